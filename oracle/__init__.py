@@ -1,0 +1,204 @@
+"""Plain fp64 CPU oracle of the MoE-ViE fine-grained MoE FFN layer forward.
+
+TEST INFRASTRUCTURE, NOT PRODUCT CODE.  Only the tests, ``__graft_entry__.smoke()``
+and the CPU-baseline leg of ``bench.py`` may import this package.  It shares no
+code with the CUDA library in ``paper_2608_17402_gb300``; the two meet only in the
+seeded input generator (``workloads``), which holds none of the method's
+arithmetic.
+
+The arithmetic lives in ``moevie_oracle.c`` (plain C, fp64, pthreads over tokens);
+this module builds it with gcc and marshals numpy arrays through ctypes.  What it
+computes, with the paper's equations:
+
+* :func:`logits`        Eq. (1), ``s = x . W_r`` (W_r stored ``[d, E]``)
+* :func:`select`        Eq. (7) selection by ``top-k(sigmoid(s) + b)``, ties to the
+  lower id, ids ascending; Eqs. (4)-(5) gates ``sigmoid(s)`` renormalised over the
+  selected experts (the bias only selects)
+* :func:`permute`       App. B, Algorithm 1 phase 1: BinCount, CumSum offsets and a
+  stable sort of the flat slots by expert
+* :func:`expert_rows`   ``E_e(x) = GELU(x W1[e]) W2[e]`` for expert-major rows
+* :func:`combine`       Eq. (6) gate-weighted sum plus ``lambda`` times the shared
+  expert
+* :func:`forward_tokens` the whole layer, token by token (Eqs. 1, 7, 4-6)
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import subprocess
+import threading
+
+import numpy as np
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+_SRC = os.path.join(_HERE, "moevie_oracle.c")
+_LIB = os.path.join(_HERE, "liboracle.so")
+_lock = threading.Lock()
+_lib = None
+
+
+def build(force: bool = False) -> str:
+    """Compile ``moevie_oracle.c`` into ``oracle/liboracle.so`` with gcc."""
+    if not force and os.path.exists(_LIB) and os.path.getmtime(_LIB) >= os.path.getmtime(_SRC):
+        return _LIB
+    cmd = ["gcc", "-O2", "-std=c11", "-ffp-contract=off", "-fno-fast-math", "-fPIC",
+           "-shared", "-pthread", _SRC, "-o", _LIB + ".tmp", "-lm"]
+    subprocess.run(cmd, check=True)
+    os.replace(_LIB + ".tmp", _LIB)
+    return _LIB
+
+
+def default_threads() -> int:
+    return max(1, os.cpu_count() or 1)
+
+
+def _load():
+    global _lib
+    with _lock:
+        if _lib is not None:
+            return _lib
+        build()
+        lib = ctypes.CDLL(_LIB)
+        P = ctypes.c_void_p
+        I64 = ctypes.c_int64
+        lib.oracle_logits.argtypes = [P, P, I64, I64, I64, P, ctypes.c_int]
+        lib.oracle_select.argtypes = [P, P, I64, I64, I64, P, P, P, ctypes.c_int]
+        lib.oracle_permute.argtypes = [P, I64, I64, I64, P, P, P, P]
+        lib.oracle_expert_rows.argtypes = [P, P, P, P, P, I64, I64, I64, I64, I64, P, I64,
+                                           ctypes.c_int, P, ctypes.c_int]
+        lib.oracle_combine.argtypes = [P, P, P, P, ctypes.c_double, I64, I64, I64, P]
+        lib.oracle_forward_tokens.argtypes = [P, P, P, P, P, P, P, ctypes.c_double,
+                                              I64, I64, I64, I64, I64, I64, P, I64,
+                                              P, P, P, P, P, ctypes.c_int]
+        for fn in (lib.oracle_logits, lib.oracle_select, lib.oracle_permute,
+                   lib.oracle_expert_rows, lib.oracle_combine, lib.oracle_forward_tokens):
+            fn.restype = ctypes.c_int
+        _lib = lib
+        return lib
+
+
+def _ptr(a):
+    return None if a is None else a.ctypes.data_as(ctypes.c_void_p)
+
+
+def _c(a, dtype):
+    """C-contiguous array of ``dtype``; bf16 data travels as uint16 bit patterns."""
+    return np.ascontiguousarray(a, dtype=dtype)
+
+
+def _check(rc, what):
+    if rc != 0:
+        raise RuntimeError(f"oracle {what} failed with code {rc}")
+
+
+def logits(x_bf16, Wr, nthreads=None):
+    """Eq. (1): ``s[t, e] = sum_i x[t, i] W_r[i, e]`` in fp64.  ``x_bf16`` uint16 [T, d]."""
+    x = _c(x_bf16, np.uint16)
+    Wr = _c(Wr, np.float32)
+    T, d = x.shape
+    E = Wr.shape[1]
+    assert Wr.shape[0] == d
+    s = np.empty((T, E), np.float64)
+    _check(_load().oracle_logits(_ptr(x), _ptr(Wr), T, d, E, _ptr(s), nthreads or default_threads()),
+           "logits")
+    return s
+
+
+def select(s, b, k, nthreads=None):
+    """Eqs. (7), (4), (5): returns ``(idx int32 [T,k], gate fp64 [T,k], margin fp64 [T])``."""
+    s = _c(s, np.float64)
+    b = _c(b, np.float32)
+    T, E = s.shape
+    idx = np.empty((T, k), np.int32)
+    gate = np.empty((T, k), np.float64)
+    margin = np.empty((T,), np.float64)
+    _check(_load().oracle_select(_ptr(s), _ptr(b), T, E, k, _ptr(idx), _ptr(gate), _ptr(margin),
+                                 nthreads or default_threads()), "select")
+    return idx, gate, margin
+
+
+def route(x_bf16, Wr, b, k, nthreads=None):
+    """Logits then selection: ``(idx, gate, margin)``."""
+    return select(logits(x_bf16, Wr, nthreads), b, k, nthreads)
+
+
+def permute(idx, E):
+    """Algorithm 1 phase 1: ``(counts [E], offsets [E+1], perm [T*k], inv [T*k])`` int32."""
+    idx = _c(idx, np.int32)
+    T, k = idx.shape
+    counts = np.empty((E,), np.int32)
+    offsets = np.empty((E + 1,), np.int32)
+    perm = np.empty((T * k,), np.int32)
+    inv = np.empty((T * k,), np.int32)
+    _check(_load().oracle_permute(_ptr(idx), T, k, E, _ptr(counts), _ptr(offsets), _ptr(perm),
+                                  _ptr(inv)), "permute")
+    return counts, offsets, perm, inv
+
+
+def expert_rows(x_bf16, perm, offsets, W1, W2, k, rows, hidden=False, nthreads=None):
+    """Un-gated ``E_e(x_t)`` (or ``GELU(x_t W1[e])`` when ``hidden``) for expert-major ``rows``."""
+    x = _c(x_bf16, np.uint16)
+    perm = _c(perm, np.int32)
+    offsets = _c(offsets, np.int32)
+    W1 = _c(W1, np.uint16)
+    W2 = None if W2 is None else _c(W2, np.uint16)
+    rows = _c(rows, np.int32)
+    T, d = x.shape
+    E, d1, h = W1.shape
+    assert d1 == d
+    width = h if hidden else d
+    out = np.empty((rows.size, width), np.float64)
+    _check(_load().oracle_expert_rows(_ptr(x), _ptr(perm), _ptr(offsets), _ptr(W1), _ptr(W2),
+                                      T, d, h, E, k, _ptr(rows), rows.size, 1 if hidden else 0,
+                                      _ptr(out), nthreads or default_threads()), "expert_rows")
+    return out
+
+
+def combine(rows_out, inv, gate, shared=None, lam=1.0):
+    """Eq. (6): ``y[t] = sum_j gate[t,j] rows_out[inv[t*k+j]] + lam * shared[t]`` (fp64)."""
+    rows_out = _c(rows_out, np.float64)
+    gate = _c(gate, np.float64)
+    inv = _c(inv, np.int32)
+    T, k = gate.shape
+    d = rows_out.shape[1]
+    sh = None if shared is None else _c(shared, np.float64)
+    y = np.empty((T, d), np.float64)
+    _check(_load().oracle_combine(_ptr(rows_out), _ptr(inv), _ptr(gate), _ptr(sh), float(lam),
+                                  T, k, d, _ptr(y)), "combine")
+    return y
+
+
+def forward_tokens(x_bf16, Wr, b, W1, W2, k, Ws1=None, Ws2=None, lam=1.0, tokens=None,
+                   nthreads=None, want_shared=False):
+    """The whole layer for ``tokens`` (all tokens when None).
+
+    Returns ``(y fp64 [n, d], idx int32 [n, k], gate fp64 [n, k], margin fp64 [n])`` and,
+    with ``want_shared``, the un-weighted shared expert output as a fifth item.
+    """
+    x = _c(x_bf16, np.uint16)
+    Wr = _c(Wr, np.float32)
+    b = _c(b, np.float32)
+    W1 = _c(W1, np.uint16)
+    W2 = _c(W2, np.uint16)
+    T, d = x.shape
+    E, _, h = W1.shape
+    hs = 0
+    if Ws1 is not None:
+        Ws1 = _c(Ws1, np.uint16)
+        Ws2 = _c(Ws2, np.uint16)
+        hs = Ws1.shape[1]
+    toks = None if tokens is None else _c(tokens, np.int32)
+    n = T if toks is None else toks.size
+    y = np.empty((n, d), np.float64)
+    idx = np.empty((n, k), np.int32)
+    gate = np.empty((n, k), np.float64)
+    margin = np.empty((n,), np.float64)
+    shared = np.empty((n, d), np.float64) if (want_shared and hs > 0) else None
+    _check(_load().oracle_forward_tokens(_ptr(x), _ptr(Wr), _ptr(b), _ptr(W1), _ptr(W2),
+                                         _ptr(Ws1), _ptr(Ws2), float(lam), T, d, E, k, h, hs,
+                                         _ptr(toks), n, _ptr(y), _ptr(idx), _ptr(gate),
+                                         _ptr(margin), _ptr(shared),
+                                         nthreads or default_threads()), "forward_tokens")
+    if want_shared:
+        return y, idx, gate, margin, shared
+    return y, idx, gate, margin

@@ -1,0 +1,379 @@
+/*
+ * moevie_oracle.c -- plain, slow, fp64 CPU oracle of the MoE-ViE fine-grained
+ * mixture-of-experts FFN layer forward pass.
+ *
+ * TEST INFRASTRUCTURE, NOT PRODUCT CODE.  This file exists only so that the
+ * CUDA library can be checked against an independent statement of the method.
+ * Only the tests, the smoke check and the benchmark's CPU-baseline leg may load
+ * it.  It shares no code, header, table or helper with the CUDA library.
+ *
+ * What it computes (paper: "MoE-ViE", Sec. 2.1-2.2, App. B):
+ *   Eq. (1)      s = W_r x                     router logits, here x.W_r with
+ *                                              W_r stored [d, E]
+ *   Eq. (7)      selection by top-k(Sigmoid(s) + b)
+ *   Eq. (4)-(5)  gates: Sigmoid(s) of the selected experts, renormalised to
+ *                sum to one (the bias b only selects; it is not part of g)
+ *   Eq. (3)/(6)  y = sum_{e in T(x)} g'_e E_e(x) + lambda * sum_shared E_s(x)
+ *   expert       E_e(x) = GELU(x W1[e]) W2[e], GELU(u) = u/2 (1 + erf(u/sqrt 2))
+ *   App. B, Algorithm 1 phase 1: the sort of the flattened routing indices by
+ *                expert, its histogram and exclusive prefix sum (offsets).
+ *
+ * Readings of points the paper leaves open (each is listed in the design notes):
+ *   - ties in the selection key go to the lower expert id;
+ *   - a token's k selected ids are stored in ascending id order;
+ *   - the sort of Algorithm 1 is stable: inside one expert's segment, rows keep
+ *     ascending flat-slot order t*k + j;
+ *   - the shared expert has its own width h_s, its weight lambda multiplies it,
+ *     and it is not renormalised together with the routed gates.
+ *
+ * Arithmetic: every input is widened exactly to double (bf16 and fp32 values
+ * are exact doubles, and so is every product x_i * w_i of a bf16 and an fp32
+ * number, since 8 + 24 mantissa bits fit in 53).  Sums run in ascending index
+ * order in double.  exp() and erf() are the C library's.  Nothing is blocked,
+ * fused or reordered beyond that.  Build with -ffp-contract=off so that no
+ * compiler contracts a*b+c into a fused multiply-add, which keeps the results
+ * the same on x86-64 and aarch64.
+ */
+#include <math.h>
+#include <pthread.h>
+#include <stdint.h>
+#include <stdlib.h>
+#include <string.h>
+
+#define ORACLE_OK 0
+#define ORACLE_ERR_ARG 1
+#define ORACLE_ERR_NOMEM 2
+
+/* ---------------------------------------------------------------- helpers */
+
+/* A bf16 value is the upper half of an IEEE fp32 value. */
+static double bf16_to_double(uint16_t v) {
+    uint32_t bits = ((uint32_t)v) << 16;
+    float f;
+    memcpy(&f, &bits, sizeof f);
+    return (double)f;
+}
+
+static double sigmoid(double s) { return 1.0 / (1.0 + exp(-s)); }
+
+static double gelu(double u) { return 0.5 * u * (1.0 + erf(u / sqrt(2.0))); }
+
+/* Parallel-for over [0, n) with plain pthreads; each worker takes a contiguous
+ * block of items.  Work items never share output memory. */
+typedef void (*item_fn)(void* ctx, int64_t begin, int64_t end);
+typedef struct { item_fn fn; void* ctx; int64_t begin, end; } worker_arg;
+
+static void* worker_main(void* p) {
+    worker_arg* a = (worker_arg*)p;
+    a->fn(a->ctx, a->begin, a->end);
+    return NULL;
+}
+
+static void parallel_for(int64_t n, int nthreads, item_fn fn, void* ctx) {
+    if (n <= 0) return;
+    if (nthreads < 1) nthreads = 1;
+    if (nthreads > 256) nthreads = 256;
+    if ((int64_t)nthreads > n) nthreads = (int)n;
+    if (nthreads == 1) { fn(ctx, 0, n); return; }
+    pthread_t th[256];
+    worker_arg args[256];
+    int started[256];
+    int64_t chunk = (n + nthreads - 1) / nthreads;
+    for (int i = 0; i < nthreads; ++i) {
+        args[i].fn = fn; args[i].ctx = ctx;
+        args[i].begin = (int64_t)i * chunk;
+        args[i].end = args[i].begin + chunk < n ? args[i].begin + chunk : n;
+        started[i] = 0;
+        if (args[i].begin >= args[i].end) continue;
+        if (pthread_create(&th[i], NULL, worker_main, &args[i]) == 0) started[i] = 1;
+        else worker_main(&args[i]);   /* could not spawn: run it here */
+    }
+    for (int i = 0; i < nthreads; ++i)
+        if (started[i]) pthread_join(th[i], NULL);
+}
+
+/* ------------------------------------------------------ Eq. (1): logits */
+
+/* s[t, e] = sum_i x[t, i] * W_r[i, e]   (x bf16 [T, d], W_r fp32 [d, E]).
+ * The loop over i is outermost so that W_r is read row by row; each s[t, e]
+ * is still one sum taken in ascending i. */
+static void logits_row(const uint16_t* xt, const float* Wr, int64_t d, int64_t E, double* st) {
+    for (int64_t e = 0; e < E; ++e) st[e] = 0.0;
+    for (int64_t i = 0; i < d; ++i) {
+        double xi = bf16_to_double(xt[i]);
+        const float* wi = Wr + i * E;
+        for (int64_t e = 0; e < E; ++e) st[e] += xi * (double)wi[e];
+    }
+}
+
+typedef struct { const uint16_t* x; const float* Wr; int64_t d, E; double* s; } logits_ctx;
+
+static void logits_items(void* p, int64_t t0, int64_t t1) {
+    logits_ctx* c = (logits_ctx*)p;
+    for (int64_t t = t0; t < t1; ++t)
+        logits_row(c->x + t * c->d, c->Wr, c->d, c->E, c->s + t * c->E);
+}
+
+int oracle_logits(const uint16_t* x, const float* Wr, int64_t T, int64_t d, int64_t E,
+                  double* s, int nthreads) {
+    if (T < 0 || d <= 0 || E <= 0 || (T > 0 && (!x || !Wr || !s))) return ORACLE_ERR_ARG;
+    logits_ctx c = { x, Wr, d, E, s };
+    parallel_for(T, nthreads, logits_items, &c);
+    return ORACLE_OK;
+}
+
+/* ------------------------------------------- Eqs. (7), (4), (5): routing */
+
+/* Select the k experts with the largest key_e = Sigmoid(s_e) + b_e (Eq. 7).
+ * Repeated arg-max over the experts not yet chosen; a tie goes to the lower id
+ * because the scan keeps the first maximum it meets.  The chosen ids are then
+ * sorted ascending.  Gates are Sigmoid(s) of the chosen experts divided by their
+ * sum (Eqs. 4-5); the bias does not enter them.  margin = (smallest chosen key)
+ * - (largest key left out), +inf when k == E. */
+static void select_one(const double* st, const float* b, int64_t E, int64_t k,
+                       int32_t* idx, double* gate, double* margin, unsigned char* taken,
+                       double* key) {
+    for (int64_t e = 0; e < E; ++e) { key[e] = sigmoid(st[e]) + (double)b[e]; taken[e] = 0; }
+    double min_chosen = INFINITY;
+    for (int64_t j = 0; j < k; ++j) {
+        int64_t best = -1;
+        for (int64_t e = 0; e < E; ++e) {
+            if (taken[e]) continue;
+            if (best < 0 || key[e] > key[best]) best = e;
+        }
+        taken[best] = 1;
+        idx[j] = (int32_t)best;
+        if (key[best] < min_chosen) min_chosen = key[best];
+    }
+    /* ascending id order (insertion sort: k is small) */
+    for (int64_t j = 1; j < k; ++j) {
+        int32_t v = idx[j];
+        int64_t i = j - 1;
+        while (i >= 0 && idx[i] > v) { idx[i + 1] = idx[i]; --i; }
+        idx[i + 1] = v;
+    }
+    double sum = 0.0;
+    for (int64_t j = 0; j < k; ++j) sum += sigmoid(st[idx[j]]);
+    for (int64_t j = 0; j < k; ++j) gate[j] = sigmoid(st[idx[j]]) / sum;
+    double max_left = -INFINITY;
+    for (int64_t e = 0; e < E; ++e)
+        if (!taken[e] && key[e] > max_left) max_left = key[e];
+    if (margin) *margin = (k == E) ? INFINITY : (min_chosen - max_left);
+}
+
+typedef struct {
+    const double* s; const float* b; int64_t E, k;
+    int32_t* idx; double* gate; double* margin; int err;
+} select_ctx;
+
+static void select_items(void* p, int64_t t0, int64_t t1) {
+    select_ctx* c = (select_ctx*)p;
+    unsigned char* taken = (unsigned char*)malloc((size_t)c->E);
+    double* key = (double*)malloc((size_t)c->E * sizeof(double));
+    if (!taken || !key) { c->err = ORACLE_ERR_NOMEM; free(taken); free(key); return; }
+    for (int64_t t = t0; t < t1; ++t)
+        select_one(c->s + t * c->E, c->b, c->E, c->k, c->idx + t * c->k, c->gate + t * c->k,
+                   c->margin ? c->margin + t : NULL, taken, key);
+    free(taken); free(key);
+}
+
+int oracle_select(const double* s, const float* b, int64_t T, int64_t E, int64_t k,
+                  int32_t* idx, double* gate, double* margin, int nthreads) {
+    if (T < 0 || E <= 0 || k < 1 || k > E) return ORACLE_ERR_ARG;
+    if (T > 0 && (!s || !b || !idx || !gate)) return ORACLE_ERR_ARG;
+    select_ctx c = { s, b, E, k, idx, gate, margin, ORACLE_OK };
+    parallel_for(T, nthreads, select_items, &c);
+    return c.err;
+}
+
+/* ------------------------------- Algorithm 1, phase 1: expert-major order */
+
+/* counts[e] = number of flat slots (t, j) with idx[t*k + j] == e (BinCount);
+ * offsets = exclusive prefix sum of counts, E + 1 entries (CumSum);
+ * perm[r] = flat slot placed at row r by a stable counting sort on the expert
+ * id (rows of one expert keep ascending slot order); inv[perm[r]] = r.
+ * The token of row r is perm[r] / k, the "index" of Algorithm 1. */
+int oracle_permute(const int32_t* idx, int64_t T, int64_t k, int64_t E,
+                   int32_t* counts, int32_t* offsets, int32_t* perm, int32_t* inv) {
+    if (T < 0 || k < 1 || E <= 0 || !counts || !offsets) return ORACLE_ERR_ARG;
+    if (T > 0 && (!idx || !perm || !inv)) return ORACLE_ERR_ARG;
+    int64_t n = T * k;
+    for (int64_t e = 0; e < E; ++e) counts[e] = 0;
+    for (int64_t i = 0; i < n; ++i) {
+        if (idx[i] < 0 || idx[i] >= E) return ORACLE_ERR_ARG;
+        counts[idx[i]] += 1;
+    }
+    offsets[0] = 0;
+    for (int64_t e = 0; e < E; ++e) offsets[e + 1] = offsets[e] + counts[e];
+    int64_t* cursor = (int64_t*)malloc((size_t)E * sizeof(int64_t));
+    if (!cursor) return ORACLE_ERR_NOMEM;
+    for (int64_t e = 0; e < E; ++e) cursor[e] = offsets[e];
+    for (int64_t i = 0; i < n; ++i) {
+        int64_t r = cursor[idx[i]]++;
+        perm[r] = (int32_t)i;
+        inv[i] = (int32_t)r;
+    }
+    free(cursor);
+    return ORACLE_OK;
+}
+
+/* ------------------------------------------------ one expert on one token */
+
+/* hidden[n] = GELU(sum_i x[i] W1[e, i, n])  for n < h   (W1 bf16 [E, d, h]).
+ * i is the outer loop (W1 read row by row); each pre-activation is still one
+ * sum in ascending i, and GELU is applied once it is complete. */
+static void expert_hidden(const uint16_t* xt, const uint16_t* W1e, int64_t d, int64_t h, double* hidden) {
+    for (int64_t n = 0; n < h; ++n) hidden[n] = 0.0;
+    for (int64_t i = 0; i < d; ++i) {
+        double xi = bf16_to_double(xt[i]);
+        const uint16_t* wi = W1e + i * h;
+        for (int64_t n = 0; n < h; ++n) hidden[n] += xi * bf16_to_double(wi[n]);
+    }
+    for (int64_t n = 0; n < h; ++n) hidden[n] = gelu(hidden[n]);
+}
+
+/* out[c] = sum_n hidden[n] W2[e, n, c]  for c < d   (W2 bf16 [E, h, d]);
+ * n outermost, each out[c] one sum in ascending n. */
+static void expert_down(const double* hidden, const uint16_t* W2e, int64_t h, int64_t d, double* out) {
+    for (int64_t c = 0; c < d; ++c) out[c] = 0.0;
+    for (int64_t n = 0; n < h; ++n) {
+        double a = hidden[n];
+        const uint16_t* wn = W2e + n * d;
+        for (int64_t c = 0; c < d; ++c) out[c] += a * bf16_to_double(wn[c]);
+    }
+}
+
+static int64_t expert_of_row(const int32_t* offsets, int64_t E, int64_t r) {
+    for (int64_t e = 0; e < E; ++e)
+        if (r >= offsets[e] && r < offsets[e + 1]) return e;
+    return -1;
+}
+
+typedef struct {
+    const uint16_t* x; const int32_t* perm; const int32_t* offsets;
+    const uint16_t* W1; const uint16_t* W2; int64_t T, d, h, E, k;
+    const int32_t* rows; double* out; int want_hidden; int err;
+} rows_ctx;
+
+static void rows_items(void* p, int64_t i0, int64_t i1) {
+    rows_ctx* c = (rows_ctx*)p;
+    double* hidden = (double*)malloc((size_t)c->h * sizeof(double));
+    if (!hidden) { c->err = ORACLE_ERR_NOMEM; return; }
+    for (int64_t i = i0; i < i1; ++i) {
+        int64_t r = c->rows[i];
+        int64_t e = expert_of_row(c->offsets, c->E, r);
+        int64_t t = c->perm[r] / c->k;
+        if (e < 0 || t < 0 || t >= c->T) { c->err = ORACLE_ERR_ARG; continue; }
+        expert_hidden(c->x + t * c->d, c->W1 + e * c->d * c->h, c->d, c->h, hidden);
+        if (c->want_hidden) memcpy(c->out + i * c->h, hidden, (size_t)c->h * sizeof(double));
+        else expert_down(hidden, c->W2 + e * c->h * c->d, c->h, c->d, c->out + i * c->d);
+    }
+    free(hidden);
+}
+
+/* Un-gated expert output of selected expert-major rows:
+ * out[i, :] = E_e(x_t) with r = rows[i], e the expert whose segment holds r,
+ * t = perm[r] / k.  want_hidden != 0 returns GELU(x_t W1[e]) ([nrows, h]) instead. */
+int oracle_expert_rows(const uint16_t* x, const int32_t* perm, const int32_t* offsets,
+                       const uint16_t* W1, const uint16_t* W2, int64_t T, int64_t d, int64_t h,
+                       int64_t E, int64_t k, const int32_t* rows, int64_t nrows, int want_hidden,
+                       double* out, int nthreads) {
+    if (T < 0 || d <= 0 || h <= 0 || E <= 0 || k < 1 || nrows < 0) return ORACLE_ERR_ARG;
+    if (nrows > 0 && (!x || !perm || !offsets || !W1 || (!want_hidden && !W2) || !rows || !out))
+        return ORACLE_ERR_ARG;
+    rows_ctx c = { x, perm, offsets, W1, W2, T, d, h, E, k, rows, out, want_hidden, ORACLE_OK };
+    parallel_for(nrows, nthreads, rows_items, &c);
+    return c.err;
+}
+
+/* ------------------------------------------------------ Eq. (6): combine */
+
+/* y[t] = sum_j gate[t*k+j] * rows_out[inv[t*k+j]] + lambda * shared[t]
+ * (shared may be NULL).  All arrays are double. */
+int oracle_combine(const double* rows_out, const int32_t* inv, const double* gate,
+                   const double* shared, double lambda, int64_t T, int64_t k, int64_t d, double* y) {
+    if (T < 0 || k < 1 || d <= 0) return ORACLE_ERR_ARG;
+    if (T > 0 && (!rows_out || !inv || !gate || !y)) return ORACLE_ERR_ARG;
+    for (int64_t t = 0; t < T; ++t)
+        for (int64_t c = 0; c < d; ++c) {
+            double acc = 0.0;
+            for (int64_t j = 0; j < k; ++j)
+                acc += gate[t * k + j] * rows_out[(int64_t)inv[t * k + j] * d + c];
+            if (shared) acc += lambda * shared[t * d + c];
+            y[t * d + c] = acc;
+        }
+    return ORACLE_OK;
+}
+
+/* ------------------------------------- the whole layer, token by token */
+
+typedef struct {
+    const uint16_t* x; const float* Wr; const float* b; const uint16_t* W1; const uint16_t* W2;
+    const uint16_t* Ws1; const uint16_t* Ws2; double lambda;
+    int64_t T, d, E, k, h, hs;
+    const int32_t* tokens; double* y; int32_t* idx; double* gate; double* margin;
+    double* shared_out; int err;
+} fwd_ctx;
+
+static void fwd_items(void* p, int64_t i0, int64_t i1) {
+    fwd_ctx* c = (fwd_ctx*)p;
+    int64_t hmax = c->h > c->hs ? c->h : c->hs;
+    double* s = (double*)malloc((size_t)c->E * sizeof(double));
+    double* key = (double*)malloc((size_t)c->E * sizeof(double));
+    unsigned char* taken = (unsigned char*)malloc((size_t)c->E);
+    double* hidden = (double*)malloc((size_t)hmax * sizeof(double));
+    double* o = (double*)malloc((size_t)c->d * sizeof(double));
+    int32_t* sel = (int32_t*)malloc((size_t)c->k * sizeof(int32_t));
+    double* g = (double*)malloc((size_t)c->k * sizeof(double));
+    if (!s || !key || !taken || !hidden || !o || !sel || !g) {
+        c->err = ORACLE_ERR_NOMEM;
+        goto done;
+    }
+    for (int64_t i = i0; i < i1; ++i) {
+        int64_t t = c->tokens ? c->tokens[i] : i;
+        if (t < 0 || t >= c->T) { c->err = ORACLE_ERR_ARG; continue; }
+        const uint16_t* xt = c->x + t * c->d;
+        logits_row(xt, c->Wr, c->d, c->E, s);                                              /* Eq. 1 */
+        double m;
+        select_one(s, c->b, c->E, c->k, sel, g, &m, taken, key);                          /* Eqs. 7, 4, 5 */
+        double* yt = c->y + i * c->d;
+        for (int64_t col = 0; col < c->d; ++col) yt[col] = 0.0;
+        for (int64_t j = 0; j < c->k; ++j) {                                               /* Eq. 6, routed */
+            int64_t e = sel[j];
+            expert_hidden(xt, c->W1 + e * c->d * c->h, c->d, c->h, hidden);
+            expert_down(hidden, c->W2 + e * c->h * c->d, c->h, c->d, o);
+            for (int64_t col = 0; col < c->d; ++col) yt[col] += g[j] * o[col];
+        }
+        if (c->hs > 0) {                                                                    /* Eq. 6, shared */
+            expert_hidden(xt, c->Ws1, c->d, c->hs, hidden);
+            expert_down(hidden, c->Ws2, c->hs, c->d, o);
+            for (int64_t col = 0; col < c->d; ++col) yt[col] += c->lambda * o[col];
+            if (c->shared_out)
+                for (int64_t col = 0; col < c->d; ++col) c->shared_out[i * c->d + col] = o[col];
+        }
+        if (c->idx) for (int64_t j = 0; j < c->k; ++j) c->idx[i * c->k + j] = sel[j];
+        if (c->gate) for (int64_t j = 0; j < c->k; ++j) c->gate[i * c->k + j] = g[j];
+        if (c->margin) c->margin[i] = m;
+    }
+done:
+    free(s); free(key); free(taken); free(hidden); free(o); free(sel); free(g);
+}
+
+/* y[i, :] for token tokens[i] (tokens may be NULL: all T tokens in order).
+ * hs == 0 means no shared expert (Ws1, Ws2 ignored).  idx, gate, margin and
+ * shared_out ([ntok, d], the un-weighted shared expert output) may be NULL. */
+int oracle_forward_tokens(const uint16_t* x, const float* Wr, const float* b,
+                          const uint16_t* W1, const uint16_t* W2,
+                          const uint16_t* Ws1, const uint16_t* Ws2, double lambda,
+                          int64_t T, int64_t d, int64_t E, int64_t k, int64_t h, int64_t hs,
+                          const int32_t* tokens, int64_t ntok,
+                          double* y, int32_t* idx, double* gate, double* margin,
+                          double* shared_out, int nthreads) {
+    if (T < 0 || d <= 0 || E <= 0 || k < 1 || k > E || h <= 0 || hs < 0 || ntok < 0) return ORACLE_ERR_ARG;
+    if (ntok > 0 && (!x || !Wr || !b || !W1 || !W2 || !y)) return ORACLE_ERR_ARG;
+    if (hs > 0 && ntok > 0 && (!Ws1 || !Ws2)) return ORACLE_ERR_ARG;
+    fwd_ctx c = { x, Wr, b, W1, W2, Ws1, Ws2, lambda, T, d, E, k, h, hs,
+                  tokens, y, idx, gate, margin, shared_out, ORACLE_OK };
+    parallel_for(ntok, nthreads, fwd_items, &c);
+    return c.err;
+}

@@ -1,0 +1,347 @@
+"""Pins of the fp64 CPU oracle against facts that do not come from the oracle.
+
+The paper prints no worked numerical example of the layer, so each pin is a
+closed form, an invariant, an exhaustive brute force on tiny inputs, an
+arbitrary-precision evaluation, or a special case that reduces to a library
+routine (torch / numpy / scipy).  Between them a dropped term, a wrong sign or
+index, or a transposed operand anywhere in the oracle fails at least one test:
+
+* logits (Eq. 1)                    exact rational sums (``fractions.Fraction``)
+* selection + tie rule (Eq. 7)      brute force over all k-subsets, keys at 60 digits
+* gates (Eqs. 4-5)                  60-digit evaluation; W_r = 0 gives exactly 1/k
+* permutation (Algorithm 1, ph. 1)  numpy stable argsort / bincount / cumsum,
+                                    permutation invariants, round trip
+* expert FFN (E=1, k=1)             torch fp64 matmul + GELU (erf form)
+* combine + gates (Eq. 6)           dense masked sum over all experts (torch einsum)
+* k = E with W_r = 0                mean of all experts
+* shared expert                     routed weights zero -> lambda * shared expert
+* token order                       permuting tokens permutes the outputs
+"""
+import itertools
+import math
+from fractions import Fraction
+
+import mpmath
+import numpy as np
+import pytest
+import scipy.special
+import torch
+
+import oracle
+import workloads
+from workloads import bf16_bits_to_f32, f32_to_bf16_bits
+
+mpmath.mp.dps = 60
+
+
+def _rng(seed):
+    return np.random.default_rng(1000 + seed)
+
+
+def _bf16(a):
+    return f32_to_bf16_bits(np.asarray(a, np.float32))
+
+
+def _exact_logits(x_bits, Wr):
+    """Exact rational logits."""
+    xf = bf16_bits_to_f32(x_bits).astype(np.float64)
+    T, d = xf.shape
+    E = Wr.shape[1]
+    out = [[sum((Fraction(float(xf[t, i])) * Fraction(float(Wr[i, e])) for i in range(d)), Fraction(0))
+             for e in range(E)] for t in range(T)]
+    return out
+
+
+def _brute_topk(keys, k):
+    """Lexicographically smallest sorted id tuple among the k-subsets whose every
+    key is >= every key left out (the lowest-id tie rule, stated as a set)."""
+    E = len(keys)
+    best = None
+    for S in itertools.combinations(range(E), k):
+        inside = min(keys[e] for e in S)
+        outside = max((keys[e] for e in range(E) if e not in S), default=None)
+        if outside is not None and inside < outside:
+            continue
+        if best is None or S < best:
+            best = S
+    return best
+
+
+def _mp_key(s_frac, b):
+    s = mpmath.mpf(s_frac.numerator) / s_frac.denominator
+    return 1 / (1 + mpmath.exp(-s)) + mpmath.mpf(float(b))
+
+
+# ------------------------------------------------------------------ logits
+
+@pytest.mark.parametrize("seed", range(6))
+def test_logits_match_exact_rationals(seed):
+    rng = _rng(seed)
+    T, d, E = 5, 7, 3          # d != E: a transposed W_r index cannot pass
+    x = _bf16(rng.standard_normal((T, d)))
+    Wr = (rng.standard_normal((d, E)) * 0.3).astype(np.float32)
+    s = oracle.logits(x, Wr)
+    ex = _exact_logits(x, Wr)
+    xf = bf16_bits_to_f32(x).astype(np.float64)
+    for t in range(T):
+        for e in range(E):
+            bound = d * 2.0 ** -53 * float(np.sum(np.abs(xf[t] * Wr[:, e])))
+            assert abs(s[t, e] - float(ex[t][e])) <= bound + 1e-300
+
+
+# --------------------------------------------------------------- selection
+
+@pytest.mark.parametrize("seed", range(40))
+def test_select_bias_only_brute_force_with_ties(seed):
+    """W_r = 0: s = 0, sigmoid = 1/2 exactly, key = 1/2 + b.  b on a dyadic grid
+    makes exact ties common.  Selection must be the brute-force top-k with the
+    lowest-id rule, and every gate exactly 1/k."""
+    rng = _rng(seed)
+    E = int(rng.integers(1, 9))
+    k = int(rng.integers(1, min(E, 4) + 1))
+    T, d = 4, 3
+    x = _bf16(rng.standard_normal((T, d)))
+    Wr = np.zeros((d, E), np.float32)
+    b = rng.choice(np.array([-0.5, -0.25, 0.0, 0.25, 0.5], np.float32), size=E).astype(np.float32)
+    idx, gate, margin = oracle.route(x, Wr, b, k)
+    want = _brute_topk([0.5 + float(v) for v in b], k)
+    for t in range(T):
+        assert tuple(idx[t]) == want
+        assert np.all(gate[t] == 1.0 / k)
+    assert len(set(want)) == k
+
+
+@pytest.mark.parametrize("seed", range(25))
+def test_select_brute_force_high_precision(seed):
+    """General logits: keys evaluated at 60 digits from exact rational logits,
+    brute force over all subsets.  Duplicated W_r columns with equal bias make
+    exact ties that must go to the lower id."""
+    rng = _rng(100 + seed)
+    E = int(rng.integers(2, 9))
+    k = int(rng.integers(1, min(E, 4) + 1))
+    T, d = 6, int(rng.integers(1, 6))
+    x = _bf16(rng.standard_normal((T, d)))
+    Wr = (rng.standard_normal((d, E)) * 0.8).astype(np.float32)
+    b = (rng.uniform(-0.1, 0.1, size=E)).astype(np.float32)
+    if E >= 3 and seed % 2 == 0:             # exact tie between experts 0 and E-1 (or a pair)
+        a, c = sorted(rng.choice(E, size=2, replace=False))
+        Wr[:, c] = Wr[:, a]
+        b[c] = b[a]
+    idx, gate, margin = oracle.route(x, Wr, b, k)
+    ex = _exact_logits(x, Wr)
+    for t in range(T):
+        keys = [_mp_key(ex[t][e], b[e]) for e in range(E)]
+        want = _brute_topk(keys, k)
+        assert tuple(idx[t]) == want, (t, keys, idx[t], want)
+        sig = [1 / (1 + mpmath.exp(-mpmath.mpf(ex[t][e].numerator) / ex[t][e].denominator)) for e in want]
+        tot = sum(sig)
+        for j, e in enumerate(want):
+            assert abs(gate[t, j] - float(sig[j] / tot)) <= 4e-16
+        left = [keys[e] for e in range(E) if e not in want]
+        if left:
+            m = float(min(keys[e] for e in want) - max(left))
+            assert abs(margin[t] - m) <= 1e-15
+        else:
+            assert margin[t] == math.inf
+
+
+def test_gates_sum_to_one_and_bias_excluded():
+    rng = _rng(7)
+    T, d, E, k = 64, 32, 16, 4
+    x = _bf16(rng.standard_normal((T, d)))
+    Wr = (rng.standard_normal((d, E)) * 0.2).astype(np.float32)
+    b = rng.uniform(-0.1, 0.1, size=E).astype(np.float32)
+    idx, gate, _ = oracle.route(x, Wr, b, k)
+    assert np.all(np.abs(gate.sum(1) - 1.0) <= 1e-15)
+    assert np.all((gate > 0) & (gate < 1))
+    # changing b may change the selection but never the gate formula: with the same
+    # selection forced (b shifted uniformly), gates are unchanged
+    idx2, gate2, _ = oracle.route(x, Wr, (b + np.float32(0.0625)).astype(np.float32), k)
+    same = np.all(idx == idx2, axis=1)
+    assert same.any()
+    assert np.array_equal(gate[same], gate2[same])
+    # ids ascending and distinct
+    assert np.all(np.diff(idx, axis=1) > 0)
+
+
+# -------------------------------------------------------------- permutation
+
+def _random_routing(rng, T, E, k, empty=()):
+    allowed = np.array([e for e in range(E) if e not in set(empty)])
+    idx = np.stack([np.sort(rng.choice(allowed, size=k, replace=False)) for _ in range(T)]).astype(np.int32)
+    return idx
+
+
+@pytest.mark.parametrize("T,E,k,empty", [(1, 1, 1, ()), (37, 5, 2, (1,)), (200, 16, 4, (0, 15)),
+                                         (129, 8, 8, ()), (0, 4, 2, ())])
+def test_permute_against_stable_argsort(T, E, k, empty):
+    rng = _rng(T + E + k)
+    idx = _random_routing(rng, T, E, k, empty) if T else np.zeros((0, k), np.int32)
+    counts, offsets, perm, inv = oracle.permute(idx, E)
+    flat = idx.ravel()
+    # library routines: bincount / cumsum / stable argsort
+    assert np.array_equal(counts, np.bincount(flat, minlength=E))
+    assert np.array_equal(offsets, np.concatenate([[0], np.cumsum(np.bincount(flat, minlength=E))]))
+    assert np.array_equal(perm, np.argsort(flat, kind="stable"))
+    # invariants
+    assert counts.sum() == T * k and offsets[-1] == T * k
+    assert np.array_equal(np.sort(perm), np.arange(T * k))
+    assert np.array_equal(inv[perm], np.arange(T * k))
+    for e in range(E):
+        seg = perm[offsets[e]:offsets[e + 1]]
+        assert np.all(flat[seg] == e)
+        assert np.all(np.diff(seg) > 0)
+    for e in empty:
+        assert counts[e] == 0
+    # round trip: unpermute(permute(v)) == v
+    v = rng.standard_normal(T * k)
+    assert np.array_equal(v[perm][inv], v)
+
+
+# ------------------------------------------------------------ expert FFN
+
+def _t64(bits):
+    return torch.from_numpy(bf16_bits_to_f32(bits).astype(np.float64))
+
+
+def _gelu_t(u):
+    return torch.nn.functional.gelu(u, approximate="none")
+
+
+def test_single_expert_is_dense_mlp():
+    """E = 1, k = 1: the layer is GELU(x W1) W2 (gate 1); d != h so a transposed
+    W1 or W2 index cannot pass."""
+    rng = _rng(11)
+    T, d, h = 9, 24, 40
+    x = _bf16(rng.standard_normal((T, d)))
+    W1 = _bf16(rng.standard_normal((1, d, h)) / np.sqrt(d))
+    W2 = _bf16(rng.standard_normal((1, h, d)) / np.sqrt(h))
+    Wr = (rng.standard_normal((d, 1)) * 0.02).astype(np.float32)
+    b = np.zeros(1, np.float32)
+    y, idx, gate, _ = oracle.forward_tokens(x, Wr, b, W1, W2, 1)
+    want = _gelu_t(_t64(x) @ _t64(W1[0])) @ _t64(W2[0])
+    assert np.all(idx == 0) and np.all(gate == 1.0)
+    np.testing.assert_allclose(y, want.numpy(), rtol=1e-12, atol=1e-12)
+
+
+def test_gelu_against_normal_cdf():
+    """GELU(u) = u Phi(u) (scipy ndtr) and GELU(u) - GELU(-u) = u, through a 1x1 expert."""
+    us = np.array([-6.0, -2.5, -1.0, -0.375, 0.0, 0.5, 1.0, 3.0, 8.0], np.float32)
+    T = us.size
+    x = _bf16(us[:, None])
+    W1 = _bf16(np.ones((1, 1, 1)))
+    W2 = _bf16(np.ones((1, 1, 1)))
+    y, *_ = oracle.forward_tokens(x, np.zeros((1, 1), np.float32), np.zeros(1, np.float32), W1, W2, 1)
+    u = bf16_bits_to_f32(x)[:, 0].astype(np.float64)
+    # the erf form 0.5 u (1 + erf(u / sqrt 2)) loses relative accuracy where 1 + erf
+    # cancels (u << 0); its absolute error stays below ~|u| * eps
+    err = np.abs(y[:, 0] - u * scipy.special.ndtr(u))
+    assert np.all(err <= 1e-14 * np.abs(u * scipy.special.ndtr(u)) + 4 * np.abs(u) * 2.0 ** -53)
+    xm = _bf16(-us[:, None])
+    ym, *_ = oracle.forward_tokens(xm, np.zeros((1, 1), np.float32), np.zeros(1, np.float32), W1, W2, 1)
+    np.testing.assert_allclose(y[:, 0] - ym[:, 0], u, rtol=0, atol=1e-15)
+
+
+def _layer(rng, T, d, E, k, h, hs=0, wr_scale=0.3):
+    x = _bf16(rng.standard_normal((T, d)))
+    Wr = (rng.standard_normal((d, E)) * wr_scale).astype(np.float32)
+    b = rng.uniform(-0.1, 0.1, size=E).astype(np.float32)
+    W1 = _bf16(rng.standard_normal((E, d, h)) / np.sqrt(d))
+    W2 = _bf16(rng.standard_normal((E, h, d)) / np.sqrt(h))
+    Ws1 = Ws2 = None
+    if hs:
+        Ws1 = _bf16(rng.standard_normal((d, hs)) / np.sqrt(d))
+        Ws2 = _bf16(rng.standard_normal((hs, d)) / np.sqrt(hs))
+    return x, Wr, b, W1, W2, Ws1, Ws2
+
+
+def _all_experts_t(x, W1, W2):
+    xt = _t64(x)
+    hid = _gelu_t(torch.einsum("td,edh->teh", xt, _t64(W1)))
+    return torch.einsum("teh,ehd->ted", hid, _t64(W2))
+
+
+@pytest.mark.parametrize("hs,lam", [(0, 1.0), (24, 1.0), (24, 0.25)])
+def test_dense_masked_formulation(hs, lam):
+    """y = sum_e mask_e g_e E_e(x) + lam S(x), with every expert evaluated densely
+    (torch einsum), using the oracle's own selection and gates."""
+    rng = _rng(21 + hs)
+    T, d, E, k, h = 40, 16, 8, 3, 20
+    x, Wr, b, W1, W2, Ws1, Ws2 = _layer(rng, T, d, E, k, h, hs)
+    y, idx, gate, _ = oracle.forward_tokens(x, Wr, b, W1, W2, k, Ws1, Ws2, lam)
+    G = torch.zeros(T, E, dtype=torch.float64)
+    G.scatter_(1, torch.from_numpy(idx.astype(np.int64)), torch.from_numpy(gate))
+    dense = torch.einsum("te,ted->td", G, _all_experts_t(x, W1, W2))
+    if hs:
+        dense = dense + lam * (_gelu_t(_t64(x) @ _t64(Ws1)) @ _t64(Ws2))
+    np.testing.assert_allclose(y, dense.numpy(), rtol=1e-12, atol=1e-12)
+
+
+def test_staged_functions_agree_with_whole_layer():
+    """permute -> expert_rows -> combine reproduces forward_tokens."""
+    rng = _rng(31)
+    T, d, E, k, h, hs = 33, 16, 6, 2, 12, 8
+    x, Wr, b, W1, W2, Ws1, Ws2 = _layer(rng, T, d, E, k, h, hs)
+    y, idx, gate, _, shared = oracle.forward_tokens(x, Wr, b, W1, W2, k, Ws1, Ws2, 0.5, want_shared=True)
+    counts, offsets, perm, inv = oracle.permute(idx, E)
+    rows = oracle.expert_rows(x, perm, offsets, W1, W2, k, np.arange(T * k, dtype=np.int32))
+    y2 = oracle.combine(rows, inv, gate, shared, 0.5)
+    np.testing.assert_allclose(y2, y, rtol=1e-13, atol=1e-13)
+    hid = oracle.expert_rows(x, perm, offsets, W1, None, k, np.arange(T * k, dtype=np.int32), hidden=True)
+    e_of_row = np.repeat(np.arange(E), counts)
+    want = _gelu_t(torch.einsum("rd,rdh->rh", _t64(x[perm // k]), _t64(W1[e_of_row])))
+    np.testing.assert_allclose(hid, want.numpy(), rtol=1e-12, atol=1e-13)
+
+
+def test_all_experts_uniform_gates():
+    """k = E and W_r = 0: every gate is 1/E and y is the mean of all experts."""
+    rng = _rng(41)
+    T, d, E, h = 12, 16, 5, 8
+    x, _, b, W1, W2, _, _ = _layer(rng, T, d, E, E, h)
+    Wr = np.zeros((d, E), np.float32)
+    y, idx, gate, margin = oracle.forward_tokens(x, Wr, b, W1, W2, E)
+    assert np.all(idx == np.arange(E)) and np.all(gate == 1.0 / E) and np.all(np.isinf(margin))
+    want = _all_experts_t(x, W1, W2).mean(1)
+    np.testing.assert_allclose(y, want.numpy(), rtol=1e-12, atol=1e-13)
+
+
+def test_shared_expert_alone():
+    """Routed experts all zero: y = lam * GELU(x Ws1) Ws2."""
+    rng = _rng(51)
+    T, d, E, k, h, hs = 10, 16, 4, 2, 8, 24
+    x, Wr, b, W1, W2, Ws1, Ws2 = _layer(rng, T, d, E, k, h, hs)
+    W1[:] = 0
+    W2[:] = 0
+    y, *_ = oracle.forward_tokens(x, Wr, b, W1, W2, k, Ws1, Ws2, 0.75)
+    want = 0.75 * (_gelu_t(_t64(x) @ _t64(Ws1)) @ _t64(Ws2))
+    np.testing.assert_allclose(y, want.numpy(), rtol=1e-12, atol=1e-13)
+
+
+def test_token_order_equivariance():
+    rng = _rng(61)
+    T, d, E, k, h = 30, 16, 8, 2, 12
+    x, Wr, b, W1, W2, _, _ = _layer(rng, T, d, E, k, h)
+    y, idx, gate, _ = oracle.forward_tokens(x, Wr, b, W1, W2, k)
+    p = rng.permutation(T)
+    y2, idx2, gate2, _ = oracle.forward_tokens(x[p], Wr, b, W1, W2, k)
+    assert np.array_equal(idx2, idx[p])
+    np.testing.assert_array_equal(gate2, gate[p])
+    np.testing.assert_array_equal(y2, y[p])
+    # a token subset gives the same rows
+    sub = np.array([3, 0, 29, 7], np.int32)
+    y3, idx3, _, _ = oracle.forward_tokens(x, Wr, b, W1, W2, k, tokens=sub)
+    np.testing.assert_array_equal(y3, y[sub])
+
+
+def test_generator_recipe_is_seeded_and_shaped():
+    cfg = workloads.small_config(T=16, d=32, E=4, k=2, h=16, h_s=8, seed=3)
+    a = workloads.make_layer(cfg)
+    b = workloads.make_layer(cfg)
+    assert np.array_equal(a.x, b.x) and np.array_equal(a.W1, b.W1) and np.array_equal(a.Ws2, b.Ws2)
+    assert a.x.shape == (16, 32) and a.Wr.shape == (32, 4) and a.W1.shape == (4, 32, 16)
+    assert a.W2.shape == (4, 16, 32) and a.Ws1.shape == (32, 8) and a.Ws2.shape == (8, 32)
+    # bf16 round trip of the generator's rounding
+    v = np.array([1.0, -2.5, 3.14159, 1e-3], np.float32)
+    back = bf16_bits_to_f32(f32_to_bf16_bits(v))
+    assert np.all(np.abs(back - v) <= np.abs(v) * 2.0 ** -8)
+    assert np.array_equal(bf16_bits_to_f32(f32_to_bf16_bits(back)), back)
