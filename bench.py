@@ -1,0 +1,337 @@
+"""Benchmark of the MoE-ViE fine-grained MoE FFN layer forward on GB300.
+
+One step = one whole layer forward (router, expert-major order, grouped up- and
+down-projection with the fused combine, shared expert, final bf16 output) over
+one batch of synthetic tokens, through the C ABI (moevie_moe_forward).
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--config c1] [--impl ours|reference]
+
+Prints one JSON line.  Default workload: the image-batch layer (c1: T=8192,
+d=1024, E=64, k=8, h=512, one shared expert h_s=1024).  Under torchrun each rank
+runs its own replica of the workload (tokens shard with no exchange step), the
+timed region is bracketed by barriers, and the slowest rank's time is used.
+`--impl reference` times the CPU oracle on a bounded token sample instead.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+import workloads  # noqa: E402
+
+METRIC = "MoE-layer tokens/sec and µs/layer on 1 GB300; achieved fraction of roofline"
+L2_FLUSH_BYTES = 512 << 20
+
+
+def parse():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=50)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--config", default="c1", choices=sorted(workloads.CONFIGS))
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    return ap.parse_args()
+
+
+def peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(path):
+        with open(path) as f:
+            mp = json.load(f)
+        return {"hbm_gbs": float(mp["hbm_gbs"]), "bf16_tflops": float(mp["bf16_tflops"]),
+                "bf16_tflops_sustained": float(mp.get("bf16_tflops_sustained", mp["bf16_tflops"])),
+                "source": "measured"}
+    return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0,
+            "source": "fallback"}
+
+
+def layer_work(cfg, counts):
+    """Algorithmic FLOPs and bytes of one layer forward (weights of touched experts)."""
+    T, d, E, k, h, hs = cfg.T, cfg.d, cfg.E, cfg.k, cfg.h, cfg.h_s
+    flops_router = 2.0 * T * d * E
+    flops_experts = 4.0 * T * k * d * h
+    flops_shared = 4.0 * T * d * hs
+    touched = int((np.asarray(counts) > 0).sum())
+    bytes_ = (T * d * 2 + T * d * 2 + d * E * 4 + E * 4 + touched * 2 * d * h * 2
+              + 2 * d * hs * 2 + 8 * T * k)
+    return {"flops": flops_router + flops_experts + flops_shared, "flops_up_gemm": 2.0 * T * k * d * h,
+            "flops_down_gemm": 2.0 * T * k * d * h, "bytes": float(bytes_), "touched_experts": touched}
+
+
+class ClockSampler:
+    """nvidia-smi clock / throttle samples during the timed region."""
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index):
+        self.gpu = gpu_index
+        self.proc = None
+        self.path = os.path.join("/tmp", f"moevie_clocks_{os.getpid()}.csv")
+
+    def __enter__(self):
+        try:
+            self.f = open(self.path, "w")
+            self.proc = subprocess.Popen(["nvidia-smi", f"--id={self.gpu}", f"--query-gpu={self.FIELDS}",
+                                          "--format=csv,noheader,nounits", "-lms", "100"],
+                                         stdout=self.f, stderr=subprocess.DEVNULL)
+            time.sleep(0.3)
+        except (OSError, FileNotFoundError):
+            self.proc = None
+        return self
+
+    def __exit__(self, *a):
+        if self.proc is not None:
+            time.sleep(0.2)
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+            self.f.close()
+
+    def summary(self):
+        if self.proc is None or not os.path.exists(self.path):
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        sm, smax, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        with open(self.path) as f:
+            for line in f:
+                p = [x.strip() for x in line.split(",")]
+                if len(p) < 9:
+                    continue
+                try:
+                    sm.append(float(p[1]))
+                    smax.append(float(p[2]))
+                except ValueError:
+                    continue
+                for n, v in zip(names, p[5:9]):
+                    if v.lower() == "active":
+                        reasons.add(n)
+        os.remove(self.path)
+        if not sm:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no samples"]}
+        loaded = [s for s in sm if s > 0.5 * max(sm)] or sm
+        return {"sm_mhz": statistics.median(loaded), "sm_max_mhz": max(smax), "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+def cpu_baseline(lay, target_s=15.0, max_tokens=None):
+    """The oracle, as it stands, on a bounded token sample (host cores)."""
+    import oracle
+    cfg = lay.cfg
+    nthreads = oracle.default_threads()
+    rng = np.random.default_rng(123)
+    probe = np.sort(rng.choice(cfg.T, size=min(cfg.T, max(nthreads, 8)), replace=False)).astype(np.int32)
+    t0 = time.perf_counter()
+    oracle.forward_tokens(lay.x, lay.Wr, lay.b, lay.W1, lay.W2, cfg.k, lay.Ws1, lay.Ws2, cfg.lam, tokens=probe)
+    per_tok = (time.perf_counter() - t0) / probe.size
+    n = int(min(cfg.T, max(nthreads, target_s / max(per_tok, 1e-9))))
+    if max_tokens:
+        n = min(n, max_tokens)
+    toks = np.sort(rng.choice(cfg.T, size=n, replace=False)).astype(np.int32)
+    t0 = time.perf_counter()
+    oracle.forward_tokens(lay.x, lay.Wr, lay.b, lay.W1, lay.W2, cfg.k, lay.Ws1, lay.Ws2, cfg.lam, tokens=toks)
+    dt = time.perf_counter() - t0
+    return {"value": n / dt, "unit": "tokens/s", "cores": nthreads, "kind": "oracle",
+            "sample": f"{n} of {cfg.T} tokens of {cfg.name} (whole layer per token: route, k experts, "
+                      f"shared expert), fp64, {nthreads} threads, {dt:.1f} s"}
+
+
+def run_reference(args, rank):
+    if rank != 0:
+        return
+    cfg = workloads.CONFIGS[args.config]
+    lay = workloads.make_layer(cfg)
+    import oracle
+    nthreads = oracle.default_threads()
+    rng = np.random.default_rng(7)
+    # size each step so the whole run stays within a few minutes
+    probe = np.arange(min(cfg.T, nthreads), dtype=np.int32)
+    t0 = time.perf_counter()
+    oracle.forward_tokens(lay.x, lay.Wr, lay.b, lay.W1, lay.W2, cfg.k, lay.Ws1, lay.Ws2, cfg.lam, tokens=probe)
+    per_tok = (time.perf_counter() - t0) / probe.size
+    budget = 150.0 / max(1, args.steps + args.warmup)
+    n = int(min(cfg.T, max(nthreads, budget / max(per_tok, 1e-9))))
+    times = []
+    for i in range(args.warmup + args.steps):
+        toks = np.sort(rng.choice(cfg.T, size=n, replace=False)).astype(np.int32)
+        t0 = time.perf_counter()
+        oracle.forward_tokens(lay.x, lay.Wr, lay.b, lay.W1, lay.W2, cfg.k, lay.Ws1, lay.Ws2, cfg.lam,
+                              tokens=toks)
+        if i >= args.warmup:
+            times.append(time.perf_counter() - t0)
+    ms = 1e3 * statistics.mean(times)
+    value = n / (ms / 1e3)
+    out = {"impl": "reference", "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": args.gpus,
+           "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True,
+           "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+           "config": {"workload": f"{cfg.name}: {cfg.note}", "T": cfg.T, "d": cfg.d, "E": cfg.E, "k": cfg.k,
+                      "h": cfg.h, "h_s": cfg.h_s, "tokens_per_step": n},
+           "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": nthreads, "kind": "oracle",
+                            "sample": f"{n} random tokens of {cfg.name} per step"},
+           "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(out), flush=True)
+
+
+def run_ours(args, rank, world):
+    import torch
+    import torch.distributed as dist
+
+    import __graft_entry__
+    from paper_2608_17402_gb300 import moevie
+
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    torch.cuda.set_device(local)
+    __graft_entry__.build()
+    cfg = workloads.CONFIGS[args.config]
+    lay = workloads.make_layer(cfg)
+
+    def bf(a):
+        return torch.from_numpy(np.ascontiguousarray(a).view(np.int16)).view(torch.bfloat16).cuda()
+
+    W = moevie.LayerWeights(W_r=torch.from_numpy(lay.Wr).cuda(), b=torch.from_numpy(lay.b).cuda(),
+                            W1=bf(lay.W1), W2=bf(lay.W2), k=cfg.k,
+                            Ws1=None if lay.Ws1 is None else bf(lay.Ws1),
+                            Ws2=None if lay.Ws2 is None else bf(lay.Ws2), lam=cfg.lam)
+    x = bf(lay.x)
+    y = torch.empty((cfg.T, cfg.d), dtype=torch.bfloat16, device="cuda")
+    ws = moevie.Workspace(cfg.T, cfg.d, cfg.E, cfg.k, cfg.h, cfg.h_s)
+    flush = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device="cuda")
+    stream = torch.cuda.current_stream()
+
+    # routing by-products once (touched experts for the byte count)
+    _, rt = moevie.moevie_moe_forward(W, x, ws, y=y, routing=True)
+    counts = rt["counts"].cpu().numpy()
+    code, detail = moevie.moevie_get_device_status(ws)
+    if code != 0:
+        raise RuntimeError(f"device status {code} {detail}")
+    work = layer_work(cfg, counts)
+
+    for _ in range(args.warmup):
+        moevie.moevie_moe_forward(W, x, ws, y=y)
+    torch.cuda.synchronize()
+
+    def barrier():
+        if world > 1:
+            dist.barrier()
+        torch.cuda.synchronize()
+
+    starts = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    ends = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    with ClockSampler(local) as clk:
+        barrier()
+        n0 = moevie.moevie_launch_count()
+        for i in range(args.steps):
+            flush.zero_()                      # L2 flush outside the timed window
+            starts[i].record(stream)
+            moevie.moevie_moe_forward(W, x, ws, y=y)
+            ends[i].record(stream)
+        barrier()
+        launches = moevie.moevie_launch_count() - n0
+    ms = statistics.mean(s.elapsed_time(e) for s, e in zip(starts, ends))
+
+    # per-stage times (events recorded between the launches, same stream)
+    nstage = len(moevie.FORWARD_STAGES)
+    stage_ms = np.zeros(nstage)
+    for i in range(args.steps):
+        evs = [torch.cuda.Event(enable_timing=True) for _ in range(nstage + 1)]
+        for e in evs:
+            e.record(stream)                   # creates the CUDA event handles
+        flush.zero_()
+        moevie.moevie_test_moe_forward_events(W, x, ws, evs, y=y)
+        torch.cuda.synchronize()
+        stage_ms += np.array([evs[j].elapsed_time(evs[j + 1]) for j in range(nstage)])
+    stage_ms /= args.steps
+    stages = dict(zip(moevie.FORWARD_STAGES, stage_ms.tolist()))
+
+    # end to end through the public API with host buffers (pinned), copies inside
+    x_host = torch.from_numpy(np.ascontiguousarray(lay.x).view(np.int16)).view(torch.bfloat16).pin_memory()
+    y_host = torch.empty((cfg.T, cfg.d), dtype=torch.bfloat16).pin_memory()
+    e2e_s = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    e2e_e = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    barrier()
+    for i in range(args.steps):
+        flush.zero_()
+        e2e_s[i].record(stream)
+        x.copy_(x_host, non_blocking=True)
+        moevie.moevie_moe_forward(W, x, ws, y=y)
+        y_host.copy_(y, non_blocking=True)
+        e2e_e[i].record(stream)
+    barrier()
+    e2e_ms = statistics.mean(s.elapsed_time(e) for s, e in zip(e2e_s, e2e_e))
+    code, detail = moevie.moevie_get_device_status(ws)
+    if code != 0:
+        raise RuntimeError(f"device status {code} {detail}")
+
+    if world > 1:
+        t = torch.tensor([ms, e2e_ms], device="cuda", dtype=torch.float64)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms, e2e_ms = float(t[0]), float(t[1])
+    if rank != 0:
+        return
+
+    pk = peaks()
+    value = world * cfg.T / (ms / 1e3)
+    dom = max(("up_gemm", "down_gemm"), key=lambda s: stages[s])
+    dom_flops = work["flops_up_gemm"] if dom == "up_gemm" else work["flops_down_gemm"]
+    achieved = dom_flops / (stages[dom] / 1e3) / 1e12
+    t_roof = max(work["flops"] / (pk["bf16_tflops"] * 1e12), work["bytes"] / (pk["hbm_gbs"] * 1e9))
+    out = {
+        "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": ms, "us_per_layer": ms * 1e3, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+        "config": {"workload": f"{cfg.name}: {cfg.note}", "T": cfg.T, "d": cfg.d, "E": cfg.E, "k": cfg.k,
+                   "h": cfg.h, "h_s": cfg.h_s, "lambda": cfg.lam, "seed": cfg.seed,
+                   "parallelism": f"replicas x{world}" if world > 1 else "single GPU",
+                   "l2": f"flushed between steps ({L2_FLUSH_BYTES >> 20} MiB write outside the timed window)"},
+        "roofline": {"bound": "tensor", "kernel": f"grouped_gemm_kernel ({dom})", "achieved": achieved,
+                     "peak": pk["bf16_tflops"], "unit": "TFLOP/s", "frac": achieved / pk["bf16_tflops"],
+                     "traffic": None, "peak_source": pk["source"] + " bf16 burst"},
+        "layer_roofline": {"flops": work["flops"], "bytes": work["bytes"], "roofline_us": t_roof * 1e6,
+                           "frac": t_roof / (ms / 1e3), "touched_experts": work["touched_experts"],
+                           "peaks": pk},
+        "stages_ms": stages,
+        "e2e": {"value": world * cfg.T / (e2e_ms / 1e3), "unit": "tokens/s",
+                "h2d_bytes_per_step": cfg.T * cfg.d * 2, "d2h_bytes_per_step": cfg.T * cfg.d * 2},
+        "gpu_launches": int(launches),
+        "clocks": clk.summary(),
+    }
+    if world == 1 and not args.no_cpu_baseline:
+        out["cpu_baseline"] = cpu_baseline(lay)
+    print(json.dumps(out), flush=True)
+
+
+def main():
+    args = parse()
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    if args.impl == "reference":
+        run_reference(args, rank)
+        return
+    if world > 1:
+        import torch
+        import torch.distributed as dist
+        torch.cuda.set_device(int(os.environ.get("LOCAL_RANK", "0")))
+        dist.init_process_group("nccl")
+    try:
+        run_ours(args, rank, world)
+    finally:
+        if world > 1:
+            import torch.distributed as dist
+            dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,161 @@
+/*
+ * moevie.h -- C ABI of the GB300 (sm_103a) MoE-ViE fine-grained MoE FFN layer.
+ *
+ * The layer (paper "MoE-ViE", Sec. 2.1-2.2 and App. B, Algorithm 1) maps tokens
+ * x[T, d] to y[T, d]:
+ *
+ *   s      = x . W_r                                  (Eq. 1; W_r stored [d, E])
+ *   T(x)   = the k experts with the largest sigmoid(s_e) + b_e      (Eq. 7)
+ *   g'_e   = sigmoid(s_e) / sum_{i in T(x)} sigmoid(s_i)            (Eqs. 4-5)
+ *   y      = sum_{e in T(x)} g'_e E_e(x) + lambda * S(x)             (Eq. 6)
+ *   E_e(x) = GELU(x W1[e]) W2[e],   S(x) = GELU(x Ws1) Ws2 (optional shared expert)
+ *
+ * GELU is the erf form u/2 (1 + erf(u / sqrt 2)).  The bias b only selects; it
+ * never enters a gate.  Ties in the selection key go to the lower expert id.  A
+ * token's k ids are stored in ascending order.  The expert-major row order is the
+ * stable sort of the flat slots t*k + j by expert id (Algorithm 1, phase 1).
+ *
+ * Conventions for every entry point
+ *  - Every array argument is DEVICE memory owned by the caller, unless a comment
+ *    says otherwise.  The library never allocates, frees or synchronises on these
+ *    calls (moevie_get_device_status excepted); all work is enqueued on `stream`
+ *    (a cudaStream_t passed as void*; NULL is the legacy default stream) and runs
+ *    asynchronously.
+ *  - bf16 tensors are passed as void* pointing at __nv_bfloat16 data.  Matrices are
+ *    row-major and dense: x[T, d], W1[E, d, h], W2[E, h, d], Ws1[d, h_s],
+ *    Ws2[h_s, d], y[T, d]; W_r[d, E] and b[E] are fp32.
+ *  - Device pointers must be 16-byte aligned.  Sizes must satisfy d % 8 == 0,
+ *    h % 16 == 0, h_s % 16 == 0, 1 <= k <= E <= 1024 and T * k < 2^31;
+ *    otherwise MOEVIE_ERR_UNSUPPORTED.  T == 0 is valid and launches nothing.
+ *  - Argument errors are reported synchronously, before anything is enqueued.
+ *    A failed kernel launch returns MOEVIE_ERR_CUDA.  Errors found on the device
+ *    (an out-of-range expert id, a pipeline wait that ran past its time limit) are
+ *    written to a status block at the start of the workspace and read back with
+ *    moevie_get_device_status; kernels never trap.
+ *  - `ws` is caller-owned device scratch of `ws_bytes` bytes.  A workspace of
+ *    moevie_workspace_size(T_max, d, E, k, h, h_s) bytes serves every entry point
+ *    for any T <= T_max with the same sizes.  It must be set up once with
+ *    moevie_workspace_init before first use.  Calls that share one workspace must
+ *    be ordered on one stream.
+ */
+#ifndef MOEVIE_H
+#define MOEVIE_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef int moevie_status;
+#define MOEVIE_OK 0
+#define MOEVIE_ERR_INVALID_ARG 1   /* null / misaligned pointer, negative size      */
+#define MOEVIE_ERR_UNSUPPORTED 2   /* sizes outside the supported set above         */
+#define MOEVIE_ERR_WORKSPACE 3     /* ws_bytes smaller than the entry point needs   */
+#define MOEVIE_ERR_CUDA 4          /* a CUDA runtime call or kernel launch failed   */
+#define MOEVIE_ERR_TIMEOUT 5       /* device: a bounded wait gave up (see status)   */
+#define MOEVIE_ERR_DEVICE 6        /* device: a bounds check failed (see status)    */
+
+/* Human-readable name of a status code (static string). */
+const char* moevie_status_string(moevie_status s);
+
+/* Library ABI version (major * 10000 + minor * 100 + patch). */
+int moevie_version(void);
+
+/* Bytes of workspace needed by moevie_moe_forward for up to T_max tokens (h_s = 0:
+ * no shared expert).  Host-only; no device query.  Monotone in T_max. */
+moevie_status moevie_workspace_size(int64_t T_max, int64_t d, int64_t E, int64_t k, int64_t h,
+                                    int64_t h_s, size_t* bytes);
+
+/* Zero the workspace's device status block (enqueued on stream).  Call once per
+ * workspace before its first use; the status is sticky until cleared again. */
+moevie_status moevie_workspace_init(void* ws, size_t ws_bytes, void* stream);
+
+/* Router (Eqs. 1, 7, 4-5).  x bf16 [T, d], W_r fp32 [d, E], b fp32 [E].
+ * Out: idx int32 [T, k] (ascending ids per token), gate fp32 [T, k] (same order).
+ * Logits are fp32; a token whose k-th and (k+1)-th keys are closer than the fp32
+ * error bound is re-decided with exactly computed (fp64) logits of the experts
+ * near its boundary, so idx equals the exact-arithmetic selection. */
+moevie_status moevie_route(const void* x, const float* W_r, const float* b, int64_t T, int64_t d,
+                           int64_t E, int64_t k, int32_t* idx, float* gate, void* ws,
+                           size_t ws_bytes, void* stream);
+
+/* Expert-major order (App. B, Algorithm 1, phase 1: Sort, index = pos // K,
+ * BinCount, CumSum).  idx int32 [T, k].  Out: counts int32 [E], offsets int32
+ * [E + 1] (exclusive prefix, offsets[E] = T*k), perm int32 [T*k] (row -> flat slot
+ * t*k + j, stable), inv int32 [T*k] (flat slot -> row).  An id outside [0, E) is a
+ * device error (MOEVIE_ERR_DEVICE in the status block; that slot is dropped). */
+moevie_status moevie_permute(const int32_t* idx, int64_t T, int64_t k, int64_t E, int32_t* counts,
+                             int32_t* offsets, int32_t* perm, int32_t* inv, void* ws,
+                             size_t ws_bytes, void* stream);
+
+/* Un-gated expert outputs in expert-major row order (App. B, Algorithm 1, Kernels
+ * 1 and 2 without the routing weight): out_rows[r, :] = GELU(x[perm[r] / k] W1[e])
+ * W2[e] for r in [offsets[e], offsets[e+1]).  out_rows bf16 [T*k, d]; fp32
+ * accumulation, the hidden activation is rounded to bf16. */
+moevie_status moevie_expert_ffn(const void* x, const int32_t* perm, const int32_t* offsets,
+                                const void* W1, const void* W2, int64_t T, int64_t d, int64_t h,
+                                int64_t E, int64_t k, void* out_rows, void* ws, size_t ws_bytes,
+                                void* stream);
+
+/* Shared expert (Sec. 2.2.1, Eq. 6, second term, without lambda):
+ * out[t, :] = GELU(x[t] Ws1) Ws2, out bf16 [T, d]. */
+moevie_status moevie_shared_expert(const void* x, const void* Ws1, const void* Ws2, int64_t T,
+                                   int64_t d, int64_t h_s, void* out, void* ws, size_t ws_bytes,
+                                   void* stream);
+
+/* Gate-weighted combine (Eq. 6): y[t] = sum_j gate[t, j] out_rows[inv[t*k + j]]
+ * + lambda * shared_out[t]   (shared_out bf16 [T, d] or NULL).  fp32 sums, y bf16. */
+moevie_status moevie_combine(const void* out_rows, const int32_t* inv, const float* gate,
+                             const void* shared_out, float lambda, int64_t T, int64_t k, int64_t d,
+                             void* y, void* stream);
+
+/* Layer description for moevie_moe_forward.  Weights are device pointers. */
+typedef struct moevie_layer {
+    int64_t d, E, k, h;
+    int64_t h_s;            /* 0: no shared expert (Ws1, Ws2 ignored) */
+    const float* W_r;       /* fp32 [d, E] */
+    const float* b;         /* fp32 [E]    */
+    const void* W1;         /* bf16 [E, d, h] */
+    const void* W2;         /* bf16 [E, h, d] */
+    const void* Ws1;        /* bf16 [d, h_s]  */
+    const void* Ws2;        /* bf16 [h_s, d]  */
+    float lambda;           /* weight of the shared expert */
+} moevie_layer;
+
+/* Optional routing by-products of moevie_moe_forward; any member may be NULL. */
+typedef struct moevie_routing {
+    int32_t* idx;       /* [T, k]   */
+    float* gate;        /* [T, k]   */
+    int32_t* counts;    /* [E]      */
+    int32_t* offsets;   /* [E + 1]  */
+    int32_t* perm;      /* [T * k]  */
+    int32_t* inv;       /* [T * k]  */
+} moevie_routing;
+
+/* The whole layer forward (Eqs. 1, 4-7; Algorithm 1): router, expert-major
+ * order, grouped up-projection with GELU fused into its epilogue and the token
+ * gather fused into its operand load, grouped down-projection whose epilogue
+ * scales each row by its gate and adds it into an fp32 accumulator of y (the
+ * scatter-add of Algorithm 1), and the shared expert.  x bf16 [T, d] -> y bf16
+ * [T, d].  `routing` may be NULL. */
+moevie_status moevie_moe_forward(const moevie_layer* layer, const void* x, int64_t T, void* y,
+                                 const moevie_routing* routing, void* ws, size_t ws_bytes,
+                                 void* stream);
+
+/* Number of kernels this library has launched since it was loaded (all
+ * threads, all devices).  Host-only. */
+uint64_t moevie_launch_count(void);
+
+/* Synchronise `stream`, then read the workspace's device status into *out
+ * (MOEVIE_OK when no device-side error was recorded).  `detail` (host, may be
+ * NULL) receives 4 ints: code, site, and two values describing the failure. */
+moevie_status moevie_get_device_status(const void* ws, void* stream, moevie_status* out,
+                                       int32_t* detail);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* MOEVIE_H */

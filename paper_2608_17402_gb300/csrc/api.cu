@@ -1,0 +1,571 @@
+// api.cu -- extern "C" entry points of the MoE-ViE layer library (moevie.h,
+// moevie_testing.h): argument checks, workspace carving and launch order.
+// Nothing here allocates, frees or synchronises on the layer path.
+#include <stdint.h>
+#include <string.h>
+
+#include <atomic>
+
+#include "internal.h"
+#include "moevie_testing.h"
+
+using namespace mv;
+
+namespace {
+std::atomic<uint64_t> g_launches{0};
+}  // namespace
+
+void mv::count_launches(int n) { g_launches.fetch_add((uint64_t)n, std::memory_order_relaxed); }
+
+namespace {
+
+constexpr uint64_t WAIT_LIMIT_NS = 2000000000ull;   // 2 s per pipeline wait
+
+inline size_t up256(size_t v) { return (v + 255) & ~static_cast<size_t>(255); }
+inline bool a16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+// Workspace carve-up.  Every buffer size is monotone in every size argument and
+// the order is fixed, so a workspace sized for the whole layer also serves each
+// stage (which passes 0 for the sizes it does not use).
+struct Layout {
+    size_t status, xnorm2, wnorm2, logits, fb_tokens;
+    size_t idx, gate, hist, counts, offsets, tile_off, perm, inv, row_tok, row_gate;
+    size_t off_s, tile_s, H, Hs, yacc;
+    size_t total;
+};
+
+Layout make_layout(int64_t T, int64_t d, int64_t E, int64_t k, int64_t h, int64_t hs) {
+    Layout L;
+    size_t o = 0;
+    auto take = [&](size_t bytes) {
+        const size_t at = o;
+        o += up256(bytes);
+        return at;
+    };
+    const int64_t n = T * k;
+    const int64_t nchunks = (n + PERM_CHUNK - 1) / PERM_CHUNK;
+    L.status = take(sizeof(DevStatus));
+    L.xnorm2 = take(4 * T);
+    L.wnorm2 = take(4 * E);
+    L.logits = take(4 * T * E);
+    L.fb_tokens = take(4 * T);
+    L.idx = take(4 * n);
+    L.gate = take(4 * n);
+    L.hist = take(4 * nchunks * E);
+    L.counts = take(4 * E);
+    L.offsets = take(4 * (E + 1));
+    L.tile_off = take(4 * (E + 1));
+    L.perm = take(4 * n);
+    L.inv = take(4 * n);
+    L.row_tok = take(4 * n);
+    L.row_gate = take(4 * n);
+    L.off_s = take(8);
+    L.tile_s = take(8);
+    L.H = take(2 * n * h);
+    L.Hs = take(2 * T * hs);
+    L.yacc = take(4 * T * d);
+    L.total = o;
+    return L;
+}
+
+template <typename P>
+P* at(void* ws, size_t off) {
+    return reinterpret_cast<P*>(static_cast<uint8_t*>(ws) + off);
+}
+
+moevie_status check_sizes(int64_t T, int64_t d, int64_t E, int64_t k, int64_t h, int64_t hs) {
+    if (T < 0 || d <= 0 || E <= 0 || k <= 0 || h < 0 || hs < 0) return MOEVIE_ERR_INVALID_ARG;
+    if (d % 8 != 0 || h % 16 != 0 || hs % 16 != 0) return MOEVIE_ERR_UNSUPPORTED;
+    if (k > E || E > 1024) return MOEVIE_ERR_UNSUPPORTED;
+    if (T * k >= (int64_t(1) << 31) || T >= (int64_t(1) << 31) || d >= (int64_t(1) << 24) ||
+        h >= (int64_t(1) << 24) || hs >= (int64_t(1) << 24))
+        return MOEVIE_ERR_UNSUPPORTED;
+    return MOEVIE_OK;
+}
+
+int num_sms() {
+    static int cache[64] = {};
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 148;
+    if (!cache[dev]) {
+        int n = 0;
+        cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev);
+        cache[dev] = n > 0 ? n : 148;
+    }
+    return cache[dev];
+}
+
+inline moevie_status cuda_status(cudaError_t e) { return e == cudaSuccess ? MOEVIE_OK : MOEVIE_ERR_CUDA; }
+
+#define MV_TRY(expr)                                     \
+    do {                                                 \
+        cudaError_t _e = (expr);                         \
+        if (_e != cudaSuccess) return MOEVIE_ERR_CUDA;   \
+    } while (0)
+
+// One grouped GEMM launch: D = A[rows] . W[g], W bf16 [G][K][N].
+struct GemmSpec {
+    const void* A;
+    int64_t lda;
+    const int32_t* a_rows;
+    int a_div;
+    int64_t a_nrows;      // rows of A
+    int64_t m_total;      // GEMM rows (segment total bound)
+    int64_t o_nrows;      // rows of yacc
+    const int32_t* offsets;
+    const int32_t* tile_off;
+    int G;
+    int64_t max_mtiles;   // host bound on the number of m-tiles
+    const void* W;
+    int K, N;
+    int epi;
+    void* out;
+    int64_t ldo;
+    float* yacc;
+    int64_t ldy;
+    const int32_t* o_rows;
+    int o_div;
+    const float* row_scale;
+    float scale;
+};
+
+moevie_status run_gemm(const GemmSpec& g, DevStatus* st, cudaStream_t s) {
+    GemmArgs a;
+    memset(&a, 0, sizeof a);
+    if (!make_weight_tmap(&a.tmB, g.W, g.N, g.K, g.G)) return MOEVIE_ERR_CUDA;
+    a.A = static_cast<const __nv_bfloat16*>(g.A);
+    a.lda = g.lda;
+    a.a_rows = g.a_rows;
+    a.a_div = g.a_div > 0 ? g.a_div : 1;
+    a.a_nrows = g.a_nrows;
+    a.m_total = g.m_total;
+    a.max_mtiles = g.max_mtiles;
+    a.o_nrows = g.o_nrows;
+    a.offsets = g.offsets;
+    a.tile_off = g.tile_off;
+    a.G = g.G;
+    a.K = g.K;
+    a.N = g.N;
+    choose_bn(g.N, &a.BN, &a.n_ntiles);
+    a.num_kb = (g.K + GM_BK - 1) / GM_BK;
+    a.nbox = (a.BN + 63) / 64;
+    a.epi = g.epi;
+    a.out = static_cast<__nv_bfloat16*>(g.out);
+    a.ldo = g.ldo;
+    a.yacc = g.yacc;
+    a.ldy = g.ldy;
+    a.o_rows = g.o_rows;
+    a.o_div = g.o_div > 0 ? g.o_div : 1;
+    a.row_scale = g.row_scale;
+    a.scale = g.scale;
+    a.status = st;
+    a.limit_ns = WAIT_LIMIT_NS;
+    const int64_t work = g.max_mtiles * a.n_ntiles;
+    const int sms = num_sms();
+    const int grid = (int)(work < sms ? (work > 0 ? work : 1) : sms);
+    return cuda_status(launch_grouped_gemm(a, grid, s));
+}
+
+}  // namespace
+
+extern "C" {
+
+const char* moevie_status_string(moevie_status s) {
+    switch (s) {
+        case MOEVIE_OK: return "MOEVIE_OK";
+        case MOEVIE_ERR_INVALID_ARG: return "MOEVIE_ERR_INVALID_ARG";
+        case MOEVIE_ERR_UNSUPPORTED: return "MOEVIE_ERR_UNSUPPORTED";
+        case MOEVIE_ERR_WORKSPACE: return "MOEVIE_ERR_WORKSPACE";
+        case MOEVIE_ERR_CUDA: return "MOEVIE_ERR_CUDA";
+        case MOEVIE_ERR_TIMEOUT: return "MOEVIE_ERR_TIMEOUT";
+        case MOEVIE_ERR_DEVICE: return "MOEVIE_ERR_DEVICE";
+        default: return "MOEVIE_ERR_UNKNOWN";
+    }
+}
+
+int moevie_version(void) { return 100; }
+
+moevie_status moevie_workspace_size(int64_t T_max, int64_t d, int64_t E, int64_t k, int64_t h,
+                                    int64_t h_s, size_t* bytes) {
+    if (!bytes) return MOEVIE_ERR_INVALID_ARG;
+    const moevie_status c = check_sizes(T_max, d, E, k, h, h_s);
+    if (c != MOEVIE_OK) return c;
+    *bytes = make_layout(T_max, d, E, k, h, h_s).total;
+    return MOEVIE_OK;
+}
+
+moevie_status moevie_workspace_init(void* ws, size_t ws_bytes, void* stream) {
+    if (!ws || ws_bytes < sizeof(DevStatus) || !a16(ws)) return MOEVIE_ERR_INVALID_ARG;
+    return cuda_status(cudaMemsetAsync(ws, 0, sizeof(DevStatus), static_cast<cudaStream_t>(stream)));
+}
+
+moevie_status moevie_route(const void* x, const float* W_r, const float* b, int64_t T, int64_t d,
+                           int64_t E, int64_t k, int32_t* idx, float* gate, void* ws,
+                           size_t ws_bytes, void* stream) {
+    moevie_status c = check_sizes(T, d, E, k, 0, 0);
+    if (c != MOEVIE_OK) return c;
+    if (T == 0) return MOEVIE_OK;
+    if (!x || !W_r || !b || !idx || !gate || !ws) return MOEVIE_ERR_INVALID_ARG;
+    if (!a16(x) || !a16(ws)) return MOEVIE_ERR_INVALID_ARG;
+    const Layout L = make_layout(T, 0, E, k, 0, 0);
+    if (ws_bytes < L.total) return MOEVIE_ERR_WORKSPACE;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    DevStatus* st = at<DevStatus>(ws, L.status);
+    RouteBufs rb{at<float>(ws, L.logits), at<float>(ws, L.xnorm2), at<float>(ws, L.wnorm2),
+                 at<int32_t>(ws, L.fb_tokens)};
+    const __nv_bfloat16* xb = static_cast<const __nv_bfloat16*>(x);
+    MV_TRY(launch_route_logits(xb, W_r, (int)T, (int)d, (int)E, rb, st, s));
+    MV_TRY(launch_route_select(xb, W_r, b, (int)T, (int)d, (int)E, (int)k, idx, gate, rb, st,
+                               num_sms(), s));
+    return MOEVIE_OK;
+}
+
+moevie_status moevie_permute(const int32_t* idx, int64_t T, int64_t k, int64_t E, int32_t* counts,
+                             int32_t* offsets, int32_t* perm, int32_t* inv, void* ws,
+                             size_t ws_bytes, void* stream) {
+    moevie_status c = check_sizes(T, 8, E, k, 0, 0);
+    if (c != MOEVIE_OK) return c;
+    if (!counts || !offsets || !ws) return MOEVIE_ERR_INVALID_ARG;
+    if (T > 0 && (!idx || !perm || !inv)) return MOEVIE_ERR_INVALID_ARG;
+    if (!a16(ws) || (idx && !a16(idx))) return MOEVIE_ERR_INVALID_ARG;
+    const Layout L = make_layout(T, 0, E, k, 0, 0);
+    if (ws_bytes < L.total) return MOEVIE_ERR_WORKSPACE;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    if (T == 0) {   // all counts and offsets are zero
+        MV_TRY(cudaMemsetAsync(counts, 0, 4 * E, s));
+        MV_TRY(cudaMemsetAsync(offsets, 0, 4 * (E + 1), s));
+        return MOEVIE_OK;
+    }
+    DevStatus* st = at<DevStatus>(ws, L.status);
+    MV_TRY(launch_permute(idx, T * k, (int)k, (int)E, GM_BM, nullptr, at<int32_t>(ws, L.hist),
+                          counts, offsets, at<int32_t>(ws, L.tile_off), perm, inv, nullptr,
+                          nullptr, st, s));
+    return MOEVIE_OK;
+}
+
+static moevie_status expert_up(const void* x, const int32_t* perm, const int32_t* offsets,
+                               const int32_t* tile_off, const void* W1, int64_t T, int64_t d,
+                               int64_t h, int64_t E, int64_t k, void* hidden, DevStatus* st,
+                               cudaStream_t s) {
+    GemmSpec g{};
+    g.A = x;
+    g.lda = d;
+    g.a_rows = perm;
+    g.a_div = (int)k;
+    g.a_nrows = T;
+    g.m_total = T * k;
+    g.offsets = offsets;
+    g.tile_off = tile_off;
+    g.G = (int)E;
+    g.max_mtiles = (T * k + GM_BM - 1) / GM_BM + E;
+    g.W = W1;
+    g.K = (int)d;
+    g.N = (int)h;
+    g.epi = EPI_GELU_BF16;
+    g.out = hidden;
+    g.ldo = h;
+    return run_gemm(g, st, s);
+}
+
+moevie_status moevie_expert_ffn(const void* x, const int32_t* perm, const int32_t* offsets,
+                                const void* W1, const void* W2, int64_t T, int64_t d, int64_t h,
+                                int64_t E, int64_t k, void* out_rows, void* ws, size_t ws_bytes,
+                                void* stream) {
+    moevie_status c = check_sizes(T, d, E, k, h, 0);
+    if (c != MOEVIE_OK) return c;
+    if (h == 0) return MOEVIE_ERR_UNSUPPORTED;
+    if (T == 0) return MOEVIE_OK;
+    if (!x || !perm || !offsets || !W1 || !W2 || !out_rows || !ws) return MOEVIE_ERR_INVALID_ARG;
+    if (!a16(x) || !a16(W1) || !a16(W2) || !a16(out_rows) || !a16(ws)) return MOEVIE_ERR_INVALID_ARG;
+    const Layout L = make_layout(T, 0, E, k, h, 0);
+    if (ws_bytes < L.total) return MOEVIE_ERR_WORKSPACE;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    DevStatus* st = at<DevStatus>(ws, L.status);
+    int32_t* tile_off = at<int32_t>(ws, L.tile_off);
+    void* H = at<void>(ws, L.H);
+    MV_TRY(launch_tile_prefix(offsets, (int)E, GM_BM, tile_off, s));
+    c = expert_up(x, perm, offsets, tile_off, W1, T, d, h, E, k, H, st, s);
+    if (c != MOEVIE_OK) return c;
+    GemmSpec g{};
+    g.A = H;
+    g.lda = h;
+    g.a_nrows = T * k;
+    g.m_total = T * k;
+    g.offsets = offsets;
+    g.tile_off = tile_off;
+    g.G = (int)E;
+    g.max_mtiles = (T * k + GM_BM - 1) / GM_BM + E;
+    g.W = W2;
+    g.K = (int)h;
+    g.N = (int)d;
+    g.epi = EPI_STORE_BF16;
+    g.out = out_rows;
+    g.ldo = d;
+    return run_gemm(g, st, s);
+}
+
+// Shared expert as one group of all T rows (identity gather).  Writes either a
+// bf16 output (out != NULL) or lambda * S(x) as the first value of the fp32 y
+// accumulator.
+static moevie_status shared_expert(const void* x, const void* Ws1, const void* Ws2, int64_t T,
+                                   int64_t d, int64_t hs, void* out, float* yacc, float lambda,
+                                   const Layout& L, void* ws, DevStatus* st, cudaStream_t s) {
+    int32_t* off_s = at<int32_t>(ws, L.off_s);
+    int32_t* tile_s = at<int32_t>(ws, L.tile_s);
+    void* Hs = at<void>(ws, L.Hs);
+    MV_TRY(launch_single_group(off_s, tile_s, (int)T, GM_BM, s));
+    GemmSpec g{};
+    g.A = x;
+    g.lda = d;
+    g.a_nrows = T;
+    g.m_total = T;
+    g.offsets = off_s;
+    g.tile_off = tile_s;
+    g.G = 1;
+    g.max_mtiles = (T + GM_BM - 1) / GM_BM;
+    g.W = Ws1;
+    g.K = (int)d;
+    g.N = (int)hs;
+    g.epi = EPI_GELU_BF16;
+    g.out = Hs;
+    g.ldo = hs;
+    moevie_status c = run_gemm(g, st, s);
+    if (c != MOEVIE_OK) return c;
+    GemmSpec g2{};
+    g2.A = Hs;
+    g2.lda = hs;
+    g2.a_nrows = T;
+    g2.m_total = T;
+    g2.o_nrows = T;
+    g2.offsets = off_s;
+    g2.tile_off = tile_s;
+    g2.G = 1;
+    g2.max_mtiles = (T + GM_BM - 1) / GM_BM;
+    g2.W = Ws2;
+    g2.K = (int)hs;
+    g2.N = (int)d;
+    if (out) {
+        g2.epi = EPI_STORE_BF16;
+        g2.out = out;
+        g2.ldo = d;
+    } else {
+        g2.epi = EPI_STORE_F32;
+        g2.yacc = yacc;
+        g2.ldy = d;
+        g2.scale = lambda;
+    }
+    return run_gemm(g2, st, s);
+}
+
+moevie_status moevie_shared_expert(const void* x, const void* Ws1, const void* Ws2, int64_t T,
+                                   int64_t d, int64_t h_s, void* out, void* ws, size_t ws_bytes,
+                                   void* stream) {
+    moevie_status c = check_sizes(T, d, 1, 1, 0, h_s);
+    if (c != MOEVIE_OK) return c;
+    if (h_s == 0) return MOEVIE_ERR_UNSUPPORTED;
+    if (T == 0) return MOEVIE_OK;
+    if (!x || !Ws1 || !Ws2 || !out || !ws) return MOEVIE_ERR_INVALID_ARG;
+    if (!a16(x) || !a16(Ws1) || !a16(Ws2) || !a16(out) || !a16(ws)) return MOEVIE_ERR_INVALID_ARG;
+    const Layout L = make_layout(T, 0, 1, 1, 0, h_s);
+    if (ws_bytes < L.total) return MOEVIE_ERR_WORKSPACE;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    return shared_expert(x, Ws1, Ws2, T, d, h_s, out, nullptr, 0.f, L, ws,
+                         at<DevStatus>(ws, L.status), s);
+}
+
+moevie_status moevie_combine(const void* out_rows, const int32_t* inv, const float* gate,
+                             const void* shared_out, float lambda, int64_t T, int64_t k, int64_t d,
+                             void* y, void* stream) {
+    moevie_status c = check_sizes(T, d, k, k, 0, 0);
+    if (c != MOEVIE_OK) return c;
+    if (T == 0) return MOEVIE_OK;
+    if (!out_rows || !inv || !gate || !y) return MOEVIE_ERR_INVALID_ARG;
+    if (!a16(out_rows) || !a16(y) || (shared_out && !a16(shared_out))) return MOEVIE_ERR_INVALID_ARG;
+    return cuda_status(launch_combine(static_cast<const __nv_bfloat16*>(out_rows), inv, gate,
+                                      static_cast<const __nv_bfloat16*>(shared_out), lambda, T,
+                                      (int)k, (int)d, static_cast<__nv_bfloat16*>(y),
+                                      static_cast<cudaStream_t>(stream)));
+}
+
+static moevie_status forward_impl(const moevie_layer* Lr, const void* x, int64_t T, void* y,
+                                  const moevie_routing* routing, void* ws, size_t ws_bytes,
+                                  void* stream, void* const* events, int n_events) {
+    if (!Lr) return MOEVIE_ERR_INVALID_ARG;
+    if (events && n_events != 7) return MOEVIE_ERR_INVALID_ARG;
+    const int64_t d = Lr->d, E = Lr->E, k = Lr->k, h = Lr->h, hs = Lr->h_s;
+    moevie_status c = check_sizes(T, d, E, k, h, hs);
+    if (c != MOEVIE_OK) return c;
+    if (h == 0) return MOEVIE_ERR_UNSUPPORTED;
+    if (T == 0) return MOEVIE_OK;
+    if (!x || !y || !ws || !Lr->W_r || !Lr->b || !Lr->W1 || !Lr->W2) return MOEVIE_ERR_INVALID_ARG;
+    if (hs > 0 && (!Lr->Ws1 || !Lr->Ws2)) return MOEVIE_ERR_INVALID_ARG;
+    if (!a16(x) || !a16(y) || !a16(ws) || !a16(Lr->W1) || !a16(Lr->W2)) return MOEVIE_ERR_INVALID_ARG;
+    if (hs > 0 && (!a16(Lr->Ws1) || !a16(Lr->Ws2))) return MOEVIE_ERR_INVALID_ARG;
+    const Layout L = make_layout(T, d, E, k, h, hs);
+    if (ws_bytes < L.total) return MOEVIE_ERR_WORKSPACE;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    DevStatus* st = at<DevStatus>(ws, L.status);
+    moevie_routing r{};
+    if (routing) r = *routing;
+    int32_t* idx = r.idx ? r.idx : at<int32_t>(ws, L.idx);
+    float* gate = r.gate ? r.gate : at<float>(ws, L.gate);
+    int32_t* offsets = r.offsets ? r.offsets : at<int32_t>(ws, L.offsets);
+    int32_t* perm = r.perm ? r.perm : at<int32_t>(ws, L.perm);
+    int32_t* inv = r.inv ? r.inv : at<int32_t>(ws, L.inv);
+    if (!a16(idx)) return MOEVIE_ERR_INVALID_ARG;
+    int32_t* tile_off = at<int32_t>(ws, L.tile_off);
+    int32_t* row_tok = at<int32_t>(ws, L.row_tok);
+    float* row_gate = at<float>(ws, L.row_gate);
+    float* yacc = at<float>(ws, L.yacc);
+    const __nv_bfloat16* xb = static_cast<const __nv_bfloat16*>(x);
+    auto mark = [&](int i) -> cudaError_t {
+        return events ? cudaEventRecord(static_cast<cudaEvent_t>(events[i]), s) : cudaSuccess;
+    };
+
+    MV_TRY(mark(0));
+    // 1. router (Eqs. 1, 7, 4-5)
+    RouteBufs rb{at<float>(ws, L.logits), at<float>(ws, L.xnorm2), at<float>(ws, L.wnorm2),
+                 at<int32_t>(ws, L.fb_tokens)};
+    MV_TRY(launch_route_logits(xb, Lr->W_r, (int)T, (int)d, (int)E, rb, st, s));
+    MV_TRY(launch_route_select(xb, Lr->W_r, Lr->b, (int)T, (int)d, (int)E, (int)k, idx, gate, rb,
+                               st, num_sms(), s));
+    MV_TRY(mark(1));
+    // 2. expert-major order (Algorithm 1, phase 1) + per-row token and gate
+    MV_TRY(launch_permute(idx, T * k, (int)k, (int)E, GM_BM, gate, at<int32_t>(ws, L.hist),
+                          r.counts, offsets, tile_off, perm, inv, row_tok, row_gate, st, s));
+    MV_TRY(mark(2));
+    // 3. y accumulator: lambda * shared expert, or zero
+    if (hs > 0) {
+        c = shared_expert(x, Lr->Ws1, Lr->Ws2, T, d, hs, nullptr, yacc, Lr->lambda, L, ws, st, s);
+        if (c != MOEVIE_OK) return c;
+    } else {
+        MV_TRY(launch_zero_f32(yacc, T * d, s));
+    }
+    MV_TRY(mark(3));
+    // 4. grouped up-projection, token gather in the operand load, GELU epilogue
+    GemmSpec up{};
+    up.A = x;
+    up.lda = d;
+    up.a_rows = row_tok;
+    up.a_div = 1;
+    up.a_nrows = T;
+    up.m_total = T * k;
+    up.offsets = offsets;
+    up.tile_off = tile_off;
+    up.G = (int)E;
+    up.max_mtiles = (T * k + GM_BM - 1) / GM_BM + E;
+    up.W = Lr->W1;
+    up.K = (int)d;
+    up.N = (int)h;
+    up.epi = EPI_GELU_BF16;
+    up.out = at<void>(ws, L.H);
+    up.ldo = h;
+    if ((c = run_gemm(up, st, s)) != MOEVIE_OK) return c;
+    MV_TRY(mark(4));
+    // 5. grouped down-projection, epilogue: gate * row added into y (scatter-add)
+    GemmSpec dn{};
+    dn.A = at<void>(ws, L.H);
+    dn.lda = h;
+    dn.a_nrows = T * k;
+    dn.m_total = T * k;
+    dn.o_nrows = T;
+    dn.offsets = offsets;
+    dn.tile_off = tile_off;
+    dn.G = (int)E;
+    dn.max_mtiles = up.max_mtiles;
+    dn.W = Lr->W2;
+    dn.K = (int)h;
+    dn.N = (int)d;
+    dn.epi = EPI_ADD_F32;
+    dn.yacc = yacc;
+    dn.ldy = d;
+    dn.o_rows = row_tok;
+    dn.o_div = 1;
+    dn.row_scale = row_gate;
+    if ((c = run_gemm(dn, st, s)) != MOEVIE_OK) return c;
+    MV_TRY(mark(5));
+    // 6. y = bf16(accumulator)
+    MV_TRY(launch_f32_to_bf16(yacc, static_cast<__nv_bfloat16*>(y), T * d, s));
+    MV_TRY(mark(6));
+    return MOEVIE_OK;
+}
+
+moevie_status moevie_moe_forward(const moevie_layer* layer, const void* x, int64_t T, void* y,
+                                 const moevie_routing* routing, void* ws, size_t ws_bytes,
+                                 void* stream) {
+    return forward_impl(layer, x, T, y, routing, ws, ws_bytes, stream, nullptr, 0);
+}
+
+uint64_t moevie_launch_count(void) { return g_launches.load(std::memory_order_relaxed); }
+
+moevie_status moevie_get_device_status(const void* ws, void* stream, moevie_status* out,
+                                       int32_t* detail) {
+    if (!ws || !out) return MOEVIE_ERR_INVALID_ARG;
+    if (cudaStreamSynchronize(static_cast<cudaStream_t>(stream)) != cudaSuccess) return MOEVIE_ERR_CUDA;
+    int32_t v[4];
+    if (cudaMemcpy(v, ws, sizeof v, cudaMemcpyDeviceToHost) != cudaSuccess) return MOEVIE_ERR_CUDA;
+    *out = v[0];
+    if (detail) memcpy(detail, v, sizeof v);
+    return MOEVIE_OK;
+}
+
+// ------------------------------------------------------------ test hooks
+
+moevie_status moevie_test_route_logits(const void* x, const float* W_r, int64_t T, int64_t d,
+                                       int64_t E, float* s_out, void* ws, size_t ws_bytes,
+                                       void* stream) {
+    moevie_status c = check_sizes(T, d, E, 1, 0, 0);
+    if (c != MOEVIE_OK) return c;
+    if (T == 0) return MOEVIE_OK;
+    if (!x || !W_r || !s_out || !ws || !a16(x) || !a16(ws)) return MOEVIE_ERR_INVALID_ARG;
+    const Layout L = make_layout(T, 0, E, 1, 0, 0);
+    if (ws_bytes < L.total) return MOEVIE_ERR_WORKSPACE;
+    RouteBufs rb{s_out, at<float>(ws, L.xnorm2), at<float>(ws, L.wnorm2), at<int32_t>(ws, L.fb_tokens)};
+    return cuda_status(launch_route_logits(static_cast<const __nv_bfloat16*>(x), W_r, (int)T, (int)d,
+                                           (int)E, rb, at<DevStatus>(ws, L.status),
+                                           static_cast<cudaStream_t>(stream)));
+}
+
+moevie_status moevie_test_fallback_count(const void* ws, void* stream, int32_t* out) {
+    if (!ws || !out) return MOEVIE_ERR_INVALID_ARG;
+    if (cudaStreamSynchronize(static_cast<cudaStream_t>(stream)) != cudaSuccess) return MOEVIE_ERR_CUDA;
+    DevStatus h;
+    if (cudaMemcpy(&h, ws, sizeof h, cudaMemcpyDeviceToHost) != cudaSuccess) return MOEVIE_ERR_CUDA;
+    *out = h.fb_count;
+    return MOEVIE_OK;
+}
+
+moevie_status moevie_test_expert_hidden(const void* x, const int32_t* perm, const int32_t* offsets,
+                                        const void* W1, int64_t T, int64_t d, int64_t h, int64_t E,
+                                        int64_t k, void* hidden, void* ws, size_t ws_bytes,
+                                        void* stream) {
+    moevie_status c = check_sizes(T, d, E, k, h, 0);
+    if (c != MOEVIE_OK) return c;
+    if (h == 0) return MOEVIE_ERR_UNSUPPORTED;
+    if (T == 0) return MOEVIE_OK;
+    if (!x || !perm || !offsets || !W1 || !hidden || !ws) return MOEVIE_ERR_INVALID_ARG;
+    if (!a16(x) || !a16(W1) || !a16(hidden) || !a16(ws)) return MOEVIE_ERR_INVALID_ARG;
+    const Layout L = make_layout(T, 0, E, k, 0, 0);
+    if (ws_bytes < L.total) return MOEVIE_ERR_WORKSPACE;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    int32_t* tile_off = at<int32_t>(ws, L.tile_off);
+    MV_TRY(launch_tile_prefix(offsets, (int)E, GM_BM, tile_off, s));
+    return expert_up(x, perm, offsets, tile_off, W1, T, d, h, E, k, hidden,
+                     at<DevStatus>(ws, L.status), s);
+}
+
+moevie_status moevie_test_moe_forward_events(const moevie_layer* layer, const void* x, int64_t T,
+                                            void* y, void* ws, size_t ws_bytes, void* stream,
+                                            void* const* events, int n_events) {
+    if (!events) return MOEVIE_ERR_INVALID_ARG;
+    return forward_impl(layer, x, T, y, nullptr, ws, ws_bytes, stream, events, n_events);
+}
+
+moevie_status moevie_test_wait_timeout(void* ws, size_t ws_bytes, uint64_t limit_ns, void* stream) {
+    if (!ws || ws_bytes < sizeof(DevStatus) || !a16(ws)) return MOEVIE_ERR_INVALID_ARG;
+    if (limit_ns == 0 || limit_ns > 10000000000ull) return MOEVIE_ERR_INVALID_ARG;
+    return cuda_status(launch_wait_probe(static_cast<DevStatus*>(ws), limit_ns,
+                                         static_cast<cudaStream_t>(stream)));
+}
+
+}  // extern "C"

@@ -1,0 +1,125 @@
+// misc.cu -- memory-bound helper kernels of the MoE-ViE layer, sm_103a.
+//   zero_f32_kernel      y accumulator := 0 (float4 stores)
+//   f32_to_bf16_kernel   y := bf16(y accumulator)  (32-byte loads, 16-byte stores)
+//   combine_kernel       Eq. (6) as a stand-alone gather-reduce over expert-major
+//                        rows: y[t] = sum_j gate[t, j] rows[inv[t*k + j]] + lambda * shared[t]
+//   wait_probe_kernel    bounded wait on a barrier nobody arrives at (error-path test)
+#include "internal.h"
+
+namespace mv {
+
+namespace {
+
+__global__ void zero_f32_kernel(float4* __restrict__ p, int64_t n4) {
+    const float4 z = make_float4(0.f, 0.f, 0.f, 0.f);
+    for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n4;
+         i += (int64_t)gridDim.x * blockDim.x)
+        p[i] = z;
+}
+
+// n8 groups of 8 values.
+__global__ void f32_to_bf16_kernel(const float4* __restrict__ src, uint4* __restrict__ dst,
+                                   int64_t n8) {
+    for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n8;
+         i += (int64_t)gridDim.x * blockDim.x) {
+        const float4 a = src[2 * i], b = src[2 * i + 1];
+        uint4 u;
+        u.x = pack_bf16x2(a.x, a.y);
+        u.y = pack_bf16x2(a.z, a.w);
+        u.z = pack_bf16x2(b.x, b.y);
+        u.w = pack_bf16x2(b.z, b.w);
+        dst[i] = u;
+    }
+}
+
+// One thread per (token, 8 columns).
+__global__ void combine_kernel(const __nv_bfloat16* __restrict__ rows,
+                               const int32_t* __restrict__ inv, const float* __restrict__ gate,
+                               const __nv_bfloat16* __restrict__ shared, float lambda, int64_t T,
+                               int k, int d, __nv_bfloat16* __restrict__ y) {
+    const int cpr = d >> 3;   // 8-column groups per row
+    for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < T * cpr;
+         i += (int64_t)gridDim.x * blockDim.x) {
+        const int64_t t = i / cpr;
+        const int c = (int)(i - t * cpr) * 8;
+        float acc[8];
+#pragma unroll
+        for (int q = 0; q < 8; ++q) acc[q] = 0.f;
+        for (int j = 0; j < k; ++j) {
+            const int r = inv[t * k + j];
+            if (r < 0 || r >= T * k) continue;   // a dropped slot contributes nothing
+            const float g = gate[t * k + j];
+            float v[8];
+            unpack_bf16x8(*reinterpret_cast<const uint4*>(rows + (int64_t)r * d + c), v);
+#pragma unroll
+            for (int q = 0; q < 8; ++q) acc[q] = fmaf(g, v[q], acc[q]);
+        }
+        if (shared) {
+            float v[8];
+            unpack_bf16x8(*reinterpret_cast<const uint4*>(shared + t * d + c), v);
+#pragma unroll
+            for (int q = 0; q < 8; ++q) acc[q] = fmaf(lambda, v[q], acc[q]);
+        }
+        uint4 u;
+        u.x = pack_bf16x2(acc[0], acc[1]);
+        u.y = pack_bf16x2(acc[2], acc[3]);
+        u.z = pack_bf16x2(acc[4], acc[5]);
+        u.w = pack_bf16x2(acc[6], acc[7]);
+        *reinterpret_cast<uint4*>(y + t * d + c) = u;
+    }
+}
+
+__global__ void wait_probe_kernel(DevStatus* st, uint64_t limit_ns) {
+    __shared__ __align__(8) uint64_t bar;
+    const uint32_t b = smem_u32(&bar);
+    if (threadIdx.x == 0) {
+        mbar_init(b, 1);
+        mbar_fence_init();
+    }
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        // Nothing ever arrives: the wait must give up after limit_ns.
+        if (!mbar_wait(b, 0, limit_ns, nullptr))
+            report(st, MOEVIE_ERR_TIMEOUT, SITE_TIMEOUT_PROBE, 0, 0);
+    }
+}
+
+int grid_for(int64_t n, int threads) {
+    int64_t g = (n + threads - 1) / threads;
+    if (g > 152 * 16) g = 152 * 16;
+    return (int)(g < 1 ? 1 : g);
+}
+
+}  // namespace
+
+cudaError_t launch_zero_f32(float* p, int64_t n, cudaStream_t s) {
+    const int64_t n4 = n / 4;   // callers pass multiples of 4
+    zero_f32_kernel<<<grid_for(n4, 256), 256, 0, s>>>(reinterpret_cast<float4*>(p), n4);
+    count_launches(1);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_f32_to_bf16(const float* src, __nv_bfloat16* dst, int64_t n, cudaStream_t s) {
+    const int64_t n8 = n / 8;   // callers pass multiples of 8
+    f32_to_bf16_kernel<<<grid_for(n8, 256), 256, 0, s>>>(reinterpret_cast<const float4*>(src),
+                                                          reinterpret_cast<uint4*>(dst), n8);
+    count_launches(1);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_combine(const __nv_bfloat16* rows, const int32_t* inv, const float* gate,
+                           const __nv_bfloat16* shared, float lambda, int64_t T, int k, int d,
+                           __nv_bfloat16* y, cudaStream_t s) {
+    const int64_t n = T * (d / 8);
+    combine_kernel<<<grid_for(n, 256), 256, 0, s>>>(rows, inv, gate, shared, lambda, T, k, d, y);
+    count_launches(1);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_wait_probe(DevStatus* st, uint64_t limit_ns, cudaStream_t s) {
+    wait_probe_kernel<<<1, 32, 0, s>>>(st, limit_ns);
+    count_launches(1);
+    return cudaGetLastError();
+}
+
+}  // namespace mv

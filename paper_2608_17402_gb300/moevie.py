@@ -1,0 +1,306 @@
+"""Python binding of ``libmoevie.so`` -- argument marshalling only.
+
+Every function below has the name of the C entry point it calls (``include/moevie.h``,
+``include/moevie_testing.h``), takes torch CUDA tensors, passes their device
+pointers and the current CUDA stream through ctypes, and raises
+:class:`MoevieError` on a non-OK status.  All computation happens in the CUDA
+library; there is no fallback of any kind: if the library is not built or no GPU
+is present, the call fails.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+from dataclasses import dataclass
+
+import torch
+
+_PKG = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_PKG, "libmoevie.so")
+_lib = None
+
+STATUS_NAMES = {0: "MOEVIE_OK", 1: "MOEVIE_ERR_INVALID_ARG", 2: "MOEVIE_ERR_UNSUPPORTED",
+                3: "MOEVIE_ERR_WORKSPACE", 4: "MOEVIE_ERR_CUDA", 5: "MOEVIE_ERR_TIMEOUT",
+                6: "MOEVIE_ERR_DEVICE"}
+C_ENTRY_POINTS = ("moevie_status_string", "moevie_version", "moevie_workspace_size",
+                  "moevie_workspace_init", "moevie_route", "moevie_permute", "moevie_expert_ffn",
+                  "moevie_shared_expert", "moevie_combine", "moevie_moe_forward",
+                  "moevie_get_device_status", "moevie_launch_count", "moevie_test_route_logits",
+                  "moevie_test_fallback_count", "moevie_test_expert_hidden",
+                  "moevie_test_moe_forward_events", "moevie_test_wait_timeout")
+
+
+class MoevieError(RuntimeError):
+    def __init__(self, fn, code):
+        super().__init__(f"{fn} returned {STATUS_NAMES.get(code, code)}")
+        self.code = code
+
+
+class _Layer(ctypes.Structure):
+    _fields_ = [("d", ctypes.c_int64), ("E", ctypes.c_int64), ("k", ctypes.c_int64),
+                ("h", ctypes.c_int64), ("h_s", ctypes.c_int64),
+                ("W_r", ctypes.c_void_p), ("b", ctypes.c_void_p), ("W1", ctypes.c_void_p),
+                ("W2", ctypes.c_void_p), ("Ws1", ctypes.c_void_p), ("Ws2", ctypes.c_void_p),
+                ("lam", ctypes.c_float)]
+
+
+class _Routing(ctypes.Structure):
+    _fields_ = [("idx", ctypes.c_void_p), ("gate", ctypes.c_void_p), ("counts", ctypes.c_void_p),
+                ("offsets", ctypes.c_void_p), ("perm", ctypes.c_void_p), ("inv", ctypes.c_void_p)]
+
+
+def load():
+    """Load the CUDA library (torch is imported first so both share one CUDA runtime)."""
+    global _lib
+    if _lib is not None:
+        return _lib
+    if not os.path.exists(LIB_PATH):
+        raise ImportError(f"{LIB_PATH} is not built; run `python -c \"import __graft_entry__ as g; "
+                          f"g.build()\"` first")
+    lib = ctypes.CDLL(LIB_PATH)
+    P, I64, SZ, F = ctypes.c_void_p, ctypes.c_int64, ctypes.c_size_t, ctypes.c_float
+    sig = {
+        "moevie_status_string": ([ctypes.c_int], ctypes.c_char_p),
+        "moevie_version": ([], ctypes.c_int),
+        "moevie_workspace_size": ([I64] * 6 + [P], ctypes.c_int),
+        "moevie_workspace_init": ([P, SZ, P], ctypes.c_int),
+        "moevie_route": ([P, P, P, I64, I64, I64, I64, P, P, P, SZ, P], ctypes.c_int),
+        "moevie_permute": ([P, I64, I64, I64, P, P, P, P, P, SZ, P], ctypes.c_int),
+        "moevie_expert_ffn": ([P, P, P, P, P, I64, I64, I64, I64, I64, P, P, SZ, P], ctypes.c_int),
+        "moevie_shared_expert": ([P, P, P, I64, I64, I64, P, P, SZ, P], ctypes.c_int),
+        "moevie_combine": ([P, P, P, P, F, I64, I64, I64, P, P], ctypes.c_int),
+        "moevie_moe_forward": ([P, P, I64, P, P, P, SZ, P], ctypes.c_int),
+        "moevie_get_device_status": ([P, P, P, P], ctypes.c_int),
+        "moevie_launch_count": ([], ctypes.c_uint64),
+        "moevie_test_route_logits": ([P, P, I64, I64, I64, P, P, SZ, P], ctypes.c_int),
+        "moevie_test_fallback_count": ([P, P, P], ctypes.c_int),
+        "moevie_test_expert_hidden": ([P, P, P, P, I64, I64, I64, I64, I64, P, P, SZ, P],
+                                      ctypes.c_int),
+        "moevie_test_moe_forward_events": ([P, P, I64, P, P, SZ, P, P, ctypes.c_int], ctypes.c_int),
+        "moevie_test_wait_timeout": ([P, SZ, ctypes.c_uint64, P], ctypes.c_int),
+    }
+    for name, (args, res) in sig.items():
+        fn = getattr(lib, name)
+        fn.argtypes = args
+        fn.restype = res
+    _lib = lib
+    return lib
+
+
+def _p(t):
+    return None if t is None else ctypes.c_void_p(t.data_ptr())
+
+
+def _stream(stream=None):
+    s = stream if stream is not None else torch.cuda.current_stream()
+    return ctypes.c_void_p(s.cuda_stream)
+
+
+def _call(name, *args):
+    rc = getattr(load(), name)(*args)
+    if rc != 0:
+        raise MoevieError(name, rc)
+
+
+def _want(t, dtype, name):
+    if not (t.is_cuda and t.dtype == dtype and t.is_contiguous()):
+        raise ValueError(f"{name}: expected a contiguous CUDA {dtype} tensor, got "
+                         f"{t.dtype} on {t.device} (contiguous={t.is_contiguous()})")
+    return t
+
+
+# ------------------------------------------------------------------ workspace
+
+def moevie_workspace_size(T_max, d, E, k, h, h_s=0) -> int:
+    out = ctypes.c_size_t(0)
+    _call("moevie_workspace_size", T_max, d, E, k, h, h_s, ctypes.byref(out))
+    return out.value
+
+
+class Workspace:
+    """Caller-owned device scratch for the layer (sized for up to ``T_max`` tokens)."""
+
+    def __init__(self, T_max, d, E, k, h, h_s=0, device="cuda", stream=None):
+        self.dims = (T_max, d, E, k, h, h_s)
+        self.nbytes = moevie_workspace_size(T_max, d, E, k, h, h_s)
+        self.buf = torch.empty(self.nbytes, dtype=torch.uint8, device=device)
+        moevie_workspace_init(self, stream)
+
+    @property
+    def ptr(self):
+        return ctypes.c_void_p(self.buf.data_ptr())
+
+
+def moevie_workspace_init(ws: Workspace, stream=None):
+    _call("moevie_workspace_init", ws.ptr, ws.nbytes, _stream(stream))
+
+
+def moevie_get_device_status(ws: Workspace, stream=None):
+    """Synchronises the stream; returns ``(code, [code, site, a, b])``."""
+    code = ctypes.c_int(0)
+    detail = (ctypes.c_int32 * 4)()
+    _call("moevie_get_device_status", ws.ptr, _stream(stream), ctypes.byref(code), detail)
+    return code.value, list(detail)
+
+
+# ----------------------------------------------------------------- the stages
+
+def moevie_route(x, W_r, b, k, ws: Workspace, idx=None, gate=None, stream=None):
+    _want(x, torch.bfloat16, "x")
+    _want(W_r, torch.float32, "W_r")
+    _want(b, torch.float32, "b")
+    T, d = x.shape
+    E = W_r.shape[1]
+    idx = idx if idx is not None else torch.empty((T, k), dtype=torch.int32, device=x.device)
+    gate = gate if gate is not None else torch.empty((T, k), dtype=torch.float32, device=x.device)
+    _call("moevie_route", _p(x), _p(W_r), _p(b), T, d, E, k, _p(idx), _p(gate), ws.ptr, ws.nbytes,
+          _stream(stream))
+    return idx, gate
+
+
+def moevie_permute(idx, E, ws: Workspace, stream=None):
+    _want(idx, torch.int32, "idx")
+    T, k = idx.shape
+    dev = idx.device
+    counts = torch.empty(E, dtype=torch.int32, device=dev)
+    offsets = torch.empty(E + 1, dtype=torch.int32, device=dev)
+    perm = torch.empty(T * k, dtype=torch.int32, device=dev)
+    inv = torch.empty(T * k, dtype=torch.int32, device=dev)
+    _call("moevie_permute", _p(idx), T, k, E, _p(counts), _p(offsets), _p(perm), _p(inv), ws.ptr,
+          ws.nbytes, _stream(stream))
+    return counts, offsets, perm, inv
+
+
+def moevie_expert_ffn(x, perm, offsets, W1, W2, k, ws: Workspace, out_rows=None, stream=None):
+    _want(x, torch.bfloat16, "x")
+    _want(W1, torch.bfloat16, "W1")
+    _want(W2, torch.bfloat16, "W2")
+    T, d = x.shape
+    E, _, h = W1.shape
+    out_rows = out_rows if out_rows is not None else torch.empty((T * k, d), dtype=torch.bfloat16,
+                                                                 device=x.device)
+    _call("moevie_expert_ffn", _p(x), _p(perm), _p(offsets), _p(W1), _p(W2), T, d, h, E, k,
+          _p(out_rows), ws.ptr, ws.nbytes, _stream(stream))
+    return out_rows
+
+
+def moevie_shared_expert(x, Ws1, Ws2, ws: Workspace, out=None, stream=None):
+    _want(x, torch.bfloat16, "x")
+    T, d = x.shape
+    hs = Ws1.shape[1]
+    out = out if out is not None else torch.empty((T, d), dtype=torch.bfloat16, device=x.device)
+    _call("moevie_shared_expert", _p(x), _p(Ws1), _p(Ws2), T, d, hs, _p(out), ws.ptr, ws.nbytes,
+          _stream(stream))
+    return out
+
+
+def moevie_combine(out_rows, inv, gate, k, shared_out=None, lam=1.0, y=None, stream=None):
+    _want(out_rows, torch.bfloat16, "out_rows")
+    T = gate.shape[0]
+    d = out_rows.shape[1]
+    y = y if y is not None else torch.empty((T, d), dtype=torch.bfloat16, device=out_rows.device)
+    _call("moevie_combine", _p(out_rows), _p(inv), _p(gate), _p(shared_out), float(lam), T, k, d,
+          _p(y), _stream(stream))
+    return y
+
+
+@dataclass
+class LayerWeights:
+    """Device weights of one layer (bf16 unless noted)."""
+    W_r: torch.Tensor           # fp32 [d, E]
+    b: torch.Tensor             # fp32 [E]
+    W1: torch.Tensor            # [E, d, h]
+    W2: torch.Tensor            # [E, h, d]
+    k: int
+    Ws1: torch.Tensor | None = None   # [d, h_s]
+    Ws2: torch.Tensor | None = None   # [h_s, d]
+    lam: float = 1.0
+
+    @property
+    def dims(self):
+        d, E = self.W_r.shape
+        h = self.W1.shape[2]
+        hs = 0 if self.Ws1 is None else self.Ws1.shape[1]
+        return d, E, self.k, h, hs
+
+    def c_struct(self) -> _Layer:
+        d, E, k, h, hs = self.dims
+        return _Layer(d, E, k, h, hs, self.W_r.data_ptr(), self.b.data_ptr(), self.W1.data_ptr(),
+                      self.W2.data_ptr(), 0 if self.Ws1 is None else self.Ws1.data_ptr(),
+                      0 if self.Ws2 is None else self.Ws2.data_ptr(), float(self.lam))
+
+
+def moevie_moe_forward(layer: LayerWeights, x, ws: Workspace, y=None, routing=False, stream=None):
+    """The fused layer forward.  With ``routing=True`` also returns a dict of the
+    routing by-products (idx, gate, counts, offsets, perm, inv)."""
+    _want(x, torch.bfloat16, "x")
+    T, d = x.shape
+    _, E, k, _, _ = layer.dims
+    dev = x.device
+    y = y if y is not None else torch.empty((T, d), dtype=torch.bfloat16, device=dev)
+    rt = None
+    rstruct = None
+    if routing:
+        rt = {"idx": torch.empty((T, k), dtype=torch.int32, device=dev),
+              "gate": torch.empty((T, k), dtype=torch.float32, device=dev),
+              "counts": torch.empty(E, dtype=torch.int32, device=dev),
+              "offsets": torch.empty(E + 1, dtype=torch.int32, device=dev),
+              "perm": torch.empty(T * k, dtype=torch.int32, device=dev),
+              "inv": torch.empty(T * k, dtype=torch.int32, device=dev)}
+        rstruct = _Routing(*(rt[n].data_ptr() for n in ("idx", "gate", "counts", "offsets", "perm",
+                                                         "inv")))
+    L = layer.c_struct()
+    _call("moevie_moe_forward", ctypes.byref(L), _p(x), T, _p(y),
+          ctypes.byref(rstruct) if rstruct is not None else None, ws.ptr, ws.nbytes,
+          _stream(stream))
+    return (y, rt) if routing else y
+
+
+def moevie_launch_count() -> int:
+    return int(load().moevie_launch_count())
+
+
+# ----------------------------------------------------------------- test hooks
+
+FORWARD_STAGES = ("route", "permute", "y_init", "up_gemm", "down_gemm", "finalize")
+
+
+def moevie_test_moe_forward_events(layer: LayerWeights, x, ws: Workspace, events, y=None,
+                                   stream=None):
+    """Forward that records the 7 stage-boundary events (torch.cuda.Event objects,
+    already recorded once so that their CUDA handles exist)."""
+    T, d = x.shape
+    y = y if y is not None else torch.empty((T, d), dtype=torch.bfloat16, device=x.device)
+    arr = (ctypes.c_void_p * 7)(*(ctypes.c_void_p(e.cuda_event) for e in events))
+    L = layer.c_struct()
+    _call("moevie_test_moe_forward_events", ctypes.byref(L), _p(x), T, _p(y), ws.ptr, ws.nbytes,
+          _stream(stream), arr, 7)
+    return y
+
+
+def moevie_test_route_logits(x, W_r, ws: Workspace, stream=None):
+    T, d = x.shape
+    E = W_r.shape[1]
+    s = torch.empty((T, E), dtype=torch.float32, device=x.device)
+    _call("moevie_test_route_logits", _p(x), _p(W_r), T, d, E, _p(s), ws.ptr, ws.nbytes,
+          _stream(stream))
+    return s
+
+
+def moevie_test_fallback_count(ws: Workspace, stream=None) -> int:
+    out = ctypes.c_int32(0)
+    _call("moevie_test_fallback_count", ws.ptr, _stream(stream), ctypes.byref(out))
+    return out.value
+
+
+def moevie_test_expert_hidden(x, perm, offsets, W1, k, ws: Workspace, stream=None):
+    T, d = x.shape
+    E, _, h = W1.shape
+    hidden = torch.empty((T * k, h), dtype=torch.bfloat16, device=x.device)
+    _call("moevie_test_expert_hidden", _p(x), _p(perm), _p(offsets), _p(W1), T, d, h, E, k,
+          _p(hidden), ws.ptr, ws.nbytes, _stream(stream))
+    return hidden
+
+
+def moevie_test_wait_timeout(ws: Workspace, limit_ns: int, stream=None):
+    _call("moevie_test_wait_timeout", ws.ptr, ws.nbytes, ctypes.c_uint64(limit_ns), _stream(stream))

@@ -1,0 +1,61 @@
+"""Helpers of the GPU parity tests: device copies of generator inputs and the
+output tolerance.  The CUDA path is always reached through the C ABI."""
+from __future__ import annotations
+
+import numpy as np
+import torch
+
+from paper_2608_17402_gb300 import moevie
+
+# Output tolerance of the layer (bf16 inputs, fp32 accumulation, bf16 hidden
+# activations and bf16 output): relative L2 error <= 1e-2 and every element within
+# 5e-2 of the RMS of the oracle output.
+REL_L2 = 1e-2
+MAX_ABS_OF_RMS = 5e-2
+# Oracle margins below this are not trusted to decide an exact tie-free order
+# between two independent fp64 evaluations (summation order, libm vs CUDA exp).
+MARGIN_PINNED = 1e-11
+
+
+def dev_bf16(a_u16: np.ndarray) -> torch.Tensor:
+    return torch.from_numpy(np.ascontiguousarray(a_u16).view(np.int16)).view(torch.bfloat16).cuda()
+
+
+def dev(a) -> torch.Tensor:
+    return torch.from_numpy(np.ascontiguousarray(a)).cuda()
+
+
+def to_np_f64(t: torch.Tensor) -> np.ndarray:
+    return t.detach().float().cpu().numpy().astype(np.float64)
+
+
+def layer_to_device(lay):
+    W = moevie.LayerWeights(
+        W_r=dev(lay.Wr), b=dev(lay.b), W1=dev_bf16(lay.W1), W2=dev_bf16(lay.W2), k=lay.cfg.k,
+        Ws1=None if lay.Ws1 is None else dev_bf16(lay.Ws1),
+        Ws2=None if lay.Ws2 is None else dev_bf16(lay.Ws2), lam=lay.cfg.lam)
+    return dev_bf16(lay.x), W
+
+
+def workspace_for(lay):
+    c = lay.cfg
+    return moevie.Workspace(c.T, c.d, c.E, c.k, c.h, c.h_s)
+
+
+def assert_close(got: np.ndarray, want: np.ndarray, what: str = "y"):
+    got = np.asarray(got, np.float64)
+    want = np.asarray(want, np.float64)
+    assert got.shape == want.shape, (got.shape, want.shape)
+    assert np.all(np.isfinite(got)), f"{what}: non-finite values"
+    rms = float(np.sqrt(np.mean(want ** 2))) if want.size else 0.0
+    err = got - want
+    rel = float(np.linalg.norm(err) / max(np.linalg.norm(want), 1e-300))
+    mx = float(np.abs(err).max()) if err.size else 0.0
+    assert rel <= REL_L2, f"{what}: relative L2 error {rel:.3e} > {REL_L2}"
+    assert mx <= MAX_ABS_OF_RMS * rms + 1e-30, f"{what}: max |err| {mx:.3e} > {MAX_ABS_OF_RMS} * RMS {rms:.3e}"
+    return rel, mx / max(rms, 1e-300)
+
+
+def check_status(ws):
+    code, detail = moevie.moevie_get_device_status(ws)
+    assert code == 0, f"device status {moevie.STATUS_NAMES.get(code, code)} detail={detail}"

@@ -1,0 +1,95 @@
+"""The C-ABI library loads and exports every entry point that include/*.h declares,
+and its host-side logic (validation, workspace sizing) behaves -- no GPU needed,
+no kernel is launched."""
+import ctypes
+import os
+import re
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+INCLUDE = os.path.join(ROOT, "include")
+
+
+def _declared():
+    names = set()
+    for f in os.listdir(INCLUDE):
+        if f.endswith(".h"):
+            src = open(os.path.join(INCLUDE, f)).read()
+            names |= set(re.findall(r"\b(moevie_\w+)\s*\(", src))
+    return names
+
+
+@pytest.fixture(scope="module")
+def lib():
+    from paper_2608_17402_gb300 import _build, moevie
+    _build.build()
+    return moevie.load()
+
+
+def test_every_declared_symbol_is_exported(lib):
+    declared = _declared()
+    assert {"moevie_route", "moevie_permute", "moevie_expert_ffn", "moevie_combine",
+            "moevie_moe_forward", "moevie_workspace_size"} <= declared
+    for name in sorted(declared):
+        assert hasattr(lib, name), name
+    from paper_2608_17402_gb300 import moevie
+    assert set(moevie.C_ENTRY_POINTS) == declared
+
+
+def test_status_strings_and_version(lib):
+    assert lib.moevie_status_string(0) == b"MOEVIE_OK"
+    assert lib.moevie_status_string(3) == b"MOEVIE_ERR_WORKSPACE"
+    assert lib.moevie_version() >= 100
+
+
+def _ws_size(lib, *dims):
+    out = ctypes.c_size_t(0)
+    rc = lib.moevie_workspace_size(*dims, ctypes.byref(out))
+    return rc, out.value
+
+
+def test_workspace_size_monotone_and_validated(lib):
+    rc, a = _ws_size(lib, 512, 768, 16, 2, 768, 0)
+    assert rc == 0 and a > 0
+    rc, b = _ws_size(lib, 1024, 768, 16, 2, 768, 0)
+    assert rc == 0 and b > a
+    rc, c = _ws_size(lib, 1024, 768, 16, 2, 768, 1024)
+    assert rc == 0 and c > b
+    assert _ws_size(lib, 512, 770, 16, 2, 768, 0)[0] == 2      # d % 8 != 0
+    assert _ws_size(lib, 512, 768, 16, 2, 760, 0)[0] == 2      # h % 16 != 0
+    assert _ws_size(lib, 512, 768, 16, 17, 768, 0)[0] == 2     # k > E
+    assert _ws_size(lib, 512, 768, 2048, 2, 768, 0)[0] == 2    # E > 1024
+    assert _ws_size(lib, -1, 768, 16, 2, 768, 0)[0] == 1
+    assert lib.moevie_workspace_size(1, 8, 1, 1, 16, 0, None) == 1
+
+
+def test_validation_happens_before_any_launch(lib):
+    P = ctypes.c_void_p
+    fake = P(0x1000)          # never dereferenced: every call below fails validation first
+    # sizes outside the supported set
+    assert lib.moevie_route(fake, fake, fake, 4, 12, 8, 2, fake, fake, fake, 1 << 20, None) == 2
+    # null pointers with T > 0
+    assert lib.moevie_route(None, fake, fake, 4, 16, 8, 2, fake, fake, fake, 1 << 20, None) == 1
+    # misaligned x
+    assert lib.moevie_route(P(0x1008), fake, fake, 4, 16, 8, 2, fake, fake, fake, 1 << 20, None) == 1
+    # workspace too small
+    assert lib.moevie_route(fake, fake, fake, 4, 16, 8, 2, fake, fake, fake, 16, None) == 3
+    # T == 0 is a valid no-op
+    assert lib.moevie_route(None, None, None, 0, 16, 8, 2, None, None, None, 0, None) == 0
+    assert lib.moevie_moe_forward(None, fake, 4, fake, None, fake, 1 << 20, None) == 1
+    assert lib.moevie_combine(fake, fake, fake, None, ctypes.c_float(1.0), 4, 2, 12, fake, None) == 2
+    assert lib.moevie_test_wait_timeout(fake, 256, 0, None) == 1
+
+
+def test_forward_rejects_bad_layer(lib):
+    from paper_2608_17402_gb300.moevie import _Layer
+    fake = 0x1000
+    L = _Layer(16, 8, 2, 32, 0, fake, fake, fake, fake, 0, 0, 1.0)
+    rc = lib.moevie_moe_forward(ctypes.byref(L), ctypes.c_void_p(fake), 4, ctypes.c_void_p(fake),
+                                None, ctypes.c_void_p(fake), 16, None)
+    assert rc == 3   # workspace too small
+    L.h = 40         # h % 16 != 0
+    rc = lib.moevie_moe_forward(ctypes.byref(L), ctypes.c_void_p(fake), 4, ctypes.c_void_p(fake),
+                                None, ctypes.c_void_p(fake), 1 << 30, None)
+    assert rc == 2

@@ -1,0 +1,99 @@
+"""Router parity (Eqs. 1, 7, 4-5): GPU selection bit-exact against the fp64 oracle,
+gates within fp32 rounding, through the C ABI."""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+import workloads
+from paper_2608_17402_gb300 import moevie
+from tests._gpu import MARGIN_PINNED, check_status, dev, dev_bf16
+
+pytestmark = pytest.mark.gpu
+
+
+def _route_case(x, Wr, b, k):
+    T, d = x.shape
+    E = Wr.shape[1]
+    ws = moevie.Workspace(T, d, E, k, 16)
+    idx, gate = moevie.moevie_route(dev_bf16(x), dev(Wr), dev(b), k, ws)
+    nfb = moevie.moevie_test_fallback_count(ws)
+    check_status(ws)
+    return idx.cpu().numpy(), gate.cpu().numpy().astype(np.float64), nfb
+
+
+def _check_against_oracle(x, Wr, b, k):
+    idx, gate, nfb = _route_case(x, Wr, b, k)
+    oidx, ogate, margin = oracle.route(x, Wr, b, k)
+    pinned = margin > MARGIN_PINNED
+    assert pinned.mean() > 0.999, "too many oracle near-ties to pin the selection"
+    assert np.array_equal(idx[pinned], oidx[pinned]), np.argwhere(np.any(idx != oidx, axis=1))[:8]
+    np.testing.assert_allclose(gate, ogate, rtol=0, atol=1e-5)
+    assert np.all(np.diff(idx, axis=1) > 0)
+    return nfb
+
+
+@pytest.mark.parametrize("T,d,E,k", [(1, 16, 8, 2), (37, 64, 16, 2), (129, 128, 64, 8),
+                                     (200, 96, 1, 1), (64, 32, 4, 4), (50, 64, 1024, 4),
+                                     (300, 256, 256, 8), (77, 48, 33, 5)])
+def test_route_small_shapes(T, d, E, k):
+    rng = np.random.default_rng(T * 7 + E)
+    x = workloads.f32_to_bf16_bits(rng.standard_normal((T, d)).astype(np.float32))
+    Wr = (rng.standard_normal((d, E)) * 0.02).astype(np.float32)
+    b = rng.uniform(-0.1, 0.1, E).astype(np.float32)
+    _check_against_oracle(x, Wr, b, k)
+
+
+def test_route_exact_ties_go_to_lower_id():
+    """Duplicated W_r columns with equal bias give exactly equal keys; the fast path
+    cannot certify them and the exact re-decision must pick the lower id."""
+    rng = np.random.default_rng(5)
+    T, d, E, k = 256, 64, 16, 3
+    x = workloads.f32_to_bf16_bits(rng.standard_normal((T, d)).astype(np.float32))
+    Wr = (rng.standard_normal((d, E)) * 0.3).astype(np.float32)
+    b = rng.uniform(-0.1, 0.1, E).astype(np.float32)
+    for a, c in [(1, 9), (4, 5), (0, 15)]:
+        Wr[:, c] = Wr[:, a]
+        b[c] = b[a]
+    idx, gate, nfb = _route_case(x, Wr, b, k)
+    oidx, ogate, _ = oracle.route(x, Wr, b, k)
+    assert np.array_equal(idx, oidx)
+    assert nfb > 0
+    np.testing.assert_allclose(gate, ogate, rtol=0, atol=1e-5)
+
+
+def test_route_bias_only():
+    """W_r = 0: every key is 1/2 + b; ties in b resolve to the lower id; gates 1/k."""
+    T, d, E, k = 40, 32, 12, 4
+    x = workloads.f32_to_bf16_bits(np.random.default_rng(1).standard_normal((T, d)).astype(np.float32))
+    Wr = np.zeros((d, E), np.float32)
+    b = np.array([0.0625, -0.5, 0.25, 0.25, 0.0, 0.25, 0.125, 0.25, -0.25, 0.0625, 0.5, 0.0],
+                 np.float32)
+    idx, gate, _ = _route_case(x, Wr, b, k)
+    want = np.array([2, 3, 5, 10])   # 0.5 (id 10), then 0.25 at ids 2, 3, 5 (7 left out)
+    assert np.all(idx == want)
+    np.testing.assert_allclose(gate, 0.25, rtol=0, atol=1e-7)
+
+
+@pytest.mark.parametrize("name", ["c0", "c1", "c2", "c3", "c4"])
+def test_route_full_configs(name):
+    lay = workloads.make_layer(workloads.CONFIGS[name])
+    nfb = _check_against_oracle(lay.x, lay.Wr, lay.b, lay.cfg.k)
+    print(f"{name}: {nfb} of {lay.cfg.T} tokens re-decided exactly")
+
+
+@pytest.mark.parametrize("name", ["c1", "c4"])
+def test_fast_logit_error_within_bound(name):
+    """The fp32 logits stay far inside the error bound the router certifies with
+    (ROUTE_TAU_C = 64 units of 2^-24 |x| max|w|): measured max below 1/4 of it."""
+    lay = workloads.make_layer(workloads.CONFIGS[name])
+    T = min(lay.cfg.T, 8192)
+    x, Wr = lay.x[:T], lay.Wr
+    ws = moevie.Workspace(T, lay.cfg.d, lay.cfg.E, 1, 16)
+    s = moevie.moevie_test_route_logits(dev_bf16(x), dev(Wr), ws).cpu().numpy().astype(np.float64)
+    so = oracle.logits(x, Wr)
+    xf = workloads.bf16_bits_to_f32(x).astype(np.float64)
+    scale = 2.0 ** -24 * np.linalg.norm(xf, axis=1)[:, None] * np.linalg.norm(Wr.astype(np.float64), axis=0).max()
+    ratio = np.abs(s - so) / scale
+    print(f"{name}: max |s_fast - s| = {ratio.max():.2f} units of 2^-24 |x| max|w|")
+    assert ratio.max() < 64 / 4

@@ -70,11 +70,14 @@ CONFIGS = {
 
 
 def f32_to_bf16_bits(a: np.ndarray) -> np.ndarray:
-    """Round fp32 values to the nearest bf16 (ties to even); return the bit patterns."""
-    a = np.ascontiguousarray(a, dtype=np.float32)
-    u = a.view(np.uint32).astype(np.uint64)
-    u = u + 0x7FFF + ((u >> 16) & 1)
-    return (u >> 16).astype(np.uint16)
+    """Round fp32 values to the nearest bf16 (ties to even); return the bit patterns.
+
+    The rounding is torch's fp32 -> bf16 conversion on the CPU (round to nearest,
+    ties to even: add 0x7FFF plus the lowest kept bit, drop the low 16 bits), used
+    here only because it is multithreaded."""
+    import torch
+    t = torch.from_numpy(np.ascontiguousarray(a, dtype=np.float32))
+    return t.to(torch.bfloat16).view(torch.int16).numpy().view(np.uint16).copy()
 
 
 def bf16_bits_to_f32(b: np.ndarray) -> np.ndarray:
@@ -99,7 +102,7 @@ class LayerInputs:
 def _normal_bf16(rng: np.random.Generator, shape, std: float) -> np.ndarray:
     v = rng.standard_normal(size=shape, dtype=np.float32)
     if std != 1.0:
-        v *= np.float32(std)
+        np.multiply(v, np.float32(std), out=v)
     return f32_to_bf16_bits(v)
 
 
