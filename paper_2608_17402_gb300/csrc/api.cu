@@ -28,9 +28,9 @@ inline bool a16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) =
 // the order is fixed, so a workspace sized for the whole layer also serves each
 // stage (which passes 0 for the sizes it does not use).
 struct Layout {
-    size_t status, xnorm2, wnorm2, logits, fb_tokens;
-    size_t idx, gate, hist, counts, offsets, tile_off, perm, inv, row_tok, row_gate;
-    size_t off_s, tile_s, H, Hs, yacc;
+    size_t status, xnorm, wnorm, wpart, wsplit, logits, fb_tokens;
+    size_t idx, gate, hist, counts, offsets, tiles, n_tiles, perm, inv, row_tok, row_gate;
+    size_t H, Hs, yacc;
     size_t total;
 };
 
@@ -43,24 +43,26 @@ Layout make_layout(int64_t T, int64_t d, int64_t E, int64_t k, int64_t h, int64_
         return at;
     };
     const int64_t n = T * k;
-    const int64_t nchunks = (n + PERM_CHUNK - 1) / PERM_CHUNK;
+    const int64_t Ep = route_epad((int)E);
+    const int64_t nchunks_max = (n + 255) / 256;   // chunks are at least 256 slots
     L.status = take(sizeof(DevStatus));
-    L.xnorm2 = take(4 * T);
-    L.wnorm2 = take(4 * E);
-    L.logits = take(4 * T * E);
+    L.xnorm = take(4 * T);
+    L.wnorm = take(4 * E);
+    L.wpart = take(4 * (int64_t)route_split_parts((int)d) * Ep);
+    L.wsplit = take(2 * 3 * (int64_t)route_dpad((int)d) * Ep);
+    L.logits = take(4 * T * Ep);
     L.fb_tokens = take(4 * T);
     L.idx = take(4 * n);
     L.gate = take(4 * n);
-    L.hist = take(4 * nchunks * E);
+    L.hist = take(4 * nchunks_max * E);
     L.counts = take(4 * E);
     L.offsets = take(4 * (E + 1));
-    L.tile_off = take(4 * (E + 1));
+    L.tiles = take(16 * max_mtiles(n, E));
+    L.n_tiles = take(4);
     L.perm = take(4 * n);
     L.inv = take(4 * n);
     L.row_tok = take(4 * n);
     L.row_gate = take(4 * n);
-    L.off_s = take(8);
-    L.tile_s = take(8);
     L.H = take(2 * n * h);
     L.Hs = take(2 * T * hs);
     L.yacc = take(4 * T * d);
@@ -77,8 +79,8 @@ moevie_status check_sizes(int64_t T, int64_t d, int64_t E, int64_t k, int64_t h,
     if (T < 0 || d <= 0 || E <= 0 || k <= 0 || h < 0 || hs < 0) return MOEVIE_ERR_INVALID_ARG;
     if (d % 8 != 0 || h % 16 != 0 || hs % 16 != 0) return MOEVIE_ERR_UNSUPPORTED;
     if (k > E || E > 1024) return MOEVIE_ERR_UNSUPPORTED;
-    if (T * k >= (int64_t(1) << 31) || T >= (int64_t(1) << 31) || d >= (int64_t(1) << 24) ||
-        h >= (int64_t(1) << 24) || hs >= (int64_t(1) << 24))
+    if (T * k >= (int64_t(1) << 31) || T * route_epad((int)E) >= (int64_t(1) << 40) ||
+        d >= (int64_t(1) << 24) || h >= (int64_t(1) << 24) || hs >= (int64_t(1) << 24))
         return MOEVIE_ERR_UNSUPPORTED;
     return MOEVIE_OK;
 }
@@ -103,26 +105,28 @@ inline moevie_status cuda_status(cudaError_t e) { return e == cudaSuccess ? MOEV
         if (_e != cudaSuccess) return MOEVIE_ERR_CUDA;   \
     } while (0)
 
-// One grouped GEMM launch: D = A[rows] . W[g], W bf16 [G][K][N].
+// One grouped GEMM launch: D = A[rows] . W[g], W bf16 [G][K][N] (row stride N_ld).
 struct GemmSpec {
     const void* A;
     int64_t lda;
+    int64_t a_cols;       // valid columns of an A row (0 = K)
     const int32_t* a_rows;
     int a_div;
+    int a_kperiod;
     int64_t a_nrows;      // rows of A
-    int64_t m_total;      // GEMM rows (segment total bound)
-    int64_t o_nrows;      // rows of yacc
-    const int32_t* offsets;
-    const int32_t* tile_off;
+    int64_t m_total;      // GEMM rows
+    const int4* tiles;    // nullptr: one dense group of m_total rows
+    const int32_t* n_tiles;
     int G;
-    int64_t max_mtiles;   // host bound on the number of m-tiles
     const void* W;
     int K, N;
+    int64_t N_ld;         // inner extent of W (>= N), 0 = N
     int epi;
     void* out;
     int64_t ldo;
     float* yacc;
     int64_t ldy;
+    int64_t o_nrows;      // rows of yacc
     const int32_t* o_rows;
     int o_div;
     const float* row_scale;
@@ -132,17 +136,20 @@ struct GemmSpec {
 moevie_status run_gemm(const GemmSpec& g, DevStatus* st, cudaStream_t s) {
     GemmArgs a;
     memset(&a, 0, sizeof a);
-    if (!make_weight_tmap(&a.tmB, g.W, g.N, g.K, g.G)) return MOEVIE_ERR_CUDA;
+    const int64_t n_ld = g.N_ld > 0 ? g.N_ld : g.N;
+    if (!make_weight_tmap(&a.tmB, g.W, n_ld, g.K, g.G)) return MOEVIE_ERR_CUDA;
+    if (!g.a_rows && !make_rows_tmap(&a.tmA, g.A, g.a_cols > 0 ? g.a_cols : g.K, g.a_nrows, g.lda))
+        return MOEVIE_ERR_CUDA;
     a.A = static_cast<const __nv_bfloat16*>(g.A);
     a.lda = g.lda;
     a.a_rows = g.a_rows;
     a.a_div = g.a_div > 0 ? g.a_div : 1;
+    a.a_kperiod = g.a_kperiod;
     a.a_nrows = g.a_nrows;
     a.m_total = g.m_total;
-    a.max_mtiles = g.max_mtiles;
-    a.o_nrows = g.o_nrows;
-    a.offsets = g.offsets;
-    a.tile_off = g.tile_off;
+    a.tiles = g.tiles;
+    a.n_tiles_dev = g.n_tiles;
+    a.max_mtiles = g.tiles ? max_mtiles(g.m_total, g.G) : (g.m_total + GM_BM - 1) / GM_BM;
     a.G = g.G;
     a.K = g.K;
     a.N = g.N;
@@ -154,16 +161,121 @@ moevie_status run_gemm(const GemmSpec& g, DevStatus* st, cudaStream_t s) {
     a.ldo = g.ldo;
     a.yacc = g.yacc;
     a.ldy = g.ldy;
+    a.o_nrows = g.o_nrows;
     a.o_rows = g.o_rows;
     a.o_div = g.o_div > 0 ? g.o_div : 1;
     a.row_scale = g.row_scale;
     a.scale = g.scale;
     a.status = st;
     a.limit_ns = WAIT_LIMIT_NS;
-    const int64_t work = g.max_mtiles * a.n_ntiles;
-    const int sms = num_sms();
-    const int grid = (int)(work < sms ? (work > 0 ? work : 1) : sms);
+    const int64_t work = a.max_mtiles * a.n_ntiles;     // one CTA pair per work item at most
+    const int sms = num_sms() & ~1;
+    const int grid = (int)(2 * work < sms ? (work > 0 ? 2 * work : 2) : sms);
     return cuda_status(launch_grouped_gemm(a, grid, s));
+}
+
+// Router (Eqs. 1, 7, 4-5): exact bf16 split of W_r, tensor-core logits,
+// certified top-k with exact re-decision of near ties.
+moevie_status route_impl(const void* x, const float* W_r, const float* b, int64_t T, int64_t d,
+                         int64_t E, int64_t k, int32_t* idx, float* gate, const Layout& L,
+                         void* ws, cudaStream_t s, bool logits_only = false,
+                         float* logits_out = nullptr) {
+    DevStatus* st = at<DevStatus>(ws, L.status);
+    const int Ep = route_epad((int)E);
+    __nv_bfloat16* wsplit = at<__nv_bfloat16>(ws, L.wsplit);
+    float* wnorm = at<float>(ws, L.wnorm);
+    float* logits = logits_out ? logits_out : at<float>(ws, L.logits);
+    MV_TRY(launch_route_split(W_r, (int)d, (int)E, wsplit, at<float>(ws, L.wpart), wnorm, s));
+    const int64_t dp = route_dpad((int)d);
+    GemmSpec g{};
+    g.A = x;
+    g.lda = d;
+    g.a_cols = d;
+    g.a_kperiod = (int)dp;         // K = 3 dp: x is read three times, once per piece
+    g.a_nrows = T;
+    g.m_total = T;
+    g.G = 1;
+    g.W = wsplit;
+    g.K = (int)(3 * dp);
+    g.N = (int)E;
+    g.N_ld = Ep;
+    g.epi = EPI_STORE_F32;
+    g.yacc = logits;
+    g.ldy = Ep;
+    g.o_nrows = T;
+    g.scale = 1.0f;
+    moevie_status c = run_gemm(g, st, s);
+    if (c != MOEVIE_OK || logits_only) return c;
+    MV_TRY(launch_route_select(static_cast<const __nv_bfloat16*>(x), W_r, b, logits, Ep, wnorm,
+                               (int)T, (int)d, (int)E, (int)k, idx, gate,
+                               at<int32_t>(ws, L.fb_tokens), at<float>(ws, L.xnorm), st,
+                               num_sms(), s));
+    return MOEVIE_OK;
+}
+
+moevie_status expert_up(const void* x, const int32_t* a_rows, int a_div, const int4* tiles,
+                        const int32_t* n_tiles, const void* W1, int64_t T, int64_t d, int64_t h,
+                        int64_t E, int64_t k, void* hidden, DevStatus* st, cudaStream_t s) {
+    GemmSpec g{};
+    g.A = x;
+    g.lda = d;
+    g.a_rows = a_rows;
+    g.a_div = a_div;
+    g.a_nrows = T;
+    g.m_total = T * k;
+    g.tiles = tiles;
+    g.n_tiles = n_tiles;
+    g.G = (int)E;
+    g.W = W1;
+    g.K = (int)d;
+    g.N = (int)h;
+    g.epi = EPI_GELU_BF16;
+    g.out = hidden;
+    g.ldo = h;
+    return run_gemm(g, st, s);
+}
+
+// Shared expert as one dense group of all T rows.  Writes either a bf16 output
+// (out != NULL) or lambda * S(x) as the first value of the fp32 y accumulator.
+moevie_status shared_expert(const void* x, const void* Ws1, const void* Ws2, int64_t T, int64_t d,
+                            int64_t hs, void* out, float* yacc, float lambda, const Layout& L,
+                            void* ws, DevStatus* st, cudaStream_t s) {
+    void* Hs = at<void>(ws, L.Hs);
+    GemmSpec g{};
+    g.A = x;
+    g.lda = d;
+    g.a_nrows = T;
+    g.m_total = T;
+    g.G = 1;
+    g.W = Ws1;
+    g.K = (int)d;
+    g.N = (int)hs;
+    g.epi = EPI_GELU_BF16;
+    g.out = Hs;
+    g.ldo = hs;
+    moevie_status c = run_gemm(g, st, s);
+    if (c != MOEVIE_OK) return c;
+    GemmSpec g2{};
+    g2.A = Hs;
+    g2.lda = hs;
+    g2.a_nrows = T;
+    g2.m_total = T;
+    g2.G = 1;
+    g2.W = Ws2;
+    g2.K = (int)hs;
+    g2.N = (int)d;
+    if (out) {
+        g2.epi = EPI_STORE_BF16;
+        g2.out = out;
+        g2.ldo = d;
+    } else {
+        g2.epi = EPI_STORE_F32;
+        g2.yacc = yacc;
+        g2.ldy = d;
+        g2.o_nrows = T;
+        g2.scale = lambda;
+    }
+    return run_gemm(g2, st, s);
 }
 
 }  // namespace
@@ -183,7 +295,9 @@ const char* moevie_status_string(moevie_status s) {
     }
 }
 
-int moevie_version(void) { return 100; }
+int moevie_version(void) { return 200; }
+
+uint64_t moevie_launch_count(void) { return g_launches.load(std::memory_order_relaxed); }
 
 moevie_status moevie_workspace_size(int64_t T_max, int64_t d, int64_t E, int64_t k, int64_t h,
                                     int64_t h_s, size_t* bytes) {
@@ -207,17 +321,9 @@ moevie_status moevie_route(const void* x, const float* W_r, const float* b, int6
     if (T == 0) return MOEVIE_OK;
     if (!x || !W_r || !b || !idx || !gate || !ws) return MOEVIE_ERR_INVALID_ARG;
     if (!a16(x) || !a16(ws)) return MOEVIE_ERR_INVALID_ARG;
-    const Layout L = make_layout(T, 0, E, k, 0, 0);
+    const Layout L = make_layout(T, d, E, k, 0, 0);
     if (ws_bytes < L.total) return MOEVIE_ERR_WORKSPACE;
-    cudaStream_t s = static_cast<cudaStream_t>(stream);
-    DevStatus* st = at<DevStatus>(ws, L.status);
-    RouteBufs rb{at<float>(ws, L.logits), at<float>(ws, L.xnorm2), at<float>(ws, L.wnorm2),
-                 at<int32_t>(ws, L.fb_tokens)};
-    const __nv_bfloat16* xb = static_cast<const __nv_bfloat16*>(x);
-    MV_TRY(launch_route_logits(xb, W_r, (int)T, (int)d, (int)E, rb, st, s));
-    MV_TRY(launch_route_select(xb, W_r, b, (int)T, (int)d, (int)E, (int)k, idx, gate, rb, st,
-                               num_sms(), s));
-    return MOEVIE_OK;
+    return route_impl(x, W_r, b, T, d, E, k, idx, gate, L, ws, static_cast<cudaStream_t>(stream));
 }
 
 moevie_status moevie_permute(const int32_t* idx, int64_t T, int64_t k, int64_t E, int32_t* counts,
@@ -237,34 +343,11 @@ moevie_status moevie_permute(const int32_t* idx, int64_t T, int64_t k, int64_t E
         return MOEVIE_OK;
     }
     DevStatus* st = at<DevStatus>(ws, L.status);
-    MV_TRY(launch_permute(idx, T * k, (int)k, (int)E, GM_BM, nullptr, at<int32_t>(ws, L.hist),
-                          counts, offsets, at<int32_t>(ws, L.tile_off), perm, inv, nullptr,
-                          nullptr, st, s));
+    const int chunk = perm_chunk(T * k, num_sms());
+    MV_TRY(launch_permute(idx, T * k, (int)k, (int)E, GM_BM, chunk, nullptr, at<int32_t>(ws, L.hist),
+                          counts, offsets, at<int4>(ws, L.tiles), at<int32_t>(ws, L.n_tiles), perm,
+                          inv, nullptr, nullptr, st, s));
     return MOEVIE_OK;
-}
-
-static moevie_status expert_up(const void* x, const int32_t* perm, const int32_t* offsets,
-                               const int32_t* tile_off, const void* W1, int64_t T, int64_t d,
-                               int64_t h, int64_t E, int64_t k, void* hidden, DevStatus* st,
-                               cudaStream_t s) {
-    GemmSpec g{};
-    g.A = x;
-    g.lda = d;
-    g.a_rows = perm;
-    g.a_div = (int)k;
-    g.a_nrows = T;
-    g.m_total = T * k;
-    g.offsets = offsets;
-    g.tile_off = tile_off;
-    g.G = (int)E;
-    g.max_mtiles = (T * k + GM_BM - 1) / GM_BM + E;
-    g.W = W1;
-    g.K = (int)d;
-    g.N = (int)h;
-    g.epi = EPI_GELU_BF16;
-    g.out = hidden;
-    g.ldo = h;
-    return run_gemm(g, st, s);
 }
 
 moevie_status moevie_expert_ffn(const void* x, const int32_t* perm, const int32_t* offsets,
@@ -281,20 +364,20 @@ moevie_status moevie_expert_ffn(const void* x, const int32_t* perm, const int32_
     if (ws_bytes < L.total) return MOEVIE_ERR_WORKSPACE;
     cudaStream_t s = static_cast<cudaStream_t>(stream);
     DevStatus* st = at<DevStatus>(ws, L.status);
-    int32_t* tile_off = at<int32_t>(ws, L.tile_off);
+    int4* tiles = at<int4>(ws, L.tiles);
+    int32_t* n_tiles = at<int32_t>(ws, L.n_tiles);
     void* H = at<void>(ws, L.H);
-    MV_TRY(launch_tile_prefix(offsets, (int)E, GM_BM, tile_off, s));
-    c = expert_up(x, perm, offsets, tile_off, W1, T, d, h, E, k, H, st, s);
+    MV_TRY(launch_tile_table(offsets, (int)E, GM_BM, tiles, n_tiles, s));
+    c = expert_up(x, perm, (int)k, tiles, n_tiles, W1, T, d, h, E, k, H, st, s);
     if (c != MOEVIE_OK) return c;
     GemmSpec g{};
     g.A = H;
     g.lda = h;
     g.a_nrows = T * k;
     g.m_total = T * k;
-    g.offsets = offsets;
-    g.tile_off = tile_off;
+    g.tiles = tiles;
+    g.n_tiles = n_tiles;
     g.G = (int)E;
-    g.max_mtiles = (T * k + GM_BM - 1) / GM_BM + E;
     g.W = W2;
     g.K = (int)h;
     g.N = (int)d;
@@ -302,59 +385,6 @@ moevie_status moevie_expert_ffn(const void* x, const int32_t* perm, const int32_
     g.out = out_rows;
     g.ldo = d;
     return run_gemm(g, st, s);
-}
-
-// Shared expert as one group of all T rows (identity gather).  Writes either a
-// bf16 output (out != NULL) or lambda * S(x) as the first value of the fp32 y
-// accumulator.
-static moevie_status shared_expert(const void* x, const void* Ws1, const void* Ws2, int64_t T,
-                                   int64_t d, int64_t hs, void* out, float* yacc, float lambda,
-                                   const Layout& L, void* ws, DevStatus* st, cudaStream_t s) {
-    int32_t* off_s = at<int32_t>(ws, L.off_s);
-    int32_t* tile_s = at<int32_t>(ws, L.tile_s);
-    void* Hs = at<void>(ws, L.Hs);
-    MV_TRY(launch_single_group(off_s, tile_s, (int)T, GM_BM, s));
-    GemmSpec g{};
-    g.A = x;
-    g.lda = d;
-    g.a_nrows = T;
-    g.m_total = T;
-    g.offsets = off_s;
-    g.tile_off = tile_s;
-    g.G = 1;
-    g.max_mtiles = (T + GM_BM - 1) / GM_BM;
-    g.W = Ws1;
-    g.K = (int)d;
-    g.N = (int)hs;
-    g.epi = EPI_GELU_BF16;
-    g.out = Hs;
-    g.ldo = hs;
-    moevie_status c = run_gemm(g, st, s);
-    if (c != MOEVIE_OK) return c;
-    GemmSpec g2{};
-    g2.A = Hs;
-    g2.lda = hs;
-    g2.a_nrows = T;
-    g2.m_total = T;
-    g2.o_nrows = T;
-    g2.offsets = off_s;
-    g2.tile_off = tile_s;
-    g2.G = 1;
-    g2.max_mtiles = (T + GM_BM - 1) / GM_BM;
-    g2.W = Ws2;
-    g2.K = (int)hs;
-    g2.N = (int)d;
-    if (out) {
-        g2.epi = EPI_STORE_BF16;
-        g2.out = out;
-        g2.ldo = d;
-    } else {
-        g2.epi = EPI_STORE_F32;
-        g2.yacc = yacc;
-        g2.ldy = d;
-        g2.scale = lambda;
-    }
-    return run_gemm(g2, st, s);
 }
 
 moevie_status moevie_shared_expert(const void* x, const void* Ws1, const void* Ws2, int64_t T,
@@ -413,26 +443,23 @@ static moevie_status forward_impl(const moevie_layer* Lr, const void* x, int64_t
     int32_t* perm = r.perm ? r.perm : at<int32_t>(ws, L.perm);
     int32_t* inv = r.inv ? r.inv : at<int32_t>(ws, L.inv);
     if (!a16(idx)) return MOEVIE_ERR_INVALID_ARG;
-    int32_t* tile_off = at<int32_t>(ws, L.tile_off);
+    int4* tiles = at<int4>(ws, L.tiles);
+    int32_t* n_tiles = at<int32_t>(ws, L.n_tiles);
     int32_t* row_tok = at<int32_t>(ws, L.row_tok);
     float* row_gate = at<float>(ws, L.row_gate);
     float* yacc = at<float>(ws, L.yacc);
-    const __nv_bfloat16* xb = static_cast<const __nv_bfloat16*>(x);
     auto mark = [&](int i) -> cudaError_t {
         return events ? cudaEventRecord(static_cast<cudaEvent_t>(events[i]), s) : cudaSuccess;
     };
 
     MV_TRY(mark(0));
     // 1. router (Eqs. 1, 7, 4-5)
-    RouteBufs rb{at<float>(ws, L.logits), at<float>(ws, L.xnorm2), at<float>(ws, L.wnorm2),
-                 at<int32_t>(ws, L.fb_tokens)};
-    MV_TRY(launch_route_logits(xb, Lr->W_r, (int)T, (int)d, (int)E, rb, st, s));
-    MV_TRY(launch_route_select(xb, Lr->W_r, Lr->b, (int)T, (int)d, (int)E, (int)k, idx, gate, rb,
-                               st, num_sms(), s));
+    if ((c = route_impl(x, Lr->W_r, Lr->b, T, d, E, k, idx, gate, L, ws, s)) != MOEVIE_OK) return c;
     MV_TRY(mark(1));
-    // 2. expert-major order (Algorithm 1, phase 1) + per-row token and gate
-    MV_TRY(launch_permute(idx, T * k, (int)k, (int)E, GM_BM, gate, at<int32_t>(ws, L.hist),
-                          r.counts, offsets, tile_off, perm, inv, row_tok, row_gate, st, s));
+    // 2. expert-major order (Algorithm 1, phase 1), per-row token and gate, m-tile table
+    const int chunk = perm_chunk(T * k, num_sms());
+    MV_TRY(launch_permute(idx, T * k, (int)k, (int)E, GM_BM, chunk, gate, at<int32_t>(ws, L.hist),
+                          r.counts, offsets, tiles, n_tiles, perm, inv, row_tok, row_gate, st, s));
     MV_TRY(mark(2));
     // 3. y accumulator: lambda * shared expert, or zero
     if (hs > 0) {
@@ -443,24 +470,9 @@ static moevie_status forward_impl(const moevie_layer* Lr, const void* x, int64_t
     }
     MV_TRY(mark(3));
     // 4. grouped up-projection, token gather in the operand load, GELU epilogue
-    GemmSpec up{};
-    up.A = x;
-    up.lda = d;
-    up.a_rows = row_tok;
-    up.a_div = 1;
-    up.a_nrows = T;
-    up.m_total = T * k;
-    up.offsets = offsets;
-    up.tile_off = tile_off;
-    up.G = (int)E;
-    up.max_mtiles = (T * k + GM_BM - 1) / GM_BM + E;
-    up.W = Lr->W1;
-    up.K = (int)d;
-    up.N = (int)h;
-    up.epi = EPI_GELU_BF16;
-    up.out = at<void>(ws, L.H);
-    up.ldo = h;
-    if ((c = run_gemm(up, st, s)) != MOEVIE_OK) return c;
+    if ((c = expert_up(x, row_tok, 1, tiles, n_tiles, Lr->W1, T, d, h, E, k, at<void>(ws, L.H),
+                       st, s)) != MOEVIE_OK)
+        return c;
     MV_TRY(mark(4));
     // 5. grouped down-projection, epilogue: gate * row added into y (scatter-add)
     GemmSpec dn{};
@@ -468,17 +480,16 @@ static moevie_status forward_impl(const moevie_layer* Lr, const void* x, int64_t
     dn.lda = h;
     dn.a_nrows = T * k;
     dn.m_total = T * k;
-    dn.o_nrows = T;
-    dn.offsets = offsets;
-    dn.tile_off = tile_off;
+    dn.tiles = tiles;
+    dn.n_tiles = n_tiles;
     dn.G = (int)E;
-    dn.max_mtiles = up.max_mtiles;
     dn.W = Lr->W2;
     dn.K = (int)h;
     dn.N = (int)d;
     dn.epi = EPI_ADD_F32;
     dn.yacc = yacc;
     dn.ldy = d;
+    dn.o_nrows = T;
     dn.o_rows = row_tok;
     dn.o_div = 1;
     dn.row_scale = row_gate;
@@ -495,8 +506,6 @@ moevie_status moevie_moe_forward(const moevie_layer* layer, const void* x, int64
                                  void* stream) {
     return forward_impl(layer, x, T, y, routing, ws, ws_bytes, stream, nullptr, 0);
 }
-
-uint64_t moevie_launch_count(void) { return g_launches.load(std::memory_order_relaxed); }
 
 moevie_status moevie_get_device_status(const void* ws, void* stream, moevie_status* out,
                                        int32_t* detail) {
@@ -517,13 +526,12 @@ moevie_status moevie_test_route_logits(const void* x, const float* W_r, int64_t 
     moevie_status c = check_sizes(T, d, E, 1, 0, 0);
     if (c != MOEVIE_OK) return c;
     if (T == 0) return MOEVIE_OK;
-    if (!x || !W_r || !s_out || !ws || !a16(x) || !a16(ws)) return MOEVIE_ERR_INVALID_ARG;
-    const Layout L = make_layout(T, 0, E, 1, 0, 0);
+    if (!x || !W_r || !s_out || !ws || !a16(x) || !a16(ws) || !a16(s_out)) return MOEVIE_ERR_INVALID_ARG;
+    const Layout L = make_layout(T, d, E, 1, 0, 0);
     if (ws_bytes < L.total) return MOEVIE_ERR_WORKSPACE;
-    RouteBufs rb{s_out, at<float>(ws, L.xnorm2), at<float>(ws, L.wnorm2), at<int32_t>(ws, L.fb_tokens)};
-    return cuda_status(launch_route_logits(static_cast<const __nv_bfloat16*>(x), W_r, (int)T, (int)d,
-                                           (int)E, rb, at<DevStatus>(ws, L.status),
-                                           static_cast<cudaStream_t>(stream)));
+    // s_out receives the padded [T, route_epad(E)] logits
+    return route_impl(x, W_r, nullptr, T, d, E, 1, nullptr, nullptr, L, ws,
+                      static_cast<cudaStream_t>(stream), true, s_out);
 }
 
 moevie_status moevie_test_fallback_count(const void* ws, void* stream, int32_t* out) {
@@ -548,15 +556,16 @@ moevie_status moevie_test_expert_hidden(const void* x, const int32_t* perm, cons
     const Layout L = make_layout(T, 0, E, k, 0, 0);
     if (ws_bytes < L.total) return MOEVIE_ERR_WORKSPACE;
     cudaStream_t s = static_cast<cudaStream_t>(stream);
-    int32_t* tile_off = at<int32_t>(ws, L.tile_off);
-    MV_TRY(launch_tile_prefix(offsets, (int)E, GM_BM, tile_off, s));
-    return expert_up(x, perm, offsets, tile_off, W1, T, d, h, E, k, hidden,
+    int4* tiles = at<int4>(ws, L.tiles);
+    int32_t* n_tiles = at<int32_t>(ws, L.n_tiles);
+    MV_TRY(launch_tile_table(offsets, (int)E, GM_BM, tiles, n_tiles, s));
+    return expert_up(x, perm, (int)k, tiles, n_tiles, W1, T, d, h, E, k, hidden,
                      at<DevStatus>(ws, L.status), s);
 }
 
 moevie_status moevie_test_moe_forward_events(const moevie_layer* layer, const void* x, int64_t T,
-                                            void* y, void* ws, size_t ws_bytes, void* stream,
-                                            void* const* events, int n_events) {
+                                             void* y, void* ws, size_t ws_bytes, void* stream,
+                                             void* const* events, int n_events) {
     if (!events) return MOEVIE_ERR_INVALID_ARG;
     return forward_impl(layer, x, T, y, nullptr, ws, ws_bytes, stream, events, n_events);
 }

@@ -1,29 +1,43 @@
-// gemm.cu -- persistent grouped GEMM on tcgen05 / TMEM for the expert FFN of the
-// MoE-ViE layer (App. B, Algorithm 1, Kernels 1 and 2), sm_103a.
+// gemm.cu -- persistent grouped GEMM on tcgen05 / TMEM with 2-SM MMAs, for the
+// MoE-ViE layer (App. B, Algorithm 1, Kernels 1 and 2; also the router logits),
+// sm_103a.
 //
 // One launch computes, for every group g (an expert) and every row r of its
-// segment [offsets[g], offsets[g+1]):   D[r, :] = A[row(r), :] . B[g]   (fp32)
-// and hands each 128 x BN tile to a fused epilogue:
+// segment:   D[r, :] = A[row(r), :] . B[g]   (bf16 inputs, fp32 accumulation)
+// and hands each tile to a fused epilogue:
 //   EPI_GELU_BF16   hidden = bf16(GELU(D))                      (Kernel 1, GELU)
 //   EPI_STORE_BF16  out    = bf16(D)
 //   EPI_ADD_F32     y[tok(r)] += gate(r) * D   (Kernel 2: routing weight + scatter-add)
-//   EPI_STORE_F32   y[tok(r)]  = scale * D     (first writer of y, e.g. the shared expert)
+//   EPI_STORE_F32   y[tok(r)]  = scale * D     (first writer of y; router logits)
 //
-// Work items are (m-tile, n-tile) pairs of all groups, in group-major order with
-// the n-tile fastest; a persistent CTA per SM walks them with a static stride.
-// There is no host read of segment sizes: the m-tile list comes from the device
-// prefix tile_off, written by the permute step.
+// CTA pairs.  The grid is made of clusters of two CTAs on neighbouring SMs.  A
+// pair computes a 256 x BN tile with tcgen05.mma.cta_group::2 (M = 256): CTA r
+// holds rows 128 r .. 128 r + 127 of A and columns r BN/2 .. (r+1) BN/2 - 1 of B
+// in its shared memory, and receives rows 128 r .. of D in its TMEM.  Per SM this
+// halves the B traffic of a 128 x BN tile, so shared memory bandwidth (the MMA
+// reads what TMA writes) no longer caps the tensor pipe.  CTA 0 of the pair (the
+// leader) issues every MMA; its commits arrive on the barriers of both CTAs.
 //
-// Warp roles (320 threads, one CTA per SM):
-//   warps 0-3  epilogue: tcgen05.ld of the fp32 accumulator rows (warp w owns TMEM
-//              lanes 32w..32w+31), fused math, global stores / vector atomics
-//   warp 4     TMEM allocation; lane 0 issues tcgen05.mma (M=128, N=BN, K=16)
-//   warp 5     lane 0 issues TMA loads of B tiles (weights, 128-byte swizzle)
-//   warps 6-9  gather A rows with 16-byte cp.async straight into the 128-byte
-//              swizzled K-major layout (the token gather fused into the operand load)
-// Shared memory: GM_STAGES x (A 128x64 + B 64x256) bf16 stages; TMEM: two fp32
-// accumulators of 256 columns, so the epilogue of one tile overlaps the
-// main loop of the next.
+// Work items are (256-row m-tile, n-tile) pairs in group-major order with the
+// n-tile fastest; a persistent pair walks them with a static stride.  The m-tiles
+// come from a device tile table {group, first row, rows <= 256} written by the
+// permute step (no host read of segment sizes), or, for one dense group, from
+// arithmetic.
+//
+// Warp roles (448 threads per CTA, one CTA per SM):
+//   warps 0-7   epilogue: tcgen05.ld of the CTA's 128 accumulator rows (warp w:
+//               TMEM lanes 32 (w%4)..+31, every other 16-column chunk), fused math,
+//               sector-wide stores (fp32 results pass a per-warp smem transpose)
+//   warp 8      TMEM allocation (both CTAs, jointly); leader lane 0 issues the MMAs
+//   warp 9      lane 0: TMA loads of the B half and, for contiguous A rows, of A;
+//               the leader posts the byte count of both CTAs on its full barrier
+//   warps 10-13 token gather: 16-byte cp.async of A rows straight into the 128-byte
+//               swizzled K-major layout, two stages in flight per thread; after a
+//               stage's copies land and are fenced to the async proxy, each warp
+//               arrives once (leader: on its full barrier; peer: on a local barrier
+//               that the peer's idle MMA-warp lane forwards to the leader)
+// Shared memory: 6 stages x (A 128x64 + B 64x128) bf16; TMEM: two fp32 accumulators
+// of 256 columns, so the epilogue of one tile overlaps the main loop of the next.
 //
 // Operand layouts (tcgen05 shared-memory descriptors, 128-byte swizzle):
 //   A  K-major : row r of the 128x64 tile at byte r*128, 16-byte chunk c stored
@@ -41,6 +55,81 @@ namespace mv {
 
 namespace {
 
+constexpr int A_LAG = 2;             // cp.async stages in flight per gather thread
+constexpr int STG_LD = GM_STG_LD;
+
+// ------------------------------------------------------------ pair helpers
+
+__device__ __forceinline__ uint32_t cluster_rank() {
+    uint32_t r;
+    asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+    return r;
+}
+// Address of the same shared-memory object in CTA `rank` of the cluster.
+__device__ __forceinline__ uint32_t peer_addr(uint32_t addr, uint32_t rank) {
+    uint32_t r;
+    asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(addr), "r"(rank));
+    return r;
+}
+__device__ __forceinline__ void cluster_sync() {
+    asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::
+                     : "memory");
+}
+__device__ __forceinline__ void mbar_arrive_remote(uint32_t bar_cluster) {
+    asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(bar_cluster)
+                 : "memory");
+}
+// TMA loads into this CTA's shared memory that complete on a barrier of either CTA
+// of the pair.
+__device__ __forceinline__ void tma_load_3d_pair(uint32_t dst, const CUtensorMap* tm,
+                                                 uint32_t bar_cluster, int c0, int c1, int c2) {
+    asm volatile(
+        "cp.async.bulk.tensor.3d.cta_group::2.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
+        " [%0], [%1, {%2, %3, %4}], [%5];" ::"r"(dst),
+        "l"(tm), "r"(c0), "r"(c1), "r"(c2), "r"(bar_cluster)
+        : "memory");
+}
+__device__ __forceinline__ void tma_load_2d_pair(uint32_t dst, const CUtensorMap* tm,
+                                                 uint32_t bar_cluster, int c0, int c1) {
+    asm volatile(
+        "cp.async.bulk.tensor.2d.cta_group::2.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
+        " [%0], [%1, {%2, %3}], [%4];" ::"r"(dst),
+        "l"(tm), "r"(c0), "r"(c1), "r"(bar_cluster)
+        : "memory");
+}
+__device__ __forceinline__ void tmem_alloc_pair(uint32_t slot, uint32_t ncols) {
+    asm volatile("tcgen05.alloc.cta_group::2.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(slot),
+                 "r"(ncols)
+                 : "memory");
+}
+__device__ __forceinline__ void tmem_relinquish_pair() {
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::2.sync.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void tmem_dealloc_pair(uint32_t taddr, uint32_t ncols) {
+    asm volatile("tcgen05.dealloc.cta_group::2.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(ncols)
+                 : "memory");
+}
+__device__ __forceinline__ void tc_mma_bf16_pair(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc,
+                                                 uint32_t idesc, uint32_t accumulate) {
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "setp.ne.b32 p, %4, 0;\n\t"
+        "tcgen05.mma.cta_group::2.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
+        "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
+        : "memory");
+}
+// Arrive once on the barrier at shared offset `bar` of both CTAs when all prior
+// tcgen05 operations of this thread have completed.
+__device__ __forceinline__ void tc_commit_pair(uint32_t bar) {
+    asm volatile(
+        "tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64"
+        " [%0], %1;" ::"r"(bar),
+        "h"((uint16_t)3)
+        : "memory");
+}
+
+// ------------------------------------------------------------------ tiles
+
 struct Tile {
     int g, row0, nrows, n0;
 };
@@ -48,34 +137,53 @@ struct Tile {
 __device__ __forceinline__ Tile decode_tile(const GemmArgs& p, int64_t w) {
     const int mt = (int)(w / p.n_ntiles);
     const int nt = (int)(w - (int64_t)mt * p.n_ntiles);
-    int lo = 0, hi = p.G - 1;   // largest g with tile_off[g] <= mt (skips empty groups)
-    while (lo < hi) {
-        const int mid = (lo + hi + 1) >> 1;
-        if (__ldg(p.tile_off + mid) <= mt) lo = mid;
-        else hi = mid - 1;
-    }
     Tile t;
-    t.g = lo;
-    const int seg0 = __ldg(p.offsets + lo), seg1 = __ldg(p.offsets + lo + 1);
-    t.row0 = seg0 + (mt - __ldg(p.tile_off + lo)) * GM_BM;
-    t.nrows = min(GM_BM, seg1 - t.row0);
-    if ((int64_t)t.row0 + t.nrows > p.m_total) {   // inconsistent offsets: write nothing
-        report(p.status, MOEVIE_ERR_DEVICE, SITE_GEMM_TILES, t.row0, seg1);
+    if (p.tiles) {
+        const int4 d = __ldg(p.tiles + mt);
+        t.g = d.x;
+        t.row0 = d.y;
+        t.nrows = d.z;
+    } else {   // one dense group of m_total rows
+        t.g = 0;
+        t.row0 = mt * GM_BM;
+        const int64_t left = p.m_total - t.row0;
+        t.nrows = (int)(left < GM_BM ? left : GM_BM);
+    }
+    if (t.nrows < 0 || t.nrows > GM_BM || t.g < 0 || t.g >= p.G ||
+        (int64_t)t.row0 + t.nrows > p.m_total) {
+        report(p.status, MOEVIE_ERR_DEVICE, SITE_GEMM_TILES, t.row0, t.nrows);
         t.nrows = 0;
+        t.g = 0;
     }
     t.n0 = nt * p.BN;
     return t;
 }
 
+// GELU(u) = u/2 (1 + erf(u / sqrt 2)) with erf from Abramowitz & Stegun 7.1.26:
+//   erf(z) = 1 - t (a1 + t (a2 + t (a3 + t (a4 + t a5)))) e^{-z^2},  t = 1 / (1 + p z),
+// z >= 0, |error| <= 1.5e-7 (the hidden activation is then rounded to bf16, 2^-9
+// relative).  With q = 1 - erf(|u| / sqrt 2), 1 + erf(u / sqrt 2) is 2 - q for
+// u >= 0 and q for u < 0, which avoids the cancellation of the erf form.
 __device__ __forceinline__ float gelu_erf(float u) {
-    return 0.5f * u * (1.0f + erff(u * 0.70710678118654752f));
+    const float z = fabsf(u) * 0.70710678118654752f;
+    const float t = __fdividef(1.0f, fmaf(0.3275911f, z, 1.0f));
+    float poly = fmaf(1.061405429f, t, -1.453152027f);
+    poly = fmaf(poly, t, 1.421413741f);
+    poly = fmaf(poly, t, -0.284496736f);
+    poly = fmaf(poly, t, 0.254829592f);
+    const float q = poly * t * __expf(-z * z);
+    return 0.5f * u * (u >= 0.0f ? 2.0f - q : q);
 }
 
 struct Smem {
     uint32_t a0, b0;          // shared addresses of stage 0
     uint32_t full, empty;     // barrier arrays (8 bytes apart)
+    uint32_t afull;           // peer CTA: its gather warps' copies of a stage have landed
     uint32_t tfull, tempty;
     uint32_t drain;
+    float* stage_out;         // epilogue transpose buffers, 32 x STG_LD floats per warp
+    uint32_t rank;            // rank of this CTA in its pair
+    int64_t pair, npairs;     // pair index and count
 };
 
 __device__ __forceinline__ void set_abort(volatile int* flag, DevStatus* st, int site, int a,
@@ -84,89 +192,171 @@ __device__ __forceinline__ void set_abort(volatile int* flag, DevStatus* st, int
     report(st, MOEVIE_ERR_TIMEOUT, site, a, b);
 }
 
-// ------------------------------------------------------------- producers
+// Rows of tile t held by this CTA: 128 rank .. 128 rank + rows_half(t) - 1.
+__device__ __forceinline__ int rows_half(const Tile& t, uint32_t rank) {
+    const int r = t.nrows - (int)rank * GM_HALF;
+    return r < 0 ? 0 : (r > GM_HALF ? GM_HALF : r);
+}
 
-__device__ void producer_a(const GemmArgs& p, const Smem& sm, int64_t n_work,
-                           volatile int* abort_flag) {
-    const int pt = threadIdx.x - 6 * 32;   // 0..127
-    const int c = pt & 7, rb = pt >> 3;     // 16-byte chunk, first row
+// --------------------------------------------------------------- producers
+
+// TMA producer (warp 9, lane 0): the CTA's half of B, and A when its rows are
+// contiguous.  The leader posts the byte count of both CTAs on its full barrier.
+__device__ void producer_tma(const GemmArgs& p, const Smem& sm, int64_t n_work,
+                             volatile int* abort_flag) {
+    tma_prefetch_desc(&p.tmB);
+    const bool gather = p.a_rows != nullptr;
+    if (!gather) tma_prefetch_desc(&p.tmA);
+    const uint32_t half_n = (uint32_t)p.BN / 2;
+    const uint32_t nboxh = (half_n + 63) / 64;
+    const uint32_t cta_bytes = nboxh * GM_BK * 128 + (gather ? 0u : (uint32_t)GM_A_BYTES);
+    const uint32_t full_leader = peer_addr(sm.full, 0);
     int s = 0;
     uint32_t ph = 0;
-    int pend = -1;                          // stage whose arrival waits for its copies
-    bool ok = true;
-    for (int64_t w = blockIdx.x; w < n_work && ok; w += gridDim.x) {
-        const Tile t = decode_tile(p, w);
-        const __nv_bfloat16* src[8];
-#pragma unroll
-        for (int j = 0; j < 8; ++j) {
-            const int r = rb + 16 * j;
-            if (r < t.nrows) {
-                const int gr = t.row0 + r;
-                const int ar = p.a_rows ? __ldg(p.a_rows + gr) / p.a_div : gr;
-                if (ar >= 0 && ar < p.a_nrows) {
-                    src[j] = p.A + (int64_t)ar * p.lda;
-                } else {   // out-of-range gather index: zero row, device error
-                    report(p.status, MOEVIE_ERR_DEVICE, SITE_GEMM_A_ROW, gr, ar);
-                    src[j] = nullptr;
-                }
-            } else {
-                src[j] = nullptr;
-            }
-        }
+    int64_t w = sm.pair;
+    Tile t{};
+    if (w < n_work) t = decode_tile(p, w);
+    for (; w < n_work; w += sm.npairs) {
+        const int64_t wn = w + sm.npairs;
+        Tile tn{};
+        if (wn < n_work) tn = decode_tile(p, wn);
         for (int kb = 0; kb < p.num_kb; ++kb) {
             if (!mbar_wait(sm.empty + 8 * s, ph ^ 1u, p.limit_ns, abort_flag)) {
-                set_abort(abort_flag, p.status, SITE_GEMM_WAIT_EMPTY, blockIdx.x, 0);
-                ok = false;
-                break;
+                set_abort(abort_flag, p.status, SITE_GEMM_WAIT_EMPTY, (int)sm.pair, 1);
+                return;
             }
-            const uint32_t dst0 = sm.a0 + s * GM_A_BYTES;
-            const int col = kb * GM_BK + c * 8;
-            const bool col_ok = col < p.K;
-#pragma unroll
-            for (int j = 0; j < 8; ++j) {
-                const int r = rb + 16 * j;
-                const uint32_t dst = dst0 + r * 128 + ((c ^ (r & 7)) << 4);
-                const bool v = col_ok && src[j] != nullptr;
-                cp_async16(dst, v ? (const void*)(src[j] + col) : (const void*)p.A, v ? 16u : 0u);
+            const uint32_t bar = full_leader + 8 * s;
+            if (sm.rank == 0) mbar_arrive_expect_tx(sm.full + 8 * s, 2 * cta_bytes);
+            const uint32_t b_dst = sm.b0 + s * GM_B_BYTES;
+            const int kk = kb * GM_BK;
+            for (uint32_t j = 0; j < nboxh; ++j)
+                tma_load_3d_pair(b_dst + j * (GM_BK * 128), &p.tmB, bar,
+                                 t.n0 + (int)(sm.rank * half_n + 64 * j), kk, t.g);
+            if (!gather) {
+                const int col = p.a_kperiod ? kk % p.a_kperiod : kk;
+                tma_load_2d_pair(sm.a0 + s * GM_A_BYTES, &p.tmA, bar, col,
+                                 t.row0 + (int)sm.rank * GM_HALF);
             }
-            cp_async_commit();
-            if (pend >= 0) {
-                cp_async_wait<1>();
-                fence_proxy_async_smem();
-                mbar_arrive(sm.full + 8 * pend);
-            }
-            pend = s;
             if (++s == GM_STAGES) {
                 s = 0;
                 ph ^= 1u;
             }
         }
-    }
-    cp_async_wait<0>();
-    if (pend >= 0) {
-        fence_proxy_async_smem();
-        mbar_arrive(sm.full + 8 * pend);
+        t = tn;
     }
 }
 
-__device__ void producer_b(const GemmArgs& p, const Smem& sm, int64_t n_work,
-                           volatile int* abort_flag) {
-    tma_prefetch_desc(&p.tmB);
-    const uint32_t stage_bytes = (uint32_t)p.nbox * GM_BK * 128;
+// A row pointers of this thread's 8 rows (r = rb + 16 j of the CTA's half).
+__device__ __forceinline__ void gather_rows(const GemmArgs& p, const Tile& t, uint32_t rank,
+                                            int rb, const __nv_bfloat16* (&src)[8]) {
+    const int nh = rows_half(t, rank);
+    int idx[8];
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+        const int r = rb + 16 * j;
+        const int gr = t.row0 + (int)rank * GM_HALF + r;
+        idx[j] = (r < nh) ? __ldg(p.a_rows + gr) / p.a_div : -1;
+    }
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+        const int r = rb + 16 * j;
+        if (r < nh && idx[j] >= 0 && idx[j] < p.a_nrows) {
+            src[j] = p.A + (int64_t)idx[j] * p.lda;
+        } else {
+            if (r < nh)
+                report(p.status, MOEVIE_ERR_DEVICE, SITE_GEMM_A_ROW, t.row0 + (int)rank * GM_HALF + r,
+                       idx[j]);
+            src[j] = nullptr;
+        }
+    }
+}
+
+// Token gather (warps 10-13): each thread copies 8 16-byte chunks per stage; once
+// the copies of a stage have landed and are fenced to the async proxy, each warp
+// arrives once at CTA scope.
+__device__ void producer_gather(const GemmArgs& p, const Smem& sm, int64_t n_work,
+                                volatile int* abort_flag) {
+    const int pt = threadIdx.x - GM_WARP_GATHER * 32;   // 0..127
+    const int lane = threadIdx.x & 31;
+    const int c = pt & 7, rb = pt >> 3;                  // 16-byte chunk, first row
+    // leader: its own full barrier; peer: its afull barrier (forwarded by gather_forwarder)
+    const uint32_t arrive_bar = sm.rank == 0 ? sm.full : sm.afull;
     int s = 0;
     uint32_t ph = 0;
-    for (int64_t w = blockIdx.x; w < n_work; w += gridDim.x) {
-        const Tile t = decode_tile(p, w);
+    int pend[A_LAG];
+    int npend = 0;
+    bool ok = true;
+    int64_t w = sm.pair;
+    const __nv_bfloat16* src[8];
+    if (w < n_work) gather_rows(p, decode_tile(p, w), sm.rank, rb, src);
+    for (; w < n_work && ok; w += sm.npairs) {
+        const int64_t wn = w + sm.npairs;
+        const __nv_bfloat16* nsrc[8];
+        if (wn < n_work) gather_rows(p, decode_tile(p, wn), sm.rank, rb, nsrc);
         for (int kb = 0; kb < p.num_kb; ++kb) {
-            if (!mbar_wait(sm.empty + 8 * s, ph ^ 1u, p.limit_ns, abort_flag)) {
-                set_abort(abort_flag, p.status, SITE_GEMM_WAIT_EMPTY, blockIdx.x, 1);
+            int good = 1;
+            if (lane == 0) good = mbar_wait(sm.empty + 8 * s, ph ^ 1u, p.limit_ns, abort_flag);
+            good = __shfl_sync(0xffffffffu, good, 0);
+            if (!good) {
+                if (lane == 0) set_abort(abort_flag, p.status, SITE_GEMM_WAIT_EMPTY, (int)sm.pair, 0);
+                ok = false;
+                break;
+            }
+            const uint32_t dst0 = sm.a0 + s * GM_A_BYTES;
+            const int kk = kb * GM_BK + c * 8;
+            const bool col_ok = kk < p.K;
+#pragma unroll
+            for (int j = 0; j < 8; ++j) {
+                const int r = rb + 16 * j;
+                const uint32_t dst = dst0 + r * 128 + ((c ^ (r & 7)) << 4);
+                const bool v = col_ok && src[j] != nullptr;
+                cp_async16(dst, v ? (const void*)(src[j] + kk) : (const void*)p.A, v ? 16u : 0u);
+            }
+            cp_async_commit();
+            if (npend == A_LAG) {
+                cp_async_wait<A_LAG>();
+                fence_proxy_async_smem();
+                __syncwarp();
+                if (lane == 0) mbar_arrive(arrive_bar + 8 * pend[0]);
+#pragma unroll
+                for (int q = 0; q + 1 < A_LAG; ++q) pend[q] = pend[q + 1];
+                --npend;
+            }
+            pend[npend++] = s;
+            if (++s == GM_STAGES) {
+                s = 0;
+                ph ^= 1u;
+            }
+        }
+        if (wn < n_work) {
+#pragma unroll
+            for (int j = 0; j < 8; ++j) src[j] = nsrc[j];
+        }
+    }
+    cp_async_wait<0>();
+    fence_proxy_async_smem();
+    __syncwarp();
+    if (lane == 0)
+        for (int q = 0; q < npend; ++q) mbar_arrive(arrive_bar + 8 * pend[q]);
+}
+
+// Peer CTA, warp 8, lane 0 (idle otherwise): once the peer's four gather warps have
+// arrived on its local afull barrier for a stage, forward one cluster-scope arrival
+// to the leader's full barrier.  A release at cluster scope costs the issuing thread
+// a wait for its outstanding memory operations; this thread has none, the gather
+// threads (with copies in flight) only release at CTA scope.
+__device__ void gather_forwarder(const GemmArgs& p, const Smem& sm, int64_t n_work,
+                                 volatile int* abort_flag) {
+    const uint32_t full_leader = peer_addr(sm.full, 0);
+    int s = 0;
+    uint32_t ph = 0;
+    for (int64_t w = sm.pair; w < n_work; w += sm.npairs) {
+        for (int kb = 0; kb < p.num_kb; ++kb) {
+            if (!mbar_wait(sm.afull + 8 * s, ph, p.limit_ns, abort_flag)) {
+                set_abort(abort_flag, p.status, SITE_GEMM_WAIT_FULL, (int)sm.pair, -1 - kb);
                 return;
             }
-            const uint32_t bar = sm.full + 8 * s;
-            mbar_arrive_expect_tx(bar, stage_bytes);
-            const uint32_t dst0 = sm.b0 + s * GM_B_BYTES;
-            for (int j = 0; j < p.nbox; ++j)
-                tma_load_3d(dst0 + j * (GM_BK * 128), &p.tmB, bar, t.n0 + 64 * j, kb * GM_BK, t.g);
+            mbar_arrive_remote(full_leader + 8 * s);
             if (++s == GM_STAGES) {
                 s = 0;
                 ph ^= 1u;
@@ -177,18 +367,19 @@ __device__ void producer_b(const GemmArgs& p, const Smem& sm, int64_t n_work,
 
 // ------------------------------------------------------------------- MMA
 
+// Leader CTA, warp 8, lane 0.
 __device__ void mma_issuer(const GemmArgs& p, const Smem& sm, uint32_t tmem, int64_t n_work,
                            volatile int* abort_flag) {
-    const uint32_t idesc = idesc_bf16_f32(GM_BM, p.BN, false, true);
+    const uint32_t idesc = idesc_bf16_f32(2 * GM_HALF, p.BN, false, true);
     int s = 0;
     uint32_t ph = 0;
     int it = 0;
     bool issued = false;
-    for (int64_t w = blockIdx.x; w < n_work; w += gridDim.x, ++it) {
+    for (int64_t w = sm.pair; w < n_work; w += sm.npairs, ++it) {
         const int acc = it & 1;
         const uint32_t aph = (uint32_t)(it >> 1) & 1u;
         if (!mbar_wait(sm.tempty + 8 * acc, aph ^ 1u, p.limit_ns, abort_flag)) {
-            set_abort(abort_flag, p.status, SITE_GEMM_WAIT_TEMPTY, blockIdx.x, it);
+            set_abort(abort_flag, p.status, SITE_GEMM_WAIT_TEMPTY, (int)sm.pair, it);
             break;
         }
         tc_fence_after();
@@ -196,7 +387,7 @@ __device__ void mma_issuer(const GemmArgs& p, const Smem& sm, uint32_t tmem, int
         bool ok = true;
         for (int kb = 0; kb < p.num_kb; ++kb) {
             if (!mbar_wait(sm.full + 8 * s, ph, p.limit_ns, abort_flag)) {
-                set_abort(abort_flag, p.status, SITE_GEMM_WAIT_FULL, blockIdx.x, kb);
+                set_abort(abort_flag, p.status, SITE_GEMM_WAIT_FULL, (int)sm.pair, kb);
                 ok = false;
                 break;
             }
@@ -207,96 +398,127 @@ __device__ void mma_issuer(const GemmArgs& p, const Smem& sm, uint32_t tmem, int
             for (int kk = 0; kk < GM_BK / 16; ++kk) {
                 const uint64_t ad = smem_desc_sw128(a_addr + kk * 32, 16, 1024);
                 const uint64_t bd = smem_desc_sw128(b_addr + kk * 2048, 8192, 1024);
-                tc_mma_bf16(d_tmem, ad, bd, idesc, (kb | kk) != 0 ? 1u : 0u);
+                tc_mma_bf16_pair(d_tmem, ad, bd, idesc, (kb | kk) != 0 ? 1u : 0u);
             }
             issued = true;
-            tc_commit(sm.empty + 8 * s);
+            tc_commit_pair(sm.empty + 8 * s);
             if (++s == GM_STAGES) {
                 s = 0;
                 ph ^= 1u;
             }
         }
         if (!ok) break;
-        tc_commit(sm.tfull + 8 * acc);
+        tc_commit_pair(sm.tfull + 8 * acc);
     }
     // Every tcgen05.mma must be complete before TMEM is released.
     if (issued) {
-        tc_commit(sm.drain);
+        tc_commit_pair(sm.drain);
         if (!mbar_wait(sm.drain, 0, p.limit_ns, nullptr))
-            report(p.status, MOEVIE_ERR_TIMEOUT, SITE_GEMM_DRAIN, blockIdx.x, 0);
+            report(p.status, MOEVIE_ERR_TIMEOUT, SITE_GEMM_DRAIN, (int)sm.pair, 0);
     }
 }
 
 // -------------------------------------------------------------- epilogue
 
+// Warp w reads TMEM lanes 32 (w % 4) .. +31 (its rows of the CTA's half) and the
+// 16-column chunks c = w / 4, w / 4 + 2, ... of each tile.  bf16 outputs: every
+// thread stores its row's 16 values as one 32-byte sector.  fp32 outputs (y
+// accumulator, logits): a shared-memory transpose first, so that 4 lanes cover 64
+// contiguous bytes of a row and each vector reduction / store touches whole sectors.
+// When a warp has read its last chunk of the accumulator it arrives (once) on the
+// leader's tempty barrier.
 __device__ void epilogue(const GemmArgs& p, const Smem& sm, uint32_t tmem, int64_t n_work,
                          volatile int* abort_flag) {
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int row = warp * 32 + lane;
+    const int quad = warp & 3, half = warp >> 2;
+    float* stg = sm.stage_out + warp * (32 * STG_LD);
+    const bool to_f32 = (p.epi == EPI_ADD_F32 || p.epi == EPI_STORE_F32);
+    const int rsub = lane >> 2, c4 = (lane & 3) * 4;   // transposed: rows 8 i + rsub, columns c4..c4+3
+    const int nchunk = (p.BN + 15) / 16;
+    const uint32_t tempty_leader = peer_addr(sm.tempty, 0);
     int it = 0;
-    for (int64_t w = blockIdx.x; w < n_work; w += gridDim.x, ++it) {
+    for (int64_t w = sm.pair; w < n_work; w += sm.npairs, ++it) {
         const Tile t = decode_tile(p, w);
         const int acc = it & 1;
         const uint32_t aph = (uint32_t)(it >> 1) & 1u;
+        const int myrow = quad * 32 + lane;
+        const int gr = t.row0 + (int)sm.rank * GM_HALF + myrow;
+        int64_t tok = gr;
+        float sc = p.scale;
+        bool ok_row = myrow < rows_half(t, sm.rank);
+        if (ok_row) {
+            if (p.o_rows) tok = __ldg(p.o_rows + gr) / p.o_div;
+            if (p.row_scale) sc = __ldg(p.row_scale + gr);
+            if (to_f32 && (tok < 0 || tok >= p.o_nrows)) {
+                report(p.status, MOEVIE_ERR_DEVICE, SITE_GEMM_OUT_ROW, gr, (int)tok);
+                ok_row = false;
+            }
+        }
         if (!mbar_wait(sm.tfull + 8 * acc, aph, p.limit_ns, abort_flag)) {
-            set_abort(abort_flag, p.status, SITE_GEMM_WAIT_TFULL, blockIdx.x, it);
+            set_abort(abort_flag, p.status, SITE_GEMM_WAIT_TFULL, (int)sm.pair, it);
             return;
         }
         tc_fence_after();
-        const bool rv = row < t.nrows;
-        const int gr = t.row0 + row;
-        int64_t tok = gr;
-        float sc = p.scale;
-        bool rv_out = rv;
-        if (rv) {
-            if (p.o_rows) tok = __ldg(p.o_rows + gr) / p.o_div;
-            if (p.row_scale) sc = __ldg(p.row_scale + gr);
-            if ((p.epi == EPI_ADD_F32 || p.epi == EPI_STORE_F32) && (tok < 0 || tok >= p.o_nrows)) {
-                report(p.status, MOEVIE_ERR_DEVICE, SITE_GEMM_OUT_ROW, gr, (int)tok);
-                rv_out = false;
-            }
+        const uint32_t tbase = tmem + ((uint32_t)(quad * 32) << 16) + (uint32_t)acc * GM_MAXBN;
+        if (half >= nchunk) {   // no columns for this warp in this tile
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive_remote(tempty_leader + 8 * acc);
         }
-        const uint32_t tbase = tmem + ((uint32_t)(warp * 32) << 16) + (uint32_t)acc * GM_MAXBN;
-        for (int c0 = 0; c0 < p.BN; c0 += 32) {
-            uint32_t v[32];
-            tmem_ld_32x32b_x32(tbase + c0, v);
+        for (int ch = half; ch < nchunk; ch += 2) {
+            const int c0 = ch * 16;
+            uint32_t v[16];
+            tmem_ld_32x32b_x16(tbase + c0, v);
             tmem_wait_ld();
-            if (!rv_out) continue;
+            if (ch + 2 >= nchunk) {   // this warp's last read of the accumulator
+                tc_fence_before();
+                __syncwarp();
+                if (lane == 0) mbar_arrive_remote(tempty_leader + 8 * acc);
+            }
+            const int n = t.n0 + c0;
+            if (!to_f32) {
+                if (ok_row) {
 #pragma unroll
-            for (int g8 = 0; g8 < 4; ++g8) {
-                const int cl = c0 + 8 * g8;      // column inside the tile
-                const int n = t.n0 + cl;         // column of the output
-                if (cl >= p.BN || n >= p.N) continue;
-                float f[8];
+                    for (int g8 = 0; g8 < 2; ++g8) {
+                        if (c0 + 8 * g8 >= p.BN || n + 8 * g8 >= p.N) continue;
+                        float f[8];
 #pragma unroll
-                for (int i = 0; i < 8; ++i) f[i] = __uint_as_float(v[8 * g8 + i]);
-                if (p.epi == EPI_GELU_BF16 || p.epi == EPI_STORE_BF16) {
-                    if (p.epi == EPI_GELU_BF16) {
-#pragma unroll
-                        for (int i = 0; i < 8; ++i) f[i] = gelu_erf(f[i]);
-                    }
-                    uint4 u;
-                    u.x = pack_bf16x2(f[0], f[1]);
-                    u.y = pack_bf16x2(f[2], f[3]);
-                    u.z = pack_bf16x2(f[4], f[5]);
-                    u.w = pack_bf16x2(f[6], f[7]);
-                    *reinterpret_cast<uint4*>(p.out + (int64_t)gr * p.ldo + n) = u;
-                } else {
-                    float4* dst = reinterpret_cast<float4*>(p.yacc + tok * p.ldy + n);
-                    const float4 lo = make_float4(sc * f[0], sc * f[1], sc * f[2], sc * f[3]);
-                    const float4 hi = make_float4(sc * f[4], sc * f[5], sc * f[6], sc * f[7]);
-                    if (p.epi == EPI_ADD_F32) {
-                        atomicAdd(dst, lo);
-                        atomicAdd(dst + 1, hi);
-                    } else {
-                        dst[0] = lo;
-                        dst[1] = hi;
+                        for (int i = 0; i < 8; ++i) {
+                            f[i] = __uint_as_float(v[8 * g8 + i]);
+                            if (p.epi == EPI_GELU_BF16) f[i] = gelu_erf(f[i]);
+                        }
+                        uint4 u;
+                        u.x = pack_bf16x2(f[0], f[1]);
+                        u.y = pack_bf16x2(f[2], f[3]);
+                        u.z = pack_bf16x2(f[4], f[5]);
+                        u.w = pack_bf16x2(f[6], f[7]);
+                        *reinterpret_cast<uint4*>(p.out + (int64_t)gr * p.ldo + n + 8 * g8) = u;
                     }
                 }
+                continue;
             }
+#pragma unroll
+            for (int q = 0; q < 4; ++q)
+                *reinterpret_cast<float4*>(stg + lane * STG_LD + 4 * q) =
+                    make_float4(__uint_as_float(v[4 * q]), __uint_as_float(v[4 * q + 1]),
+                                __uint_as_float(v[4 * q + 2]), __uint_as_float(v[4 * q + 3]));
+            __syncwarp();
+            const bool col_ok = (c0 + c4 < p.BN) && (n + c4 < p.N);
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+                const int rr = 8 * i + rsub;
+                const int64_t rtok = __shfl_sync(0xffffffffu, tok, rr);
+                const float rsc = __shfl_sync(0xffffffffu, sc, rr);
+                const bool rok = __shfl_sync(0xffffffffu, ok_row ? 1 : 0, rr) != 0;
+                const float4 f = *reinterpret_cast<const float4*>(stg + rr * STG_LD + c4);
+                if (!(rok && col_ok)) continue;
+                float4* dst = reinterpret_cast<float4*>(p.yacc + rtok * p.ldy + n + c4);
+                const float4 val = make_float4(rsc * f.x, rsc * f.y, rsc * f.z, rsc * f.w);
+                if (p.epi == EPI_ADD_F32) atomicAdd(dst, val);
+                else *dst = val;
+            }
+            __syncwarp();
         }
-        tc_fence_before();
-        mbar_arrive(sm.tempty + 8 * acc);
     }
 }
 
@@ -306,8 +528,9 @@ __global__ void __launch_bounds__(GM_THREADS, 1) grouped_gemm_kernel(const __gri
         (reinterpret_cast<uintptr_t>(gm_smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
     uint8_t* sA = smem;
     uint8_t* sB = smem + GM_STAGES * GM_A_BYTES;
-    uint64_t* bars = reinterpret_cast<uint64_t*>(sB + GM_STAGES * GM_B_BYTES);
-    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 2 * GM_STAGES + 5);
+    float* sOut = reinterpret_cast<float*>(sB + GM_STAGES * GM_B_BYTES);
+    uint64_t* bars = reinterpret_cast<uint64_t*>(sOut + GM_EPI_WARPS * 32 * STG_LD);
+    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 3 * GM_STAGES + 5);
     volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
 
     Smem sm;
@@ -315,54 +538,72 @@ __global__ void __launch_bounds__(GM_THREADS, 1) grouped_gemm_kernel(const __gri
     sm.b0 = smem_u32(sB);
     sm.full = smem_u32(bars);
     sm.empty = sm.full + 8 * GM_STAGES;
-    sm.tfull = sm.empty + 8 * GM_STAGES;
+    sm.afull = sm.empty + 8 * GM_STAGES;
+    sm.tfull = sm.afull + 8 * GM_STAGES;
     sm.tempty = sm.tfull + 16;
     sm.drain = sm.tempty + 16;
+    sm.stage_out = sOut;
+    sm.rank = cluster_rank();
+    sm.pair = blockIdx.x >> 1;
+    sm.npairs = gridDim.x >> 1;
 
     const int warp = threadIdx.x >> 5;
+    const bool gather = p.a_rows != nullptr;
     if (threadIdx.x == 0) {
         for (int s = 0; s < GM_STAGES; ++s) {
-            mbar_init(sm.full + 8 * s, 128 + 1);   // 128 gather threads + 1 TMA arrival
-            mbar_init(sm.empty + 8 * s, 1);        // tcgen05.commit
+            // leader's expect_tx arrival (+ its 4 gather warps and the peer's forwarder)
+            mbar_init(sm.full + 8 * s, 1 + (gather ? 4 + 1 : 0));
+            mbar_init(sm.empty + 8 * s, 1);         // multicast tcgen05.commit
+            mbar_init(sm.afull + 8 * s, 4);         // this CTA's gather warps
         }
         for (int a = 0; a < 2; ++a) {
-            mbar_init(sm.tfull + 8 * a, 1);        // tcgen05.commit
-            mbar_init(sm.tempty + 8 * a, 128);     // every epilogue thread
+            mbar_init(sm.tfull + 8 * a, 1);         // multicast tcgen05.commit
+            mbar_init(sm.tempty + 8 * a, 2 * GM_EPI_WARPS);   // every epilogue warp of the pair
         }
         mbar_init(sm.drain, 1);
         *abort_flag = 0;
         mbar_fence_init();
     }
-    if (warp == 4) {
-        tmem_alloc(smem_u32(tmem_slot), 2 * GM_MAXBN);
-        tmem_relinquish();
+    if (warp == GM_WARP_MMA) {
+        tmem_alloc_pair(smem_u32(tmem_slot), 2 * GM_MAXBN);
+        tmem_relinquish_pair();
     }
     tc_fence_before();
     __syncthreads();
+    cluster_sync();   // barriers of both CTAs initialised before any remote arrival
     tc_fence_after();
     const uint32_t tmem = *tmem_slot;
-    int64_t n_mtiles = __ldg(p.tile_off + p.G);
-    if (n_mtiles < 0 || n_mtiles > p.max_mtiles) {   // inconsistent offsets: do no work
-        if (threadIdx.x == 0) report(p.status, MOEVIE_ERR_DEVICE, SITE_GEMM_TILES, (int)n_mtiles, -1);
-        n_mtiles = 0;
+    int64_t n_mtiles;
+    if (p.tiles) {
+        n_mtiles = __ldg(p.n_tiles_dev);
+        if (n_mtiles < 0 || n_mtiles > p.max_mtiles) {   // inconsistent offsets: no work
+            if (threadIdx.x == 0) report(p.status, MOEVIE_ERR_DEVICE, SITE_GEMM_TILES, (int)n_mtiles, -1);
+            n_mtiles = 0;
+        }
+    } else {
+        n_mtiles = (p.m_total + GM_BM - 1) / GM_BM;
     }
     const int64_t n_work = n_mtiles * p.n_ntiles;
 
-    if (warp < 4) {
+    if (warp < GM_EPI_WARPS) {
         epilogue(p, sm, tmem, n_work, abort_flag);
-    } else if (warp == 4) {
-        if ((threadIdx.x & 31) == 0) mma_issuer(p, sm, tmem, n_work, abort_flag);
-    } else if (warp == 5) {
-        if ((threadIdx.x & 31) == 0) producer_b(p, sm, n_work, abort_flag);
-    } else {
-        producer_a(p, sm, n_work, abort_flag);
+    } else if (warp == GM_WARP_MMA) {
+        if ((threadIdx.x & 31) == 0) {
+            if (sm.rank == 0) mma_issuer(p, sm, tmem, n_work, abort_flag);
+            else if (gather) gather_forwarder(p, sm, n_work, abort_flag);
+        }
+    } else if (warp == GM_WARP_LOAD) {
+        if ((threadIdx.x & 31) == 0) producer_tma(p, sm, n_work, abort_flag);
+    } else if (gather) {
+        producer_gather(p, sm, n_work, abort_flag);
     }
 
     tc_fence_before();
     __syncthreads();
-    if (warp == 4) {
+    cluster_sync();   // the leader's MMAs have drained; both CTAs are done with TMEM
+    if (warp == GM_WARP_MMA) {
         tc_fence_after();
-        tmem_dealloc(tmem, 2 * GM_MAXBN);
+        tmem_dealloc_pair(tmem, 2 * GM_MAXBN);
     }
 }
 
@@ -394,10 +635,23 @@ bool make_weight_tmap(CUtensorMap* tm, const void* base, int64_t N, int64_t K, i
     return r == CUDA_SUCCESS;
 }
 
+bool make_rows_tmap(CUtensorMap* tm, const void* base, int64_t cols, int64_t rows, int64_t ld) {
+    PFN_cuTensorMapEncodeTiled_v12000 enc = get_encode_fn();
+    if (!enc) return false;
+    cuuint64_t dims[2] = {(cuuint64_t)cols, (cuuint64_t)rows};
+    cuuint64_t strides[1] = {(cuuint64_t)ld * 2};
+    cuuint32_t box[2] = {64, (cuuint32_t)GM_HALF};
+    cuuint32_t estr[2] = {1, 1};
+    CUresult r = enc(tm, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides,
+                     box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                     CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    return r == CUDA_SUCCESS;
+}
+
 void choose_bn(int N, int* BN, int* n_ntiles) {
     const int nt = (N + GM_MAXBN - 1) / GM_MAXBN;
     int bn = (N + nt - 1) / nt;
-    bn = (bn + 15) / 16 * 16;
+    bn = (bn + 31) / 32 * 32;   // each CTA of a pair holds BN / 2 columns, a multiple of 16
     *BN = bn;
     *n_ntiles = (N + bn - 1) / bn;
 }
@@ -413,9 +667,21 @@ cudaError_t launch_grouped_gemm(const GemmArgs& a, int grid, cudaStream_t s) {
         if (e != cudaSuccess) return e;
         attr_set[dev] = true;
     }
-    grouped_gemm_kernel<<<grid, GM_THREADS, GM_SMEM_BYTES, s>>>(a);
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3((unsigned)((grid + 1) & ~1));   // whole pairs
+    cfg.blockDim = dim3(GM_THREADS);
+    cfg.dynamicSmemBytes = GM_SMEM_BYTES;
+    cfg.stream = s;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = 2;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    cudaError_t e = cudaLaunchKernelEx(&cfg, grouped_gemm_kernel, a);
     count_launches(1);
-    return cudaGetLastError();
+    return e != cudaSuccess ? e : cudaGetLastError();
 }
 
 }  // namespace mv

@@ -14,51 +14,71 @@ void count_launches(int n);
 
 // ----------------------------------------------------------------- router
 
-// Relative bound on the fp32 logit error used to decide when a token's selection
-// must be re-decided with exact logits: |s_fast - s| <= TAU_C * 2^-24 * |x_t| * max_e |W_r[:, e]|.
-constexpr float ROUTE_TAU_C = 64.0f;
+// Error model of the fast (tensor-core, fp32-accumulated) logits used to decide
+// when a token's selection must be re-decided with exact logits:
+//   |s_fast[t, e] - s[t, e]| <= ROUTE_TAU_C * 2^-24 * |x_t| * |W_r[:, e]|.
+constexpr float ROUTE_TAU_C = 128.0f;
 // Extra allowance, in key units, for the fp32 evaluation of sigmoid(s) + b.
 constexpr float ROUTE_KEY_SLACK = 2e-6f;
 
-struct RouteBufs {
-    float* logits;      // [T, E]
-    float* xnorm2;      // [T]
-    float* wnorm2;      // [E]
-    int32_t* fb_tokens; // [T]
-};
+// Columns of the router logit buffer: E rounded up to 16 (rows stay 16-byte aligned).
+inline int route_epad(int E) { return (E + 15) / 16 * 16; }
+// Rows of each W_r piece: d rounded up to 64 (zero rows), so that no 64-wide K block
+// of the router GEMM straddles two pieces.
+inline int route_dpad(int d) { return (d + 63) / 64 * 64; }
 
-cudaError_t launch_route_logits(const __nv_bfloat16* x, const float* Wr, int T, int d, int E,
-                                const RouteBufs& rb, DevStatus* st, cudaStream_t s);
-cudaError_t launch_route_select(const __nv_bfloat16* x, const float* Wr, const float* b, int T,
+// W_r fp32 [d, E] -> three bf16 pieces [3][d_pad][E_pad] with W_r = hi + mid + lo
+// exactly (zero in the padding rows and columns), plus |W_r[:, e]| (wpart:
+// route_split_parts(d) x E_pad floats of scratch).
+int route_split_parts(int d);
+cudaError_t launch_route_split(const float* Wr, int d, int E, __nv_bfloat16* Wsplit, float* wpart,
+                               float* wnorm, cudaStream_t s);
+// Keys, warp top-k with a certificate, gates; uncertified tokens are re-decided
+// with exact (fp64) logits of the experts near their boundary.
+cudaError_t launch_route_select(const __nv_bfloat16* x, const float* Wr, const float* b,
+                                const float* logits, int ld_logits, const float* wnorm, int T,
                                 int d, int E, int k, int32_t* idx, float* gate,
-                                const RouteBufs& rb, DevStatus* st, int num_sms, cudaStream_t s);
+                                int32_t* fb_tokens, float* xnorm, DevStatus* st, int num_sms,
+                                cudaStream_t s);
 
 // ---------------------------------------------------------------- permute
 
-constexpr int PERM_CHUNK = 4096;   // flat slots per CTA of the histogram / scatter
+constexpr int PERM_CHUNK_MAX = 4096;   // flat slots per CTA of the histogram / scatter
 
-cudaError_t launch_permute(const int32_t* idx, int64_t n_slots, int k, int E, int bm,
+// Slots per CTA for n flat slots on num_sms SMs (multiple of 256, <= PERM_CHUNK_MAX).
+int perm_chunk(int64_t n, int num_sms);
+
+// Stable expert-major order; also writes the m-tile table of the grouped GEMMs
+// (tiles[i] = {expert, first row, rows, 0}, *n_tiles = their number).
+cudaError_t launch_permute(const int32_t* idx, int64_t n_slots, int k, int E, int bm, int chunk,
                            const float* gate_flat, int32_t* hist, int32_t* counts,
-                           int32_t* offsets, int32_t* tile_off, int32_t* perm, int32_t* inv,
-                           int32_t* row_tok, float* row_gate, DevStatus* st, cudaStream_t s);
+                           int32_t* offsets, int4* tiles, int32_t* n_tiles, int32_t* perm,
+                           int32_t* inv, int32_t* row_tok, float* row_gate, DevStatus* st,
+                           cudaStream_t s);
 
-// One group of T rows: offsets = {0, T}, tile_off = {0, ceil(T / bm)}.
-cudaError_t launch_single_group(int32_t* offsets, int32_t* tile_off, int T, int bm, cudaStream_t s);
-
-// Tiles of `bm` rows per group from given offsets: tile_off[g] = sum_{g'<g} ceil(cnt/bm).
-cudaError_t launch_tile_prefix(const int32_t* offsets, int G, int bm, int32_t* tile_off,
-                               cudaStream_t s);
+// m-tile table of `bm`-row tiles from given segment offsets [G + 1].
+cudaError_t launch_tile_table(const int32_t* offsets, int G, int bm, int4* tiles,
+                              int32_t* n_tiles, cudaStream_t s);
 
 // ----------------------------------------------------------- grouped GEMM
 
-constexpr int GM_BM = 128;        // rows per tile (tcgen05 M)
+constexpr int GM_BM = 256;        // rows per m-tile: one CTA pair, 128 rows per CTA
+constexpr int GM_HALF = 128;      // rows per CTA (tcgen05 M = 256 across the pair)
 constexpr int GM_BK = 64;         // K per stage: 64 bf16 = one 128-byte swizzle row
-constexpr int GM_STAGES = 4;
-constexpr int GM_MAXBN = 256;     // largest N of one tcgen05.mma with M = 128
-constexpr int GM_THREADS = 320;   // 4 epilogue warps, MMA warp, TMA warp, 4 gather warps
-constexpr int GM_A_BYTES = GM_BM * GM_BK * 2;
-constexpr int GM_B_BYTES = GM_BK * GM_MAXBN * 2;
-constexpr int GM_SMEM_BYTES = GM_STAGES * (GM_A_BYTES + GM_B_BYTES) + 1024 + 256;
+constexpr int GM_STAGES = 6;
+constexpr int GM_MAXBN = 256;     // largest N of one tcgen05.mma
+constexpr int GM_EPI_WARPS = 8;   // two warps per TMEM lane quadrant, alternate 16-column chunks
+constexpr int GM_WARP_MMA = GM_EPI_WARPS;        // TMEM allocation + tcgen05.mma issue
+constexpr int GM_WARP_LOAD = GM_EPI_WARPS + 1;   // TMA loads of B (and of contiguous A)
+constexpr int GM_WARP_GATHER = GM_EPI_WARPS + 2; // first of 4 token-gather warps
+constexpr int GM_THREADS = (GM_EPI_WARPS + 2 + 4) * 32;
+constexpr int GM_A_BYTES = GM_HALF * GM_BK * 2;           // one CTA's A rows per stage
+constexpr int GM_B_BYTES = GM_BK * (GM_MAXBN / 2) * 2;    // one CTA's half of B per stage
+constexpr int GM_STG_LD = 20;                   // floats per row of a transpose buffer
+constexpr int GM_STG_BYTES = GM_EPI_WARPS * 32 * GM_STG_LD * 4;   // epilogue transpose buffers
+constexpr int GM_SMEM_BYTES = GM_STAGES * (GM_A_BYTES + GM_B_BYTES) + GM_STG_BYTES + 1024 + 512;
+
+inline int64_t max_mtiles(int64_t rows, int64_t groups) { return (rows + GM_BM - 1) / GM_BM + groups; }
 
 enum Epilogue : int {
     EPI_GELU_BF16 = 0,   // out[r, n] = bf16(GELU(acc))
@@ -69,22 +89,25 @@ enum Epilogue : int {
 
 struct GemmArgs {
     CUtensorMap tmB;            // B = weights [G][K][N] bf16 (N contiguous), 3-D map {N, K, G}
-    const __nv_bfloat16* A;     // A rows [*, lda] bf16
+    CUtensorMap tmA;            // A = rows [a_nrows][K_A] bf16, 2-D map {K_A, a_nrows}, box
+                                // {64, 128}; used when A rows are contiguous (a_rows == nullptr)
+    const __nv_bfloat16* A;     // A rows, for the token gather
     int64_t lda;
-    const int32_t* a_rows;      // A row of GEMM row r: a_rows ? a_rows[r] / a_div : r
+    const int32_t* a_rows;      // A row of GEMM row r: a_rows ? a_rows[r] / a_div : r (gather)
     int a_div;
+    int a_kperiod;              // 0, or a multiple of 64: column of K index kk in A is kk % a_kperiod
     int64_t a_nrows;            // rows of A; a gathered row outside [0, a_nrows) is a device error
-    int64_t m_total;            // GEMM rows that may be written; tiles past it are a device error
-    int64_t max_mtiles;         // host bound on tile_off[G]
-    int64_t o_nrows;            // rows of yacc (EPI_*_F32); tokens outside are a device error
-    const int32_t* offsets;     // [G + 1] GEMM-row segment of each group
-    const int32_t* tile_off;    // [G + 1] m-tile prefix; tile_off[G] = number of m-tiles
+    int64_t m_total;            // GEMM rows that may be written
+    const int4* tiles;          // m-tile table {g, row0, nrows, 0}; nullptr: one dense group
+    const int32_t* n_tiles_dev; // number of entries of `tiles`
+    int64_t max_mtiles;         // host bound on *n_tiles_dev
     int G, K, N, BN, n_ntiles, num_kb, nbox;
     int epi;
     __nv_bfloat16* out;         // EPI_*_BF16
     int64_t ldo;
     float* yacc;                // EPI_*_F32
     int64_t ldy;
+    int64_t o_nrows;            // rows of yacc; tokens outside are a device error
     const int32_t* o_rows;      // output token of row r: o_rows ? o_rows[r] / o_div : r
     int o_div;
     const float* row_scale;     // scale(r) = row_scale ? row_scale[r] : scale
@@ -95,7 +118,10 @@ struct GemmArgs {
 
 // Encodes the 3-D weight tensor map {N, K, G} for W[G][K][N] bf16.
 bool make_weight_tmap(CUtensorMap* tm, const void* base, int64_t N, int64_t K, int64_t G);
-// Picks BN (multiple of 16, <= 256) and the number of N tiles for width N.
+// Encodes the 2-D row tensor map {cols, rows} of A[rows][cols] bf16 (row stride ld
+// elements), box {64, GM_HALF}.
+bool make_rows_tmap(CUtensorMap* tm, const void* base, int64_t cols, int64_t rows, int64_t ld);
+// Picks BN (multiple of 32, <= 256) and the number of N tiles for width N.
 void choose_bn(int N, int* BN, int* n_ntiles);
 cudaError_t launch_grouped_gemm(const GemmArgs& a, int grid, cudaStream_t s);
 

@@ -1,7 +1,7 @@
 // permute.cu -- expert-major order of the flat routing slots (App. B, Algorithm 1,
 // phase 1: Sort by expert id, index = pos // K, BinCount, CumSum), sm_103a.
 //
-// A stable counting sort over chunks of PERM_CHUNK flat slots:
+// A stable counting sort over chunks of flat slots (about two chunks per SM):
 //   perm_hist_kernel    per-chunk histograms (16-byte vector loads of idx)
 //   perm_scan_kernel    counts, exclusive offsets, each chunk's first row per
 //                       expert, and the m-tile prefix used by the grouped GEMMs
@@ -18,19 +18,18 @@ namespace {
 
 constexpr int PT = 256;                      // threads per CTA
 constexpr int PW = PT / 32;                  // warps per CTA
-constexpr int PER_WARP = PERM_CHUNK / PW;    // slots per warp in the scatter
 
 __device__ __forceinline__ bool valid_id(int e, int E) { return e >= 0 && e < E; }
 
 __global__ void __launch_bounds__(PT) perm_hist_kernel(const int32_t* __restrict__ idx,
-                                                       int64_t n, int E,
+                                                       int64_t n, int E, int chunk,
                                                        int32_t* __restrict__ hist,
                                                        DevStatus* st) {
     extern __shared__ int32_t cnt[];
     for (int e = threadIdx.x; e < E; e += PT) cnt[e] = 0;
     __syncthreads();
-    const int64_t c0 = (int64_t)blockIdx.x * PERM_CHUNK;
-    const int64_t c1 = c0 + PERM_CHUNK < n ? c0 + PERM_CHUNK : n;
+    const int64_t c0 = (int64_t)blockIdx.x * chunk;
+    const int64_t c1 = c0 + chunk < n ? c0 + chunk : n;
     const int64_t nvec = (c1 - c0) >> 2;
     const int4* v = reinterpret_cast<const int4*>(idx + c0);   // c0 % 4 == 0, idx 16-B aligned
     for (int64_t i = threadIdx.x; i < nvec; i += PT) {
@@ -80,49 +79,72 @@ __device__ int block_exclusive_scan_1024(int v, int* total) {
     return r;
 }
 
-// One thread per expert (E <= 1024).  Rewrites hist[c][e] in place with the
-// first row of expert e inside chunk c.
+// One CTA of 1024 threads.  Warp w scans the chunk histograms of experts w, w+32,
+// ... (lanes over chunks) and rewrites hist[c][e] in place with the first row of
+// expert e inside chunk c, relative to the expert's segment; then one thread per
+// expert scans counts and tile counts across experts; then warps write the m-tile
+// table (lanes over an expert's tiles).
 __global__ void __launch_bounds__(1024) perm_scan_kernel(int32_t* __restrict__ hist, int nchunks,
                                                          int E, int bm,
                                                          int32_t* __restrict__ counts,
                                                          int32_t* __restrict__ offsets,
-                                                         int32_t* __restrict__ tile_off) {
+                                                         int4* __restrict__ tiles,
+                                                         int32_t* __restrict__ n_tiles) {
     __shared__ int s_total, s_tiles;
+    __shared__ int s_cnt[1024], s_off[1024], s_toff[1024];
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    for (int e = warp; e < E; e += 32) {
+        int running = 0;
+        for (int c0 = 0; c0 < nchunks; c0 += 32) {
+            const int c = c0 + lane;
+            const int h = c < nchunks ? hist[(int64_t)c * E + e] : 0;
+            int inc = h;
+#pragma unroll
+            for (int o = 1; o < 32; o <<= 1) {
+                const int u = __shfl_up_sync(0xffffffffu, inc, o);
+                if (lane >= o) inc += u;
+            }
+            if (c < nchunks) hist[(int64_t)c * E + e] = running + inc - h;
+            running += __shfl_sync(0xffffffffu, inc, 31);
+        }
+        if (lane == 0) s_cnt[e] = running;
+    }
+    __syncthreads();
     const int e = threadIdx.x;
-    int cnt = 0;
-    if (e < E)
-        for (int c = 0; c < nchunks; ++c) cnt += hist[(int64_t)c * E + e];
-    const int off = block_exclusive_scan_1024(e < E ? cnt : 0, &s_total);
-    const int nt = (cnt + bm - 1) / bm;
-    const int toff = block_exclusive_scan_1024(e < E ? nt : 0, &s_tiles);
+    const int cnt = e < E ? s_cnt[e] : 0;
+    const int off = block_exclusive_scan_1024(cnt, &s_total);
+    const int toff = block_exclusive_scan_1024((cnt + bm - 1) / bm, &s_tiles);
     if (e < E) {
         if (counts) counts[e] = cnt;
         offsets[e] = off;
-        tile_off[e] = toff;
-        int run = off;
-        for (int c = 0; c < nchunks; ++c) {
-            const int h = hist[(int64_t)c * E + e];
-            hist[(int64_t)c * E + e] = run;
-            run += h;
-        }
+        s_off[e] = off;
+        s_toff[e] = toff;
     }
     if (e == 0) {
         offsets[E] = s_total;
-        tile_off[E] = s_tiles;
+        *n_tiles = s_tiles;
+    }
+    __syncthreads();
+    for (int g = warp; g < E; g += 32) {
+        const int c = s_cnt[g], o = s_off[g], to = s_toff[g];
+        for (int m = lane; m * bm < c; m += 32)
+            tiles[to + m] = make_int4(g, o + m * bm, min(bm, c - m * bm), 0);
     }
 }
 
-// Dynamic smem: PERM_CHUNK ints (the chunk's ids) + PW * E ints (per-warp counts).
+// Dynamic smem: chunk ints (the chunk's ids) + PW * E ints (per-warp counts).
 __global__ void __launch_bounds__(PT) perm_scatter_kernel(
-    const int32_t* __restrict__ idx, int64_t n, int k, int E, const int32_t* __restrict__ base,
+    const int32_t* __restrict__ idx, int64_t n, int k, int E, int chunk,
+    const int32_t* __restrict__ base, const int32_t* __restrict__ offsets,
     const float* __restrict__ gate_flat, int32_t* __restrict__ perm, int32_t* __restrict__ inv,
     int32_t* __restrict__ row_tok, float* __restrict__ row_gate) {
     extern __shared__ __align__(16) int32_t ps_smem[];
     int32_t* sidx = ps_smem;
-    int32_t* wc = ps_smem + PERM_CHUNK;
+    int32_t* wc = ps_smem + chunk;
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-    const int64_t c0 = (int64_t)blockIdx.x * PERM_CHUNK;
-    const int len = (int)(c0 + PERM_CHUNK < n ? PERM_CHUNK : n - c0);
+    const int per_warp = chunk / PW;
+    const int64_t c0 = (int64_t)blockIdx.x * chunk;
+    const int len = (int)(c0 + chunk < n ? chunk : n - c0);
     {
         const int nvec = len >> 2;
         const int4* v = reinterpret_cast<const int4*>(idx + c0);
@@ -132,8 +154,8 @@ __global__ void __launch_bounds__(PT) perm_scatter_kernel(
     }
     for (int i = tid; i < PW * E; i += PT) wc[i] = 0;
     __syncthreads();
-    const int wbeg = warp * PER_WARP;
-    const int wend = wbeg + PER_WARP < len ? wbeg + PER_WARP : len;
+    const int wbeg = warp * per_warp;
+    const int wend = wbeg + per_warp < len ? wbeg + per_warp : len;
     int32_t* my = wc + warp * E;
     for (int s0 = wbeg; s0 < wend; s0 += 32) {          // pass 1: per-warp histogram
         const int i = s0 + lane;
@@ -145,7 +167,7 @@ __global__ void __launch_bounds__(PT) perm_scatter_kernel(
     }
     __syncthreads();
     for (int e = tid; e < E; e += PT) {                  // pass 2: first row per (warp, e)
-        int run = base[(int64_t)blockIdx.x * E + e];
+        int run = offsets[e] + base[(int64_t)blockIdx.x * E + e];
         for (int w = 0; w < PW; ++w) {
             const int c = wc[w * E + e];
             wc[w * E + e] = run;
@@ -178,66 +200,61 @@ __global__ void __launch_bounds__(PT) perm_scatter_kernel(
     }
 }
 
-__global__ void tile_prefix_kernel(const int32_t* __restrict__ offsets, int G, int bm,
-                                   int32_t* __restrict__ tile_off) {
+// m-tile table from given offsets (one thread per group, E <= 1024).
+__global__ void __launch_bounds__(1024) tile_table_kernel(const int32_t* __restrict__ offsets,
+                                                          int G, int bm, int4* __restrict__ tiles,
+                                                          int32_t* __restrict__ n_tiles) {
     __shared__ int s_total;
-    int acc_base = 0;
-    for (int g0 = 0; g0 < G; g0 += 1024) {
-        const int g = g0 + threadIdx.x;
-        const int cnt = (g < G) ? offsets[g + 1] - offsets[g] : 0;
-        const int nt = cnt > 0 ? (cnt + bm - 1) / bm : 0;
-        const int ex = block_exclusive_scan_1024(nt, &s_total);
-        if (g < G) tile_off[g] = acc_base + ex;
-        acc_base += s_total;
-        __syncthreads();
-    }
-    if (threadIdx.x == 0) tile_off[G] = acc_base;
-}
-
-__global__ void single_group_kernel(int32_t* offsets, int32_t* tile_off, int T, int bm) {
-    offsets[0] = 0;
-    offsets[1] = T;
-    tile_off[0] = 0;
-    tile_off[1] = (T + bm - 1) / bm;
+    const int g = threadIdx.x;
+    const int cnt = (g < G) ? max(0, offsets[g + 1] - offsets[g]) : 0;
+    const int nt = (cnt + bm - 1) / bm;
+    const int toff = block_exclusive_scan_1024(nt, &s_total);
+    if (g < G)
+        for (int m = 0; m < nt; ++m)
+            tiles[toff + m] = make_int4(g, offsets[g] + m * bm, min(bm, cnt - m * bm), 0);
+    if (g == 0) *n_tiles = s_total;
 }
 
 }  // namespace
 
-cudaError_t launch_single_group(int32_t* offsets, int32_t* tile_off, int T, int bm, cudaStream_t s) {
-    single_group_kernel<<<1, 1, 0, s>>>(offsets, tile_off, T, bm);
-    count_launches(1);
-    return cudaGetLastError();
+int perm_chunk(int64_t n, int num_sms) {
+    int64_t c = (n + 2 * num_sms - 1) / (2 * num_sms);
+    c = (c + 255) / 256 * 256;
+    if (c < 256) c = 256;
+    if (c > PERM_CHUNK_MAX) c = PERM_CHUNK_MAX;
+    return (int)c;
 }
 
-cudaError_t launch_permute(const int32_t* idx, int64_t n_slots, int k, int E, int bm,
+cudaError_t launch_permute(const int32_t* idx, int64_t n_slots, int k, int E, int bm, int chunk,
                            const float* gate_flat, int32_t* hist, int32_t* counts,
-                           int32_t* offsets, int32_t* tile_off, int32_t* perm, int32_t* inv,
-                           int32_t* row_tok, float* row_gate, DevStatus* st, cudaStream_t s) {
-    const int nchunks = (int)((n_slots + PERM_CHUNK - 1) / PERM_CHUNK);
-    perm_hist_kernel<<<nchunks, PT, (size_t)E * 4, s>>>(idx, n_slots, E, hist, st);
+                           int32_t* offsets, int4* tiles, int32_t* n_tiles, int32_t* perm,
+                           int32_t* inv, int32_t* row_tok, float* row_gate, DevStatus* st,
+                           cudaStream_t s) {
+    const int nchunks = (int)((n_slots + chunk - 1) / chunk);
+    perm_hist_kernel<<<nchunks, PT, (size_t)E * 4, s>>>(idx, n_slots, E, chunk, hist, st);
     cudaError_t err = cudaGetLastError();
     if (err != cudaSuccess) return err;
-    perm_scan_kernel<<<1, 1024, 0, s>>>(hist, nchunks, E, bm, counts, offsets, tile_off);
+    perm_scan_kernel<<<1, 1024, 0, s>>>(hist, nchunks, E, bm, counts, offsets, tiles, n_tiles);
     if ((err = cudaGetLastError()) != cudaSuccess) return err;
-    const size_t smem = (size_t)(PERM_CHUNK + PW * E) * 4;
+    const size_t smem = (size_t)(chunk + PW * E) * 4;
     static bool attr_set[64] = {};
     int dev = 0;
     cudaGetDevice(&dev);
     if (dev >= 0 && dev < 64 && !attr_set[dev]) {
         err = cudaFuncSetAttribute(perm_scatter_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                   (int)((PERM_CHUNK + PW * 1024) * 4));
+                                   (int)((PERM_CHUNK_MAX + PW * 1024) * 4));
         if (err != cudaSuccess) return err;
         attr_set[dev] = true;
     }
-    perm_scatter_kernel<<<nchunks, PT, smem, s>>>(idx, n_slots, k, E, hist, gate_flat, perm, inv,
-                                                  row_tok, row_gate);
+    perm_scatter_kernel<<<nchunks, PT, smem, s>>>(idx, n_slots, k, E, chunk, hist, offsets,
+                                                  gate_flat, perm, inv, row_tok, row_gate);
     count_launches(3);
     return cudaGetLastError();
 }
 
-cudaError_t launch_tile_prefix(const int32_t* offsets, int G, int bm, int32_t* tile_off,
-                               cudaStream_t s) {
-    tile_prefix_kernel<<<1, 1024, 0, s>>>(offsets, G, bm, tile_off);
+cudaError_t launch_tile_table(const int32_t* offsets, int G, int bm, int4* tiles,
+                              int32_t* n_tiles, cudaStream_t s) {
+    tile_table_kernel<<<1, 1024, 0, s>>>(offsets, G, bm, tiles, n_tiles);
     count_launches(1);
     return cudaGetLastError();
 }

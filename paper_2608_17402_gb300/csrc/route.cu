@@ -1,15 +1,27 @@
 // route.cu -- router of the MoE-ViE layer (Eqs. 1, 7, 4-5), sm_103a.
 //
-//  1. route_logits_kernel: s = x . W_r in fp32 on CUDA cores (64 tokens x 64
-//     experts per CTA), plus |x_t|^2 and |W_r[:, e]|^2 for the error bound.
+// The logits s = x . W_r run on the tensor cores (grouped_gemm_kernel, one dense
+// group): W_r is split exactly into three bf16 pieces, W_r = hi + mid + lo, and
+// the GEMM accumulates x . [hi; mid; lo] over K = 3 d_pad in fp32 (each piece padded
+// to a multiple of 64 rows with zeros).  Every product of a
+// bf16 x and a bf16 piece is exact in fp32, so the only error is the fp32
+// accumulation.  This file holds the steps around that GEMM:
+//
+//  1. route_split_kernel / route_wnorm_kernel: the three pieces and |W_r[:, e]|.
 //  2. route_topk_kernel: one warp per token; keys sigmoid(s) + b, k rounds of warp
-//     arg-max (ties to the lower id), and a certificate: the gap between the k-th
-//     and (k+1)-th key must exceed twice the key error bound.  Certified tokens
-//     write ascending ids and gates sigmoid(s)/sum (the bias only selects).
-//  3. route_fallback_kernel: for every token without a certificate, experts whose
-//     key interval overlaps the boundary get exact logits (fp64: each product
-//     x_i * w_i of a bf16 and an fp32 value is exact in double) and the remaining
-//     places are filled from them, ties to the lower id.
+//     arg-max (ties to the lower id), and a certificate.  Every expert's key lies in
+//     [key_e - tau_e, key_e + tau_e]; tau_e is the logit error bound
+//     (ROUTE_TAU_C 2^-24 |x_t| |W_r[:, e]|) times the largest sigmoid slope inside
+//     the logit interval, plus fp32 evaluation slack.  The selection is certain when
+//     the lowest selected lower end is above the highest unselected upper end (tried
+//     first with the slope bound 1/4, then with the exact slope).  Certified tokens
+//     write ascending ids and gates sigmoid(s) / sum (the bias only selects).
+//  3. route_fallback_kernel: one warp per uncertified token.  An expert is surely in
+//     when its lower end is above the k-th largest upper end of the others, surely
+//     out when its upper end is below the k-th largest lower end; the rest get exact
+//     logits (fp64: each product of a bf16 and an fp32 value is exact in double, and
+//     the sum of d terms has relative error below d 2^-53), and the remaining places
+//     are filled from them, ties to the lower id.
 #include <math.h>
 
 #include "internal.h"
@@ -18,153 +30,134 @@ namespace mv {
 
 namespace {
 
-constexpr int LG_TT = 64;   // tokens per CTA
-constexpr int LG_TE = 64;   // experts per CTA
-constexpr int LG_TK = 32;   // K per smem stage
+constexpr int SPLIT_ROWS = 256;   // W_r rows per CTA of the split kernel
 
-__global__ void __launch_bounds__(256) route_logits_kernel(const __nv_bfloat16* __restrict__ x,
-                                                           const float* __restrict__ Wr, int T,
-                                                           int d, int E, float* __restrict__ s,
-                                                           float* __restrict__ xnorm2,
-                                                           float* __restrict__ wnorm2,
-                                                           DevStatus* st) {
-    __shared__ float xs[LG_TK][LG_TT + 4];
-    __shared__ float wsm[LG_TK][LG_TE + 4];
-    __shared__ float wred[8][LG_TE];
-    const int t0 = blockIdx.x * LG_TT, e0 = blockIdx.y * LG_TE;
-    const int tid = threadIdx.x;
-    const int ty = tid >> 4, tx = tid & 15;
-    const int xl_t = tid >> 2, xl_k = (tid & 3) * 8;      // x loader: token, first k
-    const int wl_k = tid >> 3, wl_e = (tid & 7) * 8;      // W loader: k row, first expert
-    float acc[4][4];
-#pragma unroll
-    for (int i = 0; i < 4; ++i)
-#pragma unroll
-        for (int j = 0; j < 4; ++j) acc[i][j] = 0.f;
-    float xsq = 0.f;
-    float wsq[8];
-#pragma unroll
-    for (int i = 0; i < 8; ++i) wsq[i] = 0.f;
-
-    for (int k0 = 0; k0 < d; k0 += LG_TK) {
-        {
-            const int t = t0 + xl_t, kk = k0 + xl_k;
-            float v[8];
-            if (t < T && kk < d) {   // d % 8 == 0: the 8 values are all inside the row
-                const uint4 u = *reinterpret_cast<const uint4*>(x + (int64_t)t * d + kk);
-                unpack_bf16x8(u, v);
-            } else {
-#pragma unroll
-                for (int i = 0; i < 8; ++i) v[i] = 0.f;
-            }
-#pragma unroll
-            for (int i = 0; i < 8; ++i) {
-                xs[xl_k + i][xl_t] = v[i];
-                xsq = fmaf(v[i], v[i], xsq);
-            }
-        }
-        {
-            const int kk = k0 + wl_k;
-#pragma unroll
-            for (int i = 0; i < 8; ++i) {
-                const int e = e0 + wl_e + i;
-                const float v = (kk < d && e < E) ? __ldg(Wr + (int64_t)kk * E + e) : 0.f;
-                wsm[wl_k][wl_e + i] = v;
-                wsq[i] = fmaf(v, v, wsq[i]);
-            }
-        }
-        __syncthreads();
-#pragma unroll
-        for (int kk = 0; kk < LG_TK; ++kk) {
-            float a[4], b[4];
-#pragma unroll
-            for (int i = 0; i < 4; ++i) a[i] = xs[kk][ty * 4 + i];
-#pragma unroll
-            for (int j = 0; j < 4; ++j) b[j] = wsm[kk][tx * 4 + j];
-#pragma unroll
-            for (int i = 0; i < 4; ++i)
-#pragma unroll
-                for (int j = 0; j < 4; ++j) acc[i][j] = fmaf(a[i], b[j], acc[i][j]);
-        }
-        __syncthreads();
-    }
-#pragma unroll
-    for (int i = 0; i < 4; ++i) {
-        const int t = t0 + ty * 4 + i;
-        if (t >= T) continue;
-#pragma unroll
-        for (int j = 0; j < 4; ++j) {
-            const int e = e0 + tx * 4 + j;
-            if (e < E) s[(int64_t)t * E + e] = acc[i][j];
+// CTA (bx, by): experts 32 bx .. +31, rows SPLIT_ROWS by .. +SPLIT_ROWS-1; 32 x 8 threads.
+__global__ void __launch_bounds__(256) route_split_kernel(const float* __restrict__ Wr, int d,
+                                                          int dp, int E, int Ep,
+                                                          __nv_bfloat16* __restrict__ Wsplit,
+                                                          float* __restrict__ wpart) {
+    __shared__ float red[8][32];
+    const int tx = threadIdx.x & 31, ty = threadIdx.x >> 5;
+    const int e = blockIdx.x * 32 + tx;
+    const int i0 = blockIdx.y * SPLIT_ROWS;
+    const int i1 = min(dp, i0 + SPLIT_ROWS);
+    float sq = 0.f;
+    if (e < Ep) {
+        const size_t piece = (size_t)dp * Ep;
+        for (int i = i0 + ty; i < i1; i += 8) {
+            const float w = (e < E && i < d) ? Wr[(int64_t)i * E + e] : 0.f;
+            const __nv_bfloat16 hi = __float2bfloat16_rn(w);
+            const float r1 = w - __bfloat162float(hi);          // exact
+            const __nv_bfloat16 mid = __float2bfloat16_rn(r1);
+            const __nv_bfloat16 lo = __float2bfloat16_rn(r1 - __bfloat162float(mid));   // exact
+            const size_t o = (size_t)i * Ep + e;
+            Wsplit[o] = hi;
+            Wsplit[piece + o] = mid;
+            Wsplit[2 * piece + o] = lo;
+            sq = fmaf(w, w, sq);
         }
     }
-    if (blockIdx.y == 0) {   // |x_t|^2: 4 consecutive lanes hold one token
-        xsq += __shfl_xor_sync(0xffffffffu, xsq, 1);
-        xsq += __shfl_xor_sync(0xffffffffu, xsq, 2);
-        if ((tid & 3) == 0 && t0 + xl_t < T) xnorm2[t0 + xl_t] = xsq;
+    red[ty][tx] = sq;
+    __syncthreads();
+    if (ty == 0 && e < Ep) {
+        float v = 0.f;
+        for (int q = 0; q < 8; ++q) v += red[q][tx];
+        wpart[(int64_t)blockIdx.y * Ep + e] = v;
     }
-    if (blockIdx.x == 0) {   // |W_r[:, e]|^2: lanes l, l+8, l+16, l+24 share experts
-#pragma unroll
-        for (int i = 0; i < 8; ++i) {
-            float v = wsq[i];
-            v += __shfl_xor_sync(0xffffffffu, v, 8);
-            v += __shfl_xor_sync(0xffffffffu, v, 16);
-            if ((tid & 31) < 8) wred[tid >> 5][wl_e + i] = v;
-        }
-        __syncthreads();
-        if (tid < LG_TE && e0 + tid < E) {
-            float v = 0.f;
-            for (int w = 0; w < 8; ++w) v += wred[w][tid];
-            wnorm2[e0 + tid] = v;
-        }
-    }
-    if (blockIdx.x == 0 && blockIdx.y == 0 && tid == 0) st->fb_count = 0;
 }
 
-__device__ __forceinline__ float sigmoid_f32(float v) { return 1.0f / (1.0f + expf(-v)); }
-
-// Half-width of the key interval of token t: key error <= 0.25 * logit error +
-// fp32 evaluation slack (the slope of the sigmoid is at most 1/4).
-__device__ __forceinline__ float key_tau(float xn2, float wmax2) {
-    const float tau_s = ROUTE_TAU_C * 5.9604645e-8f * sqrtf(xn2 * wmax2);
-    return 0.25f * tau_s + ROUTE_KEY_SLACK;
+// |W_r[:, e]| from the per-CTA partial sums, in a fixed order.
+__global__ void route_wnorm_kernel(const float* __restrict__ wpart, int nparts, int E, int Ep,
+                                   float* __restrict__ wnorm) {
+    const int e = blockIdx.x * blockDim.x + threadIdx.x;
+    if (e >= E) return;
+    float v = 0.f;
+    for (int p = 0; p < nparts; ++p) v += wpart[(int64_t)p * Ep + e];
+    wnorm[e] = sqrtf(v);
 }
 
-__device__ __forceinline__ float warp_max_wnorm(const float* wnorm2, int E, int lane) {
-    float wm = 0.f;
-    for (int e = lane; e < E; e += 32) wm = fmaxf(wm, wnorm2[e]);
+// Fast sigmoid: __expf (ex2.approx) and __fdividef.  For the keys compared below
+// its absolute error stays under 1e-6, inside ROUTE_KEY_SLACK (2e-6): the relative
+// error of e^{-v} is at most |v| log2(e) 2^-24 + 2^-22 and enters the sigmoid
+// multiplied by s(1 - s) <= 1/4 (and by e^{-|v|} for large |v|); the division adds
+// two ulp.
+__device__ __forceinline__ float sigmoid_fast(float v) {
+    return __fdividef(1.0f, 1.0f + __expf(-v));
+}
+
+// Logit error bound of expert e for a token: ROUTE_TAU_C 2^-24 |x_t| |W_r[:, e]|.
+__device__ __forceinline__ float logit_tau(float xn, float wn) {
+    return ROUTE_TAU_C * 5.9604645e-8f * xn * wn;
+}
+
+// Key half-width with the largest sigmoid slope inside [s - tau_s, s + tau_s]
+// (the slope s(1 - s) falls with |s|).
+__device__ __forceinline__ float key_tau_exact_slope(float s, float tau_s) {
+    const float z = fmaxf(fabsf(s) - tau_s, 0.f);
+    const float sz = sigmoid_fast(z);
+    return tau_s * (sz * (1.f - sz)) + ROUTE_KEY_SLACK;
+}
+
+__device__ __forceinline__ float warp_sum(float v) {
 #pragma unroll
-    for (int o = 16; o; o >>= 1) wm = fmaxf(wm, __shfl_xor_sync(0xffffffffu, wm, o));
-    return wm;
+    for (int o = 16; o; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+    return v;
+}
+
+// |x_t| by one warp (16-byte loads; d % 8 == 0).
+__device__ __forceinline__ float row_norm(const __nv_bfloat16* xt, int d, int lane) {
+    float acc = 0.f;
+    for (int c = lane; c < d / 8; c += 32) {
+        float v[8];
+        unpack_bf16x8(*reinterpret_cast<const uint4*>(xt + 8 * c), v);
+#pragma unroll
+        for (int q = 0; q < 8; ++q) acc = fmaf(v[q], v[q], acc);
+    }
+    return sqrtf(warp_sum(acc));
+}
+
+// Warp arg-max of (value, id): largest value, ties to the lower id.
+__device__ __forceinline__ void warp_argmax(float& v, int& id) {
+#pragma unroll
+    for (int o = 16; o; o >>= 1) {
+        const float ov = __shfl_xor_sync(0xffffffffu, v, o);
+        const int oi = __shfl_xor_sync(0xffffffffu, id, o);
+        if (ov > v || (ov == v && oi < id)) {
+            v = ov;
+            id = oi;
+        }
+    }
 }
 
 // One warp per token.  NPL = experts per lane (expert e sits in lane e % 32, slot e / 32).
 template <int NPL>
 __global__ void __launch_bounds__(256) route_topk_kernel(
-    const float* __restrict__ s, const float* __restrict__ b, const float* __restrict__ xnorm2,
-    const float* __restrict__ wnorm2, int T, int E, int k, int32_t* __restrict__ idx,
-    float* __restrict__ gate, int32_t* __restrict__ fb_tokens, DevStatus* st) {
+    const __nv_bfloat16* __restrict__ x, const float* __restrict__ s, int ld,
+    const float* __restrict__ b, const float* __restrict__ wnorm, int T, int d, int E, int k,
+    int32_t* __restrict__ idx, float* __restrict__ gate, float* __restrict__ xnorm,
+    int32_t* __restrict__ fb_tokens, DevStatus* st) {
     const int lane = threadIdx.x & 31;
-    const int t = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+    const int t = (int)(((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5);
     if (t >= T) return;
-    const float wmax2 = warp_max_wnorm(wnorm2, E, lane);
-    const float tau = key_tau(xnorm2[t], wmax2);
-    float key[NPL], sg[NPL];
+    const float xn = row_norm(x + (int64_t)t * d, d, lane);
+    if (lane == 0) xnorm[t] = xn;
+    float sv[NPL], key[NPL], ts[NPL];
 #pragma unroll
     for (int i = 0; i < NPL; ++i) {
         const int e = lane + 32 * i;
         if (e < E) {
-            sg[i] = sigmoid_f32(s[(int64_t)t * E + e]);
-            key[i] = sg[i] + b[e];
+            sv[i] = s[(int64_t)t * ld + e];
+            key[i] = sigmoid_fast(sv[i]) + b[e];
+            ts[i] = logit_tau(xn, wnorm[e]);
         } else {
-            sg[i] = 0.f;
+            sv[i] = 0.f;
             key[i] = -INFINITY;
+            ts[i] = 0.f;
         }
     }
     uint32_t taken = 0;
-    float kth = 0.f, next = -INFINITY;
-    const int rounds = (k < E) ? k + 1 : k;
-    for (int j = 0; j < rounds; ++j) {
+    for (int j = 0; j < k; ++j) {
         float bv = -INFINITY;
         int bi = 0x7fffffff;
 #pragma unroll
@@ -175,23 +168,28 @@ __global__ void __launch_bounds__(256) route_topk_kernel(
                 bi = e;
             }
         }
+        warp_argmax(bv, bi);
+        if ((bi & 31) == lane) taken |= 1u << (bi >> 5);
+    }
+    bool certain = k >= E;
+    for (int pass = 0; pass < 2 && !certain; ++pass) {
+        float lo_in = INFINITY, hi_out = -INFINITY;
+#pragma unroll
+        for (int i = 0; i < NPL; ++i) {
+            const int e = lane + 32 * i;
+            if (e >= E) continue;
+            const float tk = pass == 0 ? 0.25f * ts[i] + ROUTE_KEY_SLACK
+                                       : key_tau_exact_slope(sv[i], ts[i]);
+            if ((taken >> i) & 1u) lo_in = fminf(lo_in, key[i] - tk);
+            else hi_out = fmaxf(hi_out, key[i] + tk);
+        }
 #pragma unroll
         for (int o = 16; o; o >>= 1) {
-            const float ov = __shfl_xor_sync(0xffffffffu, bv, o);
-            const int oi = __shfl_xor_sync(0xffffffffu, bi, o);
-            if (ov > bv || (ov == bv && oi < bi)) {
-                bv = ov;
-                bi = oi;
-            }
+            lo_in = fminf(lo_in, __shfl_xor_sync(0xffffffffu, lo_in, o));
+            hi_out = fmaxf(hi_out, __shfl_xor_sync(0xffffffffu, hi_out, o));
         }
-        if (j < k) {
-            if ((bi & 31) == lane) taken |= 1u << (bi >> 5);
-            kth = bv;
-        } else {
-            next = bv;
-        }
+        certain = lo_in > hi_out;
     }
-    const bool certain = (k >= E) || (kth - next > 2.0f * tau);
     if (!certain) {
         if (lane == 0) {
             const int p = atomicAdd(&st->fb_count, 1);
@@ -200,11 +198,13 @@ __global__ void __launch_bounds__(256) route_topk_kernel(
         return;
     }
     float ssum = 0.f;
+    float sg[NPL];
 #pragma unroll
-    for (int i = 0; i < NPL; ++i)
-        if ((taken >> i) & 1u) ssum += sg[i];
-#pragma unroll
-    for (int o = 16; o; o >>= 1) ssum += __shfl_xor_sync(0xffffffffu, ssum, o);
+    for (int i = 0; i < NPL; ++i) {
+        sg[i] = ((taken >> i) & 1u) ? sigmoid_fast(sv[i]) : 0.f;
+        ssum += sg[i];
+    }
+    ssum = warp_sum(ssum);
     const uint32_t lt = (1u << lane) - 1u;
     int base = 0;
 #pragma unroll
@@ -213,137 +213,226 @@ __global__ void __launch_bounds__(256) route_topk_kernel(
         if ((taken >> i) & 1u) {
             const int pos = base + __popc(m & lt);
             idx[(int64_t)t * k + pos] = lane + 32 * i;
-            gate[(int64_t)t * k + pos] = sg[i] / ssum;
+            gate[(int64_t)t * k + pos] = __fdividef(sg[i], ssum);
         }
         base += __popc(m);
     }
 }
 
-constexpr int FB_THREADS = 256;
+constexpr int FB_BATCH = 8;   // candidates whose exact logits are summed together
 
-// Exact re-decision of uncertified tokens.  Dynamic smem: E floats (fast keys),
-// E floats (fast sigmoid), E bytes (class), E doubles (exact keys).
-__global__ void __launch_bounds__(FB_THREADS) route_fallback_kernel(
-    const __nv_bfloat16* __restrict__ x, const float* __restrict__ Wr,
-    const float* __restrict__ b, const float* __restrict__ s, const float* __restrict__ xnorm2,
-    const float* __restrict__ wnorm2, int d, int E, int k, int32_t* __restrict__ idx,
-    float* __restrict__ gate, const int32_t* __restrict__ fb_tokens, DevStatus* st) {
-    extern __shared__ __align__(16) uint8_t fb_smem[];
-    double* exk = reinterpret_cast<double*>(fb_smem);
-    float* key = reinterpret_cast<float*>(exk + E);
-    float* sg = key + E;
-    uint8_t* cls = reinterpret_cast<uint8_t*>(sg + E);   // 1 sure in, 2 sure out, 3 candidate, 4 chosen
-    __shared__ int s_in, s_cand;
-    __shared__ float s_wmax2;
-    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-    if (warp == 0) {
-        const float wm = warp_max_wnorm(wnorm2, E, lane);
-        if (lane == 0) s_wmax2 = wm;
-    }
-    __syncthreads();
-    const int nfb = st->fb_count;
-    for (int i = blockIdx.x; i < nfb; i += gridDim.x) {
-        const int t = fb_tokens[i];
-        const float tau = key_tau(xnorm2[t], s_wmax2);
-        for (int e = tid; e < E; e += FB_THREADS) {
-            sg[e] = sigmoid_f32(s[(int64_t)t * E + e]);
-            key[e] = sg[e] + b[e];
-        }
-        if (tid == 0) {
-            s_in = 0;
-            s_cand = 0;
-        }
-        __syncthreads();
-        // classify against the fast-key intervals [key - tau, key + tau]
-        for (int e = tid; e < E; e += FB_THREADS) {
-            int maybe_above = 0, surely_above = 0;
-            for (int f = 0; f < E; ++f) {
-                if (f == e) continue;
-                if (key[f] + tau >= key[e] - tau) ++maybe_above;
-                if (key[f] - tau > key[e] + tau) ++surely_above;
-            }
-            uint8_t c = 3;
-            if (maybe_above < k) c = 1;
-            else if (surely_above >= k) c = 2;
-            cls[e] = c;
-            if (c == 1) atomicAdd(&s_in, 1);
-            if (c == 3) atomicAdd(&s_cand, 1);
-        }
-        __syncthreads();
-        // exact keys of the candidates: one warp per candidate
-        for (int e = warp; e < E; e += FB_THREADS / 32) {
-            if (cls[e] != 3) continue;
-            double acc = 0.0;
-            for (int j = lane; j < d; j += 32)
-                acc += static_cast<double>(__bfloat162float(x[(int64_t)t * d + j])) *
-                       static_cast<double>(Wr[(int64_t)j * E + e]);
+// k-th and (k+1)-th largest of v over the warp (k rounds of arg-max; k <= E).
+template <int NPL>
+__device__ __forceinline__ void warp_kth_values(const float (&v)[NPL], int E, int k, int lane,
+                                                float& kth, float& kth1) {
+    uint32_t used = 0;
+    kth = -INFINITY;
+    kth1 = -INFINITY;
+    const int rounds = k < E ? k + 1 : k;
+    for (int j = 0; j < rounds; ++j) {
+        float bv = -INFINITY;
+        int bi = 0x7fffffff;
 #pragma unroll
-            for (int o = 16; o; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
-            if (lane == 0) exk[e] = 1.0 / (1.0 + exp(-acc)) + static_cast<double>(b[e]);
-        }
-        __syncthreads();
-        if (tid == 0) {
-            const int need = k - s_in;
-            if (need < 0 || need > s_cand) report(st, MOEVIE_ERR_DEVICE, SITE_ROUTE_FALLBACK, t, need);
-            for (int r = 0; r < need; ++r) {
-                int best = -1;
-                for (int e = 0; e < E; ++e)
-                    if (cls[e] == 3 && (best < 0 || exk[e] > exk[best])) best = e;
-                if (best < 0) break;
-                cls[best] = 4;
-            }
-            float ssum = 0.f;
-            for (int e = 0; e < E; ++e)
-                if (cls[e] == 1 || cls[e] == 4) ssum += sg[e];
-            int pos = 0;
-            for (int e = 0; e < E && pos < k; ++e)
-                if (cls[e] == 1 || cls[e] == 4) {
-                    idx[(int64_t)t * k + pos] = e;
-                    gate[(int64_t)t * k + pos] = sg[e] / ssum;
-                    ++pos;
-                }
-            for (; pos < k; ++pos) {   // only after a reported inconsistency
-                idx[(int64_t)t * k + pos] = 0;
-                gate[(int64_t)t * k + pos] = 0.f;
+        for (int i = 0; i < NPL; ++i) {
+            const int e = lane + 32 * i;
+            if (e < E && !((used >> i) & 1u) && (v[i] > bv || bi == 0x7fffffff)) {
+                bv = v[i];
+                bi = e;
             }
         }
-        __syncthreads();
+        warp_argmax(bv, bi);
+        if ((bi & 31) == lane) used |= 1u << (bi >> 5);
+        if (j == k - 1) kth = bv;
+        if (j == k) kth1 = bv;
     }
 }
+
+// Exact re-decision of uncertified tokens, one warp per token.
+template <int NPL>
+__global__ void __launch_bounds__(256) route_fallback_kernel(
+    const __nv_bfloat16* __restrict__ x, const float* __restrict__ Wr,
+    const float* __restrict__ b, const float* __restrict__ s, int ld,
+    const float* __restrict__ xnorm, const float* __restrict__ wnorm, int d, int E, int k,
+    int32_t* __restrict__ idx, float* __restrict__ gate, const int32_t* __restrict__ fb_tokens,
+    DevStatus* st) {
+    const int lane = threadIdx.x & 31;
+    const int64_t wid = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+    const int64_t nwarps = ((int64_t)gridDim.x * blockDim.x) >> 5;
+    const int nfb = st->fb_count;
+    for (int64_t f = wid; f < nfb; f += nwarps) {
+        const int t = fb_tokens[f];
+        const float xn = xnorm[t];
+        float sv[NPL], up[NPL], lo[NPL];
+#pragma unroll
+        for (int i = 0; i < NPL; ++i) {
+            const int e = lane + 32 * i;
+            if (e < E) {
+                sv[i] = s[(int64_t)t * ld + e];
+                const float key = sigmoid_fast(sv[i]) + b[e];
+                const float tk = key_tau_exact_slope(sv[i], logit_tau(xn, wnorm[e]));
+                up[i] = key + tk;
+                lo[i] = key - tk;
+            } else {
+                sv[i] = 0.f;
+                up[i] = lo[i] = -INFINITY;
+            }
+        }
+        // k-th / (k+1)-th largest upper ends and k-th largest lower end
+        float u_k, u_k1, l_k, l_k1;
+        warp_kth_values<NPL>(up, E, k, lane, u_k, u_k1);
+        warp_kth_values<NPL>(lo, E, k, lane, l_k, l_k1);
+        uint32_t sure_in = 0, cand = 0;
+#pragma unroll
+        for (int i = 0; i < NPL; ++i) {
+            const int e = lane + 32 * i;
+            if (e >= E) continue;
+            // k-th largest upper end among the others (u_k when e may sit at rank k: conservative)
+            const float thr = up[i] > u_k ? u_k1 : u_k;
+            if (k >= E || lo[i] > thr) sure_in |= 1u << i;
+            else if (!(up[i] < l_k)) cand |= 1u << i;
+        }
+        int n_in = 0, n_cand = 0;
+#pragma unroll
+        for (int i = 0; i < NPL; ++i) {
+            n_in += __popc(__ballot_sync(0xffffffffu, (sure_in >> i) & 1u));
+            n_cand += __popc(__ballot_sync(0xffffffffu, (cand >> i) & 1u));
+        }
+        const int need = k - n_in;
+        if (need < 0 || need > n_cand) {
+            if (lane == 0) report(st, MOEVIE_ERR_DEVICE, SITE_ROUTE_FALLBACK, t, need);
+            continue;
+        }
+        // exact keys of the candidates, FB_BATCH at a time, lanes over d
+        double exk[NPL];
+#pragma unroll
+        for (int i = 0; i < NPL; ++i) exk[i] = -INFINITY;
+        for (int done = 0; done < n_cand;) {
+            int ids[FB_BATCH];
+            int nb = 0, seen = 0;
+#pragma unroll
+            for (int i = 0; i < NPL; ++i) {
+                uint32_t m = __ballot_sync(0xffffffffu, (cand >> i) & 1u);
+                while (m && nb < FB_BATCH) {
+                    const int l = __ffs(m) - 1;
+                    m &= m - 1;
+                    if (seen++ >= done) ids[nb++] = l + 32 * i;
+                }
+            }
+#pragma unroll
+            for (int q = 0; q < FB_BATCH; ++q)
+                if (q >= nb) ids[q] = ids[0];
+            double acc[FB_BATCH];
+#pragma unroll
+            for (int q = 0; q < FB_BATCH; ++q) acc[q] = 0.0;
+            for (int j = lane; j < d; j += 32) {
+                const double xv = (double)__bfloat162float(x[(int64_t)t * d + j]);
+                const float* wrow = Wr + (int64_t)j * E;
+#pragma unroll
+                for (int q = 0; q < FB_BATCH; ++q) acc[q] += xv * (double)wrow[ids[q]];
+            }
+#pragma unroll
+            for (int q = 0; q < FB_BATCH; ++q) {
+                double v = acc[q];
+#pragma unroll
+                for (int o = 16; o; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+                const int e = ids[q];
+                if (q < nb && (e & 31) == lane) {
+                    const double key = 1.0 / (1.0 + exp(-v)) + (double)b[e];
+#pragma unroll
+                    for (int i = 0; i < NPL; ++i)
+                        if (i == (e >> 5)) exk[i] = key;
+                }
+            }
+            done += nb;
+        }
+        // choose `need` candidates by exact key, ties to the lower id
+        uint32_t chosen = sure_in;
+        for (int r = 0; r < need; ++r) {
+            double bv = -INFINITY;
+            int bi = 0x7fffffff;
+#pragma unroll
+            for (int i = 0; i < NPL; ++i) {
+                const int e = lane + 32 * i;
+                if (((cand >> i) & 1u) && !((chosen >> i) & 1u) && (exk[i] > bv || bi == 0x7fffffff)) {
+                    bv = exk[i];
+                    bi = e;
+                }
+            }
+#pragma unroll
+            for (int o = 16; o; o >>= 1) {
+                const double ov = __shfl_xor_sync(0xffffffffu, bv, o);
+                const int oi = __shfl_xor_sync(0xffffffffu, bi, o);
+                if (ov > bv || (ov == bv && oi < bi)) {
+                    bv = ov;
+                    bi = oi;
+                }
+            }
+            if ((bi & 31) == lane) chosen |= 1u << (bi >> 5);
+        }
+        float sg[NPL];
+        float ssum = 0.f;
+#pragma unroll
+        for (int i = 0; i < NPL; ++i) {
+            sg[i] = ((chosen >> i) & 1u) ? sigmoid_fast(sv[i]) : 0.f;
+            ssum += sg[i];
+        }
+        ssum = warp_sum(ssum);
+        const uint32_t lt = (1u << lane) - 1u;
+        int base = 0;
+#pragma unroll
+        for (int i = 0; i < NPL; ++i) {
+            const uint32_t m = __ballot_sync(0xffffffffu, (chosen >> i) & 1u);
+            if ((chosen >> i) & 1u) {
+                const int pos = base + __popc(m & lt);
+                idx[(int64_t)t * k + pos] = lane + 32 * i;
+                gate[(int64_t)t * k + pos] = __fdividef(sg[i], ssum);
+            }
+            base += __popc(m);
+        }
+    }
+}
+
+__global__ void reset_fallback_count(DevStatus* st) { st->fb_count = 0; }
 
 }  // namespace
 
-cudaError_t launch_route_logits(const __nv_bfloat16* x, const float* Wr, int T, int d, int E,
-                                const RouteBufs& rb, DevStatus* st, cudaStream_t s) {
-    dim3 grid((T + LG_TT - 1) / LG_TT, (E + LG_TE - 1) / LG_TE);
-    route_logits_kernel<<<grid, 256, 0, s>>>(x, Wr, T, d, E, rb.logits, rb.xnorm2, rb.wnorm2, st);
-    count_launches(1);
+int route_split_parts(int d) { return (route_dpad(d) + SPLIT_ROWS - 1) / SPLIT_ROWS; }
+
+cudaError_t launch_route_split(const float* Wr, int d, int E, __nv_bfloat16* Wsplit, float* wpart,
+                               float* wnorm, cudaStream_t s) {
+    const int Ep = route_epad(E);
+    const int parts = route_split_parts(d);
+    route_split_kernel<<<dim3((Ep + 31) / 32, parts), 256, 0, s>>>(Wr, d, route_dpad(d), E, Ep,
+                                                                   Wsplit, wpart);
+    route_wnorm_kernel<<<(E + 255) / 256, 256, 0, s>>>(wpart, parts, E, Ep, wnorm);
+    count_launches(2);
     return cudaGetLastError();
 }
 
-cudaError_t launch_route_select(const __nv_bfloat16* x, const float* Wr, const float* b, int T,
-                                int d, int E, int k, int32_t* idx, float* gate,
-                                const RouteBufs& rb, DevStatus* st, int num_sms, cudaStream_t s) {
+cudaError_t launch_route_select(const __nv_bfloat16* x, const float* Wr, const float* b,
+                                const float* logits, int ld, const float* wnorm, int T, int d,
+                                int E, int k, int32_t* idx, float* gate, int32_t* fb_tokens,
+                                float* xnorm, DevStatus* st, int num_sms, cudaStream_t s) {
+    reset_fallback_count<<<1, 1, 0, s>>>(st);
     const int blocks = (int)(((int64_t)T * 32 + 255) / 256);
+    const int64_t fb_warps = T < 16 * (int64_t)num_sms ? (int64_t)T : 16 * (int64_t)num_sms;
+    const int fb_blocks = (int)((fb_warps * 32 + 255) / 256);
     const int npl = (E + 31) / 32;
-#define MV_TOPK(N)                                                                            \
-    route_topk_kernel<N><<<blocks, 256, 0, s>>>(rb.logits, b, rb.xnorm2, rb.wnorm2, T, E, k, \
-                                                idx, gate, rb.fb_tokens, st)
-    if (npl <= 1) MV_TOPK(1);
-    else if (npl <= 2) MV_TOPK(2);
-    else if (npl <= 4) MV_TOPK(4);
-    else if (npl <= 8) MV_TOPK(8);
-    else if (npl <= 16) MV_TOPK(16);
-    else MV_TOPK(32);
-#undef MV_TOPK
-    cudaError_t err = cudaGetLastError();
-    if (err != cudaSuccess) return err;
-    const size_t smem = (size_t)E * (8 + 4 + 4 + 1);
-    const int fb_grid = T < 2 * num_sms ? T : 2 * num_sms;
-    route_fallback_kernel<<<fb_grid, FB_THREADS, smem, s>>>(x, Wr, b, rb.logits, rb.xnorm2,
-                                                            rb.wnorm2, d, E, k, idx, gate,
-                                                            rb.fb_tokens, st);
-    count_launches(2);
+#define MV_ROUTE(N)                                                                              \
+    do {                                                                                         \
+        route_topk_kernel<N><<<blocks, 256, 0, s>>>(x, logits, ld, b, wnorm, T, d, E, k, idx,    \
+                                                    gate, xnorm, fb_tokens, st);                 \
+        route_fallback_kernel<N><<<fb_blocks, 256, 0, s>>>(x, Wr, b, logits, ld, xnorm, wnorm, d, \
+                                                           E, k, idx, gate, fb_tokens, st);      \
+    } while (0)
+    if (npl <= 1) MV_ROUTE(1);
+    else if (npl <= 2) MV_ROUTE(2);
+    else if (npl <= 4) MV_ROUTE(4);
+    else if (npl <= 8) MV_ROUTE(8);
+    else if (npl <= 16) MV_ROUTE(16);
+    else MV_ROUTE(32);
+#undef MV_ROUTE
+    count_launches(3);
     return cudaGetLastError();
 }
 

@@ -279,12 +279,14 @@ def moevie_test_moe_forward_events(layer: LayerWeights, x, ws: Workspace, events
 
 
 def moevie_test_route_logits(x, W_r, ws: Workspace, stream=None):
+    """Fast-path logits [T, E] (the library writes E rounded up to 16 columns)."""
     T, d = x.shape
     E = W_r.shape[1]
-    s = torch.empty((T, E), dtype=torch.float32, device=x.device)
+    E16 = (E + 15) // 16 * 16
+    s = torch.empty((T, E16), dtype=torch.float32, device=x.device)
     _call("moevie_test_route_logits", _p(x), _p(W_r), T, d, E, _p(s), ws.ptr, ws.nbytes,
           _stream(stream))
-    return s
+    return s[:, :E]
 
 
 def moevie_test_fallback_count(ws: Workspace, stream=None) -> int:

@@ -82,18 +82,20 @@ def test_route_full_configs(name):
     print(f"{name}: {nfb} of {lay.cfg.T} tokens re-decided exactly")
 
 
-@pytest.mark.parametrize("name", ["c1", "c4"])
+@pytest.mark.parametrize("name", ["c0", "c1", "c4"])
 def test_fast_logit_error_within_bound(name):
-    """The fp32 logits stay far inside the error bound the router certifies with
-    (ROUTE_TAU_C = 64 units of 2^-24 |x| max|w|): measured max below 1/4 of it."""
+    """The tensor-core logits stay far inside the error bound the router certifies
+    with (ROUTE_TAU_C = 128 units of 2^-24 |x_t| |W_r[:, e]|): measured max below 1/4
+    of it over every token of the layer."""
     lay = workloads.make_layer(workloads.CONFIGS[name])
-    T = min(lay.cfg.T, 8192)
+    T = lay.cfg.T
     x, Wr = lay.x[:T], lay.Wr
     ws = moevie.Workspace(T, lay.cfg.d, lay.cfg.E, 1, 16)
     s = moevie.moevie_test_route_logits(dev_bf16(x), dev(Wr), ws).cpu().numpy().astype(np.float64)
+    check_status(ws)
     so = oracle.logits(x, Wr)
     xf = workloads.bf16_bits_to_f32(x).astype(np.float64)
-    scale = 2.0 ** -24 * np.linalg.norm(xf, axis=1)[:, None] * np.linalg.norm(Wr.astype(np.float64), axis=0).max()
+    scale = 2.0 ** -24 * np.linalg.norm(xf, axis=1)[:, None] * np.linalg.norm(Wr.astype(np.float64), axis=0)[None, :]
     ratio = np.abs(s - so) / scale
-    print(f"{name}: max |s_fast - s| = {ratio.max():.2f} units of 2^-24 |x| max|w|")
-    assert ratio.max() < 64 / 4
+    print(f"{name}: max |s_fast - s| = {ratio.max():.3f} units of 2^-24 |x_t| |W_r[:, e]|")
+    assert ratio.max() < 128 / 4
