@@ -144,6 +144,38 @@ moevie_status moevie_moe_forward(const moevie_layer* layer, const void* x, int64
                                  const moevie_routing* routing, void* ws, size_t ws_bytes,
                                  void* stream);
 
+/* moevie_permute without a workspace (the paper has no counterpart: this is a
+ * calling convention, not part of the method).  Same inputs, outputs, ordering and
+ * validation as moevie_permute, and bit-identical results.
+ *
+ * Who it is for: callers that cannot give the library scratch memory and cannot let
+ * it allocate any -- e.g. code running inside another framework's operator that
+ * only hands over its input and output buffers, or a process whose device memory
+ * is all reserved up front by its own pool, where a cudaMalloc would fail or would
+ * synchronise the device at a bad moment.  This entry point makes no cudaMalloc or
+ * cudaFree and calls no allocating library: its scratch is one fixed array of
+ * 2,179,584 bytes in the library's device image, one copy per device.
+ *
+ * Limits: T * k <= 1048576 (2^20) flat slots, plus the limits of moevie_permute
+ * (1 <= k <= E <= 1024); larger inputs return MOEVIE_ERR_UNSUPPORTED before
+ * anything is enqueued.
+ *
+ * Set-up: the first call on a device (with that device current) looks up the
+ * array's device address, which may load the library's device code; make that
+ * first call before any stream capture.  Later calls reuse the address.
+ *
+ * Concurrency: all calls on one device share the one array.  Two calls whose GPU
+ * work overlaps (different streams, or several host threads without ordering) race
+ * on it and give undefined results; order them on one stream or with events.
+ *
+ * Device-side errors: each call clears the array's status block; an expert id
+ * outside [0, E) drops its slot (inv = -1, not counted in counts / offsets) and is
+ * recorded there, but no entry point reads that status back -- check inv for -1
+ * where ids are untrusted. */
+moevie_status moevie_permute_static(const int32_t* idx, int64_t T, int64_t k, int64_t E,
+                                    int32_t* counts, int32_t* offsets, int32_t* perm,
+                                    int32_t* inv, void* stream);
+
 /* Number of kernels this library has launched since it was loaded (all
  * threads, all devices).  Host-only. */
 uint64_t moevie_launch_count(void);

@@ -350,6 +350,39 @@ moevie_status moevie_permute(const int32_t* idx, int64_t T, int64_t k, int64_t E
     return MOEVIE_OK;
 }
 
+moevie_status moevie_permute_static(const int32_t* idx, int64_t T, int64_t k, int64_t E,
+                                    int32_t* counts, int32_t* offsets, int32_t* perm,
+                                    int32_t* inv, void* stream) {
+    moevie_status c = check_sizes(T, 8, E, k, 0, 0);
+    if (c != MOEVIE_OK) return c;
+    if (T * k > PERM_STATIC_MAX_SLOTS) return MOEVIE_ERR_UNSUPPORTED;   // beyond the fixed scratch
+    if (!counts || !offsets) return MOEVIE_ERR_INVALID_ARG;
+    if (T > 0 && (!idx || !perm || !inv)) return MOEVIE_ERR_INVALID_ARG;
+    if (idx && !a16(idx)) return MOEVIE_ERR_INVALID_ARG;
+    unsigned char* scratch = nullptr;
+    MV_TRY(perm_static_scratch(&scratch));   // the first call on a device looks it up
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    if (T == 0) {
+        MV_TRY(cudaMemsetAsync(counts, 0, 4 * E, s));
+        MV_TRY(cudaMemsetAsync(offsets, 0, 4 * (E + 1), s));
+        return MOEVIE_OK;
+    }
+    // The status block must start at zero (a report only lands in a clear block);
+    // the histograms, tile table and tile count are fully rewritten by the kernels.
+    DevStatus* st = reinterpret_cast<DevStatus*>(scratch);
+    MV_TRY(cudaMemsetAsync(st, 0, sizeof(DevStatus), s));
+    const int64_t n = T * k;
+    int64_t chunk = perm_chunk(n, num_sms());
+    const int64_t min_chunk = ((n + PERM_STATIC_MAX_CHUNKS - 1) / PERM_STATIC_MAX_CHUNKS + 255) / 256 * 256;
+    if (chunk < min_chunk) chunk = min_chunk;   // at most PERM_STATIC_MAX_CHUNKS histograms
+    MV_TRY(launch_permute(idx, n, (int)k, (int)E, GM_BM, (int)chunk, nullptr,
+                          reinterpret_cast<int32_t*>(scratch + PERM_STATIC_HIST_OFF), counts, offsets,
+                          reinterpret_cast<int4*>(scratch + PERM_STATIC_TILES_OFF),
+                          reinterpret_cast<int32_t*>(scratch + PERM_STATIC_NTILES_OFF), perm, inv,
+                          nullptr, nullptr, st, s));
+    return MOEVIE_OK;
+}
+
 moevie_status moevie_expert_ffn(const void* x, const int32_t* perm, const int32_t* offsets,
                                 const void* W1, const void* W2, int64_t T, int64_t d, int64_t h,
                                 int64_t E, int64_t k, void* out_rows, void* ws, size_t ws_bytes,

@@ -125,6 +125,31 @@ bool make_rows_tmap(CUtensorMap* tm, const void* base, int64_t cols, int64_t row
 void choose_bn(int N, int* BN, int* n_ntiles);
 cudaError_t launch_grouped_gemm(const GemmArgs& a, int grid, cudaStream_t s);
 
+// ---------------------------------------- permute without a caller workspace
+
+// moevie_permute_static keeps its scratch in one fixed device array (in permute.cu):
+//   [0, 256)                 DevStatus (cleared by every call)
+//   [256, 260)               number of m-tiles
+//   [PERM_STATIC_HIST_OFF)   chunk histograms, <= PERM_STATIC_MAX_CHUNKS x 1024 int32
+//   [PERM_STATIC_TILES_OFF)  m-tile table, <= max_mtiles(PERM_STATIC_MAX_SLOTS, 1024) int4
+constexpr int64_t PERM_STATIC_MAX_SLOTS = int64_t(1) << 20;   // largest T * k
+constexpr int PERM_STATIC_MAX_CHUNKS = 512;
+constexpr size_t PERM_STATIC_NTILES_OFF = 256;
+constexpr size_t PERM_STATIC_HIST_OFF = 512;
+constexpr size_t PERM_STATIC_TILES_OFF =
+    PERM_STATIC_HIST_OFF + size_t(4) * PERM_STATIC_MAX_CHUNKS * 1024;
+constexpr size_t PERM_STATIC_SCRATCH_BYTES =
+    PERM_STATIC_TILES_OFF + size_t(16) * ((PERM_STATIC_MAX_SLOTS + GM_BM - 1) / GM_BM + 1024);
+
+static_assert((PERM_STATIC_MAX_SLOTS + PERM_STATIC_MAX_CHUNKS - 1) / PERM_STATIC_MAX_CHUNKS <=
+                  PERM_CHUNK_MAX,
+              "the largest permute must fit PERM_STATIC_MAX_CHUNKS chunks");
+
+// Device address of that array on the current device.  The first call on a device
+// looks the symbol up (cudaGetSymbolAddress, which may load the module); later calls
+// return the cached address.  Thread-safe.
+cudaError_t perm_static_scratch(unsigned char** out);
+
 // ------------------------------------------------------------------- misc
 
 cudaError_t launch_zero_f32(float* p, int64_t n, cudaStream_t s);

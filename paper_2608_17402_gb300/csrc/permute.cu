@@ -10,6 +10,8 @@
 //                       (warp match + per-warp running counts), and writes perm,
 //                       inv and the per-row token (pos // K) and gate.
 // Inside one expert's segment, rows keep ascending slot order t*k + j.
+#include <mutex>
+
 #include "internal.h"
 
 namespace mv {
@@ -216,6 +218,29 @@ __global__ void __launch_bounds__(1024) tile_table_kernel(const int32_t* __restr
 }
 
 }  // namespace
+
+// Scratch of moevie_permute_static: fixed size, so that entry point needs neither a
+// workspace from its caller nor an allocation of its own (layout in internal.h).
+static __device__ __align__(256) unsigned char g_perm_static_scratch[PERM_STATIC_SCRATCH_BYTES];
+
+cudaError_t perm_static_scratch(unsigned char** out) {
+    constexpr int kMaxDevices = 64;
+    static std::mutex mu;
+    static unsigned char* addr[kMaxDevices] = {};
+    int dev = -1;
+    cudaError_t err = cudaGetDevice(&dev);
+    if (err != cudaSuccess) return err;
+    if (dev < 0 || dev >= kMaxDevices) return cudaErrorInvalidDevice;
+    std::lock_guard<std::mutex> lock(mu);
+    if (!addr[dev]) {   // once per device, with that device current
+        void* p = nullptr;
+        err = cudaGetSymbolAddress(&p, g_perm_static_scratch);
+        if (err != cudaSuccess) return err;
+        addr[dev] = static_cast<unsigned char*>(p);
+    }
+    *out = addr[dev];
+    return cudaSuccess;
+}
 
 int perm_chunk(int64_t n, int num_sms) {
     int64_t c = (n + 2 * num_sms - 1) / (2 * num_sms);

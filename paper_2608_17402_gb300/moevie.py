@@ -23,7 +23,8 @@ STATUS_NAMES = {0: "MOEVIE_OK", 1: "MOEVIE_ERR_INVALID_ARG", 2: "MOEVIE_ERR_UNSU
                 3: "MOEVIE_ERR_WORKSPACE", 4: "MOEVIE_ERR_CUDA", 5: "MOEVIE_ERR_TIMEOUT",
                 6: "MOEVIE_ERR_DEVICE"}
 C_ENTRY_POINTS = ("moevie_status_string", "moevie_version", "moevie_workspace_size",
-                  "moevie_workspace_init", "moevie_route", "moevie_permute", "moevie_expert_ffn",
+                  "moevie_workspace_init", "moevie_route", "moevie_permute", "moevie_permute_static",
+                  "moevie_expert_ffn",
                   "moevie_shared_expert", "moevie_combine", "moevie_moe_forward",
                   "moevie_get_device_status", "moevie_launch_count", "moevie_test_route_logits",
                   "moevie_test_fallback_count", "moevie_test_expert_hidden",
@@ -66,6 +67,7 @@ def load():
         "moevie_workspace_init": ([P, SZ, P], ctypes.c_int),
         "moevie_route": ([P, P, P, I64, I64, I64, I64, P, P, P, SZ, P], ctypes.c_int),
         "moevie_permute": ([P, I64, I64, I64, P, P, P, P, P, SZ, P], ctypes.c_int),
+        "moevie_permute_static": ([P, I64, I64, I64, P, P, P, P, P], ctypes.c_int),
         "moevie_expert_ffn": ([P, P, P, P, P, I64, I64, I64, I64, I64, P, P, SZ, P], ctypes.c_int),
         "moevie_shared_expert": ([P, P, P, I64, I64, I64, P, P, SZ, P], ctypes.c_int),
         "moevie_combine": ([P, P, P, P, F, I64, I64, I64, P, P], ctypes.c_int),
@@ -168,6 +170,21 @@ def moevie_permute(idx, E, ws: Workspace, stream=None):
     inv = torch.empty(T * k, dtype=torch.int32, device=dev)
     _call("moevie_permute", _p(idx), T, k, E, _p(counts), _p(offsets), _p(perm), _p(inv), ws.ptr,
           ws.nbytes, _stream(stream))
+    return counts, offsets, perm, inv
+
+
+def moevie_permute_static(idx, E, stream=None):
+    """moevie_permute without a workspace: the library's fixed device scratch is used
+    (T * k <= 2^20).  Calls whose GPU work overlaps race on that scratch."""
+    _want(idx, torch.int32, "idx")
+    T, k = idx.shape
+    dev = idx.device
+    counts = torch.empty(E, dtype=torch.int32, device=dev)
+    offsets = torch.empty(E + 1, dtype=torch.int32, device=dev)
+    perm = torch.empty(T * k, dtype=torch.int32, device=dev)
+    inv = torch.empty(T * k, dtype=torch.int32, device=dev)
+    _call("moevie_permute_static", _p(idx), T, k, E, _p(counts), _p(offsets), _p(perm), _p(inv),
+          _stream(stream))
     return counts, offsets, perm, inv
 
 
