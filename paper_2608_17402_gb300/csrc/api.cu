@@ -28,7 +28,7 @@ inline bool a16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) =
 // the order is fixed, so a workspace sized for the whole layer also serves each
 // stage (which passes 0 for the sizes it does not use).
 struct Layout {
-    size_t status, xnorm, wnorm, wpart, wsplit, logits, fb_tokens;
+    size_t status, xnorm, wnorm, wpart, wsplit, wrt, logits, fb_tokens;
     size_t idx, gate, hist, counts, offsets, tiles, n_tiles, perm, inv, row_tok, row_gate;
     size_t H, Hs, yacc;
     size_t total;
@@ -50,7 +50,8 @@ Layout make_layout(int64_t T, int64_t d, int64_t E, int64_t k, int64_t h, int64_
     L.wnorm = take(4 * E);
     L.wpart = take(4 * (int64_t)route_split_parts((int)d) * Ep);
     L.wsplit = take(2 * 3 * (int64_t)route_dpad((int)d) * Ep);
-    L.logits = take(4 * T * Ep);
+    L.wrt = take(4 * E * (int64_t)route_dpad((int)d));
+    L.logits = take(4 * route_logits_rows(T, (int)d, (int)E) * Ep);
     L.fb_tokens = take(4 * T);
     L.idx = take(4 * n);
     L.gate = take(4 * n);
@@ -131,6 +132,8 @@ struct GemmSpec {
     int o_div;
     const float* row_scale;
     float scale;
+    int ksplit;              // 0 or 1: no split of K; fp32 outputs only otherwise
+    int64_t y_split_stride;  // floats between the outputs of consecutive splits
 };
 
 moevie_status run_gemm(const GemmSpec& g, DevStatus* st, cudaStream_t s) {
@@ -166,9 +169,13 @@ moevie_status run_gemm(const GemmSpec& g, DevStatus* st, cudaStream_t s) {
     a.o_div = g.o_div > 0 ? g.o_div : 1;
     a.row_scale = g.row_scale;
     a.scale = g.scale;
+    a.ksplit = g.ksplit > 1 ? g.ksplit : 1;
+    if (a.ksplit > a.num_kb) return MOEVIE_ERR_UNSUPPORTED;
+    if (a.ksplit > 1 && g.epi != EPI_STORE_F32 && g.epi != EPI_ADD_F32) return MOEVIE_ERR_UNSUPPORTED;
+    a.y_split_stride = g.y_split_stride;
     a.status = st;
     a.limit_ns = WAIT_LIMIT_NS;
-    const int64_t work = a.max_mtiles * a.n_ntiles;     // one CTA pair per work item at most
+    const int64_t work = a.max_mtiles * a.n_ntiles * a.ksplit;   // one CTA pair per work item at most
     const int sms = num_sms() & ~1;
     const int grid = (int)(2 * work < sms ? (work > 0 ? 2 * work : 2) : sms);
     return cuda_status(launch_grouped_gemm(a, grid, s));
@@ -183,9 +190,13 @@ moevie_status route_impl(const void* x, const float* W_r, const float* b, int64_
     DevStatus* st = at<DevStatus>(ws, L.status);
     const int Ep = route_epad((int)E);
     __nv_bfloat16* wsplit = at<__nv_bfloat16>(ws, L.wsplit);
+    float* wrt = at<float>(ws, L.wrt);
     float* wnorm = at<float>(ws, L.wnorm);
-    float* logits = logits_out ? logits_out : at<float>(ws, L.logits);
-    MV_TRY(launch_route_split(W_r, (int)d, (int)E, wsplit, at<float>(ws, L.wpart), wnorm, s));
+    const int ksplit = route_ksplit(T, (int)d, (int)E);
+    // partial logits: ksplit arrays [T][Ep]; straight into logits_out when unsplit
+    float* logits = (logits_out && ksplit == 1) ? logits_out : at<float>(ws, L.logits);
+    const int64_t part_stride = T * Ep;
+    MV_TRY(launch_route_split(W_r, (int)d, (int)E, wsplit, wrt, at<float>(ws, L.wpart), wnorm, s));
     const int64_t dp = route_dpad((int)d);
     GemmSpec g{};
     g.A = x;
@@ -204,10 +215,17 @@ moevie_status route_impl(const void* x, const float* W_r, const float* b, int64_
     g.ldy = Ep;
     g.o_nrows = T;
     g.scale = 1.0f;
+    g.ksplit = ksplit;
+    g.y_split_stride = part_stride;
     moevie_status c = run_gemm(g, st, s);
-    if (c != MOEVIE_OK || logits_only) return c;
-    MV_TRY(launch_route_select(static_cast<const __nv_bfloat16*>(x), W_r, b, logits, Ep, wnorm,
-                               (int)T, (int)d, (int)E, (int)k, idx, gate,
+    if (c != MOEVIE_OK) return c;
+    if (logits_only) {
+        if (logits_out && ksplit > 1)
+            MV_TRY(launch_route_sum_parts(logits, part_stride, ksplit, part_stride, logits_out, s));
+        return MOEVIE_OK;
+    }
+    MV_TRY(launch_route_select(static_cast<const __nv_bfloat16*>(x), wrt, b, logits, Ep, ksplit,
+                               part_stride, wnorm, (int)T, (int)d, (int)E, (int)k, idx, gate,
                                at<int32_t>(ws, L.fb_tokens), at<float>(ws, L.xnorm), st,
                                num_sms(), s));
     return MOEVIE_OK;
@@ -472,6 +490,7 @@ static moevie_status forward_impl(const moevie_layer* Lr, const void* x, int64_t
     if (routing) r = *routing;
     int32_t* idx = r.idx ? r.idx : at<int32_t>(ws, L.idx);
     float* gate = r.gate ? r.gate : at<float>(ws, L.gate);
+    int32_t* counts = r.counts ? r.counts : at<int32_t>(ws, L.counts);
     int32_t* offsets = r.offsets ? r.offsets : at<int32_t>(ws, L.offsets);
     int32_t* perm = r.perm ? r.perm : at<int32_t>(ws, L.perm);
     int32_t* inv = r.inv ? r.inv : at<int32_t>(ws, L.inv);
@@ -492,7 +511,7 @@ static moevie_status forward_impl(const moevie_layer* Lr, const void* x, int64_t
     // 2. expert-major order (Algorithm 1, phase 1), per-row token and gate, m-tile table
     const int chunk = perm_chunk(T * k, num_sms());
     MV_TRY(launch_permute(idx, T * k, (int)k, (int)E, GM_BM, chunk, gate, at<int32_t>(ws, L.hist),
-                          r.counts, offsets, tiles, n_tiles, perm, inv, row_tok, row_gate, st, s));
+                          counts, offsets, tiles, n_tiles, perm, inv, row_tok, row_gate, st, s));
     MV_TRY(mark(2));
     // 3. y accumulator: lambda * shared expert, or zero
     if (hs > 0) {

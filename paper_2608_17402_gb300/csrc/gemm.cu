@@ -24,7 +24,7 @@
 // permute step (no host read of segment sizes), or, for one dense group, from
 // arithmetic.
 //
-// Warp roles (448 threads per CTA, one CTA per SM):
+// Warp roles (480 threads per CTA, one CTA per SM):
 //   warps 0-7   epilogue: tcgen05.ld of the CTA's 128 accumulator rows (warp w:
 //               TMEM lanes 32 (w%4)..+31, every other 16-column chunk), fused math,
 //               sector-wide stores (fp32 results pass a per-warp smem transpose)
@@ -32,10 +32,10 @@
 //   warp 9      lane 0: TMA loads of the B half and, for contiguous A rows, of A;
 //               the leader posts the byte count of both CTAs on its full barrier
 //   warps 10-13 token gather: 16-byte cp.async of A rows straight into the 128-byte
-//               swizzled K-major layout, two stages in flight per thread; after a
-//               stage's copies land and are fenced to the async proxy, each warp
-//               arrives once (leader: on its full barrier; peer: on a local barrier
-//               that the peer's idle MMA-warp lane forwards to the leader)
+//               swizzled K-major layout; each thread hands the completion of its
+//               copies to the stage's local afull barrier and moves on
+//   warp 14     lane 0: waits for afull, fences the stage to the async proxy and
+//               arrives on the leader's full barrier (remotely from the peer)
 // Shared memory: 6 stages x (A 128x64 + B 64x128) bf16; TMEM: two fp32 accumulators
 // of 256 columns, so the epilogue of one tile overlaps the main loop of the next.
 //
@@ -55,7 +55,6 @@ namespace mv {
 
 namespace {
 
-constexpr int A_LAG = 2;             // cp.async stages in flight per gather thread
 constexpr int STG_LD = GM_STG_LD;
 
 // ------------------------------------------------------------ pair helpers
@@ -74,6 +73,16 @@ __device__ __forceinline__ uint32_t peer_addr(uint32_t addr, uint32_t rank) {
 __device__ __forceinline__ void cluster_sync() {
     asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::
                      : "memory");
+}
+// 16-byte async-proxy copy from this CTA's shared memory to `dst_cluster` (shared
+// memory of a CTA of the cluster) that completes 16 transaction bytes on the
+// barrier `bar_cluster` of that CTA.
+__device__ __forceinline__ void bulk_signal_remote(uint32_t dst_cluster, uint32_t src,
+                                                   uint32_t bar_cluster) {
+    asm volatile(
+        "cp.async.bulk.shared::cluster.shared::cta.mbarrier::complete_tx::bytes [%0], [%1], 16, [%2];" ::
+            "r"(dst_cluster), "r"(src), "r"(bar_cluster)
+        : "memory");
 }
 __device__ __forceinline__ void mbar_arrive_remote(uint32_t bar_cluster) {
     asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(bar_cluster)
@@ -132,12 +141,18 @@ __device__ __forceinline__ void tc_commit_pair(uint32_t bar) {
 
 struct Tile {
     int g, row0, nrows, n0;
+    int kb0, kb1;   // k-blocks [kb0, kb1) of this item's split of K
+    int ks;         // split index
 };
 
 __device__ __forceinline__ Tile decode_tile(const GemmArgs& p, int64_t w) {
+    Tile t;
+    t.ks = (int)(w % p.ksplit);   // split of K fastest
+    w /= p.ksplit;
+    t.kb0 = (int)((int64_t)t.ks * p.num_kb / p.ksplit);
+    t.kb1 = (int)((int64_t)(t.ks + 1) * p.num_kb / p.ksplit);
     const int mt = (int)(w / p.n_ntiles);
     const int nt = (int)(w - (int64_t)mt * p.n_ntiles);
-    Tile t;
     if (p.tiles) {
         const int4 d = __ldg(p.tiles + mt);
         t.g = d.x;
@@ -181,6 +196,7 @@ struct Smem {
     uint32_t afull;           // peer CTA: its gather warps' copies of a stage have landed
     uint32_t tfull, tempty;
     uint32_t drain;
+    uint32_t sink;            // 16 bytes: target / source of the peer's stage signals
     float* stage_out;         // epilogue transpose buffers, 32 x STG_LD floats per warp
     uint32_t rank;            // rank of this CTA in its pair
     int64_t pair, npairs;     // pair index and count
@@ -210,6 +226,8 @@ __device__ void producer_tma(const GemmArgs& p, const Smem& sm, int64_t n_work,
     const uint32_t half_n = (uint32_t)p.BN / 2;
     const uint32_t nboxh = (half_n + 63) / 64;
     const uint32_t cta_bytes = nboxh * GM_BK * 128 + (gather ? 0u : (uint32_t)GM_A_BYTES);
+    // gathering: plus the 16-byte signal with which the peer publishes its A half
+    const uint32_t stage_tx = 2 * cta_bytes + (gather ? 16u : 0u);
     const uint32_t full_leader = peer_addr(sm.full, 0);
     int s = 0;
     uint32_t ph = 0;
@@ -220,13 +238,13 @@ __device__ void producer_tma(const GemmArgs& p, const Smem& sm, int64_t n_work,
         const int64_t wn = w + sm.npairs;
         Tile tn{};
         if (wn < n_work) tn = decode_tile(p, wn);
-        for (int kb = 0; kb < p.num_kb; ++kb) {
+        for (int kb = t.kb0; kb < t.kb1; ++kb) {
             if (!mbar_wait(sm.empty + 8 * s, ph ^ 1u, p.limit_ns, abort_flag)) {
                 set_abort(abort_flag, p.status, SITE_GEMM_WAIT_EMPTY, (int)sm.pair, 1);
                 return;
             }
             const uint32_t bar = full_leader + 8 * s;
-            if (sm.rank == 0) mbar_arrive_expect_tx(sm.full + 8 * s, 2 * cta_bytes);
+            if (sm.rank == 0) mbar_arrive_expect_tx(sm.full + 8 * s, stage_tx);
             const uint32_t b_dst = sm.b0 + s * GM_B_BYTES;
             const int kk = kb * GM_BK;
             for (uint32_t j = 0; j < nboxh; ++j)
@@ -271,29 +289,34 @@ __device__ __forceinline__ void gather_rows(const GemmArgs& p, const Tile& t, ui
     }
 }
 
-// Token gather (warps 10-13): each thread copies 8 16-byte chunks per stage; once
-// the copies of a stage have landed and are fenced to the async proxy, each warp
-// arrives once at CTA scope.
+// Token gather (warps 10-13): each thread copies 8 16-byte chunks per stage straight
+// into the 128-byte swizzled K-major layout, then hands the completion of its copies
+// to the stage's afull barrier (cp.async.mbarrier.arrive.noinc) and moves on without
+// waiting; gather_forwarder publishes the stage once all 128 threads' copies landed.
 __device__ void producer_gather(const GemmArgs& p, const Smem& sm, int64_t n_work,
                                 volatile int* abort_flag) {
     const int pt = threadIdx.x - GM_WARP_GATHER * 32;   // 0..127
     const int lane = threadIdx.x & 31;
     const int c = pt & 7, rb = pt >> 3;                  // 16-byte chunk, first row
-    // leader: its own full barrier; peer: its afull barrier (forwarded by gather_forwarder)
-    const uint32_t arrive_bar = sm.rank == 0 ? sm.full : sm.afull;
     int s = 0;
     uint32_t ph = 0;
-    int pend[A_LAG];
-    int npend = 0;
     bool ok = true;
     int64_t w = sm.pair;
     const __nv_bfloat16* src[8];
-    if (w < n_work) gather_rows(p, decode_tile(p, w), sm.rank, rb, src);
+    Tile t{};
+    if (w < n_work) {
+        t = decode_tile(p, w);
+        gather_rows(p, t, sm.rank, rb, src);
+    }
     for (; w < n_work && ok; w += sm.npairs) {
         const int64_t wn = w + sm.npairs;
         const __nv_bfloat16* nsrc[8];
-        if (wn < n_work) gather_rows(p, decode_tile(p, wn), sm.rank, rb, nsrc);
-        for (int kb = 0; kb < p.num_kb; ++kb) {
+        Tile tn{};
+        if (wn < n_work) {
+            tn = decode_tile(p, wn);
+            gather_rows(p, tn, sm.rank, rb, nsrc);
+        }
+        for (int kb = t.kb0; kb < t.kb1; ++kb) {
             int good = 1;
             if (lane == 0) good = mbar_wait(sm.empty + 8 * s, ph ^ 1u, p.limit_ns, abort_flag);
             good = __shfl_sync(0xffffffffu, good, 0);
@@ -312,17 +335,7 @@ __device__ void producer_gather(const GemmArgs& p, const Smem& sm, int64_t n_wor
                 const bool v = col_ok && src[j] != nullptr;
                 cp_async16(dst, v ? (const void*)(src[j] + kk) : (const void*)p.A, v ? 16u : 0u);
             }
-            cp_async_commit();
-            if (npend == A_LAG) {
-                cp_async_wait<A_LAG>();
-                fence_proxy_async_smem();
-                __syncwarp();
-                if (lane == 0) mbar_arrive(arrive_bar + 8 * pend[0]);
-#pragma unroll
-                for (int q = 0; q + 1 < A_LAG; ++q) pend[q] = pend[q + 1];
-                --npend;
-            }
-            pend[npend++] = s;
+            cp_async_arrive_noinc(sm.afull + 8 * s);
             if (++s == GM_STAGES) {
                 s = 0;
                 ph ^= 1u;
@@ -332,31 +345,35 @@ __device__ void producer_gather(const GemmArgs& p, const Smem& sm, int64_t n_wor
 #pragma unroll
             for (int j = 0; j < 8; ++j) src[j] = nsrc[j];
         }
+        t = tn;
     }
-    cp_async_wait<0>();
-    fence_proxy_async_smem();
-    __syncwarp();
-    if (lane == 0)
-        for (int q = 0; q < npend; ++q) mbar_arrive(arrive_bar + 8 * pend[q]);
+    cp_async_wait_all();
 }
 
-// Peer CTA, warp 8, lane 0 (idle otherwise): once the peer's four gather warps have
-// arrived on its local afull barrier for a stage, forward one cluster-scope arrival
-// to the leader's full barrier.  A release at cluster scope costs the issuing thread
-// a wait for its outstanding memory operations; this thread has none, the gather
-// threads (with copies in flight) only release at CTA scope.
+// Warp GM_WARP_FWD, lane 0, in both CTAs: once all of this CTA's gather threads'
+// copies of a stage have landed (its afull barrier), make them visible to the async
+// proxy that tcgen05.mma reads shared memory through, and publish the stage on the
+// leader's full barrier: a local arrival in the leader; from the peer, a 16-byte
+// async-proxy copy into the leader that completes 16 transaction bytes on that
+// barrier (the leader's expect_tx counts them).  Being ordered after the proxy
+// fence, the copy's completion implies the gathered rows are visible to the MMA,
+// without the cost of a cluster-scope release by this thread.
 __device__ void gather_forwarder(const GemmArgs& p, const Smem& sm, int64_t n_work,
                                  volatile int* abort_flag) {
     const uint32_t full_leader = peer_addr(sm.full, 0);
+    const uint32_t sink_leader = peer_addr(sm.sink, 0);
     int s = 0;
     uint32_t ph = 0;
     for (int64_t w = sm.pair; w < n_work; w += sm.npairs) {
-        for (int kb = 0; kb < p.num_kb; ++kb) {
+        const Tile t = decode_tile(p, w);
+        for (int kb = t.kb0; kb < t.kb1; ++kb) {
             if (!mbar_wait(sm.afull + 8 * s, ph, p.limit_ns, abort_flag)) {
                 set_abort(abort_flag, p.status, SITE_GEMM_WAIT_FULL, (int)sm.pair, -1 - kb);
                 return;
             }
-            mbar_arrive_remote(full_leader + 8 * s);
+            fence_proxy_async_smem();
+            if (sm.rank == 0) mbar_arrive(sm.full + 8 * s);
+            else bulk_signal_remote(sink_leader, sm.sink, full_leader + 8 * s);
             if (++s == GM_STAGES) {
                 s = 0;
                 ph ^= 1u;
@@ -384,8 +401,9 @@ __device__ void mma_issuer(const GemmArgs& p, const Smem& sm, uint32_t tmem, int
         }
         tc_fence_after();
         const uint32_t d_tmem = tmem + (uint32_t)acc * GM_MAXBN;
+        const Tile t = decode_tile(p, w);
         bool ok = true;
-        for (int kb = 0; kb < p.num_kb; ++kb) {
+        for (int kb = t.kb0; kb < t.kb1; ++kb) {
             if (!mbar_wait(sm.full + 8 * s, ph, p.limit_ns, abort_flag)) {
                 set_abort(abort_flag, p.status, SITE_GEMM_WAIT_FULL, (int)sm.pair, kb);
                 ok = false;
@@ -398,7 +416,7 @@ __device__ void mma_issuer(const GemmArgs& p, const Smem& sm, uint32_t tmem, int
             for (int kk = 0; kk < GM_BK / 16; ++kk) {
                 const uint64_t ad = smem_desc_sw128(a_addr + kk * 32, 16, 1024);
                 const uint64_t bd = smem_desc_sw128(b_addr + kk * 2048, 8192, 1024);
-                tc_mma_bf16_pair(d_tmem, ad, bd, idesc, (kb | kk) != 0 ? 1u : 0u);
+                tc_mma_bf16_pair(d_tmem, ad, bd, idesc, (kb != t.kb0 || kk != 0) ? 1u : 0u);
             }
             issued = true;
             tc_commit_pair(sm.empty + 8 * s);
@@ -512,7 +530,8 @@ __device__ void epilogue(const GemmArgs& p, const Smem& sm, uint32_t tmem, int64
                 const bool rok = __shfl_sync(0xffffffffu, ok_row ? 1 : 0, rr) != 0;
                 const float4 f = *reinterpret_cast<const float4*>(stg + rr * STG_LD + c4);
                 if (!(rok && col_ok)) continue;
-                float4* dst = reinterpret_cast<float4*>(p.yacc + rtok * p.ldy + n + c4);
+                float4* dst = reinterpret_cast<float4*>(p.yacc + t.ks * p.y_split_stride +
+                                                        rtok * p.ldy + n + c4);
                 const float4 val = make_float4(rsc * f.x, rsc * f.y, rsc * f.z, rsc * f.w);
                 if (p.epi == EPI_ADD_F32) atomicAdd(dst, val);
                 else *dst = val;
@@ -532,6 +551,7 @@ __global__ void __launch_bounds__(GM_THREADS, 1) grouped_gemm_kernel(const __gri
     uint64_t* bars = reinterpret_cast<uint64_t*>(sOut + GM_EPI_WARPS * 32 * STG_LD);
     uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 3 * GM_STAGES + 5);
     volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+    uint8_t* sink = reinterpret_cast<uint8_t*>(bars) + 256;   // 16-byte aligned, after the barriers
 
     Smem sm;
     sm.a0 = smem_u32(sA);
@@ -542,6 +562,7 @@ __global__ void __launch_bounds__(GM_THREADS, 1) grouped_gemm_kernel(const __gri
     sm.tfull = sm.afull + 8 * GM_STAGES;
     sm.tempty = sm.tfull + 16;
     sm.drain = sm.tempty + 16;
+    sm.sink = smem_u32(sink);
     sm.stage_out = sOut;
     sm.rank = cluster_rank();
     sm.pair = blockIdx.x >> 1;
@@ -551,10 +572,11 @@ __global__ void __launch_bounds__(GM_THREADS, 1) grouped_gemm_kernel(const __gri
     const bool gather = p.a_rows != nullptr;
     if (threadIdx.x == 0) {
         for (int s = 0; s < GM_STAGES; ++s) {
-            // leader's expect_tx arrival (+ its 4 gather warps and the peer's forwarder)
-            mbar_init(sm.full + 8 * s, 1 + (gather ? 4 + 1 : 0));
+            // leader's expect_tx arrival (+ the leader's forwarder; the peer's signals
+            // are transaction bytes)
+            mbar_init(sm.full + 8 * s, 1 + (gather ? 1 : 0));
             mbar_init(sm.empty + 8 * s, 1);         // multicast tcgen05.commit
-            mbar_init(sm.afull + 8 * s, 4);         // this CTA's gather warps
+            mbar_init(sm.afull + 8 * s, 128);       // this CTA's gather threads (async arrivals)
         }
         for (int a = 0; a < 2; ++a) {
             mbar_init(sm.tfull + 8 * a, 1);         // multicast tcgen05.commit
@@ -583,17 +605,16 @@ __global__ void __launch_bounds__(GM_THREADS, 1) grouped_gemm_kernel(const __gri
     } else {
         n_mtiles = (p.m_total + GM_BM - 1) / GM_BM;
     }
-    const int64_t n_work = n_mtiles * p.n_ntiles;
+    const int64_t n_work = n_mtiles * p.n_ntiles * p.ksplit;
 
     if (warp < GM_EPI_WARPS) {
         epilogue(p, sm, tmem, n_work, abort_flag);
     } else if (warp == GM_WARP_MMA) {
-        if ((threadIdx.x & 31) == 0) {
-            if (sm.rank == 0) mma_issuer(p, sm, tmem, n_work, abort_flag);
-            else if (gather) gather_forwarder(p, sm, n_work, abort_flag);
-        }
+        if ((threadIdx.x & 31) == 0 && sm.rank == 0) mma_issuer(p, sm, tmem, n_work, abort_flag);
     } else if (warp == GM_WARP_LOAD) {
         if ((threadIdx.x & 31) == 0) producer_tma(p, sm, n_work, abort_flag);
+    } else if (warp == GM_WARP_FWD) {
+        if ((threadIdx.x & 31) == 0 && gather) gather_forwarder(p, sm, n_work, abort_flag);
     } else if (gather) {
         producer_gather(p, sm, n_work, abort_flag);
     }

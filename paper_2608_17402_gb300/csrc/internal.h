@@ -28,18 +28,36 @@ inline int route_epad(int E) { return (E + 15) / 16 * 16; }
 inline int route_dpad(int d) { return (d + 63) / 64 * 64; }
 
 // W_r fp32 [d, E] -> three bf16 pieces [3][d_pad][E_pad] with W_r = hi + mid + lo
-// exactly (zero in the padding rows and columns), plus |W_r[:, e]| (wpart:
-// route_split_parts(d) x E_pad floats of scratch).
+// exactly (zero in the padding rows and columns), the transposed fp32 copy
+// wrt [E][d_pad] (zero rows past d), and |W_r[:, e]| (wpart: route_split_parts(d) x
+// E_pad floats of scratch).
 int route_split_parts(int d);
-cudaError_t launch_route_split(const float* Wr, int d, int E, __nv_bfloat16* Wsplit, float* wpart,
-                               float* wnorm, cudaStream_t s);
+cudaError_t launch_route_split(const float* Wr, int d, int E, __nv_bfloat16* Wsplit, float* wrt,
+                               float* wpart, float* wnorm, cudaStream_t s);
+
+// Splits of K for the router GEMM: enough CTA-pair work items for about
+// ROUTE_SPLIT_TARGET items, at most ROUTE_MAX_KSPLIT, at least three K blocks each.
+// Depends on the sizes only (the workspace size uses it).
+constexpr int ROUTE_SPLIT_TARGET = 152;
+constexpr int ROUTE_MAX_KSPLIT = 16;
+int route_ksplit(int64_t T, int d, int E);
+// Rows of partial-logit storage: an upper bound of route_ksplit(T) * T that is
+// monotone in T (ROUTE_MAX_KSPLIT T, and (ROUTE_SPLIT_TARGET + m-tiles x n-tiles) x 256).
+int64_t route_logits_rows(int64_t T, int d, int E);
+
+// out = the sum over the nparts partial logit arrays (n floats each, part_stride apart).
+cudaError_t launch_route_sum_parts(const float* logits, int64_t part_stride, int nparts, int64_t n,
+                                   float* out, cudaStream_t s);
+
 // Keys, warp top-k with a certificate, gates; uncertified tokens are re-decided
-// with exact (fp64) logits of the experts near their boundary.
-cudaError_t launch_route_select(const __nv_bfloat16* x, const float* Wr, const float* b,
-                                const float* logits, int ld_logits, const float* wnorm, int T,
-                                int d, int E, int k, int32_t* idx, float* gate,
-                                int32_t* fb_tokens, float* xnorm, DevStatus* st, int num_sms,
-                                cudaStream_t s);
+// with exact (fp64) logits of the experts near their boundary.  logits: nparts
+// partial arrays [T][ld] (part_stride floats apart); part 0 is overwritten with the
+// sum for uncertified tokens.
+cudaError_t launch_route_select(const __nv_bfloat16* x, const float* wrt, const float* b,
+                                float* logits, int ld, int nparts, int64_t part_stride,
+                                const float* wnorm, int T, int d, int E, int k, int32_t* idx,
+                                float* gate, int32_t* fb_tokens, float* xnorm, DevStatus* st,
+                                int num_sms, cudaStream_t s);
 
 // ---------------------------------------------------------------- permute
 
@@ -71,7 +89,8 @@ constexpr int GM_EPI_WARPS = 8;   // two warps per TMEM lane quadrant, alternate
 constexpr int GM_WARP_MMA = GM_EPI_WARPS;        // TMEM allocation + tcgen05.mma issue
 constexpr int GM_WARP_LOAD = GM_EPI_WARPS + 1;   // TMA loads of B (and of contiguous A)
 constexpr int GM_WARP_GATHER = GM_EPI_WARPS + 2; // first of 4 token-gather warps
-constexpr int GM_THREADS = (GM_EPI_WARPS + 2 + 4) * 32;
+constexpr int GM_WARP_FWD = GM_EPI_WARPS + 6;    // publishes gathered stages
+constexpr int GM_THREADS = (GM_EPI_WARPS + 7) * 32;
 constexpr int GM_A_BYTES = GM_HALF * GM_BK * 2;           // one CTA's A rows per stage
 constexpr int GM_B_BYTES = GM_BK * (GM_MAXBN / 2) * 2;    // one CTA's half of B per stage
 constexpr int GM_STG_LD = 20;                   // floats per row of a transpose buffer
@@ -102,6 +121,8 @@ struct GemmArgs {
     const int32_t* n_tiles_dev; // number of entries of `tiles`
     int64_t max_mtiles;         // host bound on *n_tiles_dev
     int G, K, N, BN, n_ntiles, num_kb, nbox;
+    int ksplit;                 // K is split into this many parts (work items), >= 1
+    int64_t y_split_stride;     // fp32 outputs: split ks writes yacc + ks * y_split_stride
     int epi;
     __nv_bfloat16* out;         // EPI_*_BF16
     int64_t ldo;

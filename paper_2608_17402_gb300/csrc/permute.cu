@@ -2,9 +2,13 @@
 // phase 1: Sort by expert id, index = pos // K, BinCount, CumSum), sm_103a.
 //
 // A stable counting sort over chunks of flat slots (about two chunks per SM):
-//   perm_hist_kernel    per-chunk histograms (16-byte vector loads of idx)
-//   perm_scan_kernel    counts, exclusive offsets, each chunk's first row per
-//                       expert, and the m-tile prefix used by the grouped GEMMs
+//   perm_hist_kernel    per-chunk histograms (16-byte vector loads of idx), stored
+//                       expert-major: hist[e][chunk]
+//   perm_chunk_scan_kernel  one warp per expert: exclusive scan over its chunks
+//                       (each chunk's first row inside the expert's segment) and
+//                       the expert's count
+//   perm_offsets_kernel exclusive offsets over experts and the m-tile table used
+//                       by the grouped GEMMs (one CTA)
 //   perm_scatter_kernel stages its chunk in shared memory (16-byte loads), ranks
 //                       every slot among the earlier slots of the same expert
 //                       (warp match + per-warp running counts), and writes perm,
@@ -49,7 +53,7 @@ __global__ void __launch_bounds__(PT) perm_hist_kernel(const int32_t* __restrict
         else report(st, MOEVIE_ERR_DEVICE, SITE_PERMUTE_ID, (int)i, e);
     }
     __syncthreads();
-    for (int e = threadIdx.x; e < E; e += PT) hist[(int64_t)blockIdx.x * E + e] = cnt[e];
+    for (int e = threadIdx.x; e < E; e += PT) hist[(int64_t)e * gridDim.x + blockIdx.x] = cnt[e];
 }
 
 // Exclusive scan of one int per thread over a 1024-thread block.
@@ -81,44 +85,49 @@ __device__ int block_exclusive_scan_1024(int v, int* total) {
     return r;
 }
 
-// One CTA of 1024 threads.  Warp w scans the chunk histograms of experts w, w+32,
-// ... (lanes over chunks) and rewrites hist[c][e] in place with the first row of
-// expert e inside chunk c, relative to the expert's segment; then one thread per
-// expert scans counts and tile counts across experts; then warps write the m-tile
-// table (lanes over an expert's tiles).
-__global__ void __launch_bounds__(1024) perm_scan_kernel(int32_t* __restrict__ hist, int nchunks,
-                                                         int E, int bm,
-                                                         int32_t* __restrict__ counts,
-                                                         int32_t* __restrict__ offsets,
-                                                         int4* __restrict__ tiles,
-                                                         int32_t* __restrict__ n_tiles) {
+// One warp per expert: hist[e][0 .. nchunks) becomes its exclusive prefix (the first
+// row of expert e inside each chunk, relative to the expert's segment); counts[e] is
+// the total.  Coalesced: lanes over consecutive chunks.
+__global__ void __launch_bounds__(256) perm_chunk_scan_kernel(int32_t* __restrict__ hist,
+                                                              int nchunks, int E,
+                                                              int32_t* __restrict__ counts) {
+    const int lane = threadIdx.x & 31;
+    const int e = (int)(((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5);
+    if (e >= E) return;
+    int32_t* h = hist + (int64_t)e * nchunks;
+    int running = 0;
+    for (int c0 = 0; c0 < nchunks; c0 += 32) {
+        const int c = c0 + lane;
+        const int v = c < nchunks ? h[c] : 0;
+        int inc = v;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const int u = __shfl_up_sync(0xffffffffu, inc, o);
+            if (lane >= o) inc += u;
+        }
+        if (c < nchunks) h[c] = running + inc - v;
+        running += __shfl_sync(0xffffffffu, inc, 31);
+    }
+    if (lane == 0) counts[e] = running;
+}
+
+// One CTA of 1024 threads (E <= 1024): exclusive offsets over experts, the number
+// of bm-row m-tiles, and the m-tile table (warps over experts, lanes over tiles).
+__global__ void __launch_bounds__(1024) perm_offsets_kernel(const int32_t* __restrict__ counts,
+                                                            int E, int bm,
+                                                            int32_t* __restrict__ offsets,
+                                                            int4* __restrict__ tiles,
+                                                            int32_t* __restrict__ n_tiles) {
     __shared__ int s_total, s_tiles;
     __shared__ int s_cnt[1024], s_off[1024], s_toff[1024];
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-    for (int e = warp; e < E; e += 32) {
-        int running = 0;
-        for (int c0 = 0; c0 < nchunks; c0 += 32) {
-            const int c = c0 + lane;
-            const int h = c < nchunks ? hist[(int64_t)c * E + e] : 0;
-            int inc = h;
-#pragma unroll
-            for (int o = 1; o < 32; o <<= 1) {
-                const int u = __shfl_up_sync(0xffffffffu, inc, o);
-                if (lane >= o) inc += u;
-            }
-            if (c < nchunks) hist[(int64_t)c * E + e] = running + inc - h;
-            running += __shfl_sync(0xffffffffu, inc, 31);
-        }
-        if (lane == 0) s_cnt[e] = running;
-    }
-    __syncthreads();
     const int e = threadIdx.x;
-    const int cnt = e < E ? s_cnt[e] : 0;
+    const int cnt = e < E ? counts[e] : 0;
     const int off = block_exclusive_scan_1024(cnt, &s_total);
     const int toff = block_exclusive_scan_1024((cnt + bm - 1) / bm, &s_tiles);
     if (e < E) {
-        if (counts) counts[e] = cnt;
         offsets[e] = off;
+        s_cnt[e] = cnt;
         s_off[e] = off;
         s_toff[e] = toff;
     }
@@ -169,7 +178,7 @@ __global__ void __launch_bounds__(PT) perm_scatter_kernel(
     }
     __syncthreads();
     for (int e = tid; e < E; e += PT) {                  // pass 2: first row per (warp, e)
-        int run = offsets[e] + base[(int64_t)blockIdx.x * E + e];
+        int run = offsets[e] + base[(int64_t)e * gridDim.x + blockIdx.x];
         for (int w = 0; w < PW; ++w) {
             const int c = wc[w * E + e];
             wc[w * E + e] = run;
@@ -259,7 +268,9 @@ cudaError_t launch_permute(const int32_t* idx, int64_t n_slots, int k, int E, in
     perm_hist_kernel<<<nchunks, PT, (size_t)E * 4, s>>>(idx, n_slots, E, chunk, hist, st);
     cudaError_t err = cudaGetLastError();
     if (err != cudaSuccess) return err;
-    perm_scan_kernel<<<1, 1024, 0, s>>>(hist, nchunks, E, bm, counts, offsets, tiles, n_tiles);
+    perm_chunk_scan_kernel<<<(E + 7) / 8, 256, 0, s>>>(hist, nchunks, E, counts);
+    if ((err = cudaGetLastError()) != cudaSuccess) return err;
+    perm_offsets_kernel<<<1, 1024, 0, s>>>(counts, E, bm, offsets, tiles, n_tiles);
     if ((err = cudaGetLastError()) != cudaSuccess) return err;
     const size_t smem = (size_t)(chunk + PW * E) * 4;
     static bool attr_set[64] = {};
@@ -273,7 +284,7 @@ cudaError_t launch_permute(const int32_t* idx, int64_t n_slots, int k, int E, in
     }
     perm_scatter_kernel<<<nchunks, PT, smem, s>>>(idx, n_slots, k, E, chunk, hist, offsets,
                                                   gate_flat, perm, inv, row_tok, row_gate);
-    count_launches(3);
+    count_launches(4);
     return cudaGetLastError();
 }
 

@@ -5,23 +5,27 @@
 // the GEMM accumulates x . [hi; mid; lo] over K = 3 d_pad in fp32 (each piece padded
 // to a multiple of 64 rows with zeros).  Every product of a
 // bf16 x and a bf16 piece is exact in fp32, so the only error is the fp32
-// accumulation.  This file holds the steps around that GEMM:
+// accumulation.  When there are few tokens, K is split over several CTA pairs
+// (route_ksplit) and each split writes its own fp32 partial logits; they are summed
+// in a fixed order.  This file holds the steps around that GEMM:
 //
-//  1. route_split_kernel / route_wnorm_kernel: the three pieces and |W_r[:, e]|.
-//  2. route_topk_kernel: one warp per token; keys sigmoid(s) + b, k rounds of warp
-//     arg-max (ties to the lower id), and a certificate.  Every expert's key lies in
+//  1. route_split_kernel / route_wnorm_kernel: the three pieces, an fp32 copy of
+//     W_r transposed to [E][d_pad] (read by the exact re-decision), and |W_r[:, e]|.
+//  2. route_topk_kernel: one warp per token; the partial logits summed, keys
+//     sigmoid(s) + b, k rounds of warp arg-max (ties to the lower id), and a
+//     certificate.  Every expert's key lies in
 //     [key_e - tau_e, key_e + tau_e]; tau_e is the logit error bound
 //     (ROUTE_TAU_C 2^-24 |x_t| |W_r[:, e]|) times the largest sigmoid slope inside
 //     the logit interval, plus fp32 evaluation slack.  The selection is certain when
 //     the lowest selected lower end is above the highest unselected upper end (tried
 //     first with the slope bound 1/4, then with the exact slope).  Certified tokens
 //     write ascending ids and gates sigmoid(s) / sum (the bias only selects).
-//  3. route_fallback_kernel: one warp per uncertified token.  An expert is surely in
+//  3. route_fallback_kernel: one CTA per uncertified token.  An expert is surely in
 //     when its lower end is above the k-th largest upper end of the others, surely
 //     out when its upper end is below the k-th largest lower end; the rest get exact
 //     logits (fp64: each product of a bf16 and an fp32 value is exact in double, and
-//     the sum of d terms has relative error below d 2^-53), and the remaining places
-//     are filled from them, ties to the lower id.
+//     the sum of d terms has relative error below d 2^-53; one warp per candidate),
+//     and the remaining places are filled from them, ties to the lower id.
 #include <math.h>
 
 #include "internal.h"
@@ -30,23 +34,28 @@ namespace mv {
 
 namespace {
 
-constexpr int SPLIT_ROWS = 256;   // W_r rows per CTA of the split kernel
+constexpr int SPLIT_TILE = 32;    // W_r rows (and experts) per CTA of the split kernel
 
-// CTA (bx, by): experts 32 bx .. +31, rows SPLIT_ROWS by .. +SPLIT_ROWS-1; 32 x 8 threads.
+// CTA (bx, by): experts 32 bx .. +31 and rows 32 by .. +31 of W_r (rows past d are
+// zero); 32 x 8 threads.  Writes the three bf16 pieces, the transposed fp32 copy and
+// the CTA's partial sums of w^2 per expert.
 __global__ void __launch_bounds__(256) route_split_kernel(const float* __restrict__ Wr, int d,
                                                           int dp, int E, int Ep,
                                                           __nv_bfloat16* __restrict__ Wsplit,
+                                                          float* __restrict__ wrt,
                                                           float* __restrict__ wpart) {
+    __shared__ float tile[SPLIT_TILE][SPLIT_TILE + 1];
     __shared__ float red[8][32];
     const int tx = threadIdx.x & 31, ty = threadIdx.x >> 5;
-    const int e = blockIdx.x * 32 + tx;
-    const int i0 = blockIdx.y * SPLIT_ROWS;
-    const int i1 = min(dp, i0 + SPLIT_ROWS);
+    const int e = blockIdx.x * SPLIT_TILE + tx;
+    const int i0 = blockIdx.y * SPLIT_TILE;
+    const size_t piece = (size_t)dp * Ep;
     float sq = 0.f;
-    if (e < Ep) {
-        const size_t piece = (size_t)dp * Ep;
-        for (int i = i0 + ty; i < i1; i += 8) {
-            const float w = (e < E && i < d) ? Wr[(int64_t)i * E + e] : 0.f;
+#pragma unroll
+    for (int r = ty; r < SPLIT_TILE; r += 8) {
+        const int i = i0 + r;
+        const float w = (e < E && i < d) ? Wr[(int64_t)i * E + e] : 0.f;
+        if (e < Ep) {
             const __nv_bfloat16 hi = __float2bfloat16_rn(w);
             const float r1 = w - __bfloat162float(hi);          // exact
             const __nv_bfloat16 mid = __float2bfloat16_rn(r1);
@@ -55,8 +64,9 @@ __global__ void __launch_bounds__(256) route_split_kernel(const float* __restric
             Wsplit[o] = hi;
             Wsplit[piece + o] = mid;
             Wsplit[2 * piece + o] = lo;
-            sq = fmaf(w, w, sq);
         }
+        tile[r][tx] = w;
+        sq = fmaf(w, w, sq);
     }
     red[ty][tx] = sq;
     __syncthreads();
@@ -65,16 +75,26 @@ __global__ void __launch_bounds__(256) route_split_kernel(const float* __restric
         for (int q = 0; q < 8; ++q) v += red[q][tx];
         wpart[(int64_t)blockIdx.y * Ep + e] = v;
     }
+#pragma unroll
+    for (int r = ty; r < SPLIT_TILE; r += 8) {
+        const int ee = blockIdx.x * SPLIT_TILE + r;
+        if (ee < E) wrt[(int64_t)ee * dp + i0 + tx] = tile[tx][r];
+    }
 }
 
-// |W_r[:, e]| from the per-CTA partial sums, in a fixed order.
-__global__ void route_wnorm_kernel(const float* __restrict__ wpart, int nparts, int E, int Ep,
-                                   float* __restrict__ wnorm) {
-    const int e = blockIdx.x * blockDim.x + threadIdx.x;
+// |W_r[:, e]| from the per-CTA partial sums: one warp per expert, lanes over parts,
+// then a fixed shuffle tree (deterministic).
+__global__ void __launch_bounds__(256) route_wnorm_kernel(const float* __restrict__ wpart,
+                                                          int nparts, int E, int Ep,
+                                                          float* __restrict__ wnorm) {
+    const int lane = threadIdx.x & 31;
+    const int e = (int)(((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5);
     if (e >= E) return;
     float v = 0.f;
-    for (int p = 0; p < nparts; ++p) v += wpart[(int64_t)p * Ep + e];
-    wnorm[e] = sqrtf(v);
+    for (int p = lane; p < nparts; p += 32) v += wpart[(int64_t)p * Ep + e];
+#pragma unroll
+    for (int o = 16; o; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+    if (lane == 0) wnorm[e] = sqrtf(v);
 }
 
 // Fast sigmoid: __expf (ex2.approx) and __fdividef.  For the keys compared below
@@ -105,71 +125,121 @@ __device__ __forceinline__ float warp_sum(float v) {
     return v;
 }
 
-// |x_t| by one warp (16-byte loads; d % 8 == 0).
-__device__ __forceinline__ float row_norm(const __nv_bfloat16* xt, int d, int lane) {
-    float acc = 0.f;
-    for (int c = lane; c < d / 8; c += 32) {
-        float v[8];
-        unpack_bf16x8(*reinterpret_cast<const uint4*>(xt + 8 * c), v);
+__device__ __forceinline__ float sq_bf16x8(const uint4& q) {
+    float v[8];
+    unpack_bf16x8(q, v);
+    float a = 0.f;
 #pragma unroll
-        for (int q = 0; q < 8; ++q) acc = fmaf(v[q], v[q], acc);
+    for (int i = 0; i < 8; ++i) a = fmaf(v[i], v[i], a);
+    return a;
+}
+
+// |x_t| by one warp (16-byte loads, up to eight in flight per lane; d % 8 == 0).
+__device__ __forceinline__ float row_norm(const __nv_bfloat16* xt, int d, int lane) {
+    const uint4* v = reinterpret_cast<const uint4*>(xt);
+    const int nc = d / 8;
+    float acc = 0.f;
+    int c = lane;
+    for (; c + 224 < nc; c += 256) {
+        uint4 q[8];
+#pragma unroll
+        for (int u = 0; u < 8; ++u) q[u] = v[c + 32 * u];
+#pragma unroll
+        for (int u = 0; u < 8; ++u) acc += sq_bf16x8(q[u]);
     }
+    for (; c + 96 < nc; c += 128) {
+        const uint4 q0 = v[c], q1 = v[c + 32], q2 = v[c + 64], q3 = v[c + 96];
+        acc += (sq_bf16x8(q0) + sq_bf16x8(q1)) + (sq_bf16x8(q2) + sq_bf16x8(q3));
+    }
+    for (; c < nc; c += 32) acc += sq_bf16x8(v[c]);
     return sqrtf(warp_sum(acc));
 }
 
-// Warp arg-max of (value, id): largest value, ties to the lower id.
-__device__ __forceinline__ void warp_argmax(float& v, int& id) {
+// Order-preserving code of (key, id): larger key first, then the lower id.
+__device__ __forceinline__ uint64_t key_code(float key, int e) {
+    uint32_t u = __float_as_uint(key);
+    u ^= (u & 0x80000000u) ? 0xffffffffu : 0x80000000u;
+    return ((uint64_t)u << 32) | (uint32_t)(0xffffffffu - (uint32_t)e);
+}
+
+__device__ __forceinline__ uint64_t warp_max_u64(uint64_t v) {
 #pragma unroll
     for (int o = 16; o; o >>= 1) {
-        const float ov = __shfl_xor_sync(0xffffffffu, v, o);
-        const int oi = __shfl_xor_sync(0xffffffffu, id, o);
-        if (ov > v || (ov == v && oi < id)) {
-            v = ov;
-            id = oi;
-        }
+        const uint64_t u = __shfl_xor_sync(0xffffffffu, v, o);
+        v = u > v ? u : v;
     }
+    return v;
+}
+
+// Order-preserving code of a float (larger float, larger code; no NaNs here).
+__device__ __forceinline__ uint32_t ord_f32(float f) {
+    const uint32_t u = __float_as_uint(f);
+    return u ^ ((u & 0x80000000u) ? 0xffffffffu : 0x80000000u);
 }
 
 // One warp per token.  NPL = experts per lane (expert e sits in lane e % 32, slot e / 32).
+// s holds nparts partial logit arrays, part p at s + p * part_stride.  Each of the k
+// selection rounds takes the warp maximum of the keys' order codes (redux.sync) and
+// then the lowest id holding it (ballots in slot order), so ties go to the lower id.
 template <int NPL>
 __global__ void __launch_bounds__(256) route_topk_kernel(
-    const __nv_bfloat16* __restrict__ x, const float* __restrict__ s, int ld,
-    const float* __restrict__ b, const float* __restrict__ wnorm, int T, int d, int E, int k,
-    int32_t* __restrict__ idx, float* __restrict__ gate, float* __restrict__ xnorm,
-    int32_t* __restrict__ fb_tokens, DevStatus* st) {
+    const __nv_bfloat16* __restrict__ x, float* __restrict__ s, int ld, int nparts,
+    int64_t part_stride, const float* __restrict__ b, const float* __restrict__ wnorm, int T,
+    int d, int E, int k, int32_t* __restrict__ idx, float* __restrict__ gate,
+    float* __restrict__ xnorm, int32_t* __restrict__ fb_tokens, DevStatus* st) {
     const int lane = threadIdx.x & 31;
     const int t = (int)(((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5);
     if (t >= T) return;
+    float* srow = s + (int64_t)t * ld;
+    float sv[NPL];
+#pragma unroll
+    for (int i = 0; i < NPL; ++i) {
+        const int e = lane + 32 * i;
+        sv[i] = e < E ? srow[e] : 0.f;
+    }
+    for (int q = 1; q < nparts; ++q) {
+#pragma unroll
+        for (int i = 0; i < NPL; ++i) {
+            const int e = lane + 32 * i;
+            if (e < E) sv[i] += srow[q * part_stride + e];
+        }
+    }
     const float xn = row_norm(x + (int64_t)t * d, d, lane);
     if (lane == 0) xnorm[t] = xn;
-    float sv[NPL], key[NPL], ts[NPL];
+    float sg[NPL], key[NPL], ts[NPL];
+    uint32_t code[NPL];
 #pragma unroll
     for (int i = 0; i < NPL; ++i) {
         const int e = lane + 32 * i;
         if (e < E) {
-            sv[i] = s[(int64_t)t * ld + e];
-            key[i] = sigmoid_fast(sv[i]) + b[e];
+            sg[i] = sigmoid_fast(sv[i]);
+            key[i] = sg[i] + b[e];
             ts[i] = logit_tau(xn, wnorm[e]);
+            code[i] = ord_f32(key[i]);
         } else {
-            sv[i] = 0.f;
+            sg[i] = 0.f;
             key[i] = -INFINITY;
             ts[i] = 0.f;
+            code[i] = 0;
         }
     }
     uint32_t taken = 0;
     for (int j = 0; j < k; ++j) {
-        float bv = -INFINITY;
-        int bi = 0x7fffffff;
+        uint32_t best = 0;
 #pragma unroll
         for (int i = 0; i < NPL; ++i) {
-            const int e = lane + 32 * i;
-            if (e < E && !((taken >> i) & 1u) && (key[i] > bv || bi == 0x7fffffff)) {
-                bv = key[i];
-                bi = e;
+            const uint32_t c = ((taken >> i) & 1u) ? 0u : code[i];
+            best = c > best ? c : best;
+        }
+        best = __reduce_max_sync(0xffffffffu, best);
+#pragma unroll
+        for (int i = 0; i < NPL; ++i) {
+            const uint32_t m = __ballot_sync(0xffffffffu, !((taken >> i) & 1u) && code[i] == best);
+            if (m) {
+                if (lane == __ffs(m) - 1) taken |= 1u << i;
+                break;
             }
         }
-        warp_argmax(bv, bi);
-        if ((bi & 31) == lane) taken |= 1u << (bi >> 5);
     }
     bool certain = k >= E;
     for (int pass = 0; pass < 2 && !certain; ++pass) {
@@ -183,14 +253,17 @@ __global__ void __launch_bounds__(256) route_topk_kernel(
             if ((taken >> i) & 1u) lo_in = fminf(lo_in, key[i] - tk);
             else hi_out = fmaxf(hi_out, key[i] + tk);
         }
-#pragma unroll
-        for (int o = 16; o; o >>= 1) {
-            lo_in = fminf(lo_in, __shfl_xor_sync(0xffffffffu, lo_in, o));
-            hi_out = fmaxf(hi_out, __shfl_xor_sync(0xffffffffu, hi_out, o));
-        }
-        certain = lo_in > hi_out;
+        certain = __reduce_min_sync(0xffffffffu, ord_f32(lo_in)) >
+                  __reduce_max_sync(0xffffffffu, ord_f32(hi_out));
     }
     if (!certain) {
+        if (nparts > 1) {   // the re-decision reads the summed logits from part 0
+#pragma unroll
+            for (int i = 0; i < NPL; ++i) {
+                const int e = lane + 32 * i;
+                if (e < E) srow[e] = sv[i];
+            }
+        }
         if (lane == 0) {
             const int p = atomicAdd(&st->fb_count, 1);
             fb_tokens[p] = t;
@@ -198,12 +271,8 @@ __global__ void __launch_bounds__(256) route_topk_kernel(
         return;
     }
     float ssum = 0.f;
-    float sg[NPL];
 #pragma unroll
-    for (int i = 0; i < NPL; ++i) {
-        sg[i] = ((taken >> i) & 1u) ? sigmoid_fast(sv[i]) : 0.f;
-        ssum += sg[i];
-    }
+    for (int i = 0; i < NPL; ++i) ssum += ((taken >> i) & 1u) ? sg[i] : 0.f;
     ssum = warp_sum(ssum);
     const uint32_t lt = (1u << lane) - 1u;
     int base = 0;
@@ -219,211 +288,276 @@ __global__ void __launch_bounds__(256) route_topk_kernel(
     }
 }
 
-constexpr int FB_BATCH = 8;   // candidates whose exact logits are summed together
-
 // k-th and (k+1)-th largest of v over the warp (k rounds of arg-max; k <= E).
 template <int NPL>
 __device__ __forceinline__ void warp_kth_values(const float (&v)[NPL], int E, int k, int lane,
                                                 float& kth, float& kth1) {
+    uint64_t code[NPL];
+#pragma unroll
+    for (int i = 0; i < NPL; ++i) {
+        const int e = lane + 32 * i;
+        code[i] = e < E ? key_code(v[i], e) : 0ull;
+    }
     uint32_t used = 0;
     kth = -INFINITY;
     kth1 = -INFINITY;
     const int rounds = k < E ? k + 1 : k;
     for (int j = 0; j < rounds; ++j) {
-        float bv = -INFINITY;
-        int bi = 0x7fffffff;
+        uint64_t best = 0;
 #pragma unroll
         for (int i = 0; i < NPL; ++i) {
-            const int e = lane + 32 * i;
-            if (e < E && !((used >> i) & 1u) && (v[i] > bv || bi == 0x7fffffff)) {
-                bv = v[i];
-                bi = e;
-            }
+            const uint64_t c = ((used >> i) & 1u) ? 0ull : code[i];
+            best = c > best ? c : best;
         }
-        warp_argmax(bv, bi);
+        best = warp_max_u64(best);
+        const int bi = (int)(0xffffffffu - (uint32_t)best);
+        float bv = 0.f;
+#pragma unroll
+        for (int i = 0; i < NPL; ++i)
+            if (lane + 32 * i == bi) bv = v[i];
+        bv = __shfl_sync(0xffffffffu, bv, bi & 31);
         if ((bi & 31) == lane) used |= 1u << (bi >> 5);
         if (j == k - 1) kth = bv;
         if (j == k) kth1 = bv;
     }
 }
 
-// Exact re-decision of uncertified tokens, one warp per token.
+__device__ __forceinline__ double dot_bf16x8_f32x8(const uint4& xq, const float4& w0,
+                                                   const float4& w1) {
+    float xv[8];
+    unpack_bf16x8(xq, xv);
+    double a = (double)xv[0] * (double)w0.x;
+    a = fma((double)xv[1], (double)w0.y, a);
+    a = fma((double)xv[2], (double)w0.z, a);
+    a = fma((double)xv[3], (double)w0.w, a);
+    a = fma((double)xv[4], (double)w1.x, a);
+    a = fma((double)xv[5], (double)w1.y, a);
+    a = fma((double)xv[6], (double)w1.z, a);
+    a = fma((double)xv[7], (double)w1.w, a);
+    return a;
+}
+
+// Exact re-decision of uncertified tokens, one CTA (8 warps) per token.  Warp 0
+// bounds the keys and lists the candidates; every warp computes exact logits of its
+// candidates (lanes over d, reading the transposed fp32 copy of W_r); warp 0 fills
+// the remaining places from the exact keys and writes ids and gates.
 template <int NPL>
 __global__ void __launch_bounds__(256) route_fallback_kernel(
-    const __nv_bfloat16* __restrict__ x, const float* __restrict__ Wr,
+    const __nv_bfloat16* __restrict__ x, const float* __restrict__ wrt, int dp,
     const float* __restrict__ b, const float* __restrict__ s, int ld,
     const float* __restrict__ xnorm, const float* __restrict__ wnorm, int d, int E, int k,
     int32_t* __restrict__ idx, float* __restrict__ gate, const int32_t* __restrict__ fb_tokens,
     DevStatus* st) {
-    const int lane = threadIdx.x & 31;
-    const int64_t wid = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
-    const int64_t nwarps = ((int64_t)gridDim.x * blockDim.x) >> 5;
+    __shared__ int s_cand[32 * NPL];
+    __shared__ double s_key[32 * NPL];
+    __shared__ int s_ncand;
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const uint32_t lt = (1u << lane) - 1u;
     const int nfb = st->fb_count;
-    for (int64_t f = wid; f < nfb; f += nwarps) {
+    for (int f = blockIdx.x; f < nfb; f += gridDim.x) {
         const int t = fb_tokens[f];
-        const float xn = xnorm[t];
-        float sv[NPL], up[NPL], lo[NPL];
-#pragma unroll
-        for (int i = 0; i < NPL; ++i) {
-            const int e = lane + 32 * i;
-            if (e < E) {
-                sv[i] = s[(int64_t)t * ld + e];
-                const float key = sigmoid_fast(sv[i]) + b[e];
-                const float tk = key_tau_exact_slope(sv[i], logit_tau(xn, wnorm[e]));
-                up[i] = key + tk;
-                lo[i] = key - tk;
-            } else {
-                sv[i] = 0.f;
-                up[i] = lo[i] = -INFINITY;
-            }
-        }
-        // k-th / (k+1)-th largest upper ends and k-th largest lower end
-        float u_k, u_k1, l_k, l_k1;
-        warp_kth_values<NPL>(up, E, k, lane, u_k, u_k1);
-        warp_kth_values<NPL>(lo, E, k, lane, l_k, l_k1);
+        float sv[NPL];
         uint32_t sure_in = 0, cand = 0;
-#pragma unroll
-        for (int i = 0; i < NPL; ++i) {
-            const int e = lane + 32 * i;
-            if (e >= E) continue;
-            // k-th largest upper end among the others (u_k when e may sit at rank k: conservative)
-            const float thr = up[i] > u_k ? u_k1 : u_k;
-            if (k >= E || lo[i] > thr) sure_in |= 1u << i;
-            else if (!(up[i] < l_k)) cand |= 1u << i;
-        }
-        int n_in = 0, n_cand = 0;
-#pragma unroll
-        for (int i = 0; i < NPL; ++i) {
-            n_in += __popc(__ballot_sync(0xffffffffu, (sure_in >> i) & 1u));
-            n_cand += __popc(__ballot_sync(0xffffffffu, (cand >> i) & 1u));
-        }
-        const int need = k - n_in;
-        if (need < 0 || need > n_cand) {
-            if (lane == 0) report(st, MOEVIE_ERR_DEVICE, SITE_ROUTE_FALLBACK, t, need);
-            continue;
-        }
-        // exact keys of the candidates, FB_BATCH at a time, lanes over d
-        double exk[NPL];
-#pragma unroll
-        for (int i = 0; i < NPL; ++i) exk[i] = -INFINITY;
-        for (int done = 0; done < n_cand;) {
-            int ids[FB_BATCH];
-            int nb = 0, seen = 0;
-#pragma unroll
-            for (int i = 0; i < NPL; ++i) {
-                uint32_t m = __ballot_sync(0xffffffffu, (cand >> i) & 1u);
-                while (m && nb < FB_BATCH) {
-                    const int l = __ffs(m) - 1;
-                    m &= m - 1;
-                    if (seen++ >= done) ids[nb++] = l + 32 * i;
-                }
-            }
-#pragma unroll
-            for (int q = 0; q < FB_BATCH; ++q)
-                if (q >= nb) ids[q] = ids[0];
-            double acc[FB_BATCH];
-#pragma unroll
-            for (int q = 0; q < FB_BATCH; ++q) acc[q] = 0.0;
-            for (int j = lane; j < d; j += 32) {
-                const double xv = (double)__bfloat162float(x[(int64_t)t * d + j]);
-                const float* wrow = Wr + (int64_t)j * E;
-#pragma unroll
-                for (int q = 0; q < FB_BATCH; ++q) acc[q] += xv * (double)wrow[ids[q]];
-            }
-#pragma unroll
-            for (int q = 0; q < FB_BATCH; ++q) {
-                double v = acc[q];
-#pragma unroll
-                for (int o = 16; o; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
-                const int e = ids[q];
-                if (q < nb && (e & 31) == lane) {
-                    const double key = 1.0 / (1.0 + exp(-v)) + (double)b[e];
-#pragma unroll
-                    for (int i = 0; i < NPL; ++i)
-                        if (i == (e >> 5)) exk[i] = key;
-                }
-            }
-            done += nb;
-        }
-        // choose `need` candidates by exact key, ties to the lower id
-        uint32_t chosen = sure_in;
-        for (int r = 0; r < need; ++r) {
-            double bv = -INFINITY;
-            int bi = 0x7fffffff;
+        int need = 0;
+        if (warp == 0) {
+            const float xn = xnorm[t];
+            float up[NPL], lo[NPL];
 #pragma unroll
             for (int i = 0; i < NPL; ++i) {
                 const int e = lane + 32 * i;
-                if (((cand >> i) & 1u) && !((chosen >> i) & 1u) && (exk[i] > bv || bi == 0x7fffffff)) {
-                    bv = exk[i];
-                    bi = e;
+                if (e < E) {
+                    sv[i] = s[(int64_t)t * ld + e];
+                    const float key = sigmoid_fast(sv[i]) + b[e];
+                    const float tk = key_tau_exact_slope(sv[i], logit_tau(xn, wnorm[e]));
+                    up[i] = key + tk;
+                    lo[i] = key - tk;
+                } else {
+                    sv[i] = 0.f;
+                    up[i] = lo[i] = -INFINITY;
                 }
             }
+            // k-th / (k+1)-th largest upper ends and k-th largest lower end
+            float u_k, u_k1, l_k, l_k1;
+            warp_kth_values<NPL>(up, E, k, lane, u_k, u_k1);
+            warp_kth_values<NPL>(lo, E, k, lane, l_k, l_k1);
 #pragma unroll
-            for (int o = 16; o; o >>= 1) {
-                const double ov = __shfl_xor_sync(0xffffffffu, bv, o);
-                const int oi = __shfl_xor_sync(0xffffffffu, bi, o);
-                if (ov > bv || (ov == bv && oi < bi)) {
-                    bv = ov;
-                    bi = oi;
+            for (int i = 0; i < NPL; ++i) {
+                const int e = lane + 32 * i;
+                if (e >= E) continue;
+                // k-th largest upper end among the others (u_k when e may sit at rank k: conservative)
+                const float thr = up[i] > u_k ? u_k1 : u_k;
+                if (k >= E || lo[i] > thr) sure_in |= 1u << i;
+                else if (!(up[i] < l_k)) cand |= 1u << i;
+            }
+            int n_in = 0, n_cand = 0;
+#pragma unroll
+            for (int i = 0; i < NPL; ++i) {
+                n_in += __popc(__ballot_sync(0xffffffffu, (sure_in >> i) & 1u));
+                const uint32_t m = __ballot_sync(0xffffffffu, (cand >> i) & 1u);
+                if ((cand >> i) & 1u) s_cand[n_cand + __popc(m & lt)] = lane + 32 * i;
+                n_cand += __popc(m);
+            }
+            need = k - n_in;
+            const bool bad = need < 0 || need > n_cand;
+            if (lane == 0) {
+                if (bad) report(st, MOEVIE_ERR_DEVICE, SITE_ROUTE_FALLBACK, t, need);
+                s_ncand = bad ? -1 : n_cand;
+            }
+        }
+        __syncthreads();
+        const int nc = s_ncand;
+        const uint4* xr = reinterpret_cast<const uint4*>(x + (int64_t)t * d);
+        const int nchunk = d / 8;
+        for (int c = warp; c < nc; c += 8) {
+            const int e = s_cand[c];
+            const float4* wr = reinterpret_cast<const float4*>(wrt + (int64_t)e * dp);
+            double acc0 = 0.0, acc1 = 0.0;
+            int j = lane;
+            for (; j + 32 < nchunk; j += 64) {
+                const uint4 xa = xr[j], xb = xr[j + 32];
+                const float4 wa0 = wr[2 * j], wa1 = wr[2 * j + 1];
+                const float4 wb0 = wr[2 * (j + 32)], wb1 = wr[2 * (j + 32) + 1];
+                acc0 += dot_bf16x8_f32x8(xa, wa0, wa1);
+                acc1 += dot_bf16x8_f32x8(xb, wb0, wb1);
+            }
+            if (j < nchunk) acc0 += dot_bf16x8_f32x8(xr[j], wr[2 * j], wr[2 * j + 1]);
+            double v = acc0 + acc1;
+#pragma unroll
+            for (int o = 16; o; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+            if (lane == 0) s_key[c] = 1.0 / (1.0 + exp(-v)) + (double)b[e];
+        }
+        __syncthreads();
+        if (warp == 0 && nc >= 0) {
+            double exk[NPL];
+            int base = 0;
+#pragma unroll
+            for (int i = 0; i < NPL; ++i) {
+                const uint32_t m = __ballot_sync(0xffffffffu, (cand >> i) & 1u);
+                exk[i] = ((cand >> i) & 1u) ? s_key[base + __popc(m & lt)] : -INFINITY;
+                base += __popc(m);
+            }
+            // choose `need` candidates by exact key, ties to the lower id
+            uint32_t chosen = sure_in;
+            for (int r = 0; r < need; ++r) {
+                double bv = -INFINITY;
+                int bi = 0x7fffffff;
+#pragma unroll
+                for (int i = 0; i < NPL; ++i) {
+                    const int e = lane + 32 * i;
+                    if (((cand >> i) & 1u) && !((chosen >> i) & 1u) &&
+                        (exk[i] > bv || bi == 0x7fffffff)) {
+                        bv = exk[i];
+                        bi = e;
+                    }
                 }
-            }
-            if ((bi & 31) == lane) chosen |= 1u << (bi >> 5);
-        }
-        float sg[NPL];
-        float ssum = 0.f;
 #pragma unroll
-        for (int i = 0; i < NPL; ++i) {
-            sg[i] = ((chosen >> i) & 1u) ? sigmoid_fast(sv[i]) : 0.f;
-            ssum += sg[i];
-        }
-        ssum = warp_sum(ssum);
-        const uint32_t lt = (1u << lane) - 1u;
-        int base = 0;
-#pragma unroll
-        for (int i = 0; i < NPL; ++i) {
-            const uint32_t m = __ballot_sync(0xffffffffu, (chosen >> i) & 1u);
-            if ((chosen >> i) & 1u) {
-                const int pos = base + __popc(m & lt);
-                idx[(int64_t)t * k + pos] = lane + 32 * i;
-                gate[(int64_t)t * k + pos] = __fdividef(sg[i], ssum);
+                for (int o = 16; o; o >>= 1) {
+                    const double ov = __shfl_xor_sync(0xffffffffu, bv, o);
+                    const int oi = __shfl_xor_sync(0xffffffffu, bi, o);
+                    if (ov > bv || (ov == bv && oi < bi)) {
+                        bv = ov;
+                        bi = oi;
+                    }
+                }
+                if ((bi & 31) == lane) chosen |= 1u << (bi >> 5);
             }
-            base += __popc(m);
+            float sg[NPL];
+            float ssum = 0.f;
+#pragma unroll
+            for (int i = 0; i < NPL; ++i) {
+                sg[i] = ((chosen >> i) & 1u) ? sigmoid_fast(sv[i]) : 0.f;
+                ssum += sg[i];
+            }
+            ssum = warp_sum(ssum);
+            int pbase = 0;
+#pragma unroll
+            for (int i = 0; i < NPL; ++i) {
+                const uint32_t m = __ballot_sync(0xffffffffu, (chosen >> i) & 1u);
+                if ((chosen >> i) & 1u) {
+                    const int pos = pbase + __popc(m & lt);
+                    idx[(int64_t)t * k + pos] = lane + 32 * i;
+                    gate[(int64_t)t * k + pos] = __fdividef(sg[i], ssum);
+                }
+                pbase += __popc(m);
+            }
         }
+        __syncthreads();   // s_cand / s_key are reused by the next token
     }
 }
 
 __global__ void reset_fallback_count(DevStatus* st) { st->fb_count = 0; }
 
+// out[t, e] = sum of the nparts partial logits, in order (used for inspection).
+__global__ void route_sum_parts_kernel(const float* __restrict__ s, int64_t part_stride,
+                                       int nparts, int64_t n, float* __restrict__ out) {
+    const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    if (i >= n) return;
+    float v = s[i];
+    for (int q = 1; q < nparts; ++q) v += s[q * part_stride + i];
+    out[i] = v;
+}
+
 }  // namespace
 
-int route_split_parts(int d) { return (route_dpad(d) + SPLIT_ROWS - 1) / SPLIT_ROWS; }
+int route_split_parts(int d) { return route_dpad(d) / SPLIT_TILE; }
 
-cudaError_t launch_route_split(const float* Wr, int d, int E, __nv_bfloat16* Wsplit, float* wpart,
-                               float* wnorm, cudaStream_t s) {
+int route_ksplit(int64_t T, int d, int E) {
+    int BN = 0, n_ntiles = 0;
+    choose_bn(E, &BN, &n_ntiles);
+    const int64_t items = (T + GM_BM - 1) / GM_BM * n_ntiles;
+    const int nkb = 3 * route_dpad(d) / GM_BK;
+    int64_t p = items > 0 ? (ROUTE_SPLIT_TARGET + items - 1) / items : 1;
+    if (p > nkb / 3) p = nkb / 3;   // at least three K blocks per split
+    if (p > ROUTE_MAX_KSPLIT) p = ROUTE_MAX_KSPLIT;
+    return p < 1 ? 1 : (int)p;
+}
+
+int64_t route_logits_rows(int64_t T, int d, int E) {
+    (void)d;
+    int BN = 0, n_ntiles = 0;
+    choose_bn(E, &BN, &n_ntiles);
+    const int64_t a = (int64_t)ROUTE_MAX_KSPLIT * T;
+    const int64_t b = (ROUTE_SPLIT_TARGET + (T + GM_BM - 1) / GM_BM * n_ntiles) * GM_BM;
+    return a < b ? a : b;
+}
+
+cudaError_t launch_route_split(const float* Wr, int d, int E, __nv_bfloat16* Wsplit, float* wrt,
+                               float* wpart, float* wnorm, cudaStream_t s) {
     const int Ep = route_epad(E);
     const int parts = route_split_parts(d);
-    route_split_kernel<<<dim3((Ep + 31) / 32, parts), 256, 0, s>>>(Wr, d, route_dpad(d), E, Ep,
-                                                                   Wsplit, wpart);
-    route_wnorm_kernel<<<(E + 255) / 256, 256, 0, s>>>(wpart, parts, E, Ep, wnorm);
+    route_split_kernel<<<dim3((Ep + SPLIT_TILE - 1) / SPLIT_TILE, parts), 256, 0, s>>>(
+        Wr, d, route_dpad(d), E, Ep, Wsplit, wrt, wpart);
+    route_wnorm_kernel<<<(E + 7) / 8, 256, 0, s>>>(wpart, parts, E, Ep, wnorm);
     count_launches(2);
     return cudaGetLastError();
 }
 
-cudaError_t launch_route_select(const __nv_bfloat16* x, const float* Wr, const float* b,
-                                const float* logits, int ld, const float* wnorm, int T, int d,
-                                int E, int k, int32_t* idx, float* gate, int32_t* fb_tokens,
-                                float* xnorm, DevStatus* st, int num_sms, cudaStream_t s) {
+cudaError_t launch_route_sum_parts(const float* logits, int64_t part_stride, int nparts, int64_t n,
+                                   float* out, cudaStream_t s) {
+    route_sum_parts_kernel<<<(unsigned)((n + 255) / 256), 256, 0, s>>>(logits, part_stride, nparts,
+                                                                        n, out);
+    count_launches(1);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_route_select(const __nv_bfloat16* x, const float* wrt, const float* b,
+                                float* logits, int ld, int nparts, int64_t part_stride,
+                                const float* wnorm, int T, int d, int E, int k, int32_t* idx,
+                                float* gate, int32_t* fb_tokens, float* xnorm, DevStatus* st,
+                                int num_sms, cudaStream_t s) {
     reset_fallback_count<<<1, 1, 0, s>>>(st);
     const int blocks = (int)(((int64_t)T * 32 + 255) / 256);
-    const int64_t fb_warps = T < 16 * (int64_t)num_sms ? (int64_t)T : 16 * (int64_t)num_sms;
-    const int fb_blocks = (int)((fb_warps * 32 + 255) / 256);
+    const int fb_blocks = T < 4 * num_sms ? T : 4 * num_sms;
     const int npl = (E + 31) / 32;
+    const int dp = route_dpad(d);
 #define MV_ROUTE(N)                                                                              \
     do {                                                                                         \
-        route_topk_kernel<N><<<blocks, 256, 0, s>>>(x, logits, ld, b, wnorm, T, d, E, k, idx,    \
-                                                    gate, xnorm, fb_tokens, st);                 \
-        route_fallback_kernel<N><<<fb_blocks, 256, 0, s>>>(x, Wr, b, logits, ld, xnorm, wnorm, d, \
-                                                           E, k, idx, gate, fb_tokens, st);      \
+        route_topk_kernel<N><<<blocks, 256, 0, s>>>(x, logits, ld, nparts, part_stride, b,       \
+                                                    wnorm, T, d, E, k, idx, gate, xnorm,         \
+                                                    fb_tokens, st);                              \
+        route_fallback_kernel<N><<<fb_blocks, 256, 0, s>>>(x, wrt, dp, b, logits, ld, xnorm,     \
+                                                           wnorm, d, E, k, idx, gate, fb_tokens, \
+                                                           st);                                  \
     } while (0)
     if (npl <= 1) MV_ROUTE(1);
     else if (npl <= 2) MV_ROUTE(2);
