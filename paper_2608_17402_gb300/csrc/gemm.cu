@@ -26,8 +26,8 @@
 //
 // Warp roles (480 threads per CTA, one CTA per SM):
 //   warps 0-7   epilogue: tcgen05.ld of the CTA's 128 accumulator rows (warp w:
-//               TMEM lanes 32 (w%4)..+31, every other 16-column chunk), fused math,
-//               sector-wide stores (fp32 results pass a per-warp smem transpose)
+//               TMEM lanes 32 (w%4)..+31, every other 32-column chunk), fused math,
+//               and 16-byte stores / reductions of each thread's own row
 //   warp 8      TMEM allocation (both CTAs, jointly); leader lane 0 issues the MMAs
 //   warp 9      lane 0: TMA loads of the B half and, for contiguous A rows, of A;
 //               the leader posts the byte count of both CTAs on its full barrier
@@ -35,8 +35,9 @@
 //               swizzled K-major layout; each thread hands the completion of its
 //               copies to the stage's local afull barrier and moves on
 //   warp 14     lane 0: waits for afull, fences the stage to the async proxy and
-//               arrives on the leader's full barrier (remotely from the peer)
-// Shared memory: 6 stages x (A 128x64 + B 64x128) bf16; TMEM: two fp32 accumulators
+//               publishes it on the leader's full barrier (from the peer: a 16-byte
+//               bulk copy that completes transaction bytes there)
+// Shared memory: 7 stages x (A 128x64 + B 64x128) bf16; TMEM: two fp32 accumulators
 // of 256 columns, so the epilogue of one tile overlaps the main loop of the next.
 //
 // Operand layouts (tcgen05 shared-memory descriptors, 128-byte swizzle):
@@ -55,7 +56,6 @@ namespace mv {
 
 namespace {
 
-constexpr int STG_LD = GM_STG_LD;
 
 // ------------------------------------------------------------ pair helpers
 
@@ -84,9 +84,12 @@ __device__ __forceinline__ void bulk_signal_remote(uint32_t dst_cluster, uint32_
             "r"(dst_cluster), "r"(src), "r"(bar_cluster)
         : "memory");
 }
+// Arrival on a barrier of another CTA of the cluster, with the default (CTA-scope)
+// release: used where the arriving thread has nothing to publish but completed
+// tcgen05.ld reads (ordered by tcgen05 fences around the barrier), so no
+// cluster-wide release of its earlier stores is needed.
 __device__ __forceinline__ void mbar_arrive_remote(uint32_t bar_cluster) {
-    asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(bar_cluster)
-                 : "memory");
+    asm volatile("mbarrier.arrive.shared::cluster.b64 _, [%0];" ::"r"(bar_cluster) : "memory");
 }
 // TMA loads into this CTA's shared memory that complete on a barrier of either CTA
 // of the pair.
@@ -197,7 +200,6 @@ struct Smem {
     uint32_t tfull, tempty;
     uint32_t drain;
     uint32_t sink;            // 16 bytes: target / source of the peer's stage signals
-    float* stage_out;         // epilogue transpose buffers, 32 x STG_LD floats per warp
     uint32_t rank;            // rank of this CTA in its pair
     int64_t pair, npairs;     // pair index and count
 };
@@ -438,21 +440,20 @@ __device__ void mma_issuer(const GemmArgs& p, const Smem& sm, uint32_t tmem, int
 
 // -------------------------------------------------------------- epilogue
 
-// Warp w reads TMEM lanes 32 (w % 4) .. +31 (its rows of the CTA's half) and the
-// 16-column chunks c = w / 4, w / 4 + 2, ... of each tile.  bf16 outputs: every
-// thread stores its row's 16 values as one 32-byte sector.  fp32 outputs (y
-// accumulator, logits): a shared-memory transpose first, so that 4 lanes cover 64
-// contiguous bytes of a row and each vector reduction / store touches whole sectors.
-// When a warp has read its last chunk of the accumulator it arrives (once) on the
-// leader's tempty barrier.
+// Warp w reads TMEM lanes 32 (w % 4) .. +31 (its rows) and the 32-column chunks
+// c = w / 4, w / 4 + 2, ... of each tile.  bf16 outputs and fp32 stores: each thread
+// takes its own row (32x32b loads) and writes it straight from registers with
+// 16-byte stores.  fp32 reductions (the y accumulator): 16x256b loads give four
+// consecutive threads the 8 columns of one 32-byte sector of a row; one shuffle
+// between lane pairs leaves each lane 4 consecutive columns, so every 16-byte
+// vector reduction of a warp covers whole sectors in L2.  When a warp has read
+// its last chunk of the accumulator it arrives (once) on the leader's tempty barrier.
 __device__ void epilogue(const GemmArgs& p, const Smem& sm, uint32_t tmem, int64_t n_work,
                          volatile int* abort_flag) {
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int quad = warp & 3, half = warp >> 2;
-    float* stg = sm.stage_out + warp * (32 * STG_LD);
     const bool to_f32 = (p.epi == EPI_ADD_F32 || p.epi == EPI_STORE_F32);
-    const int rsub = lane >> 2, c4 = (lane & 3) * 4;   // transposed: rows 8 i + rsub, columns c4..c4+3
-    const int nchunk = (p.BN + 15) / 16;
+    const int nchunk = p.BN / 32;
     const uint32_t tempty_leader = peer_addr(sm.tempty, 0);
     int it = 0;
     for (int64_t w = sm.pair; w < n_work; w += sm.npairs, ++it) {
@@ -472,6 +473,24 @@ __device__ void epilogue(const GemmArgs& p, const Smem& sm, uint32_t tmem, int64
                 ok_row = false;
             }
         }
+        // reductions: rows quad*32 + 16 (q / 2) + 8 (q % 2) + lane / 4 of the 16x256b loads
+        int64_t yoff[4];
+        float ysc[4];
+        if (p.epi == EPI_ADD_F32) {
+#pragma unroll
+            for (int q = 0; q < 4; ++q) {
+                const int r = quad * 32 + 16 * (q >> 1) + 8 * (q & 1) + (lane >> 2);
+                const int rg = t.row0 + (int)sm.rank * GM_HALF + r;
+                yoff[q] = -1;
+                ysc[q] = p.scale;
+                if (r < rows_half(t, sm.rank)) {
+                    const int64_t tk = p.o_rows ? __ldg(p.o_rows + rg) / p.o_div : rg;
+                    if (p.row_scale) ysc[q] = __ldg(p.row_scale + rg);
+                    if (tk < 0 || tk >= p.o_nrows) report(p.status, MOEVIE_ERR_DEVICE, SITE_GEMM_OUT_ROW, rg, (int)tk);
+                    else yoff[q] = t.ks * p.y_split_stride + tk * p.ldy;
+                }
+            }
+        }
         if (!mbar_wait(sm.tfull + 8 * acc, aph, p.limit_ns, abort_flag)) {
             set_abort(abort_flag, p.status, SITE_GEMM_WAIT_TFULL, (int)sm.pair, it);
             return;
@@ -484,59 +503,80 @@ __device__ void epilogue(const GemmArgs& p, const Smem& sm, uint32_t tmem, int64
             if (lane == 0) mbar_arrive_remote(tempty_leader + 8 * acc);
         }
         for (int ch = half; ch < nchunk; ch += 2) {
-            const int c0 = ch * 16;
-            uint32_t v[16];
-            tmem_ld_32x32b_x16(tbase + c0, v);
+            const int c0 = ch * 32;
+            if (p.epi == EPI_ADD_F32) {
+                uint32_t va[16], vb[16];
+                tmem_ld_16x256b_x4(tbase + c0, va);                  // lanes +0..15
+                tmem_ld_16x256b_x4(tbase + (16u << 16) + c0, vb);    // lanes +16..31
+                tmem_wait_ld();
+                if (ch + 2 >= nchunk) {   // this warp's last read of the accumulator
+                    tc_fence_before();
+                    __syncwarp();
+                    if (lane == 0) mbar_arrive_remote(tempty_leader + 8 * acc);
+                }
+                // Lanes 2m and 2m+1 swap halves so that each holds 4 consecutive
+                // columns: the even lane of repetition j, the odd lane of j + 1.
+                const int odd = lane & 1;
+                const int colq = t.n0 + c0 + 2 * (lane & 2);
+#pragma unroll
+                for (int jp = 0; jp < 4; jp += 2) {
+#pragma unroll
+                    for (int q = 0; q < 4; ++q) {
+                        const int o = 2 * (q & 1);
+                        const uint32_t* v = (q < 2) ? va : vb;
+                        const float x0 = __uint_as_float(v[4 * jp + o]), x1 = __uint_as_float(v[4 * jp + o + 1]);
+                        const float y0 = __uint_as_float(v[4 * jp + 4 + o]),
+                                    y1 = __uint_as_float(v[4 * jp + 4 + o + 1]);
+                        const float s0 = __shfl_xor_sync(0xffffffffu, odd ? x0 : y0, 1);
+                        const float s1 = __shfl_xor_sync(0xffffffffu, odd ? x1 : y1, 1);
+                        const int col = colq + 8 * (jp + odd);
+                        if (yoff[q] < 0 || col >= p.N) continue;
+                        const float4 val = odd ? make_float4(s0, s1, y0, y1) : make_float4(x0, x1, s0, s1);
+                        const float sc4 = ysc[q];
+                        atomicAdd(reinterpret_cast<float4*>(p.yacc + yoff[q] + col),
+                                  make_float4(sc4 * val.x, sc4 * val.y, sc4 * val.z, sc4 * val.w));
+                    }
+                }
+                continue;
+            }
+            uint32_t v[32];
+            tmem_ld_32x32b_x32(tbase + c0, v);
             tmem_wait_ld();
             if (ch + 2 >= nchunk) {   // this warp's last read of the accumulator
                 tc_fence_before();
                 __syncwarp();
                 if (lane == 0) mbar_arrive_remote(tempty_leader + 8 * acc);
             }
+            if (!ok_row) continue;
             const int n = t.n0 + c0;
             if (!to_f32) {
-                if (ok_row) {
+                __nv_bfloat16* orow = p.out + (int64_t)gr * p.ldo + n;
 #pragma unroll
-                    for (int g8 = 0; g8 < 2; ++g8) {
-                        if (c0 + 8 * g8 >= p.BN || n + 8 * g8 >= p.N) continue;
-                        float f[8];
+                for (int g8 = 0; g8 < 4; ++g8) {
+                    if (n + 8 * g8 >= p.N) break;
+                    float f[8];
 #pragma unroll
-                        for (int i = 0; i < 8; ++i) {
-                            f[i] = __uint_as_float(v[8 * g8 + i]);
-                            if (p.epi == EPI_GELU_BF16) f[i] = gelu_erf(f[i]);
-                        }
-                        uint4 u;
-                        u.x = pack_bf16x2(f[0], f[1]);
-                        u.y = pack_bf16x2(f[2], f[3]);
-                        u.z = pack_bf16x2(f[4], f[5]);
-                        u.w = pack_bf16x2(f[6], f[7]);
-                        *reinterpret_cast<uint4*>(p.out + (int64_t)gr * p.ldo + n + 8 * g8) = u;
+                    for (int i = 0; i < 8; ++i) {
+                        f[i] = __uint_as_float(v[8 * g8 + i]);
+                        if (p.epi == EPI_GELU_BF16) f[i] = gelu_erf(f[i]);
                     }
+                    uint4 u;
+                    u.x = pack_bf16x2(f[0], f[1]);
+                    u.y = pack_bf16x2(f[2], f[3]);
+                    u.z = pack_bf16x2(f[4], f[5]);
+                    u.w = pack_bf16x2(f[6], f[7]);
+                    *reinterpret_cast<uint4*>(orow + 8 * g8) = u;
                 }
-                continue;
-            }
+            } else {
+                float* yrow = p.yacc + t.ks * p.y_split_stride + tok * p.ldy + n;
 #pragma unroll
-            for (int q = 0; q < 4; ++q)
-                *reinterpret_cast<float4*>(stg + lane * STG_LD + 4 * q) =
-                    make_float4(__uint_as_float(v[4 * q]), __uint_as_float(v[4 * q + 1]),
-                                __uint_as_float(v[4 * q + 2]), __uint_as_float(v[4 * q + 3]));
-            __syncwarp();
-            const bool col_ok = (c0 + c4 < p.BN) && (n + c4 < p.N);
-#pragma unroll
-            for (int i = 0; i < 4; ++i) {
-                const int rr = 8 * i + rsub;
-                const int64_t rtok = __shfl_sync(0xffffffffu, tok, rr);
-                const float rsc = __shfl_sync(0xffffffffu, sc, rr);
-                const bool rok = __shfl_sync(0xffffffffu, ok_row ? 1 : 0, rr) != 0;
-                const float4 f = *reinterpret_cast<const float4*>(stg + rr * STG_LD + c4);
-                if (!(rok && col_ok)) continue;
-                float4* dst = reinterpret_cast<float4*>(p.yacc + t.ks * p.y_split_stride +
-                                                        rtok * p.ldy + n + c4);
-                const float4 val = make_float4(rsc * f.x, rsc * f.y, rsc * f.z, rsc * f.w);
-                if (p.epi == EPI_ADD_F32) atomicAdd(dst, val);
-                else *dst = val;
+                for (int q = 0; q < 8; ++q) {
+                    if (n + 4 * q >= p.N) break;
+                    *reinterpret_cast<float4*>(yrow + 4 * q) =
+                        make_float4(sc * __uint_as_float(v[4 * q]), sc * __uint_as_float(v[4 * q + 1]),
+                                    sc * __uint_as_float(v[4 * q + 2]), sc * __uint_as_float(v[4 * q + 3]));
+                }
             }
-            __syncwarp();
         }
     }
 }
@@ -547,8 +587,7 @@ __global__ void __launch_bounds__(GM_THREADS, 1) grouped_gemm_kernel(const __gri
         (reinterpret_cast<uintptr_t>(gm_smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
     uint8_t* sA = smem;
     uint8_t* sB = smem + GM_STAGES * GM_A_BYTES;
-    float* sOut = reinterpret_cast<float*>(sB + GM_STAGES * GM_B_BYTES);
-    uint64_t* bars = reinterpret_cast<uint64_t*>(sOut + GM_EPI_WARPS * 32 * STG_LD);
+    uint64_t* bars = reinterpret_cast<uint64_t*>(sB + GM_STAGES * GM_B_BYTES);
     uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 3 * GM_STAGES + 5);
     volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
     uint8_t* sink = reinterpret_cast<uint8_t*>(bars) + 256;   // 16-byte aligned, after the barriers
@@ -563,7 +602,6 @@ __global__ void __launch_bounds__(GM_THREADS, 1) grouped_gemm_kernel(const __gri
     sm.tempty = sm.tfull + 16;
     sm.drain = sm.tempty + 16;
     sm.sink = smem_u32(sink);
-    sm.stage_out = sOut;
     sm.rank = cluster_rank();
     sm.pair = blockIdx.x >> 1;
     sm.npairs = gridDim.x >> 1;

@@ -83,9 +83,9 @@ cudaError_t launch_tile_table(const int32_t* offsets, int G, int bm, int4* tiles
 constexpr int GM_BM = 256;        // rows per m-tile: one CTA pair, 128 rows per CTA
 constexpr int GM_HALF = 128;      // rows per CTA (tcgen05 M = 256 across the pair)
 constexpr int GM_BK = 64;         // K per stage: 64 bf16 = one 128-byte swizzle row
-constexpr int GM_STAGES = 6;
+constexpr int GM_STAGES = 7;
 constexpr int GM_MAXBN = 256;     // largest N of one tcgen05.mma
-constexpr int GM_EPI_WARPS = 8;   // two warps per TMEM lane quadrant, alternate 16-column chunks
+constexpr int GM_EPI_WARPS = 8;   // two warps per TMEM lane quadrant, alternate 32-column chunks
 constexpr int GM_WARP_MMA = GM_EPI_WARPS;        // TMEM allocation + tcgen05.mma issue
 constexpr int GM_WARP_LOAD = GM_EPI_WARPS + 1;   // TMA loads of B (and of contiguous A)
 constexpr int GM_WARP_GATHER = GM_EPI_WARPS + 2; // first of 4 token-gather warps
@@ -93,9 +93,9 @@ constexpr int GM_WARP_FWD = GM_EPI_WARPS + 6;    // publishes gathered stages
 constexpr int GM_THREADS = (GM_EPI_WARPS + 7) * 32;
 constexpr int GM_A_BYTES = GM_HALF * GM_BK * 2;           // one CTA's A rows per stage
 constexpr int GM_B_BYTES = GM_BK * (GM_MAXBN / 2) * 2;    // one CTA's half of B per stage
-constexpr int GM_STG_LD = 20;                   // floats per row of a transpose buffer
-constexpr int GM_STG_BYTES = GM_EPI_WARPS * 32 * GM_STG_LD * 4;   // epilogue transpose buffers
-constexpr int GM_SMEM_BYTES = GM_STAGES * (GM_A_BYTES + GM_B_BYTES) + GM_STG_BYTES + 1024 + 512;
+// stages, 1 KB to align them, barriers / TMEM slot / flags / signal sink
+constexpr int GM_SMEM_BYTES = GM_STAGES * (GM_A_BYTES + GM_B_BYTES) + 1024 + 512;
+static_assert(GM_SMEM_BYTES <= 232448, "shared memory of one CTA");
 
 inline int64_t max_mtiles(int64_t rows, int64_t groups) { return (rows + GM_BM - 1) / GM_BM + groups; }
 
