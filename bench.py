@@ -56,6 +56,34 @@ def peaks():
             "source": "fallback"}
 
 
+GEMM_SOURCES = ("paper_2608_17402_gb300/csrc/gemm.cu", "paper_2608_17402_gb300/csrc/common.cuh",
+                "paper_2608_17402_gb300/csrc/internal.h")
+TRAFFIC_FILE = os.path.join(ROOT, "profiles", "grouped_gemm_dram_traffic.json")
+
+
+def gemm_sources_hash():
+    import hashlib
+    h = hashlib.sha256()
+    for rel in GEMM_SOURCES:
+        with open(os.path.join(ROOT, rel), "rb") as f:
+            h.update(f.read())
+    return h.hexdigest()
+
+
+def captured_traffic(cfg_name, stage):
+    """DRAM bytes (read + write) of one grouped GEMM launch from the committed ncu
+    capture, or None when there is none for this workload or the GEMM sources have
+    changed since it was taken."""
+    if not os.path.exists(TRAFFIC_FILE):
+        return None
+    with open(TRAFFIC_FILE) as f:
+        rec = json.load(f)
+    if rec.get("sources_sha256") != gemm_sources_hash():
+        return None
+    per = rec.get("workloads", {}).get(cfg_name, {}).get(stage)
+    return None if per is None else float(per["dram_bytes"])
+
+
 def layer_work(cfg, counts):
     """Algorithmic FLOPs and bytes of one layer forward (weights of touched experts)."""
     T, d, E, k, h, hs = cfg.T, cfg.d, cfg.E, cfg.k, cfg.h, cfg.h_s
@@ -191,6 +219,7 @@ def run_ours(args, rank, world):
 
     import __graft_entry__
     from paper_2608_17402_gb300 import moevie
+    from paper_2608_17402_gb300.replicas import max_over_ranks
 
     local = int(os.environ.get("LOCAL_RANK", "0"))
     torch.cuda.set_device(local)
@@ -275,10 +304,7 @@ def run_ours(args, rank, world):
     if code != 0:
         raise RuntimeError(f"device status {code} {detail}")
 
-    if world > 1:
-        t = torch.tensor([ms, e2e_ms], device="cuda", dtype=torch.float64)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        ms, e2e_ms = float(t[0]), float(t[1])
+    ms, e2e_ms = max_over_ranks([ms, e2e_ms], device="cuda")   # slowest rank
     if rank != 0:
         return
 
@@ -298,7 +324,8 @@ def run_ours(args, rank, world):
                    "l2": f"flushed between steps ({L2_FLUSH_BYTES >> 20} MiB write outside the timed window)"},
         "roofline": {"bound": "tensor", "kernel": f"grouped_gemm_kernel ({dom})", "achieved": achieved,
                      "peak": pk["bf16_tflops"], "unit": "TFLOP/s", "frac": achieved / pk["bf16_tflops"],
-                     "traffic": None, "peak_source": pk["source"] + " bf16 burst"},
+                     "traffic": captured_traffic(cfg.name, dom),
+                     "peak_source": pk["source"] + " bf16 burst (of measured)"},
         "layer_roofline": {"flops": work["flops"], "bytes": work["bytes"], "roofline_us": t_roof * 1e6,
                            "frac": t_roof / (ms / 1e3), "touched_experts": work["touched_experts"],
                            "peaks": pk},

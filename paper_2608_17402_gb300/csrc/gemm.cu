@@ -394,7 +394,11 @@ __device__ void mma_issuer(const GemmArgs& p, const Smem& sm, uint32_t tmem, int
     uint32_t ph = 0;
     int it = 0;
     bool issued = false;
+    Tile tn{};   // next item's tile, decoded one item ahead (its table read is a global load)
+    if (sm.pair < n_work) tn = decode_tile(p, sm.pair);
     for (int64_t w = sm.pair; w < n_work; w += sm.npairs, ++it) {
+        const Tile t = tn;
+        if (w + sm.npairs < n_work) tn = decode_tile(p, w + sm.npairs);
         const int acc = it & 1;
         const uint32_t aph = (uint32_t)(it >> 1) & 1u;
         if (!mbar_wait(sm.tempty + 8 * acc, aph ^ 1u, p.limit_ns, abort_flag)) {
@@ -403,15 +407,16 @@ __device__ void mma_issuer(const GemmArgs& p, const Smem& sm, uint32_t tmem, int
         }
         tc_fence_after();
         const uint32_t d_tmem = tmem + (uint32_t)acc * GM_MAXBN;
-        const Tile t = decode_tile(p, w);
         bool ok = true;
         for (int kb = t.kb0; kb < t.kb1; ++kb) {
+            // Operands in shared memory are ordered by the barrier alone (TMA bytes, or
+            // gathered rows fenced to the async proxy before they were published); the
+            // tcgen05 thread-sync fence is needed only where TMEM changes hands.
             if (!mbar_wait(sm.full + 8 * s, ph, p.limit_ns, abort_flag)) {
                 set_abort(abort_flag, p.status, SITE_GEMM_WAIT_FULL, (int)sm.pair, kb);
                 ok = false;
                 break;
             }
-            tc_fence_after();
             const uint32_t a_addr = sm.a0 + s * GM_A_BYTES;
             const uint32_t b_addr = sm.b0 + s * GM_B_BYTES;
 #pragma unroll

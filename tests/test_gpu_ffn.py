@@ -39,6 +39,7 @@ SHAPES = [
     (3, 515, 256, 6, 1, 96, [0, 1, 127, 128, 129, 130]),   # segment-length edges incl. an empty expert
     (4, 257, 1024, 3, 3, 512, None),      # k = E, long K loop
     (5, 40, 776, 2, 1, 48, None),         # d % 16 != 0 (8-column output tail), K tail in the up GEMM
+    (6, 899, 192, 6, 1, 64, [0, 1, 255, 256, 257, 130]),   # segments around the 256-row m-tile
 ]
 
 

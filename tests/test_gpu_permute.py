@@ -40,10 +40,10 @@ def test_permute_matches_oracle(T, E, k, empty, hot):
     assert np.array_equal(inv.cpu().numpy(), oi)
 
 
-def test_permute_segment_length_edges():
-    """Segments of 0, 1, 127, 128, 129 and 255 rows (the GEMM tile is 128 rows)."""
-    E, k = 6, 1
-    sizes = [0, 1, 127, 128, 129, 255]
+@pytest.mark.parametrize("sizes", [[0, 1, 127, 128, 129, 255], [0, 1, 255, 256, 257, 511, 512, 513]])
+def test_permute_segment_length_edges(sizes):
+    """Segments around the 128-row CTA half and the 256-row m-tile of the GEMMs."""
+    E, k = len(sizes), 1
     ids = np.concatenate([np.full(n, e, np.int32) for e, n in enumerate(sizes)])
     rng = np.random.default_rng(3)
     rng.shuffle(ids)
