@@ -29,7 +29,8 @@ inline bool a16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) =
 // stage (which passes 0 for the sizes it does not use).
 struct Layout {
     size_t status, xnorm, wnorm, wpart, wsplit, wrt, logits, fb_tokens;
-    size_t idx, gate, hist, counts, offsets, tiles, n_tiles, perm, inv, row_tok, row_gate;
+    size_t idx, gate, hist, counts, offsets, tiles, n_tiles, items, n_items, perm, inv, row_tok,
+        row_gate;
     size_t H, Hs, yacc;
     size_t total;
 };
@@ -59,6 +60,10 @@ Layout make_layout(int64_t T, int64_t d, int64_t E, int64_t k, int64_t h, int64_
     L.counts = take(4 * E);
     L.offsets = take(4 * (E + 1));
     L.tiles = take(16 * max_mtiles(n, E));
+    int BN = 0, n_nt = 0;
+    choose_bn((int)(d > 0 ? d : 1), &BN, &n_nt);
+    L.items = take(16 * max_mtiles(n, E) * n_nt);   // band-ordered down-projection items
+    L.n_items = take(4);
     L.n_tiles = take(4);
     L.perm = take(4 * n);
     L.inv = take(4 * n);
@@ -134,6 +139,7 @@ struct GemmSpec {
     float scale;
     int ksplit;              // 0 or 1: no split of K; fp32 outputs only otherwise
     int64_t y_split_stride;  // floats between the outputs of consecutive splits
+    int item_table;          // tiles / n_tiles hold (m-tile, n-tile) work items
 };
 
 moevie_status run_gemm(const GemmSpec& g, DevStatus* st, cudaStream_t s) {
@@ -153,6 +159,7 @@ moevie_status run_gemm(const GemmSpec& g, DevStatus* st, cudaStream_t s) {
     a.tiles = g.tiles;
     a.n_tiles_dev = g.n_tiles;
     a.max_mtiles = g.tiles ? max_mtiles(g.m_total, g.G) : (g.m_total + GM_BM - 1) / GM_BM;
+    a.item_table = g.item_table;
     a.G = g.G;
     a.K = g.K;
     a.N = g.N;
@@ -175,7 +182,11 @@ moevie_status run_gemm(const GemmSpec& g, DevStatus* st, cudaStream_t s) {
     a.y_split_stride = g.y_split_stride;
     a.status = st;
     a.limit_ns = WAIT_LIMIT_NS;
-    const int64_t work = a.max_mtiles * a.n_ntiles * a.ksplit;   // one CTA pair per work item at most
+    if (a.item_table) {
+        if (!g.tiles || a.ksplit != 1) return MOEVIE_ERR_UNSUPPORTED;
+        a.max_mtiles *= a.n_ntiles;   // bound on the item count
+    }
+    const int64_t work = a.item_table ? a.max_mtiles : a.max_mtiles * a.n_ntiles * a.ksplit;   // one CTA pair per item at most
     const int sms = num_sms() & ~1;
     const int grid = (int)(2 * work < sms ? (work > 0 ? 2 * work : 2) : sms);
     return cuda_status(launch_grouped_gemm(a, grid, s));
@@ -468,6 +479,40 @@ moevie_status moevie_combine(const void* out_rows, const int32_t* inv, const flo
                                       static_cast<cudaStream_t>(stream)));
 }
 
+// Work order of the down-projection.  Its epilogue adds every routed row into the
+// fp32 y accumulator [T, d]; when that is larger than ITEM_BAND_MIN_BYTES (it would
+// not stay in L2 next to the streamed operands) the items run in nb token bands x
+// column groups of gsz n-tiles (item_order_kernel), so that the accumulator block
+// being reduced into (at most ITEM_BLOCK_BYTES) stays in L2.  Each extra band re-reads
+// the expert weights W2, each extra column group the rows of H: the split minimises
+// that traffic under the block-size bound.
+constexpr double ITEM_BAND_MIN_BYTES = 64.0 * (1 << 20);
+constexpr double ITEM_BLOCK_BYTES = 24.0 * (1 << 20);
+struct BandPlan {
+    int nb, gsz;
+};
+BandPlan choose_bands(int64_t T, int64_t d, int64_t E, int64_t k, int64_t h) {
+    int BN = 0, nnt = 0;
+    choose_bn((int)d, &BN, &nnt);
+    const double yacc = 4.0 * T * d;
+    if (yacc <= ITEM_BAND_MIN_BYTES || max_mtiles(T * k, E) > ITEM_MAX_TILES) return {1, nnt};
+    const double Hb = 2.0 * T * k * h, Wb = 2.0 * E * h * d;
+    BandPlan best{1, nnt};
+    double best_cost = 1e300;
+    for (int nb = 1; nb <= ITEM_MAX_BANDS; ++nb)
+        for (int nc = 1; nc <= nnt; ++nc) {
+            const int gsz = (nnt + nc - 1) / nc;
+            const int groups = (nnt + gsz - 1) / gsz;
+            if (yacc / ((double)nb * groups) > ITEM_BLOCK_BYTES) continue;
+            const double cost = Hb * groups + Wb * nb;
+            if (cost < best_cost) {
+                best_cost = cost;
+                best = {nb, gsz};
+            }
+        }
+    return best;
+}
+
 static moevie_status forward_impl(const moevie_layer* Lr, const void* x, int64_t T, void* y,
                                   const moevie_routing* routing, void* ws, size_t ws_bytes,
                                   void* stream, void* const* events, int n_events) {
@@ -512,6 +557,14 @@ static moevie_status forward_impl(const moevie_layer* Lr, const void* x, int64_t
     const int chunk = perm_chunk(T * k, num_sms());
     MV_TRY(launch_permute(idx, T * k, (int)k, (int)E, GM_BM, chunk, gate, at<int32_t>(ws, L.hist),
                           counts, offsets, tiles, n_tiles, perm, inv, row_tok, row_gate, st, s));
+    int dBN = 0, dnt = 0;
+    choose_bn((int)d, &dBN, &dnt);
+    const BandPlan bp = choose_bands(T, d, E, k, h);
+    const bool banded = bp.nb > 1 || bp.gsz < dnt;
+    if (banded)
+        MV_TRY(launch_item_order(tiles, n_tiles, row_tok, T, bp.nb, dnt, bp.gsz, dBN,
+                                 (int)max_mtiles(T * k, E), at<int4>(ws, L.items),
+                                 at<int32_t>(ws, L.n_items), s));
     MV_TRY(mark(2));
     // 3. y accumulator: lambda * shared expert, or zero
     if (hs > 0) {
@@ -532,8 +585,9 @@ static moevie_status forward_impl(const moevie_layer* Lr, const void* x, int64_t
     dn.lda = h;
     dn.a_nrows = T * k;
     dn.m_total = T * k;
-    dn.tiles = tiles;
-    dn.n_tiles = n_tiles;
+    dn.tiles = banded ? at<int4>(ws, L.items) : tiles;
+    dn.n_tiles = banded ? at<int32_t>(ws, L.n_items) : n_tiles;
+    dn.item_table = banded ? 1 : 0;
     dn.G = (int)E;
     dn.W = Lr->W2;
     dn.K = (int)h;

@@ -37,7 +37,8 @@
 //   warp 14     lane 0: waits for afull, fences the stage to the async proxy and
 //               publishes it on the leader's full barrier (from the peer: a 16-byte
 //               bulk copy that completes transaction bytes there)
-// Shared memory: 7 stages x (A 128x64 + B 64x128) bf16; TMEM: two fp32 accumulators
+// Shared memory: 7 stages (6 plus a reduction staging buffer for the y-accumulator
+// epilogue) x (A 128x64 + B 64x128) bf16; TMEM: two fp32 accumulators
 // of 256 columns, so the epilogue of one tile overlaps the main loop of the next.
 //
 // Operand layouts (tcgen05 shared-memory descriptors, 128-byte swizzle):
@@ -154,6 +155,21 @@ __device__ __forceinline__ Tile decode_tile(const GemmArgs& p, int64_t w) {
     w /= p.ksplit;
     t.kb0 = (int)((int64_t)t.ks * p.num_kb / p.ksplit);
     t.kb1 = (int)((int64_t)(t.ks + 1) * p.num_kb / p.ksplit);
+    if (p.item_table) {   // an explicit (m-tile, n-tile) item
+        const int4 d = __ldg(p.tiles + w);
+        t.g = d.x;
+        t.row0 = d.y;
+        t.nrows = d.z;
+        t.n0 = d.w;
+        if (t.nrows < 0 || t.nrows > GM_BM || t.g < 0 || t.g >= p.G || t.n0 < 0 || t.n0 >= p.N ||
+            (int64_t)t.row0 + t.nrows > p.m_total) {
+            report(p.status, MOEVIE_ERR_DEVICE, SITE_GEMM_TILES, t.row0, t.nrows);
+            t.nrows = 0;
+            t.g = 0;
+            t.n0 = 0;
+        }
+        return t;
+    }
     const int mt = (int)(w / p.n_ntiles);
     const int nt = (int)(w - (int64_t)mt * p.n_ntiles);
     if (p.tiles) {
@@ -200,6 +216,8 @@ struct Smem {
     uint32_t tfull, tempty;
     uint32_t drain;
     uint32_t sink;            // 16 bytes: target / source of the peer's stage signals
+    int nstages;              // operand ring depth of this launch
+    float* stg;               // reduction staging: GM_STG_ROWS rows of GM_STG_LD floats per warp
     uint32_t rank;            // rank of this CTA in its pair
     int64_t pair, npairs;     // pair index and count
 };
@@ -257,7 +275,7 @@ __device__ void producer_tma(const GemmArgs& p, const Smem& sm, int64_t n_work,
                 tma_load_2d_pair(sm.a0 + s * GM_A_BYTES, &p.tmA, bar, col,
                                  t.row0 + (int)sm.rank * GM_HALF);
             }
-            if (++s == GM_STAGES) {
+            if (++s == sm.nstages) {
                 s = 0;
                 ph ^= 1u;
             }
@@ -338,7 +356,7 @@ __device__ void producer_gather(const GemmArgs& p, const Smem& sm, int64_t n_wor
                 cp_async16(dst, v ? (const void*)(src[j] + kk) : (const void*)p.A, v ? 16u : 0u);
             }
             cp_async_arrive_noinc(sm.afull + 8 * s);
-            if (++s == GM_STAGES) {
+            if (++s == sm.nstages) {
                 s = 0;
                 ph ^= 1u;
             }
@@ -376,7 +394,7 @@ __device__ void gather_forwarder(const GemmArgs& p, const Smem& sm, int64_t n_wo
             fence_proxy_async_smem();
             if (sm.rank == 0) mbar_arrive(sm.full + 8 * s);
             else bulk_signal_remote(sink_leader, sm.sink, full_leader + 8 * s);
-            if (++s == GM_STAGES) {
+            if (++s == sm.nstages) {
                 s = 0;
                 ph ^= 1u;
             }
@@ -390,6 +408,10 @@ __device__ void gather_forwarder(const GemmArgs& p, const Smem& sm, int64_t n_wo
 __device__ void mma_issuer(const GemmArgs& p, const Smem& sm, uint32_t tmem, int64_t n_work,
                            volatile int* abort_flag) {
     const uint32_t idesc = idesc_bf16_f32(2 * GM_HALF, p.BN, false, true);
+    // A K-major (k-slice +32 B), B MN-major (next 64-column atom LBO 8192, k-slice +2048 B)
+    const uint64_t adesc0 = smem_desc_sw128(sm.a0, 16, 1024);
+    const uint64_t bdesc0 = smem_desc_sw128(sm.b0, 8192, 1024);
+    static_assert(GM_BK == 64, "four k-slices of 16 per stage");
     int s = 0;
     uint32_t ph = 0;
     int it = 0;
@@ -417,17 +439,17 @@ __device__ void mma_issuer(const GemmArgs& p, const Smem& sm, uint32_t tmem, int
                 ok = false;
                 break;
             }
-            const uint32_t a_addr = sm.a0 + s * GM_A_BYTES;
-            const uint32_t b_addr = sm.b0 + s * GM_B_BYTES;
-#pragma unroll
-            for (int kk = 0; kk < GM_BK / 16; ++kk) {
-                const uint64_t ad = smem_desc_sw128(a_addr + kk * 32, 16, 1024);
-                const uint64_t bd = smem_desc_sw128(b_addr + kk * 2048, 8192, 1024);
-                tc_mma_bf16_pair(d_tmem, ad, bd, idesc, (kb != t.kb0 || kk != 0) ? 1u : 0u);
-            }
+            // Descriptors differ from the stage-0 ones only in the start-address field
+            // (bits 0-13, address >> 4; shared addresses stay below 256 KB, no carry).
+            const uint64_t ad = adesc0 + (uint64_t)((s * GM_A_BYTES) >> 4);
+            const uint64_t bd = bdesc0 + (uint64_t)((s * GM_B_BYTES) >> 4);
+            tc_mma_bf16_pair(d_tmem, ad, bd, idesc, kb != t.kb0 ? 1u : 0u);
+            tc_mma_bf16_pair(d_tmem, ad + (32 >> 4), bd + (2048 >> 4), idesc, 1u);
+            tc_mma_bf16_pair(d_tmem, ad + (64 >> 4), bd + (4096 >> 4), idesc, 1u);
+            tc_mma_bf16_pair(d_tmem, ad + (96 >> 4), bd + (6144 >> 4), idesc, 1u);
             issued = true;
             tc_commit_pair(sm.empty + 8 * s);
-            if (++s == GM_STAGES) {
+            if (++s == sm.nstages) {
                 s = 0;
                 ph ^= 1u;
             }
@@ -448,10 +470,9 @@ __device__ void mma_issuer(const GemmArgs& p, const Smem& sm, uint32_t tmem, int
 // Warp w reads TMEM lanes 32 (w % 4) .. +31 (its rows) and the 32-column chunks
 // c = w / 4, w / 4 + 2, ... of each tile.  bf16 outputs and fp32 stores: each thread
 // takes its own row (32x32b loads) and writes it straight from registers with
-// 16-byte stores.  fp32 reductions (the y accumulator): 16x256b loads give four
-// consecutive threads the 8 columns of one 32-byte sector of a row; one shuffle
-// between lane pairs leaves each lane 4 consecutive columns, so every 16-byte
-// vector reduction of a warp covers whole sectors in L2.  When a warp has read
+// 16-byte stores.  fp32 reductions (the y accumulator): the rows pass a small
+// per-warp staging buffer so that each 16-byte vector reduction instruction of a
+// warp covers four rows x 128 contiguous bytes, i.e. whole L2 lines.  When a warp has read
 // its last chunk of the accumulator it arrives (once) on the leader's tempty barrier.
 __device__ void epilogue(const GemmArgs& p, const Smem& sm, uint32_t tmem, int64_t n_work,
                          volatile int* abort_flag) {
@@ -478,24 +499,6 @@ __device__ void epilogue(const GemmArgs& p, const Smem& sm, uint32_t tmem, int64
                 ok_row = false;
             }
         }
-        // reductions: rows quad*32 + 16 (q / 2) + 8 (q % 2) + lane / 4 of the 16x256b loads
-        int64_t yoff[4];
-        float ysc[4];
-        if (p.epi == EPI_ADD_F32) {
-#pragma unroll
-            for (int q = 0; q < 4; ++q) {
-                const int r = quad * 32 + 16 * (q >> 1) + 8 * (q & 1) + (lane >> 2);
-                const int rg = t.row0 + (int)sm.rank * GM_HALF + r;
-                yoff[q] = -1;
-                ysc[q] = p.scale;
-                if (r < rows_half(t, sm.rank)) {
-                    const int64_t tk = p.o_rows ? __ldg(p.o_rows + rg) / p.o_div : rg;
-                    if (p.row_scale) ysc[q] = __ldg(p.row_scale + rg);
-                    if (tk < 0 || tk >= p.o_nrows) report(p.status, MOEVIE_ERR_DEVICE, SITE_GEMM_OUT_ROW, rg, (int)tk);
-                    else yoff[q] = t.ks * p.y_split_stride + tk * p.ldy;
-                }
-            }
-        }
         if (!mbar_wait(sm.tfull + 8 * acc, aph, p.limit_ns, abort_flag)) {
             set_abort(abort_flag, p.status, SITE_GEMM_WAIT_TFULL, (int)sm.pair, it);
             return;
@@ -510,37 +513,41 @@ __device__ void epilogue(const GemmArgs& p, const Smem& sm, uint32_t tmem, int64
         for (int ch = half; ch < nchunk; ch += 2) {
             const int c0 = ch * 32;
             if (p.epi == EPI_ADD_F32) {
-                uint32_t va[16], vb[16];
-                tmem_ld_16x256b_x4(tbase + c0, va);                  // lanes +0..15
-                tmem_ld_16x256b_x4(tbase + (16u << 16) + c0, vb);    // lanes +16..31
+                // Each lane holds its row's 32 columns; half the warp at a time writes
+                // its rows (scaled, plus the row's y offset) into the staging buffer,
+                // then every lane reduces 4 columns of one of 4 rows per instruction:
+                // 8 lanes cover a row's 128 contiguous bytes (a whole L2 line).
+                uint32_t v[32];
+                tmem_ld_32x32b_x32(tbase + c0, v);
                 tmem_wait_ld();
                 if (ch + 2 >= nchunk) {   // this warp's last read of the accumulator
                     tc_fence_before();
                     __syncwarp();
                     if (lane == 0) mbar_arrive_remote(tempty_leader + 8 * acc);
                 }
-                // Lanes 2m and 2m+1 swap halves so that each holds 4 consecutive
-                // columns: the even lane of repetition j, the odd lane of j + 1.
-                const int odd = lane & 1;
-                const int colq = t.n0 + c0 + 2 * (lane & 2);
+                const int n = t.n0 + c0;
+                float* stg = sm.stg + warp * (GM_STG_ROWS * GM_STG_LD);
 #pragma unroll
-                for (int jp = 0; jp < 4; jp += 2) {
+                for (int hh = 0; hh < 2; ++hh) {
+                    if ((lane >> 4) == hh) {
+                        float* row = stg + (lane & 15) * GM_STG_LD;
 #pragma unroll
-                    for (int q = 0; q < 4; ++q) {
-                        const int o = 2 * (q & 1);
-                        const uint32_t* v = (q < 2) ? va : vb;
-                        const float x0 = __uint_as_float(v[4 * jp + o]), x1 = __uint_as_float(v[4 * jp + o + 1]);
-                        const float y0 = __uint_as_float(v[4 * jp + 4 + o]),
-                                    y1 = __uint_as_float(v[4 * jp + 4 + o + 1]);
-                        const float s0 = __shfl_xor_sync(0xffffffffu, odd ? x0 : y0, 1);
-                        const float s1 = __shfl_xor_sync(0xffffffffu, odd ? x1 : y1, 1);
-                        const int col = colq + 8 * (jp + odd);
-                        if (yoff[q] < 0 || col >= p.N) continue;
-                        const float4 val = odd ? make_float4(s0, s1, y0, y1) : make_float4(x0, x1, s0, s1);
-                        const float sc4 = ysc[q];
-                        atomicAdd(reinterpret_cast<float4*>(p.yacc + yoff[q] + col),
-                                  make_float4(sc4 * val.x, sc4 * val.y, sc4 * val.z, sc4 * val.w));
+                        for (int c = 0; c < 8; ++c)
+                            *reinterpret_cast<float4*>(row + 4 * c) =
+                                make_float4(sc * __uint_as_float(v[4 * c]), sc * __uint_as_float(v[4 * c + 1]),
+                                            sc * __uint_as_float(v[4 * c + 2]), sc * __uint_as_float(v[4 * c + 3]));
+                        *reinterpret_cast<int64_t*>(row + 32) = ok_row ? t.ks * p.y_split_stride + tok * p.ldy : -1;
                     }
+                    __syncwarp();
+                    const int col = n + 4 * (lane & 7);
+#pragma unroll
+                    for (int r = 0; r < 4; ++r) {
+                        const float* row = stg + (4 * r + (lane >> 3)) * GM_STG_LD;
+                        const int64_t yo = *reinterpret_cast<const int64_t*>(row + 32);
+                        const float4 val = *reinterpret_cast<const float4*>(row + 4 * (lane & 7));
+                        if (yo >= 0 && col < p.N) atomicAdd(reinterpret_cast<float4*>(p.yacc + yo + col), val);
+                    }
+                    __syncwarp();
                 }
                 continue;
             }
@@ -591,9 +598,11 @@ __global__ void __launch_bounds__(GM_THREADS, 1) grouped_gemm_kernel(const __gri
     uint8_t* smem = reinterpret_cast<uint8_t*>(
         (reinterpret_cast<uintptr_t>(gm_smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
     uint8_t* sA = smem;
-    uint8_t* sB = smem + GM_STAGES * GM_A_BYTES;
-    uint64_t* bars = reinterpret_cast<uint64_t*>(sB + GM_STAGES * GM_B_BYTES);
-    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 3 * GM_STAGES + 5);
+    const int nst = gm_stages(p.epi);
+    uint8_t* sB = smem + nst * GM_A_BYTES;
+    uint8_t* sStg = sB + nst * GM_B_BYTES;                       // reduction staging (EPI_ADD_F32)
+    uint64_t* bars = reinterpret_cast<uint64_t*>(sStg + (p.epi == EPI_ADD_F32 ? GM_STG_BYTES : 0));
+    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 3 * GM_STAGES_MAX + 5);
     volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
     uint8_t* sink = reinterpret_cast<uint8_t*>(bars) + 256;   // 16-byte aligned, after the barriers
 
@@ -601,11 +610,13 @@ __global__ void __launch_bounds__(GM_THREADS, 1) grouped_gemm_kernel(const __gri
     sm.a0 = smem_u32(sA);
     sm.b0 = smem_u32(sB);
     sm.full = smem_u32(bars);
-    sm.empty = sm.full + 8 * GM_STAGES;
-    sm.afull = sm.empty + 8 * GM_STAGES;
-    sm.tfull = sm.afull + 8 * GM_STAGES;
+    sm.empty = sm.full + 8 * GM_STAGES_MAX;
+    sm.afull = sm.empty + 8 * GM_STAGES_MAX;
+    sm.tfull = sm.afull + 8 * GM_STAGES_MAX;
     sm.tempty = sm.tfull + 16;
     sm.drain = sm.tempty + 16;
+    sm.nstages = nst;
+    sm.stg = reinterpret_cast<float*>(sStg);
     sm.sink = smem_u32(sink);
     sm.rank = cluster_rank();
     sm.pair = blockIdx.x >> 1;
@@ -614,7 +625,7 @@ __global__ void __launch_bounds__(GM_THREADS, 1) grouped_gemm_kernel(const __gri
     const int warp = threadIdx.x >> 5;
     const bool gather = p.a_rows != nullptr;
     if (threadIdx.x == 0) {
-        for (int s = 0; s < GM_STAGES; ++s) {
+        for (int s = 0; s < nst; ++s) {
             // leader's expect_tx arrival (+ the leader's forwarder; the peer's signals
             // are transaction bytes)
             mbar_init(sm.full + 8 * s, 1 + (gather ? 1 : 0));
@@ -648,7 +659,7 @@ __global__ void __launch_bounds__(GM_THREADS, 1) grouped_gemm_kernel(const __gri
     } else {
         n_mtiles = (p.m_total + GM_BM - 1) / GM_BM;
     }
-    const int64_t n_work = n_mtiles * p.n_ntiles * p.ksplit;
+    const int64_t n_work = p.item_table ? n_mtiles * p.ksplit : n_mtiles * p.n_ntiles * p.ksplit;
 
     if (warp < GM_EPI_WARPS) {
         epilogue(p, sm, tmem, n_work, abort_flag);
@@ -727,14 +738,14 @@ cudaError_t launch_grouped_gemm(const GemmArgs& a, int grid, cudaStream_t s) {
     if (dev >= 0 && dev < 64 && !attr_set[dev]) {
         cudaError_t e = cudaFuncSetAttribute(grouped_gemm_kernel,
                                              cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                             GM_SMEM_BYTES);
+                                             GM_SMEM_BYTES_MAX);
         if (e != cudaSuccess) return e;
         attr_set[dev] = true;
     }
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3((unsigned)((grid + 1) & ~1));   // whole pairs
     cfg.blockDim = dim3(GM_THREADS);
-    cfg.dynamicSmemBytes = GM_SMEM_BYTES;
+    cfg.dynamicSmemBytes = gm_smem_bytes(a.epi);
     cfg.stream = s;
     cudaLaunchAttribute attr[1];
     attr[0].id = cudaLaunchAttributeClusterDimension;

@@ -78,12 +78,19 @@ cudaError_t launch_permute(const int32_t* idx, int64_t n_slots, int k, int E, in
 cudaError_t launch_tile_table(const int32_t* offsets, int G, int bm, int4* tiles,
                               int32_t* n_tiles, cudaStream_t s);
 
+// Band-ordered work items for the down-projection (see item_order_kernel).
+constexpr int ITEM_MAX_BANDS = 16;
+constexpr int ITEM_MAX_TILES = 24576;   // m-tiles one ordering pass holds in shared memory
+cudaError_t launch_item_order(const int4* tiles, const int32_t* n_tiles, const int32_t* row_tok,
+                              int64_t T, int nb, int n_ntiles, int gsz, int BN, int max_tiles,
+                              int4* items, int32_t* n_items, cudaStream_t s);
+
 // ----------------------------------------------------------- grouped GEMM
 
 constexpr int GM_BM = 256;        // rows per m-tile: one CTA pair, 128 rows per CTA
 constexpr int GM_HALF = 128;      // rows per CTA (tcgen05 M = 256 across the pair)
 constexpr int GM_BK = 64;         // K per stage: 64 bf16 = one 128-byte swizzle row
-constexpr int GM_STAGES = 7;
+constexpr int GM_STAGES_MAX = 7;   // operand ring depth (6 when the reduction staging is needed)
 constexpr int GM_MAXBN = 256;     // largest N of one tcgen05.mma
 constexpr int GM_EPI_WARPS = 8;   // two warps per TMEM lane quadrant, alternate 32-column chunks
 constexpr int GM_WARP_MMA = GM_EPI_WARPS;        // TMEM allocation + tcgen05.mma issue
@@ -93,9 +100,17 @@ constexpr int GM_WARP_FWD = GM_EPI_WARPS + 6;    // publishes gathered stages
 constexpr int GM_THREADS = (GM_EPI_WARPS + 7) * 32;
 constexpr int GM_A_BYTES = GM_HALF * GM_BK * 2;           // one CTA's A rows per stage
 constexpr int GM_B_BYTES = GM_BK * (GM_MAXBN / 2) * 2;    // one CTA's half of B per stage
-// stages, 1 KB to align them, barriers / TMEM slot / flags / signal sink
-constexpr int GM_SMEM_BYTES = GM_STAGES * (GM_A_BYTES + GM_B_BYTES) + 1024 + 512;
-static_assert(GM_SMEM_BYTES <= 232448, "shared memory of one CTA");
+constexpr int GM_STG_ROWS = 16;    // rows per warp in the reduction staging buffer
+constexpr int GM_STG_LD = 36;      // floats per staged row: 32 values, the row's y offset, pad
+constexpr int GM_STG_BYTES = GM_EPI_WARPS * GM_STG_ROWS * GM_STG_LD * 4;
+constexpr int GM_OVERHEAD_BYTES = 1024 + 512;   // alignment, barriers / TMEM slot / flags / sink
+__host__ __device__ constexpr int gm_stages(int epi) { return epi == 2 /* EPI_ADD_F32 */ ? 6 : 7; }
+__host__ __device__ constexpr int gm_smem_bytes(int epi) {
+    return gm_stages(epi) * (GM_A_BYTES + GM_B_BYTES) + (epi == 2 ? GM_STG_BYTES : 0) + GM_OVERHEAD_BYTES;
+}
+constexpr int GM_SMEM_BYTES_MAX = GM_STAGES_MAX * (GM_A_BYTES + GM_B_BYTES) + GM_OVERHEAD_BYTES;
+static_assert(GM_SMEM_BYTES_MAX <= 232448 && gm_smem_bytes(2) <= 232448, "shared memory of one CTA");
+static_assert(3 * GM_STAGES_MAX + 5 <= 32, "barriers fit before the signal sink at +256 bytes");
 
 inline int64_t max_mtiles(int64_t rows, int64_t groups) { return (rows + GM_BM - 1) / GM_BM + groups; }
 
@@ -105,6 +120,7 @@ enum Epilogue : int {
     EPI_ADD_F32 = 2,     // yacc[tok(r), n] += scale(r) * acc   (vector atomics)
     EPI_STORE_F32 = 3,   // yacc[tok(r), n]  = scale(r) * acc
 };
+static_assert(EPI_ADD_F32 == 2, "gm_stages / gm_smem_bytes test the reduction epilogue by value");
 
 struct GemmArgs {
     CUtensorMap tmB;            // B = weights [G][K][N] bf16 (N contiguous), 3-D map {N, K, G}
@@ -117,7 +133,9 @@ struct GemmArgs {
     int a_kperiod;              // 0, or a multiple of 64: column of K index kk in A is kk % a_kperiod
     int64_t a_nrows;            // rows of A; a gathered row outside [0, a_nrows) is a device error
     int64_t m_total;            // GEMM rows that may be written
-    const int4* tiles;          // m-tile table {g, row0, nrows, 0}; nullptr: one dense group
+    const int4* tiles;          // m-tile table {g, row0, nrows, 0}; nullptr: one dense group;
+                                // with item_table: work items {g, row0, nrows, n0}
+    int item_table;             // tiles lists (m-tile, n-tile) items; *n_tiles_dev counts items
     const int32_t* n_tiles_dev; // number of entries of `tiles`
     int64_t max_mtiles;         // host bound on *n_tiles_dev
     int G, K, N, BN, n_ntiles, num_kb, nbox;

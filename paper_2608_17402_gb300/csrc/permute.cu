@@ -226,6 +226,85 @@ __global__ void __launch_bounds__(1024) tile_table_kernel(const int32_t* __restr
     if (g == 0) *n_tiles = s_total;
 }
 
+// One CTA of 1024 threads.  Orders the (m-tile, n-tile) work items of a grouped GEMM
+// in nb token bands x column groups of gsz n-tiles: band b holds the m-tiles whose
+// middle row's token lies in [b T / nb, (b + 1) T / nb) (expert-major order kept
+// inside a band).  Items run band-major, then column group, then m-tile, then n-tile,
+// so the rows of y that the running items accumulate into stay within one band and
+// one column group, a block small enough to stay in L2.
+// items[i] = {expert, first row, rows, first column}; *n_items = m-tiles x n_ntiles.
+__global__ void __launch_bounds__(1024) item_order_kernel(
+    const int4* __restrict__ tiles, const int32_t* __restrict__ n_tiles_dev,
+    const int32_t* __restrict__ row_tok, int64_t T, int nb, int n_ntiles, int gsz, int BN,
+    int max_tiles, int4* __restrict__ items, int32_t* __restrict__ n_items) {
+    extern __shared__ int32_t io_smem[];
+    int32_t* band = io_smem;                 // [max_tiles]
+    int32_t* rank = io_smem + max_tiles;     // [max_tiles]
+    __shared__ int s_cnt[ITEM_MAX_BANDS + 1];
+    int nt = *n_tiles_dev;
+    if (nt < 0 || nt > max_tiles) nt = 0;    // the GEMM reports an inconsistent table
+    for (int i = threadIdx.x; i < nt; i += blockDim.x) {
+        const int4 t = tiles[i];
+        const int64_t tok = t.z > 0 ? row_tok[t.y + t.z / 2] : 0;
+        const int64_t b = tok * nb / (T > 0 ? T : 1);
+        band[i] = b < 0 ? 0 : (b >= nb ? nb - 1 : (int)b);
+    }
+    __syncthreads();
+    // stable rank of each m-tile inside its band, 1024 tiles per pass: warp-level ranks
+    // (match_any), then a running prefix over warps per band
+    __shared__ int s_wcnt[32][ITEM_MAX_BANDS];
+    __shared__ int s_carry[ITEM_MAX_BANDS];
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    if (threadIdx.x < ITEM_MAX_BANDS) s_carry[threadIdx.x] = 0;
+    for (int i0 = 0; i0 < nt; i0 += blockDim.x) {
+        for (int q = threadIdx.x; q < 32 * ITEM_MAX_BANDS; q += blockDim.x) (&s_wcnt[0][0])[q] = 0;
+        __syncthreads();
+        const int i = i0 + threadIdx.x;
+        const int b = i < nt ? band[i] : -1;
+        const uint32_t m = __match_any_sync(0xffffffffu, b);
+        const int lrank = __popc(m & ((1u << lane) - 1u));
+        if (b >= 0 && lrank == 0) s_wcnt[warp][b] = __popc(m);
+        __syncthreads();
+        if (threadIdx.x < nb) {
+            int run = s_carry[threadIdx.x];
+            for (int w = 0; w < 32; ++w) {
+                const int c = s_wcnt[w][threadIdx.x];
+                s_wcnt[w][threadIdx.x] = run;
+                run += c;
+            }
+            s_carry[threadIdx.x] = run;
+        }
+        __syncthreads();
+        if (b >= 0) rank[i] = s_wcnt[warp][b] + lrank;
+        __syncthreads();
+    }
+    if (threadIdx.x < nb) s_cnt[threadIdx.x] = s_carry[threadIdx.x];
+    __syncthreads();
+    if (threadIdx.x == 0) {   // exclusive prefix of the band sizes
+        int run = 0;
+        for (int b = 0; b < nb; ++b) {
+            const int c = s_cnt[b];
+            s_cnt[b] = run;
+            run += c;
+        }
+        s_cnt[nb] = run;
+        *n_items = run * n_ntiles;
+    }
+    __syncthreads();
+    for (int i = threadIdx.x; i < nt; i += blockDim.x) {
+        const int4 t = tiles[i];
+        const int b = band[i];
+        const int cnt_b = s_cnt[b + 1] - s_cnt[b];
+        for (int j = 0; j < n_ntiles; ++j) {
+            const int c = j / gsz, jl = j - c * gsz;
+            const int in_group = min(gsz, n_ntiles - c * gsz);
+            const int64_t pos = (int64_t)s_cnt[b] * n_ntiles + (int64_t)cnt_b * (c * gsz) +
+                                (int64_t)rank[i] * in_group + jl;
+            items[pos] = make_int4(t.x, t.y, t.z, j * BN);
+        }
+    }
+}
+
 }  // namespace
 
 // Scratch of moevie_permute_static: fixed size, so that entry point needs neither a
@@ -285,6 +364,28 @@ cudaError_t launch_permute(const int32_t* idx, int64_t n_slots, int k, int E, in
     perm_scatter_kernel<<<nchunks, PT, smem, s>>>(idx, n_slots, k, E, chunk, hist, offsets,
                                                   gate_flat, perm, inv, row_tok, row_gate);
     count_launches(4);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_item_order(const int4* tiles, const int32_t* n_tiles, const int32_t* row_tok,
+                              int64_t T, int nb, int n_ntiles, int gsz, int BN, int max_tiles,
+                              int4* items, int32_t* n_items, cudaStream_t s) {
+    if (nb < 1 || nb > ITEM_MAX_BANDS || max_tiles > ITEM_MAX_TILES || gsz < 1)
+        return cudaErrorInvalidValue;
+    const size_t smem = (size_t)2 * max_tiles * sizeof(int32_t);
+    static bool attr_set[64] = {};
+    int dev = 0;
+    cudaGetDevice(&dev);
+    if (dev >= 0 && dev < 64 && !attr_set[dev]) {
+        cudaError_t err = cudaFuncSetAttribute(item_order_kernel,
+                                               cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                               2 * ITEM_MAX_TILES * (int)sizeof(int32_t));
+        if (err != cudaSuccess) return err;
+        attr_set[dev] = true;
+    }
+    item_order_kernel<<<1, 1024, smem, s>>>(tiles, n_tiles, row_tok, T, nb, n_ntiles, gsz, BN,
+                                            max_tiles, items, n_items);
+    count_launches(1);
     return cudaGetLastError();
 }
 
