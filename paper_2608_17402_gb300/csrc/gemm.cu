@@ -24,17 +24,17 @@
 // permute step (no host read of segment sizes), or, for one dense group, from
 // arithmetic.
 //
-// Warp roles (480 threads per CTA, one CTA per SM):
+// Warp roles (608 threads per CTA, one CTA per SM):
 //   warps 0-7   epilogue: tcgen05.ld of the CTA's 128 accumulator rows (warp w:
 //               TMEM lanes 32 (w%4)..+31, every other 32-column chunk), fused math,
 //               and 16-byte stores / reductions of each thread's own row
 //   warp 8      TMEM allocation (both CTAs, jointly); leader lane 0 issues the MMAs
 //   warp 9      lane 0: TMA loads of the B half and, for contiguous A rows, of A;
 //               the leader posts the byte count of both CTAs on its full barrier
-//   warps 10-13 token gather: 16-byte cp.async of A rows straight into the 128-byte
+//   warps 10-17 token gather: 16-byte cp.async of A rows straight into the 128-byte
 //               swizzled K-major layout; each thread hands the completion of its
 //               copies to the stage's local afull barrier and moves on
-//   warp 14     lane 0: waits for afull, fences the stage to the async proxy and
+//   warp 18     lane 0: waits for afull, fences the stage to the async proxy and
 //               publishes it on the leader's full barrier (from the peer: a 16-byte
 //               bulk copy that completes transaction bytes there)
 // Shared memory: 7 stages (6 plus a reduction staging buffer for the y-accumulator
@@ -284,20 +284,21 @@ __device__ void producer_tma(const GemmArgs& p, const Smem& sm, int64_t n_work,
     }
 }
 
-// A row pointers of this thread's 8 rows (r = rb + 16 j of the CTA's half).
+// A row pointers of this thread's GM_GATHER_ROWS rows (r = rb + GM_GATHER_RSTEP j of the
+// CTA's half).
 __device__ __forceinline__ void gather_rows(const GemmArgs& p, const Tile& t, uint32_t rank,
-                                            int rb, const __nv_bfloat16* (&src)[8]) {
+                                            int rb, const __nv_bfloat16* (&src)[GM_GATHER_ROWS]) {
     const int nh = rows_half(t, rank);
-    int idx[8];
+    int idx[GM_GATHER_ROWS];
 #pragma unroll
-    for (int j = 0; j < 8; ++j) {
-        const int r = rb + 16 * j;
+    for (int j = 0; j < GM_GATHER_ROWS; ++j) {
+        const int r = rb + GM_GATHER_RSTEP * j;
         const int gr = t.row0 + (int)rank * GM_HALF + r;
         idx[j] = (r < nh) ? __ldg(p.a_rows + gr) / p.a_div : -1;
     }
 #pragma unroll
-    for (int j = 0; j < 8; ++j) {
-        const int r = rb + 16 * j;
+    for (int j = 0; j < GM_GATHER_ROWS; ++j) {
+        const int r = rb + GM_GATHER_RSTEP * j;
         if (r < nh && idx[j] >= 0 && idx[j] < p.a_nrows) {
             src[j] = p.A + (int64_t)idx[j] * p.lda;
         } else {
@@ -309,20 +310,20 @@ __device__ __forceinline__ void gather_rows(const GemmArgs& p, const Tile& t, ui
     }
 }
 
-// Token gather (warps 10-13): each thread copies 8 16-byte chunks per stage straight
+// Token gather (GM_GATHER_WARPS warps): each thread copies GM_GATHER_ROWS 16-byte chunks per stage straight
 // into the 128-byte swizzled K-major layout, then hands the completion of its copies
 // to the stage's afull barrier (cp.async.mbarrier.arrive.noinc) and moves on without
 // waiting; gather_forwarder publishes the stage once all 128 threads' copies landed.
 __device__ void producer_gather(const GemmArgs& p, const Smem& sm, int64_t n_work,
                                 volatile int* abort_flag) {
-    const int pt = threadIdx.x - GM_WARP_GATHER * 32;   // 0..127
+    const int pt = threadIdx.x - GM_WARP_GATHER * 32;   // 0 .. GM_GATHER_WARPS * 32 - 1
     const int lane = threadIdx.x & 31;
     const int c = pt & 7, rb = pt >> 3;                  // 16-byte chunk, first row
     int s = 0;
     uint32_t ph = 0;
     bool ok = true;
     int64_t w = sm.pair;
-    const __nv_bfloat16* src[8];
+    const __nv_bfloat16* src[GM_GATHER_ROWS];
     Tile t{};
     if (w < n_work) {
         t = decode_tile(p, w);
@@ -330,7 +331,7 @@ __device__ void producer_gather(const GemmArgs& p, const Smem& sm, int64_t n_wor
     }
     for (; w < n_work && ok; w += sm.npairs) {
         const int64_t wn = w + sm.npairs;
-        const __nv_bfloat16* nsrc[8];
+        const __nv_bfloat16* nsrc[GM_GATHER_ROWS];
         Tile tn{};
         if (wn < n_work) {
             tn = decode_tile(p, wn);
@@ -349,8 +350,8 @@ __device__ void producer_gather(const GemmArgs& p, const Smem& sm, int64_t n_wor
             const int kk = kb * GM_BK + c * 8;
             const bool col_ok = kk < p.K;
 #pragma unroll
-            for (int j = 0; j < 8; ++j) {
-                const int r = rb + 16 * j;
+            for (int j = 0; j < GM_GATHER_ROWS; ++j) {
+                const int r = rb + GM_GATHER_RSTEP * j;
                 const uint32_t dst = dst0 + r * 128 + ((c ^ (r & 7)) << 4);
                 const bool v = col_ok && src[j] != nullptr;
                 cp_async16(dst, v ? (const void*)(src[j] + kk) : (const void*)p.A, v ? 16u : 0u);
@@ -363,7 +364,7 @@ __device__ void producer_gather(const GemmArgs& p, const Smem& sm, int64_t n_wor
         }
         if (wn < n_work) {
 #pragma unroll
-            for (int j = 0; j < 8; ++j) src[j] = nsrc[j];
+            for (int j = 0; j < GM_GATHER_ROWS; ++j) src[j] = nsrc[j];
         }
         t = tn;
     }
@@ -630,7 +631,7 @@ __global__ void __launch_bounds__(GM_THREADS, 1) grouped_gemm_kernel(const __gri
             // are transaction bytes)
             mbar_init(sm.full + 8 * s, 1 + (gather ? 1 : 0));
             mbar_init(sm.empty + 8 * s, 1);         // multicast tcgen05.commit
-            mbar_init(sm.afull + 8 * s, 128);       // this CTA's gather threads (async arrivals)
+            mbar_init(sm.afull + 8 * s, GM_GATHER_WARPS * 32);   // gather threads (async arrivals)
         }
         for (int a = 0; a < 2; ++a) {
             mbar_init(sm.tfull + 8 * a, 1);         // multicast tcgen05.commit

@@ -95,9 +95,14 @@ constexpr int GM_MAXBN = 256;     // largest N of one tcgen05.mma
 constexpr int GM_EPI_WARPS = 8;   // two warps per TMEM lane quadrant, alternate 32-column chunks
 constexpr int GM_WARP_MMA = GM_EPI_WARPS;        // TMEM allocation + tcgen05.mma issue
 constexpr int GM_WARP_LOAD = GM_EPI_WARPS + 1;   // TMA loads of B (and of contiguous A)
-constexpr int GM_WARP_GATHER = GM_EPI_WARPS + 2; // first of 4 token-gather warps
-constexpr int GM_WARP_FWD = GM_EPI_WARPS + 6;    // publishes gathered stages
-constexpr int GM_THREADS = (GM_EPI_WARPS + 7) * 32;
+constexpr int GM_GATHER_WARPS = 8;               // token-gather warps
+constexpr int GM_WARP_GATHER = GM_EPI_WARPS + 2; // first token-gather warp
+constexpr int GM_WARP_FWD = GM_WARP_GATHER + GM_GATHER_WARPS;   // publishes gathered stages
+constexpr int GM_THREADS = (GM_WARP_FWD + 1) * 32;
+// Each gather thread copies one 16-byte chunk of GM_GATHER_ROWS rows per stage, rows
+// GM_GATHER_RSTEP apart (8 threads cover a row's 128 bytes).
+constexpr int GM_GATHER_RSTEP = GM_GATHER_WARPS * 32 / 8;
+constexpr int GM_GATHER_ROWS = 128 / GM_GATHER_RSTEP;
 constexpr int GM_A_BYTES = GM_HALF * GM_BK * 2;           // one CTA's A rows per stage
 constexpr int GM_B_BYTES = GM_BK * (GM_MAXBN / 2) * 2;    // one CTA's half of B per stage
 constexpr int GM_STG_ROWS = 16;    // rows per warp in the reduction staging buffer
