@@ -310,10 +310,11 @@ __device__ __forceinline__ void gather_rows(const GemmArgs& p, const Tile& t, ui
     }
 }
 
-// Token gather (GM_GATHER_WARPS warps): each thread copies GM_GATHER_ROWS 16-byte chunks per stage straight
-// into the 128-byte swizzled K-major layout, then hands the completion of its copies
-// to the stage's afull barrier (cp.async.mbarrier.arrive.noinc) and moves on without
-// waiting; gather_forwarder publishes the stage once all 128 threads' copies landed.
+// Token gather (GM_GATHER_WARPS warps): each thread copies one 16-byte chunk of
+// GM_GATHER_ROWS rows per stage straight into the 128-byte swizzled K-major layout,
+// then hands the completion of its copies to the stage's afull barrier
+// (cp.async.mbarrier.arrive.noinc) and moves on without waiting; gather_forwarder
+// publishes the stage once every gather thread's copies have landed.
 __device__ void producer_gather(const GemmArgs& p, const Smem& sm, int64_t n_work,
                                 volatile int* abort_flag) {
     const int pt = threadIdx.x - GM_WARP_GATHER * 32;   // 0 .. GM_GATHER_WARPS * 32 - 1
