@@ -207,7 +207,7 @@ moevie_status route_impl(const void* x, const float* W_r, const float* b, int64_
     // partial logits: ksplit arrays [T][Ep]; straight into logits_out when unsplit
     float* logits = (logits_out && ksplit == 1) ? logits_out : at<float>(ws, L.logits);
     const int64_t part_stride = T * Ep;
-    MV_TRY(launch_route_split(W_r, (int)d, (int)E, wsplit, wrt, at<float>(ws, L.wpart), wnorm, s));
+    MV_TRY(launch_route_split(W_r, (int)d, (int)E, wsplit, wrt, at<float>(ws, L.wpart), wnorm, st, s));
     const int64_t dp = route_dpad((int)d);
     GemmSpec g{};
     g.A = x;

@@ -30,10 +30,10 @@ inline int route_dpad(int d) { return (d + 63) / 64 * 64; }
 // W_r fp32 [d, E] -> three bf16 pieces [3][d_pad][E_pad] with W_r = hi + mid + lo
 // exactly (zero in the padding rows and columns), the transposed fp32 copy
 // wrt [E][d_pad] (zero rows past d), and |W_r[:, e]| (wpart: route_split_parts(d) x
-// E_pad floats of scratch).
+// E_pad floats of scratch).  Also clears the fallback counter in st (may be NULL).
 int route_split_parts(int d);
 cudaError_t launch_route_split(const float* Wr, int d, int E, __nv_bfloat16* Wsplit, float* wrt,
-                               float* wpart, float* wnorm, cudaStream_t s);
+                               float* wpart, float* wnorm, DevStatus* st, cudaStream_t s);
 
 // Splits of K for the router GEMM: enough CTA-pair work items for about
 // ROUTE_SPLIT_TARGET items, at most ROUTE_MAX_KSPLIT, at least three K blocks each.

@@ -43,7 +43,8 @@ __global__ void __launch_bounds__(256) route_split_kernel(const float* __restric
                                                           int dp, int E, int Ep,
                                                           __nv_bfloat16* __restrict__ Wsplit,
                                                           float* __restrict__ wrt,
-                                                          float* __restrict__ wpart) {
+                                                          float* __restrict__ wpart, DevStatus* st) {
+    if (st && blockIdx.x == 0 && blockIdx.y == 0 && threadIdx.x == 0) st->fb_count = 0;
     __shared__ float tile[SPLIT_TILE][SPLIT_TILE + 1];
     __shared__ float red[8][32];
     const int tx = threadIdx.x & 31, ty = threadIdx.x >> 5;
@@ -153,22 +154,6 @@ __device__ __forceinline__ float row_norm(const __nv_bfloat16* xt, int d, int la
     }
     for (; c < nc; c += 32) acc += sq_bf16x8(v[c]);
     return sqrtf(warp_sum(acc));
-}
-
-// Order-preserving code of (key, id): larger key first, then the lower id.
-__device__ __forceinline__ uint64_t key_code(float key, int e) {
-    uint32_t u = __float_as_uint(key);
-    u ^= (u & 0x80000000u) ? 0xffffffffu : 0x80000000u;
-    return ((uint64_t)u << 32) | (uint32_t)(0xffffffffu - (uint32_t)e);
-}
-
-__device__ __forceinline__ uint64_t warp_max_u64(uint64_t v) {
-#pragma unroll
-    for (int o = 16; o; o >>= 1) {
-        const uint64_t u = __shfl_xor_sync(0xffffffffu, v, o);
-        v = u > v ? u : v;
-    }
-    return v;
 }
 
 // Order-preserving code of a float (larger float, larger code; no NaNs here).
@@ -288,35 +273,40 @@ __global__ void __launch_bounds__(256) route_topk_kernel(
     }
 }
 
-// k-th and (k+1)-th largest of v over the warp (k rounds of arg-max; k <= E).
+__device__ __forceinline__ float from_ord_f32(uint32_t c) {
+    return __uint_as_float(c ^ ((c & 0x80000000u) ? 0x80000000u : 0xffffffffu));
+}
+
+// k-th and (k+1)-th largest of v over the warp, counting equal values separately
+// (k or k + 1 rounds: warp maximum of the order codes by redux.sync, then one holder
+// of that maximum leaves; k <= E).
 template <int NPL>
 __device__ __forceinline__ void warp_kth_values(const float (&v)[NPL], int E, int k, int lane,
                                                 float& kth, float& kth1) {
-    uint64_t code[NPL];
+    uint32_t code[NPL];
 #pragma unroll
-    for (int i = 0; i < NPL; ++i) {
-        const int e = lane + 32 * i;
-        code[i] = e < E ? key_code(v[i], e) : 0ull;
-    }
+    for (int i = 0; i < NPL; ++i) code[i] = (lane + 32 * i < E) ? ord_f32(v[i]) : 0u;
     uint32_t used = 0;
     kth = -INFINITY;
     kth1 = -INFINITY;
     const int rounds = k < E ? k + 1 : k;
     for (int j = 0; j < rounds; ++j) {
-        uint64_t best = 0;
+        uint32_t best = 0;
 #pragma unroll
         for (int i = 0; i < NPL; ++i) {
-            const uint64_t c = ((used >> i) & 1u) ? 0ull : code[i];
+            const uint32_t c = ((used >> i) & 1u) ? 0u : code[i];
             best = c > best ? c : best;
         }
-        best = warp_max_u64(best);
-        const int bi = (int)(0xffffffffu - (uint32_t)best);
-        float bv = 0.f;
+        best = __reduce_max_sync(0xffffffffu, best);
 #pragma unroll
-        for (int i = 0; i < NPL; ++i)
-            if (lane + 32 * i == bi) bv = v[i];
-        bv = __shfl_sync(0xffffffffu, bv, bi & 31);
-        if ((bi & 31) == lane) used |= 1u << (bi >> 5);
+        for (int i = 0; i < NPL; ++i) {
+            const uint32_t m = __ballot_sync(0xffffffffu, !((used >> i) & 1u) && code[i] == best);
+            if (m) {
+                if (lane == __ffs(m) - 1) used |= 1u << i;
+                break;
+            }
+        }
+        const float bv = from_ord_f32(best);
         if (j == k - 1) kth = bv;
         if (j == k) kth1 = bv;
     }
@@ -424,10 +414,13 @@ __global__ void __launch_bounds__(256) route_fallback_kernel(
             double v = acc0 + acc1;
 #pragma unroll
             for (int o = 16; o; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
-            if (lane == 0) s_key[c] = 1.0 / (1.0 + exp(-v)) + (double)b[e];
+            if (lane == 0) s_key[c] = v;   // exact logit; its key is formed below
         }
         __syncthreads();
         if (warp == 0 && nc >= 0) {
+            // keys of all candidates at once, one per lane (fp64 is slow: run it in parallel)
+            for (int c = lane; c < nc; c += 32) s_key[c] = 1.0 / (1.0 + exp(-s_key[c])) + (double)b[s_cand[c]];
+            __syncwarp();
             double exk[NPL];
             int base = 0;
 #pragma unroll
@@ -485,8 +478,6 @@ __global__ void __launch_bounds__(256) route_fallback_kernel(
     }
 }
 
-__global__ void reset_fallback_count(DevStatus* st) { st->fb_count = 0; }
-
 // out[t, e] = sum of the nparts partial logits, in order (used for inspection).
 __global__ void route_sum_parts_kernel(const float* __restrict__ s, int64_t part_stride,
                                        int nparts, int64_t n, float* __restrict__ out) {
@@ -522,11 +513,11 @@ int64_t route_logits_rows(int64_t T, int d, int E) {
 }
 
 cudaError_t launch_route_split(const float* Wr, int d, int E, __nv_bfloat16* Wsplit, float* wrt,
-                               float* wpart, float* wnorm, cudaStream_t s) {
+                               float* wpart, float* wnorm, DevStatus* st, cudaStream_t s) {
     const int Ep = route_epad(E);
     const int parts = route_split_parts(d);
     route_split_kernel<<<dim3((Ep + SPLIT_TILE - 1) / SPLIT_TILE, parts), 256, 0, s>>>(
-        Wr, d, route_dpad(d), E, Ep, Wsplit, wrt, wpart);
+        Wr, d, route_dpad(d), E, Ep, Wsplit, wrt, wpart, st);
     route_wnorm_kernel<<<(E + 7) / 8, 256, 0, s>>>(wpart, parts, E, Ep, wnorm);
     count_launches(2);
     return cudaGetLastError();
@@ -545,7 +536,6 @@ cudaError_t launch_route_select(const __nv_bfloat16* x, const float* wrt, const 
                                 const float* wnorm, int T, int d, int E, int k, int32_t* idx,
                                 float* gate, int32_t* fb_tokens, float* xnorm, DevStatus* st,
                                 int num_sms, cudaStream_t s) {
-    reset_fallback_count<<<1, 1, 0, s>>>(st);
     const int blocks = (int)(((int64_t)T * 32 + 255) / 256);
     const int fb_blocks = T < 4 * num_sms ? T : 4 * num_sms;
     const int npl = (E + 31) / 32;
@@ -566,7 +556,7 @@ cudaError_t launch_route_select(const __nv_bfloat16* x, const float* wrt, const 
     else if (npl <= 16) MV_ROUTE(16);
     else MV_ROUTE(32);
 #undef MV_ROUTE
-    count_launches(3);
+    count_launches(2);
     return cudaGetLastError();
 }
 
