@@ -320,6 +320,8 @@ __device__ void producer_gather(const GemmArgs& p, const Smem& sm, int64_t n_wor
     const int pt = threadIdx.x - GM_WARP_GATHER * 32;   // 0 .. GM_GATHER_WARPS * 32 - 1
     const int lane = threadIdx.x & 31;
     const int c = pt & 7, rb = pt >> 3;                  // 16-byte chunk, first row
+    // gathered rows are re-read by every expert of their tokens: keep them in L2
+    const uint64_t keep_pol = l2_policy_evict_last();
     int s = 0;
     uint32_t ph = 0;
     bool ok = true;
@@ -355,7 +357,8 @@ __device__ void producer_gather(const GemmArgs& p, const Smem& sm, int64_t n_wor
                 const int r = rb + GM_GATHER_RSTEP * j;
                 const uint32_t dst = dst0 + r * 128 + ((c ^ (r & 7)) << 4);
                 const bool v = col_ok && src[j] != nullptr;
-                cp_async16(dst, v ? (const void*)(src[j] + kk) : (const void*)p.A, v ? 16u : 0u);
+                cp_async16_hint(dst, v ? (const void*)(src[j] + kk) : (const void*)p.A, v ? 16u : 0u,
+                                keep_pol);
             }
             cp_async_arrive_noinc(sm.afull + 8 * s);
             if (++s == sm.nstages) {
@@ -482,6 +485,8 @@ __device__ void epilogue(const GemmArgs& p, const Smem& sm, uint32_t tmem, int64
     const int quad = warp & 3, half = warp >> 2;
     const bool to_f32 = (p.epi == EPI_ADD_F32 || p.epi == EPI_STORE_F32);
     const int nchunk = p.BN / 32;
+    // bf16 results are written once and read back later: let them leave L2 first
+    const uint64_t stream_pol = l2_policy_evict_first();
     const uint32_t tempty_leader = peer_addr(sm.tempty, 0);
     int it = 0;
     for (int64_t w = sm.pair; w < n_work; w += sm.npairs, ++it) {
@@ -579,7 +584,7 @@ __device__ void epilogue(const GemmArgs& p, const Smem& sm, uint32_t tmem, int64
                     u.y = pack_bf16x2(f[2], f[3]);
                     u.z = pack_bf16x2(f[4], f[5]);
                     u.w = pack_bf16x2(f[6], f[7]);
-                    *reinterpret_cast<uint4*>(orow + 8 * g8) = u;
+                    st_global_v4_hint(orow + 8 * g8, u, stream_pol);
                 }
             } else {
                 float* yrow = p.yacc + t.ks * p.y_split_stride + tok * p.ldy + n;
