@@ -14,6 +14,8 @@
 //                       (warp match + per-warp running counts), and writes perm,
 //                       inv and the per-row token (pos // K) and gate.
 // Inside one expert's segment, rows keep ascending slot order t*k + j.
+#include <cooperative_groups.h>
+
 #include <mutex>
 
 #include "internal.h"
@@ -27,14 +29,14 @@ constexpr int PW = PT / 32;                  // warps per CTA
 
 __device__ __forceinline__ bool valid_id(int e, int E) { return e >= 0 && e < E; }
 
-__global__ void __launch_bounds__(PT) perm_hist_kernel(const int32_t* __restrict__ idx,
-                                                       int64_t n, int E, int chunk,
-                                                       int32_t* __restrict__ hist,
-                                                       DevStatus* st) {
-    extern __shared__ int32_t cnt[];
+// Histogram of chunk b (of nchunks) into hist[e][b]; cnt: E ints of shared memory.
+__device__ __forceinline__ void perm_hist_body(const int32_t* __restrict__ idx, int64_t n, int E,
+                                               int chunk, int b, int nchunks,
+                                               int32_t* __restrict__ hist, DevStatus* st,
+                                               int32_t* cnt) {
     for (int e = threadIdx.x; e < E; e += PT) cnt[e] = 0;
     __syncthreads();
-    const int64_t c0 = (int64_t)blockIdx.x * chunk;
+    const int64_t c0 = (int64_t)b * chunk;
     const int64_t c1 = c0 + chunk < n ? c0 + chunk : n;
     const int64_t nvec = (c1 - c0) >> 2;
     const int4* v = reinterpret_cast<const int4*>(idx + c0);   // c0 % 4 == 0, idx 16-B aligned
@@ -53,10 +55,18 @@ __global__ void __launch_bounds__(PT) perm_hist_kernel(const int32_t* __restrict
         else report(st, MOEVIE_ERR_DEVICE, SITE_PERMUTE_ID, (int)i, e);
     }
     __syncthreads();
-    for (int e = threadIdx.x; e < E; e += PT) hist[(int64_t)e * gridDim.x + blockIdx.x] = cnt[e];
+    for (int e = threadIdx.x; e < E; e += PT) hist[(int64_t)e * nchunks + b] = cnt[e];
 }
 
-// Exclusive scan of one int per thread over a 1024-thread block.
+__global__ void __launch_bounds__(PT) perm_hist_kernel(const int32_t* __restrict__ idx,
+                                                       int64_t n, int E, int chunk,
+                                                       int32_t* __restrict__ hist,
+                                                       DevStatus* st) {
+    extern __shared__ int32_t cnt[];
+    perm_hist_body(idx, n, E, chunk, blockIdx.x, gridDim.x, hist, st, cnt);
+}
+
+// Exclusive scan of one int per thread over the block (up to 1024 threads).
 __device__ int block_exclusive_scan_1024(int v, int* total) {
     __shared__ int wsum[32];
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
@@ -69,7 +79,7 @@ __device__ int block_exclusive_scan_1024(int v, int* total) {
     if (lane == 31) wsum[warp] = inc;
     __syncthreads();
     if (warp == 0) {
-        const int w = wsum[lane];
+        const int w = lane < (int)(blockDim.x >> 5) ? wsum[lane] : 0;
         int wi = w;
 #pragma unroll
         for (int o = 1; o < 32; o <<= 1) {
@@ -88,17 +98,13 @@ __device__ int block_exclusive_scan_1024(int v, int* total) {
 // One warp per expert: hist[e][0 .. nchunks) becomes its exclusive prefix (the first
 // row of expert e inside each chunk, relative to the expert's segment); counts[e] is
 // the total.  Coalesced: lanes over consecutive chunks.
-__global__ void __launch_bounds__(256) perm_chunk_scan_kernel(int32_t* __restrict__ hist,
-                                                              int nchunks, int E,
-                                                              int32_t* __restrict__ counts) {
-    const int lane = threadIdx.x & 31;
-    const int e = (int)(((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5);
-    if (e >= E) return;
+__device__ __forceinline__ void perm_chunk_scan_warp(int32_t* __restrict__ hist, int nchunks, int e,
+                                                     int lane, int32_t* __restrict__ counts) {
     int32_t* h = hist + (int64_t)e * nchunks;
     int running = 0;
     for (int c0 = 0; c0 < nchunks; c0 += 32) {
         const int c = c0 + lane;
-        const int v = c < nchunks ? h[c] : 0;
+        const int v = c < nchunks ? __ldcg(h + c) : 0;   // L2: written by other CTAs
         int inc = v;
 #pragma unroll
         for (int o = 1; o < 32; o <<= 1) {
@@ -109,6 +115,14 @@ __global__ void __launch_bounds__(256) perm_chunk_scan_kernel(int32_t* __restric
         running += __shfl_sync(0xffffffffu, inc, 31);
     }
     if (lane == 0) counts[e] = running;
+}
+
+__global__ void __launch_bounds__(256) perm_chunk_scan_kernel(int32_t* __restrict__ hist,
+                                                              int nchunks, int E,
+                                                              int32_t* __restrict__ counts) {
+    const int e = (int)(((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5);
+    if (e >= E) return;
+    perm_chunk_scan_warp(hist, nchunks, e, threadIdx.x & 31, counts);
 }
 
 // One CTA of 1024 threads (E <= 1024): exclusive offsets over experts, the number
@@ -143,18 +157,18 @@ __global__ void __launch_bounds__(1024) perm_offsets_kernel(const int32_t* __res
     }
 }
 
-// Dynamic smem: chunk ints (the chunk's ids) + PW * E ints (per-warp counts).
-__global__ void __launch_bounds__(PT) perm_scatter_kernel(
-    const int32_t* __restrict__ idx, int64_t n, int k, int E, int chunk,
-    const int32_t* __restrict__ base, const int32_t* __restrict__ offsets,
+// Scatter of chunk b: ps_smem holds chunk ints (the chunk's ids) + PW * E ints
+// (per-warp counts); offsets may live in global or shared memory.
+__device__ __forceinline__ void perm_scatter_body(
+    const int32_t* __restrict__ idx, int64_t n, int k, int E, int chunk, int b, int nchunks,
+    const int32_t* __restrict__ base, const int32_t* offsets,
     const float* __restrict__ gate_flat, int32_t* __restrict__ perm, int32_t* __restrict__ inv,
-    int32_t* __restrict__ row_tok, float* __restrict__ row_gate) {
-    extern __shared__ __align__(16) int32_t ps_smem[];
+    int32_t* __restrict__ row_tok, float* __restrict__ row_gate, int32_t* ps_smem) {
     int32_t* sidx = ps_smem;
     int32_t* wc = ps_smem + chunk;
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const int per_warp = chunk / PW;
-    const int64_t c0 = (int64_t)blockIdx.x * chunk;
+    const int64_t c0 = (int64_t)b * chunk;
     const int len = (int)(c0 + chunk < n ? chunk : n - c0);
     {
         const int nvec = len >> 2;
@@ -178,7 +192,7 @@ __global__ void __launch_bounds__(PT) perm_scatter_kernel(
     }
     __syncthreads();
     for (int e = tid; e < E; e += PT) {                  // pass 2: first row per (warp, e)
-        int run = offsets[e] + base[(int64_t)e * gridDim.x + blockIdx.x];
+        int run = offsets[e] + __ldcg(base + (int64_t)e * nchunks + b);   // L2: written by other CTAs
         for (int w = 0; w < PW; ++w) {
             const int c = wc[w * E + e];
             wc[w * E + e] = run;
@@ -209,6 +223,77 @@ __global__ void __launch_bounds__(PT) perm_scatter_kernel(
             }
         }
     }
+}
+
+__global__ void __launch_bounds__(PT) perm_scatter_kernel(
+    const int32_t* __restrict__ idx, int64_t n, int k, int E, int chunk,
+    const int32_t* __restrict__ base, const int32_t* __restrict__ offsets,
+    const float* __restrict__ gate_flat, int32_t* __restrict__ perm, int32_t* __restrict__ inv,
+    int32_t* __restrict__ row_tok, float* __restrict__ row_gate) {
+    extern __shared__ __align__(16) int32_t ps_smem[];
+    perm_scatter_body(idx, n, k, E, chunk, blockIdx.x, gridDim.x, base, offsets, gate_flat, perm, inv,
+                      row_tok, row_gate, ps_smem);
+}
+
+// The whole permute in one cooperative launch (one CTA per chunk, all resident):
+// histograms, grid sync, per-expert chunk scans (warps over experts), grid sync, then
+// every CTA forms the expert offsets in shared memory (CTA 0 also writes offsets,
+// the m-tile table and its size) and scatters its chunk.
+__global__ void __launch_bounds__(PT) perm_fused_kernel(
+    const int32_t* __restrict__ idx, int64_t n, int k, int E, int bm, int chunk,
+    const float* __restrict__ gate_flat, int32_t* __restrict__ hist, int32_t* __restrict__ counts,
+    int32_t* __restrict__ offsets, int4* __restrict__ tiles, int32_t* __restrict__ n_tiles,
+    int32_t* __restrict__ perm, int32_t* __restrict__ inv, int32_t* __restrict__ row_tok,
+    float* __restrict__ row_gate, DevStatus* st) {
+    namespace cg = cooperative_groups;
+    cg::grid_group grid = cg::this_grid();
+    extern __shared__ __align__(16) int32_t ps_smem[];
+    __shared__ int s_off[1024], s_tot;
+    const int nchunks = gridDim.x;
+    const int lane = threadIdx.x & 31;
+    perm_hist_body(idx, n, E, chunk, blockIdx.x, nchunks, hist, st, ps_smem);
+    grid.sync();
+    const int gw = (int)(((int64_t)blockIdx.x * PT + threadIdx.x) >> 5);
+    for (int e = gw; e < E; e += nchunks * PW) perm_chunk_scan_warp(hist, nchunks, e, lane, counts);
+    grid.sync();
+    // exclusive offsets over the E <= 1024 experts, four per thread
+    int loc[4], sum = 0;
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+        const int e = 4 * threadIdx.x + q;
+        loc[q] = e < E ? __ldcg(counts + e) : 0;
+        sum += loc[q];
+    }
+    int ex = block_exclusive_scan_1024(sum, &s_tot);
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+        const int e = 4 * threadIdx.x + q;
+        if (e < E) s_off[e] = ex;
+        ex += loc[q];
+    }
+    __syncthreads();
+    if (blockIdx.x == 0) {
+        for (int e = threadIdx.x; e < E; e += PT) offsets[e] = s_off[e];
+        if (threadIdx.x == 0) offsets[E] = s_tot;
+        int tl[4], tsum = 0;
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+            tl[q] = (loc[q] + bm - 1) / bm;
+            tsum += tl[q];
+        }
+        __shared__ int s_ttot;
+        int tex = block_exclusive_scan_1024(tsum, &s_ttot);
+        if (threadIdx.x == 0) *n_tiles = s_ttot;
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+            const int g = 4 * threadIdx.x + q;
+            for (int m = 0; m < tl[q]; ++m)
+                tiles[tex + m] = make_int4(g, s_off[g] + m * bm, min(bm, loc[q] - m * bm), 0);
+            tex += tl[q];
+        }
+    }
+    perm_scatter_body(idx, n, k, E, chunk, blockIdx.x, nchunks, hist, s_off, gate_flat, perm, inv,
+                      row_tok, row_gate, ps_smem);
 }
 
 // m-tile table from given offsets (one thread per group, E <= 1024).
@@ -344,23 +429,44 @@ cudaError_t launch_permute(const int32_t* idx, int64_t n_slots, int k, int E, in
                            int32_t* inv, int32_t* row_tok, float* row_gate, DevStatus* st,
                            cudaStream_t s) {
     const int nchunks = (int)((n_slots + chunk - 1) / chunk);
-    perm_hist_kernel<<<nchunks, PT, (size_t)E * 4, s>>>(idx, n_slots, E, chunk, hist, st);
-    cudaError_t err = cudaGetLastError();
+    const size_t smem = (size_t)(chunk + PW * E) * 4;
+    static bool attr_set[64] = {};
+    static int coop_ctas[64] = {};   // co-resident CTAs of perm_fused_kernel (0: no cooperative launch)
+    int dev = 0;
+    cudaError_t err = cudaGetDevice(&dev);
     if (err != cudaSuccess) return err;
+    if (dev >= 0 && dev < 64 && !attr_set[dev]) {
+        const int max_smem = (int)((PERM_CHUNK_MAX + PW * 1024) * 4);
+        if ((err = cudaFuncSetAttribute(perm_scatter_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                        max_smem)) != cudaSuccess)
+            return err;
+        if ((err = cudaFuncSetAttribute(perm_fused_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                        max_smem)) != cudaSuccess)
+            return err;
+        int coop = 0, sms = 0, per_sm = 0;
+        cudaDeviceGetAttribute(&coop, cudaDevAttrCooperativeLaunch, dev);
+        cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+        if (coop && cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, perm_fused_kernel, PT,
+                                                                  (size_t)max_smem) == cudaSuccess)
+            coop_ctas[dev] = per_sm * sms;
+        attr_set[dev] = true;
+    }
+    if (dev >= 0 && dev < 64 && nchunks <= coop_ctas[dev]) {
+        void* args[] = {(void*)&idx, (void*)&n_slots, (void*)&k, (void*)&E, (void*)&bm,
+                        (void*)&chunk, (void*)&gate_flat, (void*)&hist, (void*)&counts,
+                        (void*)&offsets, (void*)&tiles, (void*)&n_tiles, (void*)&perm, (void*)&inv,
+                        (void*)&row_tok, (void*)&row_gate, (void*)&st};
+        err = cudaLaunchCooperativeKernel((const void*)perm_fused_kernel, dim3(nchunks), dim3(PT), args,
+                                          smem, s);
+        count_launches(1);
+        return err;
+    }
+    perm_hist_kernel<<<nchunks, PT, (size_t)E * 4, s>>>(idx, n_slots, E, chunk, hist, st);
+    if ((err = cudaGetLastError()) != cudaSuccess) return err;
     perm_chunk_scan_kernel<<<(E + 7) / 8, 256, 0, s>>>(hist, nchunks, E, counts);
     if ((err = cudaGetLastError()) != cudaSuccess) return err;
     perm_offsets_kernel<<<1, 1024, 0, s>>>(counts, E, bm, offsets, tiles, n_tiles);
     if ((err = cudaGetLastError()) != cudaSuccess) return err;
-    const size_t smem = (size_t)(chunk + PW * E) * 4;
-    static bool attr_set[64] = {};
-    int dev = 0;
-    cudaGetDevice(&dev);
-    if (dev >= 0 && dev < 64 && !attr_set[dev]) {
-        err = cudaFuncSetAttribute(perm_scatter_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                   (int)((PERM_CHUNK_MAX + PW * 1024) * 4));
-        if (err != cudaSuccess) return err;
-        attr_set[dev] = true;
-    }
     perm_scatter_kernel<<<nchunks, PT, smem, s>>>(idx, n_slots, k, E, chunk, hist, offsets,
                                                   gate_flat, perm, inv, row_tok, row_gate);
     count_launches(4);
