@@ -140,6 +140,8 @@ struct GemmSpec {
     int ksplit;              // 0 or 1: no split of K; fp32 outputs only otherwise
     int64_t y_split_stride;  // floats between the outputs of consecutive splits
     int item_table;          // tiles / n_tiles hold (m-tile, n-tile) work items
+    float* zero;             // dense A: also clear zero[0, zero_n) (zero_n % 4 == 0)
+    int64_t zero_n;
 };
 
 moevie_status run_gemm(const GemmSpec& g, DevStatus* st, cudaStream_t s) {
@@ -160,6 +162,9 @@ moevie_status run_gemm(const GemmSpec& g, DevStatus* st, cudaStream_t s) {
     a.n_tiles_dev = g.n_tiles;
     a.max_mtiles = g.tiles ? max_mtiles(g.m_total, g.G) : (g.m_total + GM_BM - 1) / GM_BM;
     a.item_table = g.item_table;
+    if (g.zero && (g.a_rows || g.zero_n % 4 != 0 || !a16(g.zero))) return MOEVIE_ERR_UNSUPPORTED;
+    a.zero = reinterpret_cast<float4*>(g.zero);
+    a.zero_n = g.zero ? g.zero_n / 4 : 0;
     a.G = g.G;
     a.K = g.K;
     a.N = g.N;
@@ -197,7 +202,7 @@ moevie_status run_gemm(const GemmSpec& g, DevStatus* st, cudaStream_t s) {
 moevie_status route_impl(const void* x, const float* W_r, const float* b, int64_t T, int64_t d,
                          int64_t E, int64_t k, int32_t* idx, float* gate, const Layout& L,
                          void* ws, cudaStream_t s, bool logits_only = false,
-                         float* logits_out = nullptr) {
+                         float* logits_out = nullptr, float* zero_acc = nullptr) {
     DevStatus* st = at<DevStatus>(ws, L.status);
     const int Ep = route_epad((int)E);
     __nv_bfloat16* wsplit = at<__nv_bfloat16>(ws, L.wsplit);
@@ -228,6 +233,8 @@ moevie_status route_impl(const void* x, const float* W_r, const float* b, int64_
     g.scale = 1.0f;
     g.ksplit = ksplit;
     g.y_split_stride = part_stride;
+    g.zero = zero_acc;   // fp32 [T][d] cleared by the GEMM's idle warps (or NULL)
+    g.zero_n = T * d;
     moevie_status c = run_gemm(g, st, s);
     if (c != MOEVIE_OK) return c;
     if (logits_only) {
@@ -551,7 +558,10 @@ static moevie_status forward_impl(const moevie_layer* Lr, const void* x, int64_t
 
     MV_TRY(mark(0));
     // 1. router (Eqs. 1, 7, 4-5)
-    if ((c = route_impl(x, Lr->W_r, Lr->b, T, d, E, k, idx, gate, L, ws, s)) != MOEVIE_OK) return c;
+    // without a shared expert the router GEMM's idle warps also clear the y accumulator
+    if ((c = route_impl(x, Lr->W_r, Lr->b, T, d, E, k, idx, gate, L, ws, s, false, nullptr,
+                        hs > 0 ? nullptr : yacc)) != MOEVIE_OK)
+        return c;
     MV_TRY(mark(1));
     // 2. expert-major order (Algorithm 1, phase 1), per-row token and gate, m-tile table
     const int chunk = perm_chunk(T * k, num_sms());
@@ -566,12 +576,10 @@ static moevie_status forward_impl(const moevie_layer* Lr, const void* x, int64_t
                                  (int)max_mtiles(T * k, E), at<int4>(ws, L.items),
                                  at<int32_t>(ws, L.n_items), s));
     MV_TRY(mark(2));
-    // 3. y accumulator: lambda * shared expert, or zero
+    // 3. y accumulator: lambda * shared expert (else the router GEMM cleared it)
     if (hs > 0) {
         c = shared_expert(x, Lr->Ws1, Lr->Ws2, T, d, hs, nullptr, yacc, Lr->lambda, L, ws, st, s);
         if (c != MOEVIE_OK) return c;
-    } else {
-        MV_TRY(launch_zero_f32(yacc, T * d, s));
     }
     MV_TRY(mark(3));
     // 4. grouped up-projection, token gather in the operand load, GELU epilogue

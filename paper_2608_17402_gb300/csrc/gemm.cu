@@ -678,6 +678,16 @@ __global__ void __launch_bounds__(GM_THREADS, 1) grouped_gemm_kernel(const __gri
         if ((threadIdx.x & 31) == 0 && gather) gather_forwarder(p, sm, n_work, abort_flag);
     } else if (gather) {
         producer_gather(p, sm, n_work, abort_flag);
+    } else if (p.zero && warp >= GM_WARP_GATHER && warp < GM_WARP_FWD) {
+        // side job for the gather warps of a dense-A GEMM: clear another buffer (the y
+        // accumulator) with 16-byte stores, grid-strided, while the MMAs run
+        // (evict-first: the zeros must not push the GEMM's re-read operands out of L2)
+        const uint4 z = make_uint4(0u, 0u, 0u, 0u);
+        const uint64_t pol = l2_policy_evict_first();
+        const int64_t per = (int64_t)GM_GATHER_WARPS * 32;
+        for (int64_t i = (int64_t)blockIdx.x * per + (threadIdx.x - GM_WARP_GATHER * 32); i < p.zero_n;
+             i += (int64_t)gridDim.x * per)
+            st_global_v4_hint(p.zero + i, z, pol);
     }
 
     tc_fence_before();

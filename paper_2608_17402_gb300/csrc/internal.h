@@ -156,6 +156,8 @@ struct GemmArgs {
     int o_div;
     const float* row_scale;     // scale(r) = row_scale ? row_scale[r] : scale
     float scale;
+    float4* zero;               // dense A only: the otherwise idle gather warps clear zero[0, zero_n)
+    int64_t zero_n;             //   (float4 elements), alongside the GEMM
     DevStatus* status;
     uint64_t limit_ns;
 };
