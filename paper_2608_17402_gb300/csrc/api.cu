@@ -142,6 +142,7 @@ struct GemmSpec {
     int item_table;          // tiles / n_tiles hold (m-tile, n-tile) work items
     float* zero;             // dense A: also clear zero[0, zero_n) (zero_n % 4 == 0)
     int64_t zero_n;
+    float* nrm_out;          // dense A: also nrm_out[r] = |A[r, 0:K_A]| (K_A = a_cols or K)
 };
 
 moevie_status run_gemm(const GemmSpec& g, DevStatus* st, cudaStream_t s) {
@@ -165,6 +166,14 @@ moevie_status run_gemm(const GemmSpec& g, DevStatus* st, cudaStream_t s) {
     if (g.zero && (g.a_rows || g.zero_n % 4 != 0 || !a16(g.zero))) return MOEVIE_ERR_UNSUPPORTED;
     a.zero = reinterpret_cast<float4*>(g.zero);
     a.zero_n = g.zero ? g.zero_n / 4 : 0;
+    if (g.nrm_out) {
+        const int64_t cols = g.a_cols > 0 ? g.a_cols : g.K;
+        if (g.a_rows || cols % 8 != 0 || g.lda % 8 != 0) return MOEVIE_ERR_UNSUPPORTED;
+        a.nrm_x = static_cast<const __nv_bfloat16*>(g.A);
+        a.nrm_ld = g.lda;
+        a.nrm_cols = (int)cols;
+        a.nrm_out = g.nrm_out;
+    }
     a.G = g.G;
     a.K = g.K;
     a.N = g.N;
@@ -235,6 +244,7 @@ moevie_status route_impl(const void* x, const float* W_r, const float* b, int64_
     g.y_split_stride = part_stride;
     g.zero = zero_acc;   // fp32 [T][d] cleared by the GEMM's idle warps (or NULL)
     g.zero_n = T * d;
+    g.nrm_out = logits_only ? nullptr : at<float>(ws, L.xnorm);   // |x_t| for the certificate
     moevie_status c = run_gemm(g, st, s);
     if (c != MOEVIE_OK) return c;
     if (logits_only) {

@@ -678,16 +678,45 @@ __global__ void __launch_bounds__(GM_THREADS, 1) grouped_gemm_kernel(const __gri
         if ((threadIdx.x & 31) == 0 && gather) gather_forwarder(p, sm, n_work, abort_flag);
     } else if (gather) {
         producer_gather(p, sm, n_work, abort_flag);
-    } else if (p.zero && warp >= GM_WARP_GATHER && warp < GM_WARP_FWD) {
-        // side job for the gather warps of a dense-A GEMM: clear another buffer (the y
-        // accumulator) with 16-byte stores, grid-strided, while the MMAs run
-        // (evict-first: the zeros must not push the GEMM's re-read operands out of L2)
-        const uint4 z = make_uint4(0u, 0u, 0u, 0u);
-        const uint64_t pol = l2_policy_evict_first();
-        const int64_t per = (int64_t)GM_GATHER_WARPS * 32;
-        for (int64_t i = (int64_t)blockIdx.x * per + (threadIdx.x - GM_WARP_GATHER * 32); i < p.zero_n;
-             i += (int64_t)gridDim.x * per)
-            st_global_v4_hint(p.zero + i, z, pol);
+    } else if ((p.zero || p.nrm_out) && warp >= GM_WARP_GATHER && warp < GM_WARP_FWD) {
+        // Side jobs for the gather warps of a dense-A GEMM, while the MMAs run.
+        // 1. Row norms of the A rows of this CTA's items (the router's |x_t|, read while
+        //    the TMA brings the same rows in): one warp per row, lanes over 16-byte chunks;
+        //    the K splits of an m-tile share its rows.
+        if (p.nrm_out) {
+            const int q = warp - GM_WARP_GATHER, lane = threadIdx.x & 31;
+            for (int64_t w = sm.pair; w < n_work; w += sm.npairs) {
+                const Tile t = decode_tile(p, w);
+                if (t.n0 != 0) continue;
+                const int nh = rows_half(t, sm.rank);
+                // the K splits of an m-tile share its rows: split ks takes rows ks mod ksplit
+                for (int r = t.ks + q * p.ksplit; r < nh; r += GM_GATHER_WARPS * p.ksplit) {
+                    const int64_t row = t.row0 + (int64_t)sm.rank * GM_HALF + r;
+                    const uint4* v = reinterpret_cast<const uint4*>(p.nrm_x + row * p.nrm_ld);
+                    float acc = 0.f;
+                    for (int c = lane; c < p.nrm_cols / 8; c += 32) {
+                        const uint4 u = v[c];
+                        float f[8];
+                        unpack_bf16x8(u, f);
+#pragma unroll
+                        for (int i = 0; i < 8; ++i) acc = fmaf(f[i], f[i], acc);
+                    }
+#pragma unroll
+                    for (int o = 16; o; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
+                    if (lane == 0) p.nrm_out[row] = sqrtf(acc);
+                }
+            }
+        }
+        // 2. Clear another buffer (the y accumulator) with 16-byte stores, grid-strided
+        //    (evict-first: the zeros must not push the GEMM's re-read operands out of L2).
+        if (p.zero) {
+            const uint4 z = make_uint4(0u, 0u, 0u, 0u);
+            const uint64_t pol = l2_policy_evict_first();
+            const int64_t per = (int64_t)GM_GATHER_WARPS * 32;
+            for (int64_t i = (int64_t)blockIdx.x * per + (threadIdx.x - GM_WARP_GATHER * 32);
+                 i < p.zero_n; i += (int64_t)gridDim.x * per)
+                st_global_v4_hint(p.zero + i, z, pol);
+        }
     }
 
     tc_fence_before();

@@ -158,6 +158,10 @@ struct GemmArgs {
     float scale;
     float4* zero;               // dense A only: the otherwise idle gather warps clear zero[0, zero_n)
     int64_t zero_n;             //   (float4 elements), alongside the GEMM
+    const __nv_bfloat16* nrm_x; // dense A only: the idle gather warps also write, for the rows of
+    int64_t nrm_ld;             //   every n-tile-0 item, nrm_out[r] = |nrm_x[r, 0:nrm_cols]|
+    int nrm_cols;               //   (nrm_cols % 8 == 0)
+    float* nrm_out;
     DevStatus* status;
     uint64_t limit_ns;
 };

@@ -126,36 +126,6 @@ __device__ __forceinline__ float warp_sum(float v) {
     return v;
 }
 
-__device__ __forceinline__ float sq_bf16x8(const uint4& q) {
-    float v[8];
-    unpack_bf16x8(q, v);
-    float a = 0.f;
-#pragma unroll
-    for (int i = 0; i < 8; ++i) a = fmaf(v[i], v[i], a);
-    return a;
-}
-
-// |x_t| by one warp (16-byte loads, up to eight in flight per lane; d % 8 == 0).
-__device__ __forceinline__ float row_norm(const __nv_bfloat16* xt, int d, int lane) {
-    const uint4* v = reinterpret_cast<const uint4*>(xt);
-    const int nc = d / 8;
-    float acc = 0.f;
-    int c = lane;
-    for (; c + 224 < nc; c += 256) {
-        uint4 q[8];
-#pragma unroll
-        for (int u = 0; u < 8; ++u) q[u] = v[c + 32 * u];
-#pragma unroll
-        for (int u = 0; u < 8; ++u) acc += sq_bf16x8(q[u]);
-    }
-    for (; c + 96 < nc; c += 128) {
-        const uint4 q0 = v[c], q1 = v[c + 32], q2 = v[c + 64], q3 = v[c + 96];
-        acc += (sq_bf16x8(q0) + sq_bf16x8(q1)) + (sq_bf16x8(q2) + sq_bf16x8(q3));
-    }
-    for (; c < nc; c += 32) acc += sq_bf16x8(v[c]);
-    return sqrtf(warp_sum(acc));
-}
-
 // Order-preserving code of a float (larger float, larger code; no NaNs here).
 __device__ __forceinline__ uint32_t ord_f32(float f) {
     const uint32_t u = __float_as_uint(f);
@@ -171,7 +141,7 @@ __global__ void __launch_bounds__(256) route_topk_kernel(
     const __nv_bfloat16* __restrict__ x, float* __restrict__ s, int ld, int nparts,
     int64_t part_stride, const float* __restrict__ b, const float* __restrict__ wnorm, int T,
     int d, int E, int k, int32_t* __restrict__ idx, float* __restrict__ gate,
-    float* __restrict__ xnorm, int32_t* __restrict__ fb_tokens, DevStatus* st) {
+    const float* __restrict__ xnorm, int32_t* __restrict__ fb_tokens, DevStatus* st) {
     const int lane = threadIdx.x & 31;
     const int t = (int)(((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5);
     if (t >= T) return;
@@ -189,8 +159,7 @@ __global__ void __launch_bounds__(256) route_topk_kernel(
             if (e < E) sv[i] += srow[q * part_stride + e];
         }
     }
-    const float xn = row_norm(x + (int64_t)t * d, d, lane);
-    if (lane == 0) xnorm[t] = xn;
+    const float xn = xnorm[t];   // |x_t|, written by the router GEMM
     float sg[NPL], key[NPL], ts[NPL];
     uint32_t code[NPL];
 #pragma unroll
