@@ -169,12 +169,18 @@ def cpu_baseline(lay, target_s=15.0, max_tokens=None):
     if max_tokens:
         n = min(n, max_tokens)
     toks = np.sort(rng.choice(cfg.T, size=n, replace=False)).astype(np.int32)
-    t0 = time.perf_counter()
-    oracle.forward_tokens(lay.x, lay.Wr, lay.b, lay.W1, lay.W2, cfg.k, lay.Ws1, lay.Ws2, cfg.lam, tokens=toks)
-    dt = time.perf_counter() - t0
-    return {"value": n / dt, "unit": "tokens/s", "cores": nthreads, "kind": "oracle",
-            "sample": f"{n} of {cfg.T} tokens of {cfg.name} (whole layer per token: route, k experts, "
-                      f"shared expert), fp64, {nthreads} threads, {dt:.1f} s"}
+    # whole passes over the sample until about target_s of CPU time has been spent
+    passes, t0 = 0, time.perf_counter()
+    while True:
+        oracle.forward_tokens(lay.x, lay.Wr, lay.b, lay.W1, lay.W2, cfg.k, lay.Ws1, lay.Ws2, cfg.lam,
+                              tokens=toks)
+        passes += 1
+        dt = time.perf_counter() - t0
+        if dt >= 0.66 * target_s or passes >= 8:
+            break
+    return {"value": passes * n / dt, "unit": "tokens/s", "cores": nthreads, "kind": "oracle",
+            "sample": f"{passes} pass(es) over {n} of {cfg.T} tokens of {cfg.name} (whole layer per "
+                      f"token: route, k experts, shared expert), fp64, {nthreads} threads, {dt:.1f} s"}
 
 
 def run_reference(args, rank):

@@ -86,3 +86,16 @@ def test_forward_is_deterministic_in_routing_and_repeatable():
     for k in r1:
         assert np.array_equal(r1[k], r2[k]), k
     assert_close(y2, y1, "repeat")
+
+
+def test_forward_empty_batch_launches_nothing():
+    """T = 0 is a valid call: status OK, no kernel launched, nothing written."""
+    cfg = workloads.small_config(4, 64, 4, 2, 64)
+    lay = workloads.make_layer(cfg)
+    x, W = layer_to_device(lay)
+    ws = workspace_for(lay)
+    n0 = moevie.moevie_launch_count()
+    y = moevie.moevie_moe_forward(W, x[:0], ws)
+    assert y.shape == (0, cfg.d)
+    assert moevie.moevie_launch_count() == n0
+    check_status(ws)
