@@ -48,6 +48,12 @@ __device__ __forceinline__ void report(DevStatus* st, int code, int site, int a,
     }
 }
 
+// Programmatic dependent launch: a kernel launched with programmatic stream
+// serialization may start while its predecessor finishes; it waits here (at the
+// top, before touching anything the predecessor writes) until that predecessor has
+// completed and its memory is visible.  A no-op for ordinary launches.
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+
 // ---------------------------------------------------------------- basics
 
 __device__ __forceinline__ uint64_t globaltimer_ns() {

@@ -655,6 +655,7 @@ __global__ void __launch_bounds__(GM_THREADS, 1) grouped_gemm_kernel(const __gri
     __syncthreads();
     cluster_sync();   // barriers of both CTAs initialised before any remote arrival
     tc_fence_after();
+    pdl_wait();       // the previous kernel's outputs (tile tables, A, row maps) are ready
     const uint32_t tmem = *tmem_slot;
     int64_t n_mtiles;
     if (p.tiles) {
@@ -793,13 +794,15 @@ cudaError_t launch_grouped_gemm(const GemmArgs& a, int grid, cudaStream_t s) {
     cfg.blockDim = dim3(GM_THREADS);
     cfg.dynamicSmemBytes = gm_smem_bytes(a.epi);
     cfg.stream = s;
-    cudaLaunchAttribute attr[1];
+    cudaLaunchAttribute attr[2];
     attr[0].id = cudaLaunchAttributeClusterDimension;
     attr[0].val.clusterDim.x = 2;
     attr[0].val.clusterDim.y = 1;
     attr[0].val.clusterDim.z = 1;
+    attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;   // see launch_pdl
+    attr[1].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
-    cfg.numAttrs = 1;
+    cfg.numAttrs = 2;
     cudaError_t e = cudaLaunchKernelEx(&cfg, grouped_gemm_kernel, a);
     count_launches(1);
     return e != cudaSuccess ? e : cudaGetLastError();

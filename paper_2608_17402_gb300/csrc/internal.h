@@ -12,6 +12,25 @@ namespace mv {
 // Counts kernel launches made by this library (read by moevie_launch_count).
 void count_launches(int n);
 
+// Launches kern<<<grid, block, smem, s>>>(args...) with programmatic stream
+// serialization, so that its launch overlaps the end of the previous kernel on s
+// (every kernel of this library calls pdl_wait() before reading its inputs).
+template <typename... KArgs, typename... Args>
+cudaError_t launch_pdl(void (*kern)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t s,
+                       Args... args) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = grid;
+    cfg.blockDim = block;
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = s;
+    cudaLaunchAttribute at[1];
+    at[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    at[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = at;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, kern, static_cast<KArgs>(args)...);
+}
+
 // ----------------------------------------------------------------- router
 
 // Error model of the fast (tensor-core, fp32-accumulated) logits used to decide

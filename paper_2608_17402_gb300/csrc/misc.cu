@@ -11,6 +11,7 @@ namespace mv {
 namespace {
 
 __global__ void zero_f32_kernel(float4* __restrict__ p, int64_t n4) {
+    pdl_wait();
     const float4 z = make_float4(0.f, 0.f, 0.f, 0.f);
     for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n4;
          i += (int64_t)gridDim.x * blockDim.x)
@@ -20,6 +21,7 @@ __global__ void zero_f32_kernel(float4* __restrict__ p, int64_t n4) {
 // n8 groups of 8 values.
 __global__ void f32_to_bf16_kernel(const float4* __restrict__ src, uint4* __restrict__ dst,
                                    int64_t n8) {
+    pdl_wait();
     for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n8;
          i += (int64_t)gridDim.x * blockDim.x) {
         const float4 a = src[2 * i], b = src[2 * i + 1];
@@ -37,6 +39,7 @@ __global__ void combine_kernel(const __nv_bfloat16* __restrict__ rows,
                                const int32_t* __restrict__ inv, const float* __restrict__ gate,
                                const __nv_bfloat16* __restrict__ shared, float lambda, int64_t T,
                                int k, int d, __nv_bfloat16* __restrict__ y) {
+    pdl_wait();
     const int cpr = d >> 3;   // 8-column groups per row
     for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < T * cpr;
          i += (int64_t)gridDim.x * blockDim.x) {
@@ -94,24 +97,29 @@ int grid_for(int64_t n, int threads) {
 
 cudaError_t launch_zero_f32(float* p, int64_t n, cudaStream_t s) {
     const int64_t n4 = n / 4;   // callers pass multiples of 4
-    zero_f32_kernel<<<grid_for(n4, 256), 256, 0, s>>>(reinterpret_cast<float4*>(p), n4);
+    cudaError_t e = launch_pdl(zero_f32_kernel, dim3(grid_for(n4, 256)), dim3(256), 0, s,
+                               reinterpret_cast<float4*>(p), n4);
+    if (e != cudaSuccess) return e;
     count_launches(1);
     return cudaGetLastError();
 }
 
 cudaError_t launch_f32_to_bf16(const float* src, __nv_bfloat16* dst, int64_t n, cudaStream_t s) {
     const int64_t n8 = n / 8;   // callers pass multiples of 8
-    f32_to_bf16_kernel<<<grid_for(n8, 256), 256, 0, s>>>(reinterpret_cast<const float4*>(src),
-                                                          reinterpret_cast<uint4*>(dst), n8);
+    const cudaError_t e = launch_pdl(f32_to_bf16_kernel, dim3(grid_for(n8, 256)), dim3(256), 0, s,
+                                     reinterpret_cast<const float4*>(src), reinterpret_cast<uint4*>(dst),
+                                     n8);
     count_launches(1);
-    return cudaGetLastError();
+    return e;
 }
 
 cudaError_t launch_combine(const __nv_bfloat16* rows, const int32_t* inv, const float* gate,
                            const __nv_bfloat16* shared, float lambda, int64_t T, int k, int d,
                            __nv_bfloat16* y, cudaStream_t s) {
     const int64_t n = T * (d / 8);
-    combine_kernel<<<grid_for(n, 256), 256, 0, s>>>(rows, inv, gate, shared, lambda, T, k, d, y);
+    cudaError_t e = launch_pdl(combine_kernel, dim3(grid_for(n, 256)), dim3(256), 0, s, rows, inv, gate,
+                               shared, lambda, T, k, d, y);
+    if (e != cudaSuccess) return e;
     count_launches(1);
     return cudaGetLastError();
 }

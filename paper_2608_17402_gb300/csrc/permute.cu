@@ -62,6 +62,7 @@ __global__ void __launch_bounds__(PT) perm_hist_kernel(const int32_t* __restrict
                                                        int64_t n, int E, int chunk,
                                                        int32_t* __restrict__ hist,
                                                        DevStatus* st) {
+    pdl_wait();
     extern __shared__ int32_t cnt[];
     perm_hist_body(idx, n, E, chunk, blockIdx.x, gridDim.x, hist, st, cnt);
 }
@@ -120,6 +121,7 @@ __device__ __forceinline__ void perm_chunk_scan_warp(int32_t* __restrict__ hist,
 __global__ void __launch_bounds__(256) perm_chunk_scan_kernel(int32_t* __restrict__ hist,
                                                               int nchunks, int E,
                                                               int32_t* __restrict__ counts) {
+    pdl_wait();
     const int e = (int)(((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5);
     if (e >= E) return;
     perm_chunk_scan_warp(hist, nchunks, e, threadIdx.x & 31, counts);
@@ -132,6 +134,7 @@ __global__ void __launch_bounds__(1024) perm_offsets_kernel(const int32_t* __res
                                                             int32_t* __restrict__ offsets,
                                                             int4* __restrict__ tiles,
                                                             int32_t* __restrict__ n_tiles) {
+    pdl_wait();
     __shared__ int s_total, s_tiles;
     __shared__ int s_cnt[1024], s_off[1024], s_toff[1024];
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
@@ -230,6 +233,7 @@ __global__ void __launch_bounds__(PT) perm_scatter_kernel(
     const int32_t* __restrict__ base, const int32_t* __restrict__ offsets,
     const float* __restrict__ gate_flat, int32_t* __restrict__ perm, int32_t* __restrict__ inv,
     int32_t* __restrict__ row_tok, float* __restrict__ row_gate) {
+    pdl_wait();
     extern __shared__ __align__(16) int32_t ps_smem[];
     perm_scatter_body(idx, n, k, E, chunk, blockIdx.x, gridDim.x, base, offsets, gate_flat, perm, inv,
                       row_tok, row_gate, ps_smem);
@@ -245,6 +249,7 @@ __global__ void __launch_bounds__(PT) perm_fused_kernel(
     int32_t* __restrict__ offsets, int4* __restrict__ tiles, int32_t* __restrict__ n_tiles,
     int32_t* __restrict__ perm, int32_t* __restrict__ inv, int32_t* __restrict__ row_tok,
     float* __restrict__ row_gate, DevStatus* st) {
+    pdl_wait();
     namespace cg = cooperative_groups;
     cg::grid_group grid = cg::this_grid();
     extern __shared__ __align__(16) int32_t ps_smem[];
@@ -300,6 +305,7 @@ __global__ void __launch_bounds__(PT) perm_fused_kernel(
 __global__ void __launch_bounds__(1024) tile_table_kernel(const int32_t* __restrict__ offsets,
                                                           int G, int bm, int4* __restrict__ tiles,
                                                           int32_t* __restrict__ n_tiles) {
+    pdl_wait();
     __shared__ int s_total;
     const int g = threadIdx.x;
     const int cnt = (g < G) ? max(0, offsets[g + 1] - offsets[g]) : 0;
@@ -322,6 +328,7 @@ __global__ void __launch_bounds__(1024) item_order_kernel(
     const int4* __restrict__ tiles, const int32_t* __restrict__ n_tiles_dev,
     const int32_t* __restrict__ row_tok, int64_t T, int nb, int n_ntiles, int gsz, int BN,
     int max_tiles, int4* __restrict__ items, int32_t* __restrict__ n_items) {
+    pdl_wait();
     extern __shared__ int32_t io_smem[];
     int32_t* band = io_smem;                 // [max_tiles]
     int32_t* rank = io_smem + max_tiles;     // [max_tiles]
@@ -461,16 +468,20 @@ cudaError_t launch_permute(const int32_t* idx, int64_t n_slots, int k, int E, in
         count_launches(1);
         return err;
     }
-    perm_hist_kernel<<<nchunks, PT, (size_t)E * 4, s>>>(idx, n_slots, E, chunk, hist, st);
-    if ((err = cudaGetLastError()) != cudaSuccess) return err;
-    perm_chunk_scan_kernel<<<(E + 7) / 8, 256, 0, s>>>(hist, nchunks, E, counts);
-    if ((err = cudaGetLastError()) != cudaSuccess) return err;
-    perm_offsets_kernel<<<1, 1024, 0, s>>>(counts, E, bm, offsets, tiles, n_tiles);
-    if ((err = cudaGetLastError()) != cudaSuccess) return err;
-    perm_scatter_kernel<<<nchunks, PT, smem, s>>>(idx, n_slots, k, E, chunk, hist, offsets,
-                                                  gate_flat, perm, inv, row_tok, row_gate);
+    if ((err = launch_pdl(perm_hist_kernel, dim3(nchunks), dim3(PT), (size_t)E * 4, s, idx, n_slots, E,
+                          chunk, hist, st)) != cudaSuccess)
+        return err;
+    if ((err = launch_pdl(perm_chunk_scan_kernel, dim3((E + 7) / 8), dim3(256), 0, s, hist, nchunks, E,
+                          counts)) != cudaSuccess)
+        return err;
+    if ((err = launch_pdl(perm_offsets_kernel, dim3(1), dim3(1024), 0, s, (const int32_t*)counts, E, bm,
+                          offsets, tiles, n_tiles)) != cudaSuccess)
+        return err;
+    err = launch_pdl(perm_scatter_kernel, dim3(nchunks), dim3(PT), smem, s, idx, n_slots, k, E, chunk,
+                     (const int32_t*)hist, (const int32_t*)offsets, gate_flat, perm, inv, row_tok,
+                     row_gate);
     count_launches(4);
-    return cudaGetLastError();
+    return err;
 }
 
 cudaError_t launch_item_order(const int4* tiles, const int32_t* n_tiles, const int32_t* row_tok,
@@ -489,17 +500,18 @@ cudaError_t launch_item_order(const int4* tiles, const int32_t* n_tiles, const i
         if (err != cudaSuccess) return err;
         attr_set[dev] = true;
     }
-    item_order_kernel<<<1, 1024, smem, s>>>(tiles, n_tiles, row_tok, T, nb, n_ntiles, gsz, BN,
-                                            max_tiles, items, n_items);
+    const cudaError_t err = launch_pdl(item_order_kernel, dim3(1), dim3(1024), smem, s, tiles, n_tiles,
+                                       row_tok, T, nb, n_ntiles, gsz, BN, max_tiles, items, n_items);
     count_launches(1);
-    return cudaGetLastError();
+    return err;
 }
 
 cudaError_t launch_tile_table(const int32_t* offsets, int G, int bm, int4* tiles,
                               int32_t* n_tiles, cudaStream_t s) {
-    tile_table_kernel<<<1, 1024, 0, s>>>(offsets, G, bm, tiles, n_tiles);
+    const cudaError_t err = launch_pdl(tile_table_kernel, dim3(1), dim3(1024), 0, s, offsets, G, bm, tiles,
+                                       n_tiles);
     count_launches(1);
-    return cudaGetLastError();
+    return err;
 }
 
 }  // namespace mv

@@ -44,6 +44,7 @@ __global__ void __launch_bounds__(256) route_split_kernel(const float* __restric
                                                           __nv_bfloat16* __restrict__ Wsplit,
                                                           float* __restrict__ wrt,
                                                           float* __restrict__ wpart, DevStatus* st) {
+    pdl_wait();
     if (st && blockIdx.x == 0 && blockIdx.y == 0 && threadIdx.x == 0) st->fb_count = 0;
     __shared__ float tile[SPLIT_TILE][SPLIT_TILE + 1];
     __shared__ float red[8][32];
@@ -88,6 +89,7 @@ __global__ void __launch_bounds__(256) route_split_kernel(const float* __restric
 __global__ void __launch_bounds__(256) route_wnorm_kernel(const float* __restrict__ wpart,
                                                           int nparts, int E, int Ep,
                                                           float* __restrict__ wnorm) {
+    pdl_wait();
     const int lane = threadIdx.x & 31;
     const int e = (int)(((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5);
     if (e >= E) return;
@@ -142,6 +144,7 @@ __global__ void __launch_bounds__(256) route_topk_kernel(
     int64_t part_stride, const float* __restrict__ b, const float* __restrict__ wnorm, int T,
     int d, int E, int k, int32_t* __restrict__ idx, float* __restrict__ gate,
     const float* __restrict__ xnorm, int32_t* __restrict__ fb_tokens, DevStatus* st) {
+    pdl_wait();
     const int lane = threadIdx.x & 31;
     const int t = (int)(((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5);
     if (t >= T) return;
@@ -307,6 +310,7 @@ __global__ void __launch_bounds__(256) route_fallback_kernel(
     const float* __restrict__ xnorm, const float* __restrict__ wnorm, int d, int E, int k,
     int32_t* __restrict__ idx, float* __restrict__ gate, const int32_t* __restrict__ fb_tokens,
     DevStatus* st) {
+    pdl_wait();
     __shared__ int s_cand[32 * NPL];
     __shared__ double s_key[32 * NPL];
     __shared__ int s_ncand;
@@ -450,6 +454,7 @@ __global__ void __launch_bounds__(256) route_fallback_kernel(
 // out[t, e] = sum of the nparts partial logits, in order (used for inspection).
 __global__ void route_sum_parts_kernel(const float* __restrict__ s, int64_t part_stride,
                                        int nparts, int64_t n, float* __restrict__ out) {
+    pdl_wait();
     const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
     if (i >= n) return;
     float v = s[i];
@@ -485,19 +490,20 @@ cudaError_t launch_route_split(const float* Wr, int d, int E, __nv_bfloat16* Wsp
                                float* wpart, float* wnorm, DevStatus* st, cudaStream_t s) {
     const int Ep = route_epad(E);
     const int parts = route_split_parts(d);
-    route_split_kernel<<<dim3((Ep + SPLIT_TILE - 1) / SPLIT_TILE, parts), 256, 0, s>>>(
-        Wr, d, route_dpad(d), E, Ep, Wsplit, wrt, wpart, st);
-    route_wnorm_kernel<<<(E + 7) / 8, 256, 0, s>>>(wpart, parts, E, Ep, wnorm);
+    cudaError_t e = launch_pdl(route_split_kernel, dim3((Ep + SPLIT_TILE - 1) / SPLIT_TILE, parts),
+                               dim3(256), 0, s, Wr, d, route_dpad(d), E, Ep, Wsplit, wrt, wpart, st);
+    if (e != cudaSuccess) return e;
+    e = launch_pdl(route_wnorm_kernel, dim3((E + 7) / 8), dim3(256), 0, s, wpart, parts, E, Ep, wnorm);
     count_launches(2);
-    return cudaGetLastError();
+    return e;
 }
 
 cudaError_t launch_route_sum_parts(const float* logits, int64_t part_stride, int nparts, int64_t n,
                                    float* out, cudaStream_t s) {
-    route_sum_parts_kernel<<<(unsigned)((n + 255) / 256), 256, 0, s>>>(logits, part_stride, nparts,
-                                                                        n, out);
+    const cudaError_t e = launch_pdl(route_sum_parts_kernel, dim3((unsigned)((n + 255) / 256)),
+                                     dim3(256), 0, s, logits, part_stride, nparts, n, out);
     count_launches(1);
-    return cudaGetLastError();
+    return e;
 }
 
 cudaError_t launch_route_select(const __nv_bfloat16* x, const float* wrt, const float* b,
@@ -509,14 +515,16 @@ cudaError_t launch_route_select(const __nv_bfloat16* x, const float* wrt, const 
     const int fb_blocks = T < 4 * num_sms ? T : 4 * num_sms;
     const int npl = (E + 31) / 32;
     const int dp = route_dpad(d);
-#define MV_ROUTE(N)                                                                              \
-    do {                                                                                         \
-        route_topk_kernel<N><<<blocks, 256, 0, s>>>(x, logits, ld, nparts, part_stride, b,       \
-                                                    wnorm, T, d, E, k, idx, gate, xnorm,         \
-                                                    fb_tokens, st);                              \
-        route_fallback_kernel<N><<<fb_blocks, 256, 0, s>>>(x, wrt, dp, b, logits, ld, xnorm,     \
-                                                           wnorm, d, E, k, idx, gate, fb_tokens, \
-                                                           st);                                  \
+    cudaError_t e = cudaSuccess;
+#define MV_ROUTE(N)                                                                                \
+    do {                                                                                           \
+        e = launch_pdl(route_topk_kernel<N>, dim3(blocks), dim3(256), 0, s, x, logits, ld, nparts,  \
+                       part_stride, b, wnorm, T, d, E, k, idx, gate, (const float*)xnorm,           \
+                       fb_tokens, st);                                                             \
+        if (e == cudaSuccess)                                                                      \
+            e = launch_pdl(route_fallback_kernel<N>, dim3(fb_blocks), dim3(256), 0, s, x, wrt, dp, \
+                           b, (const float*)logits, ld, (const float*)xnorm, wnorm, d, E, k, idx,  \
+                           gate, (const int32_t*)fb_tokens, st);                                   \
     } while (0)
     if (npl <= 1) MV_ROUTE(1);
     else if (npl <= 2) MV_ROUTE(2);
@@ -526,7 +534,7 @@ cudaError_t launch_route_select(const __nv_bfloat16* x, const float* wrt, const 
     else MV_ROUTE(32);
 #undef MV_ROUTE
     count_launches(2);
-    return cudaGetLastError();
+    return e;
 }
 
 }  // namespace mv
