@@ -163,6 +163,9 @@ moevie_status run_gemm(const GemmSpec& g, DevStatus* st, cudaStream_t s) {
     a.n_tiles_dev = g.n_tiles;
     a.max_mtiles = g.tiles ? max_mtiles(g.m_total, g.G) : (g.m_total + GM_BM - 1) / GM_BM;
     a.item_table = g.item_table;
+    // reduction staging: a full-warp buffer (5 stages) unless the work is band-ordered
+    // (accumulator beyond L2, DRAM-bound: the sixth stage pays more)
+    a.stg_rows = g.item_table ? 16 : 32;
     if (g.zero && (g.a_rows || g.zero_n % 4 != 0 || !a16(g.zero))) return MOEVIE_ERR_UNSUPPORTED;
     a.zero = reinterpret_cast<float4*>(g.zero);
     a.zero_n = g.zero ? g.zero_n / 4 : 0;

@@ -217,7 +217,7 @@ struct Smem {
     uint32_t drain;
     uint32_t sink;            // 16 bytes: target / source of the peer's stage signals
     int nstages;              // operand ring depth of this launch
-    float* stg;               // reduction staging: GM_STG_ROWS rows of GM_STG_LD floats per warp
+    float* stg;               // reduction staging: STG_ROWS rows of GM_STG_LD floats per warp
     uint32_t rank;            // rank of this CTA in its pair
     int64_t pair, npairs;     // pair index and count
 };
@@ -472,6 +472,40 @@ __device__ void mma_issuer(const GemmArgs& p, const Smem& sm, uint32_t tmem, int
 
 // -------------------------------------------------------------- epilogue
 
+// One 32-column chunk of the y-accumulator reductions of one warp: each lane holds
+// its row's 32 values; ROWS rows at a time (all 32, or 16 when the staging buffer is
+// halved) go to the warp's staging buffer, scaled and with the row's y offset; then
+// every lane reduces 4 columns of one of 4 rows per instruction, so 8 lanes cover a
+// row's 128 contiguous bytes (a whole L2 line).
+template <int ROWS>
+__device__ __forceinline__ void reduce_chunk(const GemmArgs& p, float* stg_all, int warp, int lane,
+                                             const uint32_t (&v)[32], float sc, int64_t my_yoff,
+                                             int n) {
+    float* stg = stg_all + warp * (ROWS * GM_STG_LD);
+    const int col = n + 4 * (lane & 7);
+#pragma unroll
+    for (int hh = 0; hh < 32 / ROWS; ++hh) {
+        if (lane / ROWS == hh) {
+            float* row = stg + (lane - hh * ROWS) * GM_STG_LD;
+#pragma unroll
+            for (int c = 0; c < 8; ++c)
+                *reinterpret_cast<float4*>(row + 4 * c) =
+                    make_float4(sc * __uint_as_float(v[4 * c]), sc * __uint_as_float(v[4 * c + 1]),
+                                sc * __uint_as_float(v[4 * c + 2]), sc * __uint_as_float(v[4 * c + 3]));
+            *reinterpret_cast<int64_t*>(row + 32) = my_yoff;
+        }
+        __syncwarp();
+#pragma unroll
+        for (int r = 0; r < ROWS / 4; ++r) {
+            const float* row = stg + (4 * r + (lane >> 3)) * GM_STG_LD;
+            const int64_t yo = *reinterpret_cast<const int64_t*>(row + 32);
+            const float4 val = *reinterpret_cast<const float4*>(row + 4 * (lane & 7));
+            if (yo >= 0 && col < p.N) atomicAdd(reinterpret_cast<float4*>(p.yacc + yo + col), val);
+        }
+        __syncwarp();
+    }
+}
+
 // Warp w reads TMEM lanes 32 (w % 4) .. +31 (its rows) and the 32-column chunks
 // c = w / 4, w / 4 + 2, ... of each tile.  bf16 outputs and fp32 stores: each thread
 // takes its own row (32x32b loads) and writes it straight from registers with
@@ -479,6 +513,7 @@ __device__ void mma_issuer(const GemmArgs& p, const Smem& sm, uint32_t tmem, int
 // per-warp staging buffer so that each 16-byte vector reduction instruction of a
 // warp covers four rows x 128 contiguous bytes, i.e. whole L2 lines.  When a warp has read
 // its last chunk of the accumulator it arrives (once) on the leader's tempty barrier.
+template <int STG_ROWS>
 __device__ void epilogue(const GemmArgs& p, const Smem& sm, uint32_t tmem, int64_t n_work,
                          volatile int* abort_flag) {
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -520,10 +555,6 @@ __device__ void epilogue(const GemmArgs& p, const Smem& sm, uint32_t tmem, int64
         for (int ch = half; ch < nchunk; ch += 2) {
             const int c0 = ch * 32;
             if (p.epi == EPI_ADD_F32) {
-                // Each lane holds its row's 32 columns; half the warp at a time writes
-                // its rows (scaled, plus the row's y offset) into the staging buffer,
-                // then every lane reduces 4 columns of one of 4 rows per instruction:
-                // 8 lanes cover a row's 128 contiguous bytes (a whole L2 line).
                 uint32_t v[32];
                 tmem_ld_32x32b_x32(tbase + c0, v);
                 tmem_wait_ld();
@@ -533,29 +564,8 @@ __device__ void epilogue(const GemmArgs& p, const Smem& sm, uint32_t tmem, int64
                     if (lane == 0) mbar_arrive_remote(tempty_leader + 8 * acc);
                 }
                 const int n = t.n0 + c0;
-                float* stg = sm.stg + warp * (GM_STG_ROWS * GM_STG_LD);
-#pragma unroll
-                for (int hh = 0; hh < 2; ++hh) {
-                    if ((lane >> 4) == hh) {
-                        float* row = stg + (lane & 15) * GM_STG_LD;
-#pragma unroll
-                        for (int c = 0; c < 8; ++c)
-                            *reinterpret_cast<float4*>(row + 4 * c) =
-                                make_float4(sc * __uint_as_float(v[4 * c]), sc * __uint_as_float(v[4 * c + 1]),
-                                            sc * __uint_as_float(v[4 * c + 2]), sc * __uint_as_float(v[4 * c + 3]));
-                        *reinterpret_cast<int64_t*>(row + 32) = ok_row ? t.ks * p.y_split_stride + tok * p.ldy : -1;
-                    }
-                    __syncwarp();
-                    const int col = n + 4 * (lane & 7);
-#pragma unroll
-                    for (int r = 0; r < 4; ++r) {
-                        const float* row = stg + (4 * r + (lane >> 3)) * GM_STG_LD;
-                        const int64_t yo = *reinterpret_cast<const int64_t*>(row + 32);
-                        const float4 val = *reinterpret_cast<const float4*>(row + 4 * (lane & 7));
-                        if (yo >= 0 && col < p.N) atomicAdd(reinterpret_cast<float4*>(p.yacc + yo + col), val);
-                    }
-                    __syncwarp();
-                }
+                const int64_t my_yoff = ok_row ? t.ks * p.y_split_stride + tok * p.ldy : -1;
+                reduce_chunk<STG_ROWS>(p, sm.stg, warp, lane, v, sc, my_yoff, n);
                 continue;
             }
             uint32_t v[32];
@@ -600,15 +610,18 @@ __device__ void epilogue(const GemmArgs& p, const Smem& sm, uint32_t tmem, int64
     }
 }
 
+// STG_ROWS: rows per warp of the reduction staging buffer (EPI_ADD_F32), one kernel
+// instance each so that the epilogue loops have constant trip counts.
+template <int STG_ROWS>
 __global__ void __launch_bounds__(GM_THREADS, 1) grouped_gemm_kernel(const __grid_constant__ GemmArgs p) {
     extern __shared__ uint8_t gm_smem_raw[];
     uint8_t* smem = reinterpret_cast<uint8_t*>(
         (reinterpret_cast<uintptr_t>(gm_smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
     uint8_t* sA = smem;
-    const int nst = gm_stages(p.epi);
+    const int nst = gm_stages(p.epi, STG_ROWS);
     uint8_t* sB = smem + nst * GM_A_BYTES;
     uint8_t* sStg = sB + nst * GM_B_BYTES;                       // reduction staging (EPI_ADD_F32)
-    uint64_t* bars = reinterpret_cast<uint64_t*>(sStg + (p.epi == EPI_ADD_F32 ? GM_STG_BYTES : 0));
+    uint64_t* bars = reinterpret_cast<uint64_t*>(sStg + gm_stg_bytes(p.epi, STG_ROWS));
     uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 3 * GM_STAGES_MAX + 5);
     volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
     uint8_t* sink = reinterpret_cast<uint8_t*>(bars) + 256;   // 16-byte aligned, after the barriers
@@ -670,7 +683,7 @@ __global__ void __launch_bounds__(GM_THREADS, 1) grouped_gemm_kernel(const __gri
     const int64_t n_work = p.item_table ? n_mtiles * p.ksplit : n_mtiles * p.n_ntiles * p.ksplit;
 
     if (warp < GM_EPI_WARPS) {
-        epilogue(p, sm, tmem, n_work, abort_flag);
+        epilogue<STG_ROWS>(p, sm, tmem, n_work, abort_flag);
     } else if (warp == GM_WARP_MMA) {
         if ((threadIdx.x & 31) == 0 && sm.rank == 0) mma_issuer(p, sm, tmem, n_work, abort_flag);
     } else if (warp == GM_WARP_LOAD) {
@@ -779,20 +792,23 @@ void choose_bn(int N, int* BN, int* n_ntiles) {
 }
 
 cudaError_t launch_grouped_gemm(const GemmArgs& a, int grid, cudaStream_t s) {
+    if (a.stg_rows != 32 && a.stg_rows != 16) return cudaErrorInvalidValue;
+    auto* kern = a.stg_rows == 32 ? grouped_gemm_kernel<32> : grouped_gemm_kernel<16>;
     static bool attr_set[64] = {};
     int dev = 0;
     cudaGetDevice(&dev);
     if (dev >= 0 && dev < 64 && !attr_set[dev]) {
-        cudaError_t e = cudaFuncSetAttribute(grouped_gemm_kernel,
-                                             cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                             GM_SMEM_BYTES_MAX);
-        if (e != cudaSuccess) return e;
+        for (auto* k : {grouped_gemm_kernel<32>, grouped_gemm_kernel<16>}) {
+            cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                                 GM_SMEM_BYTES_MAX);
+            if (e != cudaSuccess) return e;
+        }
         attr_set[dev] = true;
     }
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3((unsigned)((grid + 1) & ~1));   // whole pairs
     cfg.blockDim = dim3(GM_THREADS);
-    cfg.dynamicSmemBytes = gm_smem_bytes(a.epi);
+    cfg.dynamicSmemBytes = gm_smem_bytes(a.epi, a.stg_rows);
     cfg.stream = s;
     cudaLaunchAttribute attr[2];
     attr[0].id = cudaLaunchAttributeClusterDimension;
@@ -803,7 +819,7 @@ cudaError_t launch_grouped_gemm(const GemmArgs& a, int grid, cudaStream_t s) {
     attr[1].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
     cfg.numAttrs = 2;
-    cudaError_t e = cudaLaunchKernelEx(&cfg, grouped_gemm_kernel, a);
+    cudaError_t e = cudaLaunchKernelEx(&cfg, kern, a);
     count_launches(1);
     return e != cudaSuccess ? e : cudaGetLastError();
 }

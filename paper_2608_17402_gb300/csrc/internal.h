@@ -124,16 +124,26 @@ constexpr int GM_GATHER_RSTEP = GM_GATHER_WARPS * 32 / 8;
 constexpr int GM_GATHER_ROWS = 128 / GM_GATHER_RSTEP;
 constexpr int GM_A_BYTES = GM_HALF * GM_BK * 2;           // one CTA's A rows per stage
 constexpr int GM_B_BYTES = GM_BK * (GM_MAXBN / 2) * 2;    // one CTA's half of B per stage
-constexpr int GM_STG_ROWS = 16;    // rows per warp in the reduction staging buffer
+constexpr int GM_STG_ROWS = 32;    // rows per warp in the reduction staging buffer (at most)
 constexpr int GM_STG_LD = 36;      // floats per staged row: 32 values, the row's y offset, pad
-constexpr int GM_STG_BYTES = GM_EPI_WARPS * GM_STG_ROWS * GM_STG_LD * 4;
 constexpr int GM_OVERHEAD_BYTES = 1024 + 512;   // alignment, barriers / TMEM slot / flags / sink
-__host__ __device__ constexpr int gm_stages(int epi) { return epi == 2 /* EPI_ADD_F32 */ ? 6 : 7; }
-__host__ __device__ constexpr int gm_smem_bytes(int epi) {
-    return gm_stages(epi) * (GM_A_BYTES + GM_B_BYTES) + (epi == 2 ? GM_STG_BYTES : 0) + GM_OVERHEAD_BYTES;
+// The y-accumulator epilogue (epi 2, EPI_ADD_F32) stages stg_rows (32 or 16) rows per warp
+// and gives up operand stages for them: 32 rows -> 5 stages, 16 rows -> 6.  Other
+// epilogues run 7 stages.
+__host__ __device__ constexpr int gm_stg_bytes(int epi, int stg_rows) {
+    return epi == 2 ? GM_EPI_WARPS * stg_rows * GM_STG_LD * 4 : 0;
+}
+__host__ __device__ constexpr int gm_stages(int epi, int stg_rows) {
+    return epi == 2 ? (stg_rows > 16 ? 5 : 6) : 7;
+}
+__host__ __device__ constexpr int gm_smem_bytes(int epi, int stg_rows) {
+    return gm_stages(epi, stg_rows) * (GM_A_BYTES + GM_B_BYTES) + gm_stg_bytes(epi, stg_rows) +
+           GM_OVERHEAD_BYTES;
 }
 constexpr int GM_SMEM_BYTES_MAX = GM_STAGES_MAX * (GM_A_BYTES + GM_B_BYTES) + GM_OVERHEAD_BYTES;
-static_assert(GM_SMEM_BYTES_MAX <= 232448 && gm_smem_bytes(2) <= 232448, "shared memory of one CTA");
+static_assert(GM_SMEM_BYTES_MAX <= 232448 && gm_smem_bytes(2, 32) <= 232448 &&
+                  gm_smem_bytes(2, 16) <= 232448,
+              "shared memory of one CTA");
 static_assert(3 * GM_STAGES_MAX + 5 <= 32, "barriers fit before the signal sink at +256 bytes");
 
 inline int64_t max_mtiles(int64_t rows, int64_t groups) { return (rows + GM_BM - 1) / GM_BM + groups; }
@@ -160,6 +170,7 @@ struct GemmArgs {
     const int4* tiles;          // m-tile table {g, row0, nrows, 0}; nullptr: one dense group;
                                 // with item_table: work items {g, row0, nrows, n0}
     int item_table;             // tiles lists (m-tile, n-tile) items; *n_tiles_dev counts items
+    int stg_rows;               // EPI_ADD_F32: rows staged per warp and phase (32 or 16)
     const int32_t* n_tiles_dev; // number of entries of `tiles`
     int64_t max_mtiles;         // host bound on *n_tiles_dev
     int G, K, N, BN, n_ntiles, num_kb, nbox;
