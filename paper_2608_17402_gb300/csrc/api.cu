@@ -35,6 +35,56 @@ struct Layout {
     size_t total;
 };
 
+struct BandPlan {   // token bands and n-tiles per column group of the down-projection
+    int nb, gsz;
+};
+// Work order of the down-projection.  Its epilogue adds every routed row into the
+// fp32 y accumulator [T, d]; when that is larger than ITEM_BAND_MIN_BYTES (it would
+// not stay in L2 next to the streamed operands) the items run in nb token bands x
+// column groups of gsz n-tiles (item_order_kernel), so that the accumulator block
+// being reduced into (at most ITEM_BLOCK_BYTES) stays in L2.  Each extra band re-reads
+// the expert weights W2, each extra column group the rows of H: the split minimises
+// that traffic under the block-size bound.
+constexpr double ITEM_BAND_MIN_BYTES = 64.0 * (1 << 20);
+constexpr double ITEM_BLOCK_BYTES = 24.0 * (1 << 20);
+BandPlan choose_bands(int64_t T, int64_t d, int64_t E, int64_t k, int64_t h) {
+    int BN = 0, nnt = 0;
+    choose_bn((int)d, &BN, &nnt);
+    const double yacc = 4.0 * T * d;
+    if (yacc <= ITEM_BAND_MIN_BYTES || max_mtiles(T * k, E) > ITEM_MAX_TILES) return {1, nnt};
+    const double Hb = 2.0 * T * k * h, Wb = 2.0 * E * h * d;
+    BandPlan best{1, nnt};
+    double best_cost = 1e300;
+    for (int nb = 1; nb <= ITEM_MAX_BANDS; ++nb)
+        for (int nc = 1; nc <= nnt; ++nc) {
+            const int gsz = (nnt + nc - 1) / nc;
+            const int groups = (nnt + gsz - 1) / gsz;
+            if (yacc / ((double)nb * groups) > ITEM_BLOCK_BYTES) continue;
+            const double cost = Hb * groups + Wb * nb;
+            if (cost < best_cost) {
+                best_cost = cost;
+                best = {nb, gsz};
+            }
+        }
+    return best;
+}
+
+// The shared expert runs inside the grouped GEMMs as S = h_s / h always-on groups
+// E .. E + S - 1 (its hidden units in chunks of h: GELU acts unit by unit, so the
+// chunks' down-projections add up to the shared expert's output), every token with
+// gate lambda, when h divides h_s and the down-projection is not band-ordered.
+// 0: the shared expert runs as its own dense GEMMs.
+constexpr int64_t SHARED_MAX_CHUNKS = 16;
+int64_t shared_chunks(int64_t T, int64_t d, int64_t E, int64_t k, int64_t h, int64_t hs) {
+    if (hs <= 0 || h <= 0 || d <= 0 || T < 0 || hs % h != 0 || hs / h > SHARED_MAX_CHUNKS) return 0;
+    if (T * (k + hs / h) >= (int64_t(1) << 31)) return 0;
+    int BN = 0, nnt = 0;
+    choose_bn((int)d, &BN, &nnt);
+    const BandPlan bp = choose_bands(T, d, E, k, h);
+    if (bp.nb > 1 || bp.gsz < nnt) return 0;
+    return hs / h;
+}
+
 Layout make_layout(int64_t T, int64_t d, int64_t E, int64_t k, int64_t h, int64_t hs) {
     Layout L;
     size_t o = 0;
@@ -59,7 +109,9 @@ Layout make_layout(int64_t T, int64_t d, int64_t E, int64_t k, int64_t h, int64_
     L.hist = take(4 * nchunks_max * E);
     L.counts = take(4 * E);
     L.offsets = take(4 * (E + 1));
-    L.tiles = take(16 * max_mtiles(n, E));
+    const int64_t S = shared_chunks(T, d, E, k, h, hs);
+    const int64_t n2 = n + S * T;   // GEMM rows: routed, then the shared groups'
+    L.tiles = take(16 * (max_mtiles(n, E) + S * ((T + GM_BM - 1) / GM_BM)));
     int BN = 0, n_nt = 0;
     choose_bn((int)(d > 0 ? d : 1), &BN, &n_nt);
     L.items = take(16 * max_mtiles(n, E) * n_nt);   // band-ordered down-projection items
@@ -67,10 +119,10 @@ Layout make_layout(int64_t T, int64_t d, int64_t E, int64_t k, int64_t h, int64_
     L.n_tiles = take(4);
     L.perm = take(4 * n);
     L.inv = take(4 * n);
-    L.row_tok = take(4 * n);
-    L.row_gate = take(4 * n);
-    L.H = take(2 * n * h);
-    L.Hs = take(2 * T * hs);
+    L.row_tok = take(4 * n2);
+    L.row_gate = take(4 * n2);
+    L.H = take(2 * n2 * h);
+    L.Hs = take(S > 0 ? 0 : 2 * T * hs);
     L.yacc = take(4 * T * d);
     L.total = o;
     return L;
@@ -143,13 +195,24 @@ struct GemmSpec {
     float* zero;             // dense A: also clear zero[0, zero_n) (zero_n % 4 == 0)
     int64_t zero_n;
     float* nrm_out;          // dense A: also nrm_out[r] = |A[r, 0:K_A]| (K_A = a_cols or K)
+    const void* W2nd;        // groups g >= g_split: weights at W2nd + (g - g_split) w2_g_ld +
+    int64_t w2_k_ld;         //   kk w2_k_ld + n (elements); W then holds g_split groups
+    int64_t w2_g_ld;
+    int g_split;
 };
 
 moevie_status run_gemm(const GemmSpec& g, DevStatus* st, cudaStream_t s) {
     GemmArgs a;
     memset(&a, 0, sizeof a);
     const int64_t n_ld = g.N_ld > 0 ? g.N_ld : g.N;
-    if (!make_weight_tmap(&a.tmB, g.W, n_ld, g.K, g.G)) return MOEVIE_ERR_CUDA;
+    if (!make_weight_tmap(&a.tmB, g.W, n_ld, g.K, g.W2nd ? g.g_split : g.G)) return MOEVIE_ERR_CUDA;
+    if (g.W2nd) {
+        if (g.g_split <= 0 || g.g_split >= g.G || !a16(g.W2nd) || g.w2_k_ld % 8 != 0 ||
+            g.w2_g_ld % 8 != 0)
+            return MOEVIE_ERR_UNSUPPORTED;
+        if (!make_weight_tmap_strided(&a.tmB2, g.W2nd, g.N, g.K, g.G - g.g_split, g.w2_k_ld, g.w2_g_ld))
+            return MOEVIE_ERR_CUDA;
+    }
     if (!g.a_rows && !make_rows_tmap(&a.tmA, g.A, g.a_cols > 0 ? g.a_cols : g.K, g.a_nrows, g.lda))
         return MOEVIE_ERR_CUDA;
     a.A = static_cast<const __nv_bfloat16*>(g.A);
@@ -178,6 +241,7 @@ moevie_status run_gemm(const GemmSpec& g, DevStatus* st, cudaStream_t s) {
         a.nrm_out = g.nrm_out;
     }
     a.G = g.G;
+    a.g_split = g.W2nd ? g.g_split : g.G;
     a.K = g.K;
     a.N = g.N;
     choose_bn(g.N, &a.BN, &a.n_ntiles);
@@ -499,40 +563,6 @@ moevie_status moevie_combine(const void* out_rows, const int32_t* inv, const flo
                                       static_cast<cudaStream_t>(stream)));
 }
 
-// Work order of the down-projection.  Its epilogue adds every routed row into the
-// fp32 y accumulator [T, d]; when that is larger than ITEM_BAND_MIN_BYTES (it would
-// not stay in L2 next to the streamed operands) the items run in nb token bands x
-// column groups of gsz n-tiles (item_order_kernel), so that the accumulator block
-// being reduced into (at most ITEM_BLOCK_BYTES) stays in L2.  Each extra band re-reads
-// the expert weights W2, each extra column group the rows of H: the split minimises
-// that traffic under the block-size bound.
-constexpr double ITEM_BAND_MIN_BYTES = 64.0 * (1 << 20);
-constexpr double ITEM_BLOCK_BYTES = 24.0 * (1 << 20);
-struct BandPlan {
-    int nb, gsz;
-};
-BandPlan choose_bands(int64_t T, int64_t d, int64_t E, int64_t k, int64_t h) {
-    int BN = 0, nnt = 0;
-    choose_bn((int)d, &BN, &nnt);
-    const double yacc = 4.0 * T * d;
-    if (yacc <= ITEM_BAND_MIN_BYTES || max_mtiles(T * k, E) > ITEM_MAX_TILES) return {1, nnt};
-    const double Hb = 2.0 * T * k * h, Wb = 2.0 * E * h * d;
-    BandPlan best{1, nnt};
-    double best_cost = 1e300;
-    for (int nb = 1; nb <= ITEM_MAX_BANDS; ++nb)
-        for (int nc = 1; nc <= nnt; ++nc) {
-            const int gsz = (nnt + nc - 1) / nc;
-            const int groups = (nnt + gsz - 1) / gsz;
-            if (yacc / ((double)nb * groups) > ITEM_BLOCK_BYTES) continue;
-            const double cost = Hb * groups + Wb * nb;
-            if (cost < best_cost) {
-                best_cost = cost;
-                best = {nb, gsz};
-            }
-        }
-    return best;
-}
-
 static moevie_status forward_impl(const moevie_layer* Lr, const void* x, int64_t T, void* y,
                                   const moevie_routing* routing, void* ws, size_t ws_bytes,
                                   void* stream, void* const* events, int n_events) {
@@ -569,11 +599,14 @@ static moevie_status forward_impl(const moevie_layer* Lr, const void* x, int64_t
         return events ? cudaEventRecord(static_cast<cudaEvent_t>(events[i]), s) : cudaSuccess;
     };
 
+    const int64_t S = shared_chunks(T, d, E, k, h, hs);   // shared expert inside the grouped GEMMs
+    const int64_t n2 = T * k + S * T;
     MV_TRY(mark(0));
     // 1. router (Eqs. 1, 7, 4-5)
-    // without a shared expert the router GEMM's idle warps also clear the y accumulator
+    // unless a separate shared-expert GEMM writes it first, the router GEMM's idle
+    // warps also clear the y accumulator
     if ((c = route_impl(x, Lr->W_r, Lr->b, T, d, E, k, idx, gate, L, ws, s, false, nullptr,
-                        hs > 0 ? nullptr : yacc)) != MOEVIE_OK)
+                        (hs > 0 && S == 0) ? nullptr : yacc)) != MOEVIE_OK)
         return c;
     MV_TRY(mark(1));
     // 2. expert-major order (Algorithm 1, phase 1), per-row token and gate, m-tile table
@@ -589,28 +622,61 @@ static moevie_status forward_impl(const moevie_layer* Lr, const void* x, int64_t
                                  (int)max_mtiles(T * k, E), at<int4>(ws, L.items),
                                  at<int32_t>(ws, L.n_items), s));
     MV_TRY(mark(2));
-    // 3. y accumulator: lambda * shared expert (else the router GEMM cleared it)
-    if (hs > 0) {
+    // 3. shared expert (Eq. 3): S always-on groups of the grouped GEMMs (rows, gates
+    // lambda and m-tiles appended after the routed ones); otherwise its own GEMMs write
+    // lambda * shared expert as the first value of the y accumulator
+    if (S > 0) {
+        MV_TRY(launch_shared_rows(T, T * k, (int)S, (int)E, Lr->lambda, row_tok, row_gate, tiles,
+                                  n_tiles, max_mtiles(T * k, E), st, s));
+    } else if (hs > 0) {
         c = shared_expert(x, Lr->Ws1, Lr->Ws2, T, d, hs, nullptr, yacc, Lr->lambda, L, ws, st, s);
         if (c != MOEVIE_OK) return c;
     }
     MV_TRY(mark(3));
     // 4. grouped up-projection, token gather in the operand load, GELU epilogue
-    if ((c = expert_up(x, row_tok, 1, tiles, n_tiles, Lr->W1, T, d, h, E, k, at<void>(ws, L.H),
-                       st, s)) != MOEVIE_OK)
-        return c;
+    {
+        GemmSpec up{};
+        up.A = x;
+        up.lda = d;
+        up.a_rows = row_tok;
+        up.a_div = 1;
+        up.a_nrows = T;
+        up.m_total = n2;
+        up.tiles = tiles;
+        up.n_tiles = n_tiles;
+        up.G = (int)(E + S);
+        up.W = Lr->W1;
+        up.K = (int)d;
+        up.N = (int)h;
+        up.epi = EPI_GELU_BF16;
+        up.out = at<void>(ws, L.H);
+        up.ldo = h;
+        if (S > 0) {   // chunk c of Ws1 [d, h_s]: columns c h .. c h + h - 1
+            up.W2nd = Lr->Ws1;
+            up.w2_k_ld = hs;
+            up.w2_g_ld = h;
+            up.g_split = (int)E;
+        }
+        if ((c = run_gemm(up, st, s)) != MOEVIE_OK) return c;
+    }
     MV_TRY(mark(4));
     // 5. grouped down-projection, epilogue: gate * row added into y (scatter-add)
     GemmSpec dn{};
     dn.A = at<void>(ws, L.H);
     dn.lda = h;
-    dn.a_nrows = T * k;
-    dn.m_total = T * k;
+    dn.a_nrows = n2;
+    dn.m_total = n2;
     dn.tiles = banded ? at<int4>(ws, L.items) : tiles;
     dn.n_tiles = banded ? at<int32_t>(ws, L.n_items) : n_tiles;
     dn.item_table = banded ? 1 : 0;
-    dn.G = (int)E;
+    dn.G = (int)(E + S);
     dn.W = Lr->W2;
+    if (S > 0) {   // chunk c of Ws2 [h_s, d]: rows c h .. c h + h - 1
+        dn.W2nd = Lr->Ws2;
+        dn.w2_k_ld = d;
+        dn.w2_g_ld = h * d;
+        dn.g_split = (int)E;
+    }
     dn.K = (int)h;
     dn.N = (int)d;
     dn.epi = EPI_ADD_F32;

@@ -254,6 +254,7 @@ __device__ __forceinline__ int rows_half(const Tile& t, uint32_t rank) {
 __device__ void producer_tma(const GemmArgs& p, const Smem& sm, int64_t n_work,
                              volatile int* abort_flag) {
     tma_prefetch_desc(&p.tmB);
+    if (p.g_split < p.G) tma_prefetch_desc(&p.tmB2);
     const bool gather = p.a_rows != nullptr;
     if (!gather) tma_prefetch_desc(&p.tmA);
     const uint32_t half_n = (uint32_t)p.BN / 2;
@@ -271,6 +272,9 @@ __device__ void producer_tma(const GemmArgs& p, const Smem& sm, int64_t n_work,
         const int64_t wn = w + sm.npairs;
         Tile tn{};
         if (wn < n_work) tn = decode_tile(p, wn);
+        const bool second = t.g >= p.g_split;   // B of this group from the second map
+        const CUtensorMap* tmb = second ? &p.tmB2 : &p.tmB;
+        const int gb = second ? t.g - p.g_split : t.g;
         for (int kb = t.kb0; kb < t.kb1; ++kb) {
             if (!mbar_wait(sm.empty + 8 * s, ph ^ 1u, p.limit_ns, abort_flag)) {
                 set_abort(abort_flag, p.status, SITE_GEMM_WAIT_EMPTY, (int)sm.pair, 1);
@@ -281,8 +285,8 @@ __device__ void producer_tma(const GemmArgs& p, const Smem& sm, int64_t n_work,
             const uint32_t b_dst = sm.b0 + s * GM_B_BYTES;
             const int kk = kb * GM_BK;
             for (uint32_t j = 0; j < nboxh; ++j)
-                tma_load_3d_pair(b_dst + j * (GM_BK * 128), &p.tmB, bar,
-                                 t.n0 + (int)(sm.rank * half_n + 64 * j), kk, t.g);
+                tma_load_3d_pair(b_dst + j * (GM_BK * 128), tmb, bar,
+                                 t.n0 + (int)(sm.rank * half_n + 64 * j), kk, gb);
             if (!gather) {
                 const int col = p.a_kperiod ? kk % p.a_kperiod : kk;
                 tma_load_2d_pair(sm.a0 + s * GM_A_BYTES, &p.tmA, bar, col,
@@ -771,17 +775,22 @@ PFN_cuTensorMapEncodeTiled_v12000 get_encode_fn() {
 
 }  // namespace
 
-bool make_weight_tmap(CUtensorMap* tm, const void* base, int64_t N, int64_t K, int64_t G) {
+bool make_weight_tmap_strided(CUtensorMap* tm, const void* base, int64_t N, int64_t K, int64_t G,
+                              int64_t k_ld, int64_t g_ld) {
     PFN_cuTensorMapEncodeTiled_v12000 enc = get_encode_fn();
     if (!enc) return false;
     cuuint64_t dims[3] = {(cuuint64_t)N, (cuuint64_t)K, (cuuint64_t)G};
-    cuuint64_t strides[2] = {(cuuint64_t)N * 2, (cuuint64_t)N * K * 2};
+    cuuint64_t strides[2] = {(cuuint64_t)k_ld * 2, (cuuint64_t)g_ld * 2};
     cuuint32_t box[3] = {64, GM_BK, 1};
     cuuint32_t estr[3] = {1, 1, 1};
     CUresult r = enc(tm, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(base), dims,
                      strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
                      CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
     return r == CUDA_SUCCESS;
+}
+
+bool make_weight_tmap(CUtensorMap* tm, const void* base, int64_t N, int64_t K, int64_t G) {
+    return make_weight_tmap_strided(tm, base, N, K, G, N, N * K);
 }
 
 bool make_rows_tmap(CUtensorMap* tm, const void* base, int64_t cols, int64_t rows, int64_t ld) {

@@ -158,6 +158,7 @@ static_assert(EPI_ADD_F32 == 2, "gm_stages / gm_smem_bytes test the reduction ep
 
 struct GemmArgs {
     CUtensorMap tmB;            // B = weights [G][K][N] bf16 (N contiguous), 3-D map {N, K, G}
+    CUtensorMap tmB2;           // groups g >= g_split: B from this map, group g - g_split
     CUtensorMap tmA;            // A = rows [a_nrows][K_A] bf16, 2-D map {K_A, a_nrows}, box
                                 // {64, 128}; used when A rows are contiguous (a_rows == nullptr)
     const __nv_bfloat16* A;     // A rows, for the token gather
@@ -174,6 +175,7 @@ struct GemmArgs {
     const int32_t* n_tiles_dev; // number of entries of `tiles`
     int64_t max_mtiles;         // host bound on *n_tiles_dev
     int G, K, N, BN, n_ntiles, num_kb, nbox;
+    int g_split;                // first group read through tmB2 (G when there is none)
     int ksplit;                 // K is split into this many parts (work items), >= 1
     int64_t y_split_stride;     // fp32 outputs: split ks writes yacc + ks * y_split_stride
     int epi;
@@ -198,6 +200,10 @@ struct GemmArgs {
 
 // Encodes the 3-D weight tensor map {N, K, G} for W[G][K][N] bf16.
 bool make_weight_tmap(CUtensorMap* tm, const void* base, int64_t N, int64_t K, int64_t G);
+// The same for a strided view: element (g, kk, n) at base + g * g_ld + kk * k_ld + n
+// (strides in elements, multiples of 8).
+bool make_weight_tmap_strided(CUtensorMap* tm, const void* base, int64_t N, int64_t K, int64_t G,
+                              int64_t k_ld, int64_t g_ld);
 // Encodes the 2-D row tensor map {cols, rows} of A[rows][cols] bf16 (row stride ld
 // elements), box {64, GM_HALF}.
 bool make_rows_tmap(CUtensorMap* tm, const void* base, int64_t cols, int64_t rows, int64_t ld);
@@ -234,6 +240,12 @@ cudaError_t perm_static_scratch(unsigned char** out);
 
 cudaError_t launch_zero_f32(float* p, int64_t n, cudaStream_t s);
 cudaError_t launch_f32_to_bf16(const float* src, __nv_bfloat16* dst, int64_t n, cudaStream_t s);
+// Rows of the shared expert folded into the grouped GEMMs as S always-on groups
+// E .. E + S - 1 of T rows each, at rows base + c T + t (token t, gate lambda), and
+// their m-tiles appended to the tile table (after the *n_tiles routed ones).
+cudaError_t launch_shared_rows(int64_t T, int64_t base, int S, int E, float lambda,
+                               int32_t* row_tok, float* row_gate, int4* tiles, int32_t* n_tiles,
+                               int64_t max_routed, DevStatus* st, cudaStream_t s);
 cudaError_t launch_combine(const __nv_bfloat16* rows, const int32_t* inv, const float* gate,
                            const __nv_bfloat16* shared, float lambda, int64_t T, int k, int d,
                            __nv_bfloat16* y, cudaStream_t s);

@@ -87,6 +87,38 @@ __global__ void wait_probe_kernel(DevStatus* st, uint64_t limit_ns) {
     }
 }
 
+// Rows of the shared expert's S always-on groups (E .. E + S - 1): row base + c T + t
+// is token t with gate lambda.  Block 0 also appends the groups' m-tiles after the
+// routed ones that the permute step counted in *n_tiles.
+__global__ void shared_rows_kernel(int64_t T, int64_t base, int S, int E, float lambda,
+                                   int32_t* __restrict__ row_tok, float* __restrict__ row_gate,
+                                   int4* __restrict__ tiles, int32_t* __restrict__ n_tiles,
+                                   int64_t max_routed, DevStatus* st) {
+    pdl_wait();   // the permute step's tile count
+    const int64_t n = T * S;
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n;
+         i += (int64_t)gridDim.x * blockDim.x) {
+        row_tok[base + i] = (int32_t)(i % T);
+        row_gate[base + i] = lambda;
+    }
+    if (blockIdx.x == 0) {
+        const int n0 = *n_tiles;
+        if (n0 < 0 || n0 > max_routed) {   // inconsistent count: leave the table alone
+            if (threadIdx.x == 0) report(st, MOEVIE_ERR_DEVICE, SITE_GEMM_TILES, n0, -2);
+            return;
+        }
+        const int64_t mt = (T + GM_BM - 1) / GM_BM;
+        for (int64_t j = threadIdx.x; j < S * mt; j += blockDim.x) {
+            const int c = (int)(j / mt);
+            const int64_t r0 = (j - (int64_t)c * mt) * GM_BM;
+            const int64_t nr = T - r0 < GM_BM ? T - r0 : GM_BM;
+            tiles[n0 + j] = make_int4(E + c, (int)(base + (int64_t)c * T + r0), (int)nr, 0);
+        }
+        __syncthreads();   // every thread of the block has read *n_tiles
+        if (threadIdx.x == 0) *n_tiles = n0 + (int)(S * mt);
+    }
+}
+
 int grid_for(int64_t n, int threads) {
     int64_t g = (n + threads - 1) / threads;
     if (g > 152 * 16) g = 152 * 16;
@@ -109,6 +141,16 @@ cudaError_t launch_f32_to_bf16(const float* src, __nv_bfloat16* dst, int64_t n, 
     const cudaError_t e = launch_pdl(f32_to_bf16_kernel, dim3(grid_for(n8, 256)), dim3(256), 0, s,
                                      reinterpret_cast<const float4*>(src), reinterpret_cast<uint4*>(dst),
                                      n8);
+    count_launches(1);
+    return e;
+}
+
+cudaError_t launch_shared_rows(int64_t T, int64_t base, int S, int E, float lambda,
+                               int32_t* row_tok, float* row_gate, int4* tiles, int32_t* n_tiles,
+                               int64_t max_routed, DevStatus* st, cudaStream_t s) {
+    const cudaError_t e = launch_pdl(shared_rows_kernel, dim3(grid_for(T * S, 256)), dim3(256), 0, s, T,
+                                     base, S, E, lambda, row_tok, row_gate, tiles, n_tiles,
+                                     max_routed, st);
     count_launches(1);
     return e;
 }

@@ -43,6 +43,8 @@ def _check_routing(lay, rt, tokens=None):
 @pytest.mark.parametrize("T,d,E,k,h,hs", [
     (1, 64, 4, 2, 64, 0), (130, 128, 8, 2, 128, 0), (257, 256, 16, 4, 416, 0),
     (200, 128, 8, 8, 64, 0), (100, 96, 4, 1, 48, 0), (300, 128, 16, 4, 96, 256),
+    # h divides h_s: the shared expert runs as h_s / h always-on groups of the grouped GEMMs
+    (1, 64, 4, 2, 64, 64), (300, 128, 16, 4, 128, 256), (257, 64, 8, 2, 64, 192),
 ])
 def test_forward_small(T, d, E, k, h, hs):
     cfg = workloads.small_config(T, d, E, k, h, h_s=hs, lam=0.5 if hs else 1.0, seed=T + h)
