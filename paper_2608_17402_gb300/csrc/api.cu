@@ -611,8 +611,11 @@ static moevie_status forward_impl(const moevie_layer* Lr, const void* x, int64_t
     MV_TRY(mark(1));
     // 2. expert-major order (Algorithm 1, phase 1), per-row token and gate, m-tile table
     const int chunk = perm_chunk(T * k, num_sms());
+    // (with the shared expert's always-on groups appended: rows, gates lambda, m-tiles)
+    const SharedRows sh{(int)S, T, Lr->lambda};
     MV_TRY(launch_permute(idx, T * k, (int)k, (int)E, GM_BM, chunk, gate, at<int32_t>(ws, L.hist),
-                          counts, offsets, tiles, n_tiles, perm, inv, row_tok, row_gate, st, s));
+                          counts, offsets, tiles, n_tiles, perm, inv, row_tok, row_gate, st, s,
+                          S > 0 ? &sh : nullptr));
     int dBN = 0, dnt = 0;
     choose_bn((int)d, &dBN, &dnt);
     const BandPlan bp = choose_bands(T, d, E, k, h);
@@ -622,13 +625,10 @@ static moevie_status forward_impl(const moevie_layer* Lr, const void* x, int64_t
                                  (int)max_mtiles(T * k, E), at<int4>(ws, L.items),
                                  at<int32_t>(ws, L.n_items), s));
     MV_TRY(mark(2));
-    // 3. shared expert (Eq. 3): S always-on groups of the grouped GEMMs (rows, gates
-    // lambda and m-tiles appended after the routed ones); otherwise its own GEMMs write
-    // lambda * shared expert as the first value of the y accumulator
-    if (S > 0) {
-        MV_TRY(launch_shared_rows(T, T * k, (int)S, (int)E, Lr->lambda, row_tok, row_gate, tiles,
-                                  n_tiles, max_mtiles(T * k, E), st, s));
-    } else if (hs > 0) {
+    // 3. shared expert (Eq. 3): S always-on groups of the grouped GEMMs (appended by the
+    // permute step); otherwise its own GEMMs write lambda * shared expert as the first
+    // value of the y accumulator
+    if (S == 0 && hs > 0) {
         c = shared_expert(x, Lr->Ws1, Lr->Ws2, T, d, hs, nullptr, yacc, Lr->lambda, L, ws, st, s);
         if (c != MOEVIE_OK) return c;
     }

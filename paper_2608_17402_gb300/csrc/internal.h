@@ -85,13 +85,22 @@ constexpr int PERM_CHUNK_MAX = 4096;   // flat slots per CTA of the histogram / 
 // Slots per CTA for n flat slots on num_sms SMs (multiple of 256, <= PERM_CHUNK_MAX).
 int perm_chunk(int64_t n, int num_sms);
 
+// Always-on groups appended to the permuted rows: S groups E .. E + S - 1 of T rows
+// each (row n_slots + c T + t: token t, gate lambda).
+struct SharedRows {
+    int S;
+    int64_t T;
+    float lambda;
+};
+
 // Stable expert-major order; also writes the m-tile table of the grouped GEMMs
-// (tiles[i] = {expert, first row, rows, 0}, *n_tiles = their number).
+// (tiles[i] = {expert, first row, rows, 0}, *n_tiles = their number), followed by the
+// tiles and rows of the always-on groups `sh` describes (none when sh is null).
 cudaError_t launch_permute(const int32_t* idx, int64_t n_slots, int k, int E, int bm, int chunk,
                            const float* gate_flat, int32_t* hist, int32_t* counts,
                            int32_t* offsets, int4* tiles, int32_t* n_tiles, int32_t* perm,
                            int32_t* inv, int32_t* row_tok, float* row_gate, DevStatus* st,
-                           cudaStream_t s);
+                           cudaStream_t s, const SharedRows* sh = nullptr);
 
 // m-tile table of `bm`-row tiles from given segment offsets [G + 1].
 cudaError_t launch_tile_table(const int32_t* offsets, int G, int bm, int4* tiles,

@@ -248,7 +248,7 @@ __global__ void __launch_bounds__(PT) perm_fused_kernel(
     const float* __restrict__ gate_flat, int32_t* __restrict__ hist, int32_t* __restrict__ counts,
     int32_t* __restrict__ offsets, int4* __restrict__ tiles, int32_t* __restrict__ n_tiles,
     int32_t* __restrict__ perm, int32_t* __restrict__ inv, int32_t* __restrict__ row_tok,
-    float* __restrict__ row_gate, DevStatus* st) {
+    float* __restrict__ row_gate, DevStatus* st, int S, int64_t T, float lambda) {
     pdl_wait();
     namespace cg = cooperative_groups;
     cg::grid_group grid = cg::this_grid();
@@ -288,7 +288,15 @@ __global__ void __launch_bounds__(PT) perm_fused_kernel(
         }
         __shared__ int s_ttot;
         int tex = block_exclusive_scan_1024(tsum, &s_ttot);
-        if (threadIdx.x == 0) *n_tiles = s_ttot;
+        // the always-on groups' m-tiles follow the routed ones
+        const int64_t smt = S > 0 ? (T + bm - 1) / bm : 0;
+        for (int64_t j = threadIdx.x; j < S * smt; j += PT) {
+            const int c = (int)(j / smt);
+            const int64_t r0 = (j - (int64_t)c * smt) * bm;
+            tiles[s_ttot + j] = make_int4(E + c, (int)(n + (int64_t)c * T + r0),
+                                          (int)(T - r0 < bm ? T - r0 : bm), 0);
+        }
+        if (threadIdx.x == 0) *n_tiles = s_ttot + (int)(S * smt);
 #pragma unroll
         for (int q = 0; q < 4; ++q) {
             const int g = 4 * threadIdx.x + q;
@@ -299,6 +307,10 @@ __global__ void __launch_bounds__(PT) perm_fused_kernel(
     }
     perm_scatter_body(idx, n, k, E, chunk, blockIdx.x, nchunks, hist, s_off, gate_flat, perm, inv,
                       row_tok, row_gate, ps_smem);
+    for (int64_t i = (int64_t)blockIdx.x * PT + threadIdx.x; i < S * T; i += (int64_t)nchunks * PT) {
+        row_tok[n + i] = (int32_t)(i % T);   // always-on group c = i / T, token t = i % T
+        row_gate[n + i] = lambda;
+    }
 }
 
 // m-tile table from given offsets (one thread per group, E <= 1024).
@@ -434,8 +446,11 @@ cudaError_t launch_permute(const int32_t* idx, int64_t n_slots, int k, int E, in
                            const float* gate_flat, int32_t* hist, int32_t* counts,
                            int32_t* offsets, int4* tiles, int32_t* n_tiles, int32_t* perm,
                            int32_t* inv, int32_t* row_tok, float* row_gate, DevStatus* st,
-                           cudaStream_t s) {
+                           cudaStream_t s, const SharedRows* sh) {
     const int nchunks = (int)((n_slots + chunk - 1) / chunk);
+    int S = sh ? sh->S : 0;
+    int64_t T = sh ? sh->T : 0;
+    float lambda = sh ? sh->lambda : 0.f;
     const size_t smem = (size_t)(chunk + PW * E) * 4;
     static bool attr_set[64] = {};
     static int coop_ctas[64] = {};   // co-resident CTAs of perm_fused_kernel (0: no cooperative launch)
@@ -462,7 +477,8 @@ cudaError_t launch_permute(const int32_t* idx, int64_t n_slots, int k, int E, in
         void* args[] = {(void*)&idx, (void*)&n_slots, (void*)&k, (void*)&E, (void*)&bm,
                         (void*)&chunk, (void*)&gate_flat, (void*)&hist, (void*)&counts,
                         (void*)&offsets, (void*)&tiles, (void*)&n_tiles, (void*)&perm, (void*)&inv,
-                        (void*)&row_tok, (void*)&row_gate, (void*)&st};
+                        (void*)&row_tok, (void*)&row_gate, (void*)&st, (void*)&S, (void*)&T,
+                        (void*)&lambda};
         err = cudaLaunchCooperativeKernel((const void*)perm_fused_kernel, dim3(nchunks), dim3(PT), args,
                                           smem, s);
         count_launches(1);
@@ -481,6 +497,9 @@ cudaError_t launch_permute(const int32_t* idx, int64_t n_slots, int k, int E, in
                      (const int32_t*)hist, (const int32_t*)offsets, gate_flat, perm, inv, row_tok,
                      row_gate);
     count_launches(4);
+    if (err == cudaSuccess && S > 0)
+        err = launch_shared_rows(T, n_slots, S, E, lambda, row_tok, row_gate, tiles, n_tiles,
+                                 max_mtiles(n_slots, E), st, s);
     return err;
 }
 
