@@ -195,6 +195,9 @@ struct GemmSpec {
     float* zero;             // dense A: also clear zero[0, zero_n) (zero_n % 4 == 0)
     int64_t zero_n;
     float* nrm_out;          // dense A: also nrm_out[r] = |A[r, 0:K_A]| (K_A = a_cols or K)
+    const float* wn_part;    // dense A: also wn_out[e] = sqrt(sum_p wn_part[p wn_Ep + e])
+    int wn_nparts, wn_E, wn_Ep;
+    float* wn_out;
     const void* W2nd;        // groups g >= g_split: weights at W2nd + (g - g_split) w2_g_ld +
     int64_t w2_k_ld;         //   kk w2_k_ld + n (elements); W then holds g_split groups
     int64_t w2_g_ld;
@@ -239,6 +242,14 @@ moevie_status run_gemm(const GemmSpec& g, DevStatus* st, cudaStream_t s) {
         a.nrm_ld = g.lda;
         a.nrm_cols = (int)cols;
         a.nrm_out = g.nrm_out;
+    }
+    if (g.wn_out) {
+        if (g.a_rows || g.wn_E <= 0 || g.wn_Ep < g.wn_E || g.wn_nparts < 1) return MOEVIE_ERR_UNSUPPORTED;
+        a.wn_part = g.wn_part;
+        a.wn_nparts = g.wn_nparts;
+        a.wn_E = g.wn_E;
+        a.wn_Ep = g.wn_Ep;
+        a.wn_out = g.wn_out;
     }
     a.G = g.G;
     a.g_split = g.W2nd ? g.g_split : g.G;
@@ -288,7 +299,7 @@ moevie_status route_impl(const void* x, const float* W_r, const float* b, int64_
     // partial logits: ksplit arrays [T][Ep]; straight into logits_out when unsplit
     float* logits = (logits_out && ksplit == 1) ? logits_out : at<float>(ws, L.logits);
     const int64_t part_stride = T * Ep;
-    MV_TRY(launch_route_split(W_r, (int)d, (int)E, wsplit, wrt, at<float>(ws, L.wpart), wnorm, st, s));
+    MV_TRY(launch_route_split(W_r, (int)d, (int)E, wsplit, wrt, at<float>(ws, L.wpart), st, s));
     const int64_t dp = route_dpad((int)d);
     GemmSpec g{};
     g.A = x;
@@ -312,6 +323,13 @@ moevie_status route_impl(const void* x, const float* W_r, const float* b, int64_
     g.zero = zero_acc;   // fp32 [T][d] cleared by the GEMM's idle warps (or NULL)
     g.zero_n = T * d;
     g.nrm_out = logits_only ? nullptr : at<float>(ws, L.xnorm);   // |x_t| for the certificate
+    if (!logits_only) {   // |W_r[:, e]| for the certificate, from the split's partial sums
+        g.wn_part = at<float>(ws, L.wpart);
+        g.wn_nparts = route_split_parts((int)d);
+        g.wn_E = (int)E;
+        g.wn_Ep = Ep;
+        g.wn_out = wnorm;
+    }
     moevie_status c = run_gemm(g, st, s);
     if (c != MOEVIE_OK) return c;
     if (logits_only) {

@@ -710,7 +710,7 @@ __global__ void __launch_bounds__(GM_THREADS, 1) grouped_gemm_kernel(const __gri
         if ((threadIdx.x & 31) == 0 && gather) gather_forwarder(p, sm, n_work, abort_flag);
     } else if (gather) {
         producer_gather(p, sm, n_work, abort_flag);
-    } else if ((p.zero || p.nrm_out) && warp >= GM_WARP_GATHER && warp < GM_WARP_FWD) {
+    } else if ((p.zero || p.nrm_out || p.wn_out) && warp >= GM_WARP_GATHER && warp < GM_WARP_FWD) {
         // Side jobs for the gather warps of a dense-A GEMM, while the MMAs run.
         // 1. Row norms of the A rows of this CTA's items (the router's |x_t|, read while
         //    the TMA brings the same rows in): one warp per row, lanes over 16-byte chunks;
@@ -739,7 +739,19 @@ __global__ void __launch_bounds__(GM_THREADS, 1) grouped_gemm_kernel(const __gri
                 }
             }
         }
-        // 2. Clear another buffer (the y accumulator) with 16-byte stores, grid-strided
+        // 2. Column norms from per-CTA partial sums of squares: one warp per column,
+        //    lanes over the parts, then a fixed shuffle tree (deterministic).
+        if (p.wn_out) {
+            const int q = warp - GM_WARP_GATHER, lane = threadIdx.x & 31;
+            for (int e = blockIdx.x * GM_GATHER_WARPS + q; e < p.wn_E; e += gridDim.x * GM_GATHER_WARPS) {
+                float v = 0.f;
+                for (int pp = lane; pp < p.wn_nparts; pp += 32) v += p.wn_part[(int64_t)pp * p.wn_Ep + e];
+#pragma unroll
+                for (int o = 16; o; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+                if (lane == 0) p.wn_out[e] = sqrtf(v);
+            }
+        }
+        // 3. Clear another buffer (the y accumulator) with 16-byte stores, grid-strided
         //    (evict-first: the zeros must not push the GEMM's re-read operands out of L2).
         if (p.zero) {
             const uint4 z = make_uint4(0u, 0u, 0u, 0u);

@@ -30,6 +30,24 @@ cudaError_t launch_pdl(void (*kern)(KArgs...), dim3 grid, dim3 block, size_t sme
     cfg.numAttrs = 1;
     return cudaLaunchKernelEx(&cfg, kern, static_cast<KArgs>(args)...);
 }
+// The same for a cooperative launch (all CTAs co-resident; grid-wide barriers).
+template <typename... KArgs, typename... Args>
+cudaError_t launch_pdl_coop(void (*kern)(KArgs...), dim3 grid, dim3 block, size_t smem,
+                            cudaStream_t s, Args... args) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = grid;
+    cfg.blockDim = block;
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = s;
+    cudaLaunchAttribute at[2];
+    at[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    at[0].val.programmaticStreamSerializationAllowed = 1;
+    at[1].id = cudaLaunchAttributeCooperative;
+    at[1].val.cooperative = 1;
+    cfg.attrs = at;
+    cfg.numAttrs = 2;
+    return cudaLaunchKernelEx(&cfg, kern, static_cast<KArgs>(args)...);
+}
 
 // ----------------------------------------------------------------- router
 
@@ -48,11 +66,12 @@ inline int route_dpad(int d) { return (d + 63) / 64 * 64; }
 
 // W_r fp32 [d, E] -> three bf16 pieces [3][d_pad][E_pad] with W_r = hi + mid + lo
 // exactly (zero in the padding rows and columns), the transposed fp32 copy
-// wrt [E][d_pad] (zero rows past d), and |W_r[:, e]| (wpart: route_split_parts(d) x
-// E_pad floats of scratch).  Also clears the fallback counter in st (may be NULL).
+// wrt [E][d_pad] (zero rows past d), and per-CTA partial sums of squares of W_r's
+// columns (wpart: route_split_parts(d) x E_pad floats; |W_r[:, e]| is the square root
+// of their sum over the parts).  Also clears the fallback counter in st (may be NULL).
 int route_split_parts(int d);
 cudaError_t launch_route_split(const float* Wr, int d, int E, __nv_bfloat16* Wsplit, float* wrt,
-                               float* wpart, float* wnorm, DevStatus* st, cudaStream_t s);
+                               float* wpart, DevStatus* st, cudaStream_t s);
 
 // Splits of K for the router GEMM: enough CTA-pair work items for about
 // ROUTE_SPLIT_TARGET items, at most ROUTE_MAX_KSPLIT, at least three K blocks each.
@@ -203,6 +222,9 @@ struct GemmArgs {
     int64_t nrm_ld;             //   every n-tile-0 item, nrm_out[r] = |nrm_x[r, 0:nrm_cols]|
     int nrm_cols;               //   (nrm_cols % 8 == 0)
     float* nrm_out;
+    const float* wn_part;       // dense A only: the idle gather warps also write
+    int wn_nparts, wn_E, wn_Ep; //   wn_out[e] = sqrt(sum_p wn_part[p wn_Ep + e]), e < wn_E
+    float* wn_out;              //   (the router's |W_r[:, e]| from per-CTA partial sums)
     DevStatus* status;
     uint64_t limit_ns;
 };

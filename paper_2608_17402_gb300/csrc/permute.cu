@@ -474,13 +474,9 @@ cudaError_t launch_permute(const int32_t* idx, int64_t n_slots, int k, int E, in
         attr_set[dev] = true;
     }
     if (dev >= 0 && dev < 64 && nchunks <= coop_ctas[dev]) {
-        void* args[] = {(void*)&idx, (void*)&n_slots, (void*)&k, (void*)&E, (void*)&bm,
-                        (void*)&chunk, (void*)&gate_flat, (void*)&hist, (void*)&counts,
-                        (void*)&offsets, (void*)&tiles, (void*)&n_tiles, (void*)&perm, (void*)&inv,
-                        (void*)&row_tok, (void*)&row_gate, (void*)&st, (void*)&S, (void*)&T,
-                        (void*)&lambda};
-        err = cudaLaunchCooperativeKernel((const void*)perm_fused_kernel, dim3(nchunks), dim3(PT), args,
-                                          smem, s);
+        err = launch_pdl_coop(perm_fused_kernel, dim3(nchunks), dim3(PT), smem, s, idx, n_slots, k, E,
+                              bm, chunk, gate_flat, hist, counts, offsets, tiles, n_tiles, perm, inv,
+                              row_tok, row_gate, st, S, T, lambda);
         count_launches(1);
         return err;
     }

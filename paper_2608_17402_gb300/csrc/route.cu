@@ -9,8 +9,9 @@
 // (route_ksplit) and each split writes its own fp32 partial logits; they are summed
 // in a fixed order.  This file holds the steps around that GEMM:
 //
-//  1. route_split_kernel / route_wnorm_kernel: the three pieces, an fp32 copy of
-//     W_r transposed to [E][d_pad] (read by the exact re-decision), and |W_r[:, e]|.
+//  1. route_split_kernel: the three pieces, an fp32 copy of W_r transposed to
+//     [E][d_pad] (read by the exact re-decision), and per-CTA partial sums of squares
+//     of W_r's columns (the router GEMM's idle warps finish |W_r[:, e]| from them).
 //  2. route_topk_kernel: one warp per token; the partial logits summed, keys
 //     sigmoid(s) + b, k rounds of warp arg-max (ties to the lower id), and a
 //     certificate.  Every expert's key lies in
@@ -82,22 +83,6 @@ __global__ void __launch_bounds__(256) route_split_kernel(const float* __restric
         const int ee = blockIdx.x * SPLIT_TILE + r;
         if (ee < E) wrt[(int64_t)ee * dp + i0 + tx] = tile[tx][r];
     }
-}
-
-// |W_r[:, e]| from the per-CTA partial sums: one warp per expert, lanes over parts,
-// then a fixed shuffle tree (deterministic).
-__global__ void __launch_bounds__(256) route_wnorm_kernel(const float* __restrict__ wpart,
-                                                          int nparts, int E, int Ep,
-                                                          float* __restrict__ wnorm) {
-    pdl_wait();
-    const int lane = threadIdx.x & 31;
-    const int e = (int)(((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5);
-    if (e >= E) return;
-    float v = 0.f;
-    for (int p = lane; p < nparts; p += 32) v += wpart[(int64_t)p * Ep + e];
-#pragma unroll
-    for (int o = 16; o; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
-    if (lane == 0) wnorm[e] = sqrtf(v);
 }
 
 // Fast sigmoid: __expf (ex2.approx) and __fdividef.  For the keys compared below
@@ -487,14 +472,12 @@ int64_t route_logits_rows(int64_t T, int d, int E) {
 }
 
 cudaError_t launch_route_split(const float* Wr, int d, int E, __nv_bfloat16* Wsplit, float* wrt,
-                               float* wpart, float* wnorm, DevStatus* st, cudaStream_t s) {
+                               float* wpart, DevStatus* st, cudaStream_t s) {
     const int Ep = route_epad(E);
     const int parts = route_split_parts(d);
     cudaError_t e = launch_pdl(route_split_kernel, dim3((Ep + SPLIT_TILE - 1) / SPLIT_TILE, parts),
                                dim3(256), 0, s, Wr, d, route_dpad(d), E, Ep, Wsplit, wrt, wpart, st);
-    if (e != cudaSuccess) return e;
-    e = launch_pdl(route_wnorm_kernel, dim3((E + 7) / 8), dim3(256), 0, s, wpart, parts, E, Ep, wnorm);
-    count_launches(2);
+    count_launches(1);
     return e;
 }
 
