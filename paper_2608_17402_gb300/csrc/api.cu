@@ -279,6 +279,7 @@ moevie_status run_gemm(const GemmSpec& g, DevStatus* st, cudaStream_t s) {
         a.max_mtiles *= a.n_ntiles;   // bound on the item count
     }
     const int64_t work = a.item_table ? a.max_mtiles : a.max_mtiles * a.n_ntiles * a.ksplit;   // one CTA pair per item at most
+    if (work >= (int64_t(1) << 31)) return MOEVIE_ERR_UNSUPPORTED;   // item indices are 32-bit in the kernel
     const int sms = num_sms() & ~1;
     const int grid = (int)(2 * work < sms ? (work > 0 ? 2 * work : 2) : sms);
     return cuda_status(launch_grouped_gemm(a, grid, s));

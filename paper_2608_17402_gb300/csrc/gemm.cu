@@ -149,18 +149,43 @@ struct Tile {
     int ks;         // split index
 };
 
-__device__ __forceinline__ Tile decode_tile(const GemmArgs& p, int64_t w) {
+// A work item's table entry, loaded but not yet checked.  The roles that walk the
+// items load the entry of an item one item ahead (tile_load) and check it when the
+// item starts (tile_finish), so that no role waits on that load at an item boundary.
+struct TileLd {
+    int4 d;   // table entry (unused for one dense group)
+    int ks;   // split of K
+    int q;    // item index without the split: table entry (item table) or m-tile x n-tile
+};
+
+// Work-item counts stay far below 2^31 (m-tiles x n-tiles x K splits), so item indices
+// are split with 32-bit arithmetic, each division done once.
+__device__ __forceinline__ TileLd tile_load(const GemmArgs& p, int64_t w64) {
+    TileLd l;
+    const int w = (int)w64;
+    l.q = w / p.ksplit;   // split of K fastest
+    l.ks = w - l.q * p.ksplit;
+    if (p.item_table) l.d = __ldg(p.tiles + l.q);
+    else if (p.tiles) l.d = __ldg(p.tiles + l.q / p.n_ntiles);
+    else l.d = make_int4(0, 0, 0, 0);
+    return l;
+}
+
+// k-blocks [kb0, kb1) of split ks of K.
+__device__ __forceinline__ void tile_kb(const GemmArgs& p, int ks, int& kb0, int& kb1) {
+    kb0 = (int)((int64_t)ks * p.num_kb / p.ksplit);
+    kb1 = (int)((int64_t)(ks + 1) * p.num_kb / p.ksplit);
+}
+
+__device__ __forceinline__ Tile tile_finish(const GemmArgs& p, const TileLd& l) {
     Tile t;
-    t.ks = (int)(w % p.ksplit);   // split of K fastest
-    w /= p.ksplit;
-    t.kb0 = (int)((int64_t)t.ks * p.num_kb / p.ksplit);
-    t.kb1 = (int)((int64_t)(t.ks + 1) * p.num_kb / p.ksplit);
+    t.ks = l.ks;
+    tile_kb(p, l.ks, t.kb0, t.kb1);
     if (p.item_table) {   // an explicit (m-tile, n-tile) item
-        const int4 d = __ldg(p.tiles + w);
-        t.g = d.x;
-        t.row0 = d.y;
-        t.nrows = d.z;
-        t.n0 = d.w;
+        t.g = l.d.x;
+        t.row0 = l.d.y;
+        t.nrows = l.d.z;
+        t.n0 = l.d.w;
         if (t.nrows < 0 || t.nrows > GM_BM || t.g < 0 || t.g >= p.G || t.n0 < 0 || t.n0 >= p.N ||
             (int64_t)t.row0 + t.nrows > p.m_total) {
             report(p.status, MOEVIE_ERR_DEVICE, SITE_GEMM_TILES, t.row0, t.nrows);
@@ -170,13 +195,12 @@ __device__ __forceinline__ Tile decode_tile(const GemmArgs& p, int64_t w) {
         }
         return t;
     }
-    const int mt = (int)(w / p.n_ntiles);
-    const int nt = (int)(w - (int64_t)mt * p.n_ntiles);
+    const int mt = l.q / p.n_ntiles;
+    const int nt = l.q - mt * p.n_ntiles;
     if (p.tiles) {
-        const int4 d = __ldg(p.tiles + mt);
-        t.g = d.x;
-        t.row0 = d.y;
-        t.nrows = d.z;
+        t.g = l.d.x;
+        t.row0 = l.d.y;
+        t.nrows = l.d.z;
     } else {   // one dense group of m_total rows
         t.g = 0;
         t.row0 = mt * GM_BM;
@@ -191,6 +215,10 @@ __device__ __forceinline__ Tile decode_tile(const GemmArgs& p, int64_t w) {
     }
     t.n0 = nt * p.BN;
     return t;
+}
+
+__device__ __forceinline__ Tile decode_tile(const GemmArgs& p, int64_t w) {
+    return tile_finish(p, tile_load(p, w));
 }
 
 // GELU(u) = u/2 (1 + erf(u / sqrt 2)) = max(u, 0) - |u|/2 erfc(|u| / sqrt 2), the
@@ -251,11 +279,12 @@ __device__ __forceinline__ int rows_half(const Tile& t, uint32_t rank) {
 
 // TMA producer (warp 9, lane 0): the CTA's half of B, and A when its rows are
 // contiguous.  The leader posts the byte count of both CTAs on its full barrier.
+template <bool GATHER>
 __device__ void producer_tma(const GemmArgs& p, const Smem& sm, int64_t n_work,
                              volatile int* abort_flag) {
     tma_prefetch_desc(&p.tmB);
     if (p.g_split < p.G) tma_prefetch_desc(&p.tmB2);
-    const bool gather = p.a_rows != nullptr;
+    constexpr bool gather = GATHER;
     if (!gather) tma_prefetch_desc(&p.tmA);
     const uint32_t half_n = (uint32_t)p.BN / 2;
     const uint32_t nboxh = (half_n + 63) / 64;
@@ -270,8 +299,8 @@ __device__ void producer_tma(const GemmArgs& p, const Smem& sm, int64_t n_work,
     if (w < n_work) t = decode_tile(p, w);
     for (; w < n_work; w += sm.npairs) {
         const int64_t wn = w + sm.npairs;
-        Tile tn{};
-        if (wn < n_work) tn = decode_tile(p, wn);
+        TileLd nl{};
+        if (wn < n_work) nl = tile_load(p, wn);   // checked after this item's loads
         const bool second = t.g >= p.g_split;   // B of this group from the second map
         const CUtensorMap* tmb = second ? &p.tmB2 : &p.tmB;
         const int gb = second ? t.g - p.g_split : t.g;
@@ -297,31 +326,39 @@ __device__ void producer_tma(const GemmArgs& p, const Smem& sm, int64_t n_work,
                 ph ^= 1u;
             }
         }
-        t = tn;
+        if (wn < n_work) t = tile_finish(p, nl);
     }
 }
 
-// A row pointers of this thread's GM_GATHER_ROWS rows (r = rb + GM_GATHER_RSTEP j of the
-// CTA's half).
-__device__ __forceinline__ void gather_rows(const GemmArgs& p, const Tile& t, uint32_t rank,
-                                            int rb, const __nv_bfloat16* (&src)[GM_GATHER_ROWS]) {
+// Table rows of this thread's GM_GATHER_ROWS rows of tile t (r = rb + GM_GATHER_RSTEP j of
+// the CTA's half; -1 past the tile), loaded one item ahead of their use.
+__device__ __forceinline__ void gather_rows_load(const GemmArgs& p, const Tile& t, uint32_t rank,
+                                                 int rb, int (&raw)[GM_GATHER_ROWS]) {
     const int nh = rows_half(t, rank);
-    int idx[GM_GATHER_ROWS];
 #pragma unroll
     for (int j = 0; j < GM_GATHER_ROWS; ++j) {
         const int r = rb + GM_GATHER_RSTEP * j;
         const int gr = t.row0 + (int)rank * GM_HALF + r;
-        idx[j] = (r < nh) ? __ldg(p.a_rows + gr) / p.a_div : -1;
+        raw[j] = (r < nh) ? __ldg(p.a_rows + gr) : -1;
     }
+}
+
+// A row pointers from the loaded table rows (nullptr past the tile; an A row outside
+// [0, a_nrows) is a device error and is not read).
+__device__ __forceinline__ void gather_rows_finish(const GemmArgs& p, const Tile& t, uint32_t rank,
+                                                   int rb, const int (&raw)[GM_GATHER_ROWS],
+                                                   const __nv_bfloat16* (&src)[GM_GATHER_ROWS]) {
+    const int nh = rows_half(t, rank);
 #pragma unroll
     for (int j = 0; j < GM_GATHER_ROWS; ++j) {
         const int r = rb + GM_GATHER_RSTEP * j;
-        if (r < nh && idx[j] >= 0 && idx[j] < p.a_nrows) {
-            src[j] = p.A + (int64_t)idx[j] * p.lda;
+        const int idx = r < nh ? raw[j] / p.a_div : -1;
+        if (r < nh && idx >= 0 && idx < p.a_nrows) {
+            src[j] = p.A + (int64_t)idx * p.lda;
         } else {
             if (r < nh)
                 report(p.status, MOEVIE_ERR_DEVICE, SITE_GEMM_A_ROW, t.row0 + (int)rank * GM_HALF + r,
-                       idx[j]);
+                       idx);
             src[j] = nullptr;
         }
     }
@@ -343,20 +380,26 @@ __device__ void producer_gather(const GemmArgs& p, const Smem& sm, int64_t n_wor
     uint32_t ph = 0;
     bool ok = true;
     int64_t w = sm.pair;
+    // The per-item set-up is pipelined so that no load is waited on at an item start:
+    // item w's row pointers are ready when it starts; the next item's table rows were
+    // loaded one item earlier, after its tile entry (loaded earlier still) was checked.
     const __nv_bfloat16* src[GM_GATHER_ROWS];
-    Tile t{};
+    int nraw[GM_GATHER_ROWS];
+    Tile t{}, tn{};
+    TileLd nnl{};
     if (w < n_work) {
         t = decode_tile(p, w);
-        gather_rows(p, t, sm.rank, rb, src);
+        int raw[GM_GATHER_ROWS];
+        gather_rows_load(p, t, sm.rank, rb, raw);
+        gather_rows_finish(p, t, sm.rank, rb, raw, src);
     }
+    if (w + sm.npairs < n_work) {
+        tn = decode_tile(p, w + sm.npairs);
+        gather_rows_load(p, tn, sm.rank, rb, nraw);
+    }
+    if (w + 2 * sm.npairs < n_work) nnl = tile_load(p, w + 2 * sm.npairs);
     for (; w < n_work && ok; w += sm.npairs) {
         const int64_t wn = w + sm.npairs;
-        const __nv_bfloat16* nsrc[GM_GATHER_ROWS];
-        Tile tn{};
-        if (wn < n_work) {
-            tn = decode_tile(p, wn);
-            gather_rows(p, tn, sm.rank, rb, nsrc);
-        }
         for (int kb = t.kb0; kb < t.kb1; ++kb) {
             int good = 1;
             if (lane == 0) good = mbar_wait(sm.empty + 8 * s, ph ^ 1u, p.limit_ns, abort_flag);
@@ -383,11 +426,15 @@ __device__ void producer_gather(const GemmArgs& p, const Smem& sm, int64_t n_wor
                 ph ^= 1u;
             }
         }
-        if (wn < n_work) {
-#pragma unroll
-            for (int j = 0; j < GM_GATHER_ROWS; ++j) src[j] = nsrc[j];
+        if (wn < n_work) {   // advance: item wn's pointers, item wn + npairs's table rows
+            gather_rows_finish(p, tn, sm.rank, rb, nraw, src);
+            t = tn;
+            if (wn + sm.npairs < n_work) {
+                tn = tile_finish(p, nnl);
+                gather_rows_load(p, tn, sm.rank, rb, nraw);
+                if (wn + 2 * sm.npairs < n_work) nnl = tile_load(p, wn + 2 * sm.npairs);
+            }
         }
-        t = tn;
     }
     cp_async_wait_all();
 }
@@ -407,8 +454,9 @@ __device__ void gather_forwarder(const GemmArgs& p, const Smem& sm, int64_t n_wo
     int s = 0;
     uint32_t ph = 0;
     for (int64_t w = sm.pair; w < n_work; w += sm.npairs) {
-        const Tile t = decode_tile(p, w);
-        for (int kb = t.kb0; kb < t.kb1; ++kb) {
+        int kb0, kb1;   // the item's stages; its table entry is not needed here
+        tile_kb(p, (int)(w % p.ksplit), kb0, kb1);
+        for (int kb = kb0; kb < kb1; ++kb) {
             if (!mbar_wait(sm.afull + 8 * s, ph, p.limit_ns, abort_flag)) {
                 set_abort(abort_flag, p.status, SITE_GEMM_WAIT_FULL, (int)sm.pair, -1 - kb);
                 return;
@@ -438,11 +486,11 @@ __device__ void mma_issuer(const GemmArgs& p, const Smem& sm, uint32_t tmem, int
     uint32_t ph = 0;
     int it = 0;
     bool issued = false;
-    Tile tn{};   // next item's tile, decoded one item ahead (its table read is a global load)
-    if (sm.pair < n_work) tn = decode_tile(p, sm.pair);
+    TileLd nl{};   // next item's table entry, loaded one item ahead, checked when it starts
+    if (sm.pair < n_work) nl = tile_load(p, sm.pair);
     for (int64_t w = sm.pair; w < n_work; w += sm.npairs, ++it) {
-        const Tile t = tn;
-        if (w + sm.npairs < n_work) tn = decode_tile(p, w + sm.npairs);
+        const Tile t = tile_finish(p, nl);
+        if (w + sm.npairs < n_work) nl = tile_load(p, w + sm.npairs);
         const int acc = it & 1;
         const uint32_t aph = (uint32_t)(it >> 1) & 1u;
         if (!mbar_wait(sm.tempty + 8 * acc, aph ^ 1u, p.limit_ns, abort_flag)) {
@@ -530,7 +578,7 @@ __device__ __forceinline__ void reduce_chunk(const GemmArgs& p, float* stg_all, 
 // per-warp staging buffer so that each 16-byte vector reduction instruction of a
 // warp covers four rows x 128 contiguous bytes, i.e. whole L2 lines.  When a warp has read
 // its last chunk of the accumulator it arrives (once) on the leader's tempty barrier.
-template <int STG_ROWS>
+template <int STG_ROWS, bool GATHER>
 __device__ void epilogue(const GemmArgs& p, const Smem& sm, uint32_t tmem, int64_t n_work,
                          volatile int* abort_flag) {
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -571,7 +619,7 @@ __device__ void epilogue(const GemmArgs& p, const Smem& sm, uint32_t tmem, int64
         }
         for (int ch = half; ch < nchunk; ch += 2) {
             const int c0 = ch * 32;
-            if (p.epi == EPI_ADD_F32) {
+            if (!GATHER && p.epi == EPI_ADD_F32) {   // (a gathered GEMM never reduces)
                 uint32_t v[32];
                 tmem_ld_32x32b_x32(tbase + c0, v);
                 tmem_wait_ld();
@@ -630,7 +678,7 @@ __device__ void epilogue(const GemmArgs& p, const Smem& sm, uint32_t tmem, int64
 
 // STG_ROWS: rows per warp of the reduction staging buffer (EPI_ADD_F32), one kernel
 // instance each so that the epilogue loops have constant trip counts.
-template <int STG_ROWS>
+template <int STG_ROWS, bool GATHER>
 __global__ void __launch_bounds__(GM_THREADS, 1) grouped_gemm_kernel(const __grid_constant__ GemmArgs p) {
     extern __shared__ uint8_t gm_smem_raw[];
     uint8_t* smem = reinterpret_cast<uint8_t*>(
@@ -661,7 +709,7 @@ __global__ void __launch_bounds__(GM_THREADS, 1) grouped_gemm_kernel(const __gri
     sm.npairs = gridDim.x >> 1;
 
     const int warp = threadIdx.x >> 5;
-    const bool gather = p.a_rows != nullptr;
+    constexpr bool gather = GATHER;   // A rows gathered by the gather warps (else TMA)
     if (threadIdx.x == 0) {
         for (int s = 0; s < nst; ++s) {
             // leader's expect_tx arrival (+ the leader's forwarder; the peer's signals
@@ -701,14 +749,16 @@ __global__ void __launch_bounds__(GM_THREADS, 1) grouped_gemm_kernel(const __gri
     const int64_t n_work = p.item_table ? n_mtiles * p.ksplit : n_mtiles * p.n_ntiles * p.ksplit;
 
     if (warp < GM_EPI_WARPS) {
-        epilogue<STG_ROWS>(p, sm, tmem, n_work, abort_flag);
+        epilogue<STG_ROWS, GATHER>(p, sm, tmem, n_work, abort_flag);
     } else if (warp == GM_WARP_MMA) {
         if ((threadIdx.x & 31) == 0 && sm.rank == 0) mma_issuer(p, sm, tmem, n_work, abort_flag);
     } else if (warp == GM_WARP_LOAD) {
-        if ((threadIdx.x & 31) == 0) producer_tma(p, sm, n_work, abort_flag);
+        if ((threadIdx.x & 31) == 0) producer_tma<GATHER>(p, sm, n_work, abort_flag);
     } else if (warp == GM_WARP_FWD) {
-        if ((threadIdx.x & 31) == 0 && gather) gather_forwarder(p, sm, n_work, abort_flag);
-    } else if (gather) {
+        if constexpr (GATHER) {
+            if ((threadIdx.x & 31) == 0) gather_forwarder(p, sm, n_work, abort_flag);
+        }
+    } else if constexpr (GATHER) {
         producer_gather(p, sm, n_work, abort_flag);
     } else if ((p.zero || p.nrm_out || p.wn_out) && warp >= GM_WARP_GATHER && warp < GM_WARP_FWD) {
         // Side jobs for the gather warps of a dense-A GEMM, while the MMAs run.
@@ -828,12 +878,18 @@ void choose_bn(int N, int* BN, int* n_ntiles) {
 
 cudaError_t launch_grouped_gemm(const GemmArgs& a, int grid, cudaStream_t s) {
     if (a.stg_rows != 32 && a.stg_rows != 16) return cudaErrorInvalidValue;
-    auto* kern = a.stg_rows == 32 ? grouped_gemm_kernel<32> : grouped_gemm_kernel<16>;
+    // one instance per staging size (dense A) and one for gathered A (which never
+    // reduces): constant trip counts in the epilogue, and no code of the other mode
+    using Kern = void (*)(GemmArgs);
+    static const Kern kerns[3] = {grouped_gemm_kernel<32, false>, grouped_gemm_kernel<16, false>,
+                                  grouped_gemm_kernel<32, true>};
+    if (a.a_rows && a.epi == EPI_ADD_F32) return cudaErrorInvalidValue;
+    const Kern kern = a.a_rows ? kerns[2] : a.stg_rows == 32 ? kerns[0] : kerns[1];
     static bool attr_set[64] = {};
     int dev = 0;
     cudaGetDevice(&dev);
     if (dev >= 0 && dev < 64 && !attr_set[dev]) {
-        for (auto* k : {grouped_gemm_kernel<32>, grouped_gemm_kernel<16>}) {
+        for (Kern k : kerns) {
             cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                                  GM_SMEM_BYTES_MAX);
             if (e != cudaSuccess) return e;
