@@ -84,8 +84,10 @@ def captured_traffic(cfg_name, stage):
     return None if per is None else float(per["dram_bytes"])
 
 
-def layer_work(cfg, counts):
-    """Algorithmic FLOPs and bytes of one layer forward (weights of touched experts)."""
+def layer_work(cfg, counts, shared_groups=0):
+    """Algorithmic FLOPs and bytes of one layer forward (weights of touched experts).
+    shared_groups: always-on groups of width h that carry the shared expert inside the
+    routed up / down launches (moevie_shared_groups), counted in those launches' FLOPs."""
     T, d, E, k, h, hs = cfg.T, cfg.d, cfg.E, cfg.k, cfg.h, cfg.h_s
     flops_router = 2.0 * T * d * E
     flops_experts = 4.0 * T * k * d * h
@@ -93,8 +95,10 @@ def layer_work(cfg, counts):
     touched = int((np.asarray(counts) > 0).sum())
     bytes_ = (T * d * 2 + T * d * 2 + d * E * 4 + E * 4 + touched * 2 * d * h * 2
               + 2 * d * hs * 2 + 8 * T * k)
-    return {"flops": flops_router + flops_experts + flops_shared, "flops_up_gemm": 2.0 * T * k * d * h,
-            "flops_down_gemm": 2.0 * T * k * d * h, "bytes": float(bytes_), "touched_experts": touched}
+    folded = shared_groups * h * T * d * 2.0
+    return {"flops": flops_router + flops_experts + flops_shared,
+            "flops_up_gemm": 2.0 * T * k * d * h + folded,
+            "flops_down_gemm": 2.0 * T * k * d * h + folded, "bytes": float(bytes_), "touched_experts": touched}
 
 
 class ClockSampler:
@@ -252,7 +256,7 @@ def run_ours(args, rank, world):
     code, detail = moevie.moevie_get_device_status(ws)
     if code != 0:
         raise RuntimeError(f"device status {code} {detail}")
-    work = layer_work(cfg, counts)
+    work = layer_work(cfg, counts, moevie.moevie_shared_groups(cfg.T, cfg.d, cfg.E, cfg.k, cfg.h, cfg.h_s))
 
     for _ in range(args.warmup):
         moevie.moevie_moe_forward(W, x, ws, y=y)

@@ -180,6 +180,15 @@ moevie_status moevie_permute_static(const int32_t* idx, int64_t T, int64_t k, in
  * threads, all devices).  Host-only. */
 uint64_t moevie_launch_count(void);
 
+/* Launch plan of moevie_moe_forward for these sizes (host-only, no GPU work; the
+ * paper has no counterpart -- it describes how this library schedules Eq. 6's
+ * shared term).  Returns the number S of always-on groups of width h that carry the
+ * shared expert inside the routed up- and down-projection launches (its hidden units
+ * in S = h_s / h chunks, every token with gate lambda), or 0 when it runs as its own
+ * two GEMMs (no shared expert, h not dividing h_s, or a band-ordered down-projection).
+ * Invalid sizes return 0. */
+int64_t moevie_shared_groups(int64_t T, int64_t d, int64_t E, int64_t k, int64_t h, int64_t h_s);
+
 /* Synchronise `stream`, then read the workspace's device status into *out
  * (MOEVIE_OK when no device-side error was recorded).  `detail` (host, may be
  * NULL) receives 4 ints: code, site, and two values describing the failure. */

@@ -75,8 +75,14 @@ BandPlan choose_bands(int64_t T, int64_t d, int64_t E, int64_t k, int64_t h) {
 // gate lambda, when h divides h_s and the down-projection is not band-ordered.
 // 0: the shared expert runs as its own dense GEMMs.
 constexpr int64_t SHARED_MAX_CHUNKS = 16;
+// Always-on groups the shapes allow (h divides h_s); the workspace reserves room for
+// them whatever the band decision, so that its size stays monotone in T.
+int64_t shared_chunks_max(int64_t h, int64_t hs) {
+    if (hs <= 0 || h <= 0 || hs % h != 0 || hs / h > SHARED_MAX_CHUNKS) return 0;
+    return hs / h;
+}
 int64_t shared_chunks(int64_t T, int64_t d, int64_t E, int64_t k, int64_t h, int64_t hs) {
-    if (hs <= 0 || h <= 0 || d <= 0 || T < 0 || hs % h != 0 || hs / h > SHARED_MAX_CHUNKS) return 0;
+    if (shared_chunks_max(h, hs) == 0 || d <= 0 || T < 0) return 0;
     if (T * (k + hs / h) >= (int64_t(1) << 31)) return 0;
     int BN = 0, nnt = 0;
     choose_bn((int)d, &BN, &nnt);
@@ -109,8 +115,10 @@ Layout make_layout(int64_t T, int64_t d, int64_t E, int64_t k, int64_t h, int64_
     L.hist = take(4 * nchunks_max * E);
     L.counts = take(4 * E);
     L.offsets = take(4 * (E + 1));
-    const int64_t S = shared_chunks(T, d, E, k, h, hs);
-    const int64_t n2 = n + S * T;   // GEMM rows: routed, then the shared groups'
+    // GEMM rows: routed, then the shared expert's always-on groups (room for them
+    // whenever h divides h_s, folded or not, so that the size is monotone in T)
+    const int64_t S = shared_chunks_max(h, hs);
+    const int64_t n2 = n + S * T;
     L.tiles = take(16 * (max_mtiles(n, E) + S * ((T + GM_BM - 1) / GM_BM)));
     int BN = 0, n_nt = 0;
     choose_bn((int)(d > 0 ? d : 1), &BN, &n_nt);
@@ -122,7 +130,9 @@ Layout make_layout(int64_t T, int64_t d, int64_t E, int64_t k, int64_t h, int64_
     L.row_tok = take(4 * n2);
     L.row_gate = take(4 * n2);
     L.H = take(2 * n2 * h);
-    L.Hs = take(S > 0 ? 0 : 2 * T * hs);
+    // the shared expert's own hidden [T, h_s]: with room for always-on groups it is the
+    // tail of H (those S T rows of width h, the same bytes), used by one path or the other
+    L.Hs = S > 0 ? L.H + (size_t)(2 * n * h) : take(2 * T * hs);
     L.yacc = take(4 * T * d);
     L.total = o;
     return L;
@@ -430,6 +440,11 @@ const char* moevie_status_string(moevie_status s) {
 int moevie_version(void) { return 200; }
 
 uint64_t moevie_launch_count(void) { return g_launches.load(std::memory_order_relaxed); }
+
+int64_t moevie_shared_groups(int64_t T, int64_t d, int64_t E, int64_t k, int64_t h, int64_t h_s) {
+    if (check_sizes(T, d, E, k, h, h_s) != MOEVIE_OK) return 0;
+    return shared_chunks(T, d, E, k, h, h_s);
+}
 
 moevie_status moevie_workspace_size(int64_t T_max, int64_t d, int64_t E, int64_t k, int64_t h,
                                     int64_t h_s, size_t* bytes) {

@@ -26,7 +26,8 @@ C_ENTRY_POINTS = ("moevie_status_string", "moevie_version", "moevie_workspace_si
                   "moevie_workspace_init", "moevie_route", "moevie_permute", "moevie_permute_static",
                   "moevie_expert_ffn",
                   "moevie_shared_expert", "moevie_combine", "moevie_moe_forward",
-                  "moevie_get_device_status", "moevie_launch_count", "moevie_test_route_logits",
+                  "moevie_get_device_status", "moevie_launch_count", "moevie_shared_groups",
+                  "moevie_test_route_logits",
                   "moevie_test_fallback_count", "moevie_test_expert_hidden",
                   "moevie_test_moe_forward_events", "moevie_test_wait_timeout")
 
@@ -74,6 +75,7 @@ def load():
         "moevie_moe_forward": ([P, P, I64, P, P, P, SZ, P], ctypes.c_int),
         "moevie_get_device_status": ([P, P, P, P], ctypes.c_int),
         "moevie_launch_count": ([], ctypes.c_uint64),
+        "moevie_shared_groups": ([I64] * 6, ctypes.c_int64),
         "moevie_test_route_logits": ([P, P, I64, I64, I64, P, P, SZ, P], ctypes.c_int),
         "moevie_test_fallback_count": ([P, P, P], ctypes.c_int),
         "moevie_test_expert_hidden": ([P, P, P, P, I64, I64, I64, I64, I64, P, P, SZ, P],
@@ -275,6 +277,11 @@ def moevie_moe_forward(layer: LayerWeights, x, ws: Workspace, y=None, routing=Fa
 
 def moevie_launch_count() -> int:
     return int(load().moevie_launch_count())
+
+
+def moevie_shared_groups(T, d, E, k, h, h_s) -> int:
+    """Always-on groups that carry the shared expert inside the routed GEMMs (0: own GEMMs)."""
+    return int(load().moevie_shared_groups(T, d, E, k, h, h_s))
 
 
 # ----------------------------------------------------------------- test hooks

@@ -93,3 +93,27 @@ def test_forward_rejects_bad_layer(lib):
     rc = lib.moevie_moe_forward(ctypes.byref(L), ctypes.c_void_p(fake), 4, ctypes.c_void_p(fake),
                                 None, ctypes.c_void_p(fake), 1 << 30, None)
     assert rc == 2
+
+
+def test_shared_groups_plan_and_monotone_workspace(lib):
+    """moevie_shared_groups: the shared expert rides in the routed GEMMs as h_s / h
+    always-on groups when h divides h_s and the down-projection is not band-ordered
+    (fp32 accumulator [T, d] <= 64 MiB); the workspace size stays monotone in T across
+    that switch."""
+    g = lib.moevie_shared_groups
+    g.argtypes = [ctypes.c_int64] * 6
+    g.restype = ctypes.c_int64
+    assert g(8192, 1024, 64, 8, 512, 1024) == 2
+    assert g(300, 128, 16, 4, 128, 384) == 3
+    assert g(300, 256, 16, 4, 416, 128) == 0          # h does not divide h_s
+    assert g(8192, 1024, 64, 8, 512, 0) == 0          # no shared expert
+    assert g(65536, 1664, 256, 8, 416, 832) == 0      # band-ordered down-projection
+    assert g(8192, 1023, 64, 8, 512, 1024) == 0       # invalid sizes
+    d = 1024
+    t_switch = (64 << 20) // (4 * d)                  # accumulator reaches 64 MiB
+    assert g(t_switch, d, 64, 8, 512, 1024) == 2 and g(t_switch + 1, d, 64, 8, 512, 1024) == 0
+    prev = 0
+    for T in range(t_switch - 4, t_switch + 5):
+        rc, size = _ws_size(lib, T, d, 64, 8, 512, 1024)
+        assert rc == 0 and size >= prev, T
+        prev = size

@@ -101,3 +101,21 @@ def test_forward_empty_batch_launches_nothing():
     assert y.shape == (0, cfg.d)
     assert moevie.moevie_launch_count() == n0
     check_status(ws)
+
+
+def test_forward_banded_with_shared_expert_sampled():
+    """A layer whose fp32 accumulator exceeds 64 MiB (band-ordered down-projection)
+    with a shared expert of width 2h: the shared expert runs as its own GEMMs, its
+    hidden [T, h_s] in the workspace bytes that the always-on groups use otherwise."""
+    T, d, E, k, h, hs = 16400, 1024, 16, 2, 256, 512
+    assert moevie.moevie_shared_groups(T, d, E, k, h, hs) == 0
+    assert moevie.moevie_shared_groups(T // 2, d, E, k, h, hs) == 2
+    cfg = workloads.small_config(T, d, E, k, h, h_s=hs, lam=0.75, seed=7)
+    lay = workloads.make_layer(cfg)
+    y, rt = _run(lay)
+    _check_routing(lay, rt)
+    rng = np.random.default_rng(1)
+    toks = np.unique(np.concatenate([[0, T - 1], rng.choice(T, 48, replace=False)])).astype(np.int32)
+    want, *_ = oracle.forward_tokens(lay.x, lay.Wr, lay.b, lay.W1, lay.W2, k, lay.Ws1, lay.Ws2,
+                                     cfg.lam, tokens=toks)
+    assert_close(y[toks], want)
