@@ -280,7 +280,9 @@ moevie_status run_gemm(const GemmSpec& g, DevStatus* st, cudaStream_t s) {
     a.scale = g.scale;
     a.ksplit = g.ksplit > 1 ? g.ksplit : 1;
     if (a.ksplit > a.num_kb) return MOEVIE_ERR_UNSUPPORTED;
-    if (a.ksplit > 1 && g.epi != EPI_STORE_F32 && g.epi != EPI_ADD_F32) return MOEVIE_ERR_UNSUPPORTED;
+    if (a.ksplit > 1 && g.epi != EPI_STORE_F32 && g.epi != EPI_ADD_F32 && g.epi != EPI_SUM3_F32)
+        return MOEVIE_ERR_UNSUPPORTED;
+    if (g.epi == EPI_SUM3_F32 && (g.N % 96 != 0 || g.N > GM_MAXBN)) return MOEVIE_ERR_UNSUPPORTED;
     a.y_split_stride = g.y_split_stride;
     a.status = st;
     a.limit_ns = WAIT_LIMIT_NS;
@@ -312,19 +314,27 @@ moevie_status route_impl(const void* x, const float* W_r, const float* b, int64_
     const int64_t part_stride = T * Ep;
     MV_TRY(launch_route_split(W_r, (int)d, (int)E, wsplit, wrt, at<float>(ws, L.wpart), st, s));
     const int64_t dp = route_dpad((int)d);
+    const bool cc = route_concat((int)E);
     GemmSpec g{};
     g.A = x;
     g.lda = d;
     g.a_cols = d;
-    g.a_kperiod = (int)dp;         // K = 3 dp: x is read three times, once per piece
     g.a_nrows = T;
     g.m_total = T;
     g.G = 1;
     g.W = wsplit;
-    g.K = (int)(3 * dp);
-    g.N = (int)E;
-    g.N_ld = Ep;
-    g.epi = EPI_STORE_F32;
+    if (cc) {   // B [dp][3 Ep]: the three pieces side by side, summed by the epilogue
+        g.K = (int)dp;
+        g.N = 3 * Ep;
+        g.N_ld = 3 * Ep;
+        g.epi = EPI_SUM3_F32;
+    } else {    // B [3][dp][Ep]: K = 3 dp, x read three times, once per piece
+        g.a_kperiod = (int)dp;
+        g.K = (int)(3 * dp);
+        g.N = (int)E;
+        g.N_ld = Ep;
+        g.epi = EPI_STORE_F32;
+    }
     g.yacc = logits;
     g.ldy = Ep;
     g.o_nrows = T;

@@ -583,7 +583,7 @@ __device__ void epilogue(const GemmArgs& p, const Smem& sm, uint32_t tmem, int64
                          volatile int* abort_flag) {
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int quad = warp & 3, half = warp >> 2;
-    const bool to_f32 = (p.epi == EPI_ADD_F32 || p.epi == EPI_STORE_F32);
+    const bool to_f32 = (p.epi == EPI_ADD_F32 || p.epi == EPI_STORE_F32 || p.epi == EPI_SUM3_F32);
     const int nchunk = p.BN / 32;
     // bf16 results are written once and read back later: let them leave L2 first
     const uint64_t stream_pol = l2_policy_evict_first();
@@ -612,6 +612,44 @@ __device__ void epilogue(const GemmArgs& p, const Smem& sm, uint32_t tmem, int64
         }
         tc_fence_after();
         const uint32_t tbase = tmem + ((uint32_t)(quad * 32) << 16) + (uint32_t)acc * GM_MAXBN;
+        if (!GATHER && p.epi == EPI_SUM3_F32) {
+            // three column groups of N / 3 (one n-tile): chunk ch of the output is the sum
+            // of accumulator chunks ch, ch + nc3, ch + 2 nc3, added in that order
+            const int nc3 = nchunk / 3;
+            if (half >= nc3) {
+                tc_fence_before();
+                __syncwarp();
+                if (lane == 0) mbar_arrive_remote(tempty_leader + 8 * acc);
+            }
+            for (int ch = half; ch < nc3; ch += 2) {
+                uint32_t v[32];
+                float s3[32];
+                tmem_ld_32x32b_x32(tbase + ch * 32, v);
+                tmem_wait_ld();
+#pragma unroll
+                for (int i = 0; i < 32; ++i) s3[i] = __uint_as_float(v[i]);
+                tmem_ld_32x32b_x32(tbase + (ch + nc3) * 32, v);
+                tmem_wait_ld();
+#pragma unroll
+                for (int i = 0; i < 32; ++i) s3[i] += __uint_as_float(v[i]);
+                tmem_ld_32x32b_x32(tbase + (ch + 2 * nc3) * 32, v);
+                tmem_wait_ld();
+                if (ch + 2 >= nc3) {   // this warp's last read of the accumulator
+                    tc_fence_before();
+                    __syncwarp();
+                    if (lane == 0) mbar_arrive_remote(tempty_leader + 8 * acc);
+                }
+                if (!ok_row) continue;
+#pragma unroll
+                for (int i = 0; i < 32; ++i) s3[i] += __uint_as_float(v[i]);
+                float* yrow = p.yacc + t.ks * p.y_split_stride + tok * p.ldy + ch * 32;
+#pragma unroll
+                for (int q = 0; q < 8; ++q)
+                    *reinterpret_cast<float4*>(yrow + 4 * q) =
+                        make_float4(sc * s3[4 * q], sc * s3[4 * q + 1], sc * s3[4 * q + 2], sc * s3[4 * q + 3]);
+            }
+            continue;
+        }
         if (half >= nchunk) {   // no columns for this warp in this tile
             tc_fence_before();
             __syncwarp();

@@ -59,10 +59,14 @@ constexpr float ROUTE_TAU_C = 128.0f;
 constexpr float ROUTE_KEY_SLACK = 2e-6f;
 
 // Columns of the router logit buffer: E rounded up to 16 (rows stay 16-byte aligned).
-inline int route_epad(int E) { return (E + 15) / 16 * 16; }
+inline int route_epad(int E) { return (E + 31) / 32 * 32; }
 // Rows of each W_r piece: d rounded up to 64 (zero rows), so that no 64-wide K block
 // of the router GEMM straddles two pieces.
 inline int route_dpad(int d) { return (d + 63) / 64 * 64; }
+// The router GEMM's B holds the three bf16 pieces of W_r side by side along N
+// ([d_pad][3 E_pad]: x is read once, the epilogue sums the pieces) when they fit one
+// n-tile; otherwise one after another along K ([3][d_pad][E_pad], x read per piece).
+inline bool route_concat(int E) { return 3 * route_epad(E) <= 256; }   // 256: largest MMA N
 
 // W_r fp32 [d, E] -> three bf16 pieces [3][d_pad][E_pad] with W_r = hi + mid + lo
 // exactly (zero in the padding rows and columns), the transposed fp32 copy
@@ -181,6 +185,8 @@ enum Epilogue : int {
     EPI_STORE_BF16 = 1,  // out[r, n] = bf16(acc)
     EPI_ADD_F32 = 2,     // yacc[tok(r), n] += scale(r) * acc   (vector atomics)
     EPI_STORE_F32 = 3,   // yacc[tok(r), n]  = scale(r) * acc
+    EPI_SUM3_F32 = 4,    // yacc[tok(r), n]  = scale(r) * ((acc[n] + acc[n + N/3]) + acc[n + 2N/3]),
+                         //   n < N/3 (three column groups summed in a fixed order; one n-tile)
 };
 static_assert(EPI_ADD_F32 == 2, "gm_stages / gm_smem_bytes test the reduction epilogue by value");
 

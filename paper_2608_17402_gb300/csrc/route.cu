@@ -44,7 +44,8 @@ __global__ void __launch_bounds__(256) route_split_kernel(const float* __restric
                                                           int dp, int E, int Ep,
                                                           __nv_bfloat16* __restrict__ Wsplit,
                                                           float* __restrict__ wrt,
-                                                          float* __restrict__ wpart, DevStatus* st) {
+                                                          float* __restrict__ wpart, DevStatus* st,
+                                                          int concat) {
     pdl_wait();
     if (st && blockIdx.x == 0 && blockIdx.y == 0 && threadIdx.x == 0) st->fb_count = 0;
     __shared__ float tile[SPLIT_TILE][SPLIT_TILE + 1];
@@ -52,7 +53,9 @@ __global__ void __launch_bounds__(256) route_split_kernel(const float* __restric
     const int tx = threadIdx.x & 31, ty = threadIdx.x >> 5;
     const int e = blockIdx.x * SPLIT_TILE + tx;
     const int i0 = blockIdx.y * SPLIT_TILE;
-    const size_t piece = (size_t)dp * Ep;
+    // piece p of element (i, e): [p][dp][Ep] (along K), or [dp][3 Ep] (side by side along N)
+    const size_t piece = concat ? (size_t)Ep : (size_t)dp * Ep;
+    const size_t row = concat ? (size_t)3 * Ep : (size_t)Ep;
     float sq = 0.f;
 #pragma unroll
     for (int r = ty; r < SPLIT_TILE; r += 8) {
@@ -63,7 +66,7 @@ __global__ void __launch_bounds__(256) route_split_kernel(const float* __restric
             const float r1 = w - __bfloat162float(hi);          // exact
             const __nv_bfloat16 mid = __float2bfloat16_rn(r1);
             const __nv_bfloat16 lo = __float2bfloat16_rn(r1 - __bfloat162float(mid));   // exact
-            const size_t o = (size_t)i * Ep + e;
+            const size_t o = (size_t)i * row + e;
             Wsplit[o] = hi;
             Wsplit[piece + o] = mid;
             Wsplit[2 * piece + o] = lo;
@@ -453,9 +456,10 @@ int route_split_parts(int d) { return route_dpad(d) / SPLIT_TILE; }
 
 int route_ksplit(int64_t T, int d, int E) {
     int BN = 0, n_ntiles = 0;
-    choose_bn(E, &BN, &n_ntiles);
+    const bool cc = route_concat(E);
+    choose_bn(cc ? 3 * route_epad(E) : E, &BN, &n_ntiles);
     const int64_t items = (T + GM_BM - 1) / GM_BM * n_ntiles;
-    const int nkb = 3 * route_dpad(d) / GM_BK;
+    const int nkb = (cc ? 1 : 3) * route_dpad(d) / GM_BK;
     int64_t p = items > 0 ? (ROUTE_SPLIT_TARGET + items - 1) / items : 1;
     if (p > nkb / 3) p = nkb / 3;   // at least three K blocks per split
     if (p > ROUTE_MAX_KSPLIT) p = ROUTE_MAX_KSPLIT;
@@ -476,7 +480,8 @@ cudaError_t launch_route_split(const float* Wr, int d, int E, __nv_bfloat16* Wsp
     const int Ep = route_epad(E);
     const int parts = route_split_parts(d);
     cudaError_t e = launch_pdl(route_split_kernel, dim3((Ep + SPLIT_TILE - 1) / SPLIT_TILE, parts),
-                               dim3(256), 0, s, Wr, d, route_dpad(d), E, Ep, Wsplit, wrt, wpart, st);
+                               dim3(256), 0, s, Wr, d, route_dpad(d), E, Ep, Wsplit, wrt, wpart, st,
+                               route_concat(E) ? 1 : 0);
     count_launches(1);
     return e;
 }

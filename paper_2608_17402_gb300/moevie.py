@@ -303,11 +303,11 @@ def moevie_test_moe_forward_events(layer: LayerWeights, x, ws: Workspace, events
 
 
 def moevie_test_route_logits(x, W_r, ws: Workspace, stream=None):
-    """Fast-path logits [T, E] (the library writes E rounded up to 16 columns)."""
+    """Fast-path logits [T, E] (the library writes E rounded up to 32 columns)."""
     T, d = x.shape
     E = W_r.shape[1]
-    E16 = (E + 15) // 16 * 16
-    s = torch.empty((T, E16), dtype=torch.float32, device=x.device)
+    E32 = (E + 31) // 32 * 32
+    s = torch.empty((T, E32), dtype=torch.float32, device=x.device)
     _call("moevie_test_route_logits", _p(x), _p(W_r), T, d, E, _p(s), ws.ptr, ws.nbytes,
           _stream(stream))
     return s[:, :E]
