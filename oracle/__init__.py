@@ -67,11 +67,13 @@ def _load():
         lib.oracle_expert_rows.argtypes = [P, P, P, P, P, I64, I64, I64, I64, I64, P, I64,
                                            ctypes.c_int, P, ctypes.c_int]
         lib.oracle_combine.argtypes = [P, P, P, P, ctypes.c_double, I64, I64, I64, P]
+        lib.oracle_update_bias.argtypes = [P, I64, ctypes.c_float, ctypes.c_int, P]
         lib.oracle_forward_tokens.argtypes = [P, P, P, P, P, P, P, ctypes.c_double,
                                               I64, I64, I64, I64, I64, I64, P, I64,
                                               P, P, P, P, P, ctypes.c_int]
         for fn in (lib.oracle_logits, lib.oracle_select, lib.oracle_permute,
-                   lib.oracle_expert_rows, lib.oracle_combine, lib.oracle_forward_tokens):
+                   lib.oracle_expert_rows, lib.oracle_combine, lib.oracle_forward_tokens,
+                   lib.oracle_update_bias):
             fn.restype = ctypes.c_int
         _lib = lib
         return lib
@@ -133,6 +135,16 @@ def permute(idx, E):
     _check(_load().oracle_permute(_ptr(idx), T, k, E, _ptr(counts), _ptr(offsets), _ptr(perm),
                                   _ptr(inv)), "permute")
     return counts, offsets, perm, inv
+
+
+def update_bias(counts, b, alpha, rule="zscore"):
+    """Loss-free bias update (Sec. 2.2.2): z-score (Eq. 9) or sign (Eq. 8) rule; returns the new b (fp32)."""
+    counts = _c(counts, np.int32)
+    out = np.array(b, dtype=np.float32, copy=True)
+    r = {"zscore": 0, "sign": 1}[rule]
+    _check(_load().oracle_update_bias(_ptr(counts), counts.size, ctypes.c_float(alpha), r, _ptr(out)),
+           "update_bias")
+    return out
 
 
 def expert_rows(x_bf16, perm, offsets, W1, W2, k, rows, hidden=False, nthreads=None):

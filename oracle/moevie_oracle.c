@@ -377,3 +377,41 @@ int oracle_forward_tokens(const uint16_t* x, const float* Wr, const float* b,
     parallel_for(ntok, nthreads, fwd_items, &c);
     return c.err;
 }
+
+/* ------------------------------------------------------- bias update */
+
+/* Loss-free balancing bias update from one step's expert loads (Sec. 2.2.2):
+ * t_e = counts[e] (tokens routed to expert e), mu = their mean, sigma their
+ * (population) standard deviation over the E experts.
+ *   rule 0, z-score (Eq. 9):  b_e <- b_e - alpha (t_e - mu) / sigma
+ *                             (sigma == 0, all loads equal: b unchanged)
+ *   rule 1, sign (Eq. 8):     b_e <- b_e - alpha sign(t_e - mu), sign(0) = 0
+ * mu = (sum of t_e, an exact integer) / E; sigma = sqrt(sum_e (t_e - mu)^2 / E),
+ * summed in ascending e; each new b_e is computed in double and rounded to float. */
+int oracle_update_bias(const int32_t* counts, int64_t E, float alpha, int rule, float* b) {
+    if (E <= 0 || !counts || !b || (rule != 0 && rule != 1)) return ORACLE_ERR_ARG;
+    int64_t sum = 0;
+    for (int64_t e = 0; e < E; ++e) {
+        if (counts[e] < 0) return ORACLE_ERR_ARG;
+        sum += counts[e];
+    }
+    const double mu = (double)sum / (double)E;
+    double ss = 0.0;
+    for (int64_t e = 0; e < E; ++e) {
+        const double dev = (double)counts[e] - mu;
+        ss += dev * dev;
+    }
+    const double sigma = sqrt(ss / (double)E);
+    for (int64_t e = 0; e < E; ++e) {
+        const double dev = (double)counts[e] - mu;
+        double step;
+        if (rule == 0) {
+            if (sigma == 0.0) continue;
+            step = dev / sigma;
+        } else {
+            step = (double)((dev > 0.0) - (dev < 0.0));
+        }
+        b[e] = (float)((double)b[e] - (double)alpha * step);
+    }
+    return ORACLE_OK;
+}

@@ -345,3 +345,55 @@ def test_generator_recipe_is_seeded_and_shaped():
     back = bf16_bits_to_f32(f32_to_bf16_bits(v))
     assert np.all(np.abs(back - v) <= np.abs(v) * 2.0 ** -8)
     assert np.array_equal(bf16_bits_to_f32(f32_to_bf16_bits(back)), back)
+
+
+# --------------------------------------------------- loss-free bias update (Eqs. 8-9)
+
+def test_bias_update_zscore_closed_form():
+    """Eq. 9 on hand-made loads: counts (2, 4, 6) have mean 4 and population std
+    sqrt(8/3), so the z-scores are -sqrt(3/2), 0, +sqrt(3/2) and b moves by -alpha z."""
+    alpha = 0.5
+    b = np.float32([0.1, -0.2, 0.3])
+    out = oracle.update_bias([2, 4, 6], b, alpha)
+    z = math.sqrt(1.5)
+    want = np.float32([float(b[0]) + alpha * z, float(b[1]), float(b[2]) - alpha * z])
+    assert out[1] == b[1]
+    np.testing.assert_allclose(out, want, rtol=0, atol=6e-8)   # within one fp32 ulp
+
+
+def test_bias_update_balanced_loads_leave_b_unchanged():
+    """All loads equal: sigma = 0 (z-score, no update) and sign(0) = 0 (sign rule)."""
+    b = np.array([0.5, -1.25, 3.0, 0.0], np.float32)
+    for rule in ("zscore", "sign"):
+        np.testing.assert_array_equal(oracle.update_bias([7, 7, 7, 7], b, 0.01, rule), b)
+    np.testing.assert_array_equal(oracle.update_bias([9], [2.5], 0.1), np.float32([2.5]))   # E = 1
+
+
+def test_bias_update_sign_rule_exact():
+    """Eq. 8: each b_e moves by exactly -alpha sign(t_e - mean), mean taken in exact rationals."""
+    rng = np.random.default_rng(3)
+    counts = rng.integers(0, 400, size=37).astype(np.int32)
+    counts[5] = counts[6] = 0
+    b = rng.uniform(-0.1, 0.1, size=37).astype(np.float32)
+    alpha = 0.001
+    out = oracle.update_bias(counts, b, alpha, "sign")
+    mean = Fraction(int(counts.sum()), counts.size)
+    for e in range(counts.size):
+        sgn = (counts[e] > mean) - (counts[e] < mean)
+        assert out[e] == np.float32(float(b[e]) - alpha * sgn)
+
+
+def test_bias_update_zscore_invariants():
+    """z-scores of a population sum to 0 and their squares to E; scaling every load by
+    the same factor leaves them unchanged."""
+    rng = np.random.default_rng(4)
+    counts = rng.integers(0, 5000, size=256).astype(np.int32)
+    b0 = np.zeros(256, np.float32)
+    alpha = 1.0
+    z = -oracle.update_bias(counts, b0, alpha).astype(np.float64)
+    assert abs(z.sum()) < 1e-4 and abs((z * z).sum() - 256) < 1e-3
+    cf = counts.astype(np.float64)
+    want = (cf - cf.mean()) / cf.std()                    # numpy population std
+    np.testing.assert_allclose(z, want, rtol=0, atol=2e-7)
+    z3 = -oracle.update_bias(counts * 3, b0, alpha).astype(np.float64)
+    np.testing.assert_allclose(z3, z, rtol=0, atol=2e-7)
