@@ -180,6 +180,21 @@ moevie_status moevie_permute_static(const int32_t* idx, int64_t T, int64_t k, in
  * threads, all devices).  Host-only. */
 uint64_t moevie_launch_count(void);
 
+/* Loss-free balancing (Sec. 2.2.2): update the selection bias b[E] (fp32, device,
+ * in place) from one step's expert loads counts[E] (int32, device; e.g. the counts
+ * moevie_permute / moevie_moe_forward return), E <= 1024.  With mu the mean load and
+ * sigma the population standard deviation of the loads over the E experts:
+ *   rule 0, z-score (Eq. 9):  b_e <- b_e - alpha (t_e - mu) / sigma
+ *                              (all loads equal, sigma = 0: b unchanged)
+ *   rule 1, sign (Eq. 8):     b_e <- b_e - alpha sign(t_e - mu), sign(0) = 0.
+ * Arithmetic in fp64, each new b_e rounded to fp32.  One tiny kernel on `stream`;
+ * `ws` (>= 256 bytes, the workspace of the other entry points will do) receives the
+ * device status: a negative load leaves b unchanged and records MOEVIE_ERR_DEVICE.
+ * Argument errors (E outside [1, 1024], rule not 0 or 1, null or misaligned
+ * pointers) return before anything is enqueued. */
+moevie_status moevie_update_bias(const int32_t* counts, int64_t E, float alpha, int rule, float* b,
+                                 void* ws, size_t ws_bytes, void* stream);
+
 /* Launch plan of moevie_moe_forward for these sizes (host-only, no GPU work; the
  * paper has no counterpart -- it describes how this library schedules Eq. 6's
  * shared term).  Returns the number S of always-on groups of width h that carry the

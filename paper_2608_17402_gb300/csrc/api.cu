@@ -451,6 +451,15 @@ int moevie_version(void) { return 200; }
 
 uint64_t moevie_launch_count(void) { return g_launches.load(std::memory_order_relaxed); }
 
+moevie_status moevie_update_bias(const int32_t* counts, int64_t E, float alpha, int rule, float* b,
+                                 void* ws, size_t ws_bytes, void* stream) {
+    if (E < 1 || E > 1024 || (rule != 0 && rule != 1)) return MOEVIE_ERR_INVALID_ARG;
+    if (!counts || !b || !ws || !a16(ws)) return MOEVIE_ERR_INVALID_ARG;
+    if (ws_bytes < 256) return MOEVIE_ERR_WORKSPACE;
+    return cuda_status(launch_update_bias(counts, (int)E, alpha, rule, b, static_cast<DevStatus*>(ws),
+                                          static_cast<cudaStream_t>(stream)));
+}
+
 int64_t moevie_shared_groups(int64_t T, int64_t d, int64_t E, int64_t k, int64_t h, int64_t h_s) {
     if (check_sizes(T, d, E, k, h, h_s) != MOEVIE_OK) return 0;
     return shared_chunks(T, d, E, k, h, h_s);

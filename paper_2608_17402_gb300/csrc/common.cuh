@@ -37,6 +37,7 @@ enum Site : int {
     SITE_GEMM_OUT_ROW = 8,
     SITE_PERMUTE_ID = 10,
     SITE_ROUTE_FALLBACK = 20,
+    SITE_BIAS_COUNTS = 21,
     SITE_TIMEOUT_PROBE = 30,
 };
 

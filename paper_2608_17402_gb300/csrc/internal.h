@@ -277,6 +277,9 @@ cudaError_t perm_static_scratch(unsigned char** out);
 
 cudaError_t launch_zero_f32(float* p, int64_t n, cudaStream_t s);
 cudaError_t launch_f32_to_bf16(const float* src, __nv_bfloat16* dst, int64_t n, cudaStream_t s);
+// Loss-free bias update (Eq. 9 z-score, rule 0; Eq. 8 sign, rule 1) from counts[E], E <= 1024.
+cudaError_t launch_update_bias(const int32_t* counts, int E, float alpha, int rule, float* b,
+                               DevStatus* st, cudaStream_t s);
 // Rows of the shared expert folded into the grouped GEMMs as S always-on groups
 // E .. E + S - 1 of T rows each, at rows base + c T + t (token t, gate lambda), and
 // their m-tiles appended to the tile table (after the *n_tiles routed ones).

@@ -119,6 +119,59 @@ __global__ void shared_rows_kernel(int64_t T, int64_t base, int S, int E, float 
     }
 }
 
+// Loss-free balancing bias update from one step's expert loads t_e = counts[e]
+// (Sec. 2.2.2), one CTA of 1024 threads, one expert per thread (E <= 1024):
+//   rule 0, z-score (Eq. 9): b_e -= alpha (t_e - mu) / sigma  (sigma = 0: no update)
+//   rule 1, sign (Eq. 8):    b_e -= alpha sign(t_e - mu)
+// mu = (exact integer sum) / E and sigma = sqrt(sum (t_e - mu)^2 / E) (population) in
+// fp64; the sign is taken exactly as sign(E t_e - sum) in integers.  Each new b_e is
+// computed in fp64 with separately rounded operations and rounded to fp32.  A negative
+// load is a device error and leaves b unchanged.
+__global__ void __launch_bounds__(1024) update_bias_kernel(const int32_t* __restrict__ counts, int E,
+                                                           float alpha, int rule, float* __restrict__ b,
+                                                           DevStatus* st) {
+    pdl_wait();
+    __shared__ long long s_isum[32];
+    __shared__ double s_dsum[32];
+    __shared__ int s_bad;
+    const int e = threadIdx.x, lane = e & 31, warp = e >> 5;
+    const int t = e < E ? counts[e] : 0;
+    if (e == 0) s_bad = 0;
+    __syncthreads();
+    if (t < 0) atomicOr(&s_bad, 1);
+    long long is = t;
+#pragma unroll
+    for (int o = 16; o; o >>= 1) is += __shfl_xor_sync(0xffffffffu, is, o);
+    if (lane == 0) s_isum[warp] = is;
+    __syncthreads();
+    long long S = 0;
+    for (int w = 0; w < 32; ++w) S += s_isum[w];   // exact
+    if (s_bad) {
+        if (e == 0) report(st, MOEVIE_ERR_DEVICE, SITE_BIAS_COUNTS, 0, 0);
+        return;
+    }
+    const double mu = __ddiv_rn((double)S, (double)E);
+    const double dev = __dsub_rn((double)t, mu);
+    double sq = e < E ? __dmul_rn(dev, dev) : 0.0;
+#pragma unroll
+    for (int o = 16; o; o >>= 1) sq = __dadd_rn(sq, __shfl_xor_sync(0xffffffffu, sq, o));
+    if (lane == 0) s_dsum[warp] = sq;
+    __syncthreads();
+    double ss = 0.0;
+    for (int w = 0; w < 32; ++w) ss = __dadd_rn(ss, s_dsum[w]);
+    const double sigma = __dsqrt_rn(__ddiv_rn(ss, (double)E));
+    if (e >= E) return;
+    double step;
+    if (rule == 0) {
+        if (sigma == 0.0) return;
+        step = __ddiv_rn(dev, sigma);
+    } else {
+        const long long c = (long long)E * t - S;
+        step = (double)((c > 0) - (c < 0));
+    }
+    b[e] = __double2float_rn(__dsub_rn((double)b[e], __dmul_rn((double)alpha, step)));
+}
+
 int grid_for(int64_t n, int threads) {
     int64_t g = (n + threads - 1) / threads;
     if (g > 152 * 16) g = 152 * 16;
@@ -151,6 +204,14 @@ cudaError_t launch_shared_rows(int64_t T, int64_t base, int S, int E, float lamb
     const cudaError_t e = launch_pdl(shared_rows_kernel, dim3(grid_for(T * S, 256)), dim3(256), 0, s, T,
                                      base, S, E, lambda, row_tok, row_gate, tiles, n_tiles,
                                      max_routed, st);
+    count_launches(1);
+    return e;
+}
+
+cudaError_t launch_update_bias(const int32_t* counts, int E, float alpha, int rule, float* b,
+                               DevStatus* st, cudaStream_t s) {
+    const cudaError_t e = launch_pdl(update_bias_kernel, dim3(1), dim3(1024), 0, s, counts, E, alpha,
+                                     rule, b, st);
     count_launches(1);
     return e;
 }

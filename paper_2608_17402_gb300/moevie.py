@@ -27,6 +27,7 @@ C_ENTRY_POINTS = ("moevie_status_string", "moevie_version", "moevie_workspace_si
                   "moevie_expert_ffn",
                   "moevie_shared_expert", "moevie_combine", "moevie_moe_forward",
                   "moevie_get_device_status", "moevie_launch_count", "moevie_shared_groups",
+                  "moevie_update_bias",
                   "moevie_test_route_logits",
                   "moevie_test_fallback_count", "moevie_test_expert_hidden",
                   "moevie_test_moe_forward_events", "moevie_test_wait_timeout")
@@ -76,6 +77,7 @@ def load():
         "moevie_get_device_status": ([P, P, P, P], ctypes.c_int),
         "moevie_launch_count": ([], ctypes.c_uint64),
         "moevie_shared_groups": ([I64] * 6, ctypes.c_int64),
+        "moevie_update_bias": ([P, I64, F, ctypes.c_int, P, P, SZ, P], ctypes.c_int),
         "moevie_test_route_logits": ([P, P, I64, I64, I64, P, P, SZ, P], ctypes.c_int),
         "moevie_test_fallback_count": ([P, P, P], ctypes.c_int),
         "moevie_test_expert_hidden": ([P, P, P, P, I64, I64, I64, I64, I64, P, P, SZ, P],
@@ -277,6 +279,17 @@ def moevie_moe_forward(layer: LayerWeights, x, ws: Workspace, y=None, routing=Fa
 
 def moevie_launch_count() -> int:
     return int(load().moevie_launch_count())
+
+
+def moevie_update_bias(counts, b, alpha, ws: "Workspace", rule="zscore", stream=None):
+    """Loss-free bias update in place on b (fp32 [E]) from counts (int32 [E]): z-score
+    rule (Eq. 9) or sign rule (Eq. 8)."""
+    _want(counts, torch.int32, "counts")
+    _want(b, torch.float32, "b")
+    r = {"zscore": 0, "sign": 1}[rule]
+    _call("moevie_update_bias", _p(counts), counts.numel(), float(alpha), r, _p(b), ws.ptr, ws.nbytes,
+          _stream(stream))
+    return b
 
 
 def moevie_shared_groups(T, d, E, k, h, h_s) -> int:

@@ -117,3 +117,15 @@ def test_shared_groups_plan_and_monotone_workspace(lib):
         rc, size = _ws_size(lib, T, d, 64, 8, 512, 1024)
         assert rc == 0 and size >= prev, T
         prev = size
+
+
+def test_bias_update_validates_before_launch(lib):
+    f = lib.moevie_update_bias
+    f.argtypes = [ctypes.c_void_p, ctypes.c_int64, ctypes.c_float, ctypes.c_int, ctypes.c_void_p,
+                  ctypes.c_void_p, ctypes.c_size_t, ctypes.c_void_p]
+    p = ctypes.c_void_p(256)
+    assert f(p, 0, 0.1, 0, p, p, 4096, None) == 1        # E < 1
+    assert f(p, 1025, 0.1, 0, p, p, 4096, None) == 1     # E > 1024
+    assert f(p, 8, 0.1, 2, p, p, 4096, None) == 1        # unknown rule
+    assert f(None, 8, 0.1, 0, p, p, 4096, None) == 1     # null counts
+    assert f(p, 8, 0.1, 0, p, p, 128, None) == 3         # workspace too small
