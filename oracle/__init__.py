@@ -68,7 +68,7 @@ def _load():
                                            ctypes.c_int, P, ctypes.c_int]
         lib.oracle_combine.argtypes = [P, P, P, P, ctypes.c_double, I64, I64, I64, P]
         lib.oracle_update_bias.argtypes = [P, I64, ctypes.c_float, ctypes.c_int, P]
-        lib.oracle_forward_tokens.argtypes = [P, P, P, P, P, P, P, ctypes.c_double,
+        lib.oracle_forward_tokens.argtypes = [P, P, P, P, P, P, P, P, ctypes.c_double,
                                               I64, I64, I64, I64, I64, I64, P, I64,
                                               P, P, P, P, P, ctypes.c_int]
         for fn in (lib.oracle_logits, lib.oracle_select, lib.oracle_permute,
@@ -181,8 +181,9 @@ def combine(rows_out, inv, gate, shared=None, lam=1.0):
 
 
 def forward_tokens(x_bf16, Wr, b, W1, W2, k, Ws1=None, Ws2=None, lam=1.0, tokens=None,
-                   nthreads=None, want_shared=False):
-    """The whole layer for ``tokens`` (all tokens when None).
+                   nthreads=None, want_shared=False, W3=None):
+    """The whole layer for ``tokens`` (all tokens when None); SwiGLU experts
+    ``(SiLU(x W1[e]) * (x W3[e])) W2[e]`` when ``W3`` is given, else GELU experts.
 
     Returns ``(y fp64 [n, d], idx int32 [n, k], gate fp64 [n, k], margin fp64 [n])`` and,
     with ``want_shared``, the un-weighted shared expert output as a fifth item.
@@ -192,8 +193,10 @@ def forward_tokens(x_bf16, Wr, b, W1, W2, k, Ws1=None, Ws2=None, lam=1.0, tokens
     b = _c(b, np.float32)
     W1 = _c(W1, np.uint16)
     W2 = _c(W2, np.uint16)
+    W3 = None if W3 is None else _c(W3, np.uint16)   # SwiGLU experts when given
     T, d = x.shape
     E, _, h = W1.shape
+    assert W3 is None or W3.shape == W1.shape
     hs = 0
     if Ws1 is not None:
         Ws1 = _c(Ws1, np.uint16)
@@ -206,7 +209,7 @@ def forward_tokens(x_bf16, Wr, b, W1, W2, k, Ws1=None, Ws2=None, lam=1.0, tokens
     gate = np.empty((n, k), np.float64)
     margin = np.empty((n,), np.float64)
     shared = np.empty((n, d), np.float64) if (want_shared and hs > 0) else None
-    _check(_load().oracle_forward_tokens(_ptr(x), _ptr(Wr), _ptr(b), _ptr(W1), _ptr(W2),
+    _check(_load().oracle_forward_tokens(_ptr(x), _ptr(Wr), _ptr(b), _ptr(W1), _ptr(W2), _ptr(W3),
                                          _ptr(Ws1), _ptr(Ws2), float(lam), T, d, E, k, h, hs,
                                          _ptr(toks), n, _ptr(y), _ptr(idx), _ptr(gate),
                                          _ptr(margin), _ptr(shared),

@@ -14,7 +14,9 @@
  *   Eq. (4)-(5)  gates: Sigmoid(s) of the selected experts, renormalised to
  *                sum to one (the bias b only selects; it is not part of g)
  *   Eq. (3)/(6)  y = sum_{e in T(x)} g'_e E_e(x) + lambda * sum_shared E_s(x)
- *   expert       E_e(x) = GELU(x W1[e]) W2[e], GELU(u) = u/2 (1 + erf(u/sqrt 2))
+ *   expert       E_e(x) = GELU(x W1[e]) W2[e], GELU(u) = u/2 (1 + erf(u/sqrt 2)),
+ *                or the SwiGLU expert of App. B: (SiLU(x W1[e]) * (x W3[e])) W2[e],
+ *                SiLU(v) = v / (1 + exp(-v))
  *   App. B, Algorithm 1 phase 1: the sort of the flattened routing indices by
  *                expert, its histogram and exclusive prefix sum (offsets).
  *
@@ -232,6 +234,26 @@ static void expert_hidden(const uint16_t* xt, const uint16_t* W1e, int64_t d, in
     for (int64_t n = 0; n < h; ++n) hidden[n] = gelu(hidden[n]);
 }
 
+static double silu(double v) { return v / (1.0 + exp(-v)); }
+
+/* SwiGLU expert (the paper's own FFN, App. B):
+ * hidden[n] = SiLU(sum_i x[i] W1[e, i, n]) * (sum_i x[i] W3[e, i, n]),
+ * both sums in ascending i, the product formed once both are complete. */
+static void expert_hidden_swiglu(const uint16_t* xt, const uint16_t* W1e, const uint16_t* W3e,
+                                 int64_t d, int64_t h, double* hidden, double* up) {
+    for (int64_t n = 0; n < h; ++n) hidden[n] = up[n] = 0.0;
+    for (int64_t i = 0; i < d; ++i) {
+        double xi = bf16_to_double(xt[i]);
+        const uint16_t* wi = W1e + i * h;
+        const uint16_t* vi = W3e + i * h;
+        for (int64_t n = 0; n < h; ++n) {
+            hidden[n] += xi * bf16_to_double(wi[n]);
+            up[n] += xi * bf16_to_double(vi[n]);
+        }
+    }
+    for (int64_t n = 0; n < h; ++n) hidden[n] = silu(hidden[n]) * up[n];
+}
+
 /* out[c] = sum_n hidden[n] W2[e, n, c]  for c < d   (W2 bf16 [E, h, d]);
  * n outermost, each out[c] one sum in ascending n. */
 static void expert_down(const double* hidden, const uint16_t* W2e, int64_t h, int64_t d, double* out) {
@@ -309,7 +331,7 @@ int oracle_combine(const double* rows_out, const int32_t* inv, const double* gat
 
 typedef struct {
     const uint16_t* x; const float* Wr; const float* b; const uint16_t* W1; const uint16_t* W2;
-    const uint16_t* Ws1; const uint16_t* Ws2; double lambda;
+    const uint16_t* W3; const uint16_t* Ws1; const uint16_t* Ws2; double lambda;
     int64_t T, d, E, k, h, hs;
     const int32_t* tokens; double* y; int32_t* idx; double* gate; double* margin;
     double* shared_out; int err;
@@ -322,10 +344,11 @@ static void fwd_items(void* p, int64_t i0, int64_t i1) {
     double* key = (double*)malloc((size_t)c->E * sizeof(double));
     unsigned char* taken = (unsigned char*)malloc((size_t)c->E);
     double* hidden = (double*)malloc((size_t)hmax * sizeof(double));
+    double* up = (double*)malloc((size_t)hmax * sizeof(double));
     double* o = (double*)malloc((size_t)c->d * sizeof(double));
     int32_t* sel = (int32_t*)malloc((size_t)c->k * sizeof(int32_t));
     double* g = (double*)malloc((size_t)c->k * sizeof(double));
-    if (!s || !key || !taken || !hidden || !o || !sel || !g) {
+    if (!s || !key || !taken || !hidden || !up || !o || !sel || !g) {
         c->err = ORACLE_ERR_NOMEM;
         goto done;
     }
@@ -340,7 +363,11 @@ static void fwd_items(void* p, int64_t i0, int64_t i1) {
         for (int64_t col = 0; col < c->d; ++col) yt[col] = 0.0;
         for (int64_t j = 0; j < c->k; ++j) {                                               /* Eq. 6, routed */
             int64_t e = sel[j];
-            expert_hidden(xt, c->W1 + e * c->d * c->h, c->d, c->h, hidden);
+            if (c->W3)
+                expert_hidden_swiglu(xt, c->W1 + e * c->d * c->h, c->W3 + e * c->d * c->h, c->d, c->h,
+                                     hidden, up);
+            else
+                expert_hidden(xt, c->W1 + e * c->d * c->h, c->d, c->h, hidden);
             expert_down(hidden, c->W2 + e * c->h * c->d, c->h, c->d, o);
             for (int64_t col = 0; col < c->d; ++col) yt[col] += g[j] * o[col];
         }
@@ -356,14 +383,17 @@ static void fwd_items(void* p, int64_t i0, int64_t i1) {
         if (c->margin) c->margin[i] = m;
     }
 done:
-    free(s); free(key); free(taken); free(hidden); free(o); free(sel); free(g);
+    free(s); free(key); free(taken); free(hidden); free(up); free(o); free(sel); free(g);
 }
 
 /* y[i, :] for token tokens[i] (tokens may be NULL: all T tokens in order).
- * hs == 0 means no shared expert (Ws1, Ws2 ignored).  idx, gate, margin and
- * shared_out ([ntok, d], the un-weighted shared expert output) may be NULL. */
+ * W3 NULL: GELU experts GELU(x W1[e]) W2[e]; else SwiGLU experts
+ * (SiLU(x W1[e]) * (x W3[e])) W2[e], W3 bf16 [E, d, h].
+ * hs == 0 means no shared expert (Ws1, Ws2 ignored; the shared expert is GELU).
+ * idx, gate, margin and shared_out ([ntok, d], the un-weighted shared expert
+ * output) may be NULL. */
 int oracle_forward_tokens(const uint16_t* x, const float* Wr, const float* b,
-                          const uint16_t* W1, const uint16_t* W2,
+                          const uint16_t* W1, const uint16_t* W2, const uint16_t* W3,
                           const uint16_t* Ws1, const uint16_t* Ws2, double lambda,
                           int64_t T, int64_t d, int64_t E, int64_t k, int64_t h, int64_t hs,
                           const int32_t* tokens, int64_t ntok,
@@ -372,7 +402,7 @@ int oracle_forward_tokens(const uint16_t* x, const float* Wr, const float* b,
     if (T < 0 || d <= 0 || E <= 0 || k < 1 || k > E || h <= 0 || hs < 0 || ntok < 0) return ORACLE_ERR_ARG;
     if (ntok > 0 && (!x || !Wr || !b || !W1 || !W2 || !y)) return ORACLE_ERR_ARG;
     if (hs > 0 && ntok > 0 && (!Ws1 || !Ws2)) return ORACLE_ERR_ARG;
-    fwd_ctx c = { x, Wr, b, W1, W2, Ws1, Ws2, lambda, T, d, E, k, h, hs,
+    fwd_ctx c = { x, Wr, b, W1, W2, W3, Ws1, Ws2, lambda, T, d, E, k, h, hs,
                   tokens, y, idx, gate, margin, shared_out, ORACLE_OK };
     parallel_for(ntok, nthreads, fwd_items, &c);
     return c.err;

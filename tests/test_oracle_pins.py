@@ -397,3 +397,41 @@ def test_bias_update_zscore_invariants():
     np.testing.assert_allclose(z, want, rtol=0, atol=2e-7)
     z3 = -oracle.update_bias(counts * 3, b0, alpha).astype(np.float64)
     np.testing.assert_allclose(z3, z, rtol=0, atol=2e-7)
+
+
+# ------------------------------------------------------ SwiGLU experts (App. B)
+
+def test_single_swiglu_expert_is_dense_swiglu_mlp():
+    """E = 1, k = 1 with W3: the layer is (SiLU(x W1) * (x W3)) W2, checked against torch
+    fp64 (torch.nn.functional.silu); swapping W1 and W3 changes the result."""
+    rng = _rng(61)
+    T, d, h = 9, 24, 40
+    x = _bf16(rng.standard_normal((T, d)))
+    W1 = _bf16(rng.standard_normal((1, d, h)) / np.sqrt(d))
+    W3 = _bf16(rng.standard_normal((1, d, h)) / np.sqrt(d))
+    W2 = _bf16(rng.standard_normal((1, h, d)) / np.sqrt(h))
+    Wr = (rng.standard_normal((d, 1)) * 0.02).astype(np.float32)
+    b = np.zeros(1, np.float32)
+    y, idx, gate, _ = oracle.forward_tokens(x, Wr, b, W1, W2, 1, W3=W3)
+    xt = _t64(x)
+    want = (torch.nn.functional.silu(xt @ _t64(W1[0])) * (xt @ _t64(W3[0]))) @ _t64(W2[0])
+    assert np.all(idx == 0) and np.all(gate == 1.0)
+    np.testing.assert_allclose(y, want.numpy(), rtol=1e-12, atol=1e-12)
+    y_sw, *_ = oracle.forward_tokens(x, Wr, b, W3, W2, 1, W3=W1)
+    assert np.abs(y_sw - y).max() > 1e-3
+
+
+def test_swiglu_all_experts_uniform_gates():
+    """k = E and W_r = 0 with SwiGLU experts: y is the mean of all E SwiGLU experts
+    (a dense einsum over experts in torch fp64)."""
+    rng = _rng(62)
+    T, d, E, h = 12, 16, 5, 8
+    x, _, b, W1, W2, _, _ = _layer(rng, T, d, E, E, h)
+    W3 = _bf16(rng.standard_normal((E, d, h)) / np.sqrt(d))
+    Wr = np.zeros((d, E), np.float32)
+    y, idx, gate, _ = oracle.forward_tokens(x, Wr, b, W1, W2, E, W3=W3)
+    xt = _t64(x)
+    g = torch.einsum("td,edh->teh", xt, _t64(W1))
+    u = torch.einsum("td,edh->teh", xt, _t64(W3))
+    want = torch.einsum("teh,ehd->ted", torch.nn.functional.silu(g) * u, _t64(W2)).mean(1)
+    np.testing.assert_allclose(y, want.numpy(), rtol=1e-12, atol=1e-13)
