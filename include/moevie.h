@@ -122,6 +122,10 @@ typedef struct moevie_layer {
     const void* Ws1;        /* bf16 [d, h_s]  */
     const void* Ws2;        /* bf16 [h_s, d]  */
     float lambda;           /* weight of the shared expert */
+    const void* W3;         /* bf16 [E, d, h] or NULL.  NULL: GELU experts GELU(x W1[e]) W2[e].
+                             * Else SwiGLU experts (App. B): (SiLU(x W1[e]) * (x W3[e])) W2[e],
+                             * W1 the gate and W3 the up projection; with a SwiGLU layer
+                             * h_s must be 0 (MOEVIE_ERR_UNSUPPORTED otherwise). */
 } moevie_layer;
 
 /* Optional routing by-products of moevie_moe_forward; any member may be NULL. */

@@ -212,6 +212,7 @@ struct GemmSpec {
     int64_t w2_k_ld;         //   kk w2_k_ld + n (elements); W then holds g_split groups
     int64_t w2_g_ld;
     int g_split;
+    const void* W3;          // EPI_SWIGLU_BF16: the up projection W3 [G][K][N] beside W1 = W (gate)
 };
 
 moevie_status run_gemm(const GemmSpec& g, DevStatus* st, cudaStream_t s) {
@@ -263,9 +264,20 @@ moevie_status run_gemm(const GemmSpec& g, DevStatus* st, cudaStream_t s) {
     }
     a.G = g.G;
     a.g_split = g.W2nd ? g.g_split : g.G;
+    a.swiglu = g.epi == EPI_SWIGLU_BF16 ? 1 : 0;
+    if (a.swiglu) {   // gate (W1) and up (W3) tiles of 128 columns side by side: one N = 256 MMA
+        if (!g.W3 || !a16(g.W3) || g.W2nd || g.ksplit > 1) return MOEVIE_ERR_UNSUPPORTED;
+        if (!make_weight_tmap(&a.tmB2, g.W3, n_ld, g.K, g.G)) return MOEVIE_ERR_CUDA;
+    }
     a.K = g.K;
     a.N = g.N;
     choose_bn(g.N, &a.BN, &a.n_ntiles);
+    a.n_step = a.BN;
+    if (a.swiglu) {
+        a.BN = GM_MAXBN;
+        a.n_step = GM_MAXBN / 2;
+        a.n_ntiles = (g.N + a.n_step - 1) / a.n_step;
+    }
     a.num_kb = (g.K + GM_BK - 1) / GM_BK;
     a.nbox = (a.BN + 63) / 64;
     a.epi = g.epi;
@@ -628,7 +640,9 @@ static moevie_status forward_impl(const moevie_layer* Lr, const void* x, int64_t
     if (T == 0) return MOEVIE_OK;
     if (!x || !y || !ws || !Lr->W_r || !Lr->b || !Lr->W1 || !Lr->W2) return MOEVIE_ERR_INVALID_ARG;
     if (hs > 0 && (!Lr->Ws1 || !Lr->Ws2)) return MOEVIE_ERR_INVALID_ARG;
+    if (Lr->W3 && hs > 0) return MOEVIE_ERR_UNSUPPORTED;   // a SwiGLU layer has no shared expert here
     if (!a16(x) || !a16(y) || !a16(ws) || !a16(Lr->W1) || !a16(Lr->W2)) return MOEVIE_ERR_INVALID_ARG;
+    if (Lr->W3 && !a16(Lr->W3)) return MOEVIE_ERR_INVALID_ARG;
     if (hs > 0 && (!a16(Lr->Ws1) || !a16(Lr->Ws2))) return MOEVIE_ERR_INVALID_ARG;
     const Layout L = make_layout(T, d, E, k, h, hs);
     if (ws_bytes < L.total) return MOEVIE_ERR_WORKSPACE;
@@ -701,7 +715,8 @@ static moevie_status forward_impl(const moevie_layer* Lr, const void* x, int64_t
         up.W = Lr->W1;
         up.K = (int)d;
         up.N = (int)h;
-        up.epi = EPI_GELU_BF16;
+        up.epi = Lr->W3 ? EPI_SWIGLU_BF16 : EPI_GELU_BF16;
+        up.W3 = Lr->W3;   // SwiGLU: W1 the gate, W3 the up projection
         up.out = at<void>(ws, L.H);
         up.ldo = h;
         if (S > 0) {   // chunk c of Ws1 [d, h_s]: columns c h .. c h + h - 1

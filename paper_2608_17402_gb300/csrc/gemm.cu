@@ -213,7 +213,7 @@ __device__ __forceinline__ Tile tile_finish(const GemmArgs& p, const TileLd& l) 
         t.nrows = 0;
         t.g = 0;
     }
-    t.n0 = nt * p.BN;
+    t.n0 = nt * p.n_step;
     return t;
 }
 
@@ -283,7 +283,7 @@ template <bool GATHER>
 __device__ void producer_tma(const GemmArgs& p, const Smem& sm, int64_t n_work,
                              volatile int* abort_flag) {
     tma_prefetch_desc(&p.tmB);
-    if (p.g_split < p.G) tma_prefetch_desc(&p.tmB2);
+    if (p.g_split < p.G || p.swiglu) tma_prefetch_desc(&p.tmB2);
     constexpr bool gather = GATHER;
     if (!gather) tma_prefetch_desc(&p.tmA);
     const uint32_t half_n = (uint32_t)p.BN / 2;
@@ -301,9 +301,12 @@ __device__ void producer_tma(const GemmArgs& p, const Smem& sm, int64_t n_work,
         const int64_t wn = w + sm.npairs;
         TileLd nl{};
         if (wn < n_work) nl = tile_load(p, wn);   // checked after this item's loads
-        const bool second = t.g >= p.g_split;   // B of this group from the second map
+        // B of this group from the second map (groups >= g_split; with swiglu, the second
+        // CTA of the pair: W3 beside W1's columns)
+        const bool second = p.swiglu ? sm.rank == 1 : t.g >= p.g_split;
         const CUtensorMap* tmb = second ? &p.tmB2 : &p.tmB;
-        const int gb = second ? t.g - p.g_split : t.g;
+        const int gb = (second && !p.swiglu) ? t.g - p.g_split : t.g;
+        const int ncol0 = p.swiglu ? t.n0 : t.n0 + (int)(sm.rank * half_n);
         for (int kb = t.kb0; kb < t.kb1; ++kb) {
             if (!mbar_wait(sm.empty + 8 * s, ph ^ 1u, p.limit_ns, abort_flag)) {
                 set_abort(abort_flag, p.status, SITE_GEMM_WAIT_EMPTY, (int)sm.pair, 1);
@@ -314,8 +317,7 @@ __device__ void producer_tma(const GemmArgs& p, const Smem& sm, int64_t n_work,
             const uint32_t b_dst = sm.b0 + s * GM_B_BYTES;
             const int kk = kb * GM_BK;
             for (uint32_t j = 0; j < nboxh; ++j)
-                tma_load_3d_pair(b_dst + j * (GM_BK * 128), tmb, bar,
-                                 t.n0 + (int)(sm.rank * half_n + 64 * j), kk, gb);
+                tma_load_3d_pair(b_dst + j * (GM_BK * 128), tmb, bar, ncol0 + (int)(64 * j), kk, gb);
             if (!gather) {
                 const int col = p.a_kperiod ? kk % p.a_kperiod : kk;
                 tma_load_2d_pair(sm.a0 + s * GM_A_BYTES, &p.tmA, bar, col,
@@ -650,6 +652,51 @@ __device__ void epilogue(const GemmArgs& p, const Smem& sm, uint32_t tmem, int64
             }
             continue;
         }
+        if (GATHER && p.epi == EPI_SWIGLU_BF16) {   // (only the gathered up-projection)
+            // output chunk ch (32 columns): gate = accumulator chunk ch, up = chunk ch + nout
+            const int nout = nchunk / 2;
+            if (half >= nout) {
+                tc_fence_before();
+                __syncwarp();
+                if (lane == 0) mbar_arrive_remote(tempty_leader + 8 * acc);
+            }
+            for (int ch = half; ch < nout; ch += 2) {
+                uint32_t v[32];
+                float gt[32];
+                tmem_ld_32x32b_x32(tbase + ch * 32, v);
+                tmem_wait_ld();
+#pragma unroll
+                for (int i = 0; i < 32; ++i) gt[i] = __uint_as_float(v[i]);
+                tmem_ld_32x32b_x32(tbase + (ch + nout) * 32, v);
+                tmem_wait_ld();
+                if (ch + 2 >= nout) {   // this warp's last read of the accumulator
+                    tc_fence_before();
+                    __syncwarp();
+                    if (lane == 0) mbar_arrive_remote(tempty_leader + 8 * acc);
+                }
+                if (!ok_row) continue;
+                const int n = t.n0 + ch * 32;
+                __nv_bfloat16* orow = p.out + (int64_t)gr * p.ldo + n;
+#pragma unroll
+                for (int g8 = 0; g8 < 4; ++g8) {
+                    if (n + 8 * g8 >= p.N) break;
+                    float f[8];
+#pragma unroll
+                    for (int i = 0; i < 8; ++i) {
+                        // SiLU(g) u = g u / (1 + e^-g); e^-g = inf for g far below 0 gives 0
+                        const float g = gt[8 * g8 + i];
+                        f[i] = __fdividef(g, 1.0f + __expf(-g)) * __uint_as_float(v[8 * g8 + i]);
+                    }
+                    uint4 u;
+                    u.x = pack_bf16x2(f[0], f[1]);
+                    u.y = pack_bf16x2(f[2], f[3]);
+                    u.z = pack_bf16x2(f[4], f[5]);
+                    u.w = pack_bf16x2(f[6], f[7]);
+                    st_global_v4_hint(orow + 8 * g8, u, stream_pol);
+                }
+            }
+            continue;
+        }
         if (half >= nchunk) {   // no columns for this warp in this tile
             tc_fence_before();
             __syncwarp();
@@ -921,7 +968,8 @@ cudaError_t launch_grouped_gemm(const GemmArgs& a, int grid, cudaStream_t s) {
     using Kern = void (*)(GemmArgs);
     static const Kern kerns[3] = {grouped_gemm_kernel<32, false>, grouped_gemm_kernel<16, false>,
                                   grouped_gemm_kernel<32, true>};
-    if (a.a_rows && a.epi == EPI_ADD_F32) return cudaErrorInvalidValue;
+    if (a.a_rows && (a.epi == EPI_ADD_F32 || a.epi == EPI_SUM3_F32)) return cudaErrorInvalidValue;
+    if (!a.a_rows && a.epi == EPI_SWIGLU_BF16) return cudaErrorInvalidValue;
     const Kern kern = a.a_rows ? kerns[2] : a.stg_rows == 32 ? kerns[0] : kerns[1];
     static bool attr_set[64] = {};
     int dev = 0;

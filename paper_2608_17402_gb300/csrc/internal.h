@@ -185,6 +185,9 @@ enum Epilogue : int {
     EPI_STORE_BF16 = 1,  // out[r, n] = bf16(acc)
     EPI_ADD_F32 = 2,     // yacc[tok(r), n] += scale(r) * acc   (vector atomics)
     EPI_STORE_F32 = 3,   // yacc[tok(r), n]  = scale(r) * acc
+    EPI_SWIGLU_BF16 = 5, // out[r, n] = bf16(SiLU(acc[gate n]) * acc[up n]): accumulator columns
+                         //   0..127 from W1 (gate, the pair's first CTA's B half), 128..255 from
+                         //   W3 (up, the second CTA's); 128 output columns per n-tile
     EPI_SUM3_F32 = 4,    // yacc[tok(r), n]  = scale(r) * ((acc[n] + acc[n + N/3]) + acc[n + 2N/3]),
                          //   n < N/3 (three column groups summed in a fixed order; one n-tile)
 };
@@ -210,6 +213,8 @@ struct GemmArgs {
     int64_t max_mtiles;         // host bound on *n_tiles_dev
     int G, K, N, BN, n_ntiles, num_kb, nbox;
     int g_split;                // first group read through tmB2 (G when there is none)
+    int swiglu;                 // EPI_SWIGLU_BF16: B half of CTA rank 1 from tmB2 (W3), same columns
+    int n_step;                 // output columns per n-tile (BN; BN / 2 with swiglu)
     int ksplit;                 // K is split into this many parts (work items), >= 1
     int64_t y_split_stride;     // fp32 outputs: split ks writes yacc + ks * y_split_stride
     int epi;

@@ -47,6 +47,7 @@ class LayerConfig:
     seed: int = 0
     skew: str | None = None  # key into skew_offsets.json, or None for no skew
     note: str = ""
+    act: str = "gelu"       # expert FFN: "gelu", or "swiglu" (W1 gate, W3 up; App. B)
 
     @property
     def slots(self) -> int:
@@ -66,6 +67,9 @@ CONFIGS = {
                       note="4 clips x 32 frames x 256 patches, Zipf(1.0) loads, 4 empty experts"),
     "c4": LayerConfig("c4", T=65536, d=1664, E=256, k=8, h=416, skew="c4",
                       note="stress layer: one saturated expert, Zipf(1.1) over the rest, 3 empty"),
+    # SwiGLU experts (the paper's own FFN, App. B) at the image-batch layer's routed shape
+    "s1": LayerConfig("s1", T=8192, d=1024, E=64, k=8, h=512, act="swiglu",
+                      note="32 images x 256 patches, SwiGLU experts (W1 gate, W3 up), no shared expert"),
 }
 
 
@@ -97,6 +101,7 @@ class LayerInputs:
     Ws1: np.ndarray | None = None   # uint16 [d, h_s]
     Ws2: np.ndarray | None = None   # uint16 [h_s, d]
     extra: dict = field(default_factory=dict)
+    W3: np.ndarray | None = None    # uint16 [E, d, h], SwiGLU layers only
 
 
 def _normal_bf16(rng: np.random.Generator, shape, std: float) -> np.ndarray:
@@ -135,6 +140,9 @@ def make_layer(cfg: LayerConfig, skew_offsets: np.ndarray | None = None,
     if cfg.h_s > 0:
         Ws1 = _normal_bf16(rng, (d, cfg.h_s), 1.0 / np.sqrt(d))
         Ws2 = _normal_bf16(rng, (cfg.h_s, d), 1.0 / np.sqrt(cfg.h_s))
+    W3 = None
+    if cfg.act == "swiglu":   # drawn last: the GELU layers' draws are unchanged
+        W3 = _normal_bf16(rng, (E, d, h), 1.0 / np.sqrt(d))
     extra = {}
     if cfg.skew is not None:
         offs = skew_offsets if skew_offsets is not None else load_skew_offsets(cfg.skew)
@@ -147,12 +155,12 @@ def make_layer(cfg: LayerConfig, skew_offsets: np.ndarray | None = None,
             x[:, d - 1] = f32_to_bf16_bits(np.ones(1, np.float32))[0]
             Wr[d - 1, :] = offs
             extra["skew_offsets"] = offs
-    return LayerInputs(cfg, x, Wr, b, W1, W2, Ws1, Ws2, extra)
+    return LayerInputs(cfg, x, Wr, b, W1, W2, Ws1, Ws2, extra, W3)
 
 
-def small_config(T, d, E, k, h, h_s=0, lam=1.0, seed=0, name="small") -> LayerConfig:
+def small_config(T, d, E, k, h, h_s=0, lam=1.0, seed=0, name="small", act="gelu") -> LayerConfig:
     """An unskewed layer of arbitrary shape (tests)."""
-    return LayerConfig(name, T=T, d=d, E=E, k=k, h=h, h_s=h_s, lam=lam, seed=seed)
+    return LayerConfig(name, T=T, d=d, E=E, k=k, h=h, h_s=h_s, lam=lam, seed=seed, act=act)
 
 
 # ---------------------------------------------------------------- skew targets
