@@ -89,16 +89,18 @@ def layer_work(cfg, counts, shared_groups=0):
     shared_groups: always-on groups of width h that carry the shared expert inside the
     routed up / down launches (moevie_shared_groups), counted in those launches' FLOPs."""
     T, d, E, k, h, hs = cfg.T, cfg.d, cfg.E, cfg.k, cfg.h, cfg.h_s
+    up_mats = 2 if cfg.act == "swiglu" else 1    # SwiGLU: gate (W1) and up (W3) projections
     flops_router = 2.0 * T * d * E
-    flops_experts = 4.0 * T * k * d * h
+    flops_up = 2.0 * up_mats * T * k * d * h
+    flops_down = 2.0 * T * k * d * h
     flops_shared = 4.0 * T * d * hs
     touched = int((np.asarray(counts) > 0).sum())
-    bytes_ = (T * d * 2 + T * d * 2 + d * E * 4 + E * 4 + touched * 2 * d * h * 2
+    bytes_ = (T * d * 2 + T * d * 2 + d * E * 4 + E * 4 + touched * (up_mats + 1) * d * h * 2
               + 2 * d * hs * 2 + 8 * T * k)
     folded = shared_groups * h * T * d * 2.0
-    return {"flops": flops_router + flops_experts + flops_shared,
-            "flops_up_gemm": 2.0 * T * k * d * h + folded,
-            "flops_down_gemm": 2.0 * T * k * d * h + folded, "bytes": float(bytes_), "touched_experts": touched}
+    return {"flops": flops_router + flops_up + flops_down + flops_shared,
+            "flops_up_gemm": flops_up + folded,
+            "flops_down_gemm": flops_down + folded, "bytes": float(bytes_), "touched_experts": touched}
 
 
 class ClockSampler:
@@ -167,7 +169,7 @@ def cpu_baseline(lay, target_s=15.0, max_tokens=None):
     rng = np.random.default_rng(123)
     probe = np.sort(rng.choice(cfg.T, size=min(cfg.T, max(nthreads, 8)), replace=False)).astype(np.int32)
     t0 = time.perf_counter()
-    oracle.forward_tokens(lay.x, lay.Wr, lay.b, lay.W1, lay.W2, cfg.k, lay.Ws1, lay.Ws2, cfg.lam, tokens=probe)
+    oracle.forward_tokens(lay.x, lay.Wr, lay.b, lay.W1, lay.W2, cfg.k, lay.Ws1, lay.Ws2, cfg.lam, tokens=probe, W3=lay.W3)
     per_tok = (time.perf_counter() - t0) / probe.size
     n = int(min(cfg.T, max(nthreads, target_s / max(per_tok, 1e-9))))
     if max_tokens:
@@ -177,7 +179,7 @@ def cpu_baseline(lay, target_s=15.0, max_tokens=None):
     passes, t0 = 0, time.perf_counter()
     while True:
         oracle.forward_tokens(lay.x, lay.Wr, lay.b, lay.W1, lay.W2, cfg.k, lay.Ws1, lay.Ws2, cfg.lam,
-                              tokens=toks)
+                              tokens=toks, W3=lay.W3)
         passes += 1
         dt = time.perf_counter() - t0
         if dt >= 0.66 * target_s or passes >= 8:
@@ -198,7 +200,7 @@ def run_reference(args, rank):
     # size each step so the whole run stays within a few minutes
     probe = np.arange(min(cfg.T, nthreads), dtype=np.int32)
     t0 = time.perf_counter()
-    oracle.forward_tokens(lay.x, lay.Wr, lay.b, lay.W1, lay.W2, cfg.k, lay.Ws1, lay.Ws2, cfg.lam, tokens=probe)
+    oracle.forward_tokens(lay.x, lay.Wr, lay.b, lay.W1, lay.W2, cfg.k, lay.Ws1, lay.Ws2, cfg.lam, tokens=probe, W3=lay.W3)
     per_tok = (time.perf_counter() - t0) / probe.size
     budget = 150.0 / max(1, args.steps + args.warmup)
     n = int(min(cfg.T, max(nthreads, budget / max(per_tok, 1e-9))))
@@ -207,7 +209,7 @@ def run_reference(args, rank):
         toks = np.sort(rng.choice(cfg.T, size=n, replace=False)).astype(np.int32)
         t0 = time.perf_counter()
         oracle.forward_tokens(lay.x, lay.Wr, lay.b, lay.W1, lay.W2, cfg.k, lay.Ws1, lay.Ws2, cfg.lam,
-                              tokens=toks)
+                              tokens=toks, W3=lay.W3)
         if i >= args.warmup:
             times.append(time.perf_counter() - t0)
     ms = 1e3 * statistics.mean(times)
@@ -216,7 +218,7 @@ def run_reference(args, rank):
            "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True,
            "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
            "config": {"workload": f"{cfg.name}: {cfg.note}", "T": cfg.T, "d": cfg.d, "E": cfg.E, "k": cfg.k,
-                      "h": cfg.h, "h_s": cfg.h_s, "tokens_per_step": n},
+                      "h": cfg.h, "h_s": cfg.h_s, "act": cfg.act, "tokens_per_step": n},
            "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": nthreads, "kind": "oracle",
                             "sample": f"{n} random tokens of {cfg.name} per step"},
            "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
@@ -243,7 +245,8 @@ def run_ours(args, rank, world):
     W = moevie.LayerWeights(W_r=torch.from_numpy(lay.Wr).cuda(), b=torch.from_numpy(lay.b).cuda(),
                             W1=bf(lay.W1), W2=bf(lay.W2), k=cfg.k,
                             Ws1=None if lay.Ws1 is None else bf(lay.Ws1),
-                            Ws2=None if lay.Ws2 is None else bf(lay.Ws2), lam=cfg.lam)
+                            Ws2=None if lay.Ws2 is None else bf(lay.Ws2), lam=cfg.lam,
+                            W3=None if lay.W3 is None else bf(lay.W3))
     x = bf(lay.x)
     y = torch.empty((cfg.T, cfg.d), dtype=torch.bfloat16, device="cuda")
     ws = moevie.Workspace(cfg.T, cfg.d, cfg.E, cfg.k, cfg.h, cfg.h_s)
@@ -329,7 +332,7 @@ def run_ours(args, rank, world):
         "warmup": args.warmup, "ms_per_step": ms, "us_per_layer": ms * 1e3, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
         "config": {"workload": f"{cfg.name}: {cfg.note}", "T": cfg.T, "d": cfg.d, "E": cfg.E, "k": cfg.k,
-                   "h": cfg.h, "h_s": cfg.h_s, "lambda": cfg.lam, "seed": cfg.seed,
+                   "h": cfg.h, "h_s": cfg.h_s, "act": cfg.act, "lambda": cfg.lam, "seed": cfg.seed,
                    "parallelism": f"replicas x{world}" if world > 1 else "single GPU",
                    "l2": f"flushed between steps ({L2_FLUSH_BYTES >> 20} MiB write outside the timed window)"},
         "roofline": {"bound": "tensor", "kernel": f"grouped_gemm_kernel ({dom})", "achieved": achieved,

@@ -120,7 +120,7 @@ __global__ void shared_rows_kernel(int64_t T, int64_t base, int S, int E, float 
 }
 
 // Loss-free balancing bias update from one step's expert loads t_e = counts[e]
-// (Sec. 2.2.2), one CTA of 1024 threads, one expert per thread (E <= 1024):
+// (Sec. 2.2.2), one CTA with one thread per expert (E <= 1024):
 //   rule 0, z-score (Eq. 9): b_e -= alpha (t_e - mu) / sigma  (sigma = 0: no update)
 //   rule 1, sign (Eq. 8):    b_e -= alpha sign(t_e - mu)
 // mu = (exact integer sum) / E and sigma = sqrt(sum (t_e - mu)^2 / E) (population) in
@@ -133,8 +133,10 @@ __global__ void __launch_bounds__(1024) update_bias_kernel(const int32_t* __rest
     pdl_wait();
     __shared__ long long s_isum[32];
     __shared__ double s_dsum[32];
+    __shared__ long long s_S;
+    __shared__ double s_sigma;
     __shared__ int s_bad;
-    const int e = threadIdx.x, lane = e & 31, warp = e >> 5;
+    const int e = threadIdx.x, lane = e & 31, warp = e >> 5, nwarps = blockDim.x >> 5;
     const int t = e < E ? counts[e] : 0;
     if (e == 0) s_bad = 0;
     __syncthreads();
@@ -144,12 +146,18 @@ __global__ void __launch_bounds__(1024) update_bias_kernel(const int32_t* __rest
     for (int o = 16; o; o >>= 1) is += __shfl_xor_sync(0xffffffffu, is, o);
     if (lane == 0) s_isum[warp] = is;
     __syncthreads();
-    long long S = 0;
-    for (int w = 0; w < 32; ++w) S += s_isum[w];   // exact
+    if (warp == 0) {   // the exact integer total
+        long long v = lane < nwarps ? s_isum[lane] : 0;
+#pragma unroll
+        for (int o = 16; o; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+        if (lane == 0) s_S = v;
+    }
+    __syncthreads();
     if (s_bad) {
         if (e == 0) report(st, MOEVIE_ERR_DEVICE, SITE_BIAS_COUNTS, 0, 0);
         return;
     }
+    const long long S = s_S;
     const double mu = __ddiv_rn((double)S, (double)E);
     const double dev = __dsub_rn((double)t, mu);
     double sq = e < E ? __dmul_rn(dev, dev) : 0.0;
@@ -157,9 +165,14 @@ __global__ void __launch_bounds__(1024) update_bias_kernel(const int32_t* __rest
     for (int o = 16; o; o >>= 1) sq = __dadd_rn(sq, __shfl_xor_sync(0xffffffffu, sq, o));
     if (lane == 0) s_dsum[warp] = sq;
     __syncthreads();
-    double ss = 0.0;
-    for (int w = 0; w < 32; ++w) ss = __dadd_rn(ss, s_dsum[w]);
-    const double sigma = __dsqrt_rn(__ddiv_rn(ss, (double)E));
+    if (warp == 0) {   // population standard deviation
+        double v = lane < nwarps ? s_dsum[lane] : 0.0;
+#pragma unroll
+        for (int o = 16; o; o >>= 1) v = __dadd_rn(v, __shfl_xor_sync(0xffffffffu, v, o));
+        if (lane == 0) s_sigma = __dsqrt_rn(__ddiv_rn(v, (double)E));
+    }
+    __syncthreads();
+    const double sigma = s_sigma;
     if (e >= E) return;
     double step;
     if (rule == 0) {
@@ -210,8 +223,8 @@ cudaError_t launch_shared_rows(int64_t T, int64_t base, int S, int E, float lamb
 
 cudaError_t launch_update_bias(const int32_t* counts, int E, float alpha, int rule, float* b,
                                DevStatus* st, cudaStream_t s) {
-    const cudaError_t e = launch_pdl(update_bias_kernel, dim3(1), dim3(1024), 0, s, counts, E, alpha,
-                                     rule, b, st);
+    const cudaError_t e = launch_pdl(update_bias_kernel, dim3(1), dim3((E + 31) / 32 * 32), 0, s, counts,
+                                     E, alpha, rule, b, st);
     count_launches(1);
     return e;
 }
