@@ -68,7 +68,7 @@ def _load():
                                            ctypes.c_int, P, ctypes.c_int]
         lib.oracle_combine.argtypes = [P, P, P, P, ctypes.c_double, I64, I64, I64, P]
         lib.oracle_update_bias.argtypes = [P, I64, ctypes.c_float, ctypes.c_int, P]
-        lib.oracle_forward_tokens.argtypes = [P, P, P, P, P, P, P, P, ctypes.c_double,
+        lib.oracle_forward_tokens.argtypes = [P, P, P, P, P, P, P, P, P, ctypes.c_double,
                                               I64, I64, I64, I64, I64, I64, P, I64,
                                               P, P, P, P, P, ctypes.c_int]
         for fn in (lib.oracle_logits, lib.oracle_select, lib.oracle_permute,
@@ -181,7 +181,7 @@ def combine(rows_out, inv, gate, shared=None, lam=1.0):
 
 
 def forward_tokens(x_bf16, Wr, b, W1, W2, k, Ws1=None, Ws2=None, lam=1.0, tokens=None,
-                   nthreads=None, want_shared=False, W3=None):
+                   nthreads=None, want_shared=False, W3=None, Ws3=None):
     """The whole layer for ``tokens`` (all tokens when None); SwiGLU experts
     ``(SiLU(x W1[e]) * (x W3[e])) W2[e]`` when ``W3`` is given, else GELU experts.
 
@@ -202,6 +202,8 @@ def forward_tokens(x_bf16, Wr, b, W1, W2, k, Ws1=None, Ws2=None, lam=1.0, tokens
         Ws1 = _c(Ws1, np.uint16)
         Ws2 = _c(Ws2, np.uint16)
         hs = Ws1.shape[1]
+        Ws3 = None if Ws3 is None else _c(Ws3, np.uint16)   # SwiGLU shared expert when given
+        assert Ws3 is None or Ws3.shape == Ws1.shape
     toks = None if tokens is None else _c(tokens, np.int32)
     n = T if toks is None else toks.size
     y = np.empty((n, d), np.float64)
@@ -210,7 +212,7 @@ def forward_tokens(x_bf16, Wr, b, W1, W2, k, Ws1=None, Ws2=None, lam=1.0, tokens
     margin = np.empty((n,), np.float64)
     shared = np.empty((n, d), np.float64) if (want_shared and hs > 0) else None
     _check(_load().oracle_forward_tokens(_ptr(x), _ptr(Wr), _ptr(b), _ptr(W1), _ptr(W2), _ptr(W3),
-                                         _ptr(Ws1), _ptr(Ws2), float(lam), T, d, E, k, h, hs,
+                                         _ptr(Ws1), _ptr(Ws2), _ptr(Ws3), float(lam), T, d, E, k, h, hs,
                                          _ptr(toks), n, _ptr(y), _ptr(idx), _ptr(gate),
                                          _ptr(margin), _ptr(shared),
                                          nthreads or default_threads()), "forward_tokens")

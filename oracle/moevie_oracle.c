@@ -331,7 +331,7 @@ int oracle_combine(const double* rows_out, const int32_t* inv, const double* gat
 
 typedef struct {
     const uint16_t* x; const float* Wr; const float* b; const uint16_t* W1; const uint16_t* W2;
-    const uint16_t* W3; const uint16_t* Ws1; const uint16_t* Ws2; double lambda;
+    const uint16_t* W3; const uint16_t* Ws1; const uint16_t* Ws2; const uint16_t* Ws3; double lambda;
     int64_t T, d, E, k, h, hs;
     const int32_t* tokens; double* y; int32_t* idx; double* gate; double* margin;
     double* shared_out; int err;
@@ -372,7 +372,8 @@ static void fwd_items(void* p, int64_t i0, int64_t i1) {
             for (int64_t col = 0; col < c->d; ++col) yt[col] += g[j] * o[col];
         }
         if (c->hs > 0) {                                                                    /* Eq. 6, shared */
-            expert_hidden(xt, c->Ws1, c->d, c->hs, hidden);
+            if (c->Ws3) expert_hidden_swiglu(xt, c->Ws1, c->Ws3, c->d, c->hs, hidden, up);
+            else expert_hidden(xt, c->Ws1, c->d, c->hs, hidden);
             expert_down(hidden, c->Ws2, c->hs, c->d, o);
             for (int64_t col = 0; col < c->d; ++col) yt[col] += c->lambda * o[col];
             if (c->shared_out)
@@ -389,12 +390,13 @@ done:
 /* y[i, :] for token tokens[i] (tokens may be NULL: all T tokens in order).
  * W3 NULL: GELU experts GELU(x W1[e]) W2[e]; else SwiGLU experts
  * (SiLU(x W1[e]) * (x W3[e])) W2[e], W3 bf16 [E, d, h].
- * hs == 0 means no shared expert (Ws1, Ws2 ignored; the shared expert is GELU).
+ * hs == 0 means no shared expert (Ws1, Ws2, Ws3 ignored); Ws3 NULL: a GELU shared
+ * expert, else a SwiGLU one (SiLU(x Ws1) * (x Ws3)) Ws2, Ws3 bf16 [d, hs].
  * idx, gate, margin and shared_out ([ntok, d], the un-weighted shared expert
  * output) may be NULL. */
 int oracle_forward_tokens(const uint16_t* x, const float* Wr, const float* b,
                           const uint16_t* W1, const uint16_t* W2, const uint16_t* W3,
-                          const uint16_t* Ws1, const uint16_t* Ws2, double lambda,
+                          const uint16_t* Ws1, const uint16_t* Ws2, const uint16_t* Ws3, double lambda,
                           int64_t T, int64_t d, int64_t E, int64_t k, int64_t h, int64_t hs,
                           const int32_t* tokens, int64_t ntok,
                           double* y, int32_t* idx, double* gate, double* margin,
@@ -402,7 +404,7 @@ int oracle_forward_tokens(const uint16_t* x, const float* Wr, const float* b,
     if (T < 0 || d <= 0 || E <= 0 || k < 1 || k > E || h <= 0 || hs < 0 || ntok < 0) return ORACLE_ERR_ARG;
     if (ntok > 0 && (!x || !Wr || !b || !W1 || !W2 || !y)) return ORACLE_ERR_ARG;
     if (hs > 0 && ntok > 0 && (!Ws1 || !Ws2)) return ORACLE_ERR_ARG;
-    fwd_ctx c = { x, Wr, b, W1, W2, W3, Ws1, Ws2, lambda, T, d, E, k, h, hs,
+    fwd_ctx c = { x, Wr, b, W1, W2, W3, Ws1, Ws2, Ws3, lambda, T, d, E, k, h, hs,
                   tokens, y, idx, gate, margin, shared_out, ORACLE_OK };
     parallel_for(ntok, nthreads, fwd_items, &c);
     return c.err;

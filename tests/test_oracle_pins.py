@@ -435,3 +435,18 @@ def test_swiglu_all_experts_uniform_gates():
     u = torch.einsum("td,edh->teh", xt, _t64(W3))
     want = torch.einsum("teh,ehd->ted", torch.nn.functional.silu(g) * u, _t64(W2)).mean(1)
     np.testing.assert_allclose(y, want.numpy(), rtol=1e-12, atol=1e-13)
+
+
+def test_swiglu_shared_expert_alone():
+    """Routed experts all zero, SwiGLU shared expert: y = lam (SiLU(x Ws1) * (x Ws3)) Ws2."""
+    rng = _rng(63)
+    T, d, E, k, h, hs = 10, 16, 4, 2, 8, 24
+    x, Wr, b, W1, W2, Ws1, Ws2 = _layer(rng, T, d, E, k, h, hs)
+    W3 = _bf16(rng.standard_normal((E, d, h)) / np.sqrt(d))
+    Ws3 = _bf16(rng.standard_normal((d, hs)) / np.sqrt(d))
+    W1[:] = 0
+    W2[:] = 0
+    y, *_ = oracle.forward_tokens(x, Wr, b, W1, W2, k, Ws1, Ws2, 0.75, W3=W3, Ws3=Ws3)
+    xt = _t64(x)
+    want = 0.75 * ((torch.nn.functional.silu(xt @ _t64(Ws1)) * (xt @ _t64(Ws3))) @ _t64(Ws2))
+    np.testing.assert_allclose(y, want.numpy(), rtol=1e-12, atol=1e-13)
