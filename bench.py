@@ -93,10 +93,10 @@ def layer_work(cfg, counts, shared_groups=0):
     flops_router = 2.0 * T * d * E
     flops_up = 2.0 * up_mats * T * k * d * h
     flops_down = 2.0 * T * k * d * h
-    flops_shared = 4.0 * T * d * hs
+    flops_shared = 2.0 * (up_mats + 1) * T * d * hs
     touched = int((np.asarray(counts) > 0).sum())
     bytes_ = (T * d * 2 + T * d * 2 + d * E * 4 + E * 4 + touched * (up_mats + 1) * d * h * 2
-              + 2 * d * hs * 2 + 8 * T * k)
+              + (up_mats + 1) * d * hs * 2 + 8 * T * k)
     folded = shared_groups * h * T * d * 2.0
     return {"flops": flops_router + flops_up + flops_down + flops_shared,
             "flops_up_gemm": flops_up + folded,
@@ -169,7 +169,7 @@ def cpu_baseline(lay, target_s=15.0, max_tokens=None):
     rng = np.random.default_rng(123)
     probe = np.sort(rng.choice(cfg.T, size=min(cfg.T, max(nthreads, 8)), replace=False)).astype(np.int32)
     t0 = time.perf_counter()
-    oracle.forward_tokens(lay.x, lay.Wr, lay.b, lay.W1, lay.W2, cfg.k, lay.Ws1, lay.Ws2, cfg.lam, tokens=probe, W3=lay.W3)
+    oracle.forward_tokens(lay.x, lay.Wr, lay.b, lay.W1, lay.W2, cfg.k, lay.Ws1, lay.Ws2, cfg.lam, tokens=probe, W3=lay.W3, Ws3=lay.Ws3)
     per_tok = (time.perf_counter() - t0) / probe.size
     n = int(min(cfg.T, max(nthreads, target_s / max(per_tok, 1e-9))))
     if max_tokens:
@@ -179,7 +179,7 @@ def cpu_baseline(lay, target_s=15.0, max_tokens=None):
     passes, t0 = 0, time.perf_counter()
     while True:
         oracle.forward_tokens(lay.x, lay.Wr, lay.b, lay.W1, lay.W2, cfg.k, lay.Ws1, lay.Ws2, cfg.lam,
-                              tokens=toks, W3=lay.W3)
+                              tokens=toks, W3=lay.W3, Ws3=lay.Ws3)
         passes += 1
         dt = time.perf_counter() - t0
         if dt >= 0.66 * target_s or passes >= 8:
@@ -200,7 +200,7 @@ def run_reference(args, rank):
     # size each step so the whole run stays within a few minutes
     probe = np.arange(min(cfg.T, nthreads), dtype=np.int32)
     t0 = time.perf_counter()
-    oracle.forward_tokens(lay.x, lay.Wr, lay.b, lay.W1, lay.W2, cfg.k, lay.Ws1, lay.Ws2, cfg.lam, tokens=probe, W3=lay.W3)
+    oracle.forward_tokens(lay.x, lay.Wr, lay.b, lay.W1, lay.W2, cfg.k, lay.Ws1, lay.Ws2, cfg.lam, tokens=probe, W3=lay.W3, Ws3=lay.Ws3)
     per_tok = (time.perf_counter() - t0) / probe.size
     budget = 150.0 / max(1, args.steps + args.warmup)
     n = int(min(cfg.T, max(nthreads, budget / max(per_tok, 1e-9))))
@@ -209,7 +209,7 @@ def run_reference(args, rank):
         toks = np.sort(rng.choice(cfg.T, size=n, replace=False)).astype(np.int32)
         t0 = time.perf_counter()
         oracle.forward_tokens(lay.x, lay.Wr, lay.b, lay.W1, lay.W2, cfg.k, lay.Ws1, lay.Ws2, cfg.lam,
-                              tokens=toks, W3=lay.W3)
+                              tokens=toks, W3=lay.W3, Ws3=lay.Ws3)
         if i >= args.warmup:
             times.append(time.perf_counter() - t0)
     ms = 1e3 * statistics.mean(times)
@@ -246,7 +246,8 @@ def run_ours(args, rank, world):
                             W1=bf(lay.W1), W2=bf(lay.W2), k=cfg.k,
                             Ws1=None if lay.Ws1 is None else bf(lay.Ws1),
                             Ws2=None if lay.Ws2 is None else bf(lay.Ws2), lam=cfg.lam,
-                            W3=None if lay.W3 is None else bf(lay.W3))
+                            W3=None if lay.W3 is None else bf(lay.W3),
+                            Ws3=None if lay.Ws3 is None else bf(lay.Ws3))
     x = bf(lay.x)
     y = torch.empty((cfg.T, cfg.d), dtype=torch.bfloat16, device="cuda")
     ws = moevie.Workspace(cfg.T, cfg.d, cfg.E, cfg.k, cfg.h, cfg.h_s)

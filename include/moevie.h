@@ -124,8 +124,10 @@ typedef struct moevie_layer {
     float lambda;           /* weight of the shared expert */
     const void* W3;         /* bf16 [E, d, h] or NULL.  NULL: GELU experts GELU(x W1[e]) W2[e].
                              * Else SwiGLU experts (App. B): (SiLU(x W1[e]) * (x W3[e])) W2[e],
-                             * W1 the gate and W3 the up projection; with a SwiGLU layer
-                             * h_s must be 0 (MOEVIE_ERR_UNSUPPORTED otherwise). */
+                             * W1 the gate and W3 the up projection. */
+    const void* Ws3;        /* bf16 [d, h_s]: with W3, the shared expert's up projection
+                             * (SwiGLU shared expert (SiLU(x Ws1) * (x Ws3)) Ws2); ignored
+                             * without W3 or without a shared expert. */
 } moevie_layer;
 
 /* Optional routing by-products of moevie_moe_forward; any member may be NULL. */
@@ -199,7 +201,8 @@ uint64_t moevie_launch_count(void);
 moevie_status moevie_update_bias(const int32_t* counts, int64_t E, float alpha, int rule, float* b,
                                  void* ws, size_t ws_bytes, void* stream);
 
-/* Launch plan of moevie_moe_forward for these sizes (host-only, no GPU work; the
+/* Launch plan of moevie_moe_forward for these sizes (for a layer of GELU experts; a
+ * SwiGLU layer's shared expert always runs as its own GEMMs) (host-only, no GPU work; the
  * paper has no counterpart -- it describes how this library schedules Eq. 6's
  * shared term).  Returns the number S of always-on groups of width h that carry the
  * shared expert inside the routed up- and down-projection launches (its hidden units

@@ -213,6 +213,7 @@ struct GemmSpec {
     int64_t w2_g_ld;
     int g_split;
     const void* W3;          // EPI_SWIGLU_BF16: the up projection W3 [G][K][N] beside W1 = W (gate)
+    int a_ident;             // A rows contiguous but loaded by the gather warps (A row r = r)
 };
 
 moevie_status run_gemm(const GemmSpec& g, DevStatus* st, cudaStream_t s) {
@@ -240,6 +241,7 @@ moevie_status run_gemm(const GemmSpec& g, DevStatus* st, cudaStream_t s) {
     a.n_tiles_dev = g.n_tiles;
     a.max_mtiles = g.tiles ? max_mtiles(g.m_total, g.G) : (g.m_total + GM_BM - 1) / GM_BM;
     a.item_table = g.item_table;
+    a.a_ident = (g.a_ident && !g.a_rows) ? 1 : 0;
     // reduction staging: a full-warp buffer (5 stages) unless the work is band-ordered
     // (accumulator beyond L2, DRAM-bound: the sixth stage pays more)
     a.stg_rows = g.item_table ? 16 : 32;
@@ -403,7 +405,7 @@ moevie_status expert_up(const void* x, const int32_t* a_rows, int a_div, const i
 // (out != NULL) or lambda * S(x) as the first value of the fp32 y accumulator.
 moevie_status shared_expert(const void* x, const void* Ws1, const void* Ws2, int64_t T, int64_t d,
                             int64_t hs, void* out, float* yacc, float lambda, const Layout& L,
-                            void* ws, DevStatus* st, cudaStream_t s) {
+                            void* ws, DevStatus* st, cudaStream_t s, const void* Ws3 = nullptr) {
     void* Hs = at<void>(ws, L.Hs);
     GemmSpec g{};
     g.A = x;
@@ -415,6 +417,11 @@ moevie_status shared_expert(const void* x, const void* Ws1, const void* Ws2, int
     g.K = (int)d;
     g.N = (int)hs;
     g.epi = EPI_GELU_BF16;
+    if (Ws3) {   // SwiGLU shared expert: gate Ws1, up Ws3 (the SwiGLU epilogue runs with gathered A)
+        g.epi = EPI_SWIGLU_BF16;
+        g.W3 = Ws3;
+        g.a_ident = 1;
+    }
     g.out = Hs;
     g.ldo = hs;
     moevie_status c = run_gemm(g, st, s);
@@ -640,9 +647,10 @@ static moevie_status forward_impl(const moevie_layer* Lr, const void* x, int64_t
     if (T == 0) return MOEVIE_OK;
     if (!x || !y || !ws || !Lr->W_r || !Lr->b || !Lr->W1 || !Lr->W2) return MOEVIE_ERR_INVALID_ARG;
     if (hs > 0 && (!Lr->Ws1 || !Lr->Ws2)) return MOEVIE_ERR_INVALID_ARG;
-    if (Lr->W3 && hs > 0) return MOEVIE_ERR_UNSUPPORTED;   // a SwiGLU layer has no shared expert here
+    if (Lr->W3 && hs > 0 && !Lr->Ws3) return MOEVIE_ERR_INVALID_ARG;   // SwiGLU shared expert needs Ws3
     if (!a16(x) || !a16(y) || !a16(ws) || !a16(Lr->W1) || !a16(Lr->W2)) return MOEVIE_ERR_INVALID_ARG;
     if (Lr->W3 && !a16(Lr->W3)) return MOEVIE_ERR_INVALID_ARG;
+    if (Lr->W3 && hs > 0 && !a16(Lr->Ws3)) return MOEVIE_ERR_INVALID_ARG;
     if (hs > 0 && (!a16(Lr->Ws1) || !a16(Lr->Ws2))) return MOEVIE_ERR_INVALID_ARG;
     const Layout L = make_layout(T, d, E, k, h, hs);
     if (ws_bytes < L.total) return MOEVIE_ERR_WORKSPACE;
@@ -666,7 +674,8 @@ static moevie_status forward_impl(const moevie_layer* Lr, const void* x, int64_t
         return events ? cudaEventRecord(static_cast<cudaEvent_t>(events[i]), s) : cudaSuccess;
     };
 
-    const int64_t S = shared_chunks(T, d, E, k, h, hs);   // shared expert inside the grouped GEMMs
+    // shared expert inside the grouped GEMMs (GELU layers; a SwiGLU shared expert runs alone)
+    const int64_t S = Lr->W3 ? 0 : shared_chunks(T, d, E, k, h, hs);
     const int64_t n2 = T * k + S * T;
     MV_TRY(mark(0));
     // 1. router (Eqs. 1, 7, 4-5)
@@ -696,7 +705,8 @@ static moevie_status forward_impl(const moevie_layer* Lr, const void* x, int64_t
     // permute step); otherwise its own GEMMs write lambda * shared expert as the first
     // value of the y accumulator
     if (S == 0 && hs > 0) {
-        c = shared_expert(x, Lr->Ws1, Lr->Ws2, T, d, hs, nullptr, yacc, Lr->lambda, L, ws, st, s);
+        c = shared_expert(x, Lr->Ws1, Lr->Ws2, T, d, hs, nullptr, yacc, Lr->lambda, L, ws, st, s,
+                          Lr->W3 ? Lr->Ws3 : nullptr);
         if (c != MOEVIE_OK) return c;
     }
     MV_TRY(mark(3));

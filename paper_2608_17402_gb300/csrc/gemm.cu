@@ -341,7 +341,7 @@ __device__ __forceinline__ void gather_rows_load(const GemmArgs& p, const Tile& 
     for (int j = 0; j < GM_GATHER_ROWS; ++j) {
         const int r = rb + GM_GATHER_RSTEP * j;
         const int gr = t.row0 + (int)rank * GM_HALF + r;
-        raw[j] = (r < nh) ? __ldg(p.a_rows + gr) : -1;
+        raw[j] = (r < nh) ? (p.a_ident ? gr : __ldg(p.a_rows + gr)) : -1;
     }
 }
 
@@ -968,9 +968,10 @@ cudaError_t launch_grouped_gemm(const GemmArgs& a, int grid, cudaStream_t s) {
     using Kern = void (*)(GemmArgs);
     static const Kern kerns[3] = {grouped_gemm_kernel<32, false>, grouped_gemm_kernel<16, false>,
                                   grouped_gemm_kernel<32, true>};
-    if (a.a_rows && (a.epi == EPI_ADD_F32 || a.epi == EPI_SUM3_F32)) return cudaErrorInvalidValue;
-    if (!a.a_rows && a.epi == EPI_SWIGLU_BF16) return cudaErrorInvalidValue;
-    const Kern kern = a.a_rows ? kerns[2] : a.stg_rows == 32 ? kerns[0] : kerns[1];
+    const bool gathered = a.a_rows || a.a_ident;   // A rows through the gather warps
+    if (gathered && (a.epi == EPI_ADD_F32 || a.epi == EPI_SUM3_F32)) return cudaErrorInvalidValue;
+    if (!gathered && a.epi == EPI_SWIGLU_BF16) return cudaErrorInvalidValue;
+    const Kern kern = gathered ? kerns[2] : a.stg_rows == 32 ? kerns[0] : kerns[1];
     static bool attr_set[64] = {};
     int dev = 0;
     cudaGetDevice(&dev);

@@ -208,6 +208,7 @@ struct GemmArgs {
     const int4* tiles;          // m-tile table {g, row0, nrows, 0}; nullptr: one dense group;
                                 // with item_table: work items {g, row0, nrows, n0}
     int item_table;             // tiles lists (m-tile, n-tile) items; *n_tiles_dev counts items
+    int a_ident;                // gathered path with A row r = r (contiguous rows through cp.async)
     int stg_rows;               // EPI_ADD_F32: rows staged per warp and phase (32 or 16)
     const int32_t* n_tiles_dev; // number of entries of `tiles`
     int64_t max_mtiles;         // host bound on *n_tiles_dev

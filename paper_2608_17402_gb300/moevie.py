@@ -44,7 +44,7 @@ class _Layer(ctypes.Structure):
                 ("h", ctypes.c_int64), ("h_s", ctypes.c_int64),
                 ("W_r", ctypes.c_void_p), ("b", ctypes.c_void_p), ("W1", ctypes.c_void_p),
                 ("W2", ctypes.c_void_p), ("Ws1", ctypes.c_void_p), ("Ws2", ctypes.c_void_p),
-                ("lam", ctypes.c_float), ("W3", ctypes.c_void_p)]
+                ("lam", ctypes.c_float), ("W3", ctypes.c_void_p), ("Ws3", ctypes.c_void_p)]
 
 
 class _Routing(ctypes.Structure):
@@ -237,6 +237,7 @@ class LayerWeights:
     Ws2: torch.Tensor | None = None   # [h_s, d]
     lam: float = 1.0
     W3: torch.Tensor | None = None    # [E, d, h]: SwiGLU experts (W1 gate, W3 up); None: GELU
+    Ws3: torch.Tensor | None = None   # [d, h_s]: with W3, the SwiGLU shared expert's up projection
 
     @property
     def dims(self):
@@ -250,7 +251,8 @@ class LayerWeights:
         return _Layer(d, E, k, h, hs, self.W_r.data_ptr(), self.b.data_ptr(), self.W1.data_ptr(),
                       self.W2.data_ptr(), 0 if self.Ws1 is None else self.Ws1.data_ptr(),
                       0 if self.Ws2 is None else self.Ws2.data_ptr(), float(self.lam),
-                      0 if self.W3 is None else self.W3.data_ptr())
+                      0 if self.W3 is None else self.W3.data_ptr(),
+                      0 if self.Ws3 is None else self.Ws3.data_ptr())
 
 
 def moevie_moe_forward(layer: LayerWeights, x, ws: Workspace, y=None, routing=False, stream=None):

@@ -34,7 +34,8 @@ def layer_to_device(lay):
         W_r=dev(lay.Wr), b=dev(lay.b), W1=dev_bf16(lay.W1), W2=dev_bf16(lay.W2), k=lay.cfg.k,
         Ws1=None if lay.Ws1 is None else dev_bf16(lay.Ws1),
         Ws2=None if lay.Ws2 is None else dev_bf16(lay.Ws2), lam=lay.cfg.lam,
-        W3=None if lay.W3 is None else dev_bf16(lay.W3))
+        W3=None if lay.W3 is None else dev_bf16(lay.W3),
+        Ws3=None if lay.Ws3 is None else dev_bf16(lay.Ws3))
     return dev_bf16(lay.x), W
 
 

@@ -45,10 +45,17 @@ def test_swiglu_forward_image_batch_layer():
     print(f"s1: rel-L2 {rel:.2e}, max|err|/RMS {mx:.2e}")
 
 
-def test_swiglu_with_shared_expert_is_unsupported():
-    cfg = workloads.small_config(16, 64, 4, 2, 64, h_s=64, act="swiglu")
+@pytest.mark.parametrize("T,d,E,k,h,hs", [
+    (1, 64, 4, 2, 64, 64), (300, 128, 16, 4, 128, 256), (257, 64, 8, 2, 64, 96),
+])
+def test_swiglu_with_shared_expert(T, d, E, k, h, hs):
+    """A SwiGLU shared expert (Ws1 gate, Ws3 up) runs as its own GEMMs: the up-projection
+    through the gather warps with contiguous rows (the SwiGLU epilogue), then lambda times
+    its down-projection as the first value of the fp32 accumulator."""
+    cfg = workloads.small_config(T, d, E, k, h, h_s=hs, lam=0.5, seed=T + hs, act="swiglu")
     lay = workloads.make_layer(cfg)
-    x, W = layer_to_device(lay)
-    ws = workspace_for(lay)
-    with pytest.raises(moevie.MoevieError):
-        moevie.moevie_moe_forward(W, x, ws)
+    y, rt = _run(lay)
+    want, oidx, _, _ = oracle.forward_tokens(lay.x, lay.Wr, lay.b, lay.W1, lay.W2, k, lay.Ws1, lay.Ws2,
+                                             cfg.lam, W3=lay.W3, Ws3=lay.Ws3)
+    assert np.array_equal(rt["idx"], oidx)
+    assert_close(y, want)

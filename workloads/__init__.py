@@ -102,6 +102,7 @@ class LayerInputs:
     Ws2: np.ndarray | None = None   # uint16 [h_s, d]
     extra: dict = field(default_factory=dict)
     W3: np.ndarray | None = None    # uint16 [E, d, h], SwiGLU layers only
+    Ws3: np.ndarray | None = None   # uint16 [d, h_s], SwiGLU layers with a shared expert
 
 
 def _normal_bf16(rng: np.random.Generator, shape, std: float) -> np.ndarray:
@@ -140,9 +141,11 @@ def make_layer(cfg: LayerConfig, skew_offsets: np.ndarray | None = None,
     if cfg.h_s > 0:
         Ws1 = _normal_bf16(rng, (d, cfg.h_s), 1.0 / np.sqrt(d))
         Ws2 = _normal_bf16(rng, (cfg.h_s, d), 1.0 / np.sqrt(cfg.h_s))
-    W3 = None
+    W3 = Ws3 = None
     if cfg.act == "swiglu":   # drawn last: the GELU layers' draws are unchanged
         W3 = _normal_bf16(rng, (E, d, h), 1.0 / np.sqrt(d))
+        if cfg.h_s > 0:
+            Ws3 = _normal_bf16(rng, (d, cfg.h_s), 1.0 / np.sqrt(d))
     extra = {}
     if cfg.skew is not None:
         offs = skew_offsets if skew_offsets is not None else load_skew_offsets(cfg.skew)
@@ -155,7 +158,7 @@ def make_layer(cfg: LayerConfig, skew_offsets: np.ndarray | None = None,
             x[:, d - 1] = f32_to_bf16_bits(np.ones(1, np.float32))[0]
             Wr[d - 1, :] = offs
             extra["skew_offsets"] = offs
-    return LayerInputs(cfg, x, Wr, b, W1, W2, Ws1, Ws2, extra, W3)
+    return LayerInputs(cfg, x, Wr, b, W1, W2, Ws1, Ws2, extra, W3, Ws3)
 
 
 def small_config(T, d, E, k, h, h_s=0, lam=1.0, seed=0, name="small", act="gelu") -> LayerConfig:
