@@ -580,12 +580,12 @@ __device__ __forceinline__ void reduce_chunk(const GemmArgs& p, float* stg_all, 
 // per-warp staging buffer so that each 16-byte vector reduction instruction of a
 // warp covers four rows x 128 contiguous bytes, i.e. whole L2 lines.  When a warp has read
 // its last chunk of the accumulator it arrives (once) on the leader's tempty barrier.
-template <int STG_ROWS, bool GATHER>
+template <int STG_ROWS, bool GATHER, int ECLS>
 __device__ void epilogue(const GemmArgs& p, const Smem& sm, uint32_t tmem, int64_t n_work,
                          volatile int* abort_flag) {
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int quad = warp & 3, half = warp >> 2;
-    const bool to_f32 = (p.epi == EPI_ADD_F32 || p.epi == EPI_STORE_F32 || p.epi == EPI_SUM3_F32);
+    constexpr bool to_f32 = ECLS != ECLS_BF16;
     const int nchunk = p.BN / 32;
     // bf16 results are written once and read back later: let them leave L2 first
     const uint64_t stream_pol = l2_policy_evict_first();
@@ -614,7 +614,7 @@ __device__ void epilogue(const GemmArgs& p, const Smem& sm, uint32_t tmem, int64
         }
         tc_fence_after();
         const uint32_t tbase = tmem + ((uint32_t)(quad * 32) << 16) + (uint32_t)acc * GM_MAXBN;
-        if (!GATHER && p.epi == EPI_SUM3_F32) {
+        if (ECLS == ECLS_F32 && p.epi == EPI_SUM3_F32) {
             // three column groups of N / 3 (one n-tile): chunk ch of the output is the sum
             // of accumulator chunks ch, ch + nc3, ch + 2 nc3, added in that order
             const int nc3 = nchunk / 3;
@@ -652,7 +652,7 @@ __device__ void epilogue(const GemmArgs& p, const Smem& sm, uint32_t tmem, int64
             }
             continue;
         }
-        if (GATHER && p.epi == EPI_SWIGLU_BF16) {   // (only the gathered up-projection)
+        if (GATHER && ECLS == ECLS_BF16 && p.epi == EPI_SWIGLU_BF16) {   // (gathered A only)
             // output chunk ch (32 columns): gate = accumulator chunk ch, up = chunk ch + nout
             const int nout = nchunk / 2;
             if (half >= nout) {
@@ -704,7 +704,7 @@ __device__ void epilogue(const GemmArgs& p, const Smem& sm, uint32_t tmem, int64
         }
         for (int ch = half; ch < nchunk; ch += 2) {
             const int c0 = ch * 32;
-            if (!GATHER && p.epi == EPI_ADD_F32) {   // (a gathered GEMM never reduces)
+            if constexpr (ECLS == ECLS_ADD) {   // the y-accumulator reductions
                 uint32_t v[32];
                 tmem_ld_32x32b_x32(tbase + c0, v);
                 tmem_wait_ld();
@@ -728,7 +728,7 @@ __device__ void epilogue(const GemmArgs& p, const Smem& sm, uint32_t tmem, int64
             }
             if (!ok_row) continue;
             const int n = t.n0 + c0;
-            if (!to_f32) {
+            if constexpr (!to_f32) {
                 __nv_bfloat16* orow = p.out + (int64_t)gr * p.ldo + n;
 #pragma unroll
                 for (int g8 = 0; g8 < 4; ++g8) {
@@ -763,16 +763,16 @@ __device__ void epilogue(const GemmArgs& p, const Smem& sm, uint32_t tmem, int64
 
 // STG_ROWS: rows per warp of the reduction staging buffer (EPI_ADD_F32), one kernel
 // instance each so that the epilogue loops have constant trip counts.
-template <int STG_ROWS, bool GATHER>
+template <int STG_ROWS, bool GATHER, int ECLS>
 __global__ void __launch_bounds__(GM_THREADS, 1) grouped_gemm_kernel(const __grid_constant__ GemmArgs p) {
     extern __shared__ uint8_t gm_smem_raw[];
     uint8_t* smem = reinterpret_cast<uint8_t*>(
         (reinterpret_cast<uintptr_t>(gm_smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
     uint8_t* sA = smem;
-    const int nst = gm_stages(p.epi, STG_ROWS);
+    const int nst = gm_stages(ECLS == ECLS_ADD ? EPI_ADD_F32 : p.epi, STG_ROWS);
     uint8_t* sB = smem + nst * GM_A_BYTES;
     uint8_t* sStg = sB + nst * GM_B_BYTES;                       // reduction staging (EPI_ADD_F32)
-    uint64_t* bars = reinterpret_cast<uint64_t*>(sStg + gm_stg_bytes(p.epi, STG_ROWS));
+    uint64_t* bars = reinterpret_cast<uint64_t*>(sStg + gm_stg_bytes(ECLS == ECLS_ADD ? EPI_ADD_F32 : p.epi, STG_ROWS));
     uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 3 * GM_STAGES_MAX + 5);
     volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
     uint8_t* sink = reinterpret_cast<uint8_t*>(bars) + 256;   // 16-byte aligned, after the barriers
@@ -834,7 +834,7 @@ __global__ void __launch_bounds__(GM_THREADS, 1) grouped_gemm_kernel(const __gri
     const int64_t n_work = p.item_table ? n_mtiles * p.ksplit : n_mtiles * p.n_ntiles * p.ksplit;
 
     if (warp < GM_EPI_WARPS) {
-        epilogue<STG_ROWS, GATHER>(p, sm, tmem, n_work, abort_flag);
+        epilogue<STG_ROWS, GATHER, ECLS>(p, sm, tmem, n_work, abort_flag);
     } else if (warp == GM_WARP_MMA) {
         if ((threadIdx.x & 31) == 0 && sm.rank == 0) mma_issuer(p, sm, tmem, n_work, abort_flag);
     } else if (warp == GM_WARP_LOAD) {
@@ -845,7 +845,8 @@ __global__ void __launch_bounds__(GM_THREADS, 1) grouped_gemm_kernel(const __gri
         }
     } else if constexpr (GATHER) {
         producer_gather(p, sm, n_work, abort_flag);
-    } else if ((p.zero || p.nrm_out || p.wn_out) && warp >= GM_WARP_GATHER && warp < GM_WARP_FWD) {
+    } else if (!GATHER && ECLS == ECLS_F32 && (p.zero || p.nrm_out || p.wn_out) &&
+               warp >= GM_WARP_GATHER && warp < GM_WARP_FWD) {
         // Side jobs for the gather warps of a dense-A GEMM, while the MMAs run.
         // 1. Row norms of the A rows of this CTA's items (the router's |x_t|, read while
         //    the TMA brings the same rows in): one warp per row, lanes over 16-byte chunks;
@@ -963,15 +964,22 @@ void choose_bn(int N, int* BN, int* n_ntiles) {
 
 cudaError_t launch_grouped_gemm(const GemmArgs& a, int grid, cudaStream_t s) {
     if (a.stg_rows != 32 && a.stg_rows != 16) return cudaErrorInvalidValue;
-    // one instance per staging size (dense A) and one for gathered A (which never
-    // reduces): constant trip counts in the epilogue, and no code of the other mode
+    // one instance per (staging rows, A path, epilogue class): each holds only the code
+    // its launches run (constant trip counts, no other epilogue to crowd its registers)
     using Kern = void (*)(GemmArgs);
-    static const Kern kerns[3] = {grouped_gemm_kernel<32, false>, grouped_gemm_kernel<16, false>,
-                                  grouped_gemm_kernel<32, true>};
+    static const Kern kerns[5] = {
+        grouped_gemm_kernel<32, false, ECLS_ADD>, grouped_gemm_kernel<16, false, ECLS_ADD>,
+        grouped_gemm_kernel<32, false, ECLS_F32>, grouped_gemm_kernel<32, false, ECLS_BF16>,
+        grouped_gemm_kernel<32, true, ECLS_BF16>};
     const bool gathered = a.a_rows || a.a_ident;   // A rows through the gather warps
-    if (gathered && (a.epi == EPI_ADD_F32 || a.epi == EPI_SUM3_F32)) return cudaErrorInvalidValue;
+    const bool bf16_out = a.epi == EPI_GELU_BF16 || a.epi == EPI_STORE_BF16 || a.epi == EPI_SWIGLU_BF16;
+    if (gathered && !bf16_out) return cudaErrorInvalidValue;
     if (!gathered && a.epi == EPI_SWIGLU_BF16) return cudaErrorInvalidValue;
-    const Kern kern = gathered ? kerns[2] : a.stg_rows == 32 ? kerns[0] : kerns[1];
+    Kern kern;
+    if (gathered) kern = kerns[4];
+    else if (a.epi == EPI_ADD_F32) kern = a.stg_rows == 32 ? kerns[0] : kerns[1];
+    else if (a.epi == EPI_STORE_F32 || a.epi == EPI_SUM3_F32) kern = kerns[2];
+    else kern = kerns[3];
     static bool attr_set[64] = {};
     int dev = 0;
     cudaGetDevice(&dev);

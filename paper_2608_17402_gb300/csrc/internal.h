@@ -192,6 +192,9 @@ enum Epilogue : int {
                          //   n < N/3 (three column groups summed in a fixed order; one n-tile)
 };
 static_assert(EPI_ADD_F32 == 2, "gm_stages / gm_smem_bytes test the reduction epilogue by value");
+// Epilogue classes of the grouped GEMM's kernel instances: bf16 outputs (GELU, SwiGLU,
+// plain), fp32 stores (plain, three-group sums), fp32 reductions into the accumulator.
+enum { ECLS_BF16 = 0, ECLS_F32 = 1, ECLS_ADD = 2 };
 
 struct GemmArgs {
     CUtensorMap tmB;            // B = weights [G][K][N] bf16 (N contiguous), 3-D map {N, K, G}
