@@ -460,7 +460,10 @@ int route_ksplit(int64_t T, int d, int E) {
     choose_bn(cc ? 3 * route_epad(E) : E, &BN, &n_ntiles);
     const int64_t items = (T + GM_BM - 1) / GM_BM * n_ntiles;
     const int nkb = (cc ? 1 : 3) * route_dpad(d) / GM_BK;
-    int64_t p = items > 0 ? (ROUTE_SPLIT_TARGET + items - 1) / items : 1;
+    // work items to aim for: with the pieces side by side (K = d_pad) fewer, longer
+    // splits pay (measured: c1 64 items 4.8 us faster than 160)
+    const int64_t target = cc ? ROUTE_SPLIT_TARGET_CONCAT : ROUTE_SPLIT_TARGET;
+    int64_t p = items > 0 ? (target + items - 1) / items : 1;
     if (p > nkb / 3) p = nkb / 3;   // at least three K blocks per split
     if (p > ROUTE_MAX_KSPLIT) p = ROUTE_MAX_KSPLIT;
     return p < 1 ? 1 : (int)p;
