@@ -81,7 +81,7 @@ cudaError_t launch_route_split(const float* Wr, int d, int E, __nv_bfloat16* Wsp
 // ROUTE_SPLIT_TARGET items (ROUTE_SPLIT_TARGET_CONCAT with the pieces side by side),
 // at most ROUTE_MAX_KSPLIT, at least three K blocks each.
 // Depends on the sizes only (the workspace size uses it).
-constexpr int ROUTE_SPLIT_TARGET = 152;
+constexpr int ROUTE_SPLIT_TARGET = 76;
 constexpr int ROUTE_SPLIT_TARGET_CONCAT = 64;   // the same with the pieces side by side (E <= 64)
 constexpr int ROUTE_MAX_KSPLIT = 16;
 int route_ksplit(int64_t T, int d, int E);
