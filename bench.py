@@ -242,12 +242,15 @@ def run_ours(args, rank, world):
     def bf(a):
         return torch.from_numpy(np.ascontiguousarray(a).view(np.int16)).view(torch.bfloat16).cuda()
 
+    def rows(a):   # W1, W3, Ws1, Ws3: rows 16 bytes apart (h rounded up to 8)
+        return moevie.moevie_pad_rows(bf(a))
+
     W = moevie.LayerWeights(W_r=torch.from_numpy(lay.Wr).cuda(), b=torch.from_numpy(lay.b).cuda(),
-                            W1=bf(lay.W1), W2=bf(lay.W2), k=cfg.k,
-                            Ws1=None if lay.Ws1 is None else bf(lay.Ws1),
+                            W1=rows(lay.W1), W2=bf(lay.W2), k=cfg.k,
+                            Ws1=None if lay.Ws1 is None else rows(lay.Ws1),
                             Ws2=None if lay.Ws2 is None else bf(lay.Ws2), lam=cfg.lam,
-                            W3=None if lay.W3 is None else bf(lay.W3),
-                            Ws3=None if lay.Ws3 is None else bf(lay.Ws3))
+                            W3=None if lay.W3 is None else rows(lay.W3),
+                            Ws3=None if lay.Ws3 is None else rows(lay.Ws3))
     x = bf(lay.x)
     y = torch.empty((cfg.T, cfg.d), dtype=torch.bfloat16, device="cuda")
     ws = moevie.Workspace(cfg.T, cfg.d, cfg.E, cfg.k, cfg.h, cfg.h_s)

@@ -22,11 +22,16 @@
  *    (a cudaStream_t passed as void*; NULL is the legacy default stream) and runs
  *    asynchronously.
  *  - bf16 tensors are passed as void* pointing at __nv_bfloat16 data.  Matrices are
- *    row-major and dense: x[T, d], W1[E, d, h], W2[E, h, d], Ws1[d, h_s],
- *    Ws2[h_s, d], y[T, d]; W_r[d, E] and b[E] are fp32.
+ *    row-major: x[T, d], W1[E, d, h], W2[E, h, d], Ws1[d, h_s], Ws2[h_s, d],
+ *    y[T, d]; W_r[d, E] and b[E] are fp32.  Rows start 16 bytes apart: a matrix
+ *    whose rows hold h values has row stride hp = h rounded up to a multiple of 8
+ *    elements.  This matters only for W1 and W3 (stored [E][d][hp], expert stride
+ *    d*hp) and Ws1 and Ws3 ([d][h_s rounded up to 8]) when h or h_s is not a
+ *    multiple of 8 (the paper's L and H models: h = 684, 854); the pad columns are
+ *    never read.  Every other matrix is dense.
  *  - Device pointers must be 16-byte aligned.  Sizes must satisfy d % 8 == 0,
- *    h % 16 == 0, h_s % 16 == 0, 1 <= k <= E <= 1024 and T * k < 2^31;
- *    otherwise MOEVIE_ERR_UNSUPPORTED.  T == 0 is valid and launches nothing.
+ *    1 <= k <= E <= 1024 and T * k < 2^31; otherwise MOEVIE_ERR_UNSUPPORTED.
+ *    T == 0 is valid and launches nothing.
  *  - Argument errors are reported synchronously, before anything is enqueued.
  *    A failed kernel launch returns MOEVIE_ERR_CUDA.  Errors found on the device
  *    (an out-of-range expert id, a pipeline wait that ran past its time limit) are
@@ -117,15 +122,15 @@ typedef struct moevie_layer {
     int64_t h_s;            /* 0: no shared expert (Ws1, Ws2 ignored) */
     const float* W_r;       /* fp32 [d, E] */
     const float* b;         /* fp32 [E]    */
-    const void* W1;         /* bf16 [E, d, h] */
+    const void* W1;         /* bf16 [E, d, h], rows h rounded up to 8 apart */
     const void* W2;         /* bf16 [E, h, d] */
-    const void* Ws1;        /* bf16 [d, h_s]  */
+    const void* Ws1;        /* bf16 [d, h_s], rows h_s rounded up to 8 apart */
     const void* Ws2;        /* bf16 [h_s, d]  */
     float lambda;           /* weight of the shared expert */
-    const void* W3;         /* bf16 [E, d, h] or NULL.  NULL: GELU experts GELU(x W1[e]) W2[e].
+    const void* W3;         /* bf16 [E, d, h] (rows as W1) or NULL.  NULL: GELU experts GELU(x W1[e]) W2[e].
                              * Else SwiGLU experts (App. B): (SiLU(x W1[e]) * (x W3[e])) W2[e],
                              * W1 the gate and W3 the up projection. */
-    const void* Ws3;        /* bf16 [d, h_s]: with W3, the shared expert's up projection
+    const void* Ws3;        /* bf16 [d, h_s] (rows as Ws1): with W3, the shared expert's up projection
                              * (SwiGLU shared expert (SiLU(x Ws1) * (x Ws3)) Ws2); ignored
                              * without W3 or without a shared expert. */
 } moevie_layer;

@@ -31,7 +31,7 @@ moevie_status moevie_test_fallback_count(const void* ws, void* stream, int32_t* 
 
 /* The up-projection step alone (App. B, Algorithm 1, Kernel 1 with GELU):
  * hidden[r, :] = bf16(GELU(x[perm[r] / k] W1[e])) for r in expert e's segment.
- * hidden bf16 [T*k, h]. */
+ * hidden bf16 [T*k, h] with row stride h rounded up to a multiple of 8 (as W1). */
 moevie_status moevie_test_expert_hidden(const void* x, const int32_t* perm, const int32_t* offsets,
                                         const void* W1, int64_t T, int64_t d, int64_t h, int64_t E,
                                         int64_t k, void* hidden, void* ws, size_t ws_bytes,

@@ -23,6 +23,10 @@ constexpr uint64_t WAIT_LIMIT_NS = 2000000000ull;   // 2 s per pipeline wait
 
 inline size_t up256(size_t v) { return (v + 255) & ~static_cast<size_t>(255); }
 inline bool a16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+// Row stride (elements) of a bf16 matrix whose rows hold h values: W1, W3, Ws1, Ws3
+// and the hidden activations.  Rows start 16 bytes apart, as a TMA stride must; the
+// tensor maps cover the first h columns only, so the pad is never read.
+inline int64_t row_ld(int64_t h) { return (h + 7) / 8 * 8; }
 
 // Workspace carve-up.  Every buffer size is monotone in every size argument and
 // the order is fixed, so a workspace sized for the whole layer also serves each
@@ -77,8 +81,9 @@ BandPlan choose_bands(int64_t T, int64_t d, int64_t E, int64_t k, int64_t h) {
 constexpr int64_t SHARED_MAX_CHUNKS = 16;
 // Always-on groups the shapes allow (h divides h_s); the workspace reserves room for
 // them whatever the band decision, so that its size stays monotone in T.
+// Chunk c starts at column c h of Ws1, a TMA stride: h must be a multiple of 8.
 int64_t shared_chunks_max(int64_t h, int64_t hs) {
-    if (hs <= 0 || h <= 0 || hs % h != 0 || hs / h > SHARED_MAX_CHUNKS) return 0;
+    if (hs <= 0 || h <= 0 || h % 8 != 0 || hs % h != 0 || hs / h > SHARED_MAX_CHUNKS) return 0;
     return hs / h;
 }
 int64_t shared_chunks(int64_t T, int64_t d, int64_t E, int64_t k, int64_t h, int64_t hs) {
@@ -129,10 +134,10 @@ Layout make_layout(int64_t T, int64_t d, int64_t E, int64_t k, int64_t h, int64_
     L.inv = take(4 * n);
     L.row_tok = take(4 * n2);
     L.row_gate = take(4 * n2);
-    L.H = take(2 * n2 * h);
+    L.H = take(2 * n2 * row_ld(h));
     // the shared expert's own hidden [T, h_s]: with room for always-on groups it is the
     // tail of H (those S T rows of width h, the same bytes), used by one path or the other
-    L.Hs = S > 0 ? L.H + (size_t)(2 * n * h) : take(2 * T * hs);
+    L.Hs = S > 0 ? L.H + (size_t)(2 * n * h) : take(2 * T * row_ld(hs));
     L.yacc = take(4 * T * d);
     L.total = o;
     return L;
@@ -145,7 +150,7 @@ P* at(void* ws, size_t off) {
 
 moevie_status check_sizes(int64_t T, int64_t d, int64_t E, int64_t k, int64_t h, int64_t hs) {
     if (T < 0 || d <= 0 || E <= 0 || k <= 0 || h < 0 || hs < 0) return MOEVIE_ERR_INVALID_ARG;
-    if (d % 8 != 0 || h % 16 != 0 || hs % 16 != 0) return MOEVIE_ERR_UNSUPPORTED;
+    if (d % 8 != 0) return MOEVIE_ERR_UNSUPPORTED;
     if (k > E || E > 1024) return MOEVIE_ERR_UNSUPPORTED;
     if (T * k >= (int64_t(1) << 31) || T * route_epad((int)E) >= (int64_t(1) << 40) ||
         d >= (int64_t(1) << 24) || h >= (int64_t(1) << 24) || hs >= (int64_t(1) << 24))
@@ -174,6 +179,7 @@ inline moevie_status cuda_status(cudaError_t e) { return e == cudaSuccess ? MOEV
     } while (0)
 
 // One grouped GEMM launch: D = A[rows] . W[g], W bf16 [G][K][N] (row stride N_ld).
+// The weight tensor maps cover N columns and K rows: tiles past either edge read zeros.
 struct GemmSpec {
     const void* A;
     int64_t lda;
@@ -220,7 +226,9 @@ moevie_status run_gemm(const GemmSpec& g, DevStatus* st, cudaStream_t s) {
     GemmArgs a;
     memset(&a, 0, sizeof a);
     const int64_t n_ld = g.N_ld > 0 ? g.N_ld : g.N;
-    if (!make_weight_tmap(&a.tmB, g.W, n_ld, g.K, g.W2nd ? g.g_split : g.G)) return MOEVIE_ERR_CUDA;
+    if (n_ld < g.N || n_ld % 8 != 0) return MOEVIE_ERR_UNSUPPORTED;
+    if (!make_weight_tmap_strided(&a.tmB, g.W, g.N, g.K, g.W2nd ? g.g_split : g.G, n_ld, n_ld * g.K))
+        return MOEVIE_ERR_CUDA;
     if (g.W2nd) {
         if (g.g_split <= 0 || g.g_split >= g.G || !a16(g.W2nd) || g.w2_k_ld % 8 != 0 ||
             g.w2_g_ld % 8 != 0)
@@ -269,7 +277,8 @@ moevie_status run_gemm(const GemmSpec& g, DevStatus* st, cudaStream_t s) {
     a.swiglu = g.epi == EPI_SWIGLU_BF16 ? 1 : 0;
     if (a.swiglu) {   // gate (W1) and up (W3) tiles of 128 columns side by side: one N = 256 MMA
         if (!g.W3 || !a16(g.W3) || g.W2nd || g.ksplit > 1) return MOEVIE_ERR_UNSUPPORTED;
-        if (!make_weight_tmap(&a.tmB2, g.W3, n_ld, g.K, g.G)) return MOEVIE_ERR_CUDA;
+        if (!make_weight_tmap_strided(&a.tmB2, g.W3, g.N, g.K, g.G, n_ld, n_ld * g.K))
+            return MOEVIE_ERR_CUDA;
     }
     a.K = g.K;
     a.N = g.N;
@@ -395,9 +404,10 @@ moevie_status expert_up(const void* x, const int32_t* a_rows, int a_div, const i
     g.W = W1;
     g.K = (int)d;
     g.N = (int)h;
+    g.N_ld = row_ld(h);
     g.epi = EPI_GELU_BF16;
     g.out = hidden;
-    g.ldo = h;
+    g.ldo = row_ld(h);
     return run_gemm(g, st, s);
 }
 
@@ -416,6 +426,7 @@ moevie_status shared_expert(const void* x, const void* Ws1, const void* Ws2, int
     g.W = Ws1;
     g.K = (int)d;
     g.N = (int)hs;
+    g.N_ld = row_ld(hs);
     g.epi = EPI_GELU_BF16;
     if (Ws3) {   // SwiGLU shared expert: gate Ws1, up Ws3 (the SwiGLU epilogue runs with gathered A)
         g.epi = EPI_SWIGLU_BF16;
@@ -423,12 +434,12 @@ moevie_status shared_expert(const void* x, const void* Ws1, const void* Ws2, int
         g.a_ident = 1;
     }
     g.out = Hs;
-    g.ldo = hs;
+    g.ldo = row_ld(hs);
     moevie_status c = run_gemm(g, st, s);
     if (c != MOEVIE_OK) return c;
     GemmSpec g2{};
     g2.A = Hs;
-    g2.lda = hs;
+    g2.lda = row_ld(hs);
     g2.a_nrows = T;
     g2.m_total = T;
     g2.G = 1;
@@ -590,7 +601,7 @@ moevie_status moevie_expert_ffn(const void* x, const int32_t* perm, const int32_
     if (c != MOEVIE_OK) return c;
     GemmSpec g{};
     g.A = H;
-    g.lda = h;
+    g.lda = row_ld(h);
     g.a_nrows = T * k;
     g.m_total = T * k;
     g.tiles = tiles;
@@ -725,13 +736,14 @@ static moevie_status forward_impl(const moevie_layer* Lr, const void* x, int64_t
         up.W = Lr->W1;
         up.K = (int)d;
         up.N = (int)h;
+        up.N_ld = row_ld(h);
         up.epi = Lr->W3 ? EPI_SWIGLU_BF16 : EPI_GELU_BF16;
         up.W3 = Lr->W3;   // SwiGLU: W1 the gate, W3 the up projection
         up.out = at<void>(ws, L.H);
-        up.ldo = h;
+        up.ldo = row_ld(h);
         if (S > 0) {   // chunk c of Ws1 [d, h_s]: columns c h .. c h + h - 1
             up.W2nd = Lr->Ws1;
-            up.w2_k_ld = hs;
+            up.w2_k_ld = row_ld(hs);
             up.w2_g_ld = h;
             up.g_split = (int)E;
         }
@@ -741,7 +753,7 @@ static moevie_status forward_impl(const moevie_layer* Lr, const void* x, int64_t
     // 5. grouped down-projection, epilogue: gate * row added into y (scatter-add)
     GemmSpec dn{};
     dn.A = at<void>(ws, L.H);
-    dn.lda = h;
+    dn.lda = row_ld(h);
     dn.a_nrows = n2;
     dn.m_total = n2;
     dn.tiles = banded ? at<int4>(ws, L.items) : tiles;

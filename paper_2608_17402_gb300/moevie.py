@@ -115,6 +115,42 @@ def _want(t, dtype, name):
     return t
 
 
+def row_ld(h: int) -> int:
+    """Row stride (elements) of W1, W3, Ws1, Ws3 and the hidden activations when a
+    row holds h values: rows start 16 bytes apart (h rounded up to a multiple of 8)."""
+    return (h + 7) // 8 * 8
+
+
+def _rows_ok(t) -> bool:
+    """t [..., h] has row stride row_ld(h) and is otherwise packed."""
+    want = 1
+    for i in range(t.dim() - 1, -1, -1):
+        if t.shape[i] != 1 and t.stride(i) != want:
+            return False
+        want *= row_ld(t.shape[i]) if i == t.dim() - 1 else t.shape[i]
+    return True
+
+
+def moevie_pad_rows(w: torch.Tensor) -> torch.Tensor:
+    """``w`` [..., h] laid out as the entry points take W1, W3, Ws1 and Ws3 (row
+    stride ``row_ld(h)``, the pad never read): ``w`` itself when it already is, else
+    a copy into a zero-padded buffer, returned as its [..., h] view."""
+    if _rows_ok(w):
+        return w
+    h = w.shape[-1]
+    buf = torch.zeros(*w.shape[:-1], row_ld(h), dtype=w.dtype, device=w.device)
+    buf[..., :h].copy_(w)
+    return buf[..., :h]
+
+
+def _want_rows(t, dtype, name):
+    if not (t.is_cuda and t.dtype == dtype and _rows_ok(t)):
+        raise ValueError(f"{name}: expected a CUDA {dtype} tensor [..., h] with row stride "
+                         f"row_ld(h) (see moevie_pad_rows), got {t.dtype} on {t.device} with "
+                         f"shape {tuple(t.shape)} and strides {t.stride()}")
+    return t
+
+
 # ------------------------------------------------------------------ workspace
 
 def moevie_workspace_size(T_max, d, E, k, h, h_s=0) -> int:
@@ -194,7 +230,7 @@ def moevie_permute_static(idx, E, stream=None):
 
 def moevie_expert_ffn(x, perm, offsets, W1, W2, k, ws: Workspace, out_rows=None, stream=None):
     _want(x, torch.bfloat16, "x")
-    _want(W1, torch.bfloat16, "W1")
+    _want_rows(W1, torch.bfloat16, "W1")
     _want(W2, torch.bfloat16, "W2")
     T, d = x.shape
     E, _, h = W1.shape
@@ -207,6 +243,8 @@ def moevie_expert_ffn(x, perm, offsets, W1, W2, k, ws: Workspace, out_rows=None,
 
 def moevie_shared_expert(x, Ws1, Ws2, ws: Workspace, out=None, stream=None):
     _want(x, torch.bfloat16, "x")
+    _want_rows(Ws1, torch.bfloat16, "Ws1")
+    _want(Ws2, torch.bfloat16, "Ws2")
     T, d = x.shape
     hs = Ws1.shape[1]
     out = out if out is not None else torch.empty((T, d), dtype=torch.bfloat16, device=x.device)
@@ -230,14 +268,14 @@ class LayerWeights:
     """Device weights of one layer (bf16 unless noted)."""
     W_r: torch.Tensor           # fp32 [d, E]
     b: torch.Tensor             # fp32 [E]
-    W1: torch.Tensor            # [E, d, h]
+    W1: torch.Tensor            # [E, d, h], row stride row_ld(h) (moevie_pad_rows)
     W2: torch.Tensor            # [E, h, d]
     k: int
-    Ws1: torch.Tensor | None = None   # [d, h_s]
+    Ws1: torch.Tensor | None = None   # [d, h_s], row stride row_ld(h_s)
     Ws2: torch.Tensor | None = None   # [h_s, d]
     lam: float = 1.0
-    W3: torch.Tensor | None = None    # [E, d, h]: SwiGLU experts (W1 gate, W3 up); None: GELU
-    Ws3: torch.Tensor | None = None   # [d, h_s]: with W3, the SwiGLU shared expert's up projection
+    W3: torch.Tensor | None = None    # [E, d, h] as W1: SwiGLU experts (W1 gate, W3 up); None: GELU
+    Ws3: torch.Tensor | None = None   # [d, h_s] as Ws1: with W3, the SwiGLU shared expert's up
 
     @property
     def dims(self):
@@ -248,6 +286,9 @@ class LayerWeights:
 
     def c_struct(self) -> _Layer:
         d, E, k, h, hs = self.dims
+        for name in ("W1", "W3", "Ws1", "Ws3"):
+            if getattr(self, name) is not None:
+                _want_rows(getattr(self, name), torch.bfloat16, name)
         return _Layer(d, E, k, h, hs, self.W_r.data_ptr(), self.b.data_ptr(), self.W1.data_ptr(),
                       self.W2.data_ptr(), 0 if self.Ws1 is None else self.Ws1.data_ptr(),
                       0 if self.Ws2 is None else self.Ws2.data_ptr(), float(self.lam),
@@ -338,11 +379,12 @@ def moevie_test_fallback_count(ws: Workspace, stream=None) -> int:
 
 def moevie_test_expert_hidden(x, perm, offsets, W1, k, ws: Workspace, stream=None):
     T, d = x.shape
+    _want_rows(W1, torch.bfloat16, "W1")
     E, _, h = W1.shape
-    hidden = torch.empty((T * k, h), dtype=torch.bfloat16, device=x.device)
+    hidden = torch.empty((T * k, row_ld(h)), dtype=torch.bfloat16, device=x.device)
     _call("moevie_test_expert_hidden", _p(x), _p(perm), _p(offsets), _p(W1), T, d, h, E, k,
           _p(hidden), ws.ptr, ws.nbytes, _stream(stream))
-    return hidden
+    return hidden[:, :h]
 
 
 def moevie_test_wait_timeout(ws: Workspace, limit_ns: int, stream=None):

@@ -29,13 +29,18 @@ def to_np_f64(t: torch.Tensor) -> np.ndarray:
     return t.detach().float().cpu().numpy().astype(np.float64)
 
 
+def dev_rows(a_u16: np.ndarray) -> torch.Tensor:
+    """bf16 [..., h] with the row stride the entry points take for W1, W3, Ws1, Ws3."""
+    return moevie.moevie_pad_rows(dev_bf16(a_u16))
+
+
 def layer_to_device(lay):
     W = moevie.LayerWeights(
-        W_r=dev(lay.Wr), b=dev(lay.b), W1=dev_bf16(lay.W1), W2=dev_bf16(lay.W2), k=lay.cfg.k,
-        Ws1=None if lay.Ws1 is None else dev_bf16(lay.Ws1),
+        W_r=dev(lay.Wr), b=dev(lay.b), W1=dev_rows(lay.W1), W2=dev_bf16(lay.W2), k=lay.cfg.k,
+        Ws1=None if lay.Ws1 is None else dev_rows(lay.Ws1),
         Ws2=None if lay.Ws2 is None else dev_bf16(lay.Ws2), lam=lay.cfg.lam,
-        W3=None if lay.W3 is None else dev_bf16(lay.W3),
-        Ws3=None if lay.Ws3 is None else dev_bf16(lay.Ws3))
+        W3=None if lay.W3 is None else dev_rows(lay.W3),
+        Ws3=None if lay.Ws3 is None else dev_rows(lay.Ws3))
     return dev_bf16(lay.x), W
 
 

@@ -57,7 +57,11 @@ def test_workspace_size_monotone_and_validated(lib):
     rc, c = _ws_size(lib, 1024, 768, 16, 2, 768, 1024)
     assert rc == 0 and c > b
     assert _ws_size(lib, 512, 770, 16, 2, 768, 0)[0] == 2      # d % 8 != 0
-    assert _ws_size(lib, 512, 768, 16, 2, 760, 0)[0] == 2      # h % 16 != 0
+    # any hidden width: rows of W1 and of the hidden activations are padded to 8 elements
+    for h in (1, 13, 684, 760, 854):
+        rc, w = _ws_size(lib, 512, 768, 16, 2, h, h)
+        rc2, w2 = _ws_size(lib, 512, 768, 16, 2, h + 1, h + 1)
+        assert rc == 0 and rc2 == 0 and w2 >= w, h
     assert _ws_size(lib, 512, 768, 16, 17, 768, 0)[0] == 2     # k > E
     assert _ws_size(lib, 512, 768, 2048, 2, 768, 0)[0] == 2    # E > 1024
     assert _ws_size(lib, -1, 768, 16, 2, 768, 0)[0] == 1
@@ -89,7 +93,7 @@ def test_forward_rejects_bad_layer(lib):
     rc = lib.moevie_moe_forward(ctypes.byref(L), ctypes.c_void_p(fake), 4, ctypes.c_void_p(fake),
                                 None, ctypes.c_void_p(fake), 16, None)
     assert rc == 3   # workspace too small
-    L.h = 40         # h % 16 != 0
+    L.k = 9          # k > E
     rc = lib.moevie_moe_forward(ctypes.byref(L), ctypes.c_void_p(fake), 4, ctypes.c_void_p(fake),
                                 None, ctypes.c_void_p(fake), 1 << 30, None)
     assert rc == 2
@@ -109,6 +113,8 @@ def test_shared_groups_plan_and_monotone_workspace(lib):
     assert g(8192, 1024, 64, 8, 512, 0) == 0          # no shared expert
     assert g(65536, 1664, 256, 8, 416, 832) == 0      # band-ordered down-projection
     assert g(8192, 1023, 64, 8, 512, 1024) == 0       # invalid sizes
+    assert g(8192, 768, 31, 3, 512, 512) == 1         # the paper's B model: one shared expert
+    assert g(8192, 1024, 31, 3, 684, 684) == 0        # h % 8 != 0: chunk columns not 16-byte aligned
     d = 1024
     t_switch = (64 << 20) // (4 * d)                  # accumulator reaches 64 MiB
     assert g(t_switch, d, 64, 8, 512, 1024) == 2 and g(t_switch + 1, d, 64, 8, 512, 1024) == 0

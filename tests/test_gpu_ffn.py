@@ -8,7 +8,7 @@ import torch
 import oracle
 import workloads
 from paper_2608_17402_gb300 import moevie
-from tests._gpu import assert_close, check_status, dev, dev_bf16, to_np_f64
+from tests._gpu import assert_close, check_status, dev, dev_bf16, dev_rows, to_np_f64
 
 pytestmark = pytest.mark.gpu
 
@@ -40,6 +40,11 @@ SHAPES = [
     (4, 257, 1024, 3, 3, 512, None),      # k = E, long K loop
     (5, 40, 776, 2, 1, 48, None),         # d % 16 != 0 (8-column output tail), K tail in the up GEMM
     (6, 899, 192, 6, 1, 64, [0, 1, 255, 256, 257, 130]),   # segments around the 256-row m-tile
+    # hidden widths that are not multiples of 8 or 16 (rows of W1 and H padded to 8)
+    (7, 333, 256, 5, 2, 684, None),       # the paper's L width: N and K tails of 44
+    (8, 200, 128, 4, 2, 854, None),       # the paper's H width: 6 columns past a multiple of 8
+    (9, 150, 64, 3, 1, 13, [50, 0, 100]), # odd h below one output group
+    (10, 90, 96, 2, 2, 1, None),          # h = 1
 ]
 
 
@@ -47,7 +52,7 @@ SHAPES = [
 def test_expert_hidden_matches_oracle(seed, T, d, E, k, h, sizes):
     x, W1, W2, idx, counts, offsets, perm, inv = _case(seed, T, d, E, k, h, sizes)
     ws = moevie.Workspace(T, d, E, k, h)
-    hid = moevie.moevie_test_expert_hidden(dev_bf16(x), dev(perm), dev(offsets), dev_bf16(W1), k, ws)
+    hid = moevie.moevie_test_expert_hidden(dev_bf16(x), dev(perm), dev(offsets), dev_rows(W1), k, ws)
     check_status(ws)
     want = oracle.expert_rows(x, perm, offsets, W1, None, k, np.arange(T * k, dtype=np.int32), hidden=True)
     assert_close(to_np_f64(hid), want, "hidden")
@@ -57,20 +62,21 @@ def test_expert_hidden_matches_oracle(seed, T, d, E, k, h, sizes):
 def test_expert_ffn_matches_oracle(seed, T, d, E, k, h, sizes):
     x, W1, W2, idx, counts, offsets, perm, inv = _case(seed, T, d, E, k, h, sizes)
     ws = moevie.Workspace(T, d, E, k, h)
-    rows = moevie.moevie_expert_ffn(dev_bf16(x), dev(perm), dev(offsets), dev_bf16(W1), dev_bf16(W2), k, ws)
+    rows = moevie.moevie_expert_ffn(dev_bf16(x), dev(perm), dev(offsets), dev_rows(W1), dev_bf16(W2), k, ws)
     check_status(ws)
     want = oracle.expert_rows(x, perm, offsets, W1, W2, k, np.arange(T * k, dtype=np.int32))
     assert_close(to_np_f64(rows), want, "out_rows")
 
 
-def test_shared_expert_matches_oracle():
+@pytest.mark.parametrize("hs", [1024, 684])
+def test_shared_expert_matches_oracle(hs):
     rng = np.random.default_rng(9)
-    T, d, hs = 300, 256, 1024
+    T, d = 300, 256
     x = _bf(rng, (T, d))
     Ws1 = _bf(rng, (d, hs), 1 / np.sqrt(d))
     Ws2 = _bf(rng, (hs, d), 1 / np.sqrt(hs))
     ws = moevie.Workspace(T, d, 1, 1, 16, hs)
-    out = moevie.moevie_shared_expert(dev_bf16(x), dev_bf16(Ws1), dev_bf16(Ws2), ws)
+    out = moevie.moevie_shared_expert(dev_bf16(x), dev_rows(Ws1), dev_bf16(Ws2), ws)
     check_status(ws)
     # the shared expert is the single-expert layer E = 1, k = 1
     want, *_ = oracle.forward_tokens(x, np.zeros((d, 1), np.float32), np.zeros(1, np.float32),

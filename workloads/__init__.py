@@ -70,6 +70,16 @@ CONFIGS = {
     # SwiGLU experts (the paper's own FFN, App. B) at the image-batch layer's routed shape
     "s1": LayerConfig("s1", T=8192, d=1024, E=64, k=8, h=512, act="swiglu",
                       note="32 images x 256 patches, SwiGLU experts (W1 gate, W3 up), no shared expert"),
+    # The paper's own MoE-ViE-B / L / H layers (App. D, model table): 32 experts of width
+    # 512 / 684 / 854 per layer, one of them shared, 4 / 4 / 8 activated counting the
+    # shared one: E = 31 routed, k = 3 / 3 / 7, h_s = h, SwiGLU.  8192 tokens: 32 images
+    # x 256 patches (B, L), 8 images x 1024 patches at 448^2, patch 14 (H).
+    "pB": LayerConfig("pB", T=8192, d=768, E=31, k=3, h=512, h_s=512, act="swiglu",
+                      note="MoE-ViE-B layer: 31 routed + 1 shared SwiGLU experts of width 512"),
+    "pL": LayerConfig("pL", T=8192, d=1024, E=31, k=3, h=684, h_s=684, act="swiglu",
+                      note="MoE-ViE-L layer: 31 routed + 1 shared SwiGLU experts of width 684"),
+    "pH": LayerConfig("pH", T=8192, d=1280, E=31, k=7, h=854, h_s=854, act="swiglu",
+                      note="MoE-ViE-H layer: 31 routed + 1 shared SwiGLU experts of width 854"),
 }
 
 
