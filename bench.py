@@ -99,7 +99,7 @@ def layer_work(cfg, counts, shared_groups=0):
               + (up_mats + 1) * d * hs * 2 + 8 * T * k)
     folded = shared_groups * h * T * d * 2.0
     return {"flops": flops_router + flops_up + flops_down + flops_shared,
-            "flops_up_gemm": flops_up + folded,
+            "flops_up_gemm": flops_up + up_mats * folded,
             "flops_down_gemm": flops_down + folded, "bytes": float(bytes_), "touched_experts": touched}
 
 

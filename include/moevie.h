@@ -206,13 +206,13 @@ uint64_t moevie_launch_count(void);
 moevie_status moevie_update_bias(const int32_t* counts, int64_t E, float alpha, int rule, float* b,
                                  void* ws, size_t ws_bytes, void* stream);
 
-/* Launch plan of moevie_moe_forward for these sizes (for a layer of GELU experts; a
- * SwiGLU layer's shared expert always runs as its own GEMMs) (host-only, no GPU work; the
- * paper has no counterpart -- it describes how this library schedules Eq. 6's
- * shared term).  Returns the number S of always-on groups of width h that carry the
- * shared expert inside the routed up- and down-projection launches (its hidden units
- * in S = h_s / h chunks, every token with gate lambda), or 0 when it runs as its own
- * two GEMMs (no shared expert, h not dividing h_s, or a band-ordered down-projection).
+/* Launch plan of moevie_moe_forward for these sizes, GELU or SwiGLU experts alike
+ * (host-only, no GPU work; the paper has no counterpart -- it describes how this
+ * library schedules Eq. 6's shared term).  Returns the number S of always-on groups of
+ * width h that carry the shared expert inside the routed up- and down-projection
+ * launches (its hidden units in S = h_s / h chunks, every token with gate lambda), or 0
+ * when it runs as its own GEMMs (no shared expert, h not dividing h_s, several chunks
+ * of a width h that is not a multiple of 8, or a band-ordered down-projection).
  * Invalid sizes return 0. */
 int64_t moevie_shared_groups(int64_t T, int64_t d, int64_t E, int64_t k, int64_t h, int64_t h_s);
 

@@ -74,16 +74,19 @@ BandPlan choose_bands(int64_t T, int64_t d, int64_t E, int64_t k, int64_t h) {
 }
 
 // The shared expert runs inside the grouped GEMMs as S = h_s / h always-on groups
-// E .. E + S - 1 (its hidden units in chunks of h: GELU acts unit by unit, so the
-// chunks' down-projections add up to the shared expert's output), every token with
-// gate lambda, when h divides h_s and the down-projection is not band-ordered.
+// E .. E + S - 1 (its hidden units in chunks of h: GELU, like SiLU(gate) * up, acts
+// unit by unit, so the chunks' down-projections add up to the shared expert's output),
+// every token with gate lambda, when h divides h_s and the down-projection is not
+// band-ordered.
 // 0: the shared expert runs as its own dense GEMMs.
 constexpr int64_t SHARED_MAX_CHUNKS = 16;
 // Always-on groups the shapes allow (h divides h_s); the workspace reserves room for
 // them whatever the band decision, so that its size stays monotone in T.
-// Chunk c starts at column c h of Ws1, a TMA stride: h must be a multiple of 8.
+// Chunk c starts at column c h of Ws1 (and Ws3), h columns of a TMA stride apart: with
+// more than one chunk, h must be a multiple of 8.
 int64_t shared_chunks_max(int64_t h, int64_t hs) {
-    if (hs <= 0 || h <= 0 || h % 8 != 0 || hs % h != 0 || hs / h > SHARED_MAX_CHUNKS) return 0;
+    if (hs <= 0 || h <= 0 || hs % h != 0 || hs / h > SHARED_MAX_CHUNKS) return 0;
+    if (hs / h > 1 && h % 8 != 0) return 0;
     return hs / h;
 }
 int64_t shared_chunks(int64_t T, int64_t d, int64_t E, int64_t k, int64_t h, int64_t hs) {
@@ -137,7 +140,7 @@ Layout make_layout(int64_t T, int64_t d, int64_t E, int64_t k, int64_t h, int64_
     L.H = take(2 * n2 * row_ld(h));
     // the shared expert's own hidden [T, h_s]: with room for always-on groups it is the
     // tail of H (those S T rows of width h, the same bytes), used by one path or the other
-    L.Hs = S > 0 ? L.H + (size_t)(2 * n * h) : take(2 * T * row_ld(hs));
+    L.Hs = S > 0 ? L.H + (size_t)(2 * n * row_ld(h)) : take(2 * T * row_ld(hs));
     L.yacc = take(4 * T * d);
     L.total = o;
     return L;
@@ -219,6 +222,8 @@ struct GemmSpec {
     int64_t w2_g_ld;
     int g_split;
     const void* W3;          // EPI_SWIGLU_BF16: the up projection W3 [G][K][N] beside W1 = W (gate)
+    const void* W3_2nd;      // EPI_SWIGLU_BF16 with W2nd: the up projection of groups >= g_split
+                             //   (strides as W2nd, which then holds their gate)
     int a_ident;             // A rows contiguous but loaded by the gather warps (A row r = r)
 };
 
@@ -227,14 +232,22 @@ moevie_status run_gemm(const GemmSpec& g, DevStatus* st, cudaStream_t s) {
     memset(&a, 0, sizeof a);
     const int64_t n_ld = g.N_ld > 0 ? g.N_ld : g.N;
     if (n_ld < g.N || n_ld % 8 != 0) return MOEVIE_ERR_UNSUPPORTED;
+    const bool swiglu = g.epi == EPI_SWIGLU_BF16;
     if (!make_weight_tmap_strided(&a.tmB, g.W, g.N, g.K, g.W2nd ? g.g_split : g.G, n_ld, n_ld * g.K))
         return MOEVIE_ERR_CUDA;
-    if (g.W2nd) {
+    if (g.W2nd) {   // groups >= g_split (swiglu: their gate in tmB3, their up projection in tmB4)
         if (g.g_split <= 0 || g.g_split >= g.G || !a16(g.W2nd) || g.w2_k_ld % 8 != 0 ||
-            g.w2_g_ld % 8 != 0)
+            g.w2_g_ld % 8 != 0 || g.w2_k_ld < g.N)
             return MOEVIE_ERR_UNSUPPORTED;
-        if (!make_weight_tmap_strided(&a.tmB2, g.W2nd, g.N, g.K, g.G - g.g_split, g.w2_k_ld, g.w2_g_ld))
+        if (!make_weight_tmap_strided(swiglu ? &a.tmB3 : &a.tmB2, g.W2nd, g.N, g.K, g.G - g.g_split,
+                                      g.w2_k_ld, g.w2_g_ld))
             return MOEVIE_ERR_CUDA;
+        if (swiglu) {
+            if (!g.W3_2nd || !a16(g.W3_2nd)) return MOEVIE_ERR_UNSUPPORTED;
+            if (!make_weight_tmap_strided(&a.tmB4, g.W3_2nd, g.N, g.K, g.G - g.g_split, g.w2_k_ld,
+                                          g.w2_g_ld))
+                return MOEVIE_ERR_CUDA;
+        }
     }
     if (!g.a_rows && !make_rows_tmap(&a.tmA, g.A, g.a_cols > 0 ? g.a_cols : g.K, g.a_nrows, g.lda))
         return MOEVIE_ERR_CUDA;
@@ -274,9 +287,9 @@ moevie_status run_gemm(const GemmSpec& g, DevStatus* st, cudaStream_t s) {
     }
     a.G = g.G;
     a.g_split = g.W2nd ? g.g_split : g.G;
-    a.swiglu = g.epi == EPI_SWIGLU_BF16 ? 1 : 0;
+    a.swiglu = swiglu ? 1 : 0;
     if (a.swiglu) {   // gate (W1) and up (W3) tiles of 128 columns side by side: one N = 256 MMA
-        if (!g.W3 || !a16(g.W3) || g.W2nd || g.ksplit > 1) return MOEVIE_ERR_UNSUPPORTED;
+        if (!g.W3 || !a16(g.W3) || g.ksplit > 1) return MOEVIE_ERR_UNSUPPORTED;
         if (!make_weight_tmap_strided(&a.tmB2, g.W3, g.N, g.K, g.G, n_ld, n_ld * g.K))
             return MOEVIE_ERR_CUDA;
     }
@@ -685,8 +698,8 @@ static moevie_status forward_impl(const moevie_layer* Lr, const void* x, int64_t
         return events ? cudaEventRecord(static_cast<cudaEvent_t>(events[i]), s) : cudaSuccess;
     };
 
-    // shared expert inside the grouped GEMMs (GELU layers; a SwiGLU shared expert runs alone)
-    const int64_t S = Lr->W3 ? 0 : shared_chunks(T, d, E, k, h, hs);
+    // shared expert inside the grouped GEMMs (GELU or SwiGLU: both act unit by unit)
+    const int64_t S = shared_chunks(T, d, E, k, h, hs);
     const int64_t n2 = T * k + S * T;
     MV_TRY(mark(0));
     // 1. router (Eqs. 1, 7, 4-5)
@@ -741,10 +754,11 @@ static moevie_status forward_impl(const moevie_layer* Lr, const void* x, int64_t
         up.W3 = Lr->W3;   // SwiGLU: W1 the gate, W3 the up projection
         up.out = at<void>(ws, L.H);
         up.ldo = row_ld(h);
-        if (S > 0) {   // chunk c of Ws1 [d, h_s]: columns c h .. c h + h - 1
+        if (S > 0) {   // chunk c of Ws1 [d, h_s] (and of Ws3): columns c h .. c h + h - 1
             up.W2nd = Lr->Ws1;
+            up.W3_2nd = Lr->W3 ? Lr->Ws3 : nullptr;
             up.w2_k_ld = row_ld(hs);
-            up.w2_g_ld = h;
+            up.w2_g_ld = S > 1 ? h : row_ld(hs) * d;   // one chunk: any stride of 16-byte multiples
             up.g_split = (int)E;
         }
         if ((c = run_gemm(up, st, s)) != MOEVIE_OK) return c;

@@ -284,6 +284,10 @@ __device__ void producer_tma(const GemmArgs& p, const Smem& sm, int64_t n_work,
                              volatile int* abort_flag) {
     tma_prefetch_desc(&p.tmB);
     if (p.g_split < p.G || p.swiglu) tma_prefetch_desc(&p.tmB2);
+    if (p.g_split < p.G && p.swiglu) {
+        tma_prefetch_desc(&p.tmB3);
+        tma_prefetch_desc(&p.tmB4);
+    }
     constexpr bool gather = GATHER;
     if (!gather) tma_prefetch_desc(&p.tmA);
     const uint32_t half_n = (uint32_t)p.BN / 2;
@@ -301,11 +305,13 @@ __device__ void producer_tma(const GemmArgs& p, const Smem& sm, int64_t n_work,
         const int64_t wn = w + sm.npairs;
         TileLd nl{};
         if (wn < n_work) nl = tile_load(p, wn);   // checked after this item's loads
-        // B of this group from the second map (groups >= g_split; with swiglu, the second
-        // CTA of the pair: W3 beside W1's columns)
-        const bool second = p.swiglu ? sm.rank == 1 : t.g >= p.g_split;
-        const CUtensorMap* tmb = second ? &p.tmB2 : &p.tmB;
-        const int gb = (second && !p.swiglu) ? t.g - p.g_split : t.g;
+        // B of this group: groups >= g_split from their own map; with swiglu the second
+        // CTA of the pair loads the up projection (W3) beside the gate's (W1) columns
+        const bool tail = t.g >= p.g_split;
+        const CUtensorMap* tmb = tail ? &p.tmB2 : &p.tmB;
+        if (p.swiglu)
+            tmb = sm.rank == 1 ? (tail ? &p.tmB4 : &p.tmB2) : (tail ? &p.tmB3 : &p.tmB);
+        const int gb = tail ? t.g - p.g_split : t.g;
         const int ncol0 = p.swiglu ? t.n0 : t.n0 + (int)(sm.rank * half_n);
         for (int kb = t.kb0; kb < t.kb1; ++kb) {
             if (!mbar_wait(sm.empty + 8 * s, ph ^ 1u, p.limit_ns, abort_flag)) {

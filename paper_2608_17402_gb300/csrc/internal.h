@@ -201,6 +201,8 @@ enum { ECLS_BF16 = 0, ECLS_F32 = 1, ECLS_ADD = 2 };
 struct GemmArgs {
     CUtensorMap tmB;            // B = weights [G][K][N] bf16 (N contiguous), 3-D map {N, K, G}
     CUtensorMap tmB2;           // groups g >= g_split: B from this map, group g - g_split
+    CUtensorMap tmB3;           // swiglu with groups g >= g_split: their gate (CTA rank 0) and
+    CUtensorMap tmB4;           //   up (rank 1) weights, group g - g_split
     CUtensorMap tmA;            // A = rows [a_nrows][K_A] bf16, 2-D map {K_A, a_nrows}, box
                                 // {64, 128}; used when A rows are contiguous (a_rows == nullptr)
     const __nv_bfloat16* A;     // A rows, for the token gather
@@ -219,7 +221,8 @@ struct GemmArgs {
     int64_t max_mtiles;         // host bound on *n_tiles_dev
     int G, K, N, BN, n_ntiles, num_kb, nbox;
     int g_split;                // first group read through tmB2 (G when there is none)
-    int swiglu;                 // EPI_SWIGLU_BF16: B half of CTA rank 1 from tmB2 (W3), same columns
+    int swiglu;                 // EPI_SWIGLU_BF16: B half of CTA rank 1 from tmB2 (W3), same columns;
+                                // groups g >= g_split from tmB3 (rank 0) and tmB4 (rank 1)
     int n_step;                 // output columns per n-tile (BN; BN / 2 with swiglu)
     int ksplit;                 // K is split into this many parts (work items), >= 1
     int64_t y_split_stride;     // fp32 outputs: split ks writes yacc + ks * y_split_stride

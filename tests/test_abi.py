@@ -114,7 +114,8 @@ def test_shared_groups_plan_and_monotone_workspace(lib):
     assert g(65536, 1664, 256, 8, 416, 832) == 0      # band-ordered down-projection
     assert g(8192, 1023, 64, 8, 512, 1024) == 0       # invalid sizes
     assert g(8192, 768, 31, 3, 512, 512) == 1         # the paper's B model: one shared expert
-    assert g(8192, 1024, 31, 3, 684, 684) == 0        # h % 8 != 0: chunk columns not 16-byte aligned
+    assert g(8192, 1024, 31, 3, 684, 684) == 1        # one chunk of a width that is not a multiple of 8
+    assert g(8192, 1024, 31, 3, 684, 1368) == 0       # chunk 1 would start off a 16-byte boundary
     d = 1024
     t_switch = (64 << 20) // (4 * d)                  # accumulator reaches 64 MiB
     assert g(t_switch, d, 64, 8, 512, 1024) == 2 and g(t_switch + 1, d, 64, 8, 512, 1024) == 0

@@ -41,7 +41,7 @@ def _want(lay, tokens=None):
 
 
 @pytest.mark.parametrize("T,d,E,k,h,hs,act", [
-    (300, 256, 31, 3, 684, 684, "swiglu"),   # L widths at a small T and d
+    (300, 256, 31, 3, 684, 684, "swiglu"),   # L widths at a small T and d (shared: one always-on group)
     (257, 128, 31, 7, 854, 854, "swiglu"),   # H widths
     (130, 192, 8, 2, 684, 0, "gelu"),
     (200, 128, 8, 3, 100, 300, "gelu"),      # h % 8 == 4; the shared expert runs as its own GEMMs
@@ -58,9 +58,11 @@ def test_ragged_hidden_width_small(T, d, E, k, h, hs, act):
 
 @pytest.mark.parametrize("name", ["pB", "pL", "pH"])
 def test_paper_layer_sampled(name):
-    """Full-size layer, all routing outputs, and a sample of output rows."""
+    """Full-size layer, all routing outputs, and a sample of output rows.  The shared
+    expert (h_s = h) rides in the routed launches as one always-on group."""
     lay = workloads.make_layer(workloads.CONFIGS[name])
     c = lay.cfg
+    assert moevie.moevie_shared_groups(c.T, c.d, c.E, c.k, c.h, c.h_s) == 1
     y, rt = _run(lay)
     oidx, ogate, margin = oracle.route(lay.x, lay.Wr, lay.b, c.k)
     assert (margin > MARGIN_PINNED).all()

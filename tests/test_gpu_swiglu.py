@@ -49,9 +49,12 @@ def test_swiglu_forward_image_batch_layer():
     (1, 64, 4, 2, 64, 64), (300, 128, 16, 4, 128, 256), (257, 64, 8, 2, 64, 96),
 ])
 def test_swiglu_with_shared_expert(T, d, E, k, h, hs):
-    """A SwiGLU shared expert (Ws1 gate, Ws3 up) runs as its own GEMMs: the up-projection
-    through the gather warps with contiguous rows (the SwiGLU epilogue), then lambda times
+    """A SwiGLU shared expert (Ws1 gate, Ws3 up).  When h divides h_s it runs as h_s / h
+    always-on groups of the routed launches (the first two cases: the gate chunks of Ws1
+    on the pair's first CTA, those of Ws3 on the second); otherwise as its own GEMMs,
+    the up-projection through the gather warps with contiguous rows, then lambda times
     its down-projection as the first value of the fp32 accumulator."""
+    assert moevie.moevie_shared_groups(T, d, E, k, h, hs) == (hs // h if hs % h == 0 else 0)
     cfg = workloads.small_config(T, d, E, k, h, h_s=hs, lam=0.5, seed=T + hs, act="swiglu")
     lay = workloads.make_layer(cfg)
     y, rt = _run(lay)
