@@ -24,9 +24,10 @@
 //  3. route_fallback_kernel: one CTA per uncertified token.  An expert is surely in
 //     when its lower end is above the k-th largest upper end of the others, surely
 //     out when its upper end is below the k-th largest lower end; the rest get exact
-//     logits (fp64: each product of a bf16 and an fp32 value is exact in double, and
-//     the sum of d terms has relative error below d 2^-53; one warp per candidate),
-//     and the remaining places are filled from them, ties to the lower id.
+//     logits (each product of a bf16 and an fp32 value is an integer of at most 32 bits
+//     times a power of two; the block sums them in a 128-bit fixed-point accumulator on
+//     the integer pipes, see long_acc_term), and the remaining places are filled from
+//     their keys (fp64), ties to the lower id.
 #include <math.h>
 
 #include "internal.h"
@@ -272,27 +273,73 @@ __device__ __forceinline__ void warp_kth_values(const float (&v)[NPL], int E, in
     }
 }
 
-__device__ __forceinline__ double dot_bf16x8_f32x8(const uint4& xq, const float4& w0,
-                                                   const float4& w1) {
-    float xv[8];
-    unpack_bf16x8(xq, xv);
-    double a = (double)xv[0] * (double)w0.x;
-    a = fma((double)xv[1], (double)w0.y, a);
-    a = fma((double)xv[2], (double)w0.z, a);
-    a = fma((double)xv[3], (double)w0.w, a);
-    a = fma((double)xv[4], (double)w1.x, a);
-    a = fma((double)xv[5], (double)w1.y, a);
-    a = fma((double)xv[6], (double)w1.z, a);
-    a = fma((double)xv[7], (double)w1.w, a);
-    return a;
+// Exact logits by a long fixed-point accumulator (the exact dot product of Kulisch
+// and Miranker, with a window fitted to the operands).  A bf16 x_i is mx 2^(ex - 134)
+// and an fp32 w_i is mw 2^(ew - 150) (mx < 2^8, mw < 2^24 integers; ex, ew the biased
+// exponents, 1 for subnormals), so x_i w_i = P 2^(q - 284) with the integer P = mx mw
+// < 2^32 and q = ex + ew.  With Q >= every q, the term is P 2^(64 - (Q - q)) units of
+// 2^(Q - 348): a left shift (exact) when Q - q <= 64, else a right shift that drops less
+// than one unit.  The units of d terms sum in a 128-bit integer (|sum| < 2^120 for
+// d < 2^24), exactly and in any order; the logit is that sum times 2^(Q - 348), within
+// d 2^(Q - 348) + 2^-51 |s| of the exact value.  Q is the largest q of the candidate's
+// terms, whose P is at least 1, so d 2^(Q - 348) <= d 2^-64 sum|x_i w_i|: below the
+// d 2^-53 sum|x_i w_i| of an fp64 sum.  Everything but the final conversion runs on the
+// integer pipes.
+constexpr int FB_CB = 32;   // candidates per batch (one per lane of the finishing warp)
+
+__device__ __forceinline__ int bf16_exp_field(uint32_t hx) { return (int)((hx >> 7) & 0xffu); }
+__device__ __forceinline__ int f32_exp_field(uint32_t uw) { return (int)((uw >> 23) & 0xffu); }
+
+// q of the term x w (subnormals as exponent 1), plus 1024 when x or w is not finite.
+__device__ __forceinline__ int long_acc_q(uint32_t hx, uint32_t uw) {
+    const int ex = bf16_exp_field(hx), ew = f32_exp_field(uw);
+    return max(ex, 1) + max(ew, 1) + ((ex == 255 || ew == 255) ? 1024 : 0);
+}
+
+// acc += x w in units of 2^(Q - 348) (hx: bf16 bits of x, uw: fp32 bits of w).
+__device__ __forceinline__ void long_acc_term(uint32_t hx, uint32_t uw, int Q, unsigned __int128& acc) {
+    const int ex = bf16_exp_field(hx), ew = f32_exp_field(uw);
+    const uint64_t mx = (hx & 0x7fu) | (ex ? 0x80u : 0u);
+    const uint64_t mw = (uw & 0x7fffffu) | (ew ? 0x800000u : 0u);
+    const uint64_t P = mx * mw;
+    const int sh = 64 - (Q - (max(ex, 1) + max(ew, 1)));   // <= 64
+    unsigned __int128 t;
+    if (sh >= 0) t = (unsigned __int128)P << sh;
+    else t = sh > -64 ? (unsigned __int128)(P >> -sh) : (unsigned __int128)0;
+    if ((hx ^ (uw >> 16)) & 0x8000u) acc -= t;
+    else acc += t;
+}
+
+__device__ __forceinline__ unsigned __int128 warp_sum_u128(unsigned __int128 v) {
+#pragma unroll
+    for (int o = 16; o; o >>= 1) {
+        const uint64_t lo = __shfl_xor_sync(0xffffffffu, (unsigned long long)(uint64_t)v, o);
+        const uint64_t hi = __shfl_xor_sync(0xffffffffu, (unsigned long long)(uint64_t)(v >> 64), o);
+        v += ((unsigned __int128)hi << 64) | lo;
+    }
+    return v;
+}
+
+// The signed 128-bit sum `u` (two's complement) times 2^(Q - 348), in double: the
+// magnitude's two 64-bit words are rounded and added (relative error below 3 2^-53).
+__device__ __forceinline__ double long_acc_value(unsigned __int128 u, int Q) {
+    const bool neg = (long long)(uint64_t)(u >> 64) < 0;
+    const unsigned __int128 m = neg ? (unsigned __int128)0 - u : u;
+    const double hi = (double)(unsigned long long)(uint64_t)(m >> 64);
+    const double lo = (double)(unsigned long long)(uint64_t)m;
+    const double v = fma(hi, 18446744073709551616.0, lo);   // hi 2^64 + lo
+    // 2^(Q - 348) with 2 <= Q <= 508: a normal double, so the product is exact
+    const double r = v * __longlong_as_double((long long)((uint64_t)(Q - 348 + 1023) << 52));
+    return neg ? -r : r;
 }
 
 // Exact re-decision of uncertified tokens, one CTA (8 warps) per token.  Warp 0
-// bounds the keys and lists the candidates; every warp computes exact logits of its
-// candidates (lanes over d, reading the transposed fp32 copy of W_r); warp 0 fills
-// the remaining places from the exact keys and writes ids and gates.
+// bounds the keys and lists the candidates; then all 256 threads form the candidates'
+// logits in the long accumulator (threads over d, reading the transposed fp32 copy of
+// W_r), and warp 0
+// fills the remaining places from the exact keys and writes ids and gates.
 template <int NPL>
-__global__ void __launch_bounds__(256) route_fallback_kernel(
+__global__ void __launch_bounds__(256, 1) route_fallback_kernel(
     const __nv_bfloat16* __restrict__ x, const float* __restrict__ wrt, int dp,
     const float* __restrict__ b, const float* __restrict__ s, int ld,
     const float* __restrict__ xnorm, const float* __restrict__ wnorm, int d, int E, int k,
@@ -302,11 +349,16 @@ __global__ void __launch_bounds__(256) route_fallback_kernel(
     __shared__ int s_cand[32 * NPL];
     __shared__ double s_key[32 * NPL];
     __shared__ int s_ncand;
+    __shared__ int s_qmax[FB_CB];                 // largest term q of each batched candidate
+    __shared__ unsigned long long s_acc[2][8][FB_CB];   // per-warp sums: low, high words
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const uint32_t lt = (1u << lane) - 1u;
+    if (threadIdx.x < FB_CB) s_qmax[threadIdx.x] = 2;
+    __syncthreads();
     const int nfb = st->fb_count;
     for (int f = blockIdx.x; f < nfb; f += gridDim.x) {
         const int t = fb_tokens[f];
+        const uint16_t* xh = reinterpret_cast<const uint16_t*>(x) + (int64_t)t * d;
         float sv[NPL];
         uint32_t sure_in = 0, cand = 0;
         int need = 0;
@@ -357,27 +409,41 @@ __global__ void __launch_bounds__(256) route_fallback_kernel(
         }
         __syncthreads();
         const int nc = s_ncand;
-        const uint4* xr = reinterpret_cast<const uint4*>(x + (int64_t)t * d);
-        const int nchunk = d / 8;
-        for (int c = warp; c < nc; c += 8) {
-            const int e = s_cand[c];
-            const float4* wr = reinterpret_cast<const float4*>(wrt + (int64_t)e * dp);
-            double acc0 = 0.0, acc1 = 0.0;
-            int j = lane;
-            for (; j + 32 < nchunk; j += 64) {
-                const uint4 xa = xr[j], xb = xr[j + 32];
-                const float4 wa0 = wr[2 * j], wa1 = wr[2 * j + 1];
-                const float4 wb0 = wr[2 * (j + 32)], wb1 = wr[2 * (j + 32) + 1];
-                acc0 += dot_bf16x8_f32x8(xa, wa0, wa1);
-                acc1 += dot_bf16x8_f32x8(xb, wb0, wb1);
+        for (int c0 = 0; c0 < nc; c0 += FB_CB) {
+            const int cn = min(FB_CB, nc - c0);
+            for (int c = 0; c < cn; ++c) {   // the window of each candidate: its largest term q
+                const uint32_t* wcol = reinterpret_cast<const uint32_t*>(wrt + (int64_t)s_cand[c0 + c] * dp);
+                int m = 2;
+                for (int i = threadIdx.x; i < d; i += 256) m = max(m, long_acc_q(xh[i], wcol[i]));
+                m = __reduce_max_sync(0xffffffffu, m);
+                if (lane == 0) atomicMax(&s_qmax[c], m);
             }
-            if (j < nchunk) acc0 += dot_bf16x8_f32x8(xr[j], wr[2 * j], wr[2 * j + 1]);
-            double v = acc0 + acc1;
+            __syncthreads();
+            for (int c = 0; c < cn; ++c) {
+                const uint32_t* wcol = reinterpret_cast<const uint32_t*>(wrt + (int64_t)s_cand[c0 + c] * dp);
+                const int Q = s_qmax[c];   // the same in every thread
+                unsigned __int128 acc = 0;
+                if (Q < 1024) {   // finite inputs (else the logit is NaN): every q <= Q
+                    for (int i = threadIdx.x; i < d; i += 256) long_acc_term(xh[i], wcol[i], Q, acc);
+                    acc = warp_sum_u128(acc);
+                }
+                if (lane == 0) {
+                    s_acc[0][warp][c] = (unsigned long long)(uint64_t)acc;
+                    s_acc[1][warp][c] = (unsigned long long)(uint64_t)(acc >> 64);
+                }
+            }
+            __syncthreads();
+            if (warp == 0 && lane < cn) {   // exact logit of candidate c0 + lane (NaN for non-finite inputs)
+                unsigned __int128 u = 0;
 #pragma unroll
-            for (int o = 16; o; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
-            if (lane == 0) s_key[c] = v;   // exact logit; its key is formed below
+                for (int w = 0; w < 8; ++w)
+                    u += ((unsigned __int128)s_acc[1][w][lane] << 64) | s_acc[0][w][lane];
+                s_key[c0 + lane] = s_qmax[lane] < 1024 ? long_acc_value(u, s_qmax[lane])
+                                                       : __longlong_as_double(0x7ff8000000000000ll);
+            }
+            if (warp == 0 && lane < FB_CB) s_qmax[lane] = 2;   // for the next batch / token
+            __syncthreads();
         }
-        __syncthreads();
         if (warp == 0 && nc >= 0) {
             // keys of all candidates at once, one per lane (fp64 is slow: run it in parallel)
             for (int c = lane; c < nc; c += 32) s_key[c] = 1.0 / (1.0 + exp(-s_key[c])) + (double)b[s_cand[c]];

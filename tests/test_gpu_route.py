@@ -62,6 +62,30 @@ def test_route_exact_ties_go_to_lower_id():
     np.testing.assert_allclose(gate, ogate, rtol=0, atol=1e-5)
 
 
+def test_route_exact_redecision_stress():
+    """Inputs that send almost every token through the exact re-decision and stress its
+    long accumulator: two rows whose products cancel exactly (x[:, 1] = x[:, 0],
+    W_r[1] = -W_r[0] = 1024 r), which makes the fast-path error bound large; rows of
+    tiny (2^-40) and subnormal weights, whose products fall far below the others; and a
+    near-duplicate column whose logit differs from its twin by x[:, 10] 2^-20 only."""
+    rng = np.random.default_rng(12)
+    T, d, E, k = 256, 96, 24, 4
+    xf = rng.standard_normal((T, d)).astype(np.float32)
+    x = workloads.f32_to_bf16_bits(xf)
+    x[:, 1] = x[:, 0]
+    Wr = (rng.standard_normal((d, E)) * 0.05).astype(np.float32)
+    Wr[0] = (1024.0 * rng.uniform(0.5, 1.0, E) * rng.choice([-1.0, 1.0], E)).astype(np.float32)
+    Wr[1] = -Wr[0]
+    Wr[2:6] *= np.float32(2.0 ** -40)
+    Wr[6:10] = (rng.standard_normal((4, E)) * 1e-40).astype(np.float32)   # subnormal fp32
+    Wr[:, 17] = Wr[:, 3]
+    Wr[10, 17] = Wr[10, 3] + np.float32(2.0 ** -20)
+    b = rng.uniform(-0.1, 0.1, E).astype(np.float32)
+    b[17] = b[3]
+    nfb = _check_against_oracle(x, Wr, b, k)
+    assert nfb > T // 2, nfb
+
+
 def test_route_bias_only():
     """W_r = 0: every key is 1/2 + b; ties in b resolve to the lower id; gates 1/k."""
     T, d, E, k = 40, 32, 12, 4
