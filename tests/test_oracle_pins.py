@@ -208,11 +208,12 @@ def _gelu_t(u):
     return torch.nn.functional.gelu(u, approximate="none")
 
 
-def test_single_expert_is_dense_mlp():
+@pytest.mark.parametrize("h", [40, 13])
+def test_single_expert_is_dense_mlp(h):
     """E = 1, k = 1: the layer is GELU(x W1) W2 (gate 1); d != h so a transposed
-    W1 or W2 index cannot pass."""
+    W1 or W2 index cannot pass (h = 13: a width that is not a multiple of 8)."""
     rng = _rng(11)
-    T, d, h = 9, 24, 40
+    T, d = 9, 24
     x = _bf16(rng.standard_normal((T, d)))
     W1 = _bf16(rng.standard_normal((1, d, h)) / np.sqrt(d))
     W2 = _bf16(rng.standard_normal((1, h, d)) / np.sqrt(h))
@@ -401,11 +402,12 @@ def test_bias_update_zscore_invariants():
 
 # ------------------------------------------------------ SwiGLU experts (App. B)
 
-def test_single_swiglu_expert_is_dense_swiglu_mlp():
+@pytest.mark.parametrize("h", [40, 13])
+def test_single_swiglu_expert_is_dense_swiglu_mlp(h):
     """E = 1, k = 1 with W3: the layer is (SiLU(x W1) * (x W3)) W2, checked against torch
     fp64 (torch.nn.functional.silu); swapping W1 and W3 changes the result."""
     rng = _rng(61)
-    T, d, h = 9, 24, 40
+    T, d = 9, 24
     x = _bf16(rng.standard_normal((T, d)))
     W1 = _bf16(rng.standard_normal((1, d, h)) / np.sqrt(d))
     W3 = _bf16(rng.standard_normal((1, d, h)) / np.sqrt(d))
@@ -450,3 +452,31 @@ def test_swiglu_shared_expert_alone():
     xt = _t64(x)
     want = 0.75 * ((torch.nn.functional.silu(xt @ _t64(Ws1)) * (xt @ _t64(Ws3))) @ _t64(Ws2))
     np.testing.assert_allclose(y, want.numpy(), rtol=1e-12, atol=1e-13)
+
+
+@pytest.mark.parametrize("act", ["gelu", "swiglu"])
+def test_shared_expert_splits_into_chunks(act):
+    """The activation acts on each hidden unit separately, so a shared expert of width
+    2h equals the sum of two shared experts of width h holding its first and second h
+    hidden units (columns of Ws1 and Ws3, rows of Ws2): Eq. 6 with m = 2 shared experts
+    at the routed width, the form in which the kernels run it.  Checked on the oracle
+    with the routed experts zeroed."""
+    rng = _rng(71)
+    T, d, E, k, h = 11, 16, 4, 2, 12
+    x, Wr, b, W1, W2, Ws1, Ws2 = _layer(rng, T, d, E, k, h, 2 * h)
+    W1[:] = 0
+    W2[:] = 0
+    W3 = Ws3 = None
+    if act == "swiglu":
+        W3 = _bf16(rng.standard_normal((E, d, h)) / np.sqrt(d))
+        Ws3 = _bf16(rng.standard_normal((d, 2 * h)) / np.sqrt(d))
+    y, *_ = oracle.forward_tokens(x, Wr, b, W1, W2, k, Ws1, Ws2, 0.5, W3=W3, Ws3=Ws3)
+    parts = []
+    for c in range(2):
+        cols = slice(c * h, (c + 1) * h)
+        yc, *_ = oracle.forward_tokens(x, Wr, b, W1, W2, k, np.ascontiguousarray(Ws1[:, cols]),
+                                       np.ascontiguousarray(Ws2[cols]), 0.5, W3=W3,
+                                       Ws3=None if Ws3 is None else np.ascontiguousarray(Ws3[:, cols]))
+        parts.append(yc)
+    np.testing.assert_allclose(y, parts[0] + parts[1], rtol=1e-12, atol=1e-13)
+    assert np.abs(parts[0]).max() > 1e-3 and np.abs(parts[1]).max() > 1e-3
