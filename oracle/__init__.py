@@ -1,4 +1,5 @@
-"""Plain fp64 CPU oracle of the MoE-ViE fine-grained MoE FFN layer forward.
+"""Plain fp64 CPU oracle of the MoE-ViE fine-grained MoE FFN layer (forward, bias
+update and backward).
 
 TEST INFRASTRUCTURE, NOT PRODUCT CODE.  Only the tests, ``__graft_entry__.smoke()``
 and the CPU-baseline leg of ``bench.py`` may import this package.  It shares no
@@ -20,6 +21,10 @@ computes, with the paper's equations:
 * :func:`combine`       Eq. (6) gate-weighted sum plus ``lambda`` times the shared
   expert
 * :func:`forward_tokens` the whole layer, token by token (Eqs. 1, 7, 4-6)
+* :func:`update_bias`   the loss-free bias update, z-score (Eq. 9) or sign (Eq. 8)
+* :func:`backward`      the training path: gradients of ``sum dy . y`` with the
+  selection held fixed (through the gates of Eqs. 4-5 into ``W_r`` and ``x``, and
+  through the experts), the bias getting none
 """
 from __future__ import annotations
 
@@ -71,9 +76,11 @@ def _load():
         lib.oracle_forward_tokens.argtypes = [P, P, P, P, P, P, P, P, P, ctypes.c_double,
                                               I64, I64, I64, I64, I64, I64, P, I64,
                                               P, P, P, P, P, ctypes.c_int]
+        lib.oracle_backward.argtypes = [P, P, P, P, P, P, P, P, P, ctypes.c_double,
+                                        I64, I64, I64, I64, I64, I64, P, P, P, P, P, P, P, P, P]
         for fn in (lib.oracle_logits, lib.oracle_select, lib.oracle_permute,
                    lib.oracle_expert_rows, lib.oracle_combine, lib.oracle_forward_tokens,
-                   lib.oracle_update_bias):
+                   lib.oracle_update_bias, lib.oracle_backward):
             fn.restype = ctypes.c_int
         _lib = lib
         return lib
@@ -219,3 +226,43 @@ def forward_tokens(x_bf16, Wr, b, W1, W2, k, Ws1=None, Ws2=None, lam=1.0, tokens
     if want_shared:
         return y, idx, gate, margin, shared
     return y, idx, gate, margin
+
+
+def backward(x_bf16, Wr, b, W1, W2, k, dy, Ws1=None, Ws2=None, lam=1.0, W3=None, Ws3=None):
+    """Gradients of ``L = sum_t dy[t] . y[t]`` (``dy`` fp64 [T, d]) for the layer of
+    :func:`forward_tokens`, with the top-k selection held fixed and no gradient for
+    the bias (it only selects).  Returns a dict of fp64 arrays: ``dx`` [T, d], ``dWr``
+    [d, E], ``dW1`` [E, d, h], ``dW2`` [E, h, d], and ``dW3``, ``dWs1``, ``dWs2``,
+    ``dWs3`` when those weights are given.  One thread, tokens in ascending order."""
+    x = _c(x_bf16, np.uint16)
+    Wr = _c(Wr, np.float32)
+    b = _c(b, np.float32)
+    W1 = _c(W1, np.uint16)
+    W2 = _c(W2, np.uint16)
+    W3 = None if W3 is None else _c(W3, np.uint16)
+    dy = _c(dy, np.float64)
+    T, d = x.shape
+    E, _, h = W1.shape
+    assert dy.shape == (T, d) and (W3 is None or W3.shape == W1.shape)
+    hs = 0
+    if Ws1 is not None:
+        Ws1 = _c(Ws1, np.uint16)
+        Ws2 = _c(Ws2, np.uint16)
+        hs = Ws1.shape[1]
+        Ws3 = None if Ws3 is None else _c(Ws3, np.uint16)
+        assert Ws3 is None or Ws3.shape == Ws1.shape
+    out = {"dx": np.empty((T, d)), "dWr": np.empty((d, E)), "dW1": np.empty((E, d, h)),
+           "dW2": np.empty((E, h, d))}
+    if W3 is not None:
+        out["dW3"] = np.empty((E, d, h))
+    if hs > 0:
+        out["dWs1"] = np.empty((d, hs))
+        out["dWs2"] = np.empty((hs, d))
+        if Ws3 is not None:
+            out["dWs3"] = np.empty((d, hs))
+    _check(_load().oracle_backward(_ptr(x), _ptr(Wr), _ptr(b), _ptr(W1), _ptr(W2), _ptr(W3),
+                                   _ptr(Ws1), _ptr(Ws2), _ptr(Ws3), float(lam), T, d, E, k, h, hs,
+                                   _ptr(dy), _ptr(out["dx"]), _ptr(out["dWr"]), _ptr(out["dW1"]),
+                                   _ptr(out["dW2"]), _ptr(out.get("dW3")), _ptr(out.get("dWs1")),
+                                   _ptr(out.get("dWs2")), _ptr(out.get("dWs3"))), "backward")
+    return out

@@ -1,6 +1,6 @@
 /*
  * moevie_oracle.c -- plain, slow, fp64 CPU oracle of the MoE-ViE fine-grained
- * mixture-of-experts FFN layer forward pass.
+ * mixture-of-experts FFN layer: forward pass, bias update and backward pass.
  *
  * TEST INFRASTRUCTURE, NOT PRODUCT CODE.  This file exists only so that the
  * CUDA library can be checked against an independent statement of the method.
@@ -446,4 +446,167 @@ int oracle_update_bias(const int32_t* counts, int64_t E, float alpha, int rule, 
         b[e] = (float)((double)b[e] - (double)alpha * step);
     }
     return ORACLE_OK;
+}
+
+/* ------------------------------------------- backward of the layer (training) */
+
+/* The training path of the layer (App. B: grouped GEMMs for training, the activation
+ * a separate operator between the up- and down-projections): the gradients of
+ * L = sum_t dy[t] . y[t] with respect to the inputs and weights, given dy[T, d].
+ *
+ * Readings (listed in the design notes):
+ *   - the top-k selection is held fixed: it is piecewise constant in s, so it has no
+ *     gradient; the gradient reaches W_r and x through the gates of Eqs. 4-5 only;
+ *   - the bias b gets no gradient (it only selects; Sec. 2.2.2 updates it from the
+ *     expert loads, Eqs. 8-9, not by back-propagation).
+ *
+ * Per token t with selected experts e_j, sigma_j = Sigmoid(s_{e_j}), S = sum_j sigma_j,
+ * gates g_j = sigma_j / S, expert outputs o_j = E_{e_j}(x_t):
+ *   dg_j      = dy . o_j
+ *   dsigma_j  = (dg_j - sum_l g_l dg_l) / S            (derivative of sigma_j / S)
+ *   ds_{e_j}  = dsigma_j sigma_j (1 - sigma_j)           (Sigmoid' = sigma (1 - sigma))
+ *   dW_r[:, e_j] += x_t ds_{e_j},   dx_t += ds_{e_j} W_r[:, e_j]
+ * and through each selected expert with output weight g_j (and the shared expert
+ * with weight lambda), with a the hidden activation, u = x W1[e] (and v = x W3[e]):
+ *   dW2[e] += a^T (g dy),  da = (g dy) W2[e]^T,
+ *   GELU:   du = da GELU'(u),  GELU'(u) = Phi(u) + u phi(u)
+ *   SwiGLU: du = da v SiLU'(u), dv = da SiLU(u),  SiLU'(u) = sigma(u) (1 + u (1 - sigma(u)))
+ *   dW1[e] += x^T du,  dW3[e] += x^T dv,  dx += du W1[e]^T + dv W3[e]^T.
+ * Tokens are taken one after another in ascending t (one thread: the weight
+ * gradients are sums over tokens, accumulated in that order).  All outputs are
+ * double and are overwritten: dx [T, d], dWr [d, E], dW1 [E, d, h], dW2 [E, h, d],
+ * dW3 [E, d, h] (with W3), dWs1 [d, hs], dWs2 [hs, d], dWs3 [d, hs] (with Ws3). */
+
+static double gelu_grad(double u) {
+    const double Phi = 0.5 * (1.0 + erf(u / sqrt(2.0)));
+    const double phi = exp(-0.5 * u * u) / sqrt(2.0 * 3.14159265358979323846);
+    return Phi + u * phi;
+}
+
+/* One expert (or the shared expert) on one token: forward to its output o, then
+ * the gradient pieces for the output weight w (g_j or lambda).  W3 NULL: GELU. */
+static void expert_backward(const uint16_t* xt, const uint16_t* W1e, const uint16_t* W3e,
+                            const uint16_t* W2e, int64_t d, int64_t h, double w, const double* dyt,
+                            double* dW1e, double* dW3e, double* dW2e, double* dxt, double* o,
+                            double* u, double* v, double* a, double* da) {
+    for (int64_t n = 0; n < h; ++n) { u[n] = 0.0; v[n] = 0.0; }
+    for (int64_t i = 0; i < d; ++i) {
+        const double xi = bf16_to_double(xt[i]);
+        for (int64_t n = 0; n < h; ++n) {
+            u[n] += xi * bf16_to_double(W1e[i * h + n]);
+            if (W3e) v[n] += xi * bf16_to_double(W3e[i * h + n]);
+        }
+    }
+    for (int64_t n = 0; n < h; ++n) a[n] = W3e ? silu(u[n]) * v[n] : gelu(u[n]);
+    expert_down(a, W2e, h, d, o);
+    /* dW2[e] += a^T (w dy);  da = (w dy) W2[e]^T */
+    for (int64_t n = 0; n < h; ++n) {
+        double acc = 0.0;
+        for (int64_t c = 0; c < d; ++c) {
+            const double dO = w * dyt[c];
+            dW2e[n * d + c] += a[n] * dO;
+            acc += dO * bf16_to_double(W2e[n * d + c]);
+        }
+        da[n] = acc;
+    }
+    /* du (in u), dv (in v) */
+    for (int64_t n = 0; n < h; ++n) {
+        if (W3e) {
+            const double sg = sigmoid(u[n]);
+            const double du = da[n] * v[n] * sg * (1.0 + u[n] * (1.0 - sg));
+            const double dv = da[n] * u[n] * sg;   /* SiLU(u) = u sigma(u) */
+            u[n] = du;
+            v[n] = dv;
+        } else {
+            u[n] = da[n] * gelu_grad(u[n]);
+        }
+    }
+    for (int64_t i = 0; i < d; ++i) {
+        const double xi = bf16_to_double(xt[i]);
+        double acc = 0.0;
+        for (int64_t n = 0; n < h; ++n) {
+            dW1e[i * h + n] += xi * u[n];
+            acc += u[n] * bf16_to_double(W1e[i * h + n]);
+            if (W3e) {
+                dW3e[i * h + n] += xi * v[n];
+                acc += v[n] * bf16_to_double(W3e[i * h + n]);
+            }
+        }
+        dxt[i] += acc;
+    }
+}
+
+int oracle_backward(const uint16_t* x, const float* Wr, const float* b,
+                    const uint16_t* W1, const uint16_t* W2, const uint16_t* W3,
+                    const uint16_t* Ws1, const uint16_t* Ws2, const uint16_t* Ws3, double lambda,
+                    int64_t T, int64_t d, int64_t E, int64_t k, int64_t h, int64_t hs,
+                    const double* dy, double* dx, double* dWr, double* dW1, double* dW2,
+                    double* dW3, double* dWs1, double* dWs2, double* dWs3) {
+    if (T < 0 || d <= 0 || E <= 0 || k < 1 || k > E || h <= 0 || hs < 0) return ORACLE_ERR_ARG;
+    if (!x || !Wr || !b || !W1 || !W2 || !dy || !dx || !dWr || !dW1 || !dW2) return ORACLE_ERR_ARG;
+    if (W3 && !dW3) return ORACLE_ERR_ARG;
+    if (hs > 0 && (!Ws1 || !Ws2 || !dWs1 || !dWs2 || (Ws3 && !dWs3))) return ORACLE_ERR_ARG;
+    memset(dx, 0, (size_t)(T * d) * sizeof(double));
+    memset(dWr, 0, (size_t)(d * E) * sizeof(double));
+    memset(dW1, 0, (size_t)(E * d * h) * sizeof(double));
+    memset(dW2, 0, (size_t)(E * h * d) * sizeof(double));
+    if (W3) memset(dW3, 0, (size_t)(E * d * h) * sizeof(double));
+    if (hs > 0) {
+        memset(dWs1, 0, (size_t)(d * hs) * sizeof(double));
+        memset(dWs2, 0, (size_t)(hs * d) * sizeof(double));
+        if (Ws3) memset(dWs3, 0, (size_t)(d * hs) * sizeof(double));
+    }
+    const int64_t hmax = h > hs ? h : hs;
+    double* s = (double*)malloc((size_t)E * sizeof(double));
+    double* key = (double*)malloc((size_t)E * sizeof(double));
+    unsigned char* taken = (unsigned char*)malloc((size_t)E);
+    int32_t* sel = (int32_t*)malloc((size_t)k * sizeof(int32_t));
+    double* g = (double*)malloc((size_t)k * sizeof(double));
+    double* dg = (double*)malloc((size_t)k * sizeof(double));
+    double* o = (double*)malloc((size_t)d * sizeof(double));
+    double* u = (double*)malloc((size_t)hmax * sizeof(double));
+    double* v = (double*)malloc((size_t)hmax * sizeof(double));
+    double* a = (double*)malloc((size_t)hmax * sizeof(double));
+    double* da = (double*)malloc((size_t)hmax * sizeof(double));
+    int err = ORACLE_OK;
+    if (!s || !key || !taken || !sel || !g || !dg || !o || !u || !v || !a || !da) {
+        err = ORACLE_ERR_NOMEM;
+        goto done;
+    }
+    for (int64_t t = 0; t < T; ++t) {
+        const uint16_t* xt = x + t * d;
+        const double* dyt = dy + t * d;
+        double* dxt = dx + t * d;
+        logits_row(xt, Wr, d, E, s);                                                        /* Eq. 1 */
+        double m;
+        select_one(s, b, E, k, sel, g, &m, taken, key);                                    /* Eqs. 7, 4, 5 */
+        for (int64_t j = 0; j < k; ++j) {                                                   /* routed experts */
+            const int64_t e = sel[j];
+            expert_backward(xt, W1 + e * d * h, W3 ? W3 + e * d * h : NULL, W2 + e * h * d, d, h, g[j],
+                            dyt, dW1 + e * d * h, W3 ? dW3 + e * d * h : NULL, dW2 + e * h * d, dxt,
+                            o, u, v, a, da);
+            double acc = 0.0;
+            for (int64_t c = 0; c < d; ++c) acc += dyt[c] * o[c];
+            dg[j] = acc;                                                                    /* dy . o_j */
+        }
+        double S = 0.0, gdg = 0.0;                                                          /* Eqs. 4-5 */
+        for (int64_t j = 0; j < k; ++j) S += sigmoid(s[sel[j]]);
+        for (int64_t j = 0; j < k; ++j) gdg += g[j] * dg[j];
+        for (int64_t j = 0; j < k; ++j) {
+            const int64_t e = sel[j];
+            const double sg = sigmoid(s[e]);
+            const double ds = (dg[j] - gdg) / S * sg * (1.0 - sg);
+            for (int64_t i = 0; i < d; ++i) {
+                dWr[i * E + e] += bf16_to_double(xt[i]) * ds;
+                dxt[i] += ds * (double)Wr[i * E + e];
+            }
+        }
+        if (hs > 0)                                                                         /* Eq. 6, shared */
+            expert_backward(xt, Ws1, Ws3, Ws2, d, hs, lambda, dyt, dWs1, Ws3 ? dWs3 : NULL, dWs2, dxt,
+                            o, u, v, a, da);
+    }
+done:
+    free(s); free(key); free(taken); free(sel); free(g); free(dg); free(o); free(u); free(v);
+    free(a); free(da);
+    return err;
 }

@@ -480,3 +480,137 @@ def test_shared_expert_splits_into_chunks(act):
         parts.append(yc)
     np.testing.assert_allclose(y, parts[0] + parts[1], rtol=1e-12, atol=1e-13)
     assert np.abs(parts[0]).max() > 1e-3 and np.abs(parts[1]).max() > 1e-3
+
+
+# ------------------------------------------ backward (training path, App. B)
+
+def _torch_layer_from_oracle_routing(x, Wr, W1, W2, idx, lam, Ws1=None, Ws2=None, W3=None, Ws3=None):
+    """The layer in torch fp64 autograd with the selection idx held fixed: gates are
+    sigmoid(s) renormalised over the selected experts (Eqs. 4-5), experts GELU or
+    SwiGLU, plus lam times the shared expert (Eq. 6).  Inputs are torch leaves."""
+    s = x @ Wr
+    it = torch.from_numpy(idx.astype(np.int64))
+    sg = torch.sigmoid(torch.gather(s, 1, it))
+    g = sg / sg.sum(1, keepdim=True)
+
+    def ffn(xx, A, B, C):   # A, B: [T, d, h] per token (or [d, h]); C: [T, h, d] (or [h, d])
+        if A.dim() == 2:
+            u = xx @ A
+            a = torch.nn.functional.silu(u) * (xx @ B) if B is not None else _gelu_t(u)
+            return a @ C
+        u = torch.einsum("td,tdh->th", xx, A)
+        a = (torch.nn.functional.silu(u) * torch.einsum("td,tdh->th", xx, B) if B is not None
+             else _gelu_t(u))
+        return torch.einsum("th,thd->td", a, C)
+
+    y = 0.0
+    for j in range(idx.shape[1]):
+        e = it[:, j]
+        y = y + g[:, j:j + 1] * ffn(x, W1[e], None if W3 is None else W3[e], W2[e])
+    if Ws1 is not None:
+        y = y + lam * ffn(x, Ws1, Ws3, Ws2)
+    return y
+
+
+def _backward_case(seed, T, d, E, k, h, hs=0, swiglu=False, lam=0.5):
+    rng = _rng(seed)
+    x, Wr, b, W1, W2, Ws1, Ws2 = _layer(rng, T, d, E, k, h, hs)
+    W3 = _bf16(rng.standard_normal((E, d, h)) / np.sqrt(d)) if swiglu else None
+    Ws3 = _bf16(rng.standard_normal((d, hs)) / np.sqrt(d)) if (swiglu and hs) else None
+    dy = rng.standard_normal((T, d))
+    return x, Wr, b, W1, W2, W3, Ws1, Ws2, Ws3, dy, lam
+
+
+@pytest.mark.parametrize("T,d,E,k,h,hs,swiglu", [
+    (7, 16, 1, 1, 12, 0, False), (9, 24, 6, 2, 13, 0, False), (8, 16, 5, 3, 8, 20, False),
+    (9, 24, 6, 2, 13, 0, True), (8, 16, 5, 3, 8, 20, True), (6, 8, 4, 4, 6, 6, True),
+])
+def test_backward_matches_autograd(T, d, E, k, h, hs, swiglu):
+    """Every gradient of the oracle's backward against torch fp64 autograd of the layer
+    written with torch primitives, the selection held at the oracle's."""
+    x, Wr, b, W1, W2, W3, Ws1, Ws2, Ws3, dy, lam = _backward_case(T + E + h, T, d, E, k, h, hs, swiglu)
+    got = oracle.backward(x, Wr, b, W1, W2, k, dy, Ws1 if hs else None, Ws2 if hs else None, lam,
+                          W3=W3, Ws3=Ws3)
+    idx, _, _ = oracle.route(x, Wr, b, k)
+    leaves = {"dx": _t64(x), "dWr": torch.from_numpy(Wr.astype(np.float64)), "dW1": _t64(W1),
+              "dW2": _t64(W2)}
+    if swiglu:
+        leaves["dW3"] = _t64(W3)
+    if hs:
+        leaves["dWs1"], leaves["dWs2"] = _t64(Ws1), _t64(Ws2)
+        if swiglu:
+            leaves["dWs3"] = _t64(Ws3)
+    for v in leaves.values():
+        v.requires_grad_(True)
+    y = _torch_layer_from_oracle_routing(leaves["dx"], leaves["dWr"], leaves["dW1"], leaves["dW2"], idx,
+                                         lam, leaves.get("dWs1"), leaves.get("dWs2"), leaves.get("dW3"),
+                                         leaves.get("dWs3"))
+    (torch.from_numpy(dy) * y).sum().backward()
+    assert set(got) == set(leaves)
+    for name, leaf in leaves.items():
+        want = leaf.grad.numpy()
+        scale = max(np.abs(want).max(), 1e-300)
+        np.testing.assert_allclose(got[name], want, rtol=0, atol=1e-12 * scale, err_msg=name)
+        if not (name == "dWr" and E == 1):
+            assert np.abs(want).max() > 1e-6, name
+
+
+@pytest.mark.parametrize("swiglu", [False, True])
+def test_backward_linear_weight_identities(swiglu):
+    """y is linear in W2 (and, with SwiGLU, in W3) and the shared term in Ws2 (Ws3), so
+    <dW2, W2> = <dy, y_routed> and <dWs2, Ws2> = lam <dy, S(x)> (the same for W3, Ws3):
+    Euler's identity, checked against the pinned forward oracle."""
+    T, d, E, k, h, hs = 10, 16, 6, 2, 12, 24
+    x, Wr, b, W1, W2, W3, Ws1, Ws2, Ws3, dy, lam = _backward_case(81, T, d, E, k, h, hs, swiglu, 0.75)
+    y, _, _, _, S = oracle.forward_tokens(x, Wr, b, W1, W2, k, Ws1, Ws2, lam, want_shared=True,
+                                          W3=W3, Ws3=Ws3)
+    gr = oracle.backward(x, Wr, b, W1, W2, k, dy, Ws1, Ws2, lam, W3=W3, Ws3=Ws3)
+    routed = float(np.sum(dy * (y - lam * S)))
+    shared = float(lam * np.sum(dy * S))
+    f = lambda a: a.astype(np.float64)  # noqa: E731
+    w2 = lambda a: workloads.bf16_bits_to_f32(a).astype(np.float64)  # noqa: E731
+    assert abs(np.sum(gr["dW2"] * w2(W2)) - routed) <= 1e-11 * abs(routed) + 1e-12
+    assert abs(np.sum(gr["dWs2"] * w2(Ws2)) - shared) <= 1e-11 * abs(shared) + 1e-12
+    if swiglu:
+        assert abs(np.sum(gr["dW3"] * w2(W3)) - routed) <= 1e-11 * abs(routed) + 1e-12
+        assert abs(np.sum(gr["dWs3"] * w2(Ws3)) - shared) <= 1e-11 * abs(shared) + 1e-12
+    assert abs(routed) > 1e-3 and abs(shared) > 1e-3 and f(dy).std() > 0
+
+
+def test_backward_router_gets_no_gradient_when_gates_cannot_matter():
+    """Identical experts (every expert output equal) make sum_j g_j o = o whatever the
+    gates, so W_r gets no gradient; with one expert (E = k = 1) the gate is always 1."""
+    T, d, E, k, h = 8, 16, 5, 3, 8
+    x, Wr, b, W1, W2, W3, Ws1, Ws2, Ws3, dy, lam = _backward_case(82, T, d, E, k, h)
+    W1[:] = W1[0]
+    W2[:] = W2[0]
+    gr = oracle.backward(x, Wr, b, W1, W2, k, dy)
+    assert np.abs(gr["dWr"]).max() <= 1e-13 * np.abs(gr["dW1"]).max()
+    x1, Wr1, b1, W11, W21, *_ , dy1, _ = _backward_case(83, T, d, 1, 1, h)
+    gr1 = oracle.backward(x1, Wr1, b1, W11, W21, 1, dy1)
+    assert np.all(gr1["dWr"] == 0.0)
+
+
+@pytest.mark.parametrize("swiglu", [False, True])
+def test_backward_router_finite_differences(swiglu):
+    """Central differences of the pinned forward oracle along a direction V of W_r,
+    against <dWr, V>.  W_r and V are dyadic, so W_r +- V are exact fp32 inputs; only
+    tokens whose selection margin is far above the key change carry dy, so no
+    selection changes between the two evaluations."""
+    rng = _rng(84)
+    T, d, E, k, h = 24, 32, 8, 3, 12
+    x, _, b, W1, W2, _, _ = _layer(rng, T, d, E, k, h)
+    W3 = _bf16(rng.standard_normal((E, d, h)) / np.sqrt(d)) if swiglu else None
+    Wr = (np.round(rng.standard_normal((d, E)) * 0.3 * 2 ** 12) / 2 ** 12).astype(np.float32)
+    V = (rng.integers(-8, 9, (d, E)) * 2.0 ** -20).astype(np.float32)
+    assert np.array_equal((Wr + V) - V, Wr) and np.array_equal((Wr - V) + V, Wr)
+    _, _, margin = oracle.route(x, Wr, b, k)
+    dy = rng.standard_normal((T, d))
+    dy[margin < 1e-2] = 0.0
+    assert (margin >= 1e-2).sum() >= T // 2
+    L = lambda W: float(np.sum(dy * oracle.forward_tokens(x, W, b, W1, W2, k, W3=W3)[0]))  # noqa: E731
+    fd = (L(Wr + V) - L(Wr - V)) / 2.0
+    gr = oracle.backward(x, Wr, b, W1, W2, k, dy, W3=W3)
+    an = float(np.sum(gr["dWr"] * V.astype(np.float64)))
+    assert abs(an) > 1e-9
+    assert abs(fd - an) <= 1e-7 * abs(an), (fd, an)
