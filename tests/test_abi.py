@@ -136,3 +136,22 @@ def test_bias_update_validates_before_launch(lib):
     assert f(p, 8, 0.1, 2, p, p, 4096, None) == 1        # unknown rule
     assert f(None, 8, 0.1, 0, p, p, 4096, None) == 1     # null counts
     assert f(p, 8, 0.1, 0, p, p, 128, None) == 3         # workspace too small
+
+
+def test_row_padding_helpers():
+    """W1, W3, Ws1, Ws3 and the hidden activations have rows h rounded up to 8 elements
+    apart: moevie_pad_rows lays a tensor out that way (a view of [..., h]) and returns a
+    tensor that already is one unchanged; any other strides are rejected."""
+    import torch
+    from paper_2608_17402_gb300 import moevie
+    assert [moevie.row_ld(h) for h in (1, 7, 8, 13, 512, 684, 854)] == [8, 8, 8, 16, 512, 688, 856]
+    for shape in [(3, 5, 684), (5, 854), (2, 4, 13), (1, 3, 1)]:
+        w = torch.randn(*shape)
+        p = moevie.moevie_pad_rows(w)
+        assert p.shape == w.shape and torch.equal(p, w) and moevie._rows_ok(p)
+        assert p.stride()[-2] == moevie.row_ld(shape[-1])
+        assert not moevie._rows_ok(w.contiguous())   # dense rows of a width that is not a multiple of 8
+    w = torch.randn(4, 6, 512)
+    assert moevie.moevie_pad_rows(w) is w
+    with pytest.raises(ValueError):   # a host tensor is never accepted as device weights
+        moevie._want_rows(w, torch.float32, "W1")
