@@ -155,3 +155,18 @@ def test_row_padding_helpers():
     assert moevie.moevie_pad_rows(w) is w
     with pytest.raises(ValueError):   # a host tensor is never accepted as device weights
         moevie._want_rows(w, torch.float32, "W1")
+
+
+@pytest.mark.parametrize("d,E,k,h,hs", [(1024, 64, 8, 512, 1024), (768, 31, 3, 512, 512),
+                                        (1024, 31, 3, 684, 684), (1280, 31, 7, 854, 854),
+                                        (1664, 256, 8, 416, 0), (64, 4, 2, 13, 5), (96, 1, 1, 1, 0)])
+def test_workspace_size_monotone_and_covers_the_big_regions(lib, d, E, k, h, hs):
+    """For every T the workspace is monotone in T and at least holds the fp32 y
+    accumulator [T, d] and the hidden activations [T k, h rounded up to 8] bf16."""
+    hp = (h + 7) // 8 * 8
+    prev = 0
+    for T in list(range(0, 600, 37)) + [4095, 4096, 4097, 8192, 16383, 16384, 16385, 65536]:
+        rc, size = _ws_size(lib, T, d, E, k, h, hs)
+        assert rc == 0 and size >= prev, (T, size, prev)
+        assert size >= 4 * T * d + 2 * T * k * hp
+        prev = size
