@@ -161,16 +161,19 @@ moevie_status check_sizes(int64_t T, int64_t d, int64_t E, int64_t k, int64_t h,
     return MOEVIE_OK;
 }
 
+// SM count of the current device (GB300: 152), cached per device; safe to call from
+// several host threads at once.
 int num_sms() {
-    static int cache[64] = {};
+    static std::atomic<int> cache[64];
     int dev = 0;
-    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 148;
-    if (!cache[dev]) {
-        int n = 0;
-        cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev);
-        cache[dev] = n > 0 ? n : 148;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 152;
+    int n = cache[dev].load(std::memory_order_relaxed);
+    if (n == 0) {
+        if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n <= 0)
+            n = 152;
+        cache[dev].store(n, std::memory_order_relaxed);
     }
-    return cache[dev];
+    return n;
 }
 
 inline moevie_status cuda_status(cudaError_t e) { return e == cudaSuccess ? MOEVIE_OK : MOEVIE_ERR_CUDA; }
