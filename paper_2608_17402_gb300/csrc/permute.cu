@@ -16,6 +16,7 @@
 // Inside one expert's segment, rows keep ascending slot order t*k + j.
 #include <cooperative_groups.h>
 
+#include <atomic>
 #include <mutex>
 
 #include "internal.h"
@@ -452,28 +453,34 @@ cudaError_t launch_permute(const int32_t* idx, int64_t n_slots, int k, int E, in
     int64_t T = sh ? sh->T : 0;
     float lambda = sh ? sh->lambda : 0.f;
     const size_t smem = (size_t)(chunk + PW * E) * 4;
-    static bool attr_set[64] = {};
-    static int coop_ctas[64] = {};   // co-resident CTAs of perm_fused_kernel (0: no cooperative launch)
+    // per-device set-up on the first call (kernel attributes, co-resident CTAs of
+    // perm_fused_kernel; 0: no cooperative launch), safe for concurrent first calls
+    static std::mutex setup_mu;
+    static std::atomic<bool> attr_set[64];
+    static std::atomic<int> coop_ctas[64];
     int dev = 0;
     cudaError_t err = cudaGetDevice(&dev);
     if (err != cudaSuccess) return err;
-    if (dev >= 0 && dev < 64 && !attr_set[dev]) {
-        const int max_smem = (int)((PERM_CHUNK_MAX + PW * 1024) * 4);
-        if ((err = cudaFuncSetAttribute(perm_scatter_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                        max_smem)) != cudaSuccess)
-            return err;
-        if ((err = cudaFuncSetAttribute(perm_fused_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                        max_smem)) != cudaSuccess)
-            return err;
-        int coop = 0, sms = 0, per_sm = 0;
-        cudaDeviceGetAttribute(&coop, cudaDevAttrCooperativeLaunch, dev);
-        cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-        if (coop && cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, perm_fused_kernel, PT,
-                                                                  (size_t)max_smem) == cudaSuccess)
-            coop_ctas[dev] = per_sm * sms;
-        attr_set[dev] = true;
+    if (dev >= 0 && dev < 64 && !attr_set[dev].load(std::memory_order_acquire)) {
+        std::lock_guard<std::mutex> lock(setup_mu);
+        if (!attr_set[dev].load(std::memory_order_relaxed)) {
+            const int max_smem = (int)((PERM_CHUNK_MAX + PW * 1024) * 4);
+            if ((err = cudaFuncSetAttribute(perm_scatter_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                            max_smem)) != cudaSuccess)
+                return err;
+            if ((err = cudaFuncSetAttribute(perm_fused_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                            max_smem)) != cudaSuccess)
+                return err;
+            int coop = 0, sms = 0, per_sm = 0;
+            cudaDeviceGetAttribute(&coop, cudaDevAttrCooperativeLaunch, dev);
+            cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+            if (coop && cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, perm_fused_kernel, PT,
+                                                                      (size_t)max_smem) == cudaSuccess)
+                coop_ctas[dev].store(per_sm * sms, std::memory_order_relaxed);
+            attr_set[dev].store(true, std::memory_order_release);
+        }
     }
-    if (dev >= 0 && dev < 64 && nchunks <= coop_ctas[dev]) {
+    if (dev >= 0 && dev < 64 && nchunks <= coop_ctas[dev].load(std::memory_order_relaxed)) {
         err = launch_pdl_coop(perm_fused_kernel, dim3(nchunks), dim3(PT), smem, s, idx, n_slots, k, E,
                               bm, chunk, gate_flat, hist, counts, offsets, tiles, n_tiles, perm, inv,
                               row_tok, row_gate, st, S, T, lambda);
@@ -505,15 +512,15 @@ cudaError_t launch_item_order(const int4* tiles, const int32_t* n_tiles, const i
     if (nb < 1 || nb > ITEM_MAX_BANDS || max_tiles > ITEM_MAX_TILES || gsz < 1)
         return cudaErrorInvalidValue;
     const size_t smem = (size_t)2 * max_tiles * sizeof(int32_t);
-    static bool attr_set[64] = {};
+    static std::atomic<bool> attr_set[64];
     int dev = 0;
     cudaGetDevice(&dev);
-    if (dev >= 0 && dev < 64 && !attr_set[dev]) {
-        cudaError_t err = cudaFuncSetAttribute(item_order_kernel,
+    if (dev >= 0 && dev < 64 && !attr_set[dev].load(std::memory_order_acquire)) {
+        cudaError_t err = cudaFuncSetAttribute(item_order_kernel,   // idempotent: no lock needed
                                                cudaFuncAttributeMaxDynamicSharedMemorySize,
                                                2 * ITEM_MAX_TILES * (int)sizeof(int32_t));
         if (err != cudaSuccess) return err;
-        attr_set[dev] = true;
+        attr_set[dev].store(true, std::memory_order_release);
     }
     const cudaError_t err = launch_pdl(item_order_kernel, dim3(1), dim3(1024), smem, s, tiles, n_tiles,
                                        row_tok, T, nb, n_ntiles, gsz, BN, max_tiles, items, n_items);
