@@ -282,9 +282,9 @@ __device__ __forceinline__ void warp_kth_values(const float (&v)[NPL], int E, in
 // than one unit.  The units of d terms sum in a 128-bit integer (|sum| < 2^120 for
 // d < 2^24), exactly and in any order; the logit is that sum times 2^(Q - 348), within
 // d 2^(Q - 348) + 2^-51 |s| of the exact value.  Q is the largest q of the candidate's
-// terms, whose P is at least 1, so d 2^(Q - 348) <= d 2^-64 sum|x_i w_i|: below the
-// d 2^-53 sum|x_i w_i| of an fp64 sum.  Everything but the final conversion runs on the
-// integer pipes.
+// terms (zeros counted with their exponent fields); when that term is not zero its P is
+// at least 1, so d 2^(Q - 348) <= d 2^-64 sum|x_i w_i|, below the d 2^-53 sum|x_i w_i|
+// of an fp64 sum.  Everything but the final conversion runs on the integer pipes.
 constexpr int FB_CB = 32;   // candidates per batch (one per lane of the finishing warp)
 
 __device__ __forceinline__ int bf16_exp_field(uint32_t hx) { return (int)((hx >> 7) & 0xffu); }
@@ -336,8 +336,8 @@ __device__ __forceinline__ double long_acc_value(unsigned __int128 u, int Q) {
 // Exact re-decision of uncertified tokens, one CTA (8 warps) per token.  Warp 0
 // bounds the keys and lists the candidates; then all 256 threads form the candidates'
 // logits in the long accumulator (threads over d, reading the transposed fp32 copy of
-// W_r), and warp 0
-// fills the remaining places from the exact keys and writes ids and gates.
+// W_r), and warp 0 fills the remaining places from the exact keys and writes ids and
+// gates.
 template <int NPL>
 __global__ void __launch_bounds__(256, 1) route_fallback_kernel(
     const __nv_bfloat16* __restrict__ x, const float* __restrict__ wrt, int dp,
