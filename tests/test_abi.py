@@ -98,6 +98,19 @@ def test_forward_rejects_bad_layer(lib):
                                 None, ctypes.c_void_p(fake), 1 << 30, None)
     assert rc == 2
 
+    def fwd(layer, ws_bytes=1 << 30):
+        return lib.moevie_moe_forward(ctypes.byref(layer), ctypes.c_void_p(fake), 4,
+                                      ctypes.c_void_p(fake), None, ctypes.c_void_p(fake), ws_bytes, None)
+    # every case below fails argument validation, before the workspace size check
+    # and before anything is enqueued
+    assert fwd(_Layer(16, 8, 2, 32, 32, fake, fake, fake, fake, fake, 0, 1.0)) == 1      # shared, no Ws2
+    assert fwd(_Layer(16, 8, 2, 32, 32, fake, fake, fake, fake, fake, fake, 1.0,
+                      fake, 0)) == 1                                                     # SwiGLU shared, no Ws3
+    assert fwd(_Layer(16, 8, 2, 32, 0, fake, fake, fake, fake, 0, 0, 1.0, fake + 8)) == 1   # misaligned W3
+    assert fwd(_Layer(16, 8, 2, 32, 0, fake, fake, fake + 4, fake, 0, 0, 1.0)) == 1          # misaligned W1
+    # a hidden width that is not a multiple of 8 is supported: only the workspace is short
+    assert fwd(_Layer(16, 8, 2, 13, 13, fake, fake, fake, fake, fake, fake, 1.0), 16) == 3
+
 
 def test_shared_groups_plan_and_monotone_workspace(lib):
     """moevie_shared_groups: the shared expert rides in the routed GEMMs as h_s / h
