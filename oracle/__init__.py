@@ -25,6 +25,8 @@ computes, with the paper's equations:
 * :func:`backward`      the training path: gradients of ``sum dy . y`` with the
   selection held fixed (through the gates of Eqs. 4-5 into ``W_r`` and ``x``, and
   through the experts), the bias getting none
+* :func:`backward_rows` its routed-expert part per expert-major row: the gradients
+  at the hidden pre-activations and ``dy . E_e(x)``
 """
 from __future__ import annotations
 
@@ -78,9 +80,11 @@ def _load():
                                               P, P, P, P, P, ctypes.c_int]
         lib.oracle_backward.argtypes = [P, P, P, P, P, P, P, P, P, ctypes.c_double,
                                         I64, I64, I64, I64, I64, I64, P, P, P, P, P, P, P, P, P]
+        lib.oracle_backward_rows.argtypes = [P, P, P, P, P, P, P, P, I64, I64, I64, I64, I64, P, I64,
+                                             P, P, P]
         for fn in (lib.oracle_logits, lib.oracle_select, lib.oracle_permute,
                    lib.oracle_expert_rows, lib.oracle_combine, lib.oracle_forward_tokens,
-                   lib.oracle_update_bias, lib.oracle_backward):
+                   lib.oracle_update_bias, lib.oracle_backward, lib.oracle_backward_rows):
             fn.restype = ctypes.c_int
         _lib = lib
         return lib
@@ -265,4 +269,31 @@ def backward(x_bf16, Wr, b, W1, W2, k, dy, Ws1=None, Ws2=None, lam=1.0, W3=None,
                                    _ptr(dy), _ptr(out["dx"]), _ptr(out["dWr"]), _ptr(out["dW1"]),
                                    _ptr(out["dW2"]), _ptr(out.get("dW3")), _ptr(out.get("dWs1")),
                                    _ptr(out.get("dWs2")), _ptr(out.get("dWs3"))), "backward")
+    return out
+
+
+def backward_rows(x_bf16, perm, offsets, gate_rows, W1, W2, k, dy, rows, W3=None):
+    """Per expert-major row r = rows[i] (token perm[r] // k, gate gate_rows[r]): the
+    gradients at the hidden pre-activations, ``du`` [n, h] (and ``dv`` [n, h] with SwiGLU
+    experts), and ``dg`` [n] = dy[t] . E_e(x_t), the un-gated expert output.  Returns a
+    dict of fp64 arrays."""
+    x = _c(x_bf16, np.uint16)
+    perm = _c(perm, np.int32)
+    offsets = _c(offsets, np.int32)
+    gate_rows = _c(gate_rows, np.float64)
+    W1 = _c(W1, np.uint16)
+    W2 = _c(W2, np.uint16)
+    W3 = None if W3 is None else _c(W3, np.uint16)
+    dy = _c(dy, np.float64)
+    rows = _c(rows, np.int32)
+    T, d = x.shape
+    E, _, h = W1.shape
+    n = rows.size
+    out = {"du": np.empty((n, h)), "dg": np.empty((n,))}
+    if W3 is not None:
+        out["dv"] = np.empty((n, h))
+    _check(_load().oracle_backward_rows(_ptr(x), _ptr(perm), _ptr(offsets), _ptr(gate_rows), _ptr(W1),
+                                        _ptr(W2), _ptr(W3), _ptr(dy), T, d, h, E, k, _ptr(rows), n,
+                                        _ptr(out["du"]), _ptr(out.get("dv")), _ptr(out["dg"])),
+           "backward_rows")
     return out

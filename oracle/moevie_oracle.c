@@ -610,3 +610,71 @@ done:
     free(a); free(da);
     return err;
 }
+
+/* Staged backward of the routed experts, row by row in expert-major order (the rows of
+ * Algorithm 1): for row r of expert e (the segment holding r), token t = perm[r] / k and
+ * its gate g = gate_rows[r] (the gate of slot perm[r]):
+ *   du[i, :] = (g dy[t] W2[e]^T) * GELU'(u)      (GELU experts), or for SwiGLU experts
+ *   du[i, :] = (g dy[t] W2[e]^T) * v * SiLU'(u),  dv[i, :] = (g dy[t] W2[e]^T) * SiLU(u)
+ *   dg[i]    = dy[t] . E_e(x_t)                    (the un-gated expert output)
+ * with u = x_t W1[e], v = x_t W3[e], for r = rows[i].  These are the intermediate
+ * gradients from which dW1 = sum x^T du, dW3 = sum x^T dv, dx and the gate gradients
+ * of oracle_backward are formed.  du, dv: double [nrows, h] (dv only with W3); dg:
+ * double [nrows]. */
+int oracle_backward_rows(const uint16_t* x, const int32_t* perm, const int32_t* offsets,
+                         const double* gate_rows, const uint16_t* W1, const uint16_t* W2,
+                         const uint16_t* W3, const double* dy, int64_t T, int64_t d, int64_t h,
+                         int64_t E, int64_t k, const int32_t* rows, int64_t nrows,
+                         double* du, double* dv, double* dg) {
+    if (T < 0 || d <= 0 || h <= 0 || E <= 0 || k < 1 || nrows < 0) return ORACLE_ERR_ARG;
+    if (nrows > 0 && (!x || !perm || !offsets || !gate_rows || !W1 || !W2 || !dy || !rows || !du ||
+                      !dg || (W3 && !dv)))
+        return ORACLE_ERR_ARG;
+    double* u = (double*)malloc((size_t)h * sizeof(double));
+    double* v = (double*)malloc((size_t)h * sizeof(double));
+    double* a = (double*)malloc((size_t)h * sizeof(double));
+    double* da = (double*)malloc((size_t)h * sizeof(double));
+    double* o = (double*)malloc((size_t)d * sizeof(double));
+    int err = ORACLE_OK;
+    if (!u || !v || !a || !da || !o) { err = ORACLE_ERR_NOMEM; goto done; }
+    for (int64_t i = 0; i < nrows; ++i) {
+        const int64_t r = rows[i];
+        const int64_t e = expert_of_row(offsets, E, r);
+        const int64_t t = (e < 0) ? -1 : perm[r] / k;
+        if (e < 0 || t < 0 || t >= T) { err = ORACLE_ERR_ARG; continue; }
+        const uint16_t* xt = x + t * d;
+        const uint16_t* W1e = W1 + e * d * h;
+        const uint16_t* W3e = W3 ? W3 + e * d * h : NULL;
+        const uint16_t* W2e = W2 + e * h * d;
+        for (int64_t n = 0; n < h; ++n) { u[n] = 0.0; v[n] = 0.0; }
+        for (int64_t c = 0; c < d; ++c) {
+            const double xc = bf16_to_double(xt[c]);
+            for (int64_t n = 0; n < h; ++n) {
+                u[n] += xc * bf16_to_double(W1e[c * h + n]);
+                if (W3e) v[n] += xc * bf16_to_double(W3e[c * h + n]);
+            }
+        }
+        for (int64_t n = 0; n < h; ++n) a[n] = W3e ? silu(u[n]) * v[n] : gelu(u[n]);
+        expert_down(a, W2e, h, d, o);
+        double acc = 0.0;
+        for (int64_t c = 0; c < d; ++c) acc += dy[t * d + c] * o[c];
+        dg[i] = acc;
+        for (int64_t n = 0; n < h; ++n) {
+            double s = 0.0;
+            for (int64_t c = 0; c < d; ++c) s += gate_rows[r] * dy[t * d + c] * bf16_to_double(W2e[n * d + c]);
+            da[n] = s;
+        }
+        for (int64_t n = 0; n < h; ++n) {
+            if (W3e) {
+                const double sg = sigmoid(u[n]);
+                du[i * h + n] = da[n] * v[n] * sg * (1.0 + u[n] * (1.0 - sg));
+                dv[i * h + n] = da[n] * u[n] * sg;
+            } else {
+                du[i * h + n] = da[n] * gelu_grad(u[n]);
+            }
+        }
+    }
+done:
+    free(u); free(v); free(a); free(da); free(o);
+    return err;
+}

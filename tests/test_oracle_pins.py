@@ -614,3 +614,32 @@ def test_backward_router_finite_differences(swiglu):
     an = float(np.sum(gr["dWr"] * V.astype(np.float64)))
     assert abs(an) > 1e-9
     assert abs(fd - an) <= 1e-7 * abs(an), (fd, an)
+
+
+@pytest.mark.parametrize("swiglu", [False, True])
+def test_backward_rows_reassemble_the_layer_gradients(swiglu):
+    """The staged per-row gradients put back together: sum over the rows of expert e of
+    x_t^T du_r is the whole backward's dW1[e] (dW3[e] from dv), and
+    sum_r g_r dg_r + lam sum_t dy_t . S(x_t) is sum_t dy_t . y_t of the forward oracle."""
+    T, d, E, k, h, hs = 12, 16, 6, 2, 10, 20
+    x, Wr, b, W1, W2, W3, Ws1, Ws2, Ws3, dy, lam = _backward_case(91, T, d, E, k, h, hs, swiglu, 0.5)
+    idx, gate, _ = oracle.route(x, Wr, b, k)
+    counts, offsets, perm, inv = oracle.permute(idx, E)
+    gate_rows = gate.reshape(-1)[perm]
+    st = oracle.backward_rows(x, perm, offsets, gate_rows, W1, W2, k, dy,
+                              np.arange(T * k, dtype=np.int32), W3=W3)
+    whole = oracle.backward(x, Wr, b, W1, W2, k, dy, Ws1, Ws2, lam, W3=W3, Ws3=Ws3)
+    xf = workloads.bf16_bits_to_f32(x).astype(np.float64)
+    tok = perm // k
+    for name, g in (("dW1", st["du"]),) + ((("dW3", st.get("dv")),) if swiglu else ()):
+        got = np.zeros((E, d, h))
+        for e in range(E):
+            r = slice(offsets[e], offsets[e + 1])
+            got[e] = xf[tok[r]].T @ g[r]
+        np.testing.assert_allclose(got, whole[name], rtol=0, atol=1e-12 * np.abs(whole[name]).max(),
+                                   err_msg=name)
+    y, _, _, _, S = oracle.forward_tokens(x, Wr, b, W1, W2, k, Ws1, Ws2, lam, want_shared=True,
+                                          W3=W3, Ws3=Ws3)
+    lhs = float(np.sum(gate_rows * st["dg"]) + lam * np.sum(dy * S))
+    rhs = float(np.sum(dy * y))
+    assert abs(lhs - rhs) <= 1e-12 * max(abs(rhs), 1.0)
