@@ -473,7 +473,9 @@ int oracle_update_bias(const int32_t* counts, int64_t E, float alpha, int rule, 
  *   SwiGLU: du = da v SiLU'(u), dv = da SiLU(u),  SiLU'(u) = sigma(u) (1 + u (1 - sigma(u)))
  *   dW1[e] += x^T du,  dW3[e] += x^T dv,  dx += du W1[e]^T + dv W3[e]^T.
  * Tokens are taken one after another in ascending t (one thread: the weight
- * gradients are sums over tokens, accumulated in that order).  All outputs are
+ * gradients are sums over tokens, accumulated in that order).  A token whose dy row
+ * is all zero adds exact zeros to every gradient and is skipped, so a sampled check
+ * (dy nonzero on a few tokens) costs only those tokens.  All outputs are
  * double and are overwritten: dx [T, d], dWr [d, E], dW1 [E, d, h], dW2 [E, h, d],
  * dW3 [E, d, h] (with W3), dWs1 [d, hs], dWs2 [hs, d], dWs3 [d, hs] (with Ws3). */
 
@@ -577,6 +579,9 @@ int oracle_backward(const uint16_t* x, const float* Wr, const float* b,
         const uint16_t* xt = x + t * d;
         const double* dyt = dy + t * d;
         double* dxt = dx + t * d;
+        int64_t nz = 0;
+        while (nz < d && dyt[nz] == 0.0) ++nz;
+        if (nz == d) continue;                                      /* dy_t = 0: no contribution */
         logits_row(xt, Wr, d, E, s);                                                        /* Eq. 1 */
         double m;
         select_one(s, b, E, k, sel, g, &m, taken, key);                                    /* Eqs. 7, 4, 5 */

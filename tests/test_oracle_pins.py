@@ -643,3 +643,24 @@ def test_backward_rows_reassemble_the_layer_gradients(swiglu):
     lhs = float(np.sum(gate_rows * st["dg"]) + lam * np.sum(dy * S))
     rhs = float(np.sum(dy * y))
     assert abs(lhs - rhs) <= 1e-12 * max(abs(rhs), 1.0)
+
+
+def test_backward_skips_tokens_without_dy_exactly():
+    """A token whose dy row is zero contributes nothing: with dy on 3 of 8192 tokens the
+    backward equals, bit for bit, the backward of the 3-token layer holding those tokens
+    (same weights), and dx is zero elsewhere."""
+    lay = workloads.make_layer(workloads.small_config(8192, 128, 16, 4, 64, h_s=64, lam=0.5, seed=3))
+    c = lay.cfg
+    toks = np.array([5, 4000, 8191])
+    rng = _rng(92)
+    dy = np.zeros((c.T, c.d))
+    dy[toks] = rng.standard_normal((toks.size, c.d))
+    full = oracle.backward(lay.x, lay.Wr, lay.b, lay.W1, lay.W2, c.k, dy, lay.Ws1, lay.Ws2, c.lam)
+    part = oracle.backward(lay.x[toks], lay.Wr, lay.b, lay.W1, lay.W2, c.k, dy[toks], lay.Ws1, lay.Ws2,
+                           c.lam)
+    for name in part:
+        if name == "dx":
+            assert np.array_equal(full["dx"][toks], part["dx"])
+            assert not np.any(np.delete(full["dx"], toks, axis=0))
+        else:
+            assert np.array_equal(full[name], part[name]), name
