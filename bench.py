@@ -4,13 +4,17 @@ One step = one whole layer forward (router, expert-major order, grouped up- and
 down-projection with the fused combine, shared expert, final bf16 output) over
 one batch of synthetic tokens, through the C ABI (moevie_moe_forward).
 
-    python bench.py [--gpus N] [--steps K] [--warmup W] [--config c1] [--impl ours|reference]
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--config c4] [--extra c1,c2,c3]
+                    [--impl ours|reference]
 
-Prints one JSON line.  Default workload: the image-batch layer (c1: T=8192,
-d=1024, E=64, k=8, h=512, one shared expert h_s=1024).  Under torchrun each rank
-runs its own replica of the workload (tokens shard with no exchange step), the
-timed region is bracketed by barriers, and the slowest rank's time is used.
-`--impl reference` times the CPU oracle on a bounded token sample instead.
+Prints one JSON line.  Default workload: the largest single-GPU layer, the stress
+layer (c4: T=65536, d=1664, E=256, k=8, h=416, one saturated expert, Zipf(1.1)
+loads over the rest, 3 empty experts).  On one GPU the other layers named by
+--extra are measured after it and reported under "per_config" (device-resident
+time, layer roofline fraction, stage times, memory-bound stages).  Under torchrun
+each rank runs its own replica of the workload (tokens shard with no exchange
+step), the timed region is bracketed by barriers, and the slowest rank's time is
+used.  `--impl reference` times the CPU oracle on a bounded token sample instead.
 """
 from __future__ import annotations
 
@@ -38,7 +42,9 @@ def parse():
     ap.add_argument("--gpus", type=int, default=1)
     ap.add_argument("--steps", type=int, default=50)
     ap.add_argument("--warmup", type=int, default=5)
-    ap.add_argument("--config", default="c1", choices=sorted(workloads.CONFIGS))
+    ap.add_argument("--config", default="c4", choices=sorted(workloads.CONFIGS))
+    ap.add_argument("--extra", default="c1,c2,c3",
+                    help="other workloads measured after the main one (1 GPU only; '' for none)")
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
     return ap.parse_args()
@@ -225,20 +231,7 @@ def run_reference(args, rank):
     print(json.dumps(out), flush=True)
 
 
-def run_ours(args, rank, world):
-    import torch
-    import torch.distributed as dist
-
-    import __graft_entry__
-    from paper_2608_17402_gb300 import moevie
-    from paper_2608_17402_gb300.replicas import max_over_ranks
-
-    local = int(os.environ.get("LOCAL_RANK", "0"))
-    torch.cuda.set_device(local)
-    __graft_entry__.build()
-    cfg = workloads.CONFIGS[args.config]
-    lay = workloads.make_layer(cfg)
-
+def _device_layer(cfg, lay, moevie, torch):
     def bf(a):
         return torch.from_numpy(np.ascontiguousarray(a).view(np.int16)).view(torch.bfloat16).cuda()
 
@@ -251,7 +244,36 @@ def run_ours(args, rank, world):
                             Ws2=None if lay.Ws2 is None else bf(lay.Ws2), lam=cfg.lam,
                             W3=None if lay.W3 is None else rows(lay.W3),
                             Ws3=None if lay.Ws3 is None else rows(lay.Ws3))
-    x = bf(lay.x)
+    return W, bf(lay.x)
+
+
+def memory_bound_stages(cfg, stages, pk):
+    """Achieved HBM bandwidth of the memory-bound stages from their algorithmic bytes
+    and their CUDA-event times: the expert-major order (idx and gates read, perm, inv,
+    row token and row gate written; the band-ordered item table, when present, is
+    metadata and not counted) and the bf16 finalize (fp32 accumulator read, y written)."""
+    T, d, k = cfg.T, cfg.d, cfg.k
+    out = {}
+    for stage, kern, nbytes in (
+            ("permute", "perm_fused_kernel (+ item_order_kernel when band-ordered)", 24.0 * T * k),
+            ("finalize", "f32_to_bf16_kernel", 6.0 * T * d)):
+        us = stages[stage] * 1e3
+        gbs = nbytes / (us * 1e-6) / 1e9 if us > 0 else None
+        out[stage] = {"kernel": kern, "bytes": nbytes, "us": us, "GB/s": gbs,
+                      "frac": None if gbs is None else gbs / pk["hbm_gbs"]}
+    return out
+
+
+def measure_config(cfg, args, world, local, with_clocks):
+    """Times one workload: device-resident layer forwards (value), per-stage event
+    times, and end to end with host copies.  Returns the numbers and the layer."""
+    import torch
+    import torch.distributed as dist
+
+    from paper_2608_17402_gb300 import moevie
+
+    lay = workloads.make_layer(cfg)
+    W, x = _device_layer(cfg, lay, moevie, torch)
     y = torch.empty((cfg.T, cfg.d), dtype=torch.bfloat16, device="cuda")
     ws = moevie.Workspace(cfg.T, cfg.d, cfg.E, cfg.k, cfg.h, cfg.h_s)
     flush = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device="cuda")
@@ -276,7 +298,10 @@ def run_ours(args, rank, world):
 
     starts = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
     ends = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
-    with ClockSampler(local) as clk:
+    clk = ClockSampler(local) if with_clocks else None
+    if clk is not None:
+        clk.__enter__()
+    try:
         barrier()
         n0 = moevie.moevie_launch_count()
         for i in range(args.steps):
@@ -286,6 +311,9 @@ def run_ours(args, rank, world):
             ends[i].record(stream)
         barrier()
         launches = moevie.moevie_launch_count() - n0
+    finally:
+        if clk is not None:
+            clk.__exit__(None, None, None)
     ms = statistics.mean(s.elapsed_time(e) for s, e in zip(starts, ends))
 
     # per-stage times (events recorded between the launches, same stream)
@@ -320,17 +348,62 @@ def run_ours(args, rank, world):
     code, detail = moevie.moevie_get_device_status(ws)
     if code != 0:
         raise RuntimeError(f"device status {code} {detail}")
+    del ws, flush, W, x, y
+    torch.cuda.empty_cache()
+    return {"ms": ms, "e2e_ms": e2e_ms, "stages": stages, "work": work, "launches": int(launches),
+            "clocks": None if clk is None else clk.summary()}, lay
 
-    ms, e2e_ms = max_over_ranks([ms, e2e_ms], device="cuda")   # slowest rank
-    if rank != 0:
-        return
 
-    pk = peaks()
-    value = world * cfg.T / (ms / 1e3)
+def summarise(cfg, m, pk, world):
+    """Throughput, dominant-kernel roofline and layer roofline of one measured workload."""
+    stages, work, ms = m["stages"], m["work"], m["ms"]
     dom = max(("up_gemm", "down_gemm"), key=lambda s: stages[s])
     dom_flops = work["flops_up_gemm"] if dom == "up_gemm" else work["flops_down_gemm"]
     achieved = dom_flops / (stages[dom] / 1e3) / 1e12
     t_roof = max(work["flops"] / (pk["bf16_tflops"] * 1e12), work["bytes"] / (pk["hbm_gbs"] * 1e9))
+    roof = {"bound": "tensor", "kernel": f"grouped_gemm_kernel ({dom})", "achieved": achieved,
+            "peak": pk["bf16_tflops"], "unit": "TFLOP/s", "frac": achieved / pk["bf16_tflops"],
+            "traffic": captured_traffic(cfg.name, dom),
+            "peak_source": pk["source"] + " bf16 burst (of measured)"}
+    layer = {"flops": work["flops"], "bytes": work["bytes"], "roofline_us": t_roof * 1e6,
+             "frac": t_roof / (ms / 1e3), "touched_experts": work["touched_experts"]}
+    return roof, layer, world * cfg.T / (ms / 1e3)
+
+
+def run_ours(args, rank, world):
+    import torch
+    import torch.distributed as dist  # noqa: F401
+
+    import __graft_entry__
+    from paper_2608_17402_gb300.replicas import max_over_ranks
+
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    torch.cuda.set_device(local)
+    __graft_entry__.build()
+    cfg = workloads.CONFIGS[args.config]
+    m, lay = measure_config(cfg, args, world, local, with_clocks=True)
+    ms, e2e_ms = max_over_ranks([m["ms"], m["e2e_ms"]], device="cuda")   # slowest rank
+    m["ms"], m["e2e_ms"] = ms, e2e_ms
+
+    # the other layer workloads, one GPU only (device-resident numbers and stages)
+    extra = {}
+    if world == 1 and args.extra:
+        for name in [n for n in args.extra.split(",") if n and n != cfg.name]:
+            c2 = workloads.CONFIGS[name]
+            mc, _ = measure_config(c2, args, 1, local, with_clocks=False)
+            roof, layer, value = summarise(c2, mc, peaks(), 1)
+            extra[name] = {"workload": f"{c2.name}: {c2.note}", "tokens_per_s": value,
+                           "us_per_layer": mc["ms"] * 1e3, "layer_roofline_us": layer["roofline_us"],
+                           "layer_frac": layer["frac"], "dominant": roof,
+                           "stages_us": {k: v * 1e3 for k, v in mc["stages"].items()},
+                           "memory_bound": memory_bound_stages(c2, mc["stages"], peaks()),
+                           "e2e_tokens_per_s": c2.T / (mc["e2e_ms"] / 1e3)}
+    if rank != 0:
+        return
+
+    pk = peaks()
+    roof, layer, value = summarise(cfg, m, pk, world)
+    layer["peaks"] = pk
     out = {
         "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": ms, "us_per_layer": ms * 1e3, "higher_is_better": True,
@@ -339,19 +412,17 @@ def run_ours(args, rank, world):
                    "h": cfg.h, "h_s": cfg.h_s, "act": cfg.act, "lambda": cfg.lam, "seed": cfg.seed,
                    "parallelism": f"replicas x{world}" if world > 1 else "single GPU",
                    "l2": f"flushed between steps ({L2_FLUSH_BYTES >> 20} MiB write outside the timed window)"},
-        "roofline": {"bound": "tensor", "kernel": f"grouped_gemm_kernel ({dom})", "achieved": achieved,
-                     "peak": pk["bf16_tflops"], "unit": "TFLOP/s", "frac": achieved / pk["bf16_tflops"],
-                     "traffic": captured_traffic(cfg.name, dom),
-                     "peak_source": pk["source"] + " bf16 burst (of measured)"},
-        "layer_roofline": {"flops": work["flops"], "bytes": work["bytes"], "roofline_us": t_roof * 1e6,
-                           "frac": t_roof / (ms / 1e3), "touched_experts": work["touched_experts"],
-                           "peaks": pk},
-        "stages_ms": stages,
+        "roofline": roof,
+        "layer_roofline": layer,
+        "stages_ms": m["stages"],
+        "memory_bound": memory_bound_stages(cfg, m["stages"], pk),
         "e2e": {"value": world * cfg.T / (e2e_ms / 1e3), "unit": "tokens/s",
                 "h2d_bytes_per_step": cfg.T * cfg.d * 2, "d2h_bytes_per_step": cfg.T * cfg.d * 2},
-        "gpu_launches": int(launches),
-        "clocks": clk.summary(),
+        "gpu_launches": m["launches"],
+        "clocks": m["clocks"],
     }
+    if extra:
+        out["per_config"] = extra
     if world == 1 and not args.no_cpu_baseline:
         out["cpu_baseline"] = cpu_baseline(lay)
     print(json.dumps(out), flush=True)

@@ -79,18 +79,23 @@ moevie_status moevie_workspace_init(void* ws, size_t ws_bytes, void* stream);
 
 /* Router (Eqs. 1, 7, 4-5).  x bf16 [T, d], W_r fp32 [d, E], b fp32 [E].
  * Out: idx int32 [T, k] (ascending ids per token), gate fp32 [T, k] (same order).
- * Logits are fp32; a token whose k-th and (k+1)-th keys are closer than the fp32
- * error bound is re-decided with exactly computed (fp64) logits of the experts
- * near its boundary, so idx equals the exact-arithmetic selection. */
+ * Logits are fp32 (tensor cores); a token whose selection the fp32 logits cannot
+ * certify (its k-th and (k+1)-th keys closer than their error bounds) is re-decided
+ * from exact logits of the experts near its boundary -- an integer long accumulator
+ * of the bf16 x fp32 products, within d 2^-64 sum|x_i w_i| of the exact dot product --
+ * with the keys sigmoid(s) + b then formed in fp64, so idx equals the
+ * exact-arithmetic selection. */
 moevie_status moevie_route(const void* x, const float* W_r, const float* b, int64_t T, int64_t d,
                            int64_t E, int64_t k, int32_t* idx, float* gate, void* ws,
                            size_t ws_bytes, void* stream);
 
 /* Expert-major order (App. B, Algorithm 1, phase 1: Sort, index = pos // K,
  * BinCount, CumSum).  idx int32 [T, k].  Out: counts int32 [E], offsets int32
- * [E + 1] (exclusive prefix, offsets[E] = T*k), perm int32 [T*k] (row -> flat slot
- * t*k + j, stable), inv int32 [T*k] (flat slot -> row).  An id outside [0, E) is a
- * device error (MOEVIE_ERR_DEVICE in the status block; that slot is dropped). */
+ * [E + 1] (exclusive prefix; offsets[E] = the number of valid slots, T*k when every
+ * id is valid), perm int32 [T*k] (row -> flat slot t*k + j, stable), inv int32 [T*k]
+ * (flat slot -> row).  An id outside [0, E) is a device error (MOEVIE_ERR_DEVICE in
+ * the status block): that slot is dropped, its inv entry is -1, it is not counted in
+ * counts / offsets, and perm rows from offsets[E] to T*k are left unwritten. */
 moevie_status moevie_permute(const int32_t* idx, int64_t T, int64_t k, int64_t E, int32_t* counts,
                              int32_t* offsets, int32_t* perm, int32_t* inv, void* ws,
                              size_t ws_bytes, void* stream);
@@ -173,7 +178,9 @@ moevie_status moevie_moe_forward(const moevie_layer* layer, const void* x, int64
  *
  * Set-up: the first call on a device (with that device current) looks up the
  * array's device address, which may load the library's device code; make that
- * first call before any stream capture.  Later calls reuse the address.
+ * first call before any stream capture.  Later calls reuse the address as long as
+ * the device's context is the same; after cudaDeviceReset the next call looks it up
+ * again in the new context (again, before any capture).
  *
  * Concurrency: all calls on one device share the one array.  Two calls whose GPU
  * work overlaps (different streams, or several host threads without ordering) race

@@ -474,8 +474,12 @@ int oracle_update_bias(const int32_t* counts, int64_t E, float alpha, int rule, 
  *   dW1[e] += x^T du,  dW3[e] += x^T dv,  dx += du W1[e]^T + dv W3[e]^T.
  * Tokens are taken one after another in ascending t (one thread: the weight
  * gradients are sums over tokens, accumulated in that order).  A token whose dy row
- * is all zero adds exact zeros to every gradient and is skipped, so a sampled check
- * (dy nonzero on a few tokens) costs only those tokens.  All outputs are
+ * is all zero adds exact zeros to every gradient -- every term it contributes is a
+ * product with an element of dy_t -- as long as the other factor is finite, which
+ * holds when its input row x_t and every weight of the layer are finite; such a token
+ * is skipped, so a sampled check (dy nonzero on a few tokens) costs only those tokens.
+ * With a non-finite x_t or weight it is not skipped, so 0 * inf gives NaN exactly as
+ * the unskipped sum does.  All outputs are
  * double and are overwritten: dx [T, d], dWr [d, E], dW1 [E, d, h], dW2 [E, h, d],
  * dW3 [E, d, h] (with W3), dWs1 [d, hs], dWs2 [hs, d], dWs3 [d, hs] (with Ws3). */
 
@@ -538,6 +542,19 @@ static void expert_backward(const uint16_t* xt, const uint16_t* W1e, const uint1
     }
 }
 
+/* 1 when every value of the n bf16 values v is finite (exponent field not all ones). */
+static int bf16_all_finite(const uint16_t* v, int64_t n) {
+    for (int64_t i = 0; i < n; ++i)
+        if ((v[i] & 0x7f80u) == 0x7f80u) return 0;
+    return 1;
+}
+
+static int f32_all_finite(const float* v, int64_t n) {
+    for (int64_t i = 0; i < n; ++i)
+        if (!isfinite(v[i])) return 0;
+    return 1;
+}
+
 int oracle_backward(const uint16_t* x, const float* Wr, const float* b,
                     const uint16_t* W1, const uint16_t* W2, const uint16_t* W3,
                     const uint16_t* Ws1, const uint16_t* Ws2, const uint16_t* Ws3, double lambda,
@@ -575,13 +592,19 @@ int oracle_backward(const uint16_t* x, const float* Wr, const float* b,
         err = ORACLE_ERR_NOMEM;
         goto done;
     }
+    /* zero-cotangent tokens may be skipped only when the factors they multiply are finite */
+    const int weights_finite =
+        f32_all_finite(Wr, d * E) && f32_all_finite(b, E) && bf16_all_finite(W1, E * d * h) &&
+        bf16_all_finite(W2, E * h * d) && (!W3 || bf16_all_finite(W3, E * d * h)) &&
+        (hs == 0 || (bf16_all_finite(Ws1, d * hs) && bf16_all_finite(Ws2, hs * d) &&
+                     (!Ws3 || bf16_all_finite(Ws3, d * hs))));
     for (int64_t t = 0; t < T; ++t) {
         const uint16_t* xt = x + t * d;
         const double* dyt = dy + t * d;
         double* dxt = dx + t * d;
         int64_t nz = 0;
         while (nz < d && dyt[nz] == 0.0) ++nz;
-        if (nz == d) continue;                                      /* dy_t = 0: no contribution */
+        if (nz == d && weights_finite && bf16_all_finite(xt, d)) continue;   /* dy_t = 0: adds zeros */
         logits_row(xt, Wr, d, E, s);                                                        /* Eq. 1 */
         double m;
         select_one(s, b, E, k, sel, g, &m, taken, key);                                    /* Eqs. 7, 4, 5 */

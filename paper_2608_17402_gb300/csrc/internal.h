@@ -94,7 +94,7 @@ cudaError_t launch_route_sum_parts(const float* logits, int64_t part_stride, int
                                    float* out, cudaStream_t s);
 
 // Keys, warp top-k with a certificate, gates; uncertified tokens are re-decided
-// with exact (fp64) logits of the experts near their boundary.  logits: nparts
+// with exact logits (integer long accumulator) of the experts near their boundary.  logits: nparts
 // partial arrays [T][ld] (part_stride floats apart); part 0 is overwritten with the
 // sum for uncertified tokens.
 cudaError_t launch_route_select(const __nv_bfloat16* x, const float* wrt, const float* b,
@@ -284,7 +284,8 @@ static_assert((PERM_STATIC_MAX_SLOTS + PERM_STATIC_MAX_CHUNKS - 1) / PERM_STATIC
 
 // Device address of that array on the current device.  The first call on a device
 // looks the symbol up (cudaGetSymbolAddress, which may load the module); later calls
-// return the cached address.  Thread-safe.
+// return the cached address while the device's context is the one it was looked up in
+// (after a device reset the next call looks it up again).  Thread-safe.
 cudaError_t perm_static_scratch(unsigned char** out);
 
 // ------------------------------------------------------------------- misc

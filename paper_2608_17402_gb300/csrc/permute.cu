@@ -416,20 +416,45 @@ __global__ void __launch_bounds__(1024) item_order_kernel(
 // workspace from its caller nor an allocation of its own (layout in internal.h).
 static __device__ __align__(256) unsigned char g_perm_static_scratch[PERM_STATIC_SCRATCH_BYTES];
 
+// The current context (driver cuCtxGetCurrent, reached through the runtime's entry-point
+// query so that the library links only the runtime); nullptr when it cannot be read.
+static void* current_context() {
+    using GetCtx = CUresult (*)(CUcontext*);
+    static std::atomic<GetCtx> fn{nullptr};
+    GetCtx f = fn.load(std::memory_order_acquire);
+    if (!f) {
+        void* ptr = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuCtxGetCurrent", &ptr, 12000, cudaEnableDefault, &q) !=
+                cudaSuccess ||
+            q != cudaDriverEntryPointSuccess || !ptr)
+            return nullptr;
+        f = reinterpret_cast<GetCtx>(ptr);
+        fn.store(f, std::memory_order_release);
+    }
+    CUcontext c = nullptr;
+    return f(&c) == CUDA_SUCCESS ? static_cast<void*>(c) : nullptr;
+}
+
 cudaError_t perm_static_scratch(unsigned char** out) {
     constexpr int kMaxDevices = 64;
     static std::mutex mu;
     static unsigned char* addr[kMaxDevices] = {};
+    static void* ctx[kMaxDevices] = {};
     int dev = -1;
     cudaError_t err = cudaGetDevice(&dev);
     if (err != cudaSuccess) return err;
     if (dev < 0 || dev >= kMaxDevices) return cudaErrorInvalidDevice;
+    // The address belongs to the context it was looked up in: after a device reset
+    // the runtime makes a new primary context, and the address is looked up again.
+    void* cur = current_context();
     std::lock_guard<std::mutex> lock(mu);
-    if (!addr[dev]) {   // once per device, with that device current
+    if (!addr[dev] || cur == nullptr || cur != ctx[dev]) {   // with that device current
         void* p = nullptr;
         err = cudaGetSymbolAddress(&p, g_perm_static_scratch);
         if (err != cudaSuccess) return err;
         addr[dev] = static_cast<unsigned char*>(p);
+        ctx[dev] = current_context();   // the context the runtime has now made current
     }
     *out = addr[dev];
     return cudaSuccess;

@@ -213,16 +213,24 @@ def moevie_permute(idx, E, ws: Workspace, stream=None):
     return counts, offsets, perm, inv
 
 
-def moevie_permute_static(idx, E, stream=None):
+def moevie_permute_static(idx, E, out=None, stream=None):
     """moevie_permute without a workspace: the library's fixed device scratch is used
-    (T * k <= 2^20).  Calls whose GPU work overlaps race on that scratch."""
+    (T * k <= 2^20).  Calls whose GPU work overlaps race on that scratch.  ``out``: an
+    optional tuple of preallocated (counts [E], offsets [E + 1], perm [T*k], inv [T*k])
+    int32 tensors, so that the call itself allocates nothing."""
     _want(idx, torch.int32, "idx")
     T, k = idx.shape
     dev = idx.device
-    counts = torch.empty(E, dtype=torch.int32, device=dev)
-    offsets = torch.empty(E + 1, dtype=torch.int32, device=dev)
-    perm = torch.empty(T * k, dtype=torch.int32, device=dev)
-    inv = torch.empty(T * k, dtype=torch.int32, device=dev)
+    if out is not None:
+        counts, offsets, perm, inv = (_want(t, torch.int32, n)
+                                      for t, n in zip(out, ("counts", "offsets", "perm", "inv")))
+        if counts.numel() != E or offsets.numel() != E + 1 or perm.numel() < T * k or inv.numel() < T * k:
+            raise ValueError("moevie_permute_static: output tensors of the wrong size")
+    else:
+        counts = torch.empty(E, dtype=torch.int32, device=dev)
+        offsets = torch.empty(E + 1, dtype=torch.int32, device=dev)
+        perm = torch.empty(T * k, dtype=torch.int32, device=dev)
+        inv = torch.empty(T * k, dtype=torch.int32, device=dev)
     _call("moevie_permute_static", _p(idx), T, k, E, _p(counts), _p(offsets), _p(perm), _p(inv),
           _stream(stream))
     return counts, offsets, perm, inv

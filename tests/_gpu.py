@@ -66,3 +66,56 @@ def assert_close(got: np.ndarray, want: np.ndarray, what: str = "y"):
 def check_status(ws):
     code, detail = moevie.moevie_get_device_status(ws)
     assert code == 0, f"device status {moevie.STATUS_NAMES.get(code, code)} detail={detail}"
+
+
+def stratified_tokens(T, k, counts, offsets, perm, n_random=256, seed=0, bm=256, max_bands=16):
+    """Output rows (tokens) to compare against the oracle on a full-size layer, chosen
+    to cover the paths that only the full launch takes, by stratum:
+
+    * ``last_tile``: for every non-empty expert, the first and last two rows of its
+      last (usually partial) m-tile of ``bm`` rows;
+    * ``hot``: rows on both sides of every m-tile boundary of the most loaded expert;
+    * ``band_edges``: the tokens on both sides of every token-band boundary
+      ``ceil(b T / nb)`` of a band-ordered down-projection, for every band count
+      ``nb <= max_bands``;
+    * ``small``: the rows of the eight least loaded non-empty experts (all of them,
+      or the first and last 64 of a segment longer than 128);
+    * ``random``: ``n_random`` uniformly drawn tokens.
+
+    Returns the sorted unique tokens and a dict of stratum -> number of tokens."""
+    counts = np.asarray(counts)
+    offsets = np.asarray(offsets)
+    perm = np.asarray(perm)
+    strata = {}
+
+    def rows_to_tokens(rows):
+        rows = np.asarray([r for r in rows if 0 <= r < T * k], dtype=np.int64)
+        return np.unique(perm[rows] // k) if rows.size else np.zeros(0, np.int64)
+
+    rows = []
+    for e in np.flatnonzero(counts > 0):
+        c, o = int(counts[e]), int(offsets[e])
+        first = o + (c - 1) // bm * bm
+        rows += [first, first + 1, o + c - 2, o + c - 1]
+    strata["last_tile"] = rows_to_tokens(rows)
+    hot = int(np.argmax(counts))
+    rows = []
+    for m in range(bm, int(counts[hot]), bm):
+        rows += [offsets[hot] + m - 1, offsets[hot] + m]
+    strata["hot"] = rows_to_tokens(rows)
+    edges = set()
+    for nb in range(2, max_bands + 1):
+        for b in range(1, nb):
+            t0 = -(-b * T // nb)
+            edges.update({t0 - 1, t0})
+    strata["band_edges"] = np.array(sorted(t for t in edges if 0 <= t < T), np.int64)
+    nz = np.flatnonzero(counts > 0)
+    small = nz[np.argsort(counts[nz], kind="stable")[:8]]
+    rows = []
+    for e in small:   # every row, or the first and last 64 of a larger segment
+        o, c = int(offsets[e]), int(counts[e])
+        rows += list(range(o, o + c)) if c <= 128 else list(range(o, o + 64)) + list(range(o + c - 64, o + c))
+    strata["small"] = rows_to_tokens(rows)
+    strata["random"] = np.random.default_rng(seed).choice(T, min(n_random, T), replace=False)
+    toks = np.unique(np.concatenate([v for v in strata.values()] + [np.array([0, T - 1])]))
+    return toks.astype(np.int32), {k2: int(v.size) for k2, v in strata.items()}

@@ -12,7 +12,7 @@ import oracle
 import workloads
 from paper_2608_17402_gb300 import moevie
 from tests._gpu import (MARGIN_PINNED, assert_close, check_status, layer_to_device,
-                        to_np_f64, workspace_for)
+                        stratified_tokens, to_np_f64, workspace_for)
 
 pytestmark = pytest.mark.gpu
 
@@ -67,18 +67,23 @@ def test_forward_full_config(name):
 
 
 @pytest.mark.parametrize("name", ["c3", "c4"])
-def test_forward_large_config_sampled(name):
+def test_forward_large_config_stratified(name):
+    """The video and stress layers in the launch configuration the benchmark times:
+    every routing output bit-exact, and at least 1024 output rows against the oracle,
+    chosen by stratum (every expert's last m-tile, the hot expert's tile boundaries,
+    both sides of every possible token-band boundary, the least loaded experts, and a
+    uniform sample)."""
     lay = workloads.make_layer(workloads.CONFIGS[name])
     y, rt = _run(lay)
     counts = _check_routing(lay, rt)
     c = lay.cfg
     assert (counts == 0).sum() >= 3, "the skewed layer must keep its empty experts"
-    rng = np.random.default_rng(0)
-    toks = np.unique(np.concatenate([[0, 1, c.T // 2, c.T - 1], rng.choice(c.T, 60, replace=False)]))
+    toks, strata = stratified_tokens(c.T, c.k, counts, rt["offsets"], rt["perm"])
+    assert toks.size >= 1024, toks.size
     want, *_ = oracle.forward_tokens(lay.x, lay.Wr, lay.b, lay.W1, lay.W2, c.k, lay.Ws1, lay.Ws2,
-                                     c.lam, tokens=toks.astype(np.int32))
+                                     c.lam, tokens=toks)
     rel, mx = assert_close(y[toks], want)
-    print(f"{name}: sampled {toks.size} tokens, rel-L2 {rel:.2e}, max|err|/RMS {mx:.2e}")
+    print(f"{name}: {toks.size} tokens by stratum {strata}, rel-L2 {rel:.2e}, max|err|/RMS {mx:.2e}")
 
 
 def test_forward_is_deterministic_in_routing_and_repeatable():

@@ -14,7 +14,7 @@ import oracle
 import workloads
 from paper_2608_17402_gb300 import moevie
 from tests._gpu import (MARGIN_PINNED, assert_close, check_status, layer_to_device,
-                        to_np_f64, workspace_for)
+                        stratified_tokens, to_np_f64, workspace_for)
 
 pytestmark = pytest.mark.gpu
 
@@ -58,8 +58,9 @@ def test_ragged_hidden_width_small(T, d, E, k, h, hs, act):
 
 @pytest.mark.parametrize("name", ["pB", "pL", "pH"])
 def test_paper_layer_sampled(name):
-    """Full-size layer, all routing outputs, and a sample of output rows.  The shared
-    expert (h_s = h) rides in the routed launches as one always-on group."""
+    """Full-size layer, all routing outputs, and at least 1024 output rows chosen by
+    stratum (as for the video and stress layers).  The shared expert (h_s = h) rides
+    in the routed launches as one always-on group."""
     lay = workloads.make_layer(workloads.CONFIGS[name])
     c = lay.cfg
     assert moevie.moevie_shared_groups(c.T, c.d, c.E, c.k, c.h, c.h_s) == 1
@@ -71,11 +72,11 @@ def test_paper_layer_sampled(name):
     oc, oo, op, oi = oracle.permute(oidx, c.E)
     for key, want in (("counts", oc), ("offsets", oo), ("perm", op), ("inv", oi)):
         assert np.array_equal(rt[key], want), key
-    rng = np.random.default_rng(2)
-    toks = np.unique(np.concatenate([[0, 1, c.T - 1], rng.choice(c.T, 45, replace=False)]))
-    want, *_ = _want(lay, tokens=toks.astype(np.int32))
+    toks, strata = stratified_tokens(c.T, c.k, oc, oo, op, n_random=512, seed=2)
+    assert toks.size >= 1024, toks.size
+    want, *_ = _want(lay, tokens=toks)
     rel, mx = assert_close(y[toks], want)
-    print(f"{name}: sampled {toks.size} tokens, rel-L2 {rel:.2e}, max|err|/RMS {mx:.2e}")
+    print(f"{name}: {toks.size} tokens by stratum {strata}, rel-L2 {rel:.2e}, max|err|/RMS {mx:.2e}")
 
 
 def test_unpadded_weights_are_rejected():

@@ -106,20 +106,50 @@ def test_route_full_configs(name):
     print(f"{name}: {nfb} of {lay.cfg.T} tokens re-decided exactly")
 
 
-@pytest.mark.parametrize("name", ["c0", "c1", "c4"])
-def test_fast_logit_error_within_bound(name):
-    """The tensor-core logits stay far inside the error bound the router certifies
-    with (ROUTE_TAU_C = 128 units of 2^-24 |x_t| |W_r[:, e]|): measured max below 1/4
-    of it over every token of the layer."""
-    lay = workloads.make_layer(workloads.CONFIGS[name])
-    T = lay.cfg.T
-    x, Wr = lay.x[:T], lay.Wr
-    ws = moevie.Workspace(T, lay.cfg.d, lay.cfg.E, 1, 16)
+def _logit_error_units(x, Wr):
+    """max |s_fast - s| over the layer in units of 2^-24 |x_t| |W_r[:, e]|."""
+    T, d = x.shape
+    E = Wr.shape[1]
+    ws = moevie.Workspace(T, d, E, 1, 16)
     s = moevie.moevie_test_route_logits(dev_bf16(x), dev(Wr), ws).cpu().numpy().astype(np.float64)
     check_status(ws)
     so = oracle.logits(x, Wr)
     xf = workloads.bf16_bits_to_f32(x).astype(np.float64)
     scale = 2.0 ** -24 * np.linalg.norm(xf, axis=1)[:, None] * np.linalg.norm(Wr.astype(np.float64), axis=0)[None, :]
-    ratio = np.abs(s - so) / scale
-    print(f"{name}: max |s_fast - s| = {ratio.max():.3f} units of 2^-24 |x_t| |W_r[:, e]|")
-    assert ratio.max() < 128 / 4
+    return float((np.abs(s - so) / scale).max())
+
+
+@pytest.mark.parametrize("name", ["c0", "c1", "c2", "c3", "c4", "s1", "pB", "pL", "pH"])
+def test_fast_logit_error_within_bound(name):
+    """The tensor-core logits stay far inside the error bound the router certifies
+    with (ROUTE_TAU_C = 128 units of 2^-24 |x_t| |W_r[:, e]|): measured max below 1/4
+    of it over every token of every layer workload."""
+    lay = workloads.make_layer(workloads.CONFIGS[name])
+    r = _logit_error_units(lay.x, lay.Wr)
+    print(f"{name}: max |s_fast - s| = {r:.3f} units of 2^-24 |x_t| |W_r[:, e]|")
+    assert r < 128 / 4
+
+
+@pytest.mark.parametrize("E", [64, 256])
+@pytest.mark.parametrize("pattern", ["same_sign", "alternating", "random_sign"])
+def test_fast_logit_error_adversarial(pattern, E):
+    """Inputs built to maximise the fp32 accumulation error of the logits at the
+    stress layer's width (d = 1664): every product x_i w_i of nearly the same
+    magnitude (x_i = +-1, w_i = 0.02 (1 + small) with all 24 significand bits of w in
+    use, so all three bf16 pieces of W_r are non-zero), with the signs all equal
+    (the partial sums grow to d |x_i w_i|), alternating, or random.  E = 64 puts the
+    three pieces side by side (summed in the epilogue), E = 256 one after another
+    along K.  The error must stay below 1/4 of the certified bound."""
+    rng = np.random.default_rng(E + len(pattern))
+    T, d = 256, 1664
+    if pattern == "same_sign":
+        xs = np.ones((T, d), np.float32)
+    elif pattern == "alternating":
+        xs = np.tile(np.array([1.0, -1.0], np.float32), (T, d // 2))
+    else:
+        xs = rng.choice(np.array([1.0, -1.0], np.float32), (T, d))
+    x = workloads.f32_to_bf16_bits(xs)
+    Wr = (0.02 * (1.0 + rng.uniform(0.0, 2.0 ** -6, (d, E)))).astype(np.float32)
+    r = _logit_error_units(x, Wr)
+    print(f"{pattern}, E={E}: max |s_fast - s| = {r:.3f} units of 2^-24 |x_t| |W_r[:, e]|")
+    assert r < 128 / 4

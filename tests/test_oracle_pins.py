@@ -664,3 +664,24 @@ def test_backward_skips_tokens_without_dy_exactly():
             assert not np.any(np.delete(full["dx"], toks, axis=0))
         else:
             assert np.array_equal(full[name], part[name]), name
+
+
+def test_backward_zero_dy_token_with_nonfinite_weight_is_not_skipped():
+    """A token with dy_t = 0 adds exact zeros only when the factors its terms multiply
+    are finite.  With an infinite entry in W2 of an expert the token uses, the
+    gradient through that expert is 0 * inf = NaN, as in torch autograd of the layer;
+    the skip of zero-cotangent tokens must not hide it."""
+    x, Wr, b, W1, W2, W3, Ws1, Ws2, Ws3, dy, lam = _backward_case(5, 4, 8, 4, 2, 6)
+    idx, _, _ = oracle.route(x, Wr, b, 2)
+    dy[0] = 0.0
+    W2 = W2.copy()
+    W2[idx[0, 0], 0, 0] = 0x7F80   # bf16 +inf
+    got = oracle.backward(x, Wr, b, W1, W2, 2, dy)
+    xt, Wt = _t64(x), _t64(W2)
+    xt.requires_grad_(True)
+    y = _torch_layer_from_oracle_routing(xt, torch.from_numpy(Wr.astype(np.float64)), _t64(W1), Wt,
+                                         idx, lam)
+    (torch.from_numpy(dy) * y).sum().backward()
+    want = xt.grad.numpy()
+    assert np.isnan(want[0]).any()
+    assert np.array_equal(np.isnan(got["dx"][0]), np.isnan(want[0]))

@@ -63,3 +63,50 @@ def test_static_permute_rejects_oversize_and_accepts_empty():
     counts, offsets, _, _ = moevie.moevie_permute_static(
         torch.zeros((0, 4), dtype=torch.int32, device="cuda"), 16)
     assert int(counts.abs().sum()) == 0 and int(offsets.abs().sum()) == 0
+
+
+def test_static_permute_allocates_nothing():
+    """With its outputs preallocated, neither a second nor a third call changes the
+    device's free memory (cudaMemGetInfo) or torch's allocated bytes: the scratch is
+    the library's fixed device array.  The first call may load the library's device
+    code (set-up), so it runs before the measurement."""
+    T, E, k = 4096, 64, 8
+    idx = torch.from_numpy(_ids(T, E, k, 3)).cuda()
+    out = (torch.empty(E, dtype=torch.int32, device="cuda"),
+           torch.empty(E + 1, dtype=torch.int32, device="cuda"),
+           torch.empty(T * k, dtype=torch.int32, device="cuda"),
+           torch.empty(T * k, dtype=torch.int32, device="cuda"))
+    moevie.moevie_permute_static(idx, E, out=out)
+    torch.cuda.synchronize()
+    for _ in range(2):
+        free0, _ = torch.cuda.mem_get_info()
+        alloc0 = torch.cuda.memory_allocated()
+        moevie.moevie_permute_static(idx, E, out=out)
+        torch.cuda.synchronize()
+        free1, _ = torch.cuda.mem_get_info()
+        assert free1 == free0, (free0, free1)
+        assert torch.cuda.memory_allocated() == alloc0
+
+
+def test_static_permute_drops_out_of_range_ids():
+    """Ids -1 and E are device errors that drop their slot: inv = -1 there, counts and
+    offsets leave them out, and every valid slot keeps the stable expert-major row
+    that moevie_permute gives it (the workspace entry point, same rule)."""
+    T, E, k = 300, 16, 4
+    ids = _ids(T, E, k, 21)
+    bad = [(3, 0, -1), (77, 2, E), (299, 3, E), (150, 1, -1)]
+    for t, j, v in bad:
+        ids[t, j] = v
+    idx = torch.from_numpy(ids).cuda()
+    ws = moevie.Workspace(T, 8, E, k, 16)
+    want = [t.cpu() for t in moevie.moevie_permute(idx, E, ws)]
+    for _ in range(2):
+        counts, offsets, perm, inv = (t.cpu() for t in moevie.moevie_permute_static(idx, E))
+        for t, j, _v in bad:
+            assert int(inv[t * k + j]) == -1
+        valid = (ids >= 0) & (ids < E)
+        assert torch.equal(counts, torch.from_numpy(np.bincount(ids[valid], minlength=E).astype(np.int32)))
+        assert int(offsets[E]) == int(valid.sum())
+        assert torch.equal(counts, want[0]) and torch.equal(offsets, want[1]) and torch.equal(inv, want[3])
+        n = int(valid.sum())
+        assert torch.equal(perm[:n], want[2][:n])
