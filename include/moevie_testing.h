@@ -16,11 +16,12 @@
 extern "C" {
 #endif
 
-/* Router logits as the fast path computes them (Eq. 1: tensor cores, W_r split
- * exactly into three bf16 pieces, fp32 accumulation; for E <= 64 the three pieces'
- * products are accumulated separately and added hi + mid + lo): s[t, e] =
- * sum_i x[t, i] W_r[i, e].  s fp32 [T, E32] with E32 = E rounded up to a multiple of
- * 32 (the extra columns are zero). */
+/* Router logits as the fast path computes them (Eq. 1 on the tensor cores): W_r is
+ * split into bf16 pieces hi = bf16(w), mid = bf16(w - hi), and s[t, e] = sum_i x[t, i]
+ * (hi + mid)[i, e] with fp32 accumulation (for E <= 128 the two pieces' products are
+ * accumulated separately and added hi + mid).  The left-out lo = w - hi - mid is part of
+ * the certified error bound, not of these logits.  s fp32 [T, E32] with E32 = E rounded
+ * up to a multiple of 32 (the extra columns are zero). */
 moevie_status moevie_test_route_logits(const void* x, const float* W_r, int64_t T, int64_t d,
                                        int64_t E, float* s, void* ws, size_t ws_bytes,
                                        void* stream);

@@ -32,7 +32,7 @@ inline int64_t row_ld(int64_t h) { return (h + 7) / 8 * 8; }
 // the order is fixed, so a workspace sized for the whole layer also serves each
 // stage (which passes 0 for the sizes it does not use).
 struct Layout {
-    size_t status, xnorm, wnorm, wpart, wsplit, wrt, logits, fb_tokens;
+    size_t status, xnorm, wnorm, wpart, wexp, wsplit, wrt, logits, fb_tokens;
     size_t idx, gate, hist, counts, offsets, tiles, n_tiles, items, n_items, perm, inv, row_tok,
         row_gate;
     size_t H, Hs, yacc;
@@ -47,30 +47,28 @@ struct BandPlan {   // token bands and n-tiles per column group of the down-proj
 // not stay in L2 next to the streamed operands) the items run in nb token bands x
 // column groups of gsz n-tiles (item_order_kernel), so that the accumulator block
 // being reduced into (at most ITEM_BLOCK_BYTES) stays in L2.  Each extra band re-reads
-// the expert weights W2, each extra column group the rows of H: the split minimises
-// that traffic under the block-size bound.
+// the weights W2 of the experts with m-tiles in it, each extra column group the rows
+// of H.  Measured on GB300 (stress layer T = 65536, d = 1664, E = 256: 16 bands x 2
+// column groups 955 us, 8 x 2 990 us, 5 x 4 1016 us, 16 x 1 984 us; video layer T =
+// 32768, d = 1536, E = 128: every plan 408-411 us): the most bands, then the fewest
+// column groups whose block fits, is the best plan on both.  Skewed loads keep the W2
+// re-reads far below one per band per expert: an expert's rows span few bands unless
+// it is large, and a large one is re-read from L2 within a band.
 constexpr double ITEM_BAND_MIN_BYTES = 64.0 * (1 << 20);
 constexpr double ITEM_BLOCK_BYTES = 24.0 * (1 << 20);
 BandPlan choose_bands(int64_t T, int64_t d, int64_t E, int64_t k, int64_t h) {
+    (void)h;
     int BN = 0, nnt = 0;
     choose_bn((int)d, &BN, &nnt);
     const double yacc = 4.0 * T * d;
     if (yacc <= ITEM_BAND_MIN_BYTES || max_mtiles(T * k, E) > ITEM_MAX_TILES) return {1, nnt};
-    const double Hb = 2.0 * T * k * h, Wb = 2.0 * E * h * d;
-    BandPlan best{1, nnt};
-    double best_cost = 1e300;
-    for (int nb = 1; nb <= ITEM_MAX_BANDS; ++nb)
-        for (int nc = 1; nc <= nnt; ++nc) {
-            const int gsz = (nnt + nc - 1) / nc;
-            const int groups = (nnt + gsz - 1) / gsz;
-            if (yacc / ((double)nb * groups) > ITEM_BLOCK_BYTES) continue;
-            const double cost = Hb * groups + Wb * nb;
-            if (cost < best_cost) {
-                best_cost = cost;
-                best = {nb, gsz};
-            }
-        }
-    return best;
+    const int nb = ITEM_MAX_BANDS;
+    for (int groups = 1; groups <= nnt; ++groups) {
+        const int gsz = (nnt + groups - 1) / groups;
+        const int g = (nnt + gsz - 1) / gsz;   // groups that gsz actually gives
+        if (yacc / ((double)nb * g) <= ITEM_BLOCK_BYTES) return {nb, gsz};
+    }
+    return {nb, 1};
 }
 
 // The shared expert runs inside the grouped GEMMs as S = h_s / h always-on groups
@@ -112,9 +110,10 @@ Layout make_layout(int64_t T, int64_t d, int64_t E, int64_t k, int64_t h, int64_
     const int64_t nchunks_max = (n + 255) / 256;   // chunks are at least 256 slots
     L.status = take(sizeof(DevStatus));
     L.xnorm = take(4 * T);
-    L.wnorm = take(4 * E);
-    L.wpart = take(4 * (int64_t)route_split_parts((int)d) * Ep);
-    L.wsplit = take(2 * 3 * (int64_t)route_dpad((int)d) * Ep);
+    L.wnorm = take(4 * 2 * E);                                        // |W_r[:, e]|, |lo_e|
+    L.wpart = take(4 * 2 * (int64_t)route_split_parts((int)d) * Ep);
+    L.wexp = take(4 * (int64_t)route_split_parts((int)d) * Ep);
+    L.wsplit = take(2 * 2 * (int64_t)route_dpad((int)d) * Ep);
     L.wrt = take(4 * E * (int64_t)route_dpad((int)d));
     L.logits = take(4 * route_logits_rows(T, (int)d, (int)E) * Ep);
     L.fb_tokens = take(4 * T);
@@ -218,7 +217,7 @@ struct GemmSpec {
     int64_t zero_n;
     float* nrm_out;          // dense A: also nrm_out[r] = |A[r, 0:K_A]| (K_A = a_cols or K)
     const float* wn_part;    // dense A: also wn_out[e] = sqrt(sum_p wn_part[p wn_Ep + e])
-    int wn_nparts, wn_E, wn_Ep;
+    int wn_nparts, wn_E, wn_Ep, wn_sets;
     float* wn_out;
     const void* W2nd;        // groups g >= g_split: weights at W2nd + (g - g_split) w2_g_ld +
     int64_t w2_k_ld;         //   kk w2_k_ld + n (elements); W then holds g_split groups
@@ -281,11 +280,13 @@ moevie_status run_gemm(const GemmSpec& g, DevStatus* st, cudaStream_t s) {
         a.nrm_out = g.nrm_out;
     }
     if (g.wn_out) {
-        if (g.a_rows || g.wn_E <= 0 || g.wn_Ep < g.wn_E || g.wn_nparts < 1) return MOEVIE_ERR_UNSUPPORTED;
+        if (g.a_rows || g.wn_E <= 0 || g.wn_Ep < g.wn_E || g.wn_nparts < 1 || g.wn_sets < 1)
+            return MOEVIE_ERR_UNSUPPORTED;
         a.wn_part = g.wn_part;
         a.wn_nparts = g.wn_nparts;
         a.wn_E = g.wn_E;
         a.wn_Ep = g.wn_Ep;
+        a.wn_sets = g.wn_sets;
         a.wn_out = g.wn_out;
     }
     a.G = g.G;
@@ -319,9 +320,9 @@ moevie_status run_gemm(const GemmSpec& g, DevStatus* st, cudaStream_t s) {
     a.scale = g.scale;
     a.ksplit = g.ksplit > 1 ? g.ksplit : 1;
     if (a.ksplit > a.num_kb) return MOEVIE_ERR_UNSUPPORTED;
-    if (a.ksplit > 1 && g.epi != EPI_STORE_F32 && g.epi != EPI_ADD_F32 && g.epi != EPI_SUM3_F32)
+    if (a.ksplit > 1 && g.epi != EPI_STORE_F32 && g.epi != EPI_ADD_F32 && g.epi != EPI_SUM2_F32)
         return MOEVIE_ERR_UNSUPPORTED;
-    if (g.epi == EPI_SUM3_F32 && (g.N % 96 != 0 || g.N > GM_MAXBN)) return MOEVIE_ERR_UNSUPPORTED;
+    if (g.epi == EPI_SUM2_F32 && (g.N % 64 != 0 || g.N > GM_MAXBN)) return MOEVIE_ERR_UNSUPPORTED;
     a.y_split_stride = g.y_split_stride;
     a.status = st;
     a.limit_ns = WAIT_LIMIT_NS;
@@ -336,8 +337,8 @@ moevie_status run_gemm(const GemmSpec& g, DevStatus* st, cudaStream_t s) {
     return cuda_status(launch_grouped_gemm(a, grid, s));
 }
 
-// Router (Eqs. 1, 7, 4-5): exact bf16 split of W_r, tensor-core logits,
-// certified top-k with exact re-decision of near ties.
+// Router (Eqs. 1, 7, 4-5): bf16 pieces hi, mid of W_r, tensor-core logits x . (hi +
+// mid), certified top-k with exact re-decision of near ties.
 moevie_status route_impl(const void* x, const float* W_r, const float* b, int64_t T, int64_t d,
                          int64_t E, int64_t k, int32_t* idx, float* gate, const Layout& L,
                          void* ws, cudaStream_t s, bool logits_only = false,
@@ -351,7 +352,8 @@ moevie_status route_impl(const void* x, const float* W_r, const float* b, int64_
     // partial logits: ksplit arrays [T][Ep]; straight into logits_out when unsplit
     float* logits = (logits_out && ksplit == 1) ? logits_out : at<float>(ws, L.logits);
     const int64_t part_stride = T * Ep;
-    MV_TRY(launch_route_split(W_r, (int)d, (int)E, wsplit, wrt, at<float>(ws, L.wpart), st, s));
+    MV_TRY(launch_route_split(W_r, (int)d, (int)E, wsplit, wrt, at<float>(ws, L.wpart),
+                              at<int32_t>(ws, L.wexp), st, s));
     const int64_t dp = route_dpad((int)d);
     const bool cc = route_concat((int)E);
     GemmSpec g{};
@@ -362,14 +364,14 @@ moevie_status route_impl(const void* x, const float* W_r, const float* b, int64_
     g.m_total = T;
     g.G = 1;
     g.W = wsplit;
-    if (cc) {   // B [dp][3 Ep]: the three pieces side by side, summed by the epilogue
+    if (cc) {   // B [dp][2 Ep]: the two pieces side by side, summed by the epilogue
         g.K = (int)dp;
-        g.N = 3 * Ep;
-        g.N_ld = 3 * Ep;
-        g.epi = EPI_SUM3_F32;
-    } else {    // B [3][dp][Ep]: K = 3 dp, x read three times, once per piece
+        g.N = 2 * Ep;
+        g.N_ld = 2 * Ep;
+        g.epi = EPI_SUM2_F32;
+    } else {    // B [2][dp][Ep]: K = 2 dp, x read twice, once per piece
         g.a_kperiod = (int)dp;
-        g.K = (int)(3 * dp);
+        g.K = (int)(2 * dp);
         g.N = (int)E;
         g.N_ld = Ep;
         g.epi = EPI_STORE_F32;
@@ -380,14 +382,13 @@ moevie_status route_impl(const void* x, const float* W_r, const float* b, int64_
     g.scale = 1.0f;
     g.ksplit = ksplit;
     g.y_split_stride = part_stride;
-    g.zero = zero_acc;   // fp32 [T][d] cleared by the GEMM's idle warps (or NULL)
-    g.zero_n = T * d;
     g.nrm_out = logits_only ? nullptr : at<float>(ws, L.xnorm);   // |x_t| for the certificate
-    if (!logits_only) {   // |W_r[:, e]| for the certificate, from the split's partial sums
+    if (!logits_only) {   // |W_r[:, e]| and |lo_e| for the certificate, from the split's partial sums
         g.wn_part = at<float>(ws, L.wpart);
         g.wn_nparts = route_split_parts((int)d);
         g.wn_E = (int)E;
         g.wn_Ep = Ep;
+        g.wn_sets = 2;
         g.wn_out = wnorm;
     }
     moevie_status c = run_gemm(g, st, s);
@@ -398,9 +399,9 @@ moevie_status route_impl(const void* x, const float* W_r, const float* b, int64_
         return MOEVIE_OK;
     }
     MV_TRY(launch_route_select(static_cast<const __nv_bfloat16*>(x), wrt, b, logits, Ep, ksplit,
-                               part_stride, wnorm, (int)T, (int)d, (int)E, (int)k, idx, gate,
-                               at<int32_t>(ws, L.fb_tokens), at<float>(ws, L.xnorm), st,
-                               num_sms(), s));
+                               part_stride, wnorm, at<int32_t>(ws, L.wexp), (int)T, (int)d, (int)E,
+                               (int)k, idx, gate, at<int32_t>(ws, L.fb_tokens), at<float>(ws, L.xnorm),
+                               st, num_sms(), s, zero_acc, T * d));   // top-k also clears y's accumulator
     return MOEVIE_OK;
 }
 
@@ -706,8 +707,8 @@ static moevie_status forward_impl(const moevie_layer* Lr, const void* x, int64_t
     const int64_t n2 = T * k + S * T;
     MV_TRY(mark(0));
     // 1. router (Eqs. 1, 7, 4-5)
-    // unless a separate shared-expert GEMM writes it first, the router GEMM's idle
-    // warps also clear the y accumulator
+    // unless a separate shared-expert GEMM writes it first, the router's top-k kernel
+    // also clears the y accumulator (it leaves HBM mostly idle)
     if ((c = route_impl(x, Lr->W_r, Lr->b, T, d, E, k, idx, gate, L, ws, s, false, nullptr,
                         (hs > 0 && S == 0) ? nullptr : yacc)) != MOEVIE_OK)
         return c;

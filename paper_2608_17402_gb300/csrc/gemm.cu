@@ -620,41 +620,37 @@ __device__ void epilogue(const GemmArgs& p, const Smem& sm, uint32_t tmem, int64
         }
         tc_fence_after();
         const uint32_t tbase = tmem + ((uint32_t)(quad * 32) << 16) + (uint32_t)acc * GM_MAXBN;
-        if (ECLS == ECLS_F32 && p.epi == EPI_SUM3_F32) {
-            // three column groups of N / 3 (one n-tile): chunk ch of the output is the sum
-            // of accumulator chunks ch, ch + nc3, ch + 2 nc3, added in that order
-            const int nc3 = nchunk / 3;
-            if (half >= nc3) {
+        if (ECLS == ECLS_F32 && p.epi == EPI_SUM2_F32) {
+            // two column groups of N / 2 (one n-tile): chunk ch of the output is the sum of
+            // accumulator chunks ch and ch + nc2
+            const int nc2 = nchunk / 2;
+            if (half >= nc2) {
                 tc_fence_before();
                 __syncwarp();
                 if (lane == 0) mbar_arrive_remote(tempty_leader + 8 * acc);
             }
-            for (int ch = half; ch < nc3; ch += 2) {
+            for (int ch = half; ch < nc2; ch += 2) {
                 uint32_t v[32];
-                float s3[32];
+                float s2[32];
                 tmem_ld_32x32b_x32(tbase + ch * 32, v);
                 tmem_wait_ld();
 #pragma unroll
-                for (int i = 0; i < 32; ++i) s3[i] = __uint_as_float(v[i]);
-                tmem_ld_32x32b_x32(tbase + (ch + nc3) * 32, v);
+                for (int i = 0; i < 32; ++i) s2[i] = __uint_as_float(v[i]);
+                tmem_ld_32x32b_x32(tbase + (ch + nc2) * 32, v);
                 tmem_wait_ld();
-#pragma unroll
-                for (int i = 0; i < 32; ++i) s3[i] += __uint_as_float(v[i]);
-                tmem_ld_32x32b_x32(tbase + (ch + 2 * nc3) * 32, v);
-                tmem_wait_ld();
-                if (ch + 2 >= nc3) {   // this warp's last read of the accumulator
+                if (ch + 2 >= nc2) {   // this warp's last read of the accumulator
                     tc_fence_before();
                     __syncwarp();
                     if (lane == 0) mbar_arrive_remote(tempty_leader + 8 * acc);
                 }
                 if (!ok_row) continue;
 #pragma unroll
-                for (int i = 0; i < 32; ++i) s3[i] += __uint_as_float(v[i]);
+                for (int i = 0; i < 32; ++i) s2[i] += __uint_as_float(v[i]);
                 float* yrow = p.yacc + t.ks * p.y_split_stride + tok * p.ldy + ch * 32;
 #pragma unroll
                 for (int q = 0; q < 8; ++q)
                     *reinterpret_cast<float4*>(yrow + 4 * q) =
-                        make_float4(sc * s3[4 * q], sc * s3[4 * q + 1], sc * s3[4 * q + 2], sc * s3[4 * q + 3]);
+                        make_float4(sc * s2[4 * q], sc * s2[4 * q + 1], sc * s2[4 * q + 2], sc * s2[4 * q + 3]);
             }
             continue;
         }
@@ -881,16 +877,20 @@ __global__ void __launch_bounds__(GM_THREADS, 1) grouped_gemm_kernel(const __gri
                 }
             }
         }
-        // 2. Column norms from per-CTA partial sums of squares: one warp per column,
-        //    lanes over the parts, then a fixed shuffle tree (deterministic).
+        // 2. Column norms from per-CTA partial sums of squares (wn_sets sets of wn_nparts
+        //    parts): one warp per column, lanes over the parts, then a fixed shuffle tree
+        //    (deterministic).
         if (p.wn_out) {
             const int q = warp - GM_WARP_GATHER, lane = threadIdx.x & 31;
-            for (int e = blockIdx.x * GM_GATHER_WARPS + q; e < p.wn_E; e += gridDim.x * GM_GATHER_WARPS) {
+            for (int j = blockIdx.x * GM_GATHER_WARPS + q; j < p.wn_sets * p.wn_E;
+                 j += gridDim.x * GM_GATHER_WARPS) {
+                const int set = j / p.wn_E, e = j - set * p.wn_E;
+                const float* part = p.wn_part + (int64_t)set * p.wn_nparts * p.wn_Ep;
                 float v = 0.f;
-                for (int pp = lane; pp < p.wn_nparts; pp += 32) v += p.wn_part[(int64_t)pp * p.wn_Ep + e];
+                for (int pp = lane; pp < p.wn_nparts; pp += 32) v += part[(int64_t)pp * p.wn_Ep + e];
 #pragma unroll
                 for (int o = 16; o; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
-                if (lane == 0) p.wn_out[e] = sqrtf(v);
+                if (lane == 0) p.wn_out[j] = sqrtf(v);
             }
         }
         // 3. Clear another buffer (the y accumulator) with 16-byte stores, grid-strided
@@ -984,7 +984,7 @@ cudaError_t launch_grouped_gemm(const GemmArgs& a, int grid, cudaStream_t s) {
     Kern kern;
     if (gathered) kern = kerns[4];
     else if (a.epi == EPI_ADD_F32) kern = a.stg_rows == 32 ? kerns[0] : kerns[1];
-    else if (a.epi == EPI_STORE_F32 || a.epi == EPI_SUM3_F32) kern = kerns[2];
+    else if (a.epi == EPI_STORE_F32 || a.epi == EPI_SUM2_F32) kern = kerns[2];
     else kern = kerns[3];
     static bool attr_set[64] = {};
     int dev = 0;

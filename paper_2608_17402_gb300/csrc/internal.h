@@ -51,9 +51,14 @@ cudaError_t launch_pdl_coop(void (*kern)(KArgs...), dim3 grid, dim3 block, size_
 
 // ----------------------------------------------------------------- router
 
-// Error model of the fast (tensor-core, fp32-accumulated) logits used to decide
-// when a token's selection must be re-decided with exact logits:
-//   |s_fast[t, e] - s[t, e]| <= ROUTE_TAU_C * 2^-24 * |x_t| * |W_r[:, e]|.
+// Error model of the fast logits used to decide when a token's selection must be
+// re-decided with exact logits.  The fast logits are x . (hi + mid), two bf16 pieces of
+// W_r = hi + mid + lo (lo, the last 8 significand bits, is left out), on the tensor
+// cores with fp32 accumulation:
+//   |s_fast[t, e] - s[t, e]| <= |x_t| (ROUTE_TAU_C 2^-24 (|W_r[:, e]| + |lo_e|) + |lo_e|).
+// The |x_t| |lo_e| term bounds the left-out piece (Cauchy-Schwarz, rigorous); the first
+// term is the accumulation error, whose constant is fixed by measurement (the tensor
+// cores' accumulation order is undocumented).
 constexpr float ROUTE_TAU_C = 128.0f;
 // Extra allowance, in key units, for the fp32 evaluation of sigmoid(s) + b.
 constexpr float ROUTE_KEY_SLACK = 2e-6f;
@@ -63,26 +68,29 @@ inline int route_epad(int E) { return (E + 31) / 32 * 32; }
 // Rows of each W_r piece: d rounded up to 64 (zero rows), so that no 64-wide K block
 // of the router GEMM straddles two pieces.
 inline int route_dpad(int d) { return (d + 63) / 64 * 64; }
-// The router GEMM's B holds the three bf16 pieces of W_r side by side along N
-// ([d_pad][3 E_pad]: x is read once, the epilogue sums the pieces) when they fit one
-// n-tile; otherwise one after another along K ([3][d_pad][E_pad], x read per piece).
-inline bool route_concat(int E) { return 3 * route_epad(E) <= 256; }   // 256: largest MMA N
+// The router GEMM's B holds the two bf16 pieces hi, mid of W_r side by side along N
+// ([d_pad][2 E_pad]: x is read once, the epilogue sums the pieces) when they fit one
+// n-tile; otherwise one after another along K ([2][d_pad][E_pad], x read per piece).
+inline bool route_concat(int E) { return 2 * route_epad(E) <= 256; }   // 256: largest MMA N
 
-// W_r fp32 [d, E] -> three bf16 pieces [3][d_pad][E_pad] with W_r = hi + mid + lo
-// exactly (zero in the padding rows and columns), the transposed fp32 copy
-// wrt [E][d_pad] (zero rows past d), and per-CTA partial sums of squares of W_r's
-// columns (wpart: route_split_parts(d) x E_pad floats; |W_r[:, e]| is the square root
-// of their sum over the parts).  Also clears the fallback counter in st (may be NULL).
+// W_r fp32 [d, E] -> the bf16 pieces hi = bf16(w), mid = bf16(w - hi) (W_r = hi + mid +
+// lo exactly, lo = w - hi - mid; zero in the padding rows and columns), the transposed
+// fp32 copy wrt [E][d_pad] (zero rows past d), and per-CTA partial sums of squares of
+// W_r's columns and of lo's columns (wpart: two sets of route_split_parts(d) x E_pad
+// floats; |W_r[:, e]| and |lo_e| are the square roots of their sums over the parts).
+// It also writes each CTA's largest exponent field of each column (wexp:
+// route_split_parts(d) x E_pad ints, at least 1), which sets the exact re-decision's
+// accumulator window.  Also clears the fallback counter in st (may be NULL).
 int route_split_parts(int d);
 cudaError_t launch_route_split(const float* Wr, int d, int E, __nv_bfloat16* Wsplit, float* wrt,
-                               float* wpart, DevStatus* st, cudaStream_t s);
+                               float* wpart, int32_t* wexp, DevStatus* st, cudaStream_t s);
 
 // Splits of K for the router GEMM: enough CTA-pair work items for about
 // ROUTE_SPLIT_TARGET items (ROUTE_SPLIT_TARGET_CONCAT with the pieces side by side),
 // at most ROUTE_MAX_KSPLIT, at least three K blocks each.
 // Depends on the sizes only (the workspace size uses it).
 constexpr int ROUTE_SPLIT_TARGET = 76;
-constexpr int ROUTE_SPLIT_TARGET_CONCAT = 64;   // the same with the pieces side by side (E <= 64)
+constexpr int ROUTE_SPLIT_TARGET_CONCAT = 64;   // the same with the pieces side by side (E <= 128)
 constexpr int ROUTE_MAX_KSPLIT = 16;
 int route_ksplit(int64_t T, int d, int E);
 // Rows of partial-logit storage: an upper bound of route_ksplit(T) * T that is
@@ -93,15 +101,19 @@ int64_t route_logits_rows(int64_t T, int d, int E);
 cudaError_t launch_route_sum_parts(const float* logits, int64_t part_stride, int nparts, int64_t n,
                                    float* out, cudaStream_t s);
 
-// Keys, warp top-k with a certificate, gates; uncertified tokens are re-decided
-// with exact logits (integer long accumulator) of the experts near their boundary.  logits: nparts
-// partial arrays [T][ld] (part_stride floats apart); part 0 is overwritten with the
-// sum for uncertified tokens.
+// Keys, warp top-k with a certificate, gates; uncertified tokens are listed in
+// fb_tokens and re-decided by a second kernel with exact logits (integer long
+// accumulator) of the experts near their boundary.  wnorm: |W_r[:, e]| [E] then |lo_e|
+// [E] (the error model above); wexp: the split kernel's largest exponent fields.  The
+// top-k kernel also clears zero[0, zero_n) (16-byte aligned, zero_n % 4 == 0; NULL:
+// nothing).  logits: nparts partial arrays [T][ld] (part_stride floats apart); part 0 is
+// overwritten with the sum for uncertified tokens.
 cudaError_t launch_route_select(const __nv_bfloat16* x, const float* wrt, const float* b,
                                 float* logits, int ld, int nparts, int64_t part_stride,
-                                const float* wnorm, int T, int d, int E, int k, int32_t* idx,
-                                float* gate, int32_t* fb_tokens, float* xnorm, DevStatus* st,
-                                int num_sms, cudaStream_t s);
+                                const float* wnorm, const int32_t* wexp, int T, int d, int E, int k,
+                                int32_t* idx, float* gate, int32_t* fb_tokens, float* xnorm,
+                                DevStatus* st, int num_sms, cudaStream_t s, float* zero = nullptr,
+                                int64_t zero_n = 0);
 
 // ---------------------------------------------------------------- permute
 
@@ -190,12 +202,12 @@ enum Epilogue : int {
     EPI_SWIGLU_BF16 = 5, // out[r, n] = bf16(SiLU(acc[gate n]) * acc[up n]): accumulator columns
                          //   0..127 from W1 (gate, the pair's first CTA's B half), 128..255 from
                          //   W3 (up, the second CTA's); 128 output columns per n-tile
-    EPI_SUM3_F32 = 4,    // yacc[tok(r), n]  = scale(r) * ((acc[n] + acc[n + N/3]) + acc[n + 2N/3]),
-                         //   n < N/3 (three column groups summed in a fixed order; one n-tile)
+    EPI_SUM2_F32 = 4,    // yacc[tok(r), n]  = scale(r) * (acc[n] + acc[n + N/2]), n < N/2
+                         //   (two column groups summed; one n-tile)
 };
 static_assert(EPI_ADD_F32 == 2, "gm_stages / gm_smem_bytes test the reduction epilogue by value");
 // Epilogue classes of the grouped GEMM's kernel instances: bf16 outputs (GELU, SwiGLU,
-// plain), fp32 stores (plain, three-group sums), fp32 reductions into the accumulator.
+// plain), fp32 stores (plain, two-group sums), fp32 reductions into the accumulator.
 enum { ECLS_BF16 = 0, ECLS_F32 = 1, ECLS_ADD = 2 };
 
 struct GemmArgs {
@@ -242,9 +254,10 @@ struct GemmArgs {
     int64_t nrm_ld;             //   every n-tile-0 item, nrm_out[r] = |nrm_x[r, 0:nrm_cols]|
     int nrm_cols;               //   (nrm_cols % 8 == 0)
     float* nrm_out;
-    const float* wn_part;       // dense A only: the idle gather warps also write
-    int wn_nparts, wn_E, wn_Ep; //   wn_out[e] = sqrt(sum_p wn_part[p wn_Ep + e]), e < wn_E
-    float* wn_out;              //   (the router's |W_r[:, e]| from per-CTA partial sums)
+    const float* wn_part;       // dense A only: the idle gather warps also write, for each set
+    int wn_nparts, wn_E, wn_Ep; //   q < wn_sets and e < wn_E, wn_out[q wn_E + e] =
+    int wn_sets;                //   sqrt(sum_p wn_part[(q wn_nparts + p) wn_Ep + e])
+    float* wn_out;              //   (the router's |W_r[:, e]| and |lo_e| from per-CTA partial sums)
     DevStatus* status;
     uint64_t limit_ns;
 };

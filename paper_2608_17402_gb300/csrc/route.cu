@@ -1,31 +1,34 @@
 // route.cu -- router of the MoE-ViE layer (Eqs. 1, 7, 4-5), sm_103a.
 //
 // The logits s = x . W_r run on the tensor cores (grouped_gemm_kernel, one dense
-// group): W_r is split exactly into three bf16 pieces, W_r = hi + mid + lo, and
-// the GEMM accumulates x . [hi; mid; lo] over K = 3 d_pad in fp32 (each piece padded
-// to a multiple of 64 rows with zeros).  Every product of a
-// bf16 x and a bf16 piece is exact in fp32, so the only error is the fp32
-// accumulation.  When there are few tokens, K is split over several CTA pairs
-// (route_ksplit) and each split writes its own fp32 partial logits; they are summed
+// group): W_r is split exactly into bf16 pieces, W_r = hi + mid + lo, and the GEMM
+// accumulates the fast logits x . (hi + mid) in fp32 (each piece padded to a multiple of
+// 64 rows with zeros; for E <= 128 the two pieces sit side by side along N and the
+// epilogue adds them, otherwise one after another along K).  Every product of a bf16 x
+// and a bf16 piece is exact in fp32, so the error is the fp32 accumulation plus the
+// left-out x . lo, which Cauchy-Schwarz bounds by |x_t| |lo_e| (lo holds the last 8 of
+// w's 24 significand bits).  When there are few tokens, K is split over several CTA
+// pairs (route_ksplit) and each split writes its own fp32 partial logits; they are summed
 // in a fixed order.  This file holds the steps around that GEMM:
 //
-//  1. route_split_kernel: the three pieces, an fp32 copy of W_r transposed to
+//  1. route_split_kernel: the two pieces, an fp32 copy of W_r transposed to
 //     [E][d_pad] (read by the exact re-decision), and per-CTA partial sums of squares
-//     of W_r's columns (the router GEMM's idle warps finish |W_r[:, e]| from them).
+//     of W_r's columns and of lo's (the router GEMM's idle warps finish |W_r[:, e]| and
+//     |lo_e| from them).
 //  2. route_topk_kernel: one warp per token; the partial logits summed, keys
 //     sigmoid(s) + b, k rounds of warp arg-max (ties to the lower id), and a
 //     certificate.  Every expert's key lies in
-//     [key_e - tau_e, key_e + tau_e]; tau_e is the logit error bound
-//     (ROUTE_TAU_C 2^-24 |x_t| |W_r[:, e]|) times the largest sigmoid slope inside
-//     the logit interval, plus fp32 evaluation slack.  The selection is certain when
-//     the lowest selected lower end is above the highest unselected upper end (tried
-//     first with the slope bound 1/4, then with the exact slope).  Certified tokens
-//     write ascending ids and gates sigmoid(s) / sum (the bias only selects).
+//     [key_e - tau_e, key_e + tau_e]; tau_e is the logit error bound (logit_tau) times
+//     the largest sigmoid slope inside the logit interval, plus fp32 evaluation slack.
+//     The selection is certain when the lowest selected lower end is above the highest
+//     unselected upper end (tried first with the slope bound 1/4, then with the exact
+//     slope).  Certified tokens write ascending ids and gates sigmoid(s) / sum (the bias
+//     only selects).
 //  3. route_fallback_kernel: one CTA per uncertified token.  An expert is surely in
 //     when its lower end is above the k-th largest upper end of the others, surely
 //     out when its upper end is below the k-th largest lower end; the rest get exact
 //     logits (each product of a bf16 and an fp32 value is an integer of at most 32 bits
-//     times a power of two; the block sums them in a 128-bit fixed-point accumulator on
+//     times a power of two; the CTA sums them in 128-bit fixed-point accumulators on
 //     the integer pipes, see long_acc_term), and the remaining places are filled from
 //     their keys (fp64), ties to the lower id.
 #include <math.h>
@@ -39,48 +42,59 @@ namespace {
 constexpr int SPLIT_TILE = 32;    // W_r rows (and experts) per CTA of the split kernel
 
 // CTA (bx, by): experts 32 bx .. +31 and rows 32 by .. +31 of W_r (rows past d are
-// zero); 32 x 8 threads.  Writes the three bf16 pieces, the transposed fp32 copy and
-// the CTA's partial sums of w^2 per expert.
+// zero); 32 x 8 threads.  Writes the two bf16 pieces hi, mid, the transposed fp32 copy
+// and the CTA's partial sums of w^2 and of lo^2 per expert (lo = w - hi - mid, the
+// piece the fast logits leave out).
 __global__ void __launch_bounds__(256) route_split_kernel(const float* __restrict__ Wr, int d,
                                                           int dp, int E, int Ep,
                                                           __nv_bfloat16* __restrict__ Wsplit,
                                                           float* __restrict__ wrt,
-                                                          float* __restrict__ wpart, DevStatus* st,
-                                                          int concat) {
+                                                          float* __restrict__ wpart, int parts,
+                                                          int32_t* __restrict__ wexp,
+                                                          DevStatus* st, int concat) {
     pdl_wait();
     if (st && blockIdx.x == 0 && blockIdx.y == 0 && threadIdx.x == 0) st->fb_count = 0;
     __shared__ float tile[SPLIT_TILE][SPLIT_TILE + 1];
-    __shared__ float red[8][32];
+    __shared__ float red[2][8][32];
+    __shared__ int redx[8][32];
     const int tx = threadIdx.x & 31, ty = threadIdx.x >> 5;
     const int e = blockIdx.x * SPLIT_TILE + tx;
     const int i0 = blockIdx.y * SPLIT_TILE;
-    // piece p of element (i, e): [p][dp][Ep] (along K), or [dp][3 Ep] (side by side along N)
+    // piece p of element (i, e): [p][dp][Ep] (along K), or [dp][2 Ep] (side by side along N)
     const size_t piece = concat ? (size_t)Ep : (size_t)dp * Ep;
-    const size_t row = concat ? (size_t)3 * Ep : (size_t)Ep;
-    float sq = 0.f;
+    const size_t row = concat ? (size_t)2 * Ep : (size_t)Ep;
+    float sq = 0.f, sql = 0.f;
+    int ex = 1;   // largest exponent field (subnormals and zero count as 1)
 #pragma unroll
     for (int r = ty; r < SPLIT_TILE; r += 8) {
         const int i = i0 + r;
         const float w = (e < E && i < d) ? Wr[(int64_t)i * E + e] : 0.f;
+        ex = max(ex, (int)((__float_as_uint(w) >> 23) & 0xffu));
+        const __nv_bfloat16 hi = __float2bfloat16_rn(w);
+        const float r1 = w - __bfloat162float(hi);                 // exact
+        const __nv_bfloat16 mid = __float2bfloat16_rn(r1);
+        const float lo = r1 - __bfloat162float(mid);               // exact
         if (e < Ep) {
-            const __nv_bfloat16 hi = __float2bfloat16_rn(w);
-            const float r1 = w - __bfloat162float(hi);          // exact
-            const __nv_bfloat16 mid = __float2bfloat16_rn(r1);
-            const __nv_bfloat16 lo = __float2bfloat16_rn(r1 - __bfloat162float(mid));   // exact
             const size_t o = (size_t)i * row + e;
             Wsplit[o] = hi;
             Wsplit[piece + o] = mid;
-            Wsplit[2 * piece + o] = lo;
         }
         tile[r][tx] = w;
         sq = fmaf(w, w, sq);
+        sql = fmaf(lo, lo, sql);
     }
-    red[ty][tx] = sq;
+    red[0][ty][tx] = sq;
+    red[1][ty][tx] = sql;
+    redx[ty][tx] = ex;
     __syncthreads();
-    if (ty == 0 && e < Ep) {
+    if (ty < 2 && e < Ep) {
         float v = 0.f;
-        for (int q = 0; q < 8; ++q) v += red[q][tx];
-        wpart[(int64_t)blockIdx.y * Ep + e] = v;
+        for (int q = 0; q < 8; ++q) v += red[ty][q][tx];
+        wpart[((int64_t)ty * parts + blockIdx.y) * Ep + e] = v;
+    } else if (ty == 2 && e < Ep) {
+        int m = 1;
+        for (int q = 0; q < 8; ++q) m = max(m, redx[q][tx]);
+        wexp[(int64_t)blockIdx.y * Ep + e] = m;
     }
 #pragma unroll
     for (int r = ty; r < SPLIT_TILE; r += 8) {
@@ -98,9 +112,13 @@ __device__ __forceinline__ float sigmoid_fast(float v) {
     return __fdividef(1.0f, 1.0f + __expf(-v));
 }
 
-// Logit error bound of expert e for a token: ROUTE_TAU_C 2^-24 |x_t| |W_r[:, e]|.
-__device__ __forceinline__ float logit_tau(float xn, float wn) {
-    return ROUTE_TAU_C * 5.9604645e-8f * xn * wn;
+// Logit error bound of expert e for a token (internal.h): the accumulation error
+// ROUTE_TAU_C 2^-24 |x_t| (|W_r[:, e]| + |lo_e|) plus the left-out piece |x_t| |lo_e|,
+// rounded up by the factor 1.001: the norms are fp32 sums of squares along chains far
+// shorter than 2^14 terms, so their relative error (and that of the few operations
+// here) stays below 2^-10.
+__device__ __forceinline__ float logit_tau(float xn, float wn, float wl) {
+    return (ROUTE_TAU_C * 5.9604645e-8f * (wn + wl) + wl) * xn * 1.001f;
 }
 
 // Key half-width with the largest sigmoid slope inside [s - tau_s, s + tau_s]
@@ -123,17 +141,117 @@ __device__ __forceinline__ uint32_t ord_f32(float f) {
     return u ^ ((u & 0x80000000u) ? 0xffffffffu : 0x80000000u);
 }
 
+__device__ __forceinline__ float from_ord_f32(uint32_t c) {
+    return __uint_as_float(c ^ ((c & 0x80000000u) ? 0x80000000u : 0xffffffffu));
+}
+
+// k-th and (k+1)-th largest of v over the warp, counting equal values separately
+// (k or k + 1 rounds: warp maximum of the order codes by redux.sync, then one holder
+// of that maximum leaves; k <= E).
+template <int NPL>
+__device__ __forceinline__ void warp_kth_values(const float (&v)[NPL], int E, int k, int lane,
+                                                float& kth, float& kth1) {
+    uint32_t code[NPL];
+#pragma unroll
+    for (int i = 0; i < NPL; ++i) code[i] = (lane + 32 * i < E) ? ord_f32(v[i]) : 0u;
+    uint32_t used = 0;
+    kth = -INFINITY;
+    kth1 = -INFINITY;
+    const int rounds = k < E ? k + 1 : k;
+    for (int j = 0; j < rounds; ++j) {
+        uint32_t best = 0;
+#pragma unroll
+        for (int i = 0; i < NPL; ++i) {
+            const uint32_t c = ((used >> i) & 1u) ? 0u : code[i];
+            best = c > best ? c : best;
+        }
+        best = __reduce_max_sync(0xffffffffu, best);
+#pragma unroll
+        for (int i = 0; i < NPL; ++i) {
+            const uint32_t m = __ballot_sync(0xffffffffu, !((used >> i) & 1u) && code[i] == best);
+            if (m) {
+                if (lane == __ffs(m) - 1) used |= 1u << i;
+                break;
+            }
+        }
+        const float bv = from_ord_f32(best);
+        if (j == k - 1) kth = bv;
+        if (j == k) kth1 = bv;
+    }
+}
+
+// Exact logits by a long fixed-point accumulator (the exact dot product of Kulisch
+// and Miranker, with a window fitted to the operands).  A bf16 x_i is mx 2^(ex - 134)
+// and an fp32 w_i is mw 2^(ew - 150) (mx < 2^8, mw < 2^24 integers; ex, ew the biased
+// exponents, 1 for subnormals), so x_i w_i = P 2^(q - 284) with the integer P = mx mw
+// < 2^32 and q = ex + ew.  With a window Q >= every q, the term is P 2^(64 - (Q - q))
+// units of 2^(Q - 348): a left shift (exact) when Q - q <= 64, else a right shift that
+// drops less than one unit.  The units of d terms sum in a 128-bit integer (|sum| <
+// 2^120 for d < 2^24), exactly and in any order; the logit is that sum times
+// 2^(Q - 348), within d 2^(Q - 348) + 2^-51 |s| of the exact value.  Everything but the
+// final conversion runs on the integer pipes.
+__device__ __forceinline__ int bf16_exp_field(uint32_t hx) { return (int)((hx >> 7) & 0xffu); }
+__device__ __forceinline__ int f32_exp_field(uint32_t uw) { return (int)((uw >> 23) & 0xffu); }
+
+// acc += x w in units of 2^(Q - 348) (hx: bf16 bits of x, uw: fp32 bits of w).
+__device__ __forceinline__ void long_acc_term(uint32_t hx, uint32_t uw, int Q, unsigned __int128& acc) {
+    const int ex = bf16_exp_field(hx), ew = f32_exp_field(uw);
+    const uint64_t mx = (hx & 0x7fu) | (ex ? 0x80u : 0u);
+    const uint64_t mw = (uw & 0x7fffffu) | (ew ? 0x800000u : 0u);
+    const uint64_t P = mx * mw;
+    const int sh = 64 - (Q - (max(ex, 1) + max(ew, 1)));   // <= 64
+    unsigned __int128 t;
+    if (sh >= 0) t = (unsigned __int128)P << sh;
+    else t = sh > -64 ? (unsigned __int128)(P >> -sh) : (unsigned __int128)0;
+    if ((hx ^ (uw >> 16)) & 0x8000u) acc -= t;
+    else acc += t;
+}
+
+__device__ __forceinline__ unsigned __int128 warp_sum_u128(unsigned __int128 v) {
+#pragma unroll
+    for (int o = 16; o; o >>= 1) {
+        const uint64_t lo = __shfl_xor_sync(0xffffffffu, (unsigned long long)(uint64_t)v, o);
+        const uint64_t hi = __shfl_xor_sync(0xffffffffu, (unsigned long long)(uint64_t)(v >> 64), o);
+        v += ((unsigned __int128)hi << 64) | lo;
+    }
+    return v;
+}
+
+// The signed 128-bit sum `u` (two's complement) times 2^(Q - 348), in double: the
+// magnitude's two 64-bit words are rounded and added (relative error below 3 2^-53).
+__device__ __forceinline__ double long_acc_value(unsigned __int128 u, int Q) {
+    const bool neg = (long long)(uint64_t)(u >> 64) < 0;
+    const unsigned __int128 m = neg ? (unsigned __int128)0 - u : u;
+    const double hi = (double)(unsigned long long)(uint64_t)(m >> 64);
+    const double lo = (double)(unsigned long long)(uint64_t)m;
+    const double v = fma(hi, 18446744073709551616.0, lo);   // hi 2^64 + lo
+    // 2^(Q - 348) with 2 <= Q <= 508: a normal double, so the product is exact
+    const double r = v * __longlong_as_double((long long)((uint64_t)(Q - 348 + 1023) << 52));
+    return neg ? -r : r;
+}
+
 // One warp per token.  NPL = experts per lane (expert e sits in lane e % 32, slot e / 32).
 // s holds nparts partial logit arrays, part p at s + p * part_stride.  Each of the k
 // selection rounds takes the warp maximum of the keys' order codes (redux.sync) and
 // then the lowest id holding it (ballots in slot order), so ties go to the lower id.
+// A token the certificate cannot settle is listed for route_fallback_kernel.
 template <int NPL>
 __global__ void __launch_bounds__(256) route_topk_kernel(
     const __nv_bfloat16* __restrict__ x, float* __restrict__ s, int ld, int nparts,
     int64_t part_stride, const float* __restrict__ b, const float* __restrict__ wnorm, int T,
     int d, int E, int k, int32_t* __restrict__ idx, float* __restrict__ gate,
-    const float* __restrict__ xnorm, int32_t* __restrict__ fb_tokens, DevStatus* st) {
+    const float* __restrict__ xnorm, int32_t* __restrict__ fb_tokens, DevStatus* st,
+    float4* __restrict__ zero, int64_t zero_n4) {
     pdl_wait();
+    // Side job: clear another buffer (the layer's fp32 y accumulator) with 16-byte
+    // evict-first stores, grid-strided; this kernel leaves HBM mostly idle.
+    if (zero) {
+        const uint4 z = make_uint4(0u, 0u, 0u, 0u);
+        const uint64_t pol = l2_policy_evict_first();
+        for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < zero_n4;
+             i += (int64_t)gridDim.x * blockDim.x)
+            st_global_v4_hint(zero + i, z, pol);
+    }
     const int lane = threadIdx.x & 31;
     const int t = (int)(((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5);
     if (t >= T) return;
@@ -160,7 +278,7 @@ __global__ void __launch_bounds__(256) route_topk_kernel(
         if (e < E) {
             sg[i] = sigmoid_fast(sv[i]);
             key[i] = sg[i] + b[e];
-            ts[i] = logit_tau(xn, wnorm[e]);
+            ts[i] = logit_tau(xn, wnorm[e], wnorm[E + e]);
             code[i] = ord_f32(key[i]);
         } else {
             sg[i] = 0.f;
@@ -234,131 +352,63 @@ __global__ void __launch_bounds__(256) route_topk_kernel(
     }
 }
 
-__device__ __forceinline__ float from_ord_f32(uint32_t c) {
-    return __uint_as_float(c ^ ((c & 0x80000000u) ? 0x80000000u : 0xffffffffu));
-}
 
-// k-th and (k+1)-th largest of v over the warp, counting equal values separately
-// (k or k + 1 rounds: warp maximum of the order codes by redux.sync, then one holder
-// of that maximum leaves; k <= E).
+// Exact re-decision of uncertified tokens, one CTA (8 warps) per token.  The CTA stages
+// the token's x row in shared memory (16-byte loads) and finds its largest exponent
+// field; warp 0 bounds the keys and lists the candidates; then the candidates' exact
+// logits are formed FB_BATCH at a time by all 256 threads (threads over the d terms,
+// one long accumulator per candidate and thread, then a warp sum and a sum over the 8
+// warps, all exact), their keys in fp64; finally warp 0 fills the remaining places from
+// the exact keys, ties to the lower id, and writes ids and gates.
+//
+// The window of candidate e is Q = qx + qw(e), qx the largest exponent field of x_t and
+// qw(e) that of W_r[:, e] (both at least 1: subnormals and zeros count as exponent 1), so
+// every term's q is at most Q and one pass over the terms suffices; the logit is within
+// d 2^(Q - 348) + 2^-51 |s| of the exact value, and d 2^(Q - 348) <= d 2^-64
+// |x_t|_inf |W_r[:, e]|_inf.  A non-finite x_t or column (exponent field 255) gives a
+// NaN logit.
+constexpr int FB_BATCH = 4;       // candidates per pass over the terms
+constexpr int FB_X_SMEM = 16384;  // largest d whose x row is staged in shared memory
 template <int NPL>
-__device__ __forceinline__ void warp_kth_values(const float (&v)[NPL], int E, int k, int lane,
-                                                float& kth, float& kth1) {
-    uint32_t code[NPL];
-#pragma unroll
-    for (int i = 0; i < NPL; ++i) code[i] = (lane + 32 * i < E) ? ord_f32(v[i]) : 0u;
-    uint32_t used = 0;
-    kth = -INFINITY;
-    kth1 = -INFINITY;
-    const int rounds = k < E ? k + 1 : k;
-    for (int j = 0; j < rounds; ++j) {
-        uint32_t best = 0;
-#pragma unroll
-        for (int i = 0; i < NPL; ++i) {
-            const uint32_t c = ((used >> i) & 1u) ? 0u : code[i];
-            best = c > best ? c : best;
-        }
-        best = __reduce_max_sync(0xffffffffu, best);
-#pragma unroll
-        for (int i = 0; i < NPL; ++i) {
-            const uint32_t m = __ballot_sync(0xffffffffu, !((used >> i) & 1u) && code[i] == best);
-            if (m) {
-                if (lane == __ffs(m) - 1) used |= 1u << i;
-                break;
-            }
-        }
-        const float bv = from_ord_f32(best);
-        if (j == k - 1) kth = bv;
-        if (j == k) kth1 = bv;
-    }
-}
-
-// Exact logits by a long fixed-point accumulator (the exact dot product of Kulisch
-// and Miranker, with a window fitted to the operands).  A bf16 x_i is mx 2^(ex - 134)
-// and an fp32 w_i is mw 2^(ew - 150) (mx < 2^8, mw < 2^24 integers; ex, ew the biased
-// exponents, 1 for subnormals), so x_i w_i = P 2^(q - 284) with the integer P = mx mw
-// < 2^32 and q = ex + ew.  With Q >= every q, the term is P 2^(64 - (Q - q)) units of
-// 2^(Q - 348): a left shift (exact) when Q - q <= 64, else a right shift that drops less
-// than one unit.  The units of d terms sum in a 128-bit integer (|sum| < 2^120 for
-// d < 2^24), exactly and in any order; the logit is that sum times 2^(Q - 348), within
-// d 2^(Q - 348) + 2^-51 |s| of the exact value.  Q is the largest q of the candidate's
-// terms (zeros counted with their exponent fields); when that term is not zero its P is
-// at least 1, so d 2^(Q - 348) <= d 2^-64 sum|x_i w_i|, below the d 2^-53 sum|x_i w_i|
-// of an fp64 sum.  Everything but the final conversion runs on the integer pipes.
-constexpr int FB_CB = 32;   // candidates per batch (one per lane of the finishing warp)
-
-__device__ __forceinline__ int bf16_exp_field(uint32_t hx) { return (int)((hx >> 7) & 0xffu); }
-__device__ __forceinline__ int f32_exp_field(uint32_t uw) { return (int)((uw >> 23) & 0xffu); }
-
-// q of the term x w (subnormals as exponent 1), plus 1024 when x or w is not finite.
-__device__ __forceinline__ int long_acc_q(uint32_t hx, uint32_t uw) {
-    const int ex = bf16_exp_field(hx), ew = f32_exp_field(uw);
-    return max(ex, 1) + max(ew, 1) + ((ex == 255 || ew == 255) ? 1024 : 0);
-}
-
-// acc += x w in units of 2^(Q - 348) (hx: bf16 bits of x, uw: fp32 bits of w).
-__device__ __forceinline__ void long_acc_term(uint32_t hx, uint32_t uw, int Q, unsigned __int128& acc) {
-    const int ex = bf16_exp_field(hx), ew = f32_exp_field(uw);
-    const uint64_t mx = (hx & 0x7fu) | (ex ? 0x80u : 0u);
-    const uint64_t mw = (uw & 0x7fffffu) | (ew ? 0x800000u : 0u);
-    const uint64_t P = mx * mw;
-    const int sh = 64 - (Q - (max(ex, 1) + max(ew, 1)));   // <= 64
-    unsigned __int128 t;
-    if (sh >= 0) t = (unsigned __int128)P << sh;
-    else t = sh > -64 ? (unsigned __int128)(P >> -sh) : (unsigned __int128)0;
-    if ((hx ^ (uw >> 16)) & 0x8000u) acc -= t;
-    else acc += t;
-}
-
-__device__ __forceinline__ unsigned __int128 warp_sum_u128(unsigned __int128 v) {
-#pragma unroll
-    for (int o = 16; o; o >>= 1) {
-        const uint64_t lo = __shfl_xor_sync(0xffffffffu, (unsigned long long)(uint64_t)v, o);
-        const uint64_t hi = __shfl_xor_sync(0xffffffffu, (unsigned long long)(uint64_t)(v >> 64), o);
-        v += ((unsigned __int128)hi << 64) | lo;
-    }
-    return v;
-}
-
-// The signed 128-bit sum `u` (two's complement) times 2^(Q - 348), in double: the
-// magnitude's two 64-bit words are rounded and added (relative error below 3 2^-53).
-__device__ __forceinline__ double long_acc_value(unsigned __int128 u, int Q) {
-    const bool neg = (long long)(uint64_t)(u >> 64) < 0;
-    const unsigned __int128 m = neg ? (unsigned __int128)0 - u : u;
-    const double hi = (double)(unsigned long long)(uint64_t)(m >> 64);
-    const double lo = (double)(unsigned long long)(uint64_t)m;
-    const double v = fma(hi, 18446744073709551616.0, lo);   // hi 2^64 + lo
-    // 2^(Q - 348) with 2 <= Q <= 508: a normal double, so the product is exact
-    const double r = v * __longlong_as_double((long long)((uint64_t)(Q - 348 + 1023) << 52));
-    return neg ? -r : r;
-}
-
-// Exact re-decision of uncertified tokens, one CTA (8 warps) per token.  Warp 0
-// bounds the keys and lists the candidates; then all 256 threads form the candidates'
-// logits in the long accumulator (threads over d, reading the transposed fp32 copy of
-// W_r), and warp 0 fills the remaining places from the exact keys and writes ids and
-// gates.
-template <int NPL>
-__global__ void __launch_bounds__(256, 1) route_fallback_kernel(
+__global__ void __launch_bounds__(256) route_fallback_kernel(
     const __nv_bfloat16* __restrict__ x, const float* __restrict__ wrt, int dp,
+    const int32_t* __restrict__ wexp, int wexp_parts, int Ep,
     const float* __restrict__ b, const float* __restrict__ s, int ld,
     const float* __restrict__ xnorm, const float* __restrict__ wnorm, int d, int E, int k,
     int32_t* __restrict__ idx, float* __restrict__ gate, const int32_t* __restrict__ fb_tokens,
     DevStatus* st) {
     pdl_wait();
+    extern __shared__ __align__(16) uint16_t fb_x[];   // the token's x row when d <= FB_X_SMEM
     __shared__ int s_cand[32 * NPL];
     __shared__ double s_key[32 * NPL];
+    __shared__ unsigned long long s_acc[8][FB_BATCH][2];
+    __shared__ int s_q[FB_BATCH];
     __shared__ int s_ncand;
-    __shared__ int s_qmax[FB_CB];                 // largest term q of each batched candidate
-    __shared__ unsigned long long s_acc[2][8][FB_CB];   // per-warp sums: low, high words
+    __shared__ int s_qx;
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const uint32_t lt = (1u << lane) - 1u;
-    if (threadIdx.x < FB_CB) s_qmax[threadIdx.x] = 2;
-    __syncthreads();
     const int nfb = st->fb_count;
+    const bool staged = d <= FB_X_SMEM;
     for (int f = blockIdx.x; f < nfb; f += gridDim.x) {
         const int t = fb_tokens[f];
-        const uint16_t* xh = reinterpret_cast<const uint16_t*>(x) + (int64_t)t * d;
+        const uint16_t* xg = reinterpret_cast<const uint16_t*>(x) + (int64_t)t * d;
+        if (threadIdx.x == 0) s_qx = 1;
+        __syncthreads();
+        if (warp > 0 || !staged) {   // warps 1-7 stage x_t while warp 0 bounds the keys
+            int m = 1;
+            const int nthr = staged ? (int)blockDim.x - 32 : (int)blockDim.x;
+            const int tid = staged ? (int)threadIdx.x - 32 : (int)threadIdx.x;
+            for (int i = tid; i < d / 8; i += nthr) {   // d % 8 == 0, rows 16-byte aligned
+                const uint4 v = reinterpret_cast<const uint4*>(xg)[i];
+                if (staged) reinterpret_cast<uint4*>(fb_x)[i] = v;
+                const uint32_t w4[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+                for (int j = 0; j < 4; ++j)
+                    m = max(m, max((int)((w4[j] >> 7) & 0xffu), (int)((w4[j] >> 23) & 0xffu)));
+            }
+            m = __reduce_max_sync(0xffffffffu, m);
+            if (lane == 0) atomicMax(&s_qx, m);
+        }
         float sv[NPL];
         uint32_t sure_in = 0, cand = 0;
         int need = 0;
@@ -371,7 +421,7 @@ __global__ void __launch_bounds__(256, 1) route_fallback_kernel(
                 if (e < E) {
                     sv[i] = s[(int64_t)t * ld + e];
                     const float key = sigmoid_fast(sv[i]) + b[e];
-                    const float tk = key_tau_exact_slope(sv[i], logit_tau(xn, wnorm[e]));
+                    const float tk = key_tau_exact_slope(sv[i], logit_tau(xn, wnorm[e], wnorm[E + e]));
                     up[i] = key + tk;
                     lo[i] = key - tk;
                 } else {
@@ -404,56 +454,72 @@ __global__ void __launch_bounds__(256, 1) route_fallback_kernel(
             const bool bad = need < 0 || need > n_cand;
             if (lane == 0) {
                 if (bad) report(st, MOEVIE_ERR_DEVICE, SITE_ROUTE_FALLBACK, t, need);
-                s_ncand = bad ? -1 : n_cand;
+                s_ncand = bad ? -1 : (need == 0 ? 0 : n_cand);
             }
         }
         __syncthreads();
         const int nc = s_ncand;
-        for (int c0 = 0; c0 < nc; c0 += FB_CB) {
-            const int cn = min(FB_CB, nc - c0);
-            for (int c = 0; c < cn; ++c) {   // the window of each candidate: its largest term q
-                const uint32_t* wcol = reinterpret_cast<const uint32_t*>(wrt + (int64_t)s_cand[c0 + c] * dp);
-                int m = 2;
-                for (int i = threadIdx.x; i < d; i += 256) m = max(m, long_acc_q(xh[i], wcol[i]));
-                m = __reduce_max_sync(0xffffffffu, m);
-                if (lane == 0) atomicMax(&s_qmax[c], m);
+        const int qx = s_qx;
+        const uint16_t* xs = staged ? fb_x : xg;
+        for (int c0 = 0; c0 < nc; c0 += FB_BATCH) {
+            const int cn = min(FB_BATCH, nc - c0);
+            if (warp < cn) {   // warp c: the window of candidate c0 + c
+                const int e = s_cand[c0 + warp];
+                int qw = 1;
+                for (int pp = lane; pp < wexp_parts; pp += 32) qw = max(qw, __ldg(wexp + (int64_t)pp * Ep + e));
+                qw = __reduce_max_sync(0xffffffffu, qw);
+                if (lane == 0) s_q[warp] = (qx == 255 || qw == 255) ? -1 : qx + qw;   // -1: NaN
             }
             __syncthreads();
-            for (int c = 0; c < cn; ++c) {
-                const uint32_t* wcol = reinterpret_cast<const uint32_t*>(wrt + (int64_t)s_cand[c0 + c] * dp);
-                const int Q = s_qmax[c];   // the same in every thread
-                unsigned __int128 acc = 0;
-                if (Q < 1024) {   // finite inputs (else the logit is NaN): every q <= Q
-                    for (int i = threadIdx.x; i < d; i += 256) long_acc_term(xh[i], wcol[i], Q, acc);
-                    acc = warp_sum_u128(acc);
-                }
-                if (lane == 0) {
-                    s_acc[0][warp][c] = (unsigned long long)(uint64_t)acc;
-                    s_acc[1][warp][c] = (unsigned long long)(uint64_t)(acc >> 64);
-                }
-            }
-            __syncthreads();
-            if (warp == 0 && lane < cn) {   // exact logit of candidate c0 + lane (NaN for non-finite inputs)
-                unsigned __int128 u = 0;
+            unsigned __int128 acc[FB_BATCH];
+            int Q[FB_BATCH];
+            const float* wc[FB_BATCH];
 #pragma unroll
-                for (int w = 0; w < 8; ++w)
-                    u += ((unsigned __int128)s_acc[1][w][lane] << 64) | s_acc[0][w][lane];
-                s_key[c0 + lane] = s_qmax[lane] < 1024 ? long_acc_value(u, s_qmax[lane])
-                                                       : __longlong_as_double(0x7ff8000000000000ll);
+            for (int c = 0; c < FB_BATCH; ++c) {
+                acc[c] = 0;
+                Q[c] = c < cn ? s_q[c] : -1;
+                wc[c] = wrt + (int64_t)s_cand[c0 + (c < cn ? c : 0)] * dp;
             }
-            if (warp == 0 && lane < FB_CB) s_qmax[lane] = 2;   // for the next batch / token
+            for (int i = threadIdx.x; i < d; i += blockDim.x) {
+                const uint32_t hx = xs[i];
+                uint32_t uw[FB_BATCH];
+#pragma unroll
+                for (int c = 0; c < FB_BATCH; ++c) uw[c] = Q[c] > 0 ? __float_as_uint(__ldg(wc[c] + i)) : 0u;
+#pragma unroll
+                for (int c = 0; c < FB_BATCH; ++c)
+                    if (Q[c] > 0) long_acc_term(hx, uw[c], Q[c], acc[c]);
+            }
+#pragma unroll
+            for (int c = 0; c < FB_BATCH; ++c) {
+                if (Q[c] <= 0) continue;   // uniform over the CTA
+                const unsigned __int128 a = warp_sum_u128(acc[c]);
+                if (lane == 0) {
+                    s_acc[warp][c][0] = (unsigned long long)(uint64_t)a;
+                    s_acc[warp][c][1] = (unsigned long long)(uint64_t)(a >> 64);
+                }
+            }
+            __syncthreads();
+            if (warp == 0 && lane < cn) {   // candidate c0 + lane: the sum over the 8 warps
+                const int q = s_q[lane];
+                double v = __longlong_as_double(0x7ff8000000000000ll);
+                if (q > 0) {
+                    unsigned __int128 u = 0;
+#pragma unroll
+                    for (int w = 0; w < 8; ++w)
+                        u += ((unsigned __int128)s_acc[w][lane][1] << 64) | s_acc[w][lane][0];
+                    v = long_acc_value(u, q);
+                }
+                s_key[c0 + lane] = 1.0 / (1.0 + exp(-v)) + (double)b[s_cand[c0 + lane]];
+            }
             __syncthreads();
         }
         if (warp == 0 && nc >= 0) {
-            // keys of all candidates at once, one per lane (fp64 is slow: run it in parallel)
-            for (int c = lane; c < nc; c += 32) s_key[c] = 1.0 / (1.0 + exp(-s_key[c])) + (double)b[s_cand[c]];
-            __syncwarp();
             double exk[NPL];
             int base = 0;
 #pragma unroll
             for (int i = 0; i < NPL; ++i) {
                 const uint32_t m = __ballot_sync(0xffffffffu, (cand >> i) & 1u);
-                exk[i] = ((cand >> i) & 1u) ? s_key[base + __popc(m & lt)] : -INFINITY;
+                exk[i] = ((cand >> i) & 1u && nc > 0) ? s_key[base + __popc(m & lt)] : -INFINITY;
                 base += __popc(m);
             }
             // choose `need` candidates by exact key, ties to the lower id
@@ -501,7 +567,7 @@ __global__ void __launch_bounds__(256, 1) route_fallback_kernel(
                 pbase += __popc(m);
             }
         }
-        __syncthreads();   // s_cand / s_key are reused by the next token
+        __syncthreads();   // s_cand / s_key / s_ncand / s_qx / fb_x are reused by the next token
     }
 }
 
@@ -523,9 +589,9 @@ int route_split_parts(int d) { return route_dpad(d) / SPLIT_TILE; }
 int route_ksplit(int64_t T, int d, int E) {
     int BN = 0, n_ntiles = 0;
     const bool cc = route_concat(E);
-    choose_bn(cc ? 3 * route_epad(E) : E, &BN, &n_ntiles);
+    choose_bn(cc ? 2 * route_epad(E) : E, &BN, &n_ntiles);
     const int64_t items = (T + GM_BM - 1) / GM_BM * n_ntiles;
-    const int nkb = (cc ? 1 : 3) * route_dpad(d) / GM_BK;
+    const int nkb = (cc ? 1 : 2) * route_dpad(d) / GM_BK;
     // work items to aim for: with the pieces side by side (K = d_pad) fewer, longer
     // splits pay (measured: c1 64 items 4.8 us faster than 160)
     const int64_t target = cc ? ROUTE_SPLIT_TARGET_CONCAT : ROUTE_SPLIT_TARGET;
@@ -545,12 +611,12 @@ int64_t route_logits_rows(int64_t T, int d, int E) {
 }
 
 cudaError_t launch_route_split(const float* Wr, int d, int E, __nv_bfloat16* Wsplit, float* wrt,
-                               float* wpart, DevStatus* st, cudaStream_t s) {
+                               float* wpart, int32_t* wexp, DevStatus* st, cudaStream_t s) {
     const int Ep = route_epad(E);
     const int parts = route_split_parts(d);
     cudaError_t e = launch_pdl(route_split_kernel, dim3((Ep + SPLIT_TILE - 1) / SPLIT_TILE, parts),
-                               dim3(256), 0, s, Wr, d, route_dpad(d), E, Ep, Wsplit, wrt, wpart, st,
-                               route_concat(E) ? 1 : 0);
+                               dim3(256), 0, s, Wr, d, route_dpad(d), E, Ep, Wsplit, wrt, wpart, parts,
+                               wexp, st, route_concat(E) ? 1 : 0);
     count_launches(1);
     return e;
 }
@@ -565,23 +631,27 @@ cudaError_t launch_route_sum_parts(const float* logits, int64_t part_stride, int
 
 cudaError_t launch_route_select(const __nv_bfloat16* x, const float* wrt, const float* b,
                                 float* logits, int ld, int nparts, int64_t part_stride,
-                                const float* wnorm, int T, int d, int E, int k, int32_t* idx,
-                                float* gate, int32_t* fb_tokens, float* xnorm, DevStatus* st,
-                                int num_sms, cudaStream_t s) {
+                                const float* wnorm, const int32_t* wexp, int T, int d, int E, int k,
+                                int32_t* idx, float* gate, int32_t* fb_tokens, float* xnorm,
+                                DevStatus* st, int num_sms, cudaStream_t s, float* zero,
+                                int64_t zero_n) {
     const int blocks = (int)(((int64_t)T * 32 + 255) / 256);
-    const int fb_blocks = T < 4 * num_sms ? T : 4 * num_sms;
+    const int fb_blocks = T < 3 * num_sms ? T : 3 * num_sms;   // about one wave
+    const size_t fb_smem = d <= FB_X_SMEM ? (size_t)2 * d : 0;
     const int npl = (E + 31) / 32;
     const int dp = route_dpad(d);
+    const int parts = route_split_parts(d), Ep = route_epad(E);
     cudaError_t e = cudaSuccess;
 #define MV_ROUTE(N)                                                                                \
     do {                                                                                           \
         e = launch_pdl(route_topk_kernel<N>, dim3(blocks), dim3(256), 0, s, x, logits, ld, nparts,  \
                        part_stride, b, wnorm, T, d, E, k, idx, gate, (const float*)xnorm,           \
-                       fb_tokens, st);                                                             \
+                       fb_tokens, st, reinterpret_cast<float4*>(zero), zero ? zero_n / 4 : 0);      \
         if (e == cudaSuccess)                                                                      \
-            e = launch_pdl(route_fallback_kernel<N>, dim3(fb_blocks), dim3(256), 0, s, x, wrt, dp, \
-                           b, (const float*)logits, ld, (const float*)xnorm, wnorm, d, E, k, idx,  \
-                           gate, (const int32_t*)fb_tokens, st);                                   \
+            e = launch_pdl(route_fallback_kernel<N>, dim3(fb_blocks), dim3(256), fb_smem, s, x,    \
+                           wrt, dp, wexp, parts, Ep, b, (const float*)logits, ld,                  \
+                           (const float*)xnorm, wnorm, d, E, k, idx, gate,                          \
+                           (const int32_t*)fb_tokens, st);                                         \
     } while (0)
     if (npl <= 1) MV_ROUTE(1);
     else if (npl <= 2) MV_ROUTE(2);
