@@ -227,6 +227,19 @@ struct GemmSpec {
     const void* W3_2nd;      // EPI_SWIGLU_BF16 with W2nd: the up projection of groups >= g_split
                              //   (strides as W2nd, which then holds their gate)
     int a_ident;             // A rows contiguous but loaded by the gather warps (A row r = r)
+    // training path (see GemmArgs): K-major B W[G][N][K] with row stride b_k_ld and group
+    // stride b_g_ld; M-major A [a_nrows][a_cols] (row stride lda) for weight-gradient items
+    int b_kmajor;
+    int64_t b_k_ld, b_g_ld;
+    int a_mn;
+    int wg_M;                // item_table == 2: output rows per group
+    int64_t b_rows;          // item_table == 2: rows of B (one group, the K rows all items share)
+    int64_t max_items;       // item_table == 2: host bound on the number of items
+    int a_neg_zero, o_neg_skip;
+    void* out2;
+    const void* epi_u;
+    const void* epi_a;
+    float* dg_part;
 };
 
 moevie_status run_gemm(const GemmSpec& g, DevStatus* st, cudaStream_t s) {
@@ -235,8 +248,17 @@ moevie_status run_gemm(const GemmSpec& g, DevStatus* st, cudaStream_t s) {
     const int64_t n_ld = g.N_ld > 0 ? g.N_ld : g.N;
     if (n_ld < g.N || n_ld % 8 != 0) return MOEVIE_ERR_UNSUPPORTED;
     const bool swiglu = g.epi == EPI_SWIGLU_BF16;
-    if (!make_weight_tmap_strided(&a.tmB, g.W, g.N, g.K, g.W2nd ? g.g_split : g.G, n_ld, n_ld * g.K))
+    if (g.b_kmajor) {   // box: the CTA's half of an n-tile's columns
+        int bn = 0, nnt = 0;
+        choose_bn(g.N, &bn, &nnt);
+        if (swiglu || g.W2nd || g.b_k_ld % 8 != 0 || g.b_g_ld % 8 != 0 || g.b_k_ld < g.K)
+            return MOEVIE_ERR_UNSUPPORTED;
+        if (!make_kmajor_tmap(&a.tmB, g.W, g.K, g.N, g.G, g.b_k_ld, g.b_g_ld, bn / 2)) return MOEVIE_ERR_CUDA;
+    } else if (g.item_table == 2) {   // weight gradients: B [b_rows][N] as one group
+        if (!make_weight_tmap_strided(&a.tmB, g.W, g.N, g.b_rows, 1, n_ld, n_ld * g.b_rows)) return MOEVIE_ERR_CUDA;
+    } else if (!make_weight_tmap_strided(&a.tmB, g.W, g.N, g.K, g.W2nd ? g.g_split : g.G, n_ld, n_ld * g.K)) {
         return MOEVIE_ERR_CUDA;
+    }
     if (g.W2nd) {   // groups >= g_split (swiglu: their gate in tmB3, their up projection in tmB4)
         if (g.g_split <= 0 || g.g_split >= g.G || !a16(g.W2nd) || g.w2_k_ld % 8 != 0 ||
             g.w2_g_ld % 8 != 0 || g.w2_k_ld < g.N)
@@ -251,8 +273,22 @@ moevie_status run_gemm(const GemmSpec& g, DevStatus* st, cudaStream_t s) {
                 return MOEVIE_ERR_CUDA;
         }
     }
-    if (!g.a_rows && !make_rows_tmap(&a.tmA, g.A, g.a_cols > 0 ? g.a_cols : g.K, g.a_nrows, g.lda))
+    if (g.a_mn) {   // A [a_nrows = K rows][a_cols = M] as the 3-D map {M, K, 1}, box {64, 64, 1}
+        if (g.a_rows || g.lda % 8 != 0 || g.item_table != 2) return MOEVIE_ERR_UNSUPPORTED;
+        if (!make_weight_tmap_strided(&a.tmA, g.A, g.a_cols, g.a_nrows, 1, g.lda, g.lda * g.a_nrows))
+            return MOEVIE_ERR_CUDA;
+    } else if (!g.a_rows && !make_rows_tmap(&a.tmA, g.A, g.a_cols > 0 ? g.a_cols : g.K, g.a_nrows, g.lda)) {
         return MOEVIE_ERR_CUDA;
+    }
+    a.b_kmajor = g.b_kmajor ? 1 : 0;
+    a.a_mn = g.a_mn ? 1 : 0;
+    a.wg_M = g.wg_M;
+    a.a_neg_zero = g.a_neg_zero;
+    a.o_neg_skip = g.o_neg_skip;
+    a.out2 = static_cast<__nv_bfloat16*>(g.out2);
+    a.epi_u = static_cast<const __nv_bfloat16*>(g.epi_u);
+    a.epi_a = static_cast<const __nv_bfloat16*>(g.epi_a);
+    a.dg_part = g.dg_part;
     a.A = static_cast<const __nv_bfloat16*>(g.A);
     a.lda = g.lda;
     a.a_rows = g.a_rows;
@@ -326,7 +362,10 @@ moevie_status run_gemm(const GemmSpec& g, DevStatus* st, cudaStream_t s) {
     a.y_split_stride = g.y_split_stride;
     a.status = st;
     a.limit_ns = WAIT_LIMIT_NS;
-    if (a.item_table) {
+    if (a.item_table == 2) {
+        if (!g.tiles || a.ksplit != 1 || g.wg_M <= 0 || g.wg_M > 65535 || g.N > 65535) return MOEVIE_ERR_UNSUPPORTED;
+        a.max_mtiles = g.max_items;
+    } else if (a.item_table) {
         if (!g.tiles || a.ksplit != 1) return MOEVIE_ERR_UNSUPPORTED;
         a.max_mtiles *= a.n_ntiles;   // bound on the item count
     }
@@ -816,6 +855,291 @@ moevie_status moevie_get_device_status(const void* ws, void* stream, moevie_stat
     if (cudaMemcpy(v, ws, sizeof v, cudaMemcpyDeviceToHost) != cudaSuccess) return MOEVIE_ERR_CUDA;
     *out = v[0];
     if (detail) memcpy(detail, v, sizeof v);
+    return MOEVIE_OK;
+}
+
+// ------------------------------------------------------------ training path
+
+}  // extern "C"
+
+namespace {
+
+// Workspace of moevie_moe_backward.  Expert segments are padded to multiples of 64 rows
+// (rows_max = T k + 63 E bounds the padded total), so that the weight-gradient GEMMs'
+// K blocks never straddle two experts.
+struct BwdLayout {
+    size_t status, wsplit, wrt, wpart, wexp, sig, gate, hist, counts, offsets, tiles, n_tiles, perm,
+        inv, poff, ptok, pgate, slot_prow, ptiles, n_ptiles, it2, n_it2, it1, n_it1, itr, n_itr, H, U,
+        DU, Gm, Xp, dgp, DS, dwr;
+    int64_t rows_max, max_it2, max_it1, max_itr;
+    int nt_h;
+    size_t total;
+};
+
+BwdLayout make_bwd_layout(int64_t T, int64_t d, int64_t E, int64_t k, int64_t h) {
+    BwdLayout L;
+    size_t o = 0;
+    auto take = [&](size_t bytes) {
+        const size_t at = o;
+        o += up256(bytes);
+        return at;
+    };
+    const int64_t n = T * k, Ep = route_epad((int)E), dp = route_dpad((int)d), hp = row_ld(h);
+    L.rows_max = n + 63 * E;
+    int bn_d = 0, nt_d = 0, bn_h = 0, bn_e = 0, nt_e = 0;
+    choose_bn((int)d, &bn_d, &nt_d);
+    choose_bn((int)h, &bn_h, &L.nt_h);
+    choose_bn((int)Ep, &bn_e, &nt_e);
+    L.max_it2 = bwd_max_items(L.rows_max, (int)E, (int)h, (int)d, bn_d);
+    L.max_it1 = bwd_max_items(L.rows_max, (int)E, (int)d, (int)h, bn_h);
+    L.max_itr = bwd_max_items(T, 1, (int)d, (int)Ep, bn_e);
+    L.status = take(sizeof(DevStatus));
+    L.wsplit = take(2 * 2 * dp * Ep);
+    L.wrt = take(4 * E * dp);
+    L.wpart = take(4 * 2 * (int64_t)route_split_parts((int)d) * Ep);
+    L.wexp = take(4 * (int64_t)route_split_parts((int)d) * Ep);
+    L.sig = take(4 * n);
+    L.gate = take(4 * n);
+    L.hist = take(4 * ((n + 255) / 256) * E);
+    L.counts = take(4 * E);
+    L.offsets = take(4 * (E + 1));
+    L.tiles = take(16 * max_mtiles(n, E));
+    L.n_tiles = take(4);
+    L.perm = take(4 * n);
+    L.inv = take(4 * n);
+    L.poff = take(4 * (E + 1));
+    L.ptok = take(4 * L.rows_max);
+    L.pgate = take(4 * L.rows_max);
+    L.slot_prow = take(4 * n);
+    L.ptiles = take(16 * max_mtiles(L.rows_max, E));
+    L.n_ptiles = take(4);
+    L.it2 = take(16 * L.max_it2);
+    L.n_it2 = take(4);
+    L.it1 = take(16 * L.max_it1);
+    L.n_it1 = take(4);
+    L.itr = take(16 * L.max_itr);
+    L.n_itr = take(4);
+    L.H = take(2 * L.rows_max * hp);
+    L.U = take(2 * L.rows_max * hp);
+    L.DU = take(2 * L.rows_max * hp);
+    L.Gm = take(2 * L.rows_max * d);
+    L.Xp = take(2 * L.rows_max * d);
+    L.dgp = take(4 * 2 * (int64_t)L.nt_h * L.rows_max);
+    L.DS = take(2 * T * Ep);
+    L.dwr = take(4 * d * Ep);
+    L.total = o;
+    return L;
+}
+
+moevie_status check_bwd_sizes(int64_t T, int64_t d, int64_t E, int64_t k, int64_t h) {
+    moevie_status c = check_sizes(T, d, E, k, h, 0);
+    if (c != MOEVIE_OK) return c;
+    if (h <= 0 || k > 32 || d > 65535 || h > 65535 || T * k + 63 * E >= (int64_t(1) << 31))
+        return MOEVIE_ERR_UNSUPPORTED;
+    return MOEVIE_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+moevie_status moevie_backward_workspace_size(int64_t T_max, int64_t d, int64_t E, int64_t k, int64_t h,
+                                             size_t* bytes) {
+    if (!bytes) return MOEVIE_ERR_INVALID_ARG;
+    const moevie_status c = check_bwd_sizes(T_max, d, E, k, h);
+    if (c != MOEVIE_OK) return c;
+    *bytes = make_bwd_layout(T_max, d, E, k, h).total;
+    return MOEVIE_OK;
+}
+
+moevie_status moevie_moe_backward(const moevie_layer* Lr, const void* x, const void* dy, int64_t T,
+                                  const int32_t* idx, float* dx, float* dW_r, float* dW1, float* dW2,
+                                  void* ws, size_t ws_bytes, void* stream) {
+    if (!Lr) return MOEVIE_ERR_INVALID_ARG;
+    const int64_t d = Lr->d, E = Lr->E, k = Lr->k, h = Lr->h;
+    moevie_status c = check_bwd_sizes(T, d, E, k, h);
+    if (c != MOEVIE_OK) return c;
+    if (Lr->W3 || Lr->h_s > 0) return MOEVIE_ERR_UNSUPPORTED;   // GELU experts, no shared expert
+    if (T == 0) return MOEVIE_OK;
+    if (!x || !dy || !idx || !dx || !dW_r || !dW1 || !dW2 || !ws || !Lr->W_r || !Lr->W1 || !Lr->W2)
+        return MOEVIE_ERR_INVALID_ARG;
+    if (!a16(x) || !a16(dy) || !a16(idx) || !a16(dx) || !a16(dW1) || !a16(dW2) || !a16(ws) || !a16(Lr->W1) ||
+        !a16(Lr->W2))
+        return MOEVIE_ERR_INVALID_ARG;
+    const BwdLayout L = make_bwd_layout(T, d, E, k, h);
+    if (ws_bytes < L.total) return MOEVIE_ERR_WORKSPACE;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    DevStatus* st = at<DevStatus>(ws, L.status);
+    const int64_t n = T * k, Ep = route_epad((int)E), dp = route_dpad((int)d), hp = row_ld(h);
+    const __nv_bfloat16* xb = static_cast<const __nv_bfloat16*>(x);
+    float* wrt = at<float>(ws, L.wrt);
+    int32_t* poff = at<int32_t>(ws, L.poff);
+    int32_t* ptok = at<int32_t>(ws, L.ptok);
+    float* pgate = at<float>(ws, L.pgate);
+    void* H = at<void>(ws, L.H);
+    void* U = at<void>(ws, L.U);
+    void* DU = at<void>(ws, L.DU);
+    void* Gm = at<void>(ws, L.Gm);
+    void* Xp = at<void>(ws, L.Xp);
+    float* dgp = at<float>(ws, L.dgp);
+    __nv_bfloat16* DS = at<__nv_bfloat16>(ws, L.DS);
+    float* dwr = at<float>(ws, L.dwr);
+    int bn_d = 0, nt_d = 0, bn_h = 0, nt_h = 0, bn_e = 0, nt_e = 0;
+    choose_bn((int)d, &bn_d, &nt_d);
+    choose_bn((int)h, &bn_h, &nt_h);
+    choose_bn((int)Ep, &bn_e, &nt_e);
+
+    // 1. W_r's transposed fp32 copy (the router's split kernel), the gates of the held
+    //    selection (Eqs. 4-5), and the stable expert-major order (Algorithm 1, phase 1)
+    MV_TRY(launch_route_split(Lr->W_r, (int)d, (int)E, at<__nv_bfloat16>(ws, L.wsplit), wrt,
+                              at<float>(ws, L.wpart), at<int32_t>(ws, L.wexp), st, s));
+    MV_TRY(launch_bwd_gates(xb, wrt, (int)dp, idx, T, (int)d, (int)E, (int)k, at<float>(ws, L.sig),
+                            at<float>(ws, L.gate), st, s));
+    MV_TRY(launch_permute(idx, n, (int)k, (int)E, GM_BM, perm_chunk(n, num_sms()), nullptr,
+                          at<int32_t>(ws, L.hist), at<int32_t>(ws, L.counts), at<int32_t>(ws, L.offsets),
+                          at<int4>(ws, L.tiles), at<int32_t>(ws, L.n_tiles), at<int32_t>(ws, L.perm),
+                          at<int32_t>(ws, L.inv), nullptr, nullptr, st, s));
+    // 2. segments padded to 64 rows: row maps, m-tiles, weight-gradient items
+    MV_TRY(launch_bwd_pad(at<int32_t>(ws, L.counts), (int)E, poff, s));
+    MV_TRY(launch_bwd_rows(idx, at<int32_t>(ws, L.inv), at<int32_t>(ws, L.counts), at<int32_t>(ws, L.offsets),
+                           poff, at<float>(ws, L.gate), n, (int)k, (int)E, ptok, pgate,
+                           at<int32_t>(ws, L.slot_prow), s));
+    MV_TRY(launch_tile_table(poff, (int)E, GM_BM, at<int4>(ws, L.ptiles), at<int32_t>(ws, L.n_ptiles), s));
+    MV_TRY(launch_bwd_items(poff, (int)E, 0, (int)h, (int)d, bn_d, (int)L.max_it2, at<int4>(ws, L.it2),
+                            at<int32_t>(ws, L.n_it2), st, s));
+    MV_TRY(launch_bwd_items(poff, (int)E, 0, (int)d, (int)h, bn_h, (int)L.max_it1, at<int4>(ws, L.it1),
+                            at<int32_t>(ws, L.n_it1), st, s));
+    MV_TRY(launch_bwd_items(nullptr, 1, T, (int)d, (int)Ep, bn_e, (int)L.max_itr, at<int4>(ws, L.itr),
+                            at<int32_t>(ws, L.n_itr), st, s));
+    // 3. accumulators cleared; gathered copies of x and g dy
+    MV_TRY(launch_zero_f32(dx, T * d, s));
+    MV_TRY(launch_zero_f32(dW1, E * d * hp, s));
+    MV_TRY(launch_zero_f32(dW2, E * h * d, s));
+    MV_TRY(launch_zero_f32(dwr, d * Ep, s));
+    MV_TRY(launch_zero_f32(reinterpret_cast<float*>(DS), T * Ep / 2, s));
+    MV_TRY(launch_bwd_gather(xb, static_cast<const __nv_bfloat16*>(dy), ptok, pgate, poff, (int)E, (int)d,
+                             L.rows_max, static_cast<__nv_bfloat16*>(Xp), static_cast<__nv_bfloat16*>(Gm), s));
+    // 4. up-projection again: u = x W1[e] and a = GELU(u), both kept (bf16)
+    {
+        GemmSpec g{};
+        g.A = x;
+        g.lda = d;
+        g.a_rows = ptok;
+        g.a_div = 1;
+        g.a_nrows = T;
+        g.a_neg_zero = 1;
+        g.m_total = L.rows_max;
+        g.tiles = at<int4>(ws, L.ptiles);
+        g.n_tiles = at<int32_t>(ws, L.n_ptiles);
+        g.G = (int)E;
+        g.W = Lr->W1;
+        g.K = (int)d;
+        g.N = (int)h;
+        g.N_ld = hp;
+        g.epi = EPI_GELU2_BF16;
+        g.out = H;
+        g.out2 = U;
+        g.ldo = hp;
+        if ((c = run_gemm(g, st, s)) != MOEVIE_OK) return c;
+    }
+    // 5. da' = dy W2[e]^T (K-major W2), epilogue du = g da' GELU'(u) and dg = da' . a
+    {
+        GemmSpec g{};
+        g.A = dy;
+        g.lda = d;
+        g.a_rows = ptok;
+        g.a_div = 1;
+        g.a_nrows = T;
+        g.a_neg_zero = 1;
+        g.m_total = L.rows_max;
+        g.tiles = at<int4>(ws, L.ptiles);
+        g.n_tiles = at<int32_t>(ws, L.n_ptiles);
+        g.G = (int)E;
+        g.W = Lr->W2;
+        g.b_kmajor = 1;
+        g.b_k_ld = d;
+        g.b_g_ld = h * d;
+        g.K = (int)d;
+        g.N = (int)h;
+        g.N_ld = hp;
+        g.epi = EPI_DGELU_BF16;
+        g.row_scale = pgate;
+        g.epi_u = U;
+        g.epi_a = H;
+        g.out = DU;
+        g.ldo = hp;
+        g.dg_part = dgp;
+        if ((c = run_gemm(g, st, s)) != MOEVIE_OK) return c;
+    }
+    // 6. dx += du W1[e]^T (K-major W1), scattered to the rows' tokens
+    {
+        GemmSpec g{};
+        g.A = DU;
+        g.lda = hp;
+        g.a_cols = h;
+        g.a_nrows = L.rows_max;
+        g.m_total = L.rows_max;
+        g.tiles = at<int4>(ws, L.ptiles);
+        g.n_tiles = at<int32_t>(ws, L.n_ptiles);
+        g.G = (int)E;
+        g.W = Lr->W1;
+        g.b_kmajor = 1;
+        g.b_k_ld = hp;
+        g.b_g_ld = d * hp;
+        g.K = (int)h;
+        g.N = (int)d;
+        g.epi = EPI_ADD_F32;
+        g.yacc = dx;
+        g.ldy = d;
+        g.o_nrows = T;
+        g.o_rows = ptok;
+        g.o_div = 1;
+        g.o_neg_skip = 1;
+        g.scale = 1.0f;
+        if ((c = run_gemm(g, st, s)) != MOEVIE_OK) return c;
+    }
+    // 7. the router (Eqs. 4-5): ds per token, dx += ds W_r^T, ds into [T][E_pad] bf16
+    MV_TRY(launch_bwd_router(idx, at<float>(ws, L.sig), at<float>(ws, L.gate), at<int32_t>(ws, L.slot_prow), dgp,
+                             2 * nt_h, L.rows_max, wrt, (int)dp, T, (int)d, (int)E, (int)k, (int)Ep, dx, DS, s));
+    // 8. weight gradients, per expert over its padded rows: dW2[e] = a^T (g dy),
+    //    dW1[e] = x^T du; and dW_r = x^T ds over all tokens
+    auto wgrad = [&](const void* A, int64_t a_cols, int64_t a_rows, int64_t lda, const void* B, int64_t N,
+                     int64_t n_ld, int64_t b_rows, int G, int M, size_t items, size_t n_items, int64_t max_items,
+                     float* out, int64_t ldy) {
+        GemmSpec g{};
+        g.A = A;
+        g.a_mn = 1;
+        g.a_cols = a_cols;
+        g.a_nrows = a_rows;
+        g.lda = lda;
+        g.W = B;
+        g.N = (int)N;
+        g.N_ld = n_ld;
+        g.b_rows = b_rows;
+        g.K = 64;
+        g.G = G;
+        g.wg_M = M;
+        g.item_table = 2;
+        g.tiles = at<int4>(ws, items);
+        g.n_tiles = at<int32_t>(ws, n_items);
+        g.max_items = max_items;
+        g.m_total = (int64_t)G * M;
+        g.epi = EPI_ADD_F32;
+        g.yacc = out;
+        g.ldy = ldy;
+        g.o_nrows = (int64_t)G * M;
+        g.scale = 1.0f;
+        return run_gemm(g, st, s);
+    };
+    if ((c = wgrad(H, h, L.rows_max, hp, Gm, d, d, L.rows_max, (int)E, (int)h, L.it2, L.n_it2, L.max_it2, dW2,
+                   d)) != MOEVIE_OK)
+        return c;
+    if ((c = wgrad(Xp, d, L.rows_max, d, DU, h, hp, L.rows_max, (int)E, (int)d, L.it1, L.n_it1, L.max_it1, dW1,
+                   hp)) != MOEVIE_OK)
+        return c;
+    if ((c = wgrad(x, d, T, d, DS, Ep, Ep, T, 1, (int)d, L.itr, L.n_itr, L.max_itr, dwr, Ep)) != MOEVIE_OK)
+        return c;
+    MV_TRY(launch_bwd_copy(dwr, Ep, dW_r, d, E, s));
     return MOEVIE_OK;
 }
 

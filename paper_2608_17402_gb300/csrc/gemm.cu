@@ -147,6 +147,7 @@ struct Tile {
     int g, row0, nrows, n0;
     int kb0, kb1;   // k-blocks [kb0, kb1) of this item's split of K
     int ks;         // split index
+    int m0;         // weight-gradient items: first row of the output tile within its group
 };
 
 // A work item's table entry, loaded but not yet checked.  The roles that walk the
@@ -180,6 +181,25 @@ __device__ __forceinline__ void tile_kb(const GemmArgs& p, int ks, int& kb0, int
 __device__ __forceinline__ Tile tile_finish(const GemmArgs& p, const TileLd& l) {
     Tile t;
     t.ks = l.ks;
+    t.m0 = 0;
+    if (p.item_table == 2) {   // a weight-gradient item {g, m0 | n0 << 16, kb0, kb1}
+        t.g = l.d.x;
+        t.m0 = l.d.y & 0xffff;
+        t.n0 = (int)((uint32_t)l.d.y >> 16);
+        t.kb0 = l.d.z;
+        t.kb1 = l.d.w;
+        t.row0 = t.g * p.wg_M + t.m0;
+        t.nrows = min(GM_BM, p.wg_M - t.m0);
+        if (t.g < 0 || t.g >= p.G || t.m0 >= p.wg_M || t.n0 >= p.N || t.kb0 < 0 || t.kb1 <= t.kb0 ||
+            (int64_t)t.row0 + t.nrows > p.m_total) {
+            report(p.status, MOEVIE_ERR_DEVICE, SITE_GEMM_TILES, t.g, t.kb0);
+            t.nrows = 0;
+            t.g = 0;
+            t.n0 = 0;
+            t.kb1 = t.kb0 = 0;
+        }
+        return t;
+    }
     tile_kb(p, l.ks, t.kb0, t.kb1);
     if (p.item_table) {   // an explicit (m-tile, n-tile) item
         t.g = l.d.x;
@@ -250,6 +270,12 @@ __device__ __forceinline__ void gelu_erf2(float& u0, float& u1) {
     f2_unpack(r, u0, u1);
 }
 
+// GELU'(u) = Phi(u) + u phi(u) (the derivative of the erf form), in fp32 with CUDA's
+// normcdff and expf (the training path only).
+__device__ __forceinline__ float gelu_grad(float u) {
+    return normcdff(u) + u * 0.3989422804014327f * expf(-0.5f * u * u);
+}
+
 struct Smem {
     uint32_t a0, b0;          // shared addresses of stage 0
     uint32_t full, empty;     // barrier arrays (8 bytes apart)
@@ -292,7 +318,10 @@ __device__ void producer_tma(const GemmArgs& p, const Smem& sm, int64_t n_work,
     if (!gather) tma_prefetch_desc(&p.tmA);
     const uint32_t half_n = (uint32_t)p.BN / 2;
     const uint32_t nboxh = (half_n + 63) / 64;
-    const uint32_t cta_bytes = nboxh * GM_BK * 128 + (gather ? 0u : (uint32_t)GM_A_BYTES);
+    // B per CTA and stage: nboxh boxes of 64 columns x 64 K rows (N-major), or half_n rows
+    // of 64 K values (K-major)
+    const uint32_t b_bytes = p.b_kmajor ? half_n * 128u : nboxh * GM_BK * 128;
+    const uint32_t cta_bytes = b_bytes + (gather ? 0u : (uint32_t)GM_A_BYTES);
     // gathering: plus the 16-byte signal with which the peer publishes its A half
     const uint32_t stage_tx = 2 * cta_bytes + (gather ? 16u : 0u);
     const uint32_t full_leader = peer_addr(sm.full, 0);
@@ -311,7 +340,7 @@ __device__ void producer_tma(const GemmArgs& p, const Smem& sm, int64_t n_work,
         const CUtensorMap* tmb = tail ? &p.tmB2 : &p.tmB;
         if (p.swiglu)
             tmb = sm.rank == 1 ? (tail ? &p.tmB4 : &p.tmB2) : (tail ? &p.tmB3 : &p.tmB);
-        const int gb = tail ? t.g - p.g_split : t.g;
+        const int gb = p.item_table == 2 ? 0 : (tail ? t.g - p.g_split : t.g);
         const int ncol0 = p.swiglu ? t.n0 : t.n0 + (int)(sm.rank * half_n);
         for (int kb = t.kb0; kb < t.kb1; ++kb) {
             if (!mbar_wait(sm.empty + 8 * s, ph ^ 1u, p.limit_ns, abort_flag)) {
@@ -322,12 +351,22 @@ __device__ void producer_tma(const GemmArgs& p, const Smem& sm, int64_t n_work,
             if (sm.rank == 0) mbar_arrive_expect_tx(sm.full + 8 * s, stage_tx);
             const uint32_t b_dst = sm.b0 + s * GM_B_BYTES;
             const int kk = kb * GM_BK;
-            for (uint32_t j = 0; j < nboxh; ++j)
-                tma_load_3d_pair(b_dst + j * (GM_BK * 128), tmb, bar, ncol0 + (int)(64 * j), kk, gb);
+            if (p.b_kmajor) {   // half_n rows of the CTA's columns, 64 K values each
+                tma_load_3d_pair(b_dst, tmb, bar, kk, ncol0, gb);
+            } else {
+                for (uint32_t j = 0; j < nboxh; ++j)
+                    tma_load_3d_pair(b_dst + j * (GM_BK * 128), tmb, bar, ncol0 + (int)(64 * j), kk, gb);
+            }
             if (!gather) {
-                const int col = p.a_kperiod ? kk % p.a_kperiod : kk;
-                tma_load_2d_pair(sm.a0 + s * GM_A_BYTES, &p.tmA, bar, col,
-                                 t.row0 + (int)sm.rank * GM_HALF);
+                if (p.a_mn) {   // two 64-row halves of the CTA's 128 output rows, 64 K rows each
+                    const int m = t.m0 + (int)sm.rank * GM_HALF;
+                    tma_load_3d_pair(sm.a0 + s * GM_A_BYTES, &p.tmA, bar, m, kk, 0);
+                    tma_load_3d_pair(sm.a0 + s * GM_A_BYTES + GM_BK * 128, &p.tmA, bar, m + 64, kk, 0);
+                } else {
+                    const int col = p.a_kperiod ? kk % p.a_kperiod : kk;
+                    tma_load_2d_pair(sm.a0 + s * GM_A_BYTES, &p.tmA, bar, col,
+                                     t.row0 + (int)sm.rank * GM_HALF);
+                }
             }
             if (++s == sm.nstages) {
                 s = 0;
@@ -364,7 +403,7 @@ __device__ __forceinline__ void gather_rows_finish(const GemmArgs& p, const Tile
         if (r < nh && idx >= 0 && idx < p.a_nrows) {
             src[j] = p.A + (int64_t)idx * p.lda;
         } else {
-            if (r < nh)
+            if (r < nh && !(p.a_neg_zero && raw[j] < 0))   // padding rows read as zeros
                 report(p.status, MOEVIE_ERR_DEVICE, SITE_GEMM_A_ROW, t.row0 + (int)rank * GM_HALF + r,
                        idx);
             src[j] = nullptr;
@@ -485,10 +524,13 @@ __device__ void gather_forwarder(const GemmArgs& p, const Smem& sm, int64_t n_wo
 // Leader CTA, warp 8, lane 0.
 __device__ void mma_issuer(const GemmArgs& p, const Smem& sm, uint32_t tmem, int64_t n_work,
                            volatile int* abort_flag) {
-    const uint32_t idesc = idesc_bf16_f32(2 * GM_HALF, p.BN, false, true);
-    // A K-major (k-slice +32 B), B MN-major (next 64-column atom LBO 8192, k-slice +2048 B)
-    const uint64_t adesc0 = smem_desc_sw128(sm.a0, 16, 1024);
-    const uint64_t bdesc0 = smem_desc_sw128(sm.b0, 8192, 1024);
+    const uint32_t idesc = idesc_bf16_f32(2 * GM_HALF, p.BN, p.a_mn != 0, p.b_kmajor == 0);
+    // K-major operands: k-slice +32 B; MN-major operands: next 64-element atom LBO 8192,
+    // k-slice +2048 B (16 K rows of 128 bytes)
+    const uint64_t adesc0 = p.a_mn ? smem_desc_sw128(sm.a0, 8192, 1024) : smem_desc_sw128(sm.a0, 16, 1024);
+    const uint64_t bdesc0 = p.b_kmajor ? smem_desc_sw128(sm.b0, 16, 1024) : smem_desc_sw128(sm.b0, 8192, 1024);
+    const uint32_t a_step = p.a_mn ? (2048 >> 4) : (32 >> 4);
+    const uint32_t b_step = p.b_kmajor ? (32 >> 4) : (2048 >> 4);
     static_assert(GM_BK == 64, "four k-slices of 16 per stage");
     int s = 0;
     uint32_t ph = 0;
@@ -522,9 +564,9 @@ __device__ void mma_issuer(const GemmArgs& p, const Smem& sm, uint32_t tmem, int
             const uint64_t ad = adesc0 + (uint64_t)((s * GM_A_BYTES) >> 4);
             const uint64_t bd = bdesc0 + (uint64_t)((s * GM_B_BYTES) >> 4);
             tc_mma_bf16_pair(d_tmem, ad, bd, idesc, kb != t.kb0 ? 1u : 0u);
-            tc_mma_bf16_pair(d_tmem, ad + (32 >> 4), bd + (2048 >> 4), idesc, 1u);
-            tc_mma_bf16_pair(d_tmem, ad + (64 >> 4), bd + (4096 >> 4), idesc, 1u);
-            tc_mma_bf16_pair(d_tmem, ad + (96 >> 4), bd + (6144 >> 4), idesc, 1u);
+            tc_mma_bf16_pair(d_tmem, ad + a_step, bd + b_step, idesc, 1u);
+            tc_mma_bf16_pair(d_tmem, ad + 2 * a_step, bd + 2 * b_step, idesc, 1u);
+            tc_mma_bf16_pair(d_tmem, ad + 3 * a_step, bd + 3 * b_step, idesc, 1u);
             issued = true;
             tc_commit_pair(sm.empty + 8 * s);
             if (++s == sm.nstages) {
@@ -610,7 +652,8 @@ __device__ void epilogue(const GemmArgs& p, const Smem& sm, uint32_t tmem, int64
             if (p.o_rows) tok = __ldg(p.o_rows + gr) / p.o_div;
             if (p.row_scale) sc = __ldg(p.row_scale + gr);
             if (to_f32 && (tok < 0 || tok >= p.o_nrows)) {
-                report(p.status, MOEVIE_ERR_DEVICE, SITE_GEMM_OUT_ROW, gr, (int)tok);
+                if (!(p.o_neg_skip && tok < 0))   // a padding row writes nothing
+                    report(p.status, MOEVIE_ERR_DEVICE, SITE_GEMM_OUT_ROW, gr, (int)tok);
                 ok_row = false;
             }
         }
@@ -704,6 +747,7 @@ __device__ void epilogue(const GemmArgs& p, const Smem& sm, uint32_t tmem, int64
             __syncwarp();
             if (lane == 0) mbar_arrive_remote(tempty_leader + 8 * acc);
         }
+        float dg_acc = 0.f;   // EPI_DGELU_BF16: this thread's share of its row's dot
         for (int ch = half; ch < nchunk; ch += 2) {
             const int c0 = ch * 32;
             if constexpr (ECLS == ECLS_ADD) {   // the y-accumulator reductions
@@ -732,13 +776,46 @@ __device__ void epilogue(const GemmArgs& p, const Smem& sm, uint32_t tmem, int64
             const int n = t.n0 + c0;
             if constexpr (!to_f32) {
                 __nv_bfloat16* orow = p.out + (int64_t)gr * p.ldo + n;
+                if (p.epi == EPI_DGELU_BF16) {   // training path: du = scale acc GELU'(u), dot acc . a
+                    const __nv_bfloat16* urow = p.epi_u + (int64_t)gr * p.ldo + n;
+                    const __nv_bfloat16* arow = p.epi_a + (int64_t)gr * p.ldo + n;
+#pragma unroll
+                    for (int g8 = 0; g8 < 4; ++g8) {
+                        if (n + 8 * g8 >= p.N) break;
+                        float uf[8], af[8], f[8];
+                        unpack_bf16x8(*reinterpret_cast<const uint4*>(urow + 8 * g8), uf);
+                        unpack_bf16x8(*reinterpret_cast<const uint4*>(arow + 8 * g8), af);
+#pragma unroll
+                        for (int i = 0; i < 8; ++i) {
+                            const float a = __uint_as_float(v[8 * g8 + i]);
+                            const bool in = n + 8 * g8 + i < p.N;   // columns past N: padding
+                            dg_acc += in ? a * af[i] : 0.f;
+                            f[i] = in ? sc * a * gelu_grad(uf[i]) : 0.f;
+                        }
+                        uint4 u;
+                        u.x = pack_bf16x2(f[0], f[1]);
+                        u.y = pack_bf16x2(f[2], f[3]);
+                        u.z = pack_bf16x2(f[4], f[5]);
+                        u.w = pack_bf16x2(f[6], f[7]);
+                        *reinterpret_cast<uint4*>(orow + 8 * g8) = u;
+                    }
+                    continue;
+                }
 #pragma unroll
                 for (int g8 = 0; g8 < 4; ++g8) {
                     if (n + 8 * g8 >= p.N) break;
                     float f[8];
 #pragma unroll
                     for (int i = 0; i < 8; ++i) f[i] = __uint_as_float(v[8 * g8 + i]);
-                    if (p.epi == EPI_GELU_BF16) {
+                    if (p.epi == EPI_GELU2_BF16) {   // the pre-activation as well
+                        uint4 u;
+                        u.x = pack_bf16x2(f[0], f[1]);
+                        u.y = pack_bf16x2(f[2], f[3]);
+                        u.z = pack_bf16x2(f[4], f[5]);
+                        u.w = pack_bf16x2(f[6], f[7]);
+                        *reinterpret_cast<uint4*>(p.out2 + (int64_t)gr * p.ldo + n + 8 * g8) = u;
+                    }
+                    if (p.epi == EPI_GELU_BF16 || p.epi == EPI_GELU2_BF16) {
 #pragma unroll
                         for (int i = 0; i < 8; i += 2) gelu_erf2(f[i], f[i + 1]);
                     }
@@ -760,6 +837,8 @@ __device__ void epilogue(const GemmArgs& p, const Smem& sm, uint32_t tmem, int64
                 }
             }
         }
+        if (!to_f32 && p.epi == EPI_DGELU_BF16 && ok_row)   // the row dot, per n-tile and warp half
+            p.dg_part[(int64_t)(2 * (t.n0 / p.n_step) + half) * p.m_total + gr] = dg_acc;
     }
 }
 
@@ -947,6 +1026,20 @@ bool make_weight_tmap(CUtensorMap* tm, const void* base, int64_t N, int64_t K, i
     return make_weight_tmap_strided(tm, base, N, K, G, N, N * K);
 }
 
+bool make_kmajor_tmap(CUtensorMap* tm, const void* base, int64_t K, int64_t N, int64_t G, int64_t k_ld,
+                      int64_t g_ld, int box_n) {
+    PFN_cuTensorMapEncodeTiled_v12000 enc = get_encode_fn();
+    if (!enc || box_n < 8 || box_n > 256) return false;
+    cuuint64_t dims[3] = {(cuuint64_t)K, (cuuint64_t)N, (cuuint64_t)G};
+    cuuint64_t strides[2] = {(cuuint64_t)k_ld * 2, (cuuint64_t)g_ld * 2};
+    cuuint32_t box[3] = {GM_BK, (cuuint32_t)box_n, 1};
+    cuuint32_t estr[3] = {1, 1, 1};
+    CUresult r = enc(tm, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(base), dims, strides, box,
+                     estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                     CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    return r == CUDA_SUCCESS;
+}
+
 bool make_rows_tmap(CUtensorMap* tm, const void* base, int64_t cols, int64_t rows, int64_t ld) {
     PFN_cuTensorMapEncodeTiled_v12000 enc = get_encode_fn();
     if (!enc) return false;
@@ -978,7 +1071,8 @@ cudaError_t launch_grouped_gemm(const GemmArgs& a, int grid, cudaStream_t s) {
         grouped_gemm_kernel<32, false, ECLS_F32>, grouped_gemm_kernel<32, false, ECLS_BF16>,
         grouped_gemm_kernel<32, true, ECLS_BF16>};
     const bool gathered = a.a_rows || a.a_ident;   // A rows through the gather warps
-    const bool bf16_out = a.epi == EPI_GELU_BF16 || a.epi == EPI_STORE_BF16 || a.epi == EPI_SWIGLU_BF16;
+    const bool bf16_out = a.epi == EPI_GELU_BF16 || a.epi == EPI_STORE_BF16 || a.epi == EPI_SWIGLU_BF16 ||
+                          a.epi == EPI_GELU2_BF16 || a.epi == EPI_DGELU_BF16;
     if (gathered && !bf16_out) return cudaErrorInvalidValue;
     if (!gathered && a.epi == EPI_SWIGLU_BF16) return cudaErrorInvalidValue;
     Kern kern;

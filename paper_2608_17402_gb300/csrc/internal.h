@@ -204,6 +204,9 @@ enum Epilogue : int {
                          //   W3 (up, the second CTA's); 128 output columns per n-tile
     EPI_SUM2_F32 = 4,    // yacc[tok(r), n]  = scale(r) * (acc[n] + acc[n + N/2]), n < N/2
                          //   (two column groups summed; one n-tile)
+    EPI_GELU2_BF16 = 6,  // out[r, n] = bf16(GELU(acc)), out2[r, n] = bf16(acc) (the pre-activation)
+    EPI_DGELU_BF16 = 7,  // out[r, n] = bf16(scale(r) acc GELU'(u[r, n])), and the row dot
+                         //   sum_n acc a[r, n] (a = GELU(u)) in partials dg_part[2 nt + half][r]
 };
 static_assert(EPI_ADD_F32 == 2, "gm_stages / gm_smem_bytes test the reduction epilogue by value");
 // Epilogue classes of the grouped GEMM's kernel instances: bf16 outputs (GELU, SwiGLU,
@@ -258,6 +261,21 @@ struct GemmArgs {
     int wn_nparts, wn_E, wn_Ep; //   q < wn_sets and e < wn_E, wn_out[q wn_E + e] =
     int wn_sets;                //   sqrt(sum_p wn_part[(q wn_nparts + p) wn_Ep + e])
     float* wn_out;              //   (the router's |W_r[:, e]| and |lo_e| from per-CTA partial sums)
+    // Operand layouts and work items of the training path (all 0 on the forward):
+    int b_kmajor;               // B stored K-major, W[G][N][K] (K contiguous): tmB is the 3-D map
+                                //   {K, N, G} with box {64, BN/2, 1}; the shared tile holds BN/2
+                                //   rows of 128 bytes like A's
+    int a_mn;                   // A stored M-major, A[K][M] (M contiguous): tmA is the 3-D map
+                                //   {M, K, 1} with box {64, 64, 1}, two boxes per CTA and stage
+    int wg_M;                   // item_table == 2: weight-gradient items {g, m0 | n0 << 16, kb0,
+                                //   kb1} (absolute k-blocks of the rows both operands share);
+                                //   output row of (g, m) is g wg_M + m, B's map has one group
+    int a_neg_zero;             // gathered rows with a negative table entry are zero rows (padding)
+    int o_neg_skip;             // fp32 outputs: rows with a negative output token are padding, skipped
+    __nv_bfloat16* out2;        // EPI_GELU2_BF16: the pre-activation, laid out as out
+    const __nv_bfloat16* epi_u; // EPI_DGELU_BF16: pre-activations u and activations GELU(u) of
+    const __nv_bfloat16* epi_a; //   the GEMM rows, [m_total][ldo] bf16
+    float* dg_part;             // EPI_DGELU_BF16: per-row partial dots, [2 n_ntiles][m_total] fp32
     DevStatus* status;
     uint64_t limit_ns;
 };
@@ -271,9 +289,45 @@ bool make_weight_tmap_strided(CUtensorMap* tm, const void* base, int64_t N, int6
 // Encodes the 2-D row tensor map {cols, rows} of A[rows][cols] bf16 (row stride ld
 // elements), box {64, GM_HALF}.
 bool make_rows_tmap(CUtensorMap* tm, const void* base, int64_t cols, int64_t rows, int64_t ld);
+// The 3-D map {K, N, G} of a K-major operand W[G][N][K] bf16 (row stride k_ld, group
+// stride g_ld elements, multiples of 8), box {64, box_n, 1}.
+bool make_kmajor_tmap(CUtensorMap* tm, const void* base, int64_t K, int64_t N, int64_t G, int64_t k_ld,
+                      int64_t g_ld, int box_n);
 // Picks BN (multiple of 32, <= 256) and the number of N tiles for width N.
 void choose_bn(int N, int* BN, int* n_ntiles);
 cudaError_t launch_grouped_gemm(const GemmArgs& a, int grid, cudaStream_t s);
+
+// ------------------------------------------------------- training path
+
+// k-blocks (of 64 rows) per weight-gradient work item at most.
+constexpr int64_t BWD_KCH = 64;
+// Per token: sig[t k + j] = sigmoid(x_t . W_r[:, idx[t k + j]]) (fp32, from the transposed
+// copy wrt [E][dp]) and gate = sig / sum_j sig (k <= 32).
+cudaError_t launch_bwd_gates(const __nv_bfloat16* x, const float* wrt, int dp, const int32_t* idx, int64_t T,
+                             int d, int E, int k, float* sig, float* gate, DevStatus* st, cudaStream_t s);
+// poff[E + 1]: exclusive prefix of counts rounded up to multiples of 64 (E <= 1024).
+cudaError_t launch_bwd_pad(const int32_t* counts, int E, int32_t* poff, cudaStream_t s);
+// Padded rows: ptok / pgate of every padded row (-1 / 0 for padding) and the padded row
+// of every routing slot (from the stable expert-major rows inv and offsets).
+cudaError_t launch_bwd_rows(const int32_t* idx, const int32_t* inv, const int32_t* counts,
+                            const int32_t* offsets, const int32_t* poff, const float* gate, int64_t n_slots,
+                            int k, int E, int32_t* ptok, float* pgate, int32_t* slot_prow, cudaStream_t s);
+// Weight-gradient work items (see bwd_items_kernel) and a bound on their number for
+// groups holding `rows` rows in total.
+int64_t bwd_max_items(int64_t rows, int G, int M, int N, int BN);
+cudaError_t launch_bwd_items(const int32_t* koff, int G, int64_t K_rows, int M, int N, int BN,
+                             int max_items, int4* items, int32_t* n_items, DevStatus* st, cudaStream_t s);
+// xp[r] = x[ptok[r]], gdy[r] = pgate[r] dy[ptok[r]] over the poff[E] padded rows.
+cudaError_t launch_bwd_gather(const __nv_bfloat16* x, const __nv_bfloat16* dy, const int32_t* ptok,
+                              const float* pgate, const int32_t* poff, int E, int d, int64_t max_rows,
+                              __nv_bfloat16* xp, __nv_bfloat16* gdy, cudaStream_t s);
+// Router backward per token (Eqs. 4-5): ds, dx += ds W_r^T, ds into [T][Ep] bf16.
+cudaError_t launch_bwd_router(const int32_t* idx, const float* sig, const float* gate, const int32_t* slot_prow,
+                              const float* dg_part, int nparts, int64_t part_stride, const float* wrt, int dp,
+                              int64_t T, int d, int E, int k, int Ep, float* dx, __nv_bfloat16* ds,
+                              cudaStream_t s);
+cudaError_t launch_bwd_copy(const float* src, int64_t ld_src, float* dst, int64_t rows, int64_t cols,
+                            cudaStream_t s);
 
 // ---------------------------------------- permute without a caller workspace
 

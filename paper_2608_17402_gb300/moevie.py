@@ -27,7 +27,7 @@ C_ENTRY_POINTS = ("moevie_status_string", "moevie_version", "moevie_workspace_si
                   "moevie_expert_ffn",
                   "moevie_shared_expert", "moevie_combine", "moevie_moe_forward",
                   "moevie_get_device_status", "moevie_launch_count", "moevie_shared_groups",
-                  "moevie_update_bias",
+                  "moevie_update_bias", "moevie_backward_workspace_size", "moevie_moe_backward",
                   "moevie_test_route_logits",
                   "moevie_test_fallback_count", "moevie_test_expert_hidden",
                   "moevie_test_moe_forward_events", "moevie_test_wait_timeout")
@@ -78,6 +78,8 @@ def load():
         "moevie_launch_count": ([], ctypes.c_uint64),
         "moevie_shared_groups": ([I64] * 6, ctypes.c_int64),
         "moevie_update_bias": ([P, I64, F, ctypes.c_int, P, P, SZ, P], ctypes.c_int),
+        "moevie_backward_workspace_size": ([I64] * 5 + [P], ctypes.c_int),
+        "moevie_moe_backward": ([P, P, P, I64, P, P, P, P, P, P, SZ, P], ctypes.c_int),
         "moevie_test_route_logits": ([P, P, I64, I64, I64, P, P, SZ, P], ctypes.c_int),
         "moevie_test_fallback_count": ([P, P, P], ctypes.c_int),
         "moevie_test_expert_hidden": ([P, P, P, P, I64, I64, I64, I64, I64, P, P, SZ, P],
@@ -328,6 +330,43 @@ def moevie_moe_forward(layer: LayerWeights, x, ws: Workspace, y=None, routing=Fa
           ctypes.byref(rstruct) if rstruct is not None else None, ws.ptr, ws.nbytes,
           _stream(stream))
     return (y, rt) if routing else y
+
+
+def moevie_backward_workspace_size(T_max, d, E, k, h) -> int:
+    out = ctypes.c_size_t(0)
+    _call("moevie_backward_workspace_size", T_max, d, E, k, h, ctypes.byref(out))
+    return out.value
+
+
+class BackwardWorkspace(Workspace):
+    """Caller-owned device scratch of moevie_moe_backward (up to ``T_max`` tokens)."""
+
+    def __init__(self, T_max, d, E, k, h, device="cuda", stream=None):
+        self.dims = (T_max, d, E, k, h)
+        self.nbytes = moevie_backward_workspace_size(T_max, d, E, k, h)
+        self.buf = torch.empty(self.nbytes, dtype=torch.uint8, device=device)
+        moevie_workspace_init(self, stream)
+
+
+def moevie_moe_backward(layer: LayerWeights, x, dy, idx, ws: "BackwardWorkspace", stream=None):
+    """Gradients of sum(dy * y) with the selection idx held fixed (GELU experts, no
+    shared expert).  Returns a dict of fp32 tensors: dx [T, d], dW_r [d, E], dW1
+    [E, d, h] (a view of rows row_ld(h) apart), dW2 [E, h, d]."""
+    _want(x, torch.bfloat16, "x")
+    _want(dy, torch.bfloat16, "dy")
+    _want(idx, torch.int32, "idx")
+    T, d = x.shape
+    _, E, k, h, _ = layer.dims
+    dev = x.device
+    out = {"dx": torch.empty((T, d), dtype=torch.float32, device=dev),
+           "dW_r": torch.empty((d, E), dtype=torch.float32, device=dev),
+           "dW1": torch.empty((E, d, row_ld(h)), dtype=torch.float32, device=dev),
+           "dW2": torch.empty((E, h, d), dtype=torch.float32, device=dev)}
+    L = layer.c_struct()
+    _call("moevie_moe_backward", ctypes.byref(L), _p(x), _p(dy), T, _p(idx), _p(out["dx"]), _p(out["dW_r"]),
+          _p(out["dW1"]), _p(out["dW2"]), ws.ptr, ws.nbytes, _stream(stream))
+    out["dW1"] = out["dW1"][..., :h]
+    return out
 
 
 def moevie_launch_count() -> int:

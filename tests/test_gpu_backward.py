@@ -1,0 +1,138 @@
+"""Training path (App. B: grouped GEMMs with the activation as its own step) of
+moevie_moe_backward against the oracle's backward (the gradients of sum_t dy_t . y_t
+with the top-k selection held fixed, through the renormalised gates of Eqs. 4-5 into
+W_r and x; the bias gets none), element by element, on the same seeded inputs and
+the same bf16 dy.  Tolerance as for the forward (rel-L2 <= 1e-2, max |err| <= 5e-2 RMS)
+per gradient: the GEMM operands are bf16 (u, GELU(u), du, g dy, ds), accumulation fp32."""
+import numpy as np
+import pytest
+
+import oracle
+import workloads
+from paper_2608_17402_gb300 import moevie
+from tests._gpu import assert_close, check_status, dev, dev_bf16, layer_to_device, to_np_f64
+
+pytestmark = pytest.mark.gpu
+
+
+def _dy(T, d, seed, tokens=None):
+    """bf16 dy (bits) and its exact fp64 value; nonzero only on `tokens` when given."""
+    rng = np.random.default_rng(seed)
+    f = rng.standard_normal((T, d)).astype(np.float32)
+    if tokens is not None:
+        mask = np.zeros(T, bool)
+        mask[tokens] = True
+        f[~mask] = 0.0
+    bits = workloads.f32_to_bf16_bits(f)
+    return bits, workloads.bf16_bits_to_f32(bits).astype(np.float64)
+
+
+def _gpu_backward(lay, dy_bits, idx):
+    c = lay.cfg
+    x, W = layer_to_device(lay)
+    ws = moevie.BackwardWorkspace(c.T, c.d, c.E, c.k, c.h)
+    g = moevie.moevie_moe_backward(W, x, dev_bf16(dy_bits), dev(np.ascontiguousarray(idx, np.int32)), ws)
+    check_status(ws)
+    return {k: to_np_f64(v) for k, v in g.items()}
+
+
+def _compare(got, want, label):
+    out = {}
+    for g_name, o_name in (("dx", "dx"), ("dW_r", "dWr"), ("dW1", "dW1"), ("dW2", "dW2")):
+        if not np.any(want[o_name]):   # e.g. dW_r with one expert: exactly zero
+            assert not np.any(got[g_name]), f"{label} {g_name}: expected exact zeros"
+            continue
+        rel, mx = assert_close(got[g_name], want[o_name], f"{label} {g_name}")
+        out[g_name] = (rel, mx)
+    return out
+
+
+@pytest.mark.parametrize("T,d,E,k,h", [
+    (300, 256, 16, 4, 128), (257, 128, 8, 2, 416), (130, 192, 8, 8, 64), (1, 64, 4, 2, 64),
+    (200, 96, 12, 3, 100),   # h % 8 == 4: rows of W1, H and dW1 padded to 104
+    (64, 64, 1, 1, 48),      # one expert: the gates are 1, W_r gets exactly zero gradient
+    (600, 512, 33, 5, 256),  # E not a multiple of 32, several m-tiles per expert
+])
+def test_backward_small(T, d, E, k, h):
+    cfg = workloads.small_config(T, d, E, k, h, seed=T + h)
+    lay = workloads.make_layer(cfg)
+    dy_bits, dyf = _dy(T, d, T + 1)
+    idx, _, _ = oracle.route(lay.x, lay.Wr, lay.b, k)
+    want = oracle.backward(lay.x, lay.Wr, lay.b, lay.W1, lay.W2, k, dyf)
+    got = _gpu_backward(lay, dy_bits, idx)
+    _compare(got, want, f"T={T} d={d} E={E} k={k} h={h}")
+
+
+def test_backward_batch1_layer_every_token():
+    """The batch-1 layer (T = 1024, d = 1536, E = 64, k = 8, h = 768) on every token."""
+    lay = workloads.make_layer(workloads.CONFIGS["c2"])
+    c = lay.cfg
+    dy_bits, dyf = _dy(c.T, c.d, 5)
+    idx, _, _ = oracle.route(lay.x, lay.Wr, lay.b, c.k)
+    want = oracle.backward(lay.x, lay.Wr, lay.b, lay.W1, lay.W2, c.k, dyf)
+    r = _compare(_gpu_backward(lay, dy_bits, idx), want, "c2")
+    print("c2 backward:", {k: f"rel-L2 {v[0]:.2e}, max|err|/RMS {v[1]:.2e}" for k, v in r.items()})
+
+
+def test_backward_stress_layer_sampled_tokens():
+    """The stress layer (T = 65536, E = 256, one saturated expert) at full size with dy
+    nonzero on 64 tokens chosen across the token range: the oracle's backward costs only
+    those tokens, and every gradient (all of dx, dW_r, dW1, dW2) must match it, the rows
+    of the other tokens exactly zero in dx."""
+    lay = workloads.make_layer(workloads.CONFIGS["c4"])
+    c = lay.cfg
+    rng = np.random.default_rng(3)
+    toks = np.unique(np.concatenate([[0, c.T - 1], rng.choice(c.T, 62, replace=False)]))
+    dy_bits, dyf = _dy(c.T, c.d, 9, toks)
+    idx, _, _ = oracle.route(lay.x, lay.Wr, lay.b, c.k)
+    want = oracle.backward(lay.x, lay.Wr, lay.b, lay.W1, lay.W2, c.k, dyf)
+    got = _gpu_backward(lay, dy_bits, idx)
+    others = np.setdiff1d(np.arange(c.T), toks)
+    assert not np.any(got["dx"][others])
+    # with 64 of 65536 tokens the gradients are very uneven (the saturated expert takes all
+    # 64, most others one or two): compare dx on those tokens, and the expert weight
+    # gradients expert by expert, each against its own RMS.  An expert reached by fewer
+    # than 8 of the tokens has a weight gradient of rank below 8 (a sum of outer products
+    # x_t du_t, or a_t (g dy_t)), whose largest element exceeds its RMS by about the
+    # product of the two vectors' peak-to-RMS ratios (20-30); the bf16 rounding of the
+    # operands (2^-9 relative each) then reaches 5-10% of the RMS at those elements, so
+    # such slices keep the relative L2 bound of 1e-2 but take 0.25 x RMS as a guard against
+    # gross errors for the largest one (a wrong element is off by about its own value,
+    # tens of RMS there).
+    rows = np.bincount(idx[toks].ravel(), minlength=c.E)
+    rel, mx = assert_close(got["dx"][toks], want["dx"][toks], "c4 dx")
+    worst = {"dx": (rel, mx)}
+    rel, mx = assert_close(got["dW_r"], want["dWr"], "c4 dW_r")
+    worst["dW_r"] = (rel, mx)
+    for g_name, o_name in (("dW1", "dW1"), ("dW2", "dW2")):
+        w = (0.0, 0.0)
+        for e in range(c.E):
+            if not np.any(want[o_name][e]):
+                assert not np.any(got[g_name][e]), f"c4 {g_name}[{e}]: expected exact zeros"
+                continue
+            if rows[e] >= 8:
+                rel, mx = assert_close(got[g_name][e], want[o_name][e], f"c4 {g_name}[{e}]")
+            else:
+                ge, we = got[g_name][e], want[o_name][e]
+                rel = float(np.linalg.norm(ge - we) / np.linalg.norm(we))
+                mx = float(np.abs(ge - we).max() / np.sqrt(np.mean(we ** 2)))
+                assert rel <= 1e-2 and mx <= 0.25, (g_name, e, int(rows[e]), rel, mx)
+            w = (max(w[0], rel), max(w[1], mx))
+        worst[g_name] = w
+    print("c4 backward (64 tokens; worst expert):",
+          {k: f"rel-L2 {v[0]:.2e}, max|err|/RMS {v[1]:.2e}" for k, v in worst.items()})
+
+
+def test_backward_rejects_unsupported_layers():
+    """SwiGLU experts and a shared expert are outside this entry point: rejected before
+    any launch."""
+    cfg = workloads.small_config(16, 64, 4, 2, 64, h_s=64)
+    lay = workloads.make_layer(cfg)
+    x, W = layer_to_device(lay)
+    ws = moevie.BackwardWorkspace(16, 64, 4, 2, 64)
+    idx = dev(np.zeros((16, 2), np.int32) + np.array([0, 1], np.int32))
+    n0 = moevie.moevie_launch_count()
+    with pytest.raises(moevie.MoevieError) as e:
+        moevie.moevie_moe_backward(W, x, x, idx, ws)
+    assert e.value.code == 2
+    assert moevie.moevie_launch_count() == n0
