@@ -348,10 +348,47 @@ def measure_config(cfg, args, world, local, with_clocks):
     code, detail = moevie.moevie_get_device_status(ws)
     if code != 0:
         raise RuntimeError(f"device status {code} {detail}")
+    bwd = None
+    if cfg.act == "gelu" and cfg.h_s == 0:   # the training path (GELU experts, no shared expert)
+        bwd = measure_backward(cfg, W, x, rt["idx"], args, flush, stream)
     del ws, flush, W, x, y
     torch.cuda.empty_cache()
     return {"ms": ms, "e2e_ms": e2e_ms, "stages": stages, "work": work, "launches": int(launches),
-            "clocks": None if clk is None else clk.summary()}, lay
+            "clocks": None if clk is None else clk.summary(), "backward": bwd}, lay
+
+
+def measure_backward(cfg, W, x, idx, args, flush, stream):
+    """CUDA-event time of moevie_moe_backward (inputs resident, L2 flushed between calls)
+    and its GEMM rate: five grouped GEMMs of 2 T k d h FLOPs each (up-projection again,
+    dy W2^T, du W1^T, dW2, dW1) plus dW_r = x^T ds (2 T d E)."""
+    import torch
+
+    from paper_2608_17402_gb300 import moevie
+    T, d, E, k, h = cfg.T, cfg.d, cfg.E, cfg.k, cfg.h
+    g = torch.Generator(device="cuda")
+    g.manual_seed(cfg.seed + 17)
+    dy = torch.randn((T, d), generator=g, device="cuda").to(torch.bfloat16)
+    bws = moevie.BackwardWorkspace(T, d, E, k, h)
+    steps = max(1, min(args.steps, 10))
+    for _ in range(max(1, min(args.warmup, 3))):
+        moevie.moevie_moe_backward(W, x, dy, idx, bws)
+    torch.cuda.synchronize()
+    st = [torch.cuda.Event(enable_timing=True) for _ in range(steps)]
+    en = [torch.cuda.Event(enable_timing=True) for _ in range(steps)]
+    for i in range(steps):
+        flush.zero_()
+        st[i].record(stream)
+        moevie.moevie_moe_backward(W, x, dy, idx, bws)
+        en[i].record(stream)
+    torch.cuda.synchronize()
+    code, detail = moevie.moevie_get_device_status(bws)
+    if code != 0:
+        raise RuntimeError(f"backward device status {code} {detail}")
+    ms = statistics.mean(a.elapsed_time(b) for a, b in zip(st, en))
+    flops = 10.0 * T * k * d * h + 2.0 * T * d * E
+    del bws, dy
+    return {"us": ms * 1e3, "flops": flops, "tflops": flops / (ms / 1e3) / 1e12, "steps": steps,
+            "what": "moevie_moe_backward: dx, dW_r, dW1, dW2 of sum(dy . y), selection held fixed"}
 
 
 def summarise(cfg, m, pk, world):
@@ -398,6 +435,8 @@ def run_ours(args, rank, world):
                            "stages_us": {k: v * 1e3 for k, v in mc["stages"].items()},
                            "memory_bound": memory_bound_stages(c2, mc["stages"], peaks()),
                            "e2e_tokens_per_s": c2.T / (mc["e2e_ms"] / 1e3)}
+            if mc.get("backward"):
+                extra[name]["backward"] = mc["backward"]
     if rank != 0:
         return
 
@@ -421,6 +460,8 @@ def run_ours(args, rank, world):
         "gpu_launches": m["launches"],
         "clocks": m["clocks"],
     }
+    if m.get("backward"):
+        out["backward"] = m["backward"]
     if extra:
         out["per_config"] = extra
     if world == 1 and not args.no_cpu_baseline:

@@ -305,7 +305,7 @@ __device__ __forceinline__ int rows_half(const Tile& t, uint32_t rank) {
 
 // TMA producer (warp 9, lane 0): the CTA's half of B, and A when its rows are
 // contiguous.  The leader posts the byte count of both CTAs on its full barrier.
-template <bool GATHER>
+template <bool GATHER, bool TRAIN>
 __device__ void producer_tma(const GemmArgs& p, const Smem& sm, int64_t n_work,
                              volatile int* abort_flag) {
     tma_prefetch_desc(&p.tmB);
@@ -320,7 +320,7 @@ __device__ void producer_tma(const GemmArgs& p, const Smem& sm, int64_t n_work,
     const uint32_t nboxh = (half_n + 63) / 64;
     // B per CTA and stage: nboxh boxes of 64 columns x 64 K rows (N-major), or half_n rows
     // of 64 K values (K-major)
-    const uint32_t b_bytes = p.b_kmajor ? half_n * 128u : nboxh * GM_BK * 128;
+    const uint32_t b_bytes = (TRAIN && p.b_kmajor) ? half_n * 128u : nboxh * GM_BK * 128;
     const uint32_t cta_bytes = b_bytes + (gather ? 0u : (uint32_t)GM_A_BYTES);
     // gathering: plus the 16-byte signal with which the peer publishes its A half
     const uint32_t stage_tx = 2 * cta_bytes + (gather ? 16u : 0u);
@@ -340,7 +340,7 @@ __device__ void producer_tma(const GemmArgs& p, const Smem& sm, int64_t n_work,
         const CUtensorMap* tmb = tail ? &p.tmB2 : &p.tmB;
         if (p.swiglu)
             tmb = sm.rank == 1 ? (tail ? &p.tmB4 : &p.tmB2) : (tail ? &p.tmB3 : &p.tmB);
-        const int gb = p.item_table == 2 ? 0 : (tail ? t.g - p.g_split : t.g);
+        const int gb = (TRAIN && p.item_table == 2) ? 0 : (tail ? t.g - p.g_split : t.g);
         const int ncol0 = p.swiglu ? t.n0 : t.n0 + (int)(sm.rank * half_n);
         for (int kb = t.kb0; kb < t.kb1; ++kb) {
             if (!mbar_wait(sm.empty + 8 * s, ph ^ 1u, p.limit_ns, abort_flag)) {
@@ -351,14 +351,14 @@ __device__ void producer_tma(const GemmArgs& p, const Smem& sm, int64_t n_work,
             if (sm.rank == 0) mbar_arrive_expect_tx(sm.full + 8 * s, stage_tx);
             const uint32_t b_dst = sm.b0 + s * GM_B_BYTES;
             const int kk = kb * GM_BK;
-            if (p.b_kmajor) {   // half_n rows of the CTA's columns, 64 K values each
+            if (TRAIN && p.b_kmajor) {   // half_n rows of the CTA's columns, 64 K values each
                 tma_load_3d_pair(b_dst, tmb, bar, kk, ncol0, gb);
             } else {
                 for (uint32_t j = 0; j < nboxh; ++j)
                     tma_load_3d_pair(b_dst + j * (GM_BK * 128), tmb, bar, ncol0 + (int)(64 * j), kk, gb);
             }
             if (!gather) {
-                if (p.a_mn) {   // two 64-row halves of the CTA's 128 output rows, 64 K rows each
+                if (TRAIN && p.a_mn) {   // two 64-row halves of the CTA's 128 output rows, 64 K rows each
                     const int m = t.m0 + (int)sm.rank * GM_HALF;
                     tma_load_3d_pair(sm.a0 + s * GM_A_BYTES, &p.tmA, bar, m, kk, 0);
                     tma_load_3d_pair(sm.a0 + s * GM_A_BYTES + GM_BK * 128, &p.tmA, bar, m + 64, kk, 0);
@@ -522,15 +522,17 @@ __device__ void gather_forwarder(const GemmArgs& p, const Smem& sm, int64_t n_wo
 // ------------------------------------------------------------------- MMA
 
 // Leader CTA, warp 8, lane 0.
+template <bool TRAIN>
 __device__ void mma_issuer(const GemmArgs& p, const Smem& sm, uint32_t tmem, int64_t n_work,
                            volatile int* abort_flag) {
-    const uint32_t idesc = idesc_bf16_f32(2 * GM_HALF, p.BN, p.a_mn != 0, p.b_kmajor == 0);
     // K-major operands: k-slice +32 B; MN-major operands: next 64-element atom LBO 8192,
-    // k-slice +2048 B (16 K rows of 128 bytes)
-    const uint64_t adesc0 = p.a_mn ? smem_desc_sw128(sm.a0, 8192, 1024) : smem_desc_sw128(sm.a0, 16, 1024);
-    const uint64_t bdesc0 = p.b_kmajor ? smem_desc_sw128(sm.b0, 16, 1024) : smem_desc_sw128(sm.b0, 8192, 1024);
-    const uint32_t a_step = p.a_mn ? (2048 >> 4) : (32 >> 4);
-    const uint32_t b_step = p.b_kmajor ? (32 >> 4) : (2048 >> 4);
+    // k-slice +2048 B (16 K rows of 128 bytes).  The forward's A is K-major, its B MN-major.
+    const bool a_mn = TRAIN && p.a_mn, b_km = TRAIN && p.b_kmajor;
+    const uint32_t idesc = idesc_bf16_f32(2 * GM_HALF, p.BN, a_mn, !b_km);
+    const uint64_t adesc0 = a_mn ? smem_desc_sw128(sm.a0, 8192, 1024) : smem_desc_sw128(sm.a0, 16, 1024);
+    const uint64_t bdesc0 = b_km ? smem_desc_sw128(sm.b0, 16, 1024) : smem_desc_sw128(sm.b0, 8192, 1024);
+    const uint32_t a_step = a_mn ? (2048 >> 4) : (32 >> 4);
+    const uint32_t b_step = b_km ? (32 >> 4) : (2048 >> 4);
     static_assert(GM_BK == 64, "four k-slices of 16 per stage");
     int s = 0;
     uint32_t ph = 0;
@@ -628,7 +630,7 @@ __device__ __forceinline__ void reduce_chunk(const GemmArgs& p, float* stg_all, 
 // per-warp staging buffer so that each 16-byte vector reduction instruction of a
 // warp covers four rows x 128 contiguous bytes, i.e. whole L2 lines.  When a warp has read
 // its last chunk of the accumulator it arrives (once) on the leader's tempty barrier.
-template <int STG_ROWS, bool GATHER, int ECLS>
+template <int STG_ROWS, bool GATHER, int ECLS, bool TRAIN>
 __device__ void epilogue(const GemmArgs& p, const Smem& sm, uint32_t tmem, int64_t n_work,
                          volatile int* abort_flag) {
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -776,7 +778,7 @@ __device__ void epilogue(const GemmArgs& p, const Smem& sm, uint32_t tmem, int64
             const int n = t.n0 + c0;
             if constexpr (!to_f32) {
                 __nv_bfloat16* orow = p.out + (int64_t)gr * p.ldo + n;
-                if (p.epi == EPI_DGELU_BF16) {   // training path: du = scale acc GELU'(u), dot acc . a
+                if (TRAIN && p.epi == EPI_DGELU_BF16) {   // training path: du = scale acc GELU'(u), dot acc . a
                     const __nv_bfloat16* urow = p.epi_u + (int64_t)gr * p.ldo + n;
                     const __nv_bfloat16* arow = p.epi_a + (int64_t)gr * p.ldo + n;
 #pragma unroll
@@ -807,7 +809,7 @@ __device__ void epilogue(const GemmArgs& p, const Smem& sm, uint32_t tmem, int64
                     float f[8];
 #pragma unroll
                     for (int i = 0; i < 8; ++i) f[i] = __uint_as_float(v[8 * g8 + i]);
-                    if (p.epi == EPI_GELU2_BF16) {   // the pre-activation as well
+                    if (TRAIN && p.epi == EPI_GELU2_BF16) {   // the pre-activation as well
                         uint4 u;
                         u.x = pack_bf16x2(f[0], f[1]);
                         u.y = pack_bf16x2(f[2], f[3]);
@@ -815,7 +817,7 @@ __device__ void epilogue(const GemmArgs& p, const Smem& sm, uint32_t tmem, int64
                         u.w = pack_bf16x2(f[6], f[7]);
                         *reinterpret_cast<uint4*>(p.out2 + (int64_t)gr * p.ldo + n + 8 * g8) = u;
                     }
-                    if (p.epi == EPI_GELU_BF16 || p.epi == EPI_GELU2_BF16) {
+                    if (p.epi == EPI_GELU_BF16 || (TRAIN && p.epi == EPI_GELU2_BF16)) {
 #pragma unroll
                         for (int i = 0; i < 8; i += 2) gelu_erf2(f[i], f[i + 1]);
                     }
@@ -837,14 +839,14 @@ __device__ void epilogue(const GemmArgs& p, const Smem& sm, uint32_t tmem, int64
                 }
             }
         }
-        if (!to_f32 && p.epi == EPI_DGELU_BF16 && ok_row)   // the row dot, per n-tile and warp half
+        if (TRAIN && !to_f32 && p.epi == EPI_DGELU_BF16 && ok_row)   // the row dot, per n-tile and warp half
             p.dg_part[(int64_t)(2 * (t.n0 / p.n_step) + half) * p.m_total + gr] = dg_acc;
     }
 }
 
 // STG_ROWS: rows per warp of the reduction staging buffer (EPI_ADD_F32), one kernel
 // instance each so that the epilogue loops have constant trip counts.
-template <int STG_ROWS, bool GATHER, int ECLS>
+template <int STG_ROWS, bool GATHER, int ECLS, bool TRAIN>
 __global__ void __launch_bounds__(GM_THREADS, 1) grouped_gemm_kernel(const __grid_constant__ GemmArgs p) {
     extern __shared__ uint8_t gm_smem_raw[];
     uint8_t* smem = reinterpret_cast<uint8_t*>(
@@ -915,11 +917,11 @@ __global__ void __launch_bounds__(GM_THREADS, 1) grouped_gemm_kernel(const __gri
     const int64_t n_work = p.item_table ? n_mtiles * p.ksplit : n_mtiles * p.n_ntiles * p.ksplit;
 
     if (warp < GM_EPI_WARPS) {
-        epilogue<STG_ROWS, GATHER, ECLS>(p, sm, tmem, n_work, abort_flag);
+        epilogue<STG_ROWS, GATHER, ECLS, TRAIN>(p, sm, tmem, n_work, abort_flag);
     } else if (warp == GM_WARP_MMA) {
-        if ((threadIdx.x & 31) == 0 && sm.rank == 0) mma_issuer(p, sm, tmem, n_work, abort_flag);
+        if ((threadIdx.x & 31) == 0 && sm.rank == 0) mma_issuer<TRAIN>(p, sm, tmem, n_work, abort_flag);
     } else if (warp == GM_WARP_LOAD) {
-        if ((threadIdx.x & 31) == 0) producer_tma<GATHER>(p, sm, n_work, abort_flag);
+        if ((threadIdx.x & 31) == 0) producer_tma<GATHER, TRAIN>(p, sm, n_work, abort_flag);
     } else if (warp == GM_WARP_FWD) {
         if constexpr (GATHER) {
             if ((threadIdx.x & 31) == 0) gather_forwarder(p, sm, n_work, abort_flag);
@@ -1063,20 +1065,30 @@ void choose_bn(int N, int* BN, int* n_ntiles) {
 
 cudaError_t launch_grouped_gemm(const GemmArgs& a, int grid, cudaStream_t s) {
     if (a.stg_rows != 32 && a.stg_rows != 16) return cudaErrorInvalidValue;
-    // one instance per (staging rows, A path, epilogue class): each holds only the code
-    // its launches run (constant trip counts, no other epilogue to crowd its registers)
+    // one instance per (staging rows, A path, epilogue class, training-path layouts): each
+    // holds only the code its launches run (constant trip counts, no other epilogue or
+    // operand layout to crowd its registers)
     using Kern = void (*)(GemmArgs);
-    static const Kern kerns[5] = {
-        grouped_gemm_kernel<32, false, ECLS_ADD>, grouped_gemm_kernel<16, false, ECLS_ADD>,
-        grouped_gemm_kernel<32, false, ECLS_F32>, grouped_gemm_kernel<32, false, ECLS_BF16>,
-        grouped_gemm_kernel<32, true, ECLS_BF16>};
+    static const Kern kerns[8] = {
+        grouped_gemm_kernel<32, false, ECLS_ADD, false>, grouped_gemm_kernel<16, false, ECLS_ADD, false>,
+        grouped_gemm_kernel<32, false, ECLS_F32, false>, grouped_gemm_kernel<32, false, ECLS_BF16, false>,
+        grouped_gemm_kernel<32, true, ECLS_BF16, false>,
+        // the training path: K-major B, M-major A, weight-gradient items, backward epilogues
+        grouped_gemm_kernel<32, true, ECLS_BF16, true>, grouped_gemm_kernel<32, false, ECLS_ADD, true>,
+        grouped_gemm_kernel<16, false, ECLS_ADD, true>};
     const bool gathered = a.a_rows || a.a_ident;   // A rows through the gather warps
+    const bool train = a.b_kmajor || a.a_mn || a.item_table == 2 || a.epi == EPI_GELU2_BF16 ||
+                       a.epi == EPI_DGELU_BF16;
     const bool bf16_out = a.epi == EPI_GELU_BF16 || a.epi == EPI_STORE_BF16 || a.epi == EPI_SWIGLU_BF16 ||
                           a.epi == EPI_GELU2_BF16 || a.epi == EPI_DGELU_BF16;
     if (gathered && !bf16_out) return cudaErrorInvalidValue;
     if (!gathered && a.epi == EPI_SWIGLU_BF16) return cudaErrorInvalidValue;
     Kern kern;
-    if (gathered) kern = kerns[4];
+    if (train) {
+        if (gathered) kern = kerns[5];
+        else if (a.epi == EPI_ADD_F32) kern = a.stg_rows == 32 ? kerns[6] : kerns[7];
+        else return cudaErrorInvalidValue;
+    } else if (gathered) kern = kerns[4];
     else if (a.epi == EPI_ADD_F32) kern = a.stg_rows == 32 ? kerns[0] : kerns[1];
     else if (a.epi == EPI_STORE_F32 || a.epi == EPI_SUM2_F32) kern = kerns[2];
     else kern = kerns[3];
