@@ -22,7 +22,9 @@ struct DevStatus {
     int site;        // which check (Site)
     int a, b;        // two values describing it
     int fb_count;    // router: tokens re-decided with exact logits in the last call
-    int pad[59];
+    int bar_count;   // grid barrier of a cooperative launch: arrivals so far (0 between barriers)
+    int bar_gen;     //   and the barrier's generation (bumped by the last arrival)
+    int pad[57];
 };
 static_assert(sizeof(DevStatus) == 256, "status block is 256 bytes");
 
@@ -39,6 +41,7 @@ enum Site : int {
     SITE_ROUTE_FALLBACK = 20,
     SITE_BIAS_COUNTS = 21,
     SITE_TIMEOUT_PROBE = 30,
+    SITE_PERMUTE_BARRIER = 31,
 };
 
 __device__ __forceinline__ void report(DevStatus* st, int code, int site, int a, int b) {
@@ -47,6 +50,45 @@ __device__ __forceinline__ void report(DevStatus* st, int code, int site, int a,
         st->a = a;
         st->b = b;
     }
+}
+
+// Grid-wide barrier of a cooperative launch (all nblocks CTAs co-resident) with a time
+// limit: the last CTA to arrive resets the count and bumps the generation; the others
+// wait for the bump for at most limit_ns.  Returns false (after recording
+// MOEVIE_ERR_TIMEOUT at `site`) when the wait ran out; the caller then stops.  The count
+// starts at 0 (a zeroed status block) and returns to 0 after every barrier.
+__device__ __forceinline__ bool grid_barrier(DevStatus* st, unsigned nblocks, uint64_t limit_ns, int site) {
+    __shared__ int s_ok;
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        volatile int* genp = &st->bar_gen;
+        const int gen = *genp;
+        __threadfence();   // this CTA's writes before its arrival
+        int ok = 1;
+        if (atomicAdd(&st->bar_count, 1) == (int)nblocks - 1) {
+            st->bar_count = 0;
+            __threadfence();
+            atomicAdd(&st->bar_gen, 1);
+        } else {
+            uint64_t t0;
+            asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t0));
+            for (uint32_t i = 1; *genp == gen; ++i) {
+                if ((i & 63u) == 0u) {
+                    uint64_t t1;
+                    asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t1));
+                    if (t1 - t0 > limit_ns) {
+                        ok = 0;
+                        report(st, MOEVIE_ERR_TIMEOUT, site, (int)blockIdx.x, gen);
+                        break;
+                    }
+                }
+            }
+        }
+        __threadfence();   // the other CTAs' writes after the barrier
+        s_ok = ok;
+    }
+    __syncthreads();
+    return s_ok != 0;
 }
 
 // Programmatic dependent launch: a kernel launched with programmatic stream

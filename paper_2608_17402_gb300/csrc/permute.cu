@@ -14,8 +14,6 @@
 //                       (warp match + per-warp running counts), and writes perm,
 //                       inv and the per-row token (pos // K) and gate.
 // Inside one expert's segment, rows keep ascending slot order t*k + j.
-#include <cooperative_groups.h>
-
 #include <atomic>
 #include <mutex>
 
@@ -241,9 +239,16 @@ __global__ void __launch_bounds__(PT) perm_scatter_kernel(
 }
 
 // The whole permute in one cooperative launch (one CTA per chunk, all resident):
-// histograms, grid sync, per-expert chunk scans (warps over experts), grid sync, then
-// every CTA forms the expert offsets in shared memory (CTA 0 also writes offsets,
-// the m-tile table and its size) and scatters its chunk.
+// histograms, grid barrier, per-expert chunk scans (warps over experts), grid barrier,
+// then every CTA forms the expert offsets in shared memory (CTA 0 also writes offsets,
+// the m-tile table and its size) and scatters its chunk.  The barriers are bounded
+// (grid_barrier: 2 s, then MOEVIE_ERR_TIMEOUT and the CTA stops).  Launched with
+// programmatic stream serialization as well: every CTA first waits (griddepcontrol.wait)
+// for the previous kernel to complete, so by the time any CTA reaches a barrier the
+// previous kernel has released its SMs and the whole cooperative grid (sized from the
+// occupancy of an idle device) is resident; the previous kernel never waits on this
+// one, so a late CTA only delays the barrier, it cannot block it.
+constexpr uint64_t PERM_BARRIER_LIMIT_NS = 2000000000ull;
 __global__ void __launch_bounds__(PT) perm_fused_kernel(
     const int32_t* __restrict__ idx, int64_t n, int k, int E, int bm, int chunk,
     const float* __restrict__ gate_flat, int32_t* __restrict__ hist, int32_t* __restrict__ counts,
@@ -251,17 +256,15 @@ __global__ void __launch_bounds__(PT) perm_fused_kernel(
     int32_t* __restrict__ perm, int32_t* __restrict__ inv, int32_t* __restrict__ row_tok,
     float* __restrict__ row_gate, DevStatus* st, int S, int64_t T, float lambda) {
     pdl_wait();
-    namespace cg = cooperative_groups;
-    cg::grid_group grid = cg::this_grid();
     extern __shared__ __align__(16) int32_t ps_smem[];
     __shared__ int s_off[1024], s_tot;
     const int nchunks = gridDim.x;
     const int lane = threadIdx.x & 31;
     perm_hist_body(idx, n, E, chunk, blockIdx.x, nchunks, hist, st, ps_smem);
-    grid.sync();
+    if (!grid_barrier(st, gridDim.x, PERM_BARRIER_LIMIT_NS, SITE_PERMUTE_BARRIER)) return;
     const int gw = (int)(((int64_t)blockIdx.x * PT + threadIdx.x) >> 5);
     for (int e = gw; e < E; e += nchunks * PW) perm_chunk_scan_warp(hist, nchunks, e, lane, counts);
-    grid.sync();
+    if (!grid_barrier(st, gridDim.x, PERM_BARRIER_LIMIT_NS, SITE_PERMUTE_BARRIER)) return;
     // exclusive offsets over the E <= 1024 experts, four per thread
     int loc[4], sum = 0;
 #pragma unroll

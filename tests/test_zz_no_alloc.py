@@ -2,6 +2,8 @@
 caller workspace) against moevie_permute, through the C ABI: identical outputs on
 two calls in a row, and oversized inputs rejected before anything is enqueued.
 This file is collected last so that it also runs after every other GPU test."""
+import gc
+
 import numpy as np
 import pytest
 import torch
@@ -78,14 +80,19 @@ def test_static_permute_allocates_nothing():
            torch.empty(T * k, dtype=torch.int32, device="cuda"))
     moevie.moevie_permute_static(idx, E, out=out)
     torch.cuda.synchronize()
-    for _ in range(2):
-        free0, _ = torch.cuda.mem_get_info()
-        alloc0 = torch.cuda.memory_allocated()
-        moevie.moevie_permute_static(idx, E, out=out)
-        torch.cuda.synchronize()
-        free1, _ = torch.cuda.mem_get_info()
-        assert free1 == free0, (free0, free1)
-        assert torch.cuda.memory_allocated() == alloc0
+    gc.collect()   # tensors left by earlier tests are freed now, not during the measurement
+    gc.disable()
+    try:
+        for _ in range(2):
+            free0, _ = torch.cuda.mem_get_info()
+            alloc0 = torch.cuda.memory_allocated()
+            moevie.moevie_permute_static(idx, E, out=out)
+            torch.cuda.synchronize()
+            free1, _ = torch.cuda.mem_get_info()
+            assert free1 == free0, (free0, free1)
+            assert torch.cuda.memory_allocated() == alloc0
+    finally:
+        gc.enable()
 
 
 def test_static_permute_drops_out_of_range_ids():
