@@ -47,6 +47,7 @@ def parse():
                     help="other workloads measured after the main one (1 GPU only; '' for none)")
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-backward", action="store_true", help="skip timing the training path")
     return ap.parse_args()
 
 
@@ -349,7 +350,7 @@ def measure_config(cfg, args, world, local, with_clocks):
     if code != 0:
         raise RuntimeError(f"device status {code} {detail}")
     bwd = None
-    if cfg.act == "gelu" and cfg.h_s == 0:   # the training path (GELU experts, no shared expert)
+    if cfg.act == "gelu" and cfg.h_s == 0 and not args.no_backward:   # the training path (GELU experts, no shared expert)
         bwd = measure_backward(cfg, W, x, rt["idx"], args, flush, stream)
     del ws, flush, W, x, y
     torch.cuda.empty_cache()

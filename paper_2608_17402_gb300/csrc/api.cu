@@ -869,8 +869,8 @@ namespace {
 // K blocks never straddle two experts.
 struct BwdLayout {
     size_t status, wsplit, wrt, wpart, wexp, sig, gate, hist, counts, offsets, tiles, n_tiles, perm,
-        inv, poff, ptok, pgate, slot_prow, ptiles, n_ptiles, it2, n_it2, it1, n_it1, itr, n_itr, H, U,
-        DU, Gm, Xp, dgp, DS, dwr;
+        inv, poff, ptok, pgate, slot_prow, ptiles, n_ptiles, dx_items, n_dx_items, it2, n_it2, it1, n_it1,
+        itr, n_itr, H, U, DU, Gm, Xp, dgp, DS, dwr;
     int64_t rows_max, max_it2, max_it1, max_itr;
     int nt_h;
     size_t total;
@@ -913,6 +913,8 @@ BwdLayout make_bwd_layout(int64_t T, int64_t d, int64_t E, int64_t k, int64_t h)
     L.slot_prow = take(4 * n);
     L.ptiles = take(16 * max_mtiles(L.rows_max, E));
     L.n_ptiles = take(4);
+    L.dx_items = take(16 * max_mtiles(L.rows_max, E) * nt_d);   // band-ordered dx GEMM items
+    L.n_dx_items = take(4);
     L.it2 = take(16 * L.max_it2);
     L.n_it2 = take(4);
     L.it1 = take(16 * L.max_it1);
@@ -1071,16 +1073,24 @@ moevie_status moevie_moe_backward(const moevie_layer* Lr, const void* x, const v
         g.dg_part = dgp;
         if ((c = run_gemm(g, st, s)) != MOEVIE_OK) return c;
     }
-    // 6. dx += du W1[e]^T (K-major W1), scattered to the rows' tokens
+    // 6. dx += du W1[e]^T (K-major W1), scattered to the rows' tokens; band-ordered like the
+    //    forward's down-projection when the fp32 dx would not stay in L2
     {
+        const BandPlan bp = choose_bands(T, d, E, k, h);
+        const bool banded = (bp.nb > 1 || bp.gsz < nt_d) && max_mtiles(L.rows_max, E) <= ITEM_MAX_TILES;
+        if (banded)
+            MV_TRY(launch_item_order(at<int4>(ws, L.ptiles), at<int32_t>(ws, L.n_ptiles), ptok, T, bp.nb, nt_d,
+                                     bp.gsz, bn_d, (int)max_mtiles(L.rows_max, E), at<int4>(ws, L.dx_items),
+                                     at<int32_t>(ws, L.n_dx_items), s));
         GemmSpec g{};
         g.A = DU;
         g.lda = hp;
         g.a_cols = h;
         g.a_nrows = L.rows_max;
         g.m_total = L.rows_max;
-        g.tiles = at<int4>(ws, L.ptiles);
-        g.n_tiles = at<int32_t>(ws, L.n_ptiles);
+        g.tiles = banded ? at<int4>(ws, L.dx_items) : at<int4>(ws, L.ptiles);
+        g.n_tiles = banded ? at<int32_t>(ws, L.n_dx_items) : at<int32_t>(ws, L.n_ptiles);
+        g.item_table = banded ? 1 : 0;
         g.G = (int)E;
         g.W = Lr->W1;
         g.b_kmajor = 1;

@@ -30,8 +30,10 @@ __device__ __forceinline__ float warp_sum_f(float v) {
     return v;
 }
 
-// One warp per token: s_j = x_t . W_r[:, e_j] for its k experts (fp32, lanes over d),
-// sigma_j = 1 / (1 + e^-s_j), S = sum_j sigma_j, g_j = sigma_j / S.
+// One warp per token: s_j = x_t . W_r[:, e_j] for its k experts (fp32, lanes over d; the
+// k dot products advance together, so each lane has k loads in flight per step),
+// sigma_j = 1 / (1 + e^-s_j), S = sum_j sigma_j, g_j = sigma_j / S.  KB >= k.
+template <int KB>
 __global__ void __launch_bounds__(256) bwd_gates_kernel(const __nv_bfloat16* __restrict__ x,
                                                         const float* __restrict__ wrt, int dp,
                                                         const int32_t* __restrict__ idx, int64_t T,
@@ -42,20 +44,29 @@ __global__ void __launch_bounds__(256) bwd_gates_kernel(const __nv_bfloat16* __r
     const int64_t t = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
     if (t >= T) return;
     const __nv_bfloat16* xr = x + t * d;
+    const float* w[KB];
+    float acc[KB];
+#pragma unroll
+    for (int j = 0; j < KB; ++j) {
+        acc[j] = 0.f;
+        const int e = j < k ? idx[t * k + j] : 0;
+        const bool ok = e >= 0 && e < E;
+        if (j < k && !ok && lane == 0) report(st, MOEVIE_ERR_DEVICE, SITE_PERMUTE_ID, (int)(t * k + j), e);
+        w[j] = (j < k && ok) ? wrt + (int64_t)e * dp : nullptr;
+    }
+    for (int i = lane; i < d; i += 32) {
+        const float xi = __bfloat162float(xr[i]);
+#pragma unroll
+        for (int j = 0; j < KB; ++j)
+            if (w[j]) acc[j] = fmaf(xi, __ldg(w[j] + i), acc[j]);
+    }
     float ssum = 0.f, mine = 0.f;   // lane j keeps sigma_j
-    for (int j = 0; j < k; ++j) {
-        const int e = idx[t * k + j];
-        float acc = 0.f;
-        if (e >= 0 && e < E) {
-            const float* w = wrt + (int64_t)e * dp;
-            for (int i = lane; i < d; i += 32) acc = fmaf(__bfloat162float(xr[i]), w[i], acc);
-        } else if (lane == 0) {
-            report(st, MOEVIE_ERR_DEVICE, SITE_PERMUTE_ID, (int)(t * k + j), e);
-        }
-        acc = warp_sum_f(acc);
-        const float sg = 1.0f / (1.0f + expf(-acc));
-        if (lane == j) mine = sg;
-        ssum += sg;
+#pragma unroll
+    for (int j = 0; j < KB; ++j) {
+        if (j >= k) break;
+        const float sgm = 1.0f / (1.0f + expf(-warp_sum_f(acc[j])));
+        if (lane == j) mine = sgm;
+        ssum += sgm;
     }
     if (lane < k) {
         sig[t * k + lane] = mine;
@@ -221,8 +232,9 @@ __global__ void bwd_gather_kernel(const __nv_bfloat16* __restrict__ x, const __n
 
 // One warp per token (Eqs. 4-5 backward): dg_j = sum of the nparts partial row dots of
 // its padded row, gdg = sum_j g_j dg_j, ds_j = sigma_j (1 - sigma_j) (dg_j - gdg) / S;
-// dx_t += sum_j ds_j W_r[:, e_j] (after the grouped dx GEMM, same stream), and ds_j into
-// ds[t][e_j] (bf16, the rest of the row already zero).
+// dx_t += sum_j ds_j W_r[:, e_j] (after the grouped dx GEMM, same stream; the k columns
+// advance together), and ds_j into ds[t][e_j] (bf16, the rest of the row already zero).
+template <int KB>
 __global__ void __launch_bounds__(256) bwd_router_kernel(
     const int32_t* __restrict__ idx, const float* __restrict__ sig, const float* __restrict__ gate,
     const int32_t* __restrict__ slot_prow, const float* __restrict__ dg_part, int nparts,
@@ -247,13 +259,21 @@ __global__ void __launch_bounds__(256) bwd_router_kernel(
     const float gdg = warp_sum_f(g * dg);
     const float ds = lane < k ? sg * (1.f - sg) * (dg - gdg) / S : 0.f;
     if (lane < k && e >= 0 && e < E) ds_out[t * Ep + e] = __float2bfloat16_rn(ds);
-    float* dxr = dx + t * d;
-    for (int j = 0; j < k; ++j) {
-        const float dsj = __shfl_sync(0xffffffffu, ds, j);
+    const float* w[KB];
+    float dsj[KB];
+#pragma unroll
+    for (int j = 0; j < KB; ++j) {
+        dsj[j] = __shfl_sync(0xffffffffu, ds, j);
         const int ej = __shfl_sync(0xffffffffu, e, j);
-        if (ej < 0 || ej >= E) continue;
-        const float* w = wrt + (int64_t)ej * dp;
-        for (int i = lane; i < d; i += 32) dxr[i] = fmaf(dsj, w[i], dxr[i]);
+        w[j] = (j < k && ej >= 0 && ej < E) ? wrt + (int64_t)ej * dp : nullptr;
+    }
+    float* dxr = dx + t * d;
+    for (int i = lane; i < d; i += 32) {
+        float a = dxr[i];
+#pragma unroll
+        for (int j = 0; j < KB; ++j)
+            if (w[j]) a = fmaf(dsj[j], __ldg(w[j] + i), a);
+        dxr[i] = a;
     }
 }
 
@@ -278,9 +298,11 @@ int grid_of(int64_t n, int threads) {
 
 cudaError_t launch_bwd_gates(const __nv_bfloat16* x, const float* wrt, int dp, const int32_t* idx, int64_t T,
                              int d, int E, int k, float* sig, float* gate, DevStatus* st, cudaStream_t s) {
-    if (k > 32) return cudaErrorInvalidValue;
-    const cudaError_t e = launch_pdl(bwd_gates_kernel, dim3((unsigned)((T * 32 + 255) / 256)), dim3(256), 0, s,
-                                     x, wrt, dp, idx, T, d, E, k, sig, gate, st);
+    const dim3 grid((unsigned)((T * 32 + 255) / 256));
+    cudaError_t e;
+    if (k <= 8) e = launch_pdl(bwd_gates_kernel<8>, grid, dim3(256), 0, s, x, wrt, dp, idx, T, d, E, k, sig, gate, st);
+    else if (k <= 32) e = launch_pdl(bwd_gates_kernel<32>, grid, dim3(256), 0, s, x, wrt, dp, idx, T, d, E, k, sig, gate, st);
+    else return cudaErrorInvalidValue;
     count_launches(1);
     return e;
 }
@@ -328,10 +350,16 @@ cudaError_t launch_bwd_router(const int32_t* idx, const float* sig, const float*
                               const float* dg_part, int nparts, int64_t part_stride, const float* wrt, int dp,
                               int64_t T, int d, int E, int k, int Ep, float* dx, __nv_bfloat16* ds,
                               cudaStream_t s) {
-    if (k > 32) return cudaErrorInvalidValue;
-    const cudaError_t e = launch_pdl(bwd_router_kernel, dim3((unsigned)((T * 32 + 255) / 256)), dim3(256), 0, s,
-                                     idx, sig, gate, slot_prow, dg_part, nparts, part_stride, wrt, dp, T, d, E, k,
-                                     Ep, dx, ds);
+    const dim3 grid((unsigned)((T * 32 + 255) / 256));
+    cudaError_t e;
+    if (k <= 8)
+        e = launch_pdl(bwd_router_kernel<8>, grid, dim3(256), 0, s, idx, sig, gate, slot_prow, dg_part, nparts,
+                       part_stride, wrt, dp, T, d, E, k, Ep, dx, ds);
+    else if (k <= 32)
+        e = launch_pdl(bwd_router_kernel<32>, grid, dim3(256), 0, s, idx, sig, gate, slot_prow, dg_part, nparts,
+                       part_stride, wrt, dp, T, d, E, k, Ep, dx, ds);
+    else
+        return cudaErrorInvalidValue;
     count_launches(1);
     return e;
 }
