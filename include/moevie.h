@@ -225,37 +225,40 @@ int64_t moevie_shared_groups(int64_t T, int64_t d, int64_t E, int64_t k, int64_t
 
 /* ---------------------------------------------------------------- training path
  *
- * Backward pass of the layer for GELU experts without a shared expert (App. B: the
- * paper trains with grouped GEMMs and applies the activation as its own step).  Given the
- * forward's selection idx (held fixed: top-k is piecewise constant in the logits, so it
- * has no gradient) and the output gradient dy, it returns the gradients of
+ * Backward pass of the layer without a shared expert, GELU or SwiGLU experts (App. B:
+ * the paper trains with grouped GEMMs and applies the activation as its own step).  Given
+ * the forward's selection idx (held fixed: top-k is piecewise constant in the logits, so
+ * it has no gradient) and the output gradient dy, it returns the gradients of
  * L = sum_t dy_t . y_t:
- *   through each selected expert e of token t, with gate g (Eqs. 4-5) and u = x_t W1[e]:
- *     dW2[e] += GELU(u)^T (g dy_t),   du = (g dy_t W2[e]^T) GELU'(u),
- *     dW1[e] += x_t^T du,             dx_t += du W1[e]^T;
+ *   through each selected expert e of token t, with gate g (Eqs. 4-5) and the hidden
+ *   activation a (GELU(u), u = x_t W1[e]; SwiGLU: SiLU(u) v, v = x_t W3[e]):
+ *     dW2[e] += a^T (g dy_t),   da = g dy_t W2[e]^T,
+ *     GELU:   du = da GELU'(u);   SwiGLU: du = da v SiLU'(u), dv = da SiLU(u),
+ *     dW1[e] += x_t^T du,  dW3[e] += x_t^T dv,  dx_t += du W1[e]^T + dv W3[e]^T;
  *   through the gates (Eqs. 4-5), with sigma_j = sigmoid(s_{e_j}), S = sum_j sigma_j and
  *   dg_j = dy_t . E_{e_j}(x_t):
  *     ds_{e_j} = sigma_j (1 - sigma_j) (dg_j - sum_l g_l dg_l) / S,
  *     dW_r[:, e_j] += x_t ds_{e_j},   dx_t += ds_{e_j} W_r[:, e_j].
  * The bias b gets no gradient (it only selects; moevie_update_bias moves it).
  *
- * Inputs: the layer (W_r, W1, W2 as for moevie_moe_forward; W3 must be NULL and h_s 0,
- * else MOEVIE_ERR_UNSUPPORTED), x bf16 [T, d], dy bf16 [T, d], idx int32 [T, k] (the
- * forward's selection, e.g. moevie_routing.idx; ids in [0, E)).  Outputs, fp32, all
- * overwritten: dx [T, d], dW_r [d, E], dW1 [E, d, h] with rows h rounded up to 8 apart
- * (as W1; the pad columns hold zeros), dW2 [E, h, d].  The gates are recomputed from x
- * and W_r in fp32.  Arithmetic: bf16 GEMM operands with fp32 accumulation (the hidden
- * pre-activations, activations, their gradients, g dy and ds are rounded to bf16 as GEMM
- * operands); the weight gradients are summed over tokens with fp32 reductions, so their
- * last bits depend on the order in which the GEMM's work items finish.  Sizes: k <= 32,
- * d and h <= 65535, plus the limits of moevie_moe_forward.  `ws`: moevie_backward_
- * workspace_size(T_max, d, E, k, h) bytes, set up with moevie_workspace_init; device
- * errors land in its status block. */
+ * Inputs: the layer (W_r, W1, W2 and, for SwiGLU experts, W3, as for moevie_moe_forward;
+ * h_s must be 0, else MOEVIE_ERR_UNSUPPORTED), x bf16 [T, d], dy bf16 [T, d], idx int32
+ * [T, k] (the forward's selection, e.g. moevie_routing.idx; ids in [0, E)).  Outputs,
+ * fp32, all overwritten: dx [T, d], dW_r [d, E], dW1 [E, d, h] with rows h rounded up to
+ * 8 apart (as W1; the pad columns hold zeros), dW2 [E, h, d], and for SwiGLU experts dW3
+ * laid out as dW1 (NULL otherwise).  The gates are recomputed from x and W_r in fp32.
+ * Arithmetic: bf16 GEMM operands with fp32 accumulation (the recomputed pre-activations,
+ * activations, their gradients, g dy and ds are rounded to bf16 as GEMM operands); the
+ * weight gradients are summed over tokens with fp32 reductions, so their last bits
+ * depend on the order in which the GEMM's work items finish.  Sizes: k <= 32, d and h <=
+ * 65535, plus the limits of moevie_moe_forward.  `ws`: moevie_backward_workspace_size(
+ * T_max, d, E, k, h, swiglu) bytes (swiglu nonzero for SwiGLU experts), set up with
+ * moevie_workspace_init; device errors land in its status block. */
 moevie_status moevie_backward_workspace_size(int64_t T_max, int64_t d, int64_t E, int64_t k, int64_t h,
-                                             size_t* bytes);
+                                             int swiglu, size_t* bytes);
 moevie_status moevie_moe_backward(const moevie_layer* layer, const void* x, const void* dy, int64_t T,
                                   const int32_t* idx, float* dx, float* dW_r, float* dW1, float* dW2,
-                                  void* ws, size_t ws_bytes, void* stream);
+                                  float* dW3, void* ws, size_t ws_bytes, void* stream);
 
 /* Synchronise `stream`, then read the workspace's device status into *out
  * (MOEVIE_OK when no device-side error was recorded).  `detail` (host, may be

@@ -237,7 +237,9 @@ struct GemmSpec {
     int64_t max_items;       // item_table == 2: host bound on the number of items
     int a_neg_zero, o_neg_skip;
     void* out2;
+    void* out3;
     const void* epi_u;
+    const void* epi_v;
     const void* epi_a;
     float* dg_part;
 };
@@ -286,7 +288,9 @@ moevie_status run_gemm(const GemmSpec& g, DevStatus* st, cudaStream_t s) {
     a.a_neg_zero = g.a_neg_zero;
     a.o_neg_skip = g.o_neg_skip;
     a.out2 = static_cast<__nv_bfloat16*>(g.out2);
+    a.out3 = static_cast<__nv_bfloat16*>(g.out3);
     a.epi_u = static_cast<const __nv_bfloat16*>(g.epi_u);
+    a.epi_v = static_cast<const __nv_bfloat16*>(g.epi_v);
     a.epi_a = static_cast<const __nv_bfloat16*>(g.epi_a);
     a.dg_part = g.dg_part;
     a.A = static_cast<const __nv_bfloat16*>(g.A);
@@ -870,13 +874,13 @@ namespace {
 struct BwdLayout {
     size_t status, wsplit, wrt, wpart, wexp, sig, gate, hist, counts, offsets, tiles, n_tiles, perm,
         inv, poff, ptok, pgate, slot_prow, ptiles, n_ptiles, dx_items, n_dx_items, it2, n_it2, it1, n_it1,
-        itr, n_itr, H, U, DU, Gm, Xp, dgp, DS, dwr;
+        itr, n_itr, H, U, DU, V, DV, Gm, Xp, dgp, DS, dwr;
     int64_t rows_max, max_it2, max_it1, max_itr;
     int nt_h;
     size_t total;
 };
 
-BwdLayout make_bwd_layout(int64_t T, int64_t d, int64_t E, int64_t k, int64_t h) {
+BwdLayout make_bwd_layout(int64_t T, int64_t d, int64_t E, int64_t k, int64_t h, bool swiglu) {
     BwdLayout L;
     size_t o = 0;
     auto take = [&](size_t bytes) {
@@ -924,6 +928,8 @@ BwdLayout make_bwd_layout(int64_t T, int64_t d, int64_t E, int64_t k, int64_t h)
     L.H = take(2 * L.rows_max * hp);
     L.U = take(2 * L.rows_max * hp);
     L.DU = take(2 * L.rows_max * hp);
+    L.V = swiglu ? take(2 * L.rows_max * hp) : 0;    // SwiGLU: the up projection's pre-activation
+    L.DV = swiglu ? take(2 * L.rows_max * hp) : 0;   //   and its gradient
     L.Gm = take(2 * L.rows_max * d);
     L.Xp = take(2 * L.rows_max * d);
     L.dgp = take(4 * 2 * (int64_t)L.nt_h * L.rows_max);
@@ -946,29 +952,31 @@ moevie_status check_bwd_sizes(int64_t T, int64_t d, int64_t E, int64_t k, int64_
 extern "C" {
 
 moevie_status moevie_backward_workspace_size(int64_t T_max, int64_t d, int64_t E, int64_t k, int64_t h,
-                                             size_t* bytes) {
+                                             int swiglu, size_t* bytes) {
     if (!bytes) return MOEVIE_ERR_INVALID_ARG;
     const moevie_status c = check_bwd_sizes(T_max, d, E, k, h);
     if (c != MOEVIE_OK) return c;
-    *bytes = make_bwd_layout(T_max, d, E, k, h).total;
+    *bytes = make_bwd_layout(T_max, d, E, k, h, swiglu != 0).total;
     return MOEVIE_OK;
 }
 
 moevie_status moevie_moe_backward(const moevie_layer* Lr, const void* x, const void* dy, int64_t T,
                                   const int32_t* idx, float* dx, float* dW_r, float* dW1, float* dW2,
-                                  void* ws, size_t ws_bytes, void* stream) {
+                                  float* dW3, void* ws, size_t ws_bytes, void* stream) {
     if (!Lr) return MOEVIE_ERR_INVALID_ARG;
     const int64_t d = Lr->d, E = Lr->E, k = Lr->k, h = Lr->h;
     moevie_status c = check_bwd_sizes(T, d, E, k, h);
     if (c != MOEVIE_OK) return c;
-    if (Lr->W3 || Lr->h_s > 0) return MOEVIE_ERR_UNSUPPORTED;   // GELU experts, no shared expert
+    if (Lr->h_s > 0) return MOEVIE_ERR_UNSUPPORTED;   // no shared expert on this path
+    const bool swiglu = Lr->W3 != nullptr;
     if (T == 0) return MOEVIE_OK;
     if (!x || !dy || !idx || !dx || !dW_r || !dW1 || !dW2 || !ws || !Lr->W_r || !Lr->W1 || !Lr->W2)
         return MOEVIE_ERR_INVALID_ARG;
+    if (swiglu && (!dW3 || !a16(dW3) || !a16(Lr->W3))) return MOEVIE_ERR_INVALID_ARG;
     if (!a16(x) || !a16(dy) || !a16(idx) || !a16(dx) || !a16(dW1) || !a16(dW2) || !a16(ws) || !a16(Lr->W1) ||
         !a16(Lr->W2))
         return MOEVIE_ERR_INVALID_ARG;
-    const BwdLayout L = make_bwd_layout(T, d, E, k, h);
+    const BwdLayout L = make_bwd_layout(T, d, E, k, h, swiglu);
     if (ws_bytes < L.total) return MOEVIE_ERR_WORKSPACE;
     cudaStream_t s = static_cast<cudaStream_t>(stream);
     DevStatus* st = at<DevStatus>(ws, L.status);
@@ -981,6 +989,8 @@ moevie_status moevie_moe_backward(const moevie_layer* Lr, const void* x, const v
     void* H = at<void>(ws, L.H);
     void* U = at<void>(ws, L.U);
     void* DU = at<void>(ws, L.DU);
+    void* V = swiglu ? at<void>(ws, L.V) : nullptr;
+    void* DV = swiglu ? at<void>(ws, L.DV) : nullptr;
     void* Gm = at<void>(ws, L.Gm);
     void* Xp = at<void>(ws, L.Xp);
     float* dgp = at<float>(ws, L.dgp);
@@ -1017,6 +1027,7 @@ moevie_status moevie_moe_backward(const moevie_layer* Lr, const void* x, const v
     MV_TRY(launch_zero_f32(dx, T * d, s));
     MV_TRY(launch_zero_f32(dW1, E * d * hp, s));
     MV_TRY(launch_zero_f32(dW2, E * h * d, s));
+    if (swiglu) MV_TRY(launch_zero_f32(dW3, E * d * hp, s));
     MV_TRY(launch_zero_f32(dwr, d * Ep, s));
     MV_TRY(launch_zero_f32(reinterpret_cast<float*>(DS), T * Ep / 2, s));
     MV_TRY(launch_bwd_gather(xb, static_cast<const __nv_bfloat16*>(dy), ptok, pgate, poff, (int)E, (int)d,
@@ -1039,6 +1050,11 @@ moevie_status moevie_moe_backward(const moevie_layer* Lr, const void* x, const v
         g.N = (int)h;
         g.N_ld = hp;
         g.epi = EPI_GELU2_BF16;
+        if (swiglu) {   // a = SiLU(u) v with u = x W1[e] (gate), v = x W3[e] (up); u and v kept
+            g.epi = EPI_SWIGLU_BF16;
+            g.W3 = Lr->W3;
+            g.out3 = V;
+        }
         g.out = H;
         g.out2 = U;
         g.ldo = hp;
@@ -1064,11 +1080,13 @@ moevie_status moevie_moe_backward(const moevie_layer* Lr, const void* x, const v
         g.K = (int)d;
         g.N = (int)h;
         g.N_ld = hp;
-        g.epi = EPI_DGELU_BF16;
+        g.epi = swiglu ? EPI_DSWIGLU_BF16 : EPI_DGELU_BF16;
         g.row_scale = pgate;
         g.epi_u = U;
+        g.epi_v = V;
         g.epi_a = H;
         g.out = DU;
+        g.out2 = DV;
         g.ldo = hp;
         g.dg_part = dgp;
         if ((c = run_gemm(g, st, s)) != MOEVIE_OK) return c;
@@ -1082,31 +1100,33 @@ moevie_status moevie_moe_backward(const moevie_layer* Lr, const void* x, const v
             MV_TRY(launch_item_order(at<int4>(ws, L.ptiles), at<int32_t>(ws, L.n_ptiles), ptok, T, bp.nb, nt_d,
                                      bp.gsz, bn_d, (int)max_mtiles(L.rows_max, E), at<int4>(ws, L.dx_items),
                                      at<int32_t>(ws, L.n_dx_items), s));
-        GemmSpec g{};
-        g.A = DU;
-        g.lda = hp;
-        g.a_cols = h;
-        g.a_nrows = L.rows_max;
-        g.m_total = L.rows_max;
-        g.tiles = banded ? at<int4>(ws, L.dx_items) : at<int4>(ws, L.ptiles);
-        g.n_tiles = banded ? at<int32_t>(ws, L.n_dx_items) : at<int32_t>(ws, L.n_ptiles);
-        g.item_table = banded ? 1 : 0;
-        g.G = (int)E;
-        g.W = Lr->W1;
-        g.b_kmajor = 1;
-        g.b_k_ld = hp;
-        g.b_g_ld = d * hp;
-        g.K = (int)h;
-        g.N = (int)d;
-        g.epi = EPI_ADD_F32;
-        g.yacc = dx;
-        g.ldy = d;
-        g.o_nrows = T;
-        g.o_rows = ptok;
-        g.o_div = 1;
-        g.o_neg_skip = 1;
-        g.scale = 1.0f;
-        if ((c = run_gemm(g, st, s)) != MOEVIE_OK) return c;
+        for (int pass = 0; pass < (swiglu ? 2 : 1); ++pass) {   // du W1^T, then dv W3^T (SwiGLU)
+            GemmSpec g{};
+            g.A = pass ? DV : DU;
+            g.lda = hp;
+            g.a_cols = h;
+            g.a_nrows = L.rows_max;
+            g.m_total = L.rows_max;
+            g.tiles = banded ? at<int4>(ws, L.dx_items) : at<int4>(ws, L.ptiles);
+            g.n_tiles = banded ? at<int32_t>(ws, L.n_dx_items) : at<int32_t>(ws, L.n_ptiles);
+            g.item_table = banded ? 1 : 0;
+            g.G = (int)E;
+            g.W = pass ? Lr->W3 : Lr->W1;
+            g.b_kmajor = 1;
+            g.b_k_ld = hp;
+            g.b_g_ld = d * hp;
+            g.K = (int)h;
+            g.N = (int)d;
+            g.epi = EPI_ADD_F32;
+            g.yacc = dx;
+            g.ldy = d;
+            g.o_nrows = T;
+            g.o_rows = ptok;
+            g.o_div = 1;
+            g.o_neg_skip = 1;
+            g.scale = 1.0f;
+            if ((c = run_gemm(g, st, s)) != MOEVIE_OK) return c;
+        }
     }
     // 7. the router (Eqs. 4-5): ds per token, dx += ds W_r^T, ds into [T][E_pad] bf16
     MV_TRY(launch_bwd_router(idx, at<float>(ws, L.sig), at<float>(ws, L.gate), at<int32_t>(ws, L.slot_prow), dgp,
@@ -1146,6 +1166,9 @@ moevie_status moevie_moe_backward(const moevie_layer* Lr, const void* x, const v
         return c;
     if ((c = wgrad(Xp, d, L.rows_max, d, DU, h, hp, L.rows_max, (int)E, (int)d, L.it1, L.n_it1, L.max_it1, dW1,
                    hp)) != MOEVIE_OK)
+        return c;
+    if (swiglu && (c = wgrad(Xp, d, L.rows_max, d, DV, h, hp, L.rows_max, (int)E, (int)d, L.it1, L.n_it1,
+                             L.max_it1, dW3, hp)) != MOEVIE_OK)   // dW3[e] = x^T dv
         return c;
     if ((c = wgrad(x, d, T, d, DS, Ep, Ep, T, 1, (int)d, L.itr, L.n_itr, L.max_itr, dwr, Ep)) != MOEVIE_OK)
         return c;

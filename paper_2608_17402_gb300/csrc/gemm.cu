@@ -728,6 +728,19 @@ __device__ void epilogue(const GemmArgs& p, const Smem& sm, uint32_t tmem, int64
                 for (int g8 = 0; g8 < 4; ++g8) {
                     if (n + 8 * g8 >= p.N) break;
                     float f[8];
+                    if (TRAIN && p.out2) {   // the training path keeps u and v as well
+                        uint4 uu, vv;
+                        uu.x = pack_bf16x2(gt[8 * g8 + 0], gt[8 * g8 + 1]);
+                        uu.y = pack_bf16x2(gt[8 * g8 + 2], gt[8 * g8 + 3]);
+                        uu.z = pack_bf16x2(gt[8 * g8 + 4], gt[8 * g8 + 5]);
+                        uu.w = pack_bf16x2(gt[8 * g8 + 6], gt[8 * g8 + 7]);
+                        vv.x = pack_bf16x2(__uint_as_float(v[8 * g8 + 0]), __uint_as_float(v[8 * g8 + 1]));
+                        vv.y = pack_bf16x2(__uint_as_float(v[8 * g8 + 2]), __uint_as_float(v[8 * g8 + 3]));
+                        vv.z = pack_bf16x2(__uint_as_float(v[8 * g8 + 4]), __uint_as_float(v[8 * g8 + 5]));
+                        vv.w = pack_bf16x2(__uint_as_float(v[8 * g8 + 6]), __uint_as_float(v[8 * g8 + 7]));
+                        *reinterpret_cast<uint4*>(p.out2 + (int64_t)gr * p.ldo + n + 8 * g8) = uu;
+                        *reinterpret_cast<uint4*>(p.out3 + (int64_t)gr * p.ldo + n + 8 * g8) = vv;
+                    }
 #pragma unroll
                     for (int i = 0; i < 8; ++i) {
                         // SiLU(g) u = g u / (1 + e^-g); e^-g = inf for g far below 0 gives 0
@@ -778,6 +791,40 @@ __device__ void epilogue(const GemmArgs& p, const Smem& sm, uint32_t tmem, int64
             const int n = t.n0 + c0;
             if constexpr (!to_f32) {
                 __nv_bfloat16* orow = p.out + (int64_t)gr * p.ldo + n;
+                if (TRAIN && p.epi == EPI_DSWIGLU_BF16) {   // SwiGLU: du, dv and the dot acc . a
+                    const __nv_bfloat16* urow = p.epi_u + (int64_t)gr * p.ldo + n;
+                    const __nv_bfloat16* vrow = p.epi_v + (int64_t)gr * p.ldo + n;
+                    const __nv_bfloat16* arow = p.epi_a + (int64_t)gr * p.ldo + n;
+#pragma unroll
+                    for (int g8 = 0; g8 < 4; ++g8) {
+                        if (n + 8 * g8 >= p.N) break;
+                        float uf[8], vf[8], af[8], fu[8], fv[8];
+                        unpack_bf16x8(*reinterpret_cast<const uint4*>(urow + 8 * g8), uf);
+                        unpack_bf16x8(*reinterpret_cast<const uint4*>(vrow + 8 * g8), vf);
+                        unpack_bf16x8(*reinterpret_cast<const uint4*>(arow + 8 * g8), af);
+#pragma unroll
+                        for (int i = 0; i < 8; ++i) {
+                            const float a = __uint_as_float(v[8 * g8 + i]);
+                            const bool in = n + 8 * g8 + i < p.N;   // columns past N: padding
+                            dg_acc += in ? a * af[i] : 0.f;
+                            const float sg = 1.0f / (1.0f + expf(-uf[i]));   // SiLU(u) = u sg
+                            fu[i] = in ? sc * a * vf[i] * sg * (1.0f + uf[i] * (1.0f - sg)) : 0.f;
+                            fv[i] = in ? sc * a * uf[i] * sg : 0.f;
+                        }
+                        uint4 u, w;
+                        u.x = pack_bf16x2(fu[0], fu[1]);
+                        u.y = pack_bf16x2(fu[2], fu[3]);
+                        u.z = pack_bf16x2(fu[4], fu[5]);
+                        u.w = pack_bf16x2(fu[6], fu[7]);
+                        w.x = pack_bf16x2(fv[0], fv[1]);
+                        w.y = pack_bf16x2(fv[2], fv[3]);
+                        w.z = pack_bf16x2(fv[4], fv[5]);
+                        w.w = pack_bf16x2(fv[6], fv[7]);
+                        *reinterpret_cast<uint4*>(orow + 8 * g8) = u;
+                        *reinterpret_cast<uint4*>(p.out2 + (int64_t)gr * p.ldo + n + 8 * g8) = w;
+                    }
+                    continue;
+                }
                 if (TRAIN && p.epi == EPI_DGELU_BF16) {   // training path: du = scale acc GELU'(u), dot acc . a
                     const __nv_bfloat16* urow = p.epi_u + (int64_t)gr * p.ldo + n;
                     const __nv_bfloat16* arow = p.epi_a + (int64_t)gr * p.ldo + n;
@@ -839,7 +886,7 @@ __device__ void epilogue(const GemmArgs& p, const Smem& sm, uint32_t tmem, int64
                 }
             }
         }
-        if (TRAIN && !to_f32 && p.epi == EPI_DGELU_BF16 && ok_row)   // the row dot, per n-tile and warp half
+        if (TRAIN && !to_f32 && (p.epi == EPI_DGELU_BF16 || p.epi == EPI_DSWIGLU_BF16) && ok_row)   // row dot
             p.dg_part[(int64_t)(2 * (t.n0 / p.n_step) + half) * p.m_total + gr] = dg_acc;
     }
 }
@@ -1078,9 +1125,9 @@ cudaError_t launch_grouped_gemm(const GemmArgs& a, int grid, cudaStream_t s) {
         grouped_gemm_kernel<16, false, ECLS_ADD, true>};
     const bool gathered = a.a_rows || a.a_ident;   // A rows through the gather warps
     const bool train = a.b_kmajor || a.a_mn || a.item_table == 2 || a.epi == EPI_GELU2_BF16 ||
-                       a.epi == EPI_DGELU_BF16;
+                       a.epi == EPI_DGELU_BF16 || a.epi == EPI_DSWIGLU_BF16 || a.out2 != nullptr;
     const bool bf16_out = a.epi == EPI_GELU_BF16 || a.epi == EPI_STORE_BF16 || a.epi == EPI_SWIGLU_BF16 ||
-                          a.epi == EPI_GELU2_BF16 || a.epi == EPI_DGELU_BF16;
+                          a.epi == EPI_GELU2_BF16 || a.epi == EPI_DGELU_BF16 || a.epi == EPI_DSWIGLU_BF16;
     if (gathered && !bf16_out) return cudaErrorInvalidValue;
     if (!gathered && a.epi == EPI_SWIGLU_BF16) return cudaErrorInvalidValue;
     Kern kern;

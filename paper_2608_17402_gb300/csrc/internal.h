@@ -207,6 +207,8 @@ enum Epilogue : int {
     EPI_GELU2_BF16 = 6,  // out[r, n] = bf16(GELU(acc)), out2[r, n] = bf16(acc) (the pre-activation)
     EPI_DGELU_BF16 = 7,  // out[r, n] = bf16(scale(r) acc GELU'(u[r, n])), and the row dot
                          //   sum_n acc a[r, n] (a = GELU(u)) in partials dg_part[2 nt + half][r]
+    EPI_DSWIGLU_BF16 = 8,// SwiGLU a = SiLU(u) v: out = du = bf16(scale acc v SiLU'(u)), out2 = dv =
+                         //   bf16(scale acc SiLU(u)), and the row dot sum_n acc a as for EPI_DGELU_BF16
 };
 static_assert(EPI_ADD_F32 == 2, "gm_stages / gm_smem_bytes test the reduction epilogue by value");
 // Epilogue classes of the grouped GEMM's kernel instances: bf16 outputs (GELU, SwiGLU,
@@ -272,10 +274,13 @@ struct GemmArgs {
                                 //   output row of (g, m) is g wg_M + m, B's map has one group
     int a_neg_zero;             // gathered rows with a negative table entry are zero rows (padding)
     int o_neg_skip;             // fp32 outputs: rows with a negative output token are padding, skipped
-    __nv_bfloat16* out2;        // EPI_GELU2_BF16: the pre-activation, laid out as out
-    const __nv_bfloat16* epi_u; // EPI_DGELU_BF16: pre-activations u and activations GELU(u) of
-    const __nv_bfloat16* epi_a; //   the GEMM rows, [m_total][ldo] bf16
-    float* dg_part;             // EPI_DGELU_BF16: per-row partial dots, [2 n_ntiles][m_total] fp32
+    __nv_bfloat16* out2;        // EPI_GELU2_BF16: the pre-activation, laid out as out; with
+    __nv_bfloat16* out3;        //   EPI_SWIGLU_BF16 (training instances): u in out2, v in out3;
+                                //   EPI_DSWIGLU_BF16: dv in out2
+    const __nv_bfloat16* epi_u; // EPI_DGELU_BF16 / EPI_DSWIGLU_BF16: pre-activations u (and v)
+    const __nv_bfloat16* epi_v; //   and activations a of the GEMM rows, [m_total][ldo] bf16
+    const __nv_bfloat16* epi_a;
+    float* dg_part;             // EPI_D*_BF16: per-row partial dots, [2 n_ntiles][m_total] fp32
     DevStatus* status;
     uint64_t limit_ns;
 };

@@ -1,5 +1,5 @@
 """Training path (App. B: grouped GEMMs with the activation as its own step) of
-moevie_moe_backward against the oracle's backward (the gradients of sum_t dy_t . y_t
+moevie_moe_backward, GELU and SwiGLU experts, against the oracle's backward (the gradients of sum_t dy_t . y_t
 with the top-k selection held fixed, through the renormalised gates of Eqs. 4-5 into
 W_r and x; the bias gets none), element by element, on the same seeded inputs and
 the same bf16 dy.  Tolerance as for the forward (rel-L2 <= 1e-2, max |err| <= 5e-2 RMS)
@@ -30,7 +30,7 @@ def _dy(T, d, seed, tokens=None):
 def _gpu_backward(lay, dy_bits, idx):
     c = lay.cfg
     x, W = layer_to_device(lay)
-    ws = moevie.BackwardWorkspace(c.T, c.d, c.E, c.k, c.h)
+    ws = moevie.BackwardWorkspace(c.T, c.d, c.E, c.k, c.h, swiglu=lay.W3 is not None)
     g = moevie.moevie_moe_backward(W, x, dev_bf16(dy_bits), dev(np.ascontiguousarray(idx, np.int32)), ws)
     check_status(ws)
     return {k: to_np_f64(v) for k, v in g.items()}
@@ -38,7 +38,10 @@ def _gpu_backward(lay, dy_bits, idx):
 
 def _compare(got, want, label):
     out = {}
-    for g_name, o_name in (("dx", "dx"), ("dW_r", "dWr"), ("dW1", "dW1"), ("dW2", "dW2")):
+    names = [("dx", "dx"), ("dW_r", "dWr"), ("dW1", "dW1"), ("dW2", "dW2")]
+    if "dW3" in want:
+        names.append(("dW3", "dW3"))
+    for g_name, o_name in names:
         if not np.any(want[o_name]):   # e.g. dW_r with one expert: exactly zero
             assert not np.any(got[g_name]), f"{label} {g_name}: expected exact zeros"
             continue
@@ -61,6 +64,31 @@ def test_backward_small(T, d, E, k, h):
     want = oracle.backward(lay.x, lay.Wr, lay.b, lay.W1, lay.W2, k, dyf)
     got = _gpu_backward(lay, dy_bits, idx)
     _compare(got, want, f"T={T} d={d} E={E} k={k} h={h}")
+
+
+@pytest.mark.parametrize("T,d,E,k,h", [
+    (300, 256, 16, 4, 128), (257, 128, 8, 2, 416), (200, 96, 12, 3, 100), (64, 64, 1, 1, 48),
+])
+def test_backward_swiglu_small(T, d, E, k, h):
+    """SwiGLU experts (App. B: a = SiLU(x W1) (x W3), W1 the gate): dW3 besides the rest."""
+    cfg = workloads.small_config(T, d, E, k, h, seed=T + 2 * h, act="swiglu")
+    lay = workloads.make_layer(cfg)
+    dy_bits, dyf = _dy(T, d, T + 3)
+    idx, _, _ = oracle.route(lay.x, lay.Wr, lay.b, k)
+    want = oracle.backward(lay.x, lay.Wr, lay.b, lay.W1, lay.W2, k, dyf, W3=lay.W3)
+    got = _gpu_backward(lay, dy_bits, idx)
+    _compare(got, want, f"swiglu T={T} d={d} E={E} k={k} h={h}")
+
+
+def test_backward_swiglu_image_layer_every_token():
+    """The SwiGLU workload (s1: T = 8192, d = 1024, E = 64, k = 8, h = 512) on every token."""
+    lay = workloads.make_layer(workloads.CONFIGS["s1"])
+    c = lay.cfg
+    dy_bits, dyf = _dy(c.T, c.d, 15)
+    idx, _, _ = oracle.route(lay.x, lay.Wr, lay.b, c.k)
+    want = oracle.backward(lay.x, lay.Wr, lay.b, lay.W1, lay.W2, c.k, dyf, W3=lay.W3)
+    r = _compare(_gpu_backward(lay, dy_bits, idx), want, "s1")
+    print("s1 backward:", {k: f"rel-L2 {v[0]:.2e}, max|err|/RMS {v[1]:.2e}" for k, v in r.items()})
 
 
 def test_backward_batch1_layer_every_token():
@@ -124,8 +152,7 @@ def test_backward_stress_layer_sampled_tokens():
 
 
 def test_backward_rejects_unsupported_layers():
-    """SwiGLU experts and a shared expert are outside this entry point: rejected before
-    any launch."""
+    """A shared expert is outside this entry point: rejected before any launch."""
     cfg = workloads.small_config(16, 64, 4, 2, 64, h_s=64)
     lay = workloads.make_layer(cfg)
     x, W = layer_to_device(lay)
