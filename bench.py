@@ -350,7 +350,7 @@ def measure_config(cfg, args, world, local, with_clocks):
     if code != 0:
         raise RuntimeError(f"device status {code} {detail}")
     bwd = None
-    if cfg.h_s == 0 and not args.no_backward:   # the training path (no shared expert)
+    if not args.no_backward:   # the training path
         bwd = measure_backward(cfg, W, x, rt["idx"], args, flush, stream)
     del ws, flush, W, x, y
     torch.cuda.empty_cache()
@@ -362,7 +362,8 @@ def measure_backward(cfg, W, x, idx, args, flush, stream):
     """CUDA-event time of moevie_moe_backward (inputs resident, L2 flushed between calls)
     and its GEMM rate: grouped GEMMs of 2 T k d h FLOPs each -- GELU: up-projection again,
     dy W2^T, du W1^T, dW2, dW1 (5); SwiGLU: gate and up again, dy W2^T, du W1^T, dv W3^T,
-    dW2, dW1, dW3 (8) -- plus dW_r = x^T ds (2 T d E)."""
+    dW2, dW1, dW3 (8) -- plus dW_r = x^T ds (2 T d E), and the shared expert's own GEMMs
+    (the same 5 or 8, of 2 T d h_s FLOPs each)."""
     import torch
 
     from paper_2608_17402_gb300 import moevie
@@ -371,7 +372,7 @@ def measure_backward(cfg, W, x, idx, args, flush, stream):
     g.manual_seed(cfg.seed + 17)
     dy = torch.randn((T, d), generator=g, device="cuda").to(torch.bfloat16)
     swiglu = cfg.act == "swiglu"
-    bws = moevie.BackwardWorkspace(T, d, E, k, h, swiglu=swiglu)
+    bws = moevie.BackwardWorkspace(T, d, E, k, h, h_s=cfg.h_s, swiglu=swiglu)
     steps = max(1, min(args.steps, 10))
     for _ in range(max(1, min(args.warmup, 3))):
         moevie.moevie_moe_backward(W, x, dy, idx, bws)
@@ -388,10 +389,11 @@ def measure_backward(cfg, W, x, idx, args, flush, stream):
     if code != 0:
         raise RuntimeError(f"backward device status {code} {detail}")
     ms = statistics.mean(a.elapsed_time(b) for a, b in zip(st, en))
-    flops = (16.0 if swiglu else 10.0) * T * k * d * h + 2.0 * T * d * E
+    flops = (16.0 if swiglu else 10.0) * T * d * (k * h + cfg.h_s) + 2.0 * T * d * E
     del bws, dy
     return {"us": ms * 1e3, "flops": flops, "tflops": flops / (ms / 1e3) / 1e12, "steps": steps,
-            "what": "moevie_moe_backward: dx, dW_r, dW1, dW2 (and dW3 for SwiGLU) of sum(dy . y), selection held fixed"}
+            "what": "moevie_moe_backward: dx, dW_r, dW1, dW2 (dW3 for SwiGLU; dWs1, dWs2, dWs3 with a shared "
+                    "expert) of sum(dy . y), selection held fixed"}
 
 
 def summarise(cfg, m, pk, world):

@@ -225,7 +225,7 @@ int64_t moevie_shared_groups(int64_t T, int64_t d, int64_t E, int64_t k, int64_t
 
 /* ---------------------------------------------------------------- training path
  *
- * Backward pass of the layer without a shared expert, GELU or SwiGLU experts (App. B:
+ * Backward pass of the layer, GELU or SwiGLU experts, with or without a shared expert (App. B:
  * the paper trains with grouped GEMMs and applies the activation as its own step).  Given
  * the forward's selection idx (held fixed: top-k is piecewise constant in the logits, so
  * it has no gradient) and the output gradient dy, it returns the gradients of
@@ -238,27 +238,34 @@ int64_t moevie_shared_groups(int64_t T, int64_t d, int64_t E, int64_t k, int64_t
  *   through the gates (Eqs. 4-5), with sigma_j = sigmoid(s_{e_j}), S = sum_j sigma_j and
  *   dg_j = dy_t . E_{e_j}(x_t):
  *     ds_{e_j} = sigma_j (1 - sigma_j) (dg_j - sum_l g_l dg_l) / S,
- *     dW_r[:, e_j] += x_t ds_{e_j},   dx_t += ds_{e_j} W_r[:, e_j].
+ *     dW_r[:, e_j] += x_t ds_{e_j},   dx_t += ds_{e_j} W_r[:, e_j];
+ *   through the shared expert (Eq. 6, second term; h_s > 0), every token with the
+ *   constant weight lambda, the expert's rules with g = lambda and Ws1, Ws2, Ws3 in place
+ *   of W1[e], W2[e], W3[e] (lambda gets no gradient).
  * The bias b gets no gradient (it only selects; moevie_update_bias moves it).
  *
- * Inputs: the layer (W_r, W1, W2 and, for SwiGLU experts, W3, as for moevie_moe_forward;
- * h_s must be 0, else MOEVIE_ERR_UNSUPPORTED), x bf16 [T, d], dy bf16 [T, d], idx int32
- * [T, k] (the forward's selection, e.g. moevie_routing.idx; ids in [0, E)).  Outputs,
- * fp32, all overwritten: dx [T, d], dW_r [d, E], dW1 [E, d, h] with rows h rounded up to
- * 8 apart (as W1; the pad columns hold zeros), dW2 [E, h, d], and for SwiGLU experts dW3
- * laid out as dW1 (NULL otherwise).  The gates are recomputed from x and W_r in fp32.
+ * Inputs: the layer (W_r, W1, W2, for SwiGLU experts W3, and the shared expert's Ws1, Ws2,
+ * Ws3 and lambda when h_s > 0, as for moevie_moe_forward), x bf16 [T, d], dy bf16 [T, d],
+ * idx int32 [T, k] (the forward's selection, e.g. moevie_routing.idx; ids in [0, E)).
+ * Outputs, fp32, all overwritten: dx [T, d], dW_r [d, E], dW1 [E, d, h] with rows h
+ * rounded up to 8 apart (as W1; the pad columns hold zeros), dW2 [E, h, d], for SwiGLU
+ * experts dW3 laid out as dW1 (NULL otherwise); with a shared expert dWs1 [d, h_s] with
+ * rows h_s rounded up to 8 apart (as Ws1), dWs2 [h_s, d] and, for SwiGLU, dWs3 laid out as
+ * dWs1 (all three NULL without one).  The gates are recomputed from x and W_r in fp32.
  * Arithmetic: bf16 GEMM operands with fp32 accumulation (the recomputed pre-activations,
  * activations, their gradients, g dy and ds are rounded to bf16 as GEMM operands); the
  * weight gradients are summed over tokens with fp32 reductions, so their last bits
  * depend on the order in which the GEMM's work items finish.  Sizes: k <= 32, d and h <=
- * 65535, plus the limits of moevie_moe_forward.  `ws`: moevie_backward_workspace_size(
- * T_max, d, E, k, h, swiglu) bytes (swiglu nonzero for SwiGLU experts), set up with
- * moevie_workspace_init; device errors land in its status block. */
+ * 65535 (h_s too), plus the limits of moevie_moe_forward.  `ws`:
+ * moevie_backward_workspace_size(T_max, d, E, k, h, h_s, swiglu) bytes (swiglu nonzero for
+ * SwiGLU experts), set up with moevie_workspace_init; device errors land in its status
+ * block. */
 moevie_status moevie_backward_workspace_size(int64_t T_max, int64_t d, int64_t E, int64_t k, int64_t h,
-                                             int swiglu, size_t* bytes);
+                                             int64_t h_s, int swiglu, size_t* bytes);
 moevie_status moevie_moe_backward(const moevie_layer* layer, const void* x, const void* dy, int64_t T,
                                   const int32_t* idx, float* dx, float* dW_r, float* dW1, float* dW2,
-                                  float* dW3, void* ws, size_t ws_bytes, void* stream);
+                                  float* dW3, float* dWs1, float* dWs2, float* dWs3, void* ws,
+                                  size_t ws_bytes, void* stream);
 
 /* Synchronise `stream`, then read the workspace's device status into *out
  * (MOEVIE_OK when no device-side error was recorded).  `detail` (host, may be

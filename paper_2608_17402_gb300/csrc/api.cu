@@ -874,13 +874,13 @@ namespace {
 struct BwdLayout {
     size_t status, wsplit, wrt, wpart, wexp, sig, gate, hist, counts, offsets, tiles, n_tiles, perm,
         inv, poff, ptok, pgate, slot_prow, ptiles, n_ptiles, dx_items, n_dx_items, it2, n_it2, it1, n_it1,
-        itr, n_itr, H, U, DU, V, DV, Gm, Xp, dgp, DS, dwr;
-    int64_t rows_max, max_it2, max_it1, max_itr;
+        itr, n_itr, H, U, DU, V, DV, Gm, Xp, dgp, DS, dwr, its2, n_its2, its1, n_its1, Hs, Us, DUs, Vs, DVs;
+    int64_t rows_max, max_it2, max_it1, max_itr, max_its2, max_its1;
     int nt_h;
     size_t total;
 };
 
-BwdLayout make_bwd_layout(int64_t T, int64_t d, int64_t E, int64_t k, int64_t h, bool swiglu) {
+BwdLayout make_bwd_layout(int64_t T, int64_t d, int64_t E, int64_t k, int64_t h, int64_t hs, bool swiglu) {
     BwdLayout L;
     size_t o = 0;
     auto take = [&](size_t bytes) {
@@ -897,6 +897,10 @@ BwdLayout make_bwd_layout(int64_t T, int64_t d, int64_t E, int64_t k, int64_t h,
     L.max_it2 = bwd_max_items(L.rows_max, (int)E, (int)h, (int)d, bn_d);
     L.max_it1 = bwd_max_items(L.rows_max, (int)E, (int)d, (int)h, bn_h);
     L.max_itr = bwd_max_items(T, 1, (int)d, (int)Ep, bn_e);
+    int bn_s = 0, nt_s = 0;
+    if (hs > 0) choose_bn((int)hs, &bn_s, &nt_s);
+    L.max_its2 = hs > 0 ? bwd_max_items(T, 1, (int)hs, (int)d, bn_d) : 0;   // dWs2 [h_s, d]
+    L.max_its1 = hs > 0 ? bwd_max_items(T, 1, (int)d, (int)hs, bn_s) : 0;   // dWs1 [d, h_s]
     L.status = take(sizeof(DevStatus));
     L.wsplit = take(2 * 2 * dp * Ep);
     L.wrt = take(4 * E * dp);
@@ -935,14 +939,26 @@ BwdLayout make_bwd_layout(int64_t T, int64_t d, int64_t E, int64_t k, int64_t h,
     L.dgp = take(4 * 2 * (int64_t)L.nt_h * L.rows_max);
     L.DS = take(2 * T * Ep);
     L.dwr = take(4 * d * Ep);
+    if (hs > 0) {   // the shared expert: every token, one dense group of h_s hidden units
+        const int64_t hsp = row_ld(hs);
+        L.its2 = take(16 * L.max_its2);
+        L.n_its2 = take(4);
+        L.its1 = take(16 * L.max_its1);
+        L.n_its1 = take(4);
+        L.Hs = take(2 * T * hsp);
+        L.Us = take(2 * T * hsp);
+        L.DUs = take(2 * T * hsp);
+        L.Vs = swiglu ? take(2 * T * hsp) : 0;
+        L.DVs = swiglu ? take(2 * T * hsp) : 0;
+    }
     L.total = o;
     return L;
 }
 
-moevie_status check_bwd_sizes(int64_t T, int64_t d, int64_t E, int64_t k, int64_t h) {
-    moevie_status c = check_sizes(T, d, E, k, h, 0);
+moevie_status check_bwd_sizes(int64_t T, int64_t d, int64_t E, int64_t k, int64_t h, int64_t hs) {
+    moevie_status c = check_sizes(T, d, E, k, h, hs);
     if (c != MOEVIE_OK) return c;
-    if (h <= 0 || k > 32 || d > 65535 || h > 65535 || T * k + 63 * E >= (int64_t(1) << 31))
+    if (h <= 0 || k > 32 || d > 65535 || h > 65535 || hs > 65535 || T * k + 63 * E >= (int64_t(1) << 31))
         return MOEVIE_ERR_UNSUPPORTED;
     return MOEVIE_OK;
 }
@@ -952,23 +968,24 @@ moevie_status check_bwd_sizes(int64_t T, int64_t d, int64_t E, int64_t k, int64_
 extern "C" {
 
 moevie_status moevie_backward_workspace_size(int64_t T_max, int64_t d, int64_t E, int64_t k, int64_t h,
-                                             int swiglu, size_t* bytes) {
+                                             int64_t h_s, int swiglu, size_t* bytes) {
     if (!bytes) return MOEVIE_ERR_INVALID_ARG;
-    const moevie_status c = check_bwd_sizes(T_max, d, E, k, h);
+    const moevie_status c = check_bwd_sizes(T_max, d, E, k, h, h_s);
     if (c != MOEVIE_OK) return c;
-    *bytes = make_bwd_layout(T_max, d, E, k, h, swiglu != 0).total;
+    *bytes = make_bwd_layout(T_max, d, E, k, h, h_s, swiglu != 0).total;
     return MOEVIE_OK;
 }
 
 moevie_status moevie_moe_backward(const moevie_layer* Lr, const void* x, const void* dy, int64_t T,
                                   const int32_t* idx, float* dx, float* dW_r, float* dW1, float* dW2,
-                                  float* dW3, void* ws, size_t ws_bytes, void* stream) {
+                                  float* dW3, float* dWs1, float* dWs2, float* dWs3, void* ws, size_t ws_bytes,
+                                  void* stream) {
     if (!Lr) return MOEVIE_ERR_INVALID_ARG;
-    const int64_t d = Lr->d, E = Lr->E, k = Lr->k, h = Lr->h;
-    moevie_status c = check_bwd_sizes(T, d, E, k, h);
+    const int64_t d = Lr->d, E = Lr->E, k = Lr->k, h = Lr->h, hs = Lr->h_s;
+    moevie_status c = check_bwd_sizes(T, d, E, k, h, hs);
     if (c != MOEVIE_OK) return c;
-    if (Lr->h_s > 0) return MOEVIE_ERR_UNSUPPORTED;   // no shared expert on this path
     const bool swiglu = Lr->W3 != nullptr;
+    const bool shared = hs > 0;
     if (T == 0) return MOEVIE_OK;
     if (!x || !dy || !idx || !dx || !dW_r || !dW1 || !dW2 || !ws || !Lr->W_r || !Lr->W1 || !Lr->W2)
         return MOEVIE_ERR_INVALID_ARG;
@@ -976,7 +993,13 @@ moevie_status moevie_moe_backward(const moevie_layer* Lr, const void* x, const v
     if (!a16(x) || !a16(dy) || !a16(idx) || !a16(dx) || !a16(dW1) || !a16(dW2) || !a16(ws) || !a16(Lr->W1) ||
         !a16(Lr->W2))
         return MOEVIE_ERR_INVALID_ARG;
-    const BwdLayout L = make_bwd_layout(T, d, E, k, h, swiglu);
+    if (shared) {   // the shared expert's weights and gradients (Ws3, dWs3 with SwiGLU experts)
+        if (!Lr->Ws1 || !Lr->Ws2 || !dWs1 || !dWs2 || !a16(Lr->Ws1) || !a16(Lr->Ws2) || !a16(dWs1) ||
+            !a16(dWs2))
+            return MOEVIE_ERR_INVALID_ARG;
+        if (swiglu && (!Lr->Ws3 || !dWs3 || !a16(Lr->Ws3) || !a16(dWs3))) return MOEVIE_ERR_INVALID_ARG;
+    }
+    const BwdLayout L = make_bwd_layout(T, d, E, k, h, hs, swiglu);
     if (ws_bytes < L.total) return MOEVIE_ERR_WORKSPACE;
     cudaStream_t s = static_cast<cudaStream_t>(stream);
     DevStatus* st = at<DevStatus>(ws, L.status);
@@ -1023,11 +1046,25 @@ moevie_status moevie_moe_backward(const moevie_layer* Lr, const void* x, const v
                             at<int32_t>(ws, L.n_it1), st, s));
     MV_TRY(launch_bwd_items(nullptr, 1, T, (int)d, (int)Ep, bn_e, (int)L.max_itr, at<int4>(ws, L.itr),
                             at<int32_t>(ws, L.n_itr), st, s));
+    int bn_s = 0, nt_s = 0;
+    const int64_t hsp = shared ? row_ld(hs) : 0;
+    if (shared) {
+        choose_bn((int)hs, &bn_s, &nt_s);
+        MV_TRY(launch_bwd_items(nullptr, 1, T, (int)hs, (int)d, bn_d, (int)L.max_its2, at<int4>(ws, L.its2),
+                                at<int32_t>(ws, L.n_its2), st, s));
+        MV_TRY(launch_bwd_items(nullptr, 1, T, (int)d, (int)hs, bn_s, (int)L.max_its1, at<int4>(ws, L.its1),
+                                at<int32_t>(ws, L.n_its1), st, s));
+    }
     // 3. accumulators cleared; gathered copies of x and g dy
     MV_TRY(launch_zero_f32(dx, T * d, s));
     MV_TRY(launch_zero_f32(dW1, E * d * hp, s));
     MV_TRY(launch_zero_f32(dW2, E * h * d, s));
     if (swiglu) MV_TRY(launch_zero_f32(dW3, E * d * hp, s));
+    if (shared) {
+        MV_TRY(launch_zero_f32(dWs1, d * hsp, s));
+        MV_TRY(launch_zero_f32(dWs2, hs * d, s));
+        if (swiglu) MV_TRY(launch_zero_f32(dWs3, d * hsp, s));
+    }
     MV_TRY(launch_zero_f32(dwr, d * Ep, s));
     MV_TRY(launch_zero_f32(reinterpret_cast<float*>(DS), T * Ep / 2, s));
     MV_TRY(launch_bwd_gather(xb, static_cast<const __nv_bfloat16*>(dy), ptok, pgate, poff, (int)E, (int)d,
@@ -1135,7 +1172,7 @@ moevie_status moevie_moe_backward(const moevie_layer* Lr, const void* x, const v
     //    dW1[e] = x^T du; and dW_r = x^T ds over all tokens
     auto wgrad = [&](const void* A, int64_t a_cols, int64_t a_rows, int64_t lda, const void* B, int64_t N,
                      int64_t n_ld, int64_t b_rows, int G, int M, size_t items, size_t n_items, int64_t max_items,
-                     float* out, int64_t ldy) {
+                     float* out, int64_t ldy, float scale = 1.0f) {
         GemmSpec g{};
         g.A = A;
         g.a_mn = 1;
@@ -1158,7 +1195,7 @@ moevie_status moevie_moe_backward(const moevie_layer* Lr, const void* x, const v
         g.yacc = out;
         g.ldy = ldy;
         g.o_nrows = (int64_t)G * M;
-        g.scale = 1.0f;
+        g.scale = scale;
         return run_gemm(g, st, s);
     };
     if ((c = wgrad(H, h, L.rows_max, hp, Gm, d, d, L.rows_max, (int)E, (int)h, L.it2, L.n_it2, L.max_it2, dW2,
@@ -1173,6 +1210,94 @@ moevie_status moevie_moe_backward(const moevie_layer* Lr, const void* x, const v
     if ((c = wgrad(x, d, T, d, DS, Ep, Ep, T, 1, (int)d, L.itr, L.n_itr, L.max_itr, dwr, Ep)) != MOEVIE_OK)
         return c;
     MV_TRY(launch_bwd_copy(dwr, Ep, dW_r, d, E, s));
+    if (!shared) return MOEVIE_OK;
+    // 9. the shared expert (Eq. 6, second term), every token with the constant weight lambda,
+    //    one dense group of h_s hidden units through the same GEMMs: u_s = x Ws1 and a_s again,
+    //    du_s = lambda (dy Ws2^T) GELU'(u_s) (SwiGLU: du_s, dv_s), dx += du_s Ws1^T (+ dv_s Ws3^T),
+    //    dWs2 = lambda a_s^T dy, dWs1 = x^T du_s, dWs3 = x^T dv_s
+    void* Hs = at<void>(ws, L.Hs);
+    void* Us = at<void>(ws, L.Us);
+    void* DUs = at<void>(ws, L.DUs);
+    void* Vs = swiglu ? at<void>(ws, L.Vs) : nullptr;
+    void* DVs = swiglu ? at<void>(ws, L.DVs) : nullptr;
+    {
+        GemmSpec g{};
+        g.A = x;
+        g.lda = d;
+        g.a_ident = 1;
+        g.a_nrows = T;
+        g.m_total = T;
+        g.G = 1;
+        g.W = Lr->Ws1;
+        g.K = (int)d;
+        g.N = (int)hs;
+        g.N_ld = hsp;
+        g.epi = EPI_GELU2_BF16;
+        if (swiglu) {
+            g.epi = EPI_SWIGLU_BF16;
+            g.W3 = Lr->Ws3;
+            g.out3 = Vs;
+        }
+        g.out = Hs;
+        g.out2 = Us;
+        g.ldo = hsp;
+        if ((c = run_gemm(g, st, s)) != MOEVIE_OK) return c;
+    }
+    {
+        GemmSpec g{};
+        g.A = dy;
+        g.lda = d;
+        g.a_ident = 1;
+        g.a_nrows = T;
+        g.m_total = T;
+        g.G = 1;
+        g.W = Lr->Ws2;
+        g.b_kmajor = 1;
+        g.b_k_ld = d;
+        g.b_g_ld = hs * d;
+        g.K = (int)d;
+        g.N = (int)hs;
+        g.N_ld = hsp;
+        g.epi = swiglu ? EPI_DSWIGLU_BF16 : EPI_DGELU_BF16;
+        g.scale = Lr->lambda;
+        g.epi_u = Us;
+        g.epi_v = Vs;
+        g.epi_a = Hs;
+        g.out = DUs;
+        g.out2 = DVs;
+        g.ldo = hsp;
+        if ((c = run_gemm(g, st, s)) != MOEVIE_OK) return c;
+    }
+    for (int pass = 0; pass < (swiglu ? 2 : 1); ++pass) {
+        GemmSpec g{};
+        g.A = pass ? DVs : DUs;
+        g.lda = hsp;
+        g.a_cols = hs;
+        g.a_nrows = T;
+        g.m_total = T;
+        g.G = 1;
+        g.W = pass ? Lr->Ws3 : Lr->Ws1;
+        g.b_kmajor = 1;
+        g.b_k_ld = hsp;
+        g.b_g_ld = d * hsp;
+        g.K = (int)hs;
+        g.N = (int)d;
+        g.epi = EPI_ADD_F32;
+        g.yacc = dx;
+        g.ldy = d;
+        g.o_nrows = T;
+        g.scale = 1.0f;
+        if ((c = run_gemm(g, st, s)) != MOEVIE_OK) return c;
+    }
+    if ((c = wgrad(Hs, hs, T, hsp, dy, d, d, T, 1, (int)hs, L.its2, L.n_its2, L.max_its2, dWs2, d,
+                   Lr->lambda)) != MOEVIE_OK)
+        return c;
+    if ((c = wgrad(x, d, T, d, DUs, hs, hsp, T, 1, (int)d, L.its1, L.n_its1, L.max_its1, dWs1, hsp)) !=
+        MOEVIE_OK)
+        return c;
+    if (swiglu && (c = wgrad(x, d, T, d, DVs, hs, hsp, T, 1, (int)d, L.its1, L.n_its1, L.max_its1, dWs3,
+                             hsp)) != MOEVIE_OK)
+        return c;
     return MOEVIE_OK;
 }
 

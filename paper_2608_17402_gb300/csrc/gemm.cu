@@ -886,7 +886,8 @@ __device__ void epilogue(const GemmArgs& p, const Smem& sm, uint32_t tmem, int64
                 }
             }
         }
-        if (TRAIN && !to_f32 && (p.epi == EPI_DGELU_BF16 || p.epi == EPI_DSWIGLU_BF16) && ok_row)   // row dot
+        if (TRAIN && !to_f32 && (p.epi == EPI_DGELU_BF16 || p.epi == EPI_DSWIGLU_BF16) && ok_row &&
+            p.dg_part)   // row dot (the gates' gradient; none for the shared expert)
             p.dg_part[(int64_t)(2 * (t.n0 / p.n_step) + half) * p.m_total + gr] = dg_acc;
     }
 }

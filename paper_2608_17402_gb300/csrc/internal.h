@@ -280,7 +280,7 @@ struct GemmArgs {
     const __nv_bfloat16* epi_u; // EPI_DGELU_BF16 / EPI_DSWIGLU_BF16: pre-activations u (and v)
     const __nv_bfloat16* epi_v; //   and activations a of the GEMM rows, [m_total][ldo] bf16
     const __nv_bfloat16* epi_a;
-    float* dg_part;             // EPI_D*_BF16: per-row partial dots, [2 n_ntiles][m_total] fp32
+    float* dg_part;             // EPI_D*_BF16: per-row partial dots, [2 n_ntiles][m_total] fp32 (or NULL: none)
     DevStatus* status;
     uint64_t limit_ns;
 };

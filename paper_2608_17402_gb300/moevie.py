@@ -78,8 +78,8 @@ def load():
         "moevie_launch_count": ([], ctypes.c_uint64),
         "moevie_shared_groups": ([I64] * 6, ctypes.c_int64),
         "moevie_update_bias": ([P, I64, F, ctypes.c_int, P, P, SZ, P], ctypes.c_int),
-        "moevie_backward_workspace_size": ([I64] * 5 + [ctypes.c_int, P], ctypes.c_int),
-        "moevie_moe_backward": ([P, P, P, I64, P, P, P, P, P, P, P, SZ, P], ctypes.c_int),
+        "moevie_backward_workspace_size": ([I64] * 6 + [ctypes.c_int, P], ctypes.c_int),
+        "moevie_moe_backward": ([P, P, P, I64, P, P, P, P, P, P, P, P, P, P, SZ, P], ctypes.c_int),
         "moevie_test_route_logits": ([P, P, I64, I64, I64, P, P, SZ, P], ctypes.c_int),
         "moevie_test_fallback_count": ([P, P, P], ctypes.c_int),
         "moevie_test_expert_hidden": ([P, P, P, P, I64, I64, I64, I64, I64, P, P, SZ, P],
@@ -332,33 +332,34 @@ def moevie_moe_forward(layer: LayerWeights, x, ws: Workspace, y=None, routing=Fa
     return (y, rt) if routing else y
 
 
-def moevie_backward_workspace_size(T_max, d, E, k, h, swiglu=False) -> int:
+def moevie_backward_workspace_size(T_max, d, E, k, h, h_s=0, swiglu=False) -> int:
     out = ctypes.c_size_t(0)
-    _call("moevie_backward_workspace_size", T_max, d, E, k, h, int(bool(swiglu)), ctypes.byref(out))
+    _call("moevie_backward_workspace_size", T_max, d, E, k, h, h_s, int(bool(swiglu)), ctypes.byref(out))
     return out.value
 
 
 class BackwardWorkspace(Workspace):
     """Caller-owned device scratch of moevie_moe_backward (up to ``T_max`` tokens;
-    ``swiglu`` for SwiGLU experts)."""
+    ``h_s`` the shared expert's width, 0 for none; ``swiglu`` for SwiGLU experts)."""
 
-    def __init__(self, T_max, d, E, k, h, swiglu=False, device="cuda", stream=None):
-        self.dims = (T_max, d, E, k, h, swiglu)
-        self.nbytes = moevie_backward_workspace_size(T_max, d, E, k, h, swiglu)
+    def __init__(self, T_max, d, E, k, h, h_s=0, swiglu=False, device="cuda", stream=None):
+        self.dims = (T_max, d, E, k, h, h_s, swiglu)
+        self.nbytes = moevie_backward_workspace_size(T_max, d, E, k, h, h_s, swiglu)
         self.buf = torch.empty(self.nbytes, dtype=torch.uint8, device=device)
         moevie_workspace_init(self, stream)
 
 
 def moevie_moe_backward(layer: LayerWeights, x, dy, idx, ws: "BackwardWorkspace", stream=None):
     """Gradients of sum(dy * y) with the selection idx held fixed (GELU or SwiGLU
-    experts, no shared expert).  Returns a dict of fp32 tensors: dx [T, d], dW_r [d, E],
-    dW1 [E, d, h] (a view of rows row_ld(h) apart), dW2 [E, h, d], and dW3 (as dW1) for
-    SwiGLU experts."""
+    experts, with or without a shared expert).  Returns a dict of fp32 tensors: dx [T, d],
+    dW_r [d, E], dW1 [E, d, h] (a view of rows row_ld(h) apart), dW2 [E, h, d], dW3 (as
+    dW1) for SwiGLU experts, and with a shared expert dWs1 [d, h_s] (a view of rows
+    row_ld(h_s) apart), dWs2 [h_s, d] and, for SwiGLU, dWs3 (as dWs1)."""
     _want(x, torch.bfloat16, "x")
     _want(dy, torch.bfloat16, "dy")
     _want(idx, torch.int32, "idx")
     T, d = x.shape
-    _, E, k, h, _ = layer.dims
+    _, E, k, h, hs = layer.dims
     dev = x.device
     out = {"dx": torch.empty((T, d), dtype=torch.float32, device=dev),
            "dW_r": torch.empty((d, E), dtype=torch.float32, device=dev),
@@ -366,12 +367,19 @@ def moevie_moe_backward(layer: LayerWeights, x, dy, idx, ws: "BackwardWorkspace"
            "dW2": torch.empty((E, h, d), dtype=torch.float32, device=dev)}
     if layer.W3 is not None:
         out["dW3"] = torch.empty((E, d, row_ld(h)), dtype=torch.float32, device=dev)
+    if hs > 0:
+        out["dWs1"] = torch.empty((d, row_ld(hs)), dtype=torch.float32, device=dev)
+        out["dWs2"] = torch.empty((hs, d), dtype=torch.float32, device=dev)
+        if layer.W3 is not None:
+            out["dWs3"] = torch.empty((d, row_ld(hs)), dtype=torch.float32, device=dev)
     L = layer.c_struct()
     _call("moevie_moe_backward", ctypes.byref(L), _p(x), _p(dy), T, _p(idx), _p(out["dx"]), _p(out["dW_r"]),
-          _p(out["dW1"]), _p(out["dW2"]), _p(out.get("dW3")), ws.ptr, ws.nbytes, _stream(stream))
+          _p(out["dW1"]), _p(out["dW2"]), _p(out.get("dW3")), _p(out.get("dWs1")), _p(out.get("dWs2")),
+          _p(out.get("dWs3")), ws.ptr, ws.nbytes, _stream(stream))
     out["dW1"] = out["dW1"][..., :h]
-    if "dW3" in out:
-        out["dW3"] = out["dW3"][..., :h]
+    for name, w in (("dW3", h), ("dWs1", hs), ("dWs3", hs)):
+        if name in out:
+            out[name] = out[name][..., :w]
     return out
 
 

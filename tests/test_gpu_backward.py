@@ -1,5 +1,6 @@
 """Training path (App. B: grouped GEMMs with the activation as its own step) of
-moevie_moe_backward, GELU and SwiGLU experts, against the oracle's backward (the gradients of sum_t dy_t . y_t
+moevie_moe_backward, GELU and SwiGLU experts, with and without the shared expert of Eq. 6,
+against the oracle's backward (the gradients of sum_t dy_t . y_t
 with the top-k selection held fixed, through the renormalised gates of Eqs. 4-5 into
 W_r and x; the bias gets none), element by element, on the same seeded inputs and
 the same bf16 dy.  Tolerance as for the forward (rel-L2 <= 1e-2, max |err| <= 5e-2 RMS)
@@ -30,7 +31,7 @@ def _dy(T, d, seed, tokens=None):
 def _gpu_backward(lay, dy_bits, idx):
     c = lay.cfg
     x, W = layer_to_device(lay)
-    ws = moevie.BackwardWorkspace(c.T, c.d, c.E, c.k, c.h, swiglu=lay.W3 is not None)
+    ws = moevie.BackwardWorkspace(c.T, c.d, c.E, c.k, c.h, h_s=c.h_s, swiglu=lay.W3 is not None)
     g = moevie.moevie_moe_backward(W, x, dev_bf16(dy_bits), dev(np.ascontiguousarray(idx, np.int32)), ws)
     check_status(ws)
     return {k: to_np_f64(v) for k, v in g.items()}
@@ -39,8 +40,8 @@ def _gpu_backward(lay, dy_bits, idx):
 def _compare(got, want, label):
     out = {}
     names = [("dx", "dx"), ("dW_r", "dWr"), ("dW1", "dW1"), ("dW2", "dW2")]
-    if "dW3" in want:
-        names.append(("dW3", "dW3"))
+    names += [(n, n) for n in ("dW3", "dWs1", "dWs2", "dWs3") if n in want]
+    assert sorted(got) == sorted(g for g, _ in names), (sorted(got), names)
     for g_name, o_name in names:
         if not np.any(want[o_name]):   # e.g. dW_r with one expert: exactly zero
             assert not np.any(got[g_name]), f"{label} {g_name}: expected exact zeros"
@@ -102,62 +103,130 @@ def test_backward_batch1_layer_every_token():
     print("c2 backward:", {k: f"rel-L2 {v[0]:.2e}, max|err|/RMS {v[1]:.2e}" for k, v in r.items()})
 
 
+def _compare_sampled(got, want, idx, toks, T, E, label):
+    """Gradients of a full-size layer whose dy is nonzero on the tokens `toks` only: the
+    other tokens' rows of dx exactly zero; dx on `toks`, dW_r and the shared expert's
+    gradients against their own RMS; the experts' gradients expert by expert.
+
+    With a few dozen of the tokens the experts' gradients are very uneven (a saturated
+    expert takes them all, most others one or two): an expert reached by fewer than 8 of
+    the tokens has a weight gradient of rank below 8 (a sum of outer products x_t du_t, or
+    a_t (g dy_t)), whose largest element exceeds its RMS by about the product of the two
+    vectors' peak-to-RMS ratios (20-30); the bf16 rounding of the operands (2^-9 relative
+    each) then reaches 5-10% of the RMS at those elements, so such slices keep the relative
+    L2 bound of 1e-2 but take 0.25 x RMS as a guard against gross errors for the largest one
+    (a wrong element is off by about its own value, tens of RMS there)."""
+    others = np.setdiff1d(np.arange(T), toks)
+    assert not np.any(got["dx"][others])
+    rows = np.bincount(idx[toks].ravel(), minlength=E)
+    worst = {"dx": assert_close(got["dx"][toks], want["dx"][toks], f"{label} dx"),
+             "dW_r": assert_close(got["dW_r"], want["dWr"], f"{label} dW_r")}
+    for name in ("dWs1", "dWs2", "dWs3"):
+        if name in want:
+            worst[name] = assert_close(got[name], want[name], f"{label} {name}")
+    for name in ("dW1", "dW2", "dW3"):
+        if name not in want:
+            continue
+        w = (0.0, 0.0)
+        for e in range(E):
+            if not np.any(want[name][e]):
+                assert not np.any(got[name][e]), f"{label} {name}[{e}]: expected exact zeros"
+                continue
+            if rows[e] >= 8:
+                rel, mx = assert_close(got[name][e], want[name][e], f"{label} {name}[{e}]")
+            else:
+                ge, we = got[name][e], want[name][e]
+                rel = float(np.linalg.norm(ge - we) / np.linalg.norm(we))
+                mx = float(np.abs(ge - we).max() / np.sqrt(np.mean(we ** 2)))
+                assert rel <= 1e-2 and mx <= 0.25, (label, name, e, int(rows[e]), rel, mx)
+            w = (max(w[0], rel), max(w[1], mx))
+        worst[name] = w
+    return worst
+
+
+def _sampled_run(name, n_tok, seed):
+    lay = workloads.make_layer(workloads.CONFIGS[name])
+    c = lay.cfg
+    rng = np.random.default_rng(seed)
+    toks = np.unique(np.concatenate([[0, c.T - 1], rng.choice(c.T, n_tok - 2, replace=False)]))
+    dy_bits, dyf = _dy(c.T, c.d, seed + 6, toks)
+    idx, _, _ = oracle.route(lay.x, lay.Wr, lay.b, c.k)
+    want = oracle.backward(lay.x, lay.Wr, lay.b, lay.W1, lay.W2, c.k, dyf, Ws1=lay.Ws1, Ws2=lay.Ws2,
+                           lam=c.lam, W3=lay.W3, Ws3=lay.Ws3)
+    got = _gpu_backward(lay, dy_bits, idx)
+    worst = _compare_sampled(got, want, idx, toks, c.T, c.E, name)
+    print(f"{name} backward ({len(toks)} tokens; worst expert):",
+          {k: f"rel-L2 {v[0]:.2e}, max|err|/RMS {v[1]:.2e}" for k, v in worst.items()})
+
+
 def test_backward_stress_layer_sampled_tokens():
     """The stress layer (T = 65536, E = 256, one saturated expert) at full size with dy
     nonzero on 64 tokens chosen across the token range: the oracle's backward costs only
     those tokens, and every gradient (all of dx, dW_r, dW1, dW2) must match it, the rows
     of the other tokens exactly zero in dx."""
-    lay = workloads.make_layer(workloads.CONFIGS["c4"])
+    _sampled_run("c4", 64, 3)
+
+
+@pytest.mark.parametrize("name", ["pB", "pL"])
+def test_backward_paper_layers_every_token(name):
+    """The paper's B and L layers (31 routed SwiGLU experts plus a SwiGLU shared expert
+    of the same width; L's h = 684 leaves K and N tails) on every token."""
+    lay = workloads.make_layer(workloads.CONFIGS[name])
     c = lay.cfg
-    rng = np.random.default_rng(3)
-    toks = np.unique(np.concatenate([[0, c.T - 1], rng.choice(c.T, 62, replace=False)]))
-    dy_bits, dyf = _dy(c.T, c.d, 9, toks)
+    dy_bits, dyf = _dy(c.T, c.d, 35)
     idx, _, _ = oracle.route(lay.x, lay.Wr, lay.b, c.k)
-    want = oracle.backward(lay.x, lay.Wr, lay.b, lay.W1, lay.W2, c.k, dyf)
+    want = oracle.backward(lay.x, lay.Wr, lay.b, lay.W1, lay.W2, c.k, dyf, Ws1=lay.Ws1, Ws2=lay.Ws2,
+                           lam=c.lam, W3=lay.W3, Ws3=lay.Ws3)
+    r = _compare(_gpu_backward(lay, dy_bits, idx), want, name)
+    print(f"{name} backward:", {k: f"rel-L2 {v[0]:.2e}, max|err|/RMS {v[1]:.2e}" for k, v in r.items()})
+
+
+def test_backward_paper_huge_layer_sampled_tokens():
+    """The paper's H layer (h = 854, k = 7, with the shared expert) at full size, dy nonzero
+    on 2048 tokens (every expert then sees more than 150 of them)."""
+    _sampled_run("pH", 2048, 11)
+
+
+@pytest.mark.parametrize("T,d,E,k,h,h_s,lam,act", [
+    (300, 256, 16, 4, 128, 256, 1.0, "gelu"),
+    (257, 128, 8, 2, 96, 100, 0.5, "gelu"),     # h_s % 8 == 4: rows of Ws1 and dWs1 104 apart
+    (1, 64, 4, 2, 64, 64, 1.0, "gelu"),
+    (200, 96, 12, 3, 100, 64, 1.0, "swiglu"),
+    (64, 64, 1, 1, 48, 48, 2.0, "swiglu"),       # one expert: W_r's gradient exactly zero
+    (600, 512, 33, 5, 256, 1024, 1.0, "swiglu"),
+])
+def test_backward_shared_small(T, d, E, k, h, h_s, lam, act):
+    """With the shared expert (Eq. 6, weight lambda): dWs1, dWs2 (and dWs3 for SwiGLU)
+    beside the routed gradients, and its share of dx."""
+    cfg = workloads.small_config(T, d, E, k, h, h_s=h_s, lam=lam, seed=T + h_s, act=act)
+    lay = workloads.make_layer(cfg)
+    dy_bits, dyf = _dy(T, d, T + 7)
+    idx, _, _ = oracle.route(lay.x, lay.Wr, lay.b, k)
+    want = oracle.backward(lay.x, lay.Wr, lay.b, lay.W1, lay.W2, k, dyf, Ws1=lay.Ws1, Ws2=lay.Ws2, lam=lam,
+                           W3=lay.W3, Ws3=lay.Ws3)
     got = _gpu_backward(lay, dy_bits, idx)
-    others = np.setdiff1d(np.arange(c.T), toks)
-    assert not np.any(got["dx"][others])
-    # with 64 of 65536 tokens the gradients are very uneven (the saturated expert takes all
-    # 64, most others one or two): compare dx on those tokens, and the expert weight
-    # gradients expert by expert, each against its own RMS.  An expert reached by fewer
-    # than 8 of the tokens has a weight gradient of rank below 8 (a sum of outer products
-    # x_t du_t, or a_t (g dy_t)), whose largest element exceeds its RMS by about the
-    # product of the two vectors' peak-to-RMS ratios (20-30); the bf16 rounding of the
-    # operands (2^-9 relative each) then reaches 5-10% of the RMS at those elements, so
-    # such slices keep the relative L2 bound of 1e-2 but take 0.25 x RMS as a guard against
-    # gross errors for the largest one (a wrong element is off by about its own value,
-    # tens of RMS there).
-    rows = np.bincount(idx[toks].ravel(), minlength=c.E)
-    rel, mx = assert_close(got["dx"][toks], want["dx"][toks], "c4 dx")
-    worst = {"dx": (rel, mx)}
-    rel, mx = assert_close(got["dW_r"], want["dWr"], "c4 dW_r")
-    worst["dW_r"] = (rel, mx)
-    for g_name, o_name in (("dW1", "dW1"), ("dW2", "dW2")):
-        w = (0.0, 0.0)
-        for e in range(c.E):
-            if not np.any(want[o_name][e]):
-                assert not np.any(got[g_name][e]), f"c4 {g_name}[{e}]: expected exact zeros"
-                continue
-            if rows[e] >= 8:
-                rel, mx = assert_close(got[g_name][e], want[o_name][e], f"c4 {g_name}[{e}]")
-            else:
-                ge, we = got[g_name][e], want[o_name][e]
-                rel = float(np.linalg.norm(ge - we) / np.linalg.norm(we))
-                mx = float(np.abs(ge - we).max() / np.sqrt(np.mean(we ** 2)))
-                assert rel <= 1e-2 and mx <= 0.25, (g_name, e, int(rows[e]), rel, mx)
-            w = (max(w[0], rel), max(w[1], mx))
-        worst[g_name] = w
-    print("c4 backward (64 tokens; worst expert):",
-          {k: f"rel-L2 {v[0]:.2e}, max|err|/RMS {v[1]:.2e}" for k, v in worst.items()})
+    _compare(got, want, f"shared {act} T={T} d={d} E={E} k={k} h={h} h_s={h_s}")
+
+
+def test_backward_shared_expert_layer_every_token():
+    """The image layer with a shared expert (c1: T = 8192, d = 1024, E = 64, k = 8, h = 512,
+    h_s = 1024) on every token."""
+    lay = workloads.make_layer(workloads.CONFIGS["c1"])
+    c = lay.cfg
+    dy_bits, dyf = _dy(c.T, c.d, 25)
+    idx, _, _ = oracle.route(lay.x, lay.Wr, lay.b, c.k)
+    want = oracle.backward(lay.x, lay.Wr, lay.b, lay.W1, lay.W2, c.k, dyf, Ws1=lay.Ws1, Ws2=lay.Ws2, lam=c.lam)
+    r = _compare(_gpu_backward(lay, dy_bits, idx), want, "c1")
+    print("c1 backward:", {k: f"rel-L2 {v[0]:.2e}, max|err|/RMS {v[1]:.2e}" for k, v in r.items()})
 
 
 def test_backward_rejects_unsupported_layers():
-    """A shared expert is outside this entry point: rejected before any launch."""
-    cfg = workloads.small_config(16, 64, 4, 2, 64, h_s=64)
+    """k above 32 is outside this entry point: rejected before any launch."""
+    cfg = workloads.small_config(16, 64, 40, 33, 64)
     lay = workloads.make_layer(cfg)
     x, W = layer_to_device(lay)
-    ws = moevie.BackwardWorkspace(16, 64, 4, 2, 64)
-    idx = dev(np.zeros((16, 2), np.int32) + np.array([0, 1], np.int32))
+    ws = moevie.BackwardWorkspace(16, 64, 40, 32, 64)
+    idx = dev(np.zeros((16, 33), np.int32) + np.arange(33, dtype=np.int32))
     n0 = moevie.moevie_launch_count()
     with pytest.raises(moevie.MoevieError) as e:
         moevie.moevie_moe_backward(W, x, x, idx, ws)
