@@ -48,6 +48,10 @@ def parse():
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-backward", action="store_true", help="skip timing the training path")
+    ap.add_argument("--gemm-calibration", action="store_true",
+                    help="instead of a layer: the library's dense GEMM pair (moevie_shared_expert: "
+                         "x Ws1 with GELU, then . Ws2) against cuBLAS (torch.matmul) on a few shapes, "
+                         "one JSON line each")
     return ap.parse_args()
 
 
@@ -474,10 +478,71 @@ def run_ours(args, rank, world):
     print(json.dumps(out), flush=True)
 
 
+CALIBRATION_SHAPES = ((16384, 4096, 8192), (8192, 8192, 8192), (65536, 1664, 3328), (65536, 1664, 512))
+
+
+def gemm_calibration(args):
+    """The grouped GEMM kernel on plain dense problems, beside cuBLAS on the same shapes:
+    moevie_shared_expert runs it twice (T x d by d x h_s with the GELU epilogue, then
+    T x h_s by h_s x d), both operands by TMA, no gather, no reductions.  This separates
+    the kernel's main loop from what the grouped layer adds (partial m-tiles, the token
+    gather, the y reductions).  L2 flushed before every timed call; CUDA events; median
+    of `steps` calls."""
+    import torch
+
+    from paper_2608_17402_gb300 import moevie
+    torch.cuda.set_device(0)
+    flush = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device="cuda")
+    pk = peaks()
+
+    def timeit(fn):
+        for _ in range(max(3, args.warmup)):
+            fn()
+        torch.cuda.synchronize()
+        ts = []
+        for _ in range(max(1, args.steps)):
+            flush.zero_()
+            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            a.record()
+            fn()
+            b.record()
+            torch.cuda.synchronize()
+            ts.append(a.elapsed_time(b))
+        return statistics.median(ts) * 1e3   # µs
+
+    g = torch.Generator(device="cuda")
+    g.manual_seed(0)
+    for T, d, hs in CALIBRATION_SHAPES:
+        x = torch.randn((T, d), generator=g, device="cuda").to(torch.bfloat16)
+        W1 = (torch.randn((d, hs), generator=g, device="cuda") / d ** 0.5).to(torch.bfloat16)
+        W2 = (torch.randn((hs, d), generator=g, device="cuda") / hs ** 0.5).to(torch.bfloat16)
+        ws = moevie.Workspace(T, d, 1, 1, hs, hs)
+        out = torch.empty((T, d), dtype=torch.bfloat16, device="cuda")
+        hbuf = torch.empty((T, hs), dtype=torch.bfloat16, device="cuda")
+        ours = timeit(lambda: moevie.moevie_shared_expert(x, W1, W2, ws, out=out))
+        code, detail = moevie.moevie_get_device_status(ws)
+        if code != 0:
+            raise RuntimeError(f"device status {code} {detail}")
+        up = timeit(lambda: torch.matmul(x, W1, out=hbuf))
+        down = timeit(lambda: torch.matmul(hbuf, W2, out=out))
+        fl = 2.0 * T * d * hs
+        print(json.dumps({"gemm_calibration": {"T": T, "d": d, "h_s": hs},
+                          "ours_us": ours, "ours_tflops": 2 * fl / ours / 1e6,
+                          "cublas_us": up + down, "cublas_tflops": 2 * fl / (up + down) / 1e6,
+                          "cublas_up_tflops": fl / up / 1e6, "cublas_down_tflops": fl / down / 1e6,
+                          "peak_bf16_tflops": pk["bf16_tflops"], "ours_frac_of_cublas": (up + down) / ours}),
+              flush=True)
+        del x, W1, W2, ws, out, hbuf
+        torch.cuda.empty_cache()
+
+
 def main():
     args = parse()
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
+    if args.gemm_calibration:
+        gemm_calibration(args)
+        return
     if args.impl == "reference":
         run_reference(args, rank)
         return

@@ -874,7 +874,8 @@ namespace {
 struct BwdLayout {
     size_t status, wsplit, wrt, wpart, wexp, sig, gate, hist, counts, offsets, tiles, n_tiles, perm,
         inv, poff, ptok, pgate, slot_prow, ptiles, n_ptiles, dx_items, n_dx_items, it2, n_it2, it1, n_it1,
-        itr, n_itr, H, U, DU, V, DV, Gm, Xp, dgp, DS, dwr, its2, n_its2, its1, n_its1, Hs, Us, DUs, Vs, DVs;
+        itr, n_itr, H, U, DU, V, DV, Gm, Xp, dgp, DS, dwr, its2, n_its2, its1, n_its1, Hs, Us, DUs, Vs, DVs,
+        gc2, gc1, gcr, gcs2, gcs1;   // per group of each item set: 1 = its gradient is cleared first
     int64_t rows_max, max_it2, max_it1, max_itr, max_its2, max_its1;
     int nt_h;
     size_t total;
@@ -929,6 +930,11 @@ BwdLayout make_bwd_layout(int64_t T, int64_t d, int64_t E, int64_t k, int64_t h,
     L.n_it1 = take(4);
     L.itr = take(16 * L.max_itr);
     L.n_itr = take(4);
+    L.gc2 = take(4 * E);
+    L.gc1 = take(4 * E);
+    L.gcr = take(4);
+    L.gcs2 = take(4);
+    L.gcs1 = take(4);
     L.H = take(2 * L.rows_max * hp);
     L.U = take(2 * L.rows_max * hp);
     L.DU = take(2 * L.rows_max * hp);
@@ -1041,35 +1047,37 @@ moevie_status moevie_moe_backward(const moevie_layer* Lr, const void* x, const v
                            at<int32_t>(ws, L.slot_prow), s));
     MV_TRY(launch_tile_table(poff, (int)E, GM_BM, at<int4>(ws, L.ptiles), at<int32_t>(ws, L.n_ptiles), s));
     MV_TRY(launch_bwd_items(poff, (int)E, 0, (int)h, (int)d, bn_d, (int)L.max_it2, at<int4>(ws, L.it2),
-                            at<int32_t>(ws, L.n_it2), st, s));
+                            at<int32_t>(ws, L.n_it2), at<int32_t>(ws, L.gc2), st, s));
     MV_TRY(launch_bwd_items(poff, (int)E, 0, (int)d, (int)h, bn_h, (int)L.max_it1, at<int4>(ws, L.it1),
-                            at<int32_t>(ws, L.n_it1), st, s));
+                            at<int32_t>(ws, L.n_it1), at<int32_t>(ws, L.gc1), st, s));
     MV_TRY(launch_bwd_items(nullptr, 1, T, (int)d, (int)Ep, bn_e, (int)L.max_itr, at<int4>(ws, L.itr),
-                            at<int32_t>(ws, L.n_itr), st, s));
+                            at<int32_t>(ws, L.n_itr), at<int32_t>(ws, L.gcr), st, s));
     int bn_s = 0, nt_s = 0;
     const int64_t hsp = shared ? row_ld(hs) : 0;
     if (shared) {
         choose_bn((int)hs, &bn_s, &nt_s);
         MV_TRY(launch_bwd_items(nullptr, 1, T, (int)hs, (int)d, bn_d, (int)L.max_its2, at<int4>(ws, L.its2),
-                                at<int32_t>(ws, L.n_its2), st, s));
+                                at<int32_t>(ws, L.n_its2), at<int32_t>(ws, L.gcs2), st, s));
         MV_TRY(launch_bwd_items(nullptr, 1, T, (int)d, (int)hs, bn_s, (int)L.max_its1, at<int4>(ws, L.its1),
-                                at<int32_t>(ws, L.n_its1), st, s));
+                                at<int32_t>(ws, L.n_its1), at<int32_t>(ws, L.gcs1), st, s));
     }
-    // 3. accumulators cleared; gathered copies of x and g dy
+    // 3. accumulators cleared (of the weight gradients only what their items will add
+    //    into, or not write at all); gathered copies of x and g dy
+    const int sms = num_sms();
     MV_TRY(launch_zero_f32(dx, T * d, s));
-    MV_TRY(launch_zero_f32(dW1, E * d * hp, s));
-    MV_TRY(launch_zero_f32(dW2, E * h * d, s));
-    if (swiglu) MV_TRY(launch_zero_f32(dW3, E * d * hp, s));
+    MV_TRY(launch_bwd_zero(at<int32_t>(ws, L.gc1), (int)E, (int)d, (int)h, hp, dW1, sms, s));
+    MV_TRY(launch_bwd_zero(at<int32_t>(ws, L.gc2), (int)E, (int)h, (int)d, d, dW2, sms, s));
+    if (swiglu) MV_TRY(launch_bwd_zero(at<int32_t>(ws, L.gc1), (int)E, (int)d, (int)h, hp, dW3, sms, s));
     if (shared) {
-        MV_TRY(launch_zero_f32(dWs1, d * hsp, s));
-        MV_TRY(launch_zero_f32(dWs2, hs * d, s));
-        if (swiglu) MV_TRY(launch_zero_f32(dWs3, d * hsp, s));
+        MV_TRY(launch_bwd_zero(at<int32_t>(ws, L.gcs1), 1, (int)d, (int)hs, hsp, dWs1, sms, s));
+        MV_TRY(launch_bwd_zero(at<int32_t>(ws, L.gcs2), 1, (int)hs, (int)d, d, dWs2, sms, s));
+        if (swiglu) MV_TRY(launch_bwd_zero(at<int32_t>(ws, L.gcs1), 1, (int)d, (int)hs, hsp, dWs3, sms, s));
     }
-    MV_TRY(launch_zero_f32(dwr, d * Ep, s));
+    MV_TRY(launch_bwd_zero(at<int32_t>(ws, L.gcr), 1, (int)d, (int)Ep, Ep, dwr, sms, s));
     MV_TRY(launch_zero_f32(reinterpret_cast<float*>(DS), T * Ep / 2, s));
     MV_TRY(launch_bwd_gather(xb, static_cast<const __nv_bfloat16*>(dy), ptok, pgate, poff, (int)E, (int)d,
                              L.rows_max, static_cast<__nv_bfloat16*>(Xp), static_cast<__nv_bfloat16*>(Gm), s));
-    // 4. up-projection again: u = x W1[e] and a = GELU(u), both kept (bf16)
+    // 4. up-projection again: u = x W1[e] and a = GELU(u), both kept (bf16; SwiGLU: u, v and a)
     {
         GemmSpec g{};
         g.A = x;

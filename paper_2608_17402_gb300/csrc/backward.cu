@@ -18,6 +18,8 @@
 //                      [T][E_pad] bf16 matrix for dW_r = x^T ds
 #include <math.h>
 
+#include <algorithm>
+
 #include "internal.h"
 
 namespace mv {
@@ -142,11 +144,15 @@ __global__ void bwd_rows_kernel(const int32_t* __restrict__ idx, const int32_t* 
 // [koff[g] / 64, koff[g + 1] / 64) (koff == nullptr: one group of ceil(K_rows / 64)
 // k-blocks), cut into chunks of at most kch; its items are every (m-tile of 256 of M rows,
 // n-tile of BN of N columns, chunk).  items[i] = {g, m0 | n0 << 16, kb0, kb1}; *n_items =
-// their number (at most max_items; more is a device error and none are listed).
+// their number (at most max_items; more is a device error and none are listed).  A group
+// of one chunk writes each of its gradient's elements once: its items carry
+// BWD_STORE_BIT in kb1 (the GEMM stores instead of adding) and gclear[g] = 0; a group
+// with no rows or several chunks has gclear[g] = 1 (its gradient is cleared first).
 __global__ void __launch_bounds__(1024) bwd_items_kernel(const int32_t* __restrict__ koff, int G,
                                                          int64_t K_rows, int M, int N, int BN, int kch,
                                                          int max_items, int4* __restrict__ items,
-                                                         int32_t* __restrict__ n_items, DevStatus* st) {
+                                                         int32_t* __restrict__ n_items,
+                                                         int32_t* __restrict__ gclear, DevStatus* st) {
     pdl_wait();
     __shared__ int wsum[32];
     __shared__ int s_total;
@@ -192,12 +198,35 @@ __global__ void __launch_bounds__(1024) bwd_items_kernel(const int32_t* __restri
         return;
     }
     int pos = wsum[warp] + inc - v;
+    const int store = chunks == 1 ? BWD_STORE_BIT : 0;
     for (int c = 0; c < chunks; ++c) {
         const int a = kb0 + c * kch, b = min(kb1, a + kch);
         for (int m = 0; m < mt; ++m)
-            for (int n = 0; n < nt; ++n) items[pos++] = make_int4(g, (m * GM_BM) | ((n * BN) << 16), a, b);
+            for (int n = 0; n < nt; ++n)
+                items[pos++] = make_int4(g, (m * GM_BM) | ((n * BN) << 16), a, b | store);
     }
+    if (g < G) gclear[g] = chunks == 1 ? 0 : 1;
     if (g == 0) *n_items = total;
+}
+
+// The part of a weight gradient out [G][M][ld] (fp32) that the GEMM's items will not
+// write: every row of a group with gclear[g] set, and the pad columns [N, ld) of the
+// other groups' rows.  One warp per row, grid-strided; ld % 4 == 0.
+__global__ void __launch_bounds__(256) bwd_zero_kernel(const int32_t* __restrict__ gclear, int G, int M,
+                                                       int N, int64_t ld, float* __restrict__ out) {
+    pdl_wait();
+    const int lane = threadIdx.x & 31;
+    const int64_t rows = (int64_t)G * M;
+    for (int64_t q = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5; q < rows;
+         q += ((int64_t)gridDim.x * blockDim.x) >> 5) {
+        float* row = out + q * ld;
+        if (gclear[q / M]) {
+            float4* r4 = reinterpret_cast<float4*>(row);
+            for (int64_t c = lane; c < ld / 4; c += 32) r4[c] = make_float4(0.f, 0.f, 0.f, 0.f);
+        } else {
+            for (int64_t c = N + lane; c < ld; c += 32) row[c] = 0.f;
+        }
+    }
 }
 
 // Padded rows r (threads over r and 8-column groups): xp[r] = x[ptok[r]], gdy[r] =
@@ -329,10 +358,22 @@ int64_t bwd_max_items(int64_t rows, int G, int M, int N, int BN) {
 }
 
 cudaError_t launch_bwd_items(const int32_t* koff, int G, int64_t K_rows, int M, int N, int BN,
-                             int max_items, int4* items, int32_t* n_items, DevStatus* st, cudaStream_t s) {
+                             int max_items, int4* items, int32_t* n_items, int32_t* gclear, DevStatus* st,
+                             cudaStream_t s) {
     if (G > 1024) return cudaErrorInvalidValue;
     const cudaError_t e = launch_pdl(bwd_items_kernel, dim3(1), dim3(1024), 0, s, koff, G, K_rows, M, N, BN,
-                                     (int)BWD_KCH, max_items, items, n_items, st);
+                                     (int)BWD_KCH, max_items, items, n_items, gclear, st);
+    count_launches(1);
+    return e;
+}
+
+cudaError_t launch_bwd_zero(const int32_t* gclear, int G, int M, int N, int64_t ld, float* out, int num_sms,
+                            cudaStream_t s) {
+    if (ld % 4 != 0 || N > ld) return cudaErrorInvalidValue;
+    const int64_t warps = (int64_t)G * M;
+    const int64_t blocks = std::min<int64_t>((warps + 7) / 8, (int64_t)num_sms * 8);
+    const cudaError_t e = launch_pdl(bwd_zero_kernel, dim3((unsigned)std::max<int64_t>(blocks, 1)), dim3(256), 0, s,
+                                     gclear, G, M, N, ld, out);
     count_launches(1);
     return e;
 }

@@ -148,6 +148,7 @@ struct Tile {
     int kb0, kb1;   // k-blocks [kb0, kb1) of this item's split of K
     int ks;         // split index
     int m0;         // weight-gradient items: first row of the output tile within its group
+    int store;      // weight-gradient items: the only item of its output tile (store, not add)
 };
 
 // A work item's table entry, loaded but not yet checked.  The roles that walk the
@@ -182,12 +183,14 @@ __device__ __forceinline__ Tile tile_finish(const GemmArgs& p, const TileLd& l) 
     Tile t;
     t.ks = l.ks;
     t.m0 = 0;
-    if (p.item_table == 2) {   // a weight-gradient item {g, m0 | n0 << 16, kb0, kb1}
+    t.store = 0;
+    if (p.item_table == 2) {   // a weight-gradient item {g, m0 | n0 << 16, kb0, kb1 (| store bit)}
         t.g = l.d.x;
         t.m0 = l.d.y & 0xffff;
         t.n0 = (int)((uint32_t)l.d.y >> 16);
         t.kb0 = l.d.z;
-        t.kb1 = l.d.w;
+        t.kb1 = l.d.w & (BWD_STORE_BIT - 1);
+        t.store = (l.d.w & BWD_STORE_BIT) ? 1 : 0;
         t.row0 = t.g * p.wg_M + t.m0;
         t.nrows = min(GM_BM, p.wg_M - t.m0);
         if (t.g < 0 || t.g >= p.G || t.m0 >= p.wg_M || t.n0 >= p.N || t.kb0 < 0 || t.kb1 <= t.kb0 ||
@@ -249,9 +252,8 @@ __device__ __forceinline__ Tile decode_tile(const GemmArgs& p, int64_t w) {
 // below fp32 resolution).  Evaluated in fp32 the GELU error stays below 1e-6 in
 // absolute value; the hidden activation is then rounded to bf16 (2^-9 relative).
 // Two values at a time with the packed fp32x2 instructions.
-__device__ __forceinline__ void gelu_erf2(float& u0, float& u1) {
-    const uint64_t a = f2_pack(fabsf(u0), fabsf(u1));
-    const uint64_t z = f2_mul(a, f2_pack(0.70710678118654752f, 0.70710678118654752f));
+__device__ __forceinline__ void erfc_as2(float a0, float a1, float& q0, float& q1) {   // a0, a1 >= 0
+    const uint64_t z = f2_mul(f2_pack(a0, a1), f2_pack(0.70710678118654752f, 0.70710678118654752f));
     uint64_t P = f2_fma(z, f2_pack(0.0000430638f, 0.0000430638f), f2_pack(0.0002765672f, 0.0002765672f));
     P = f2_fma(P, z, f2_pack(0.0001520143f, 0.0001520143f));
     P = f2_fma(P, z, f2_pack(0.0092705272f, 0.0092705272f));
@@ -264,16 +266,29 @@ __device__ __forceinline__ void gelu_erf2(float& u0, float& u1) {
     P = f2_mul(P, P);
     float p0, p1;
     f2_unpack(P, p0, p1);
-    const uint64_t q = f2_pack(rcp_approx(p0), rcp_approx(p1));
-    const uint64_t r = f2_fma(f2_mul(a, f2_pack(-0.5f, -0.5f)), q,
+    q0 = rcp_approx(p0);
+    q1 = rcp_approx(p1);
+}
+
+__device__ __forceinline__ void gelu_erf2(float& u0, float& u1) {
+    float q0, q1;
+    erfc_as2(fabsf(u0), fabsf(u1), q0, q1);
+    const uint64_t r = f2_fma(f2_mul(f2_pack(fabsf(u0), fabsf(u1)), f2_pack(-0.5f, -0.5f)), f2_pack(q0, q1),
                               f2_pack(fmaxf(u0, 0.0f), fmaxf(u1, 0.0f)));
     f2_unpack(r, u0, u1);
 }
 
-// GELU'(u) = Phi(u) + u phi(u) (the derivative of the erf form), in fp32 with CUDA's
-// normcdff and expf (the training path only).
-__device__ __forceinline__ float gelu_grad(float u) {
-    return normcdff(u) + u * 0.3989422804014327f * expf(-0.5f * u * u);
+// GELU'(u) = Phi(u) + u phi(u) (the derivative of the erf form) of two values, for the
+// training path: Phi(u) = erfc(-u / sqrt 2) / 2 from the erfc above (1 - q / 2 for
+// u >= 0, q / 2 below), phi(u) = exp(-u^2 / 2) / sqrt(2 pi) with CUDA's __expf.
+// Absolute error below 1e-6.
+__device__ __forceinline__ void gelu_grad2(float& u0, float& u1) {
+    float q0, q1;
+    erfc_as2(fabsf(u0), fabsf(u1), q0, q1);
+    const float c0 = u0 >= 0.0f ? 1.0f - 0.5f * q0 : 0.5f * q0;
+    const float c1 = u1 >= 0.0f ? 1.0f - 0.5f * q1 : 0.5f * q1;
+    u0 = fmaf(u0, 0.3989422804014327f * __expf(-0.5f * u0 * u0), c0);
+    u1 = fmaf(u1, 0.3989422804014327f * __expf(-0.5f * u1 * u1), c1);
 }
 
 struct Smem {
@@ -597,7 +612,7 @@ __device__ void mma_issuer(const GemmArgs& p, const Smem& sm, uint32_t tmem, int
 template <int ROWS>
 __device__ __forceinline__ void reduce_chunk(const GemmArgs& p, float* stg_all, int warp, int lane,
                                              const uint32_t (&v)[32], float sc, int64_t my_yoff,
-                                             int n) {
+                                             int n, bool store) {
     float* stg = stg_all + warp * (ROWS * GM_STG_LD);
     const int col = n + 4 * (lane & 7);
 #pragma unroll
@@ -617,7 +632,11 @@ __device__ __forceinline__ void reduce_chunk(const GemmArgs& p, float* stg_all, 
             const float* row = stg + (4 * r + (lane >> 3)) * GM_STG_LD;
             const int64_t yo = *reinterpret_cast<const int64_t*>(row + 32);
             const float4 val = *reinterpret_cast<const float4*>(row + 4 * (lane & 7));
-            if (yo >= 0 && col < p.N) atomicAdd(reinterpret_cast<float4*>(p.yacc + yo + col), val);
+            if (yo >= 0 && col < p.N) {
+                float4* dst = reinterpret_cast<float4*>(p.yacc + yo + col);
+                if (store) *dst = val;   // the only contribution to these elements
+                else atomicAdd(dst, val);
+            }
         }
         __syncwarp();
     }
@@ -776,7 +795,7 @@ __device__ void epilogue(const GemmArgs& p, const Smem& sm, uint32_t tmem, int64
                 }
                 const int n = t.n0 + c0;
                 const int64_t my_yoff = ok_row ? t.ks * p.y_split_stride + tok * p.ldy : -1;
-                reduce_chunk<STG_ROWS>(p, sm.stg, warp, lane, v, sc, my_yoff, n);
+                reduce_chunk<STG_ROWS>(p, sm.stg, warp, lane, v, sc, my_yoff, n, TRAIN && t.store);
                 continue;
             }
             uint32_t v[32];
@@ -807,7 +826,7 @@ __device__ void epilogue(const GemmArgs& p, const Smem& sm, uint32_t tmem, int64
                             const float a = __uint_as_float(v[8 * g8 + i]);
                             const bool in = n + 8 * g8 + i < p.N;   // columns past N: padding
                             dg_acc += in ? a * af[i] : 0.f;
-                            const float sg = 1.0f / (1.0f + expf(-uf[i]));   // SiLU(u) = u sg
+                            const float sg = __fdividef(1.0f, 1.0f + __expf(-uf[i]));   // SiLU(u) = u sg
                             fu[i] = in ? sc * a * vf[i] * sg * (1.0f + uf[i] * (1.0f - sg)) : 0.f;
                             fv[i] = in ? sc * a * uf[i] * sg : 0.f;
                         }
@@ -835,11 +854,13 @@ __device__ void epilogue(const GemmArgs& p, const Smem& sm, uint32_t tmem, int64
                         unpack_bf16x8(*reinterpret_cast<const uint4*>(urow + 8 * g8), uf);
                         unpack_bf16x8(*reinterpret_cast<const uint4*>(arow + 8 * g8), af);
 #pragma unroll
+                        for (int i = 0; i < 8; i += 2) gelu_grad2(uf[i], uf[i + 1]);   // GELU'(u)
+#pragma unroll
                         for (int i = 0; i < 8; ++i) {
                             const float a = __uint_as_float(v[8 * g8 + i]);
                             const bool in = n + 8 * g8 + i < p.N;   // columns past N: padding
                             dg_acc += in ? a * af[i] : 0.f;
-                            f[i] = in ? sc * a * gelu_grad(uf[i]) : 0.f;
+                            f[i] = in ? sc * a * uf[i] : 0.f;
                         }
                         uint4 u;
                         u.x = pack_bf16x2(f[0], f[1]);

@@ -306,6 +306,9 @@ cudaError_t launch_grouped_gemm(const GemmArgs& a, int grid, cudaStream_t s);
 
 // k-blocks (of 64 rows) per weight-gradient work item at most.
 constexpr int64_t BWD_KCH = 64;
+// Set in a weight-gradient item's end k-block when its group has one chunk of K: the item
+// is the only one writing its output tile, so the GEMM stores instead of adding.
+constexpr int BWD_STORE_BIT = 1 << 30;
 // Per token: sig[t k + j] = sigmoid(x_t . W_r[:, idx[t k + j]]) (fp32, from the transposed
 // copy wrt [E][dp]) and gate = sig / sum_j sig (k <= 32).
 cudaError_t launch_bwd_gates(const __nv_bfloat16* x, const float* wrt, int dp, const int32_t* idx, int64_t T,
@@ -321,7 +324,13 @@ cudaError_t launch_bwd_rows(const int32_t* idx, const int32_t* inv, const int32_
 // groups holding `rows` rows in total.
 int64_t bwd_max_items(int64_t rows, int G, int M, int N, int BN);
 cudaError_t launch_bwd_items(const int32_t* koff, int G, int64_t K_rows, int M, int N, int BN,
-                             int max_items, int4* items, int32_t* n_items, DevStatus* st, cudaStream_t s);
+                             int max_items, int4* items, int32_t* n_items, int32_t* gclear, DevStatus* st,
+                             cudaStream_t s);
+// Clears what the weight-gradient items will not write of out [G][M][ld] (fp32): the
+// groups with gclear[g] set (no rows, or several chunks adding up), and the pad columns
+// [N, ld) of the others.
+cudaError_t launch_bwd_zero(const int32_t* gclear, int G, int M, int N, int64_t ld, float* out, int num_sms,
+                            cudaStream_t s);
 // xp[r] = x[ptok[r]], gdy[r] = pgate[r] dy[ptok[r]] over the poff[E] padded rows.
 cudaError_t launch_bwd_gather(const __nv_bfloat16* x, const __nv_bfloat16* dy, const int32_t* ptok,
                               const float* pgate, const int32_t* poff, int E, int d, int64_t max_rows,
