@@ -160,6 +160,26 @@ moevie_status moevie_moe_forward(const moevie_layer* layer, const void* x, int64
                                  const moevie_routing* routing, void* ws, size_t ws_bytes,
                                  void* stream);
 
+/* The layer from host memory to host memory, the copies overlapped with the compute.
+ * Every token's output depends on that token alone (Eqs. 4-7: routing, gates and the
+ * experts act per token), so the layer runs chunk by chunk over contiguous token ranges:
+ * chunk i holds tokens [i Tc, min(T, (i + 1) Tc)), Tc = ceil(T / chunks).  Its rows of x
+ * go from x_host to x_dev on the library's copy-in stream, moevie_moe_forward runs it on
+ * `stream`, and its rows of y go from y_dev to y_host on the copy-out stream, so chunk
+ * i's layer overlaps the copies of its neighbours.  `stream` completes after the last
+ * copy out: synchronise it (or wait on it) before reading y_host.
+ * x_host, y_host: host memory [T, d] bf16 (pinned, for the copies to be asynchronous);
+ * x_dev, y_dev: caller-owned device buffers [T, d] bf16, 16-byte aligned; ws:
+ * moevie_workspace_size(Tc, ...) bytes at least, set up with moevie_workspace_init;
+ * 1 <= chunks <= MOEVIE_HOST_MAX_CHUNKS, else MOEVIE_ERR_UNSUPPORTED.  The first call in a
+ * context creates the two copy streams and their events (make it before any stream
+ * capture); calls on one device share them, so calls from several host threads must
+ * not overlap.  Errors as for moevie_moe_forward; device errors land in ws's status. */
+#define MOEVIE_HOST_MAX_CHUNKS 16
+moevie_status moevie_moe_forward_host(const moevie_layer* layer, const void* x_host, int64_t T, void* y_host,
+                                      void* x_dev, void* y_dev, int64_t chunks, void* ws, size_t ws_bytes,
+                                      void* stream);
+
 /* moevie_permute without a workspace (the paper has no counterpart: this is a
  * calling convention, not part of the method).  Same inputs, outputs, ordering and
  * validation as moevie_permute, and bit-identical results.

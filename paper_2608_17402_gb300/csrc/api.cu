@@ -4,7 +4,9 @@
 #include <stdint.h>
 #include <string.h>
 
+#include <algorithm>
 #include <atomic>
+#include <mutex>
 
 #include "internal.h"
 #include "moevie_testing.h"
@@ -849,6 +851,102 @@ moevie_status moevie_moe_forward(const moevie_layer* layer, const void* x, int64
                                  const moevie_routing* routing, void* ws, size_t ws_bytes,
                                  void* stream) {
     return forward_impl(layer, x, T, y, routing, ws, ws_bytes, stream, nullptr, 0);
+}
+
+}  // extern "C"
+
+namespace {
+
+// Copy streams and events of moevie_moe_forward_host, one set per device, created by the
+// first call in a context (and again in a new context after a device reset).
+struct HostPipe {
+    void* ctx = nullptr;
+    cudaStream_t in = nullptr, out = nullptr;
+    cudaEvent_t start = nullptr, done = nullptr;
+    cudaEvent_t ev_in[MOEVIE_HOST_MAX_CHUNKS] = {}, ev_out[MOEVIE_HOST_MAX_CHUNKS] = {};
+};
+
+cudaError_t host_pipe(HostPipe** out) {
+    constexpr int kMaxDevices = 64;
+    static std::mutex mu;
+    static HostPipe pipes[kMaxDevices];
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    if (dev < 0 || dev >= kMaxDevices) return cudaErrorInvalidDevice;
+    std::lock_guard<std::mutex> lock(mu);
+    HostPipe& p = pipes[dev];
+    void* cur = current_context();
+    if (!p.in || cur == nullptr || cur != p.ctx) {
+        HostPipe n;
+        const unsigned ef = cudaEventDisableTiming;
+        if ((e = cudaStreamCreateWithFlags(&n.in, cudaStreamNonBlocking)) != cudaSuccess ||
+            (e = cudaStreamCreateWithFlags(&n.out, cudaStreamNonBlocking)) != cudaSuccess ||
+            (e = cudaEventCreateWithFlags(&n.start, ef)) != cudaSuccess ||
+            (e = cudaEventCreateWithFlags(&n.done, ef)) != cudaSuccess)
+            return e;
+        for (int c = 0; c < MOEVIE_HOST_MAX_CHUNKS; ++c)
+            if ((e = cudaEventCreateWithFlags(&n.ev_in[c], ef)) != cudaSuccess ||
+                (e = cudaEventCreateWithFlags(&n.ev_out[c], ef)) != cudaSuccess)
+                return e;
+        n.ctx = current_context();
+        p = n;
+    }
+    *out = &p;
+    return cudaSuccess;
+}
+
+}  // namespace
+
+extern "C" {
+
+moevie_status moevie_moe_forward_host(const moevie_layer* layer, const void* x_host, int64_t T, void* y_host,
+                                      void* x_dev, void* y_dev, int64_t chunks, void* ws, size_t ws_bytes,
+                                      void* stream) {
+    if (!layer) return MOEVIE_ERR_INVALID_ARG;
+    const int64_t d = layer->d;
+    moevie_status c = check_sizes(T, d, layer->E, layer->k, layer->h, layer->h_s);
+    if (c != MOEVIE_OK) return c;
+    if (chunks < 1 || chunks > MOEVIE_HOST_MAX_CHUNKS) return MOEVIE_ERR_UNSUPPORTED;
+    if (T == 0) return MOEVIE_OK;
+    if (!x_host || !y_host || !x_dev || !y_dev || !ws || !a16(x_dev) || !a16(y_dev)) return MOEVIE_ERR_INVALID_ARG;
+    const int64_t Tc = (T + chunks - 1) / chunks;   // tokens per chunk (the last one may have fewer)
+    const int64_t n_chunks = (T + Tc - 1) / Tc;
+    if (ws_bytes < make_layout(Tc, d, layer->E, layer->k, layer->h, layer->h_s).total) return MOEVIE_ERR_WORKSPACE;
+    HostPipe* p = nullptr;
+    MV_TRY(host_pipe(&p));
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    const size_t row_bytes = 2 * (size_t)d;
+    const uint8_t* xh = static_cast<const uint8_t*>(x_host);
+    uint8_t* yh = static_cast<uint8_t*>(y_host);
+    uint8_t* xd = static_cast<uint8_t*>(x_dev);
+    uint8_t* yd = static_cast<uint8_t*>(y_dev);
+    // the copies into x_dev wait for the work already on `stream` (an earlier call's chunks
+    // still reading x_dev); every chunk's rows are copied in, back to back
+    MV_TRY(cudaEventRecord(p->start, s));
+    MV_TRY(cudaStreamWaitEvent(p->in, p->start, 0));
+    for (int64_t i = 0; i < n_chunks; ++i) {
+        const int64_t t0 = i * Tc, n = std::min(Tc, T - t0);
+        MV_TRY(cudaMemcpyAsync(xd + t0 * row_bytes, xh + t0 * row_bytes, n * row_bytes, cudaMemcpyHostToDevice,
+                               p->in));
+        MV_TRY(cudaEventRecord(p->ev_in[i], p->in));
+    }
+    // each chunk's layer once its rows are in, its rows of y out once it is done
+    for (int64_t i = 0; i < n_chunks; ++i) {
+        const int64_t t0 = i * Tc, n = std::min(Tc, T - t0);
+        MV_TRY(cudaStreamWaitEvent(s, p->ev_in[i], 0));
+        if ((c = forward_impl(layer, xd + t0 * row_bytes, n, yd + t0 * row_bytes, nullptr, ws, ws_bytes, stream,
+                              nullptr, 0)) != MOEVIE_OK)
+            return c;
+        MV_TRY(cudaEventRecord(p->ev_out[i], s));
+        MV_TRY(cudaStreamWaitEvent(p->out, p->ev_out[i], 0));
+        MV_TRY(cudaMemcpyAsync(yh + t0 * row_bytes, yd + t0 * row_bytes, n * row_bytes, cudaMemcpyDeviceToHost,
+                               p->out));
+    }
+    // `stream` completes after the last copy out
+    MV_TRY(cudaEventRecord(p->done, p->out));
+    MV_TRY(cudaStreamWaitEvent(s, p->done, 0));
+    return MOEVIE_OK;
 }
 
 moevie_status moevie_get_device_status(const void* ws, void* stream, moevie_status* out,

@@ -11,7 +11,10 @@
 //   bwd_rows_kernel    per padded row its token (-1 for padding) and gate (0), and per
 //                      routing slot its padded row
 //   bwd_items_kernel   the weight-gradient work items {g, m0 | n0 << 16, kb0, kb1}: per
-//                      group, output tiles x chunks of at most BWD_KCH k-blocks
+//                      group, output tiles x chunks of at most BWD_KCH k-blocks (a group of
+//                      one chunk stores its gradient instead of adding into it)
+//   bwd_zero_kernel    clears what the items will add into or not write: the gradients of
+//                      groups with no rows or several chunks, and pad columns
 //   bwd_gather_kernel  the padded rows of x and of g dy (bf16; zero rows for padding)
 //   bwd_router_kernel  per token: dg_j = dy . E_j(x) from the partial row dots, the gate
 //                      derivative ds (Eqs. 4-5), dx += ds W_r^T, and ds into a dense

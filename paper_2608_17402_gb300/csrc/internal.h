@@ -368,6 +368,9 @@ static_assert((PERM_STATIC_MAX_SLOTS + PERM_STATIC_MAX_CHUNKS - 1) / PERM_STATIC
 // return the cached address while the device's context is the one it was looked up in
 // (after a device reset the next call looks it up again).  Thread-safe.
 cudaError_t perm_static_scratch(unsigned char** out);
+// The calling thread's current CUDA context (an opaque handle; nullptr when it cannot be
+// read), for per-context caches of device-side objects.
+void* current_context();
 
 // ------------------------------------------------------------------- misc
 

@@ -421,7 +421,7 @@ static __device__ __align__(256) unsigned char g_perm_static_scratch[PERM_STATIC
 
 // The current context (driver cuCtxGetCurrent, reached through the runtime's entry-point
 // query so that the library links only the runtime); nullptr when it cannot be read.
-static void* current_context() {
+void* current_context() {
     using GetCtx = CUresult (*)(CUcontext*);
     static std::atomic<GetCtx> fn{nullptr};
     GetCtx f = fn.load(std::memory_order_acquire);

@@ -25,7 +25,7 @@ STATUS_NAMES = {0: "MOEVIE_OK", 1: "MOEVIE_ERR_INVALID_ARG", 2: "MOEVIE_ERR_UNSU
 C_ENTRY_POINTS = ("moevie_status_string", "moevie_version", "moevie_workspace_size",
                   "moevie_workspace_init", "moevie_route", "moevie_permute", "moevie_permute_static",
                   "moevie_expert_ffn",
-                  "moevie_shared_expert", "moevie_combine", "moevie_moe_forward",
+                  "moevie_shared_expert", "moevie_combine", "moevie_moe_forward", "moevie_moe_forward_host",
                   "moevie_get_device_status", "moevie_launch_count", "moevie_shared_groups",
                   "moevie_update_bias", "moevie_backward_workspace_size", "moevie_moe_backward",
                   "moevie_test_route_logits",
@@ -74,6 +74,7 @@ def load():
         "moevie_shared_expert": ([P, P, P, I64, I64, I64, P, P, SZ, P], ctypes.c_int),
         "moevie_combine": ([P, P, P, P, F, I64, I64, I64, P, P], ctypes.c_int),
         "moevie_moe_forward": ([P, P, I64, P, P, P, SZ, P], ctypes.c_int),
+        "moevie_moe_forward_host": ([P, P, I64, P, P, P, I64, P, SZ, P], ctypes.c_int),
         "moevie_get_device_status": ([P, P, P, P], ctypes.c_int),
         "moevie_launch_count": ([], ctypes.c_uint64),
         "moevie_shared_groups": ([I64] * 6, ctypes.c_int64),
@@ -330,6 +331,39 @@ def moevie_moe_forward(layer: LayerWeights, x, ws: Workspace, y=None, routing=Fa
           ctypes.byref(rstruct) if rstruct is not None else None, ws.ptr, ws.nbytes,
           _stream(stream))
     return (y, rt) if routing else y
+
+
+HOST_MAX_CHUNKS = 16   # MOEVIE_HOST_MAX_CHUNKS
+
+
+def host_chunks(T: int) -> int:
+    """A token-chunk count for moevie_moe_forward_host: chunks of at least 8192 tokens (a
+    chunk is a whole layer forward, and smaller ones lose more to weight reads and partial
+    tiles than the overlap wins), at most 4 (measured on GB300: T = 65536 in 4 chunks
+    3.11 ms against 4.20 ms in one and 3.59 ms in 8; T = 32768 in 4 chunks 1.44 ms against
+    1.92 ms; T = 8192 best in one)."""
+    return max(1, min(4, T // 8192))
+
+
+def moevie_moe_forward_host(layer: LayerWeights, x_host, y_host, x_dev, y_dev, ws: Workspace, chunks: int,
+                            stream=None):
+    """The layer from host to host memory with the copies overlapped (moevie_moe_forward_host):
+    x_host, y_host CPU bf16 [T, d] (pinned for overlap); x_dev, y_dev CUDA bf16 [T, d] scratch;
+    ws a Workspace for ceil(T / chunks) tokens.  Asynchronous on `stream`, which completes
+    after the last row of y_host is written."""
+    _want(x_dev, torch.bfloat16, "x_dev")
+    _want(y_dev, torch.bfloat16, "y_dev")
+    for name, t in (("x_host", x_host), ("y_host", y_host)):
+        if t.device.type != "cpu" or t.dtype != torch.bfloat16 or not t.is_contiguous():
+            raise ValueError(f"{name}: expected a contiguous CPU bfloat16 tensor")
+    T, d = x_host.shape
+    if tuple(y_host.shape) != (T, d) or tuple(x_dev.shape) != (T, d) or tuple(y_dev.shape) != (T, d):
+        raise ValueError("x_host, y_host, x_dev and y_dev must all be [T, d]")
+    L = layer.c_struct()
+    _call("moevie_moe_forward_host", ctypes.byref(L), ctypes.c_void_p(x_host.data_ptr()), T,
+          ctypes.c_void_p(y_host.data_ptr()), _p(x_dev), _p(y_dev), int(chunks), ws.ptr, ws.nbytes,
+          _stream(stream))
+    return y_host
 
 
 def moevie_backward_workspace_size(T_max, d, E, k, h, h_s=0, swiglu=False) -> int:
