@@ -183,3 +183,60 @@ def test_workspace_size_monotone_and_covers_the_big_regions(lib, d, E, k, h, hs)
         assert rc == 0 and size >= prev, (T, size, prev)
         assert size >= 4 * T * d + 2 * T * k * hp
         prev = size
+
+
+def test_backward_workspace_and_validation(lib):
+    """moevie_backward_workspace_size grows with the shared expert's width and with SwiGLU,
+    and moevie_moe_backward validates its layer and gradient pointers before any launch."""
+    from paper_2608_17402_gb300.moevie import _Layer
+
+    def size(*dims):
+        out = ctypes.c_size_t(0)
+        rc = lib.moevie_backward_workspace_size(*dims, ctypes.byref(out))
+        return rc, out.value
+    rc0, a = size(1024, 256, 16, 4, 128, 0, 0)
+    rc1, b = size(1024, 256, 16, 4, 128, 256, 0)
+    rc2, c = size(1024, 256, 16, 4, 128, 256, 1)
+    assert rc0 == rc1 == rc2 == 0 and a < b < c
+    assert size(2048, 256, 16, 4, 128, 256, 1)[1] > c          # monotone in T
+    assert size(1024, 256, 16, 4, 128, 70000, 0)[0] == 2       # h_s above 65535
+    assert size(1024, 256, 40, 33, 128, 0, 0)[0] == 2          # k above 32
+    fake = 0x1000
+    P = ctypes.c_void_p
+
+    def bwd(layer, dWs1=fake, dWs2=fake, dWs3=None, ws_bytes=1 << 30):
+        g = [P(fake)] * 5   # dx, dW_r, dW1, dW2 and (SwiGLU) dW3
+        return lib.moevie_moe_backward(ctypes.byref(layer), P(fake), P(fake), 4, P(fake), g[0], g[1], g[2], g[3],
+                                       None if layer.W3 == 0 else g[4], None if dWs1 is None else P(dWs1),
+                                       None if dWs2 is None else P(dWs2), None if dWs3 is None else P(dWs3),
+                                       P(fake), ws_bytes, None)
+    shared = _Layer(16, 8, 2, 32, 32, fake, fake, fake, fake, fake, fake, 1.0)
+    assert bwd(shared, ws_bytes=16) == 3                        # workspace too small
+    assert bwd(shared, dWs1=None) == 1                          # shared expert without dWs1
+    assert bwd(shared, dWs2=fake + 4) == 1                      # misaligned dWs2
+    swiglu = _Layer(16, 8, 2, 32, 32, fake, fake, fake, fake, fake, fake, 1.0, fake, fake)
+    assert bwd(swiglu) == 1                                     # SwiGLU shared expert without dWs3
+    assert bwd(_Layer(16, 8, 2, 32, 32, fake, fake, fake, fake, fake, fake, 1.0, fake, 0), dWs3=fake) == 1
+
+
+def test_forward_host_validation(lib):
+    """moevie_moe_forward_host checks the chunk count, its buffers and the workspace (sized
+    for one chunk) before creating its streams or enqueueing anything."""
+    from paper_2608_17402_gb300 import moevie
+    from paper_2608_17402_gb300.moevie import _Layer
+    fake = 0x1000
+    P = ctypes.c_void_p
+    L = _Layer(16, 8, 2, 32, 0, fake, fake, fake, fake, 0, 0, 1.0)
+
+    def fwd(T, chunks, ws_bytes, x_dev=fake, x_host=fake):
+        return lib.moevie_moe_forward_host(ctypes.byref(L), None if x_host is None else P(x_host), T, P(fake),
+                                           P(x_dev), P(fake), chunks, P(fake), ws_bytes, None)
+    assert fwd(64, 0, 1 << 30) == 2
+    assert fwd(64, moevie.HOST_MAX_CHUNKS + 1, 1 << 30) == 2
+    assert fwd(64, 4, 1 << 30, x_dev=fake + 8) == 1             # misaligned device buffer
+    assert fwd(64, 4, 1 << 30, x_host=None) == 1
+    assert fwd(0, 4, 0) == 0                                    # T == 0: nothing to do
+    out = ctypes.c_size_t(0)
+    assert lib.moevie_workspace_size(16, 16, 8, 2, 32, 0, ctypes.byref(out)) == 0
+    assert fwd(64, 2, out.value) == 3                           # chunks of 32 tokens need more room
+    assert [moevie.host_chunks(T) for T in (1024, 8192, 16384, 32768, 65536, 1 << 20)] == [1, 1, 2, 4, 4, 4]
