@@ -162,11 +162,13 @@ moevie_status moevie_moe_forward(const moevie_layer* layer, const void* x, int64
 
 /* The layer from host memory to host memory, the copies overlapped with the compute.
  * Every token's output depends on that token alone (Eqs. 4-7: routing, gates and the
- * experts act per token), so the layer runs chunk by chunk over contiguous token ranges:
- * chunk i holds tokens [i Tc, min(T, (i + 1) Tc)), Tc = ceil(T / chunks).  Its rows of x
+ * experts act per token), so the layer runs piece by piece over contiguous token ranges
+ * of at most Tc = ceil(T / chunks) tokens: one piece with chunks = 1; otherwise a first
+ * piece of ceil(Tc / 2) tokens, then pieces of Tc, the last one what is left (so the first
+ * copy in and the last copy out, which no layer hides, are short).  A piece's rows of x
  * go from x_host to x_dev on the library's copy-in stream, moevie_moe_forward runs it on
- * `stream`, and its rows of y go from y_dev to y_host on the copy-out stream, so chunk
- * i's layer overlaps the copies of its neighbours.  `stream` completes after the last
+ * `stream`, and its rows of y go from y_dev to y_host on the copy-out stream, so each
+ * piece's layer overlaps the copies of its neighbours.  `stream` completes after the last
  * copy out: synchronise it (or wait on it) before reading y_host.
  * x_host, y_host: host memory [T, d] bf16 (pinned, for the copies to be asynchronous);
  * x_dev, y_dev: caller-owned device buffers [T, d] bf16, 16-byte aligned; ws:

@@ -863,7 +863,7 @@ struct HostPipe {
     void* ctx = nullptr;
     cudaStream_t in = nullptr, out = nullptr;
     cudaEvent_t start = nullptr, done = nullptr;
-    cudaEvent_t ev_in[MOEVIE_HOST_MAX_CHUNKS] = {}, ev_out[MOEVIE_HOST_MAX_CHUNKS] = {};
+    cudaEvent_t ev_in[MOEVIE_HOST_MAX_CHUNKS + 1] = {}, ev_out[MOEVIE_HOST_MAX_CHUNKS + 1] = {};   // per piece
 };
 
 cudaError_t host_pipe(HostPipe** out) {
@@ -885,7 +885,7 @@ cudaError_t host_pipe(HostPipe** out) {
             (e = cudaEventCreateWithFlags(&n.start, ef)) != cudaSuccess ||
             (e = cudaEventCreateWithFlags(&n.done, ef)) != cudaSuccess)
             return e;
-        for (int c = 0; c < MOEVIE_HOST_MAX_CHUNKS; ++c)
+        for (int c = 0; c <= MOEVIE_HOST_MAX_CHUNKS; ++c)
             if ((e = cudaEventCreateWithFlags(&n.ev_in[c], ef)) != cudaSuccess ||
                 (e = cudaEventCreateWithFlags(&n.ev_out[c], ef)) != cudaSuccess)
                 return e;
@@ -910,9 +910,24 @@ moevie_status moevie_moe_forward_host(const moevie_layer* layer, const void* x_h
     if (chunks < 1 || chunks > MOEVIE_HOST_MAX_CHUNKS) return MOEVIE_ERR_UNSUPPORTED;
     if (T == 0) return MOEVIE_OK;
     if (!x_host || !y_host || !x_dev || !y_dev || !ws || !a16(x_dev) || !a16(y_dev)) return MOEVIE_ERR_INVALID_ARG;
-    const int64_t Tc = (T + chunks - 1) / chunks;   // tokens per chunk (the last one may have fewer)
-    const int64_t n_chunks = (T + Tc - 1) / Tc;
+    const int64_t Tc = (T + chunks - 1) / chunks;   // tokens per chunk
     if (ws_bytes < make_layout(Tc, d, layer->E, layer->k, layer->h, layer->h_s).total) return MOEVIE_ERR_WORKSPACE;
+    // the pieces the layer runs on: with several chunks a half chunk first, whole chunks,
+    // and what is left last (another half chunk when Tc divides T), so that the first
+    // copy in and the last copy out, the two no layer hides, are half as long
+    int64_t bnd[MOEVIE_HOST_MAX_CHUNKS + 2];
+    int64_t n_chunks = 0;
+    bnd[0] = 0;
+    if (chunks == 1) {
+        bnd[++n_chunks] = T;
+    } else {
+        int64_t t = std::min(T, (Tc + 1) / 2);
+        bnd[++n_chunks] = t;
+        while (t < T) {
+            t = std::min(T, t + Tc);
+            bnd[++n_chunks] = t;
+        }
+    }
     HostPipe* p = nullptr;
     MV_TRY(host_pipe(&p));
     cudaStream_t s = static_cast<cudaStream_t>(stream);
@@ -926,14 +941,14 @@ moevie_status moevie_moe_forward_host(const moevie_layer* layer, const void* x_h
     MV_TRY(cudaEventRecord(p->start, s));
     MV_TRY(cudaStreamWaitEvent(p->in, p->start, 0));
     for (int64_t i = 0; i < n_chunks; ++i) {
-        const int64_t t0 = i * Tc, n = std::min(Tc, T - t0);
+        const int64_t t0 = bnd[i], n = bnd[i + 1] - bnd[i];
         MV_TRY(cudaMemcpyAsync(xd + t0 * row_bytes, xh + t0 * row_bytes, n * row_bytes, cudaMemcpyHostToDevice,
                                p->in));
         MV_TRY(cudaEventRecord(p->ev_in[i], p->in));
     }
     // each chunk's layer once its rows are in, its rows of y out once it is done
     for (int64_t i = 0; i < n_chunks; ++i) {
-        const int64_t t0 = i * Tc, n = std::min(Tc, T - t0);
+        const int64_t t0 = bnd[i], n = bnd[i + 1] - bnd[i];
         MV_TRY(cudaStreamWaitEvent(s, p->ev_in[i], 0));
         if ((c = forward_impl(layer, xd + t0 * row_bytes, n, yd + t0 * row_bytes, nullptr, ws, ws_bytes, stream,
                               nullptr, 0)) != MOEVIE_OK)

@@ -337,12 +337,12 @@ HOST_MAX_CHUNKS = 16   # MOEVIE_HOST_MAX_CHUNKS
 
 
 def host_chunks(T: int) -> int:
-    """A token-chunk count for moevie_moe_forward_host: chunks of at least 8192 tokens (a
-    chunk is a whole layer forward, and smaller ones lose more to weight reads and partial
-    tiles than the overlap wins), at most 4 (measured on GB300: T = 65536 in 4 chunks
-    3.11 ms against 4.20 ms in one and 3.59 ms in 8; T = 32768 in 4 chunks 1.44 ms against
-    1.92 ms; T = 8192 best in one)."""
-    return max(1, min(4, T // 8192))
+    """A chunk count for moevie_moe_forward_host: pieces of at least 32768 tokens (each
+    piece is a whole layer forward, and smaller ones lose more to weight reads and partial
+    tiles than the overlap wins), at most 16.  Measured on GB300 with the half-size first
+    and last pieces: T = 65536 in 2 chunks 2.90 ms against 4.20 ms in one and 3.02 ms in
+    4; T = 32768 in 2 chunks 1.37 ms against 1.92 ms; T = 8192 best in one."""
+    return 1 if T < 32768 else max(2, min(HOST_MAX_CHUNKS, T // 32768))
 
 
 def moevie_moe_forward_host(layer: LayerWeights, x_host, y_host, x_dev, y_dev, ws: Workspace, chunks: int,

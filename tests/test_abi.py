@@ -239,4 +239,4 @@ def test_forward_host_validation(lib):
     out = ctypes.c_size_t(0)
     assert lib.moevie_workspace_size(16, 16, 8, 2, 32, 0, ctypes.byref(out)) == 0
     assert fwd(64, 2, out.value) == 3                           # chunks of 32 tokens need more room
-    assert [moevie.host_chunks(T) for T in (1024, 8192, 16384, 32768, 65536, 1 << 20)] == [1, 1, 2, 4, 4, 4]
+    assert [moevie.host_chunks(T) for T in (1024, 8192, 16384, 32768, 65536, 1 << 20)] == [1, 1, 1, 2, 2, 16]
