@@ -276,9 +276,10 @@ int64_t moevie_shared_groups(int64_t T, int64_t d, int64_t E, int64_t k, int64_t
  * dWs1 (all three NULL without one).  The gates are recomputed from x and W_r in fp32.
  * Arithmetic: bf16 GEMM operands with fp32 accumulation (the recomputed pre-activations,
  * activations, their gradients, g dy and ds are rounded to bf16 as GEMM operands); dx,
- * and the weight gradients of experts with more than 4096 rows (summed over several
- * chunks of rows), take fp32 reductions, so their last bits depend on the order in which
- * the GEMM's work items finish; the other weight gradients are written once.  Sizes: k <= 32, d and h <=
+ * and every weight gradient summed over more than 4096 rows (an expert's rows padded to
+ * 64; all T tokens for dW_r and the shared expert's), take fp32 reductions over chunks of
+ * rows, so their last bits depend on the order in which the GEMM's work items finish;
+ * the other weight gradients are written once.  Sizes: k <= 32, d and h <=
  * 65535 (h_s too), plus the limits of moevie_moe_forward.  `ws`:
  * moevie_backward_workspace_size(T_max, d, E, k, h, h_s, swiglu) bytes (swiglu nonzero for
  * SwiGLU experts), set up with moevie_workspace_init; device errors land in its status
