@@ -240,3 +240,32 @@ def test_forward_host_validation(lib):
     assert lib.moevie_workspace_size(16, 16, 8, 2, 32, 0, ctypes.byref(out)) == 0
     assert fwd(64, 2, out.value) == 3                           # chunks of 32 tokens need more room
     assert [moevie.host_chunks(T) for T in (1024, 8192, 16384, 32768, 65536, 1 << 20)] == [1, 1, 1, 2, 2, 16]
+
+
+def test_header_is_plain_c(lib, tmp_path):
+    """include/*.h compile as C11 (no C++ in the ABI), and a C program links against the
+    library and calls a host-only entry point."""
+    import shutil
+    import subprocess
+    gcc = shutil.which("gcc")
+    if gcc is None:
+        pytest.skip("no C compiler")
+    src = tmp_path / "abi.c"
+    src.write_text(
+        '#include <stdio.h>\n#include "moevie.h"\n#include "moevie_testing.h"\n'
+        "int main(void) {\n"
+        "    size_t bytes = 0;\n"
+        "    moevie_layer layer = {0};\n"
+        "    moevie_status s = moevie_workspace_size(512, 768, 16, 2, 768, 0, &bytes);\n"
+        "    (void)layer;\n"
+        '    printf("%d %zu\\n", (int)s, bytes);\n'
+        "    return s;\n"
+        "}\n")
+    libdir = os.path.dirname(lib._name)
+    exe = tmp_path / "abi"
+    subprocess.run([gcc, "-std=c11", "-Wall", "-Wextra", "-Werror", "-I", INCLUDE, str(src), "-o", str(exe),
+                    "-L", libdir, "-lmoevie", "-Wl,--unresolved-symbols=ignore-in-shared-libs",
+                    f"-Wl,-rpath,{libdir}"], check=True, capture_output=True)
+    out = subprocess.run([str(exe)], check=True, capture_output=True, text=True).stdout.split()
+    rc, want = _ws_size(lib, 512, 768, 16, 2, 768, 0)
+    assert out == ["0", str(want)] and rc == 0
