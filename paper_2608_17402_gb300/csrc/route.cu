@@ -369,8 +369,11 @@ __global__ void __launch_bounds__(256) route_topk_kernel(
 // NaN logit.
 constexpr int FB_BATCH = 4;       // candidates per pass over the terms
 constexpr int FB_X_SMEM = 16384;  // largest d whose x row is staged in shared memory
+// CTAs per SM the re-decision keeps resident for E <= 256 (its registers allow five), so
+// that up to five tokens per SM are re-decided at once
+constexpr int FB_CTAS_PER_SM = 5;
 template <int NPL>
-__global__ void __launch_bounds__(256) route_fallback_kernel(
+__global__ void __launch_bounds__(256, (NPL <= 8 ? FB_CTAS_PER_SM : 1)) route_fallback_kernel(
     const __nv_bfloat16* __restrict__ x, const float* __restrict__ wrt, int dp,
     const int32_t* __restrict__ wexp, int wexp_parts, int Ep,
     const float* __restrict__ b, const float* __restrict__ s, int ld,
@@ -636,7 +639,8 @@ cudaError_t launch_route_select(const __nv_bfloat16* x, const float* wrt, const 
                                 DevStatus* st, int num_sms, cudaStream_t s, float* zero,
                                 int64_t zero_n) {
     const int blocks = (int)(((int64_t)T * 32 + 255) / 256);
-    const int fb_blocks = T < 3 * num_sms ? T : 3 * num_sms;   // about one wave
+    const int fb_per_sm = (E + 31) / 32 <= 8 ? FB_CTAS_PER_SM : 3;
+    const int fb_blocks = T < fb_per_sm * num_sms ? T : fb_per_sm * num_sms;   // one resident wave
     const size_t fb_smem = d <= FB_X_SMEM ? (size_t)2 * d : 0;
     const int npl = (E + 31) / 32;
     const int dp = route_dpad(d);
